@@ -71,7 +71,8 @@ def smoothing_factors(ax: np.ndarray, aw: np.ndarray, alpha: float = 0.5):
     """Eq. delta-attn / delta-lmhead: delta_j = max_t|X_tj|^alpha / max_i|W_ij|^(1-alpha).
 
     alpha = 0.5 (the paper's value) is evaluated as fl32(sqrt(ax)) / fl32(sqrt(aw)), each step
-    correctly rounded.  Any other alpha is evaluated in fp64 and rounded once to fp32.
+    correctly rounded.  Any other alpha is taken as an fp32 number (the precision in which it is
+    specified), and the quotient is evaluated in fp64 and rounded once to fp32.
     A zero statistic on either side gives delta_j = 1.  Returns (delta, inv_delta) with
     inv_delta = fl32(1 / delta).
     """
@@ -81,8 +82,9 @@ def smoothing_factors(ax: np.ndarray, aw: np.ndarray, alpha: float = 0.5):
         with np.errstate(divide="ignore", invalid="ignore"):
             delta = (np.sqrt(ax) / np.sqrt(aw)).astype(np.float32)
     else:
+        a = float(np.float32(alpha))
         with np.errstate(divide="ignore", invalid="ignore"):
-            d64 = np.power(ax.astype(np.float64), alpha) / np.power(aw.astype(np.float64), 1.0 - alpha)
+            d64 = np.power(ax.astype(np.float64), a) / np.power(aw.astype(np.float64), 1.0 - a)
         delta = d64.astype(np.float32)
     degenerate = (ax == 0) | (aw == 0) | ~np.isfinite(delta) | (delta == 0)
     delta = np.where(degenerate, F32(1.0), delta).astype(np.float32)
