@@ -1,0 +1,194 @@
+/*
+ * w8a8.h - C ABI of libw8a8.so: the W8A8 SmoothQuant hot path of
+ * "A Method for Layer Bit-Width Allocation in LLM Quantization via Performance Maximization
+ * Under a Quality-Degradation Constraint" (arXiv 2608.28003) on one GB300 (sm_103a).
+ *
+ * Conventions (every entry point):
+ *   - Returns a w8a8_status.  Nothing is thrown across the ABI.  On a non-OK status,
+ *     w8a8_last_error() returns a message for the calling thread.
+ *   - Tensors are caller-owned DEVICE pointers unless a parameter says "host".  The library
+ *     allocates no device memory on any compute entry point; scratch space comes from a
+ *     caller-provided workspace whose size a *_workspace_size query returns.
+ *   - bf16 and fp16 tensors are passed as uint16_t bit patterns.  Matrices are row-major.  A
+ *     weight [N, K] has one row per output channel i and one column per input channel j
+ *     (the paper's W_{i,j}).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Compute
+ *     calls are asynchronous on it.  Errors found on the host (arguments, shapes,
+ *     alignment) are reported before anything is launched.  Errors of a launch are
+ *     reported as W8A8_ERR_CUDA.
+ *   - Alignment: every tensor pointer must be 16-byte aligned, and every K (input channels)
+ *     must be a multiple of 16.  Otherwise the call returns W8A8_ERR_ALIGN or W8A8_ERR_SHAPE.
+ *   - Workspace: its first W8A8_WS_RESERVED bytes hold split-K arrival counters.  They must be
+ *     zero before the workspace is first used (cudaMemset once after allocating).  Every call
+ *     leaves them zero again when it completes.  A workspace must not be used by two calls
+ *     that can run concurrently.
+ *   - Exactness: INT8 codes and INT32 accumulators are exact.  Every step that decides an INT8
+ *     code runs in IEEE fp32 with round-to-nearest-even, in the order documented below.
+ */
+#ifndef W8A8_H
+#define W8A8_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  W8A8_OK = 0,
+  W8A8_ERR_INVALID_ARG = 1, /* a required pointer is NULL, a size is negative, an enum is out of range */
+  W8A8_ERR_SHAPE = 2,       /* a shape the entry point does not support (K % 16 != 0, a limit exceeded) */
+  W8A8_ERR_ALIGN = 3,       /* a tensor pointer is not 16-byte aligned */
+  W8A8_ERR_CUDA = 4,        /* a CUDA runtime call or a kernel launch failed */
+  W8A8_ERR_UNSUPPORTED = 5, /* the current device is not an sm_103 GPU, or the feature is not built */
+  W8A8_ERR_TIMEOUT = 6,     /* a bounded device-side wait gave up (the kernel returned early) */
+  W8A8_ERR_WORKSPACE = 7    /* the workspace is NULL or smaller than the size query returned */
+} w8a8_status;
+
+enum { W8A8_PREC_BF16 = 0, W8A8_PREC_W8A8 = 1 };
+
+#define W8A8_WS_RESERVED 65536 /* bytes of counters at the start of every workspace */
+#define W8A8_MAX_K 65536       /* largest K (input channels) any entry point accepts */
+
+/* Version of this ABI (incremented on incompatible changes). */
+int w8a8_abi_version(void);
+
+/* Message for the last non-OK status returned on the calling thread ("" if none). */
+const char* w8a8_last_error(void);
+
+/* ---------------------------------------------------------------------------------------
+ * Prepared W8A8 weight of one linear (produced by w8a8_prepare_weights /
+ * w8a8_prepare_gate_up, owned by the caller).
+ *   wq        [n, k] INT8 codes of the smoothed weight, in [-127, 127]          (Eq. si, what-ffn)
+ *   s_w       [n]    per-output-channel scale s_i^W = max_j |W_hat_ij| / 127      (Eq. si)
+ *   inv_delta [k]    1 / delta_j, the activation side of the smoothing            (Eq. xhat-lmhead)
+ *   wq_f16    [n, k] nullable: the same codes as fp16 values (exact).  Linears with large
+ *                    token counts use it as the tensor-core operand.
+ * ------------------------------------------------------------------------------------- */
+typedef struct {
+  int32_t n, k;
+  const int8_t* wq;
+  const float* s_w;
+  const float* inv_delta;
+  const uint16_t* wq_f16;
+} w8a8_qweight;
+
+/* Optional per-call debug outputs of w8a8_linear (each pointer nullable). */
+typedef struct {
+  int8_t* xq;   /* [M, K] INT8 activation codes (Eq. xint8) */
+  float* s_x;   /* [M]    per-token scale s_t^x (Eq. stx) */
+  int32_t* acc; /* [M, N] INT32 accumulator sum_j xq_tj * wq_ij (Eq. gemm-final) */
+} w8a8_debug;
+
+/* ------------------------------------------------------------------ calibration (offline)
+ * Running per-channel maximum of |X| over calibration tokens, the max_t |X_{t,j}| of
+ * Eq. delta-attn / delta-lmhead (LM Head section: collected by a forward hook).
+ *   X       [T, K] bf16 activations at a linear's input
+ *   absmax  [K] fp32, in/out: absmax[j] = max(absmax[j], max_t |X_tj|).  Zero it before the
+ *           first batch.  Entries must be non-negative.
+ * T == 0 is a no-op. */
+w8a8_status w8a8_act_absmax(const uint16_t* X, int T, int K, float* absmax, void* stream);
+
+/* ------------------------------------------------------------ weight preparation (offline)
+ * SmoothQuant preparation of one linear (Eq. delta-attn / delta-lmhead, what-lmhead, then
+ * Eq. si / what-ffn on the smoothed rows):
+ *   delta_j   = max_t|X_tj|^alpha / max_i|W_ij|^(1-alpha).  For alpha == 0.5 this is
+ *               fl32(sqrt(ax_j)) / fl32(sqrt(aw_j)) exactly rounded.  Other alpha values are
+ *               evaluated in fp64 and rounded once.  delta_j = 1 where either statistic is 0.
+ *   inv_delta = fl32(1 / delta)
+ *   W_hat_ij  = fl32(W_ij * delta_j);  m_i = max_j |W_hat_ij|;  s_w_i = fl32(m_i / 127)
+ *   wq_ij     = clamp(rint(fl32(W_hat_ij * fl32(127 / m_i))), -127, 127)  (0 for an all-zero row)
+ * W [N, K] bf16; act_absmax [K] from w8a8_act_absmax.  smooth == 0 gives delta = 1 (the
+ * paper's no-smoothing ablation).  Outputs (caller-owned): wq [N, K], s_w [N], delta [K],
+ * inv_delta [K].  wq_f16 (nullable) receives the codes as fp16. */
+w8a8_status w8a8_prepare_weights(const uint16_t* W, int N, int K, const float* act_absmax,
+                                 float alpha, int smooth, int8_t* wq, float* s_w, float* delta,
+                                 float* inv_delta, uint16_t* wq_f16, void* stream);
+
+/* Fused gate/up preparation for the FFN block (FFN section).  gate and up share their input, so
+ * one delta is computed over the column maxima of BOTH matrices (2F rows).  Output row p of the
+ * fused [2F, H] matrix holds, for block q = p / 16 and r = p % 16:
+ *   r < 8 : gate row 8q + r        r >= 8 : up row 8q + r - 8
+ * (blocks of 8 gate rows then the 8 matching up rows), and s_w follows the same order.
+ * F must be a multiple of 8. */
+w8a8_status w8a8_prepare_gate_up(const uint16_t* W_gate, const uint16_t* W_up, int F, int H,
+                                 const float* act_absmax, float alpha, int smooth, int8_t* wq,
+                                 float* s_w, float* delta, float* inv_delta, uint16_t* wq_f16,
+                                 void* stream);
+
+/* The same 8-row interleave for a bf16 pass-through gate/up pair: out [2F, H] bf16. */
+w8a8_status w8a8_interleave_gate_up(const uint16_t* W_gate, const uint16_t* W_up, int F, int H,
+                                    uint16_t* out, void* stream);
+
+/* ------------------------------------------------------ per-token activation quantisation
+ * Dynamic per-token quantisation of the smoothed input (Eq. xhat-lmhead, stx, xint8):
+ *   x_hat_tj = fl32(x_tj * inv_delta_j);  m_t = max_j |x_hat_tj|;  s_x_t = fl32(m_t / 127)
+ *   xq_tj    = clamp(rint(fl32(x_hat_tj * fl32(127 / m_t))), -127, 127)   (0 for a zero row)
+ * X [M, K] bf16.  Outputs: xq [M, K] int8 (nullable), xq_f16 [M, K] the same codes as fp16
+ * (nullable), s_x [M] fp32. */
+w8a8_status w8a8_quantize_activations(const uint16_t* X, int M, int K, const float* inv_delta,
+                                      int8_t* xq, uint16_t* xq_f16, float* s_x, void* stream);
+
+/* ------------------------------------------------------------------------ W8A8 linear
+ * Y = W8A8 linear of X (LM Head section, Eq. xhat-lmhead .. gemm-final):
+ *   acc_ti = sum_j xq_tj * wq_ij (exact INT32);
+ *   y_ti   = fl32(fl32(s_x_t * s_w_i) * fl32(acc_ti)), then + bias_i (fp32), then bf16 (RNE).
+ * X [M, K] bf16, Y [M, N] bf16, bias [N] fp32 nullable.  dbg nullable. */
+w8a8_status w8a8_linear_workspace_size(int M, int N, int K, size_t* bytes);
+w8a8_status w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias,
+                        uint16_t* Y, const w8a8_debug* dbg, void* workspace, size_t ws_bytes,
+                        void* stream);
+
+/* bf16 pass-through linear of a layer outside the INT8 set (FFN section: such layers keep the
+ * original precision): Y = bf16(sum_j x_tj * w_ij (fp32 accumulation) + bias_i).
+ * W [N, K] bf16. */
+w8a8_status w8a8_linear_bf16_workspace_size(int M, int N, int K, size_t* bytes);
+w8a8_status w8a8_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int M,
+                             const float* bias, uint16_t* Y, void* workspace, size_t ws_bytes,
+                             void* stream);
+
+/* ------------------------------------------------------------------------- FFN block
+ * Gemma-3 FFN (FFN section): [g | u] = gate/up linear of X (fp32 out of the epilogue),
+ * h = bf16(gelu_tanh(g) * u), Y = down linear of h (bf16).  precision W8A8_PREC_W8A8 uses
+ * w8a8 (both linears W8A8), W8A8_PREC_BF16 uses the bf16 weights.
+ * gelu_tanh is evaluated by a fixed fp32 recipe (every operation rounded to nearest-even in
+ * this order): g2 = g*g; g3 = g2*g; t = g + 0.044715f*g3; z = 0.7978845608f*t;
+ * w = clamp(-2.8853900818f*z, -126, 126); e = 2^w, where 2^w = 2^n * p(f) with n = rint(w),
+ * f = w - n and p the degree-7 Taylor polynomial of 2^f by Horner's rule; gelu = g / (1 + e).
+ *   h_dbg [M, F] bf16 nullable: receives h. */
+typedef struct {
+  int32_t hidden, inter;
+  w8a8_qweight gate_up;         /* n = 2*inter, k = hidden, 8-row interleave */
+  w8a8_qweight down;            /* n = hidden, k = inter */
+  const uint16_t* gate_up_bf16; /* [2*inter, hidden] bf16, 8-row interleave; nullable if unused */
+  const uint16_t* down_bf16;    /* [hidden, inter] bf16; nullable if unused */
+} w8a8_ffn_weights;
+
+w8a8_status w8a8_ffn_workspace_size(int M, int hidden, int inter, size_t* bytes);
+w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* ffn, int precision, const uint16_t* X, int M,
+                           uint16_t* Y, uint16_t* h_dbg, void* workspace, size_t ws_bytes,
+                           void* stream);
+
+/* --------------------------------------------------------------------------- lm_head
+ * Logits over the tied [V, d] table (LM Head section) and the top-1 index.
+ *   W8A8: logits_tv = fl32(fl32(s_x_t * s_w_v) * fl32(acc_tv)) (fp32, not rounded further).
+ *   BF16: logits_tv = sum_j x_tj * w_vj in fp32.
+ *   top1_t = argmax_v logits_tv (ties go to the lowest v).
+ * X [M, d] bf16 (the final-norm output); logits [M, V] fp32 nullable; top1 [M] int32. */
+typedef struct {
+  int32_t vocab, hidden;
+  w8a8_qweight q;        /* n = vocab, k = hidden */
+  const uint16_t* bf16;  /* [vocab, hidden] bf16 (the embedding table); nullable if unused */
+} w8a8_head_weights;
+
+w8a8_status w8a8_lm_head_workspace_size(int M, int vocab, int hidden, size_t* bytes);
+w8a8_status w8a8_lm_head(const w8a8_head_weights* head, int precision, const uint16_t* X, int M,
+                         float* logits, int32_t* top1, void* workspace, size_t ws_bytes,
+                         void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* W8A8_H */

@@ -1,0 +1,317 @@
+"""Thin ctypes binding of libw8a8.so (argument marshalling only).
+
+Every computation runs in the library's CUDA kernels; this module only turns torch tensors
+(device memory owned by the caller) into the pointers and descriptors of ``include/w8a8.h``,
+allocates output tensors and workspaces with torch, and raises on a non-OK status.  There is
+no CPU fallback: if the library is missing or the device is not sm_103, calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libw8a8.so")
+
+W8A8_PREC_BF16 = 0
+W8A8_PREC_W8A8 = 1
+WS_RESERVED = 65536
+
+STATUS = {0: "OK", 1: "ERR_INVALID_ARG", 2: "ERR_SHAPE", 3: "ERR_ALIGN", 4: "ERR_CUDA", 5: "ERR_UNSUPPORTED",
+          6: "ERR_TIMEOUT", 7: "ERR_WORKSPACE"}
+
+
+class W8A8Error(RuntimeError):
+    def __init__(self, name, status, msg):
+        super().__init__(f"{name} -> {STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int
+_f32 = ctypes.c_float
+_sz = ctypes.c_size_t
+
+
+class QWeightC(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int32), ("k", ctypes.c_int32), ("wq", _vp), ("s_w", _vp), ("inv_delta", _vp),
+                ("wq_f16", _vp)]
+
+
+class DebugC(ctypes.Structure):
+    _fields_ = [("xq", _vp), ("s_x", _vp), ("acc", _vp)]
+
+
+class FfnC(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_int32), ("inter", ctypes.c_int32), ("gate_up", QWeightC), ("down", QWeightC),
+                ("gate_up_bf16", _vp), ("down_bf16", _vp)]
+
+
+class HeadC(ctypes.Structure):
+    _fields_ = [("vocab", ctypes.c_int32), ("hidden", ctypes.c_int32), ("q", QWeightC), ("bf16", _vp)]
+
+
+# name -> (restype, argtypes)
+SIGNATURES = {
+    "w8a8_abi_version": (_i32, []),
+    "w8a8_last_error": (ctypes.c_char_p, []),
+    "w8a8_act_absmax": (_i32, [_vp, _i32, _i32, _vp, _vp]),
+    "w8a8_prepare_weights": (_i32, [_vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "w8a8_prepare_gate_up": (_i32, [_vp, _vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "w8a8_interleave_gate_up": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
+    "w8a8_quantize_activations": (_i32, [_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp]),
+    "w8a8_linear_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
+    "w8a8_linear": (_i32, [ctypes.POINTER(QWeightC), _vp, _i32, _vp, _vp, ctypes.POINTER(DebugC), _vp, _sz, _vp]),
+    "w8a8_linear_bf16_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
+    "w8a8_linear_bf16": (_i32, [_vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+    "w8a8_ffn_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
+    "w8a8_ffn_block": (_i32, [ctypes.POINTER(FfnC), _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+    "w8a8_lm_head_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
+    "w8a8_lm_head": (_i32, [ctypes.POINTER(HeadC), _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+}
+
+_LIB = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libw8a8.so (built by ``paper_2608_28003_gb300.build.build()``); raise if it is absent."""
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built: run paper_2608_28003_gb300.build.build() "
+                               "(the W8A8 path has no CPU fallback)")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _LIB = L
+    return _LIB
+
+
+def _check(name: str, status: int) -> None:
+    if status != 0:
+        raise W8A8Error(name, status, lib().w8a8_last_error().decode())
+
+
+def _p(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _bits(t: torch.Tensor) -> torch.Tensor:
+    assert t.is_cuda and t.is_contiguous(), "tensors must be contiguous CUDA tensors"
+    return t
+
+
+# ------------------------------------------------------------------------------ workspace
+class Workspace:
+    """A zero-initialised device byte buffer, grown on demand (re-zeroed when regrown)."""
+
+    def __init__(self, device=None):
+        self.device = device or torch.device("cuda")
+        self.buf = torch.zeros(WS_RESERVED, dtype=torch.uint8, device=self.device)
+
+    def get(self, nbytes: int) -> torch.Tensor:
+        if self.buf.numel() < nbytes:
+            self.buf = torch.zeros(int(nbytes * 1.25) + 256, dtype=torch.uint8, device=self.device)
+        return self.buf
+
+
+_DEFAULT_WS = {}
+
+
+def default_workspace() -> Workspace:
+    dev = torch.cuda.current_device()
+    if dev not in _DEFAULT_WS:
+        _DEFAULT_WS[dev] = Workspace(torch.device("cuda", dev))
+    return _DEFAULT_WS[dev]
+
+
+def _size(fn_name, *args) -> int:
+    out = ctypes.c_size_t(0)
+    _check(fn_name, getattr(lib(), fn_name)(*args, ctypes.byref(out)))
+    return out.value
+
+
+# ---------------------------------------------------------------------------- descriptors
+@dataclass
+class QWeight:
+    """A prepared W8A8 weight (tensors owned here; the C descriptor points into them)."""
+    wq: torch.Tensor
+    s_w: torch.Tensor
+    delta: torch.Tensor
+    inv_delta: torch.Tensor
+    wq_f16: Optional[torch.Tensor] = None
+
+    @property
+    def n(self):
+        return self.wq.shape[0]
+
+    @property
+    def k(self):
+        return self.wq.shape[1]
+
+    def c(self) -> QWeightC:
+        return QWeightC(self.n, self.k, self.wq.data_ptr(), self.s_w.data_ptr(), self.inv_delta.data_ptr(),
+                        self.wq_f16.data_ptr() if self.wq_f16 is not None else None)
+
+
+# ---------------------------------------------------------------------------- entry points
+def abi_version() -> int:
+    return lib().w8a8_abi_version()
+
+
+def act_absmax(X: torch.Tensor, absmax: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    T, K = X.shape
+    if absmax is None:
+        absmax = torch.zeros(K, dtype=torch.float32, device=X.device)
+    _check("w8a8_act_absmax", lib().w8a8_act_absmax(_p(_bits(X)), T, K, _p(absmax), _stream(stream)))
+    return absmax
+
+
+def prepare_weights(W: torch.Tensor, act_stat: Optional[torch.Tensor], alpha: float = 0.5, smooth: bool = True,
+                    want_f16: bool = False, stream=None) -> QWeight:
+    N, K = W.shape
+    dev = W.device
+    q = QWeight(torch.empty(N, K, dtype=torch.int8, device=dev), torch.empty(N, dtype=torch.float32, device=dev),
+                torch.empty(K, dtype=torch.float32, device=dev), torch.empty(K, dtype=torch.float32, device=dev),
+                torch.empty(N, K, dtype=torch.float16, device=dev) if want_f16 else None)
+    _check("w8a8_prepare_weights", lib().w8a8_prepare_weights(
+        _p(_bits(W)), N, K, _p(act_stat), float(alpha), int(smooth), _p(q.wq), _p(q.s_w), _p(q.delta),
+        _p(q.inv_delta), _p(q.wq_f16), _stream(stream)))
+    return q
+
+
+def prepare_gate_up(W_gate: torch.Tensor, W_up: torch.Tensor, act_stat: Optional[torch.Tensor], alpha: float = 0.5,
+                    smooth: bool = True, want_f16: bool = False, stream=None) -> QWeight:
+    F, H = W_gate.shape
+    dev = W_gate.device
+    q = QWeight(torch.empty(2 * F, H, dtype=torch.int8, device=dev),
+                torch.empty(2 * F, dtype=torch.float32, device=dev),
+                torch.empty(H, dtype=torch.float32, device=dev), torch.empty(H, dtype=torch.float32, device=dev),
+                torch.empty(2 * F, H, dtype=torch.float16, device=dev) if want_f16 else None)
+    _check("w8a8_prepare_gate_up", lib().w8a8_prepare_gate_up(
+        _p(_bits(W_gate)), _p(_bits(W_up)), F, H, _p(act_stat), float(alpha), int(smooth), _p(q.wq), _p(q.s_w),
+        _p(q.delta), _p(q.inv_delta), _p(q.wq_f16), _stream(stream)))
+    return q
+
+
+def interleave_gate_up(W_gate: torch.Tensor, W_up: torch.Tensor, stream=None) -> torch.Tensor:
+    F, H = W_gate.shape
+    out = torch.empty(2 * F, H, dtype=W_gate.dtype, device=W_gate.device)
+    _check("w8a8_interleave_gate_up", lib().w8a8_interleave_gate_up(
+        _p(_bits(W_gate)), _p(_bits(W_up)), F, H, _p(out), _stream(stream)))
+    return out
+
+
+def quantize_activations(X: torch.Tensor, inv_delta: torch.Tensor, stream=None):
+    M, K = X.shape
+    xq = torch.empty(M, K, dtype=torch.int8, device=X.device)
+    xf = torch.empty(M, K, dtype=torch.float16, device=X.device)
+    s_x = torch.empty(M, dtype=torch.float32, device=X.device)
+    _check("w8a8_quantize_activations", lib().w8a8_quantize_activations(
+        _p(_bits(X)), M, K, _p(inv_delta), _p(xq), _p(xf), _p(s_x), _stream(stream)))
+    return xq, xf, s_x
+
+
+def linear(w: QWeight, X: torch.Tensor, bias: Optional[torch.Tensor] = None, debug: bool = False,
+           out: Optional[torch.Tensor] = None, ws: Optional[Workspace] = None, stream=None):
+    M = X.shape[0]
+    Y = out if out is not None else torch.empty(M, w.n, dtype=torch.bfloat16, device=X.device)
+    nbytes = _size("w8a8_linear_workspace_size", M, w.n, w.k)
+    buf = (ws or default_workspace()).get(nbytes)
+    dbg = None
+    dbg_t = None
+    if debug:
+        dbg_t = (torch.empty(M, w.k, dtype=torch.int8, device=X.device),
+                 torch.empty(M, dtype=torch.float32, device=X.device),
+                 torch.empty(M, w.n, dtype=torch.int32, device=X.device))
+        dbg = DebugC(*(t.data_ptr() for t in dbg_t))
+    wc = w.c()
+    _check("w8a8_linear", lib().w8a8_linear(ctypes.byref(wc), _p(_bits(X)), M, _p(bias), _p(Y),
+                                            ctypes.byref(dbg) if dbg is not None else None, _p(buf),
+                                            buf.numel(), _stream(stream)))
+    if debug:
+        return Y, {"xq": dbg_t[0], "s_x": dbg_t[1], "acc": dbg_t[2]}
+    return Y
+
+
+def linear_bf16(W: torch.Tensor, X: torch.Tensor, bias: Optional[torch.Tensor] = None,
+                out: Optional[torch.Tensor] = None, ws: Optional[Workspace] = None, stream=None) -> torch.Tensor:
+    N, K = W.shape
+    M = X.shape[0]
+    Y = out if out is not None else torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+    nbytes = _size("w8a8_linear_bf16_workspace_size", M, N, K)
+    buf = (ws or default_workspace()).get(nbytes)
+    _check("w8a8_linear_bf16", lib().w8a8_linear_bf16(_p(_bits(W)), N, K, _p(_bits(X)), M, _p(bias), _p(Y), _p(buf),
+                                                      buf.numel(), _stream(stream)))
+    return Y
+
+
+@dataclass
+class FfnWeights:
+    hidden: int
+    inter: int
+    gate_up: Optional[QWeight] = None
+    down: Optional[QWeight] = None
+    gate_up_bf16: Optional[torch.Tensor] = None
+    down_bf16: Optional[torch.Tensor] = None
+
+    def c(self) -> FfnC:
+        empty = QWeightC(0, 0, None, None, None, None)
+        return FfnC(self.hidden, self.inter, self.gate_up.c() if self.gate_up else empty,
+                    self.down.c() if self.down else empty,
+                    self.gate_up_bf16.data_ptr() if self.gate_up_bf16 is not None else None,
+                    self.down_bf16.data_ptr() if self.down_bf16 is not None else None)
+
+
+def ffn_block(f: FfnWeights, precision: int, X: torch.Tensor, want_h: bool = False,
+              out: Optional[torch.Tensor] = None, ws: Optional[Workspace] = None, stream=None):
+    M = X.shape[0]
+    Y = out if out is not None else torch.empty(M, f.hidden, dtype=torch.bfloat16, device=X.device)
+    h = torch.empty(M, f.inter, dtype=torch.bfloat16, device=X.device) if want_h else None
+    nbytes = _size("w8a8_ffn_workspace_size", M, f.hidden, f.inter)
+    buf = (ws or default_workspace()).get(nbytes)
+    fc = f.c()
+    _check("w8a8_ffn_block", lib().w8a8_ffn_block(ctypes.byref(fc), int(precision), _p(_bits(X)), M, _p(Y), _p(h),
+                                                  _p(buf), buf.numel(), _stream(stream)))
+    return (Y, h) if want_h else Y
+
+
+@dataclass
+class HeadWeights:
+    vocab: int
+    hidden: int
+    q: Optional[QWeight] = None
+    bf16: Optional[torch.Tensor] = None
+
+    def c(self) -> HeadC:
+        empty = QWeightC(0, 0, None, None, None, None)
+        return HeadC(self.vocab, self.hidden, self.q.c() if self.q else empty,
+                     self.bf16.data_ptr() if self.bf16 is not None else None)
+
+
+def lm_head(hd: HeadWeights, precision: int, X: torch.Tensor, want_logits: bool = True,
+            logits: Optional[torch.Tensor] = None, top1: Optional[torch.Tensor] = None,
+            ws: Optional[Workspace] = None, stream=None):
+    M = X.shape[0]
+    if want_logits and logits is None:
+        logits = torch.empty(M, hd.vocab, dtype=torch.float32, device=X.device)
+    if top1 is None:
+        top1 = torch.empty(M, dtype=torch.int32, device=X.device)
+    nbytes = _size("w8a8_lm_head_workspace_size", M, hd.vocab, hd.hidden)
+    buf = (ws or default_workspace()).get(nbytes)
+    hc = hd.c()
+    _check("w8a8_lm_head", lib().w8a8_lm_head(ctypes.byref(hc), int(precision), _p(_bits(X)), M,
+                                              _p(logits) if want_logits else None, _p(top1), _p(buf), buf.numel(),
+                                              _stream(stream)))
+    return (logits if want_logits else None), top1

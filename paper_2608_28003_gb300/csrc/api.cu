@@ -1,0 +1,377 @@
+// C-ABI entry points of libw8a8: argument checks, workspace carve-up and kernel dispatch for the
+// W8A8 linear, the bf16 pass-through linear, the FFN block and lm_head.
+#include <cstdarg>
+#include <cstdio>
+#include <mutex>
+
+#include "common.cuh"
+#include "stream_gemm.cuh"
+
+namespace w8a8 {
+
+static thread_local char g_err[512] = "";
+
+void set_error(const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+}
+const char* get_error() { return g_err; }
+
+w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* inv_delta, int8_t* xq,
+                                 uint16_t* xq_f16, float* s_x, cudaStream_t st);
+
+// Per-device facts, looked up once per device.
+struct DevInfo {
+  int ok = -1;  // -1 unknown, 0 unsupported, 1 sm_103
+  int sms = 0;
+};
+static DevInfo g_dev[64];
+static std::mutex g_dev_mu;
+
+static w8a8_status dev_info(DevInfo* out) {
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  W8A8_CHECK_ARG(dev >= 0 && dev < 64, W8A8_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  DevInfo& d = g_dev[dev];
+  if (d.ok < 0) {
+    int major = 0, minor = 0, sms = 0;
+    W8A8_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
+    W8A8_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
+    W8A8_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    d.ok = (major == 10 && minor == 3) ? 1 : 0;
+    d.sms = sms;
+  }
+  W8A8_CHECK_ARG(d.ok == 1, W8A8_ERR_UNSUPPORTED, "libw8a8 is built for sm_103 (GB300) only");
+  *out = d;
+  return W8A8_OK;
+}
+
+w8a8_status check_device() {
+  DevInfo d;
+  return dev_info(&d);
+}
+
+int device_sms() {
+  DevInfo d;
+  return dev_info(&d) == W8A8_OK ? d.sms : 152;
+}
+
+// ------------------------------------------------------------------------ workspace plans
+// Layout: [reserved counters | x codes fp16 [M,K] | s_x [M] | partials]
+struct LinearWs {
+  size_t xf16, sx, part, total;
+};
+
+static LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
+  LinearWs w{};
+  size_t off = W8A8_WS_RESERVED;
+  w.xf16 = off;
+  if (int8_path) off += round_up((size_t)M * K * 2, 256);
+  w.sx = off;
+  if (int8_path) off += round_up((size_t)M * 4, 256);
+  w.part = off;
+  off += round_up(make_stream_plan(M, N, K, sms).partial_bytes, 256);
+  w.total = off;
+  return w;
+}
+
+static w8a8_status check_qweight(const char* who, const w8a8_qweight* w) {
+  W8A8_CHECK_ARG(w != nullptr, W8A8_ERR_INVALID_ARG, "%s: null weight descriptor", who);
+  W8A8_CHECK_ARG(w->n > 0 && w->k > 0, W8A8_ERR_SHAPE, "%s: weight shape [%d, %d] must be positive", who, w->n, w->k);
+  W8A8_CHECK_ARG(w->k % 16 == 0 && w->k <= W8A8_MAX_K, W8A8_ERR_SHAPE, "%s: K=%d must be a multiple of 16 and <= %d",
+                 who, w->k, W8A8_MAX_K);
+  W8A8_CHECK_ARG(w->wq && w->s_w && w->inv_delta, W8A8_ERR_INVALID_ARG, "%s: null weight pointer", who);
+  W8A8_CHECK_ARG(aligned16(w->wq) && aligned16(w->s_w) && aligned16(w->inv_delta) && (!w->wq_f16 || aligned16(w->wq_f16)),
+                 W8A8_ERR_ALIGN, "%s: weight pointers must be 16-byte aligned", who);
+  return W8A8_OK;
+}
+
+static w8a8_status check_ws(const char* who, void* ws, size_t have, size_t need) {
+  W8A8_CHECK_ARG(ws != nullptr && have >= need, W8A8_ERR_WORKSPACE, "%s: workspace %zu bytes, need %zu", who,
+                 ws ? have : 0, need);
+  W8A8_CHECK_ARG(aligned16(ws), W8A8_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
+  return W8A8_OK;
+}
+
+#define W8A8_TRY(expr)              \
+  do {                              \
+    w8a8_status s_ = (expr);        \
+    if (s_ != W8A8_OK) return s_;   \
+  } while (0)
+
+// One W8A8 linear: K1 then the streaming GEMM.  s_x/xf16 live in the workspace.
+static w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
+                                   uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
+                                   int sms, cudaStream_t st) {
+  const int N = w->n, K = w->k;
+  LinearWs L = linear_ws(M, N, K, true, sms);
+  char* base = reinterpret_cast<char*>(ws);
+  uint16_t* xf16 = reinterpret_cast<uint16_t*>(base + L.xf16);
+  float* s_x = reinterpret_cast<float*>(base + L.sx);
+  W8A8_TRY(launch_quantize_rows(X, M, K, w->inv_delta, dbg ? dbg->xq : nullptr, xf16, s_x, st));
+  if (dbg && dbg->s_x) W8A8_CUDA(cudaMemcpyAsync(dbg->s_x, s_x, sizeof(float) * M, cudaMemcpyDeviceToDevice, st));
+  StreamArgs a{};
+  a.W = w->wq;
+  a.X = xf16;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.p = make_stream_plan(M, N, K, sms);
+  a.kind = kind;
+  a.s_x = s_x;
+  a.s_w = w->s_w;
+  a.bias = bias;
+  a.y = Y;
+  a.logits = logits;
+  a.top1 = top1;
+  a.acc_dbg = dbg ? dbg->acc : nullptr;
+  a.partials = base + L.part;
+  attach_reserved(a, ws);
+  return launch_stream_gemm(true, a, st);
+}
+
+static w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias,
+                                   int kind, uint16_t* Y, float* logits, int32_t* top1, void* ws, int sms,
+                                   cudaStream_t st) {
+  LinearWs L = linear_ws(M, N, K, false, sms);
+  StreamArgs a{};
+  a.W = W;
+  a.X = X;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.p = make_stream_plan(M, N, K, sms);
+  a.kind = kind;
+  a.bias = bias;
+  a.y = Y;
+  a.logits = logits;
+  a.top1 = top1;
+  a.partials = reinterpret_cast<char*>(ws) + L.part;
+  attach_reserved(a, ws);
+  return launch_stream_gemm(false, a, st);
+}
+
+}  // namespace w8a8
+
+using namespace w8a8;
+
+extern "C" int w8a8_abi_version(void) { return 1; }
+extern "C" const char* w8a8_last_error(void) { return get_error(); }
+
+// ---------------------------------------------------------------------------- linear
+extern "C" w8a8_status w8a8_linear_workspace_size(int M, int N, int K, size_t* bytes) {
+  W8A8_CHECK_ARG(bytes && M >= 0 && N >= 0 && K >= 0, W8A8_ERR_INVALID_ARG, "w8a8_linear_workspace_size: bad argument");
+  *bytes = linear_ws(M, N, K, true, device_sms()).total;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, uint16_t* Y,
+                                   const w8a8_debug* dbg, void* workspace, size_t ws_bytes, void* stream) {
+  W8A8_TRY(check_qweight("w8a8_linear", w));
+  W8A8_CHECK_ARG(M >= 0, W8A8_ERR_INVALID_ARG, "w8a8_linear: M=%d is negative", M);
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(X && Y, W8A8_ERR_INVALID_ARG, "w8a8_linear: null X or Y");
+  W8A8_CHECK_ARG(aligned16(X) && aligned16(Y) && (!bias || aligned16(bias)), W8A8_ERR_ALIGN,
+                 "w8a8_linear: X, Y and bias must be 16-byte aligned");
+  if (dbg)
+    W8A8_CHECK_ARG((!dbg->xq || aligned16(dbg->xq)) && (!dbg->s_x || aligned16(dbg->s_x)) &&
+                       (!dbg->acc || aligned16(dbg->acc)),
+                   W8A8_ERR_ALIGN, "w8a8_linear: debug outputs must be 16-byte aligned");
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));
+  W8A8_TRY(check_ws("w8a8_linear", workspace, ws_bytes, linear_ws(M, w->n, w->k, true, d.sms).total));
+  return run_w8a8_linear(w, X, M, bias, EPI_BF16, Y, nullptr, nullptr, dbg, workspace, d.sms, as_stream(stream));
+}
+
+extern "C" w8a8_status w8a8_linear_bf16_workspace_size(int M, int N, int K, size_t* bytes) {
+  W8A8_CHECK_ARG(bytes && M >= 0 && N >= 0 && K >= 0, W8A8_ERR_INVALID_ARG,
+                 "w8a8_linear_bf16_workspace_size: bad argument");
+  *bytes = linear_ws(M, N, K, false, device_sms()).total;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_linear_bf16(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias,
+                                        uint16_t* Y, void* workspace, size_t ws_bytes, void* stream) {
+  W8A8_CHECK_ARG(M >= 0 && N > 0 && K > 0, W8A8_ERR_SHAPE, "w8a8_linear_bf16: bad shape M=%d N=%d K=%d", M, N, K);
+  W8A8_CHECK_ARG(K % 16 == 0 && K <= W8A8_MAX_K, W8A8_ERR_SHAPE, "w8a8_linear_bf16: K=%d must be a multiple of 16", K);
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(W && X && Y, W8A8_ERR_INVALID_ARG, "w8a8_linear_bf16: null pointer");
+  W8A8_CHECK_ARG(aligned16(W) && aligned16(X) && aligned16(Y) && (!bias || aligned16(bias)), W8A8_ERR_ALIGN,
+                 "w8a8_linear_bf16: pointers must be 16-byte aligned");
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));
+  W8A8_TRY(check_ws("w8a8_linear_bf16", workspace, ws_bytes, linear_ws(M, N, K, false, d.sms).total));
+  return run_bf16_linear(W, N, K, X, M, bias, EPI_BF16, Y, nullptr, nullptr, workspace, d.sms, as_stream(stream));
+}
+
+// ------------------------------------------------------------------------------- FFN
+// Layout: [reserved | h bf16 [M,F] | gate/up linear scratch | down linear scratch]
+struct FfnWs {
+  size_t h, gu, dn, total;
+};
+static FfnWs ffn_ws(int M, int H, int F, int sms) {
+  FfnWs w{};
+  size_t off = W8A8_WS_RESERVED;
+  w.h = off;
+  off += round_up((size_t)M * F * 2, 256);
+  const LinearWs a = linear_ws(M, 2 * F, H, true, sms);
+  const LinearWs b = linear_ws(M, H, F, true, sms);
+  w.gu = off;
+  off += a.total - W8A8_WS_RESERVED;
+  w.dn = off;
+  off += b.total - W8A8_WS_RESERVED;
+  w.total = off;
+  return w;
+}
+
+extern "C" w8a8_status w8a8_ffn_workspace_size(int M, int hidden, int inter, size_t* bytes) {
+  W8A8_CHECK_ARG(bytes && M >= 0 && hidden >= 0 && inter >= 0, W8A8_ERR_INVALID_ARG, "w8a8_ffn_workspace_size: bad argument");
+  *bytes = ffn_ws(M, hidden, inter, device_sms()).total;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y,
+                                      uint16_t* h_dbg, void* workspace, size_t ws_bytes, void* stream) {
+  W8A8_CHECK_ARG(f != nullptr, W8A8_ERR_INVALID_ARG, "w8a8_ffn_block: null FFN descriptor");
+  W8A8_CHECK_ARG(precision == W8A8_PREC_BF16 || precision == W8A8_PREC_W8A8, W8A8_ERR_INVALID_ARG,
+                 "w8a8_ffn_block: precision %d", precision);
+  const int H = f->hidden, F = f->inter;
+  W8A8_CHECK_ARG(H > 0 && F > 0 && H % 16 == 0 && F % 16 == 0 && H <= W8A8_MAX_K && F <= W8A8_MAX_K, W8A8_ERR_SHAPE,
+                 "w8a8_ffn_block: hidden=%d inter=%d must be positive multiples of 16", H, F);
+  W8A8_CHECK_ARG(M >= 0, W8A8_ERR_INVALID_ARG, "w8a8_ffn_block: M=%d is negative", M);
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(X && Y, W8A8_ERR_INVALID_ARG, "w8a8_ffn_block: null X or Y");
+  W8A8_CHECK_ARG(aligned16(X) && aligned16(Y) && (!h_dbg || aligned16(h_dbg)), W8A8_ERR_ALIGN,
+                 "w8a8_ffn_block: X, Y, h must be 16-byte aligned");
+  if (precision == W8A8_PREC_W8A8) {
+    W8A8_TRY(check_qweight("w8a8_ffn_block(gate_up)", &f->gate_up));
+    W8A8_TRY(check_qweight("w8a8_ffn_block(down)", &f->down));
+    W8A8_CHECK_ARG(f->gate_up.n == 2 * F && f->gate_up.k == H && f->down.n == H && f->down.k == F, W8A8_ERR_SHAPE,
+                   "w8a8_ffn_block: weight shapes do not match hidden=%d inter=%d", H, F);
+  } else {
+    W8A8_CHECK_ARG(f->gate_up_bf16 && f->down_bf16, W8A8_ERR_INVALID_ARG, "w8a8_ffn_block: null bf16 weights");
+    W8A8_CHECK_ARG(aligned16(f->gate_up_bf16) && aligned16(f->down_bf16), W8A8_ERR_ALIGN,
+                   "w8a8_ffn_block: bf16 weights must be 16-byte aligned");
+  }
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));
+  const FfnWs L = ffn_ws(M, H, F, d.sms);
+  W8A8_TRY(check_ws("w8a8_ffn_block", workspace, ws_bytes, L.total));
+  cudaStream_t st = as_stream(stream);
+  char* base = reinterpret_cast<char*>(workspace);
+  uint16_t* h = h_dbg ? h_dbg : reinterpret_cast<uint16_t*>(base + L.h);
+  // The two linears run one after the other on `stream` and share the FFN workspace's reserved
+  // counters (each leaves them zero); their scratch regions are disjoint.
+  if (precision == W8A8_PREC_W8A8) {
+    // gate/up: scratch at L.gu
+    {
+      const LinearWs A = linear_ws(M, 2 * F, H, true, d.sms);
+      uint16_t* xf16 = reinterpret_cast<uint16_t*>(base + L.gu + (A.xf16 - W8A8_WS_RESERVED));
+      float* s_x = reinterpret_cast<float*>(base + L.gu + (A.sx - W8A8_WS_RESERVED));
+      W8A8_TRY(launch_quantize_rows(X, M, H, f->gate_up.inv_delta, nullptr, xf16, s_x, st));
+      StreamArgs a{};
+      a.W = f->gate_up.wq;
+      a.X = xf16;
+      a.M = M;
+      a.N = 2 * F;
+      a.K = H;
+      a.p = make_stream_plan(M, 2 * F, H, d.sms);
+      a.kind = EPI_GEGLU;
+      a.s_x = s_x;
+      a.s_w = f->gate_up.s_w;
+      a.y = h;
+      a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(true, a, st));
+    }
+    {
+      const LinearWs B = linear_ws(M, H, F, true, d.sms);
+      uint16_t* xf16 = reinterpret_cast<uint16_t*>(base + L.dn + (B.xf16 - W8A8_WS_RESERVED));
+      float* s_x = reinterpret_cast<float*>(base + L.dn + (B.sx - W8A8_WS_RESERVED));
+      W8A8_TRY(launch_quantize_rows(h, M, F, f->down.inv_delta, nullptr, xf16, s_x, st));
+      StreamArgs a{};
+      a.W = f->down.wq;
+      a.X = xf16;
+      a.M = M;
+      a.N = H;
+      a.K = F;
+      a.p = make_stream_plan(M, H, F, d.sms);
+      a.kind = EPI_BF16;
+      a.s_x = s_x;
+      a.s_w = f->down.s_w;
+      a.y = Y;
+      a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(true, a, st));
+    }
+  } else {
+    {
+      const LinearWs A = linear_ws(M, 2 * F, H, false, d.sms);
+      StreamArgs a{};
+      a.W = f->gate_up_bf16;
+      a.X = X;
+      a.M = M;
+      a.N = 2 * F;
+      a.K = H;
+      a.p = make_stream_plan(M, 2 * F, H, d.sms);
+      a.kind = EPI_GEGLU;
+      a.y = h;
+      a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(false, a, st));
+    }
+    {
+      const LinearWs B = linear_ws(M, H, F, false, d.sms);
+      StreamArgs a{};
+      a.W = f->down_bf16;
+      a.X = h;
+      a.M = M;
+      a.N = H;
+      a.K = F;
+      a.p = make_stream_plan(M, H, F, d.sms);
+      a.kind = EPI_BF16;
+      a.y = Y;
+      a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(false, a, st));
+    }
+  }
+  return W8A8_OK;
+}
+
+// --------------------------------------------------------------------------- lm_head
+extern "C" w8a8_status w8a8_lm_head_workspace_size(int M, int vocab, int hidden, size_t* bytes) {
+  W8A8_CHECK_ARG(bytes && M >= 0 && vocab >= 0 && hidden >= 0, W8A8_ERR_INVALID_ARG, "w8a8_lm_head_workspace_size: bad argument");
+  *bytes = linear_ws(M, vocab, hidden, true, device_sms()).total;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_lm_head(const w8a8_head_weights* hd, int precision, const uint16_t* X, int M, float* logits,
+                                    int32_t* top1, void* workspace, size_t ws_bytes, void* stream) {
+  W8A8_CHECK_ARG(hd != nullptr, W8A8_ERR_INVALID_ARG, "w8a8_lm_head: null head descriptor");
+  W8A8_CHECK_ARG(precision == W8A8_PREC_BF16 || precision == W8A8_PREC_W8A8, W8A8_ERR_INVALID_ARG,
+                 "w8a8_lm_head: precision %d", precision);
+  const int V = hd->vocab, D = hd->hidden;
+  W8A8_CHECK_ARG(V > 0 && D > 0 && D % 16 == 0 && D <= W8A8_MAX_K, W8A8_ERR_SHAPE, "w8a8_lm_head: vocab=%d hidden=%d", V, D);
+  W8A8_CHECK_ARG(M >= 0, W8A8_ERR_INVALID_ARG, "w8a8_lm_head: M=%d is negative", M);
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(M <= max_top_keys(), W8A8_ERR_SHAPE, "w8a8_lm_head: M=%d exceeds %d tokens per call", M, max_top_keys());
+  W8A8_CHECK_ARG(X && top1, W8A8_ERR_INVALID_ARG, "w8a8_lm_head: null X or top1");
+  W8A8_CHECK_ARG(aligned16(X) && aligned16(top1) && (!logits || aligned16(logits)), W8A8_ERR_ALIGN,
+                 "w8a8_lm_head: pointers must be 16-byte aligned");
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));
+  cudaStream_t st = as_stream(stream);
+  if (precision == W8A8_PREC_W8A8) {
+    W8A8_TRY(check_qweight("w8a8_lm_head", &hd->q));
+    W8A8_CHECK_ARG(hd->q.n == V && hd->q.k == D, W8A8_ERR_SHAPE, "w8a8_lm_head: weight shape mismatch");
+    W8A8_TRY(check_ws("w8a8_lm_head", workspace, ws_bytes, linear_ws(M, V, D, true, d.sms).total));
+    return run_w8a8_linear(&hd->q, X, M, nullptr, EPI_F32, nullptr, logits, top1, nullptr, workspace, d.sms, st);
+  }
+  W8A8_CHECK_ARG(hd->bf16 && aligned16(hd->bf16), W8A8_ERR_INVALID_ARG, "w8a8_lm_head: null or unaligned bf16 table");
+  W8A8_TRY(check_ws("w8a8_lm_head", workspace, ws_bytes, linear_ws(M, V, D, false, d.sms).total));
+  return run_bf16_linear(hd->bf16, V, D, X, M, nullptr, EPI_F32, nullptr, logits, top1, workspace, d.sms, st);
+}

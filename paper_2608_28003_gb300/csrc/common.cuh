@@ -1,0 +1,155 @@
+// Shared device/host helpers of libw8a8 (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "../../include/w8a8.h"
+
+namespace w8a8 {
+
+// ------------------------------------------------------------------------- host status
+void set_error(const char* fmt, ...);
+const char* get_error();
+
+#define W8A8_CHECK_ARG(cond, code, ...)   \
+  do {                                    \
+    if (!(cond)) {                        \
+      ::w8a8::set_error(__VA_ARGS__);     \
+      return code;                        \
+    }                                     \
+  } while (0)
+
+#define W8A8_CUDA(call)                                                                        \
+  do {                                                                                         \
+    cudaError_t e_ = (call);                                                                   \
+    if (e_ != cudaSuccess) {                                                                   \
+      ::w8a8::set_error("CUDA error %s at %s:%d", cudaGetErrorString(e_), __FILE__, __LINE__); \
+      return W8A8_ERR_CUDA;                                                                    \
+    }                                                                                          \
+  } while (0)
+
+#define W8A8_LAUNCH_CHECK() W8A8_CUDA(cudaGetLastError())
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
+inline size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+w8a8_status check_device();  // current device must be sm_103
+
+// ---------------------------------------------------------------------- exact conversions
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint16_t f32_to_bf16_bits(float x) {
+  __nv_bfloat16 b = __float2bfloat16_rn(x);
+  return *reinterpret_cast<uint16_t*>(&b);
+}
+
+// int8 code (as int) -> fp16 bit pattern; exact for |q| <= 2048.
+__device__ __forceinline__ uint16_t int_to_f16_bits(int q) {
+  __half h = __int2half_rn(q);
+  return *reinterpret_cast<uint16_t*>(&h);
+}
+
+// Four signed bytes of `w` (byte b0 lowest) -> two f16x2 words {f16(b0), f16(b1)} and
+// {f16(b2), f16(b3)}, exact for codes in [-128, 127].  Flipping the sign bit of each byte gives
+// u = b + 128 in [0, 255]; the half 0x6400 | u is 1024 + u exactly, so subtracting 1152 leaves b.
+__device__ __forceinline__ void i8x4_to_f16x2x2(uint32_t w, uint32_t& lo, uint32_t& hi) {
+  const uint32_t u = w ^ 0x80808080u;
+  const uint32_t plo = __byte_perm(u, 0x64646464u, 0x4140u);
+  const uint32_t phi = __byte_perm(u, 0x64646464u, 0x4342u);
+  const __half2 bias = __halves2half2(__ushort_as_half(0x6480u), __ushort_as_half(0x6480u));  // 1152
+  __half2 a = __hsub2(*reinterpret_cast<const __half2*>(&plo), bias);
+  __half2 b = __hsub2(*reinterpret_cast<const __half2*>(&phi), bias);
+  lo = *reinterpret_cast<uint32_t*>(&a);
+  hi = *reinterpret_cast<uint32_t*>(&b);
+}
+
+// ------------------------------------------------------------------------- legacy MMA
+// D[16x8] += A[16x16] * B[16x8], fp32 accumulate.
+__device__ __forceinline__ void mma_f16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                              uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                               uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// ----------------------------------------------------------------- streaming global loads
+__device__ __forceinline__ uint4 ldg_stream(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint4 ldg_keep(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// --------------------------------------------------------------------- GeGLU fp32 recipe
+// gelu_tanh(g) = g / (1 + 2^w), w = -2 log2(e) * sqrt(2/pi) * (g + 0.044715 g^3), each step one
+// IEEE fp32 operation rounded to nearest-even, in the order below (no contraction into FMA).
+// 2^w = 2^n * p(f), n = rint(w), f = w - n in [-1/2, 1/2], p = degree-7 Taylor polynomial of
+// e^{f ln 2} (coefficients (ln 2)^k / k! rounded to fp32), Horner's rule.
+__device__ __forceinline__ float exp2_recipe(float w) {
+  const float n = rintf(w);
+  const float f = __fsub_rn(w, n);
+  float p = __uint_as_float(0x377fe5feu);  // (ln2)^7/7!
+  p = __fadd_rn(__fmul_rn(p, f), __uint_as_float(0x39218489u));  // (ln2)^6/6!
+  p = __fadd_rn(__fmul_rn(p, f), __uint_as_float(0x3aaec3ffu));  // (ln2)^5/5!
+  p = __fadd_rn(__fmul_rn(p, f), __uint_as_float(0x3c1d955bu));  // (ln2)^4/4!
+  p = __fadd_rn(__fmul_rn(p, f), __uint_as_float(0x3d635847u));  // (ln2)^3/3!
+  p = __fadd_rn(__fmul_rn(p, f), __uint_as_float(0x3e75fdf0u));  // (ln2)^2/2!
+  p = __fadd_rn(__fmul_rn(p, f), __uint_as_float(0x3f317218u));  // ln2
+  p = __fadd_rn(__fmul_rn(p, f), 1.0f);
+  const int ni = __float2int_rn(n);                      // |n| <= 126
+  const float scale = __int_as_float((ni + 127) << 23);  // 2^n, a normal number
+  return __fmul_rn(p, scale);
+}
+
+__device__ __forceinline__ float gelu_tanh_recipe(float g) {
+  const float g2 = __fmul_rn(g, g);
+  const float g3 = __fmul_rn(g2, g);
+  const float t = __fadd_rn(g, __fmul_rn(__uint_as_float(0x3d372713u), g3));  // 0.044715
+  const float z = __fmul_rn(__uint_as_float(0x3f4c422au), t);                  // sqrt(2/pi)
+  float w = __fmul_rn(__uint_as_float(0xc038aa3bu), z);                        // -2 log2(e)
+  w = fminf(fmaxf(w, -126.0f), 126.0f);
+  const float e = exp2_recipe(w);
+  return __fdiv_rn(g, __fadd_rn(1.0f, e));
+}
+
+__device__ __forceinline__ float geglu_recipe(float g, float u) { return __fmul_rn(gelu_tanh_recipe(g), u); }
+
+// ------------------------------------------------------------------------- reductions
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Orderable key for a float (NaN-free): larger float -> larger key.
+__device__ __forceinline__ uint32_t float_order_key(float v) {
+  const uint32_t b = __float_as_uint(v + 0.0f);  // -0 -> +0
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+}  // namespace w8a8

@@ -1,0 +1,196 @@
+"""GPU parity of the W8A8 linear path against the oracle, through the C ABI.
+
+Bar: INT8 codes, INT32 accumulators, fp32 scales, bf16/fp32 outputs of the W8A8 path are
+bit-exact; the bf16 pass-through is within 1 bf16 ulp plus the fp32 accumulation bound
+(K * 2^-24 * sum |x w|) of the oracle's fp64 sum.
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import blocks as OB
+from oracle import w8a8 as OW
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def B():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2608_28003_gb300 import build
+    build.build()
+    from paper_2608_28003_gb300 import binding
+    return binding
+
+
+def cu(t):
+    return t.contiguous().cuda()
+
+
+def bits16(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def f32_of_bf16(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().float().numpy()
+
+
+def _case(M, N, K, seed, n_out=4):
+    x32, x, ch = synth.activations(M, K, min(n_out, K), seed)
+    w32, w = synth.weight(N, K, seed)
+    c32, c, _ = synth.activations(max(M, 8), K, min(n_out, K), seed, stream=1, channels=ch)
+    return x32, x, w32, w, c32, c
+
+
+# ------------------------------------------------------------------ K1 activation quantiser
+@pytest.mark.parametrize("M,K", [(1, 1152), (16, 1152), (3, 16), (37, 6912), (5, 9216), (130, 1040)])
+def test_quantize_activations_bit_exact(B, M, K):
+    x32, x, _ = synth.activations(M, K, min(8, K), seed=M + K)
+    inv = np.random.default_rng(K).uniform(0.05, 20.0, K).astype(np.float32)
+    if M > 2:
+        x32[2] = 0.0
+        x[2] = 0
+    xq, xf, sx = B.quantize_activations(cu(x), cu(torch.from_numpy(inv)))
+    oq, os_ = OW.quantize_activations(x32, inv)
+    assert np.array_equal(xq.cpu().numpy(), oq)
+    assert np.array_equal(sx.cpu().numpy().view(np.uint32), os_.view(np.uint32))
+    assert np.array_equal(xf.cpu().float().numpy(), oq.astype(np.float32))
+
+
+def test_act_absmax_bit_exact(B):
+    x32, x, _ = synth.activations(300, 1152, 12, seed=5)
+    am = B.act_absmax(cu(x))
+    am = B.act_absmax(cu(x[:7] * 3), am)
+    ref = np.maximum(OW.act_absmax(x32), OW.act_absmax((x[:7] * 3).float().numpy()))
+    assert np.array_equal(am.cpu().numpy(), ref)
+
+
+# ------------------------------------------------------------------------- weight prep
+@pytest.mark.parametrize("N,K,alpha,smooth", [(6912, 1152, 0.5, True), (100, 64, 0.5, False), (40, 6912, 0.5, True),
+                                              (33, 1040, 0.3, True)])
+def test_prepare_weights(B, N, K, alpha, smooth):
+    _, _, w32, w, c32, c = _case(8, N, K, seed=N)
+    stat = OW.act_absmax(c32)
+    stat[5] = 0.0
+    q = B.prepare_weights(cu(w), cu(torch.from_numpy(stat)), alpha, smooth, want_f16=True)
+    ref = OW.prepare_weights(w32, stat, alpha, smooth)
+    if alpha == 0.5:
+        assert np.array_equal(q.delta.cpu().numpy(), ref["delta"])
+        assert np.array_equal(q.inv_delta.cpu().numpy(), ref["inv_delta"])
+        assert np.array_equal(q.wq.cpu().numpy(), ref["wq"])
+        assert np.array_equal(q.s_w.cpu().numpy(), ref["s_w"])
+    else:  # fp64 pow on both sides, one rounding to fp32: at most 1 ulp apart
+        d = q.delta.cpu().numpy()
+        assert np.all(np.abs(d.view(np.int32) - ref["delta"].view(np.int32)) <= 1)
+        same = d == ref["delta"]
+        assert same.mean() > 0.99
+        assert np.array_equal(q.wq.cpu().numpy()[:, same], ref["wq"][:, same])
+    assert np.array_equal(q.wq_f16.cpu().float().numpy(), q.wq.cpu().numpy().astype(np.float32))
+
+
+def deinterleave_rows(a: np.ndarray, F: int) -> np.ndarray:
+    """Inverse of the 8-row gate/up interleave: fused row p -> [gate; up] row."""
+    p = np.arange(2 * F)
+    q, r = p // 16, p % 16
+    dst = np.where(r < 8, 8 * q + r, F + 8 * q + r - 8)
+    out = np.empty_like(a)
+    out[dst] = a
+    return out
+
+
+def test_prepare_gate_up_and_interleave(B):
+    F, H = 6912, 1152
+    c = synth.ffn_case(4, seed=3, calib_rows=64)
+    stat = OW.act_absmax(c["calib32"])
+    q = B.prepare_gate_up(cu(c["wg"]), cu(c["wu"]), cu(torch.from_numpy(stat)))
+    ref = OW.prepare_weights(np.concatenate([c["wg32"], c["wu32"]]), stat)
+    assert np.array_equal(q.delta.cpu().numpy(), ref["delta"])
+    assert np.array_equal(deinterleave_rows(q.wq.cpu().numpy(), F), ref["wq"])
+    assert np.array_equal(deinterleave_rows(q.s_w.cpu().numpy(), F), ref["s_w"])
+    il = B.interleave_gate_up(cu(c["wg"]), cu(c["wu"]))
+    assert np.array_equal(deinterleave_rows(bits16(il), F), np.concatenate([bits16(c["wg"]), bits16(c["wu"])]))
+
+
+# ------------------------------------------------------------------------- W8A8 linear
+LINEAR_SHAPES = [
+    (16, 6912, 1152),   # the single-linear workload (gate_proj shape, M = 16)
+    (1, 1000, 1152),    # ragged N
+    (3, 24, 64),
+    (9, 4112, 1040),    # ragged K (not a multiple of 64)
+    (17, 200, 6912),    # K-split across CTAs
+    (33, 520, 1152),
+    (64, 1152, 6912),   # down_proj shape
+    (130, 300, 256),    # several token groups with a ragged tail
+]
+
+
+@pytest.mark.parametrize("M,N,K", LINEAR_SHAPES)
+def test_w8a8_linear_bit_exact(B, M, N, K):
+    x32, x, w32, w, c32, c = _case(M, N, K, seed=M * 7 + N)
+    stat = OW.act_absmax(np.concatenate([c32, x32]))
+    q = B.prepare_weights(cu(w), cu(torch.from_numpy(stat)))
+    bias = None
+    if N == 1000:
+        bias = np.random.default_rng(1).standard_normal(N).astype(np.float32)
+    Y, dbg = B.linear(q, cu(x), bias=cu(torch.from_numpy(bias)) if bias is not None else None, debug=True)
+    prep = OW.prepare_weights(w32, stat)
+    r = OW.w8a8_linear(x32, prep, bias=bias, out="bf16")
+    assert np.array_equal(dbg["xq"].cpu().numpy(), r["xq"])
+    assert np.array_equal(dbg["s_x"].cpu().numpy(), r["s_x"])
+    assert np.array_equal(dbg["acc"].cpu().numpy().astype(np.int64), r["acc"])
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+
+
+def test_single_linear_workload_calibrated_on_its_input(B):
+    """M = 16, K = 1152, N = 6912, 8 outlier channels x20, delta from X itself (seed 0)."""
+    c = synth.linear_case()
+    stat = OW.act_absmax(c["calib32"])
+    q = B.prepare_weights(cu(c["w"]), cu(torch.from_numpy(stat)))
+    Y, dbg = B.linear(q, cu(c["x"]), debug=True)
+    r = OW.w8a8_linear(c["x32"], OW.prepare_weights(c["w32"], stat), out="bf16")
+    assert np.array_equal(dbg["acc"].cpu().numpy().astype(np.int64), r["acc"])
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+    # every token row has an outlier channel mapped to +-127
+    assert np.all(np.abs(r["xq"].astype(int)).max(axis=1) == 127)
+
+
+@pytest.mark.parametrize("K", [1024, 1152, 6912])
+def test_w8a8_accumulator_exact_at_extremes(B, K):
+    """All codes +-127 (delta = 1, constant-magnitude rows), |acc| up to 127^2 K > 2^24: the fp32
+    MMA accumulation is folded into INT32 before it can round."""
+    M, N = 8, 48
+    g = np.random.default_rng(K)
+    x = np.where(g.random((M, K)) < 0.5, -1.0, 1.0).astype(np.float32)
+    x[0] = 1.0
+    w = np.where(g.random((N, K)) < 0.5, -0.5, 0.5).astype(np.float32)
+    w[0] = 0.5
+    w[1] = -0.5
+    w[2, : K // 2] = 0.5
+    w[2, K // 2:] = -0.5
+    xt = torch.from_numpy(x).to(torch.bfloat16)
+    wt = torch.from_numpy(w).to(torch.bfloat16)
+    q = B.prepare_weights(cu(wt), None, 0.5, False)
+    assert np.all(np.abs(q.wq.cpu().numpy()) == 127)
+    Y, dbg = B.linear(q, cu(xt), debug=True)
+    r = OW.w8a8_linear(x, OW.prepare_weights(w, None, smooth=False), out="bf16")
+    acc = dbg["acc"].cpu().numpy().astype(np.int64)
+    assert np.array_equal(acc, r["acc"]) and acc[0, 0] == 127 * 127 * K
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+
+
+# ---------------------------------------------------------------------- bf16 pass-through
+def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarray):
+    K = X.shape[1]
+    mag = np.abs(X).astype(np.float64) @ np.abs(W).astype(np.float64).T
+    ulp = np.spacing(np.abs(y_ref).astype(np.float32)) * 2 ** 16  # bf16 ulp = 2^16 fp32 ulps
+    bound = ulp + K * 2.0 ** -24 * mag + 1e-30
+    assert np.all(np.abs(y_gpu.astype(np.float64) - y_ref) <= bound)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040)])
+def test_bf16_linear_within_tolerance(B, M, N, K):
+    x32, x, w32, w, _, _ = _case(M, N, K, seed=11 + M)
+    Y = B.linear_bf16(cu(w), cu(x))
+    ref = OW.bf16_linear(x32, w32, out="bf16")
+    _bf16_close(f32_of_bf16(Y), x32, w32, ref)
