@@ -57,6 +57,20 @@ int w8a8_abi_version(void);
 /* Message for the last non-OK status returned on the calling thread ("" if none). */
 const char* w8a8_last_error(void);
 
+/* Waits for `stream`, then reads and clears the workspace's device error word.  Kernels never
+ * wait without a bound: a wait that gives up (about 2 s) sets a bit of this word, skips the rest
+ * of its work and returns, so the context stays usable.  Returns W8A8_ERR_TIMEOUT if any bit was
+ * set since the last check (the outputs of the calls in between are then undefined), W8A8_OK
+ * otherwise.  This call is synchronous. */
+w8a8_status w8a8_workspace_check(void* workspace, void* stream);
+
+/* Measurement aid: the calling thread's next weight-streaming GEMM launch (inside w8a8_linear,
+ * w8a8_linear_bf16, w8a8_ffn_block or w8a8_lm_head) records `start_event` (a cudaEvent_t) on its
+ * stream just before the kernel and `stop_event` just after it, then forgets both.  The events
+ * bracket the GEMM kernel alone, not the per-token quantiser launched before it.  Both or
+ * neither (NULL, NULL clears a pending request). */
+w8a8_status w8a8_set_kernel_events(void* start_event, void* stop_event);
+
 /* ---------------------------------------------------------------------------------------
  * Prepared W8A8 weight of one linear (produced by w8a8_prepare_weights /
  * w8a8_prepare_gate_up, owned by the caller).

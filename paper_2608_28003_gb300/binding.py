@@ -59,6 +59,8 @@ class HeadC(ctypes.Structure):
 SIGNATURES = {
     "w8a8_abi_version": (_i32, []),
     "w8a8_last_error": (ctypes.c_char_p, []),
+    "w8a8_workspace_check": (_i32, [_vp, _vp]),
+    "w8a8_set_kernel_events": (_i32, [_vp, _vp]),
     "w8a8_act_absmax": (_i32, [_vp, _i32, _i32, _vp, _vp]),
     "w8a8_prepare_weights": (_i32, [_vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
     "w8a8_prepare_gate_up": (_i32, [_vp, _vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -134,6 +136,19 @@ def default_workspace() -> Workspace:
     if dev not in _DEFAULT_WS:
         _DEFAULT_WS[dev] = Workspace(torch.device("cuda", dev))
     return _DEFAULT_WS[dev]
+
+
+def workspace_check(ws: "Workspace", stream=None) -> None:
+    """Raise W8A8Error(ERR_TIMEOUT) if a kernel using `ws` recorded a device-side timeout."""
+    _check("w8a8_workspace_check", lib().w8a8_workspace_check(_p(ws.buf), _stream(stream)))
+
+
+def set_kernel_events(start, stop) -> None:
+    """Record the torch.cuda.Events `start`/`stop` around the next weight-streaming GEMM kernel
+    launched by this thread (measurement aid)."""
+    _check("w8a8_set_kernel_events", lib().w8a8_set_kernel_events(
+        ctypes.c_void_p(start.cuda_event) if start is not None else None,
+        ctypes.c_void_p(stop.cuda_event) if stop is not None else None))
 
 
 def _size(fn_name, *args) -> int:

@@ -73,7 +73,7 @@ static LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
   w.sx = off;
   if (int8_path) off += round_up((size_t)M * 4, 256);
   w.part = off;
-  off += round_up(make_stream_plan(M, N, K, sms).partial_bytes, 256);
+  off += round_up(make_stream_plan(int8_path, M, N, K, sms).partial_bytes, 256);
   w.total = off;
   return w;
 }
@@ -96,30 +96,37 @@ static w8a8_status check_ws(const char* who, void* ws, size_t have, size_t need)
   return W8A8_OK;
 }
 
-#define W8A8_TRY(expr)              \
-  do {                              \
-    w8a8_status s_ = (expr);        \
-    if (s_ != W8A8_OK) return s_;   \
-  } while (0)
 
-// One W8A8 linear: K1 then the streaming GEMM.  s_x/xf16 live in the workspace.
+// Per-token quantiser for a W8A8 GEMM plan: INT8 codes for the dp4a GEMV, fp16 codes for the MMA
+// kernel, written to `codes` (workspace); `xq_dbg` (nullable) also receives the INT8 codes.
+static w8a8_status quantize_for(const StreamPlan& p, const uint16_t* X, int M, int K, const float* inv_delta,
+                                void* codes, int8_t* xq_dbg, float* s_x, cudaStream_t st) {
+  if (p.dp4a) {
+    W8A8_TRY(launch_quantize_rows(X, M, K, inv_delta, reinterpret_cast<int8_t*>(codes), nullptr, s_x, st));
+    if (xq_dbg) W8A8_CUDA(cudaMemcpyAsync(xq_dbg, codes, (size_t)M * K, cudaMemcpyDeviceToDevice, st));
+    return W8A8_OK;
+  }
+  return launch_quantize_rows(X, M, K, inv_delta, xq_dbg, reinterpret_cast<uint16_t*>(codes), s_x, st);
+}
+
+// One W8A8 linear: K1 then the streaming GEMM.  s_x and the codes live in the workspace.
 static w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
                                    uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
                                    int sms, cudaStream_t st) {
   const int N = w->n, K = w->k;
   LinearWs L = linear_ws(M, N, K, true, sms);
   char* base = reinterpret_cast<char*>(ws);
-  uint16_t* xf16 = reinterpret_cast<uint16_t*>(base + L.xf16);
+  void* codes = base + L.xf16;
   float* s_x = reinterpret_cast<float*>(base + L.sx);
-  W8A8_TRY(launch_quantize_rows(X, M, K, w->inv_delta, dbg ? dbg->xq : nullptr, xf16, s_x, st));
-  if (dbg && dbg->s_x) W8A8_CUDA(cudaMemcpyAsync(dbg->s_x, s_x, sizeof(float) * M, cudaMemcpyDeviceToDevice, st));
   StreamArgs a{};
+  a.p = make_stream_plan(true, M, N, K, sms);
+  W8A8_TRY(quantize_for(a.p, X, M, K, w->inv_delta, codes, dbg ? dbg->xq : nullptr, s_x, st));
+  if (dbg && dbg->s_x) W8A8_CUDA(cudaMemcpyAsync(dbg->s_x, s_x, sizeof(float) * M, cudaMemcpyDeviceToDevice, st));
   a.W = w->wq;
-  a.X = xf16;
+  a.X = codes;
   a.M = M;
   a.N = N;
   a.K = K;
-  a.p = make_stream_plan(M, N, K, sms);
   a.kind = kind;
   a.s_x = s_x;
   a.s_w = w->s_w;
@@ -143,7 +150,7 @@ static w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16
   a.M = M;
   a.N = N;
   a.K = K;
-  a.p = make_stream_plan(M, N, K, sms);
+  a.p = make_stream_plan(false, M, N, K, sms);
   a.kind = kind;
   a.bias = bias;
   a.y = Y;
@@ -159,6 +166,28 @@ static w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16
 using namespace w8a8;
 
 extern "C" int w8a8_abi_version(void) { return 1; }
+
+extern "C" w8a8_status w8a8_set_kernel_events(void* start_event, void* stop_event) {
+  W8A8_CHECK_ARG((start_event == nullptr) == (stop_event == nullptr), W8A8_ERR_INVALID_ARG,
+                 "w8a8_set_kernel_events: give both events or neither");
+  set_kernel_events(start_event, stop_event);
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_workspace_check(void* workspace, void* stream) {
+  W8A8_CHECK_ARG(workspace != nullptr, W8A8_ERR_INVALID_ARG, "w8a8_workspace_check: null workspace");
+  cudaStream_t st = as_stream(stream);
+  unsigned int* err = reinterpret_cast<unsigned int*>(reinterpret_cast<char*>(workspace) + kErrWordOffset);
+  unsigned int host = 0;
+  W8A8_CUDA(cudaMemcpyAsync(&host, err, sizeof(host), cudaMemcpyDeviceToHost, st));
+  W8A8_CUDA(cudaStreamSynchronize(st));
+  if (host == 0) return W8A8_OK;
+  W8A8_CUDA(cudaMemsetAsync(err, 0, sizeof(unsigned int), st));
+  W8A8_CUDA(cudaStreamSynchronize(st));
+  set_error("a device-side wait gave up (error bits 0x%x: 1 consumer, 2 producer, 4 drain); results of the "
+            "affected calls are undefined", host);
+  return W8A8_ERR_TIMEOUT;
+}
 extern "C" const char* w8a8_last_error(void) { return get_error(); }
 
 // ---------------------------------------------------------------------------- linear
@@ -269,16 +298,16 @@ extern "C" w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* f, int precision, 
     // gate/up: scratch at L.gu
     {
       const LinearWs A = linear_ws(M, 2 * F, H, true, d.sms);
-      uint16_t* xf16 = reinterpret_cast<uint16_t*>(base + L.gu + (A.xf16 - W8A8_WS_RESERVED));
+      void* codes = base + L.gu + (A.xf16 - W8A8_WS_RESERVED);
       float* s_x = reinterpret_cast<float*>(base + L.gu + (A.sx - W8A8_WS_RESERVED));
-      W8A8_TRY(launch_quantize_rows(X, M, H, f->gate_up.inv_delta, nullptr, xf16, s_x, st));
       StreamArgs a{};
+      a.p = make_stream_plan(true, M, 2 * F, H, d.sms);
+      W8A8_TRY(quantize_for(a.p, X, M, H, f->gate_up.inv_delta, codes, nullptr, s_x, st));
       a.W = f->gate_up.wq;
-      a.X = xf16;
+      a.X = codes;
       a.M = M;
       a.N = 2 * F;
       a.K = H;
-      a.p = make_stream_plan(M, 2 * F, H, d.sms);
       a.kind = EPI_GEGLU;
       a.s_x = s_x;
       a.s_w = f->gate_up.s_w;
@@ -289,16 +318,16 @@ extern "C" w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* f, int precision, 
     }
     {
       const LinearWs B = linear_ws(M, H, F, true, d.sms);
-      uint16_t* xf16 = reinterpret_cast<uint16_t*>(base + L.dn + (B.xf16 - W8A8_WS_RESERVED));
+      void* codes = base + L.dn + (B.xf16 - W8A8_WS_RESERVED);
       float* s_x = reinterpret_cast<float*>(base + L.dn + (B.sx - W8A8_WS_RESERVED));
-      W8A8_TRY(launch_quantize_rows(h, M, F, f->down.inv_delta, nullptr, xf16, s_x, st));
       StreamArgs a{};
+      a.p = make_stream_plan(true, M, H, F, d.sms);
+      W8A8_TRY(quantize_for(a.p, h, M, F, f->down.inv_delta, codes, nullptr, s_x, st));
       a.W = f->down.wq;
-      a.X = xf16;
+      a.X = codes;
       a.M = M;
       a.N = H;
       a.K = F;
-      a.p = make_stream_plan(M, H, F, d.sms);
       a.kind = EPI_BF16;
       a.s_x = s_x;
       a.s_w = f->down.s_w;
@@ -316,7 +345,7 @@ extern "C" w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* f, int precision, 
       a.M = M;
       a.N = 2 * F;
       a.K = H;
-      a.p = make_stream_plan(M, 2 * F, H, d.sms);
+      a.p = make_stream_plan(false, M, 2 * F, H, d.sms);
       a.kind = EPI_GEGLU;
       a.y = h;
       a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
@@ -331,7 +360,7 @@ extern "C" w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* f, int precision, 
       a.M = M;
       a.N = H;
       a.K = F;
-      a.p = make_stream_plan(M, H, F, d.sms);
+      a.p = make_stream_plan(false, M, H, F, d.sms);
       a.kind = EPI_BF16;
       a.y = Y;
       a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);

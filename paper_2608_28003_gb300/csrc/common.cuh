@@ -34,6 +34,12 @@ const char* get_error();
 
 #define W8A8_LAUNCH_CHECK() W8A8_CUDA(cudaGetLastError())
 
+#define W8A8_TRY(expr)            \
+  do {                            \
+    w8a8_status s_ = (expr);      \
+    if (s_ != W8A8_OK) return s_; \
+  } while (0)
+
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
 inline size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -104,6 +110,70 @@ __device__ __forceinline__ uint4 ldg_keep(const void* p) {
                : "l"(p));
   return v;
 }
+
+// ------------------------------------------------------------- mbarrier and bulk copies
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory"); }
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Wait for the phase with the given parity to complete, for at most `budget` SM cycles.
+// Returns false on timeout (the caller records an error and stops waiting).
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, long long budget) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > budget) return false;
+  return true;
+}
+// 2-D tiled TMA load of one box (coordinates: c0 = innermost element index, c1 = row) into shared
+// memory; completion is counted on `bar` in bytes (out-of-bounds elements are zero-filled and counted).
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int c0, int c1, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+// 1-D bulk copy global -> shared (async proxy); completion is counted on `bar` in bytes.
+// dst and src 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
+}
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
+// Device-side error bits (reserved workspace word at kErrWordOffset): set by a bounded wait
+// that gave up; read and cleared by w8a8_workspace_check.
+enum DevErr : unsigned int { DEVERR_CONSUMER_WAIT = 1u, DEVERR_PRODUCER_WAIT = 2u, DEVERR_DRAIN_WAIT = 4u };
+constexpr size_t kErrWordOffset = 36864;
+constexpr long long kWaitBudgetCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 // --------------------------------------------------------------------- GeGLU fp32 recipe
 // gelu_tanh(g) = g / (1 + 2^w), w = -2 log2(e) * sqrt(2/pi) * (g + 0.044715 g^3), each step one

@@ -1,374 +1,865 @@
-// Weight-streaming GEMM for decode-sized token counts, legacy tensor-core MMA (m16n8k16).
+// Weight-streaming GEMM for decode-sized token counts on the m16n8k16 tensor-core MMA.
 //
-// Computes acc_ti = sum_j X_tj * W_ij for W [N, K] (row = output channel) and X [M, K]
-// (Eq. gemm-final for the W8A8 path; the bf16 pass-through of the FFN section otherwise), then
-// the epilogue of the calling layer.  The weights are the streamed operand (decode is
-// HBM-bound on them); tokens ride in the MMA's N dimension (8 per block).
+// Computes acc_ti = sum_j X_tj * W_ij for W [N, K] (row = output channel) and X [M, K]: the INT8
+// sum of Eq. gemm-final on the W8A8 path, the bf16 pass-through of the FFN section otherwise,
+// followed by the calling layer's epilogue.  Decode is HBM-bound on W, so the kernel is built
+// around moving W at full bandwidth:
 //
-// W8A8 path: INT8 codes are loaded straight from global memory into registers and widened to
-// fp16 in registers (exact); X arrives as fp16 codes.  fp16 x fp16 products of codes are exact
-// integers below 2^14 and every partial sum of at most 1024 products stays below 2^24, where
-// fp32 represents integers exactly, so each warp folds its fp32 accumulator into INT32 every
-// 16 k-steps (1024 k): the INT32 result is exact whatever order the hardware adds in.
-//
-// Fragment layout: lane = 4g + t.  In a 64-wide k step the lane loads k = 16t .. 16t+15 of
-// weight rows g and g+8 and of token g.  The m16n8k16 fragments of MMA j (j = 0..3) take the
-// lane's k = 16t+4j .. 16t+4j+3 for both operands, so every MMA pairs the same physical k on
-// A and B, and the four MMAs of a step cover all 64 k: a k permutation that a dot product
-// does not see.
-//
-// Work split: 16-row tiles x k slices; a CTA holds RPC row tiles x WS k slices (one warp
-// each) and reduces its slices in shared memory.  Small-N layers also split k across CTAs
-// (CS > 1): each CTA writes its partial tile, and the last CTA to arrive (an atomic counter,
-// no waiting) sums the partials in a fixed order and runs the epilogue.  INT32 partials make
-// this exact; fp32 partials (bf16 path) are summed in a fixed order, so results are
-// deterministic.
+//  * Persistent grid, one CTA per SM (two for a single token block): 1 producer warp + 8 consumer
+//    warps each.  The work is the list
+//    of units (token group z, 128-row weight group g, k chunk of 64..256 bytes per row), ordered
+//    z-major, then g, then k; CTA c takes the contiguous range [c U / P, (c+1) U / P), so every
+//    CTA streams the same number of bytes (stream-K style balance, no wave tail); the chunk
+//    shrinks for small layers so that there are at least as many units as SMs.
+//  * One producer thread loads each unit with 2-D TMA (cp.async.bulk.tensor): 128-byte-wide boxes
+//    of 128 weight rows and of the unit's token rows of X, 128-byte swizzled, zero-filled outside
+//    the tensors, into a ring of shared-memory stages guarded by mbarriers; consumers release a
+//    stage through a second mbarrier.
+//  * Consumer warp w owns tile rows 16w .. 16w+15 of every unit.  Lane 4g + t loads k = 16t .. 16t+15
+//    (of each 64-wide step) of MMA rows g and g+8 and of token g, and feeds MMA j (j = 0..3) the
+//    lane's k = 16t+4j .. 16t+4j+3 on both operands, a k permutation that a dot product does not
+//    see.  MMA row g reads tile row perm(g): the identity for bf16, and for INT8 (lanes read 16 of
+//    each row's 128 swizzled bytes) the pairing (2p, 2p+1) -> (p, p+4), so the two rows a phase of
+//    8 lanes touches use opposite halves of the banks.
+//  * W8A8 path: INT8 codes are widened to fp16 in registers (exact); X holds fp16 codes.  Each
+//    product of codes is an integer below 2^14 and any partial sum of at most 1024 of them stays
+//    below 2^24, where fp32 is exact, so the fp32 accumulator is folded into INT32 every 16 steps
+//    (1024 k) and the INT32 result is exact in any summation order.
+//  * A (z, g) whose k range spans several CTAs is finished by the last CTA to arrive: each
+//    contributor writes its partial tile, bumps a counter (no waiting), and the last one sums the
+//    partials in CTA order (exact for INT32; a fixed order for fp32) and runs the epilogue.
+//  * Every mbarrier wait is bounded: on timeout the kernel sets a bit in the workspace's error
+//    word, stops waiting, lets its own copies in flight land (again bounded) and returns.
 #include <algorithm>
 
 #include "stream_gemm.cuh"
+#include "tmap.cuh"
 
 namespace w8a8 {
 
 namespace {
 
+constexpr int kTileCounterSlots = 8192;                      // uint32 slots at workspace offset 0
+constexpr size_t kGridCounterOffset = 8192 * 4;              // one uint32
+constexpr size_t kTopKeysOffset = 40960;                     // uint64 keys
+constexpr int kMaxTopKeys = (W8A8_WS_RESERVED - 40960) / 8;  // 3072
+constexpr int kConsumerWarps = 8;
+constexpr int kThreads = (kConsumerWarps + 1) * 32;
+constexpr int kSmemLimit = 227 * 1024;   // shared memory per SM available to CTAs
+constexpr int kStaticReserve = 8192;     // static shared memory of the kernel (barrier flags, top-1 keys)
+constexpr int kBox = 16384;  // one weight box: 128 rows x 128 bytes
+
+template <bool kInt8>
+struct Geo {
+  static constexpr int EB = kInt8 ? 1 : 2;           // weight element bytes
+  static constexpr int KCMAX = kInt8 ? 256 : 128;    // stage capacity in k elements (2 weight boxes)
+  static constexpr int BOXK = 128 / EB;              // k elements per weight box
+};
+
+__host__ __device__ constexpr int stage_bytes_for(bool int8, int tok) {
+  // 2 weight boxes + (KCMAX / 64) token boxes of TOK rows x 128 bytes, all 1024-byte aligned
+  return 2 * kBox + (int8 ? 4 : 2) * tok * 128;
+}
+
 __device__ __forceinline__ uint32_t u4c(const uint4& v, int c) {
   return c == 0 ? v.x : c == 1 ? v.y : c == 2 ? v.z : v.w;
 }
 
-constexpr int kTileCounterSlots = 8192;                    // uint32 slots at workspace offset 0
-constexpr size_t kGridCounterOffset = 8192 * 4;            // one uint32
-constexpr size_t kTopKeysOffset = 40960;                   // uint64 keys
-constexpr int kMaxTopKeys = (W8A8_WS_RESERVED - 40960) / 8;  // 3072
+// tile row read by MMA row g (0..7)
+template <bool kInt8>
+__device__ __forceinline__ int row_perm(int g) {
+  return kInt8 ? ((g >> 1) | ((g & 1) << 2)) : g;
+}
 
-template <bool kInt8, int NB, int U>
-__global__ void __launch_bounds__(256) stream_gemm_kernel(const StreamArgs a) {
+// CTAs per SM: two for up to 16 tokens (registers allow it), else one.
+template <int NB>
+struct Cps {
+  static constexpr int value = NB == 1 ? 2 : 1;
+};
+
+template <bool kInt8, int NB, int STEPS>
+__global__ void __launch_bounds__(kThreads, Cps<NB>::value)
+    stream_gemm_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                       const StreamArgs a) {
+  using GG = Geo<kInt8>;
   constexpr int TOK = 8 * NB;
-  constexpr int WV = kInt8 ? 1 : 2;  // 16-byte vectors per 16-k weight chunk
-  constexpr int EB = kInt8 ? 1 : 2;  // weight element bytes
-  __shared__ uint32_t red[8 * 16 * TOK];
-  __shared__ unsigned long long skeys[TOK];
-  __shared__ int s_last;
+  constexpr int BOXK = GG::BOXK;
+  constexpr int KC = STEPS * 64;  // k elements per unit
+  constexpr int CH = NB >= 4 ? 1 : 4 / NB;  // independent accumulator chains per token block
+  constexpr int XBOX = TOK * 128;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ int s_flag;
+  __shared__ unsigned long long s_best[kConsumerWarps][TOK];  // top-1: per-warp best key per token slot
 
   const StreamPlan& p = a.p;
+  const int S = p.stages, SB = p.stage_bytes;
+  // 128-byte swizzle repeats every 1024 bytes: align the ring to 1024
+  const uint32_t raw_u32 = smem_u32(smem_raw);
+  const uint32_t ring = (raw_u32 + 1023u) & ~1023u;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (ring - raw_u32) + (size_t)S * SB);
+  uint64_t* empty = full + S;
+
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = lane >> 2, t = lane & 3;
-  const int group = blockIdx.x / p.CS, cs = blockIdx.x % p.CS;
-  const int z = blockIdx.z;
-  const int tok0 = z * TOK;
-  const int rt_local = warp / p.WS, ws = warp % p.WS;
-  const int rt = group * p.RPC + rt_local;
-  const int sl = cs * p.WS + ws;
-  const int s_begin = sl * p.sps;
-  const int s_end = rt < p.RT ? min(p.KS, s_begin + p.sps) : s_begin;
-  const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
+  const int G = p.G, C = p.C, Z = p.Z;
+  const long long U = (long long)Z * G * C;
+  const int P = gridDim.x, cta = blockIdx.x;
+  // Unit range of this CTA: whole (z, g) groups when there are at least as many groups as CTAs
+  // (no group is split, no partial tiles), else an even split of the units (stream-K).
+  const long long ZG = (long long)Z * G;
+  const long long u0 = p.whole ? (long long)cta * ZG / P * C : (long long)cta * U / P;
+  const long long u1 = p.whole ? (long long)(cta + 1) * ZG / P * C : (long long)(cta + 1) * U / P;
+  auto cta_of = [&](long long u) -> int { return (int)(((u + 1) * P + U - 1) / U - 1); };
 
-  if (want_top)
-    for (int i = threadIdx.x; i < TOK; i += blockDim.x) skeys[i] = 0ull;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(full + s), 1);
+      mbar_init(smem_u32(empty + s), kConsumerWarps);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (u0 >= u1) return;
 
-  const int row_a = rt * 16 + g, row_b = row_a + 8;
-  const bool va = row_a < a.N, vb = row_b < a.N;
-  const char* wa_ptr = reinterpret_cast<const char*>(a.W) + (size_t)(va ? row_a : 0) * a.K * EB;
-  const char* wb_ptr = reinterpret_cast<const char*>(a.W) + (size_t)(vb ? row_b : 0) * a.K * EB;
+  // ------------------------------------------------------------------------ producer thread
+  if (warp == kConsumerWarps) {
+    if (lane != 0) return;
+    constexpr int nw = KC / BOXK, nx = KC / 64;
+    const uint32_t tx = (uint32_t)(nw * kBox + nx * XBOX);
+    bool ok = true;
+    long long it = 0;
+    for (long long u = u0; u < u1; ++u, ++it) {
+      const int s = (int)(it % S);
+      const uint32_t ph = (uint32_t)((it / S) & 1);
+      if (!mbar_wait_bounded(smem_u32(empty + s), ph ^ 1u, kWaitBudgetCycles)) {
+        ok = false;
+        break;
+      }
+      const int zg = (int)(u / C), ch = (int)(u % C);
+      const int z = zg / G, g = zg % G;
+      const uint32_t bar = smem_u32(full + s);
+      const uint32_t sb = ring + (uint32_t)s * SB;
+      mbar_arrive_expect_tx(bar, tx);
+      for (int b = 0; b < nw; ++b) tma_load_2d(sb + b * kBox, &tmW, ch * KC + b * BOXK, g * 128, bar);
+      for (int b = 0; b < nx; ++b) tma_load_2d(sb + 2 * kBox + b * XBOX, &tmX, ch * KC + b * 64, z * TOK, bar);
+    }
+    if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
+    // Let the copies of the last stages land before this CTA can exit (bounded).
+    for (long long j = it > S ? it - S : 0; j < it; ++j) {
+      if (!mbar_wait_bounded(smem_u32(full + (int)(j % S)), (uint32_t)((j / S) & 1), kWaitBudgetCycles)) {
+        atomicOr(a.err, DEVERR_DRAIN_WAIT);
+        break;
+      }
+    }
+    return;
+  }
 
-  float acc[NB][4];
+  // ----------------------------------------------------------------------- consumer warps
+  const int w = warp;
+  const int gl = lane >> 2, t = lane & 3;
+  const int pr = row_perm<kInt8>(gl);  // tile row (within 16) of MMA row gl; MMA row gl+8 -> pr+8
+  float acc[CH][NB][4];
   int iacc[NB][4];
-#pragma unroll
-  for (int nb = 0; nb < NB; ++nb)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      acc[nb][e] = 0.0f;
-      iacc[nb][e] = 0;
-    }
   int since = 0;
-  const uint4 zero4 = make_uint4(0, 0, 0, 0);
+  bool ok = true;
+  // top-1: the warp's best key per token slot of token group best_z (in s_best), published with
+  // one atomicMax per token when the token group changes and at the end
+  int best_z = -1;
 
-  for (int s0 = s_begin; s0 < s_end; s0 += U) {
-    uint4 wa[U][WV], wb[U][WV];
-    uint4 xv[U][NB][2];
+  auto zero_acc = [&]() {
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int s = s0 + u;
-      const int k = s * 64 + t * 16;
-      const bool kv = (s < s_end) && (k < a.K);
+    for (int c = 0; c < CH; ++c)
 #pragma unroll
-      for (int v = 0; v < WV; ++v) {
-        wa[u][v] = (kv && va) ? ldg_stream(wa_ptr + (size_t)k * EB + 16 * v) : zero4;
-        wb[u][v] = (kv && vb) ? ldg_stream(wb_ptr + (size_t)k * EB + 16 * v) : zero4;
-      }
+      for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-      for (int nb = 0; nb < NB; ++nb) {
-        const int tok = tok0 + nb * 8 + g;
-        const bool tv = kv && tok < a.M;
-        const uint16_t* xp = a.X + (size_t)(tv ? tok : 0) * a.K + (tv ? k : 0);
-        xv[u][nb][0] = tv ? ldg_keep(xp) : zero4;
-        xv[u][nb][1] = tv ? ldg_keep(xp + 8) : zero4;
-      }
+        for (int e = 0; e < 4; ++e) acc[c][nb][e] = 0.0f;
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) iacc[nb][e] = 0;
+    since = 0;
+  };
+
+  auto publish_top = [&]() {
+    if (best_z < 0) return;
+    __syncwarp();
+    for (int i = lane; i < TOK; i += 32) {
+      const int tk = best_z * TOK + i;
+      const unsigned long long k = s_best[w][i];
+      if (tk < a.M && k != 0ull) atomicMax(a.top_keys + tk, k);
+    }
+    __syncwarp();
+    best_z = -1;
+  };
+
+  // dequantised (or bf16-path) fp32 value of an accumulator, before the bias
+  auto value_f32 = [&](uint32_t v, int i, int tk) -> float {
+    if constexpr (kInt8) {
+      const float sc = __fmul_rn(a.s_x[tk], a.s_w[i]);  // s_t^x * s_i^W
+      return __fmul_rn(sc, __int2float_rn((int)v));
+    } else {
+      return __uint_as_float(v);
+    }
+  };
+
+  const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
+  auto epilogue = [&](int z, int g, uint32_t (&v)[NB][4]) {
+    const int ra = g * 128 + 16 * w + pr, rb = ra + 8;
+    if (want_top && z != best_z) {
+      publish_top();
+      best_z = z;
+      for (int i = lane; i < TOK; i += 32) s_best[w][i] = 0ull;
+      __syncwarp();
     }
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
+    for (int nb = 0; nb < NB; ++nb) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        unsigned long long best = 0ull;
+        const int tk = z * TOK + nb * 8 + 2 * t + h;
+        if (tk >= a.M) {
+        } else if (a.kind == EPI_GEGLU) {
+          if (rb >= a.N) continue;
+          float gv = value_f32(v[nb][h], ra, tk), uv = value_f32(v[nb][2 + h], rb, tk);
+          if (a.bias) {
+            gv = __fadd_rn(gv, a.bias[ra]);
+            uv = __fadd_rn(uv, a.bias[rb]);
+          }
+          if constexpr (kInt8) {
+            if (a.acc_dbg) {
+              a.acc_dbg[(size_t)tk * a.N + ra] = (int)v[nb][h];
+              a.acc_dbg[(size_t)tk * a.N + rb] = (int)v[nb][2 + h];
+            }
+          }
+          a.y[(size_t)tk * (a.N >> 1) + ((g * 128 + 16 * w) >> 1) + pr] = f32_to_bf16_bits(geglu_recipe(gv, uv));
+        } else {
+#pragma unroll
+          for (int side = 0; side < 2; ++side) {
+            const int i = side ? rb : ra;
+            if (i >= a.N) continue;
+            const uint32_t raw = v[nb][2 * side + h];
+            float y = value_f32(raw, i, tk);
+            if (a.bias) y = __fadd_rn(y, a.bias[i]);
+            if constexpr (kInt8) {
+              if (a.acc_dbg) a.acc_dbg[(size_t)tk * a.N + i] = (int)raw;
+            }
+            if (a.kind == EPI_BF16) {
+              a.y[(size_t)tk * a.N + i] = f32_to_bf16_bits(y);
+            } else {
+              if (a.logits) a.logits[(size_t)tk * a.N + i] = y;
+              const unsigned long long key =
+                  ((unsigned long long)float_order_key(y) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)i);
+              best = key > best ? key : best;
+            }
+          }
+        }
+        if (want_top) {  // max over the 8 row pairs (lanes with equal t)
+#pragma unroll
+          for (int o = 4; o < 32; o <<= 1) {
+            const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+            best = other > best ? other : best;
+          }
+          if (gl == 0 && best > s_best[w][nb * 8 + 2 * t + h]) s_best[w][nb * 8 + 2 * t + h] = best;
+        }
+      }
+    }
+  };
+
+  auto flush = [&](int zg, int chf, int chl) {
+    uint32_t v[NB][4];
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if constexpr (kInt8) {
+          int sum = iacc[nb][e];
+#pragma unroll
+          for (int c = 0; c < CH; ++c) sum += __float2int_rn(acc[c][nb][e]);
+          v[nb][e] = (uint32_t)sum;
+        } else {
+          float sum = acc[0][nb][e];
+#pragma unroll
+          for (int c = 1; c < CH; ++c) sum += acc[c][nb][e];
+          v[nb][e] = __float_as_uint(sum);
+        }
+      }
+    const int z = zg / G, g = zg % G;
+    if (!(chf == 0 && chl == C - 1)) {
+      const long long ub = (long long)zg * C;
+      const int f = cta_of(ub), l = cta_of(ub + C - 1);
+      uint32_t* part = reinterpret_cast<uint32_t*>(a.partials);
+      auto slot_base = [&](int c) -> uint32_t* {
+        const long long cu0 = (long long)c * U / P;
+        const int slot = (zg == (int)(cu0 / C)) ? 0 : 1;
+        return part + ((size_t)(c * 2 + slot) * 128) * TOK;
+      };
+      uint32_t* mine = slot_base(cta);
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          mine[(16 * w + pr + (e >> 1) * 8) * TOK + nb * 8 + 2 * t + (e & 1)] = v[nb][e];
+      __threadfence();
+      named_bar_sync(1, kConsumerWarps * 32);
+      if (threadIdx.x == 0) {
+        const unsigned int prev = atomicAdd(a.tile_counters + f, 1u);
+        const int is_last = prev == (unsigned int)(l - f);
+        if (is_last) a.tile_counters[f] = 0u;
+        s_flag = is_last;
+      }
+      named_bar_sync(1, kConsumerWarps * 32);
+      if (!s_flag) return;
+      __threadfence();
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) v[nb][e] = 0u;
+      for (int c = f; c <= l; ++c) {
+        const uint32_t* src = slot_base(c);
+#pragma unroll
+        for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const uint32_t x = __ldcg(src + (16 * w + pr + (e >> 1) * 8) * TOK + nb * 8 + 2 * t + (e & 1));
+            v[nb][e] = kInt8 ? (uint32_t)((int)v[nb][e] + (int)x)
+                             : __float_as_uint(__uint_as_float(v[nb][e]) + __uint_as_float(x));
+          }
+      }
+    }
+    epilogue(z, g, v);
+  };
+
+  zero_acc();
+  int cur = -1, chf = 0, chl = 0;
+  long long it = 0;
+  const uint32_t rowA = (uint32_t)(16 * w + pr) * 128u, rowB = rowA + 8u * 128u;
+  for (long long u = u0; u < u1; ++u, ++it) {
+    const int zg = (int)(u / C), ch = (int)(u % C);
+    if (zg != cur) {
+      if (cur >= 0) flush(cur, chf, chl);
+      cur = zg;
+      chf = ch;
+      zero_acc();
+    }
+    chl = ch;
+    const int s = (int)(it % S);
+    const uint32_t ph = (uint32_t)((it / S) & 1);
+    if (ok) {
+      bool got = true;
+      if (lane == 0) got = mbar_wait_bounded(smem_u32(full + s), ph, kWaitBudgetCycles);
+      got = __shfl_sync(0xffffffffu, got, 0);
+      if (!got) {
+        ok = false;
+        if (lane == 0) atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+      }
+    }
+    if (!ok) continue;  // no data: skip the math and do not release the stage
+
+    const uint32_t sb = ring + (uint32_t)s * SB;
+#pragma unroll
+    for (int st = 0; st < STEPS; ++st) {
+      uint4 wa[2], wb[2];
+      if constexpr (kInt8) {
+        // weight box st/2, logical 16-byte chunk 4(st%2) + t of rows pr and pr+8 (row & 7 == pr)
+        const uint32_t wbox = sb + (uint32_t)(st >> 1) * kBox;
+        const uint32_t off = (uint32_t)(((4 * (st & 1) + t) ^ pr) << 4);
+        wa[0] = lds128(wbox + rowA + off);
+        wb[0] = lds128(wbox + rowB + off);
+      } else {
+        // weight box st, logical chunks 2t and 2t+1 of rows gl and gl+8
+        const uint32_t wbox = sb + (uint32_t)st * kBox;
+        const uint32_t o0 = (uint32_t)(((2 * t) ^ pr) << 4), o1 = (uint32_t)(((2 * t + 1) ^ pr) << 4);
+        wa[0] = lds128(wbox + rowA + o0);
+        wa[1] = lds128(wbox + rowA + o1);
+        wb[0] = lds128(wbox + rowB + o0);
+        wb[1] = lds128(wbox + rowB + o1);
+      }
+      // A fragments of the four MMAs of this step (INT8 codes widened to fp16 in registers)
+      uint32_t af[4][4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        uint32_t a0, a1, a2, a3;
         if constexpr (kInt8) {
-          i8x4_to_f16x2x2(u4c(wa[u][0], j), a0, a2);
-          i8x4_to_f16x2x2(u4c(wb[u][0], j), a1, a3);
+          i8x4_to_f16x2x2(u4c(wa[0], j), af[j][0], af[j][2]);
+          i8x4_to_f16x2x2(u4c(wb[0], j), af[j][1], af[j][3]);
         } else {
-          a0 = u4c(wa[u][j >> 1], (2 * j) & 3);
-          a2 = u4c(wa[u][j >> 1], (2 * j + 1) & 3);
-          a1 = u4c(wb[u][j >> 1], (2 * j) & 3);
-          a3 = u4c(wb[u][j >> 1], (2 * j + 1) & 3);
+          af[j][0] = u4c(wa[j >> 1], (2 * j) & 3);
+          af[j][2] = u4c(wa[j >> 1], (2 * j + 1) & 3);
+          af[j][1] = u4c(wb[j >> 1], (2 * j) & 3);
+          af[j][3] = u4c(wb[j >> 1], (2 * j + 1) & 3);
         }
+      }
+      const uint32_t xbox = sb + 2 * kBox + (uint32_t)st * XBOX;
 #pragma unroll
-        for (int nb = 0; nb < NB; ++nb) {
-          const uint32_t b0 = u4c(xv[u][nb][j >> 1], (2 * j) & 3);
-          const uint32_t b1 = u4c(xv[u][nb][j >> 1], (2 * j + 1) & 3);
+      for (int nb = 0; nb < NB; ++nb) {
+        const uint32_t xr = xbox + (uint32_t)(nb * 8 + gl) * 128u;  // token row & 7 == gl
+        const uint4 x0 = lds128(xr + (uint32_t)(((2 * t) ^ gl) << 4));
+        const uint4 x1 = lds128(xr + (uint32_t)(((2 * t + 1) ^ gl) << 4));
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint4& xv = (j >> 1) ? x1 : x0;
+          const uint32_t b0 = u4c(xv, (2 * j) & 3);
+          const uint32_t b1 = u4c(xv, (2 * j + 1) & 3);
           if constexpr (kInt8)
-            mma_f16_16816(acc[nb], a0, a1, a2, a3, b0, b1);
+            mma_f16_16816(acc[j % CH][nb], af[j][0], af[j][1], af[j][2], af[j][3], b0, b1);
           else
-            mma_bf16_16816(acc[nb], a0, a1, a2, a3, b0, b1);
+            mma_bf16_16816(acc[j % CH][nb], af[j][0], af[j][1], af[j][2], af[j][3], b0, b1);
         }
       }
     }
     if constexpr (kInt8) {
-      since += U;
+      since += STEPS;
       if (since >= 16) {  // 16 steps = 1024 k: every partial sum so far is below 2^24
 #pragma unroll
         for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            iacc[nb][e] += __float2int_rn(acc[nb][e]);
-            acc[nb][e] = 0.0f;
+#pragma unroll
+            for (int c = 0; c < CH; ++c) {
+              iacc[nb][e] += __float2int_rn(acc[c][nb][e]);
+              acc[c][nb][e] = 0.0f;
+            }
           }
         since = 0;
       }
     }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(empty + s));
   }
-
-  // ---- per-warp tile -> shared memory: red[warp][row][tok]
-  {
-    uint32_t* r = red + warp * 16 * TOK;
-#pragma unroll
-    for (int nb = 0; nb < NB; ++nb) {
-      const int c0 = nb * 8 + 2 * t;
-      uint32_t v[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e)
-        v[e] = kInt8 ? (uint32_t)(iacc[nb][e] + __float2int_rn(acc[nb][e])) : __float_as_uint(acc[nb][e]);
-      r[g * TOK + c0] = v[0];
-      r[g * TOK + c0 + 1] = v[1];
-      r[(g + 8) * TOK + c0] = v[2];
-      r[(g + 8) * TOK + c0 + 1] = v[3];
-    }
+  if (cur >= 0) flush(cur, chf, chl);
+  if (!want_top) return;
+  // top-1 across the grid: every CTA publishes its maxima, then counts itself once; the last CTA
+  // decodes the keys into indices and clears them
+  publish_top();
+  __threadfence();
+  named_bar_sync(1, kConsumerWarps * 32);
+  if (threadIdx.x == 0) {
+    const unsigned int prev = atomicAdd(a.grid_counter, 1u);
+    s_flag = prev == (unsigned int)(P - 1);
+    if (s_flag) *a.grid_counter = 0u;
   }
-  __syncthreads();
-
-  // ---- reduce the WS slices of each row tile in place into slot ws = 0
-  const int nthreads = blockDim.x;
-  const int E = p.RPC * 16 * TOK;
-  auto fin_index = [&](int e) {  // element e = (rtl * 16 + row) * TOK + tok
-    const int rtl = e / (16 * TOK);
-    const int rem = e - rtl * 16 * TOK;
-    return (rtl * p.WS) * 16 * TOK + rem;
-  };
-  for (int e = threadIdx.x; e < E; e += nthreads) {
-    const int rtl = e / (16 * TOK);
-    const int rem = e - rtl * 16 * TOK;
-    const uint32_t* base = red + (rtl * p.WS) * 16 * TOK + rem;
-    if constexpr (kInt8) {
-      int s = 0;
-      for (int w = 0; w < p.WS; ++w) s += (int)base[w * 16 * TOK];
-      red[fin_index(e)] = (uint32_t)s;
-    } else {
-      float s = 0.0f;
-      for (int w = 0; w < p.WS; ++w) s += __uint_as_float(base[w * 16 * TOK]);
-      red[fin_index(e)] = __float_as_uint(s);
-    }
-  }
-
-  // ---- cross-CTA k split: partials + last-arriver reduction (no waiting)
-  if (p.CS > 1) {
-    uint32_t* part = reinterpret_cast<uint32_t*>(a.partials);
-    const size_t rows_total = (size_t)p.RT * 16;
-    for (int e = threadIdx.x; e < E; e += nthreads) {
-      const int rtl = e / (16 * TOK);
-      const int rem = e - rtl * 16 * TOK;
-      const int rtg = group * p.RPC + rtl;
-      if (rtg < p.RT) part[((size_t)(z * p.CS + cs) * rows_total + (size_t)rtg * 16) * TOK + rem] = red[fin_index(e)];
-    }
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned int* ctr = a.tile_counters + z * p.groups + group;
-      const unsigned int prev = atomicAdd(ctr, 1u);
-      s_last = (prev == (unsigned int)(p.CS - 1));
-      if (s_last) *ctr = 0u;  // every CTA of this tile has arrived: reset for the next call
-    }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    for (int e = threadIdx.x; e < E; e += nthreads) {
-      const int rtl = e / (16 * TOK);
-      const int rem = e - rtl * 16 * TOK;
-      const int rtg = group * p.RPC + rtl;
-      if (rtg >= p.RT) continue;
-      if constexpr (kInt8) {
-        int s = 0;
-        for (int c = 0; c < p.CS; ++c)
-          s += (int)__ldcg(part + ((size_t)(z * p.CS + c) * rows_total + (size_t)rtg * 16) * TOK + rem);
-        red[fin_index(e)] = (uint32_t)s;
-      } else {
-        float s = 0.0f;
-        for (int c = 0; c < p.CS; ++c)
-          s += __uint_as_float(__ldcg(part + ((size_t)(z * p.CS + c) * rows_total + (size_t)rtg * 16) * TOK + rem));
-        red[fin_index(e)] = __float_as_uint(s);
-      }
-    }
-  }
-  __syncthreads();
-
-  // ---- epilogue
-  auto value_f32 = [&](int e, int i, int tk) -> float {  // dequantised fp32 value (before bias)
-    const uint32_t r = red[fin_index(e)];
-    if constexpr (kInt8) {
-      const float sc = __fmul_rn(a.s_x[tk], a.s_w[i]);  // s_t^x * s_i^W
-      return __fmul_rn(sc, __int2float_rn((int)r));
-    } else {
-      return __uint_as_float(r);
-    }
-  };
-  if (a.kind == EPI_GEGLU) {
-    const int E2 = p.RPC * 8 * TOK;
-    const int F = a.N >> 1;
-    for (int e2 = threadIdx.x; e2 < E2; e2 += nthreads) {
-      const int rtl = e2 / (8 * TOK);
-      const int rem = e2 - rtl * 8 * TOK;
-      const int r = rem / TOK, tok = rem - (rem / TOK) * TOK;
-      const int rtg = group * p.RPC + rtl;
-      const int tk = tok0 + tok;
-      const int ig = rtg * 16 + r, iu = ig + 8;
-      if (rtg >= p.RT || iu >= a.N || tk >= a.M) continue;
-      const int eg = (rtl * 16 + r) * TOK + tok, eu = (rtl * 16 + r + 8) * TOK + tok;
-      float gv = value_f32(eg, ig, tk), uv = value_f32(eu, iu, tk);
-      if (a.bias) {
-        gv = __fadd_rn(gv, a.bias[ig]);
-        uv = __fadd_rn(uv, a.bias[iu]);
-      }
-      if constexpr (kInt8) {
-        if (a.acc_dbg) {
-          a.acc_dbg[(size_t)tk * a.N + ig] = (int)red[fin_index(eg)];
-          a.acc_dbg[(size_t)tk * a.N + iu] = (int)red[fin_index(eu)];
-        }
-      }
-      a.y[(size_t)tk * F + rtg * 8 + r] = f32_to_bf16_bits(geglu_recipe(gv, uv));
-    }
-  } else {
-    for (int e = threadIdx.x; e < E; e += nthreads) {
-      const int rtl = e / (16 * TOK);
-      const int rem = e - rtl * 16 * TOK;
-      const int row = rem / TOK, tok = rem - row * TOK;
-      const int rtg = group * p.RPC + rtl;
-      const int i = rtg * 16 + row, tk = tok0 + tok;
-      if (rtg >= p.RT || i >= a.N || tk >= a.M) continue;
-      float y = value_f32(e, i, tk);
-      if (a.bias) y = __fadd_rn(y, a.bias[i]);
-      if constexpr (kInt8) {
-        if (a.acc_dbg) a.acc_dbg[(size_t)tk * a.N + i] = (int)red[fin_index(e)];
-      }
-      if (a.kind == EPI_BF16) {
-        a.y[(size_t)tk * a.N + i] = f32_to_bf16_bits(y);
-      } else {
-        if (a.logits) a.logits[(size_t)tk * a.N + i] = y;
-        if (want_top) {
-          const unsigned long long key =
-              ((unsigned long long)float_order_key(y) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)i);
-          atomicMax(&skeys[tok], key);
-        }
-      }
-    }
-  }
-
-  // ---- top-1 across the grid: CTA maxima -> global keys; the last finalising CTA decodes them
-  if (want_top) {
-    __syncthreads();
-    for (int i = threadIdx.x; i < TOK; i += blockDim.x)
-      if (tok0 + i < a.M && skeys[i] != 0ull) atomicMax(a.top_keys + tok0 + i, skeys[i]);
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      const unsigned int total = (unsigned int)(p.groups * p.zgroups);
-      const unsigned int prev = atomicAdd(a.grid_counter, 1u);
-      s_last = (prev == total - 1);
-      if (s_last) *a.grid_counter = 0u;
-    }
-    __syncthreads();
-    if (s_last) {
-      __threadfence();
-      for (int tk = threadIdx.x; tk < a.M; tk += nthreads) {
-        const unsigned long long key = atomicExch(a.top_keys + tk, 0ull);
-        a.top1[tk] = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
-      }
-    }
+  named_bar_sync(1, kConsumerWarps * 32);
+  if (!s_flag) return;
+  __threadfence();
+  for (int tk = threadIdx.x; tk < a.M; tk += kConsumerWarps * 32) {
+    const unsigned long long key = atomicExch(a.top_keys + tk, 0ull);
+    a.top1[tk] = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
   }
 }
 
-template <bool kInt8, int NB, int U>
-w8a8_status launch_nb(const StreamArgs& a, cudaStream_t st) {
-  const StreamPlan& p = a.p;
-  dim3 grid(p.groups * p.CS, 1, p.zgroups);
-  dim3 block(32 * p.RPC * p.WS);
-  stream_gemm_kernel<kInt8, NB, U><<<grid, block, 0, st>>>(a);
+template <bool kInt8, int NB, int STEPS>
+w8a8_status launch_steps(const StreamArgs& a, cudaStream_t st) {
+  static bool attr_set[64] = {};
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    W8A8_CUDA(cudaFuncSetAttribute(stream_gemm_kernel<kInt8, NB, STEPS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemLimit / Cps<NB>::value - kStaticReserve));
+    attr_set[dev] = true;
+  }
+  constexpr int EB = kInt8 ? 1 : 2;
+  CUtensorMap tw, tx;
+  W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 128));
+  W8A8_TRY(make_tmap_2d(&tx, a.X, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, 64, 8 * NB));
+  stream_gemm_kernel<kInt8, NB, STEPS><<<a.p.P, kThreads, a.p.smem_bytes, st>>>(tw, tx, a);
   W8A8_LAUNCH_CHECK();
   return W8A8_OK;
+}
+
+template <bool kInt8, int NB>
+w8a8_status launch_nb(const StreamArgs& a, cudaStream_t st) {
+  constexpr int full = Geo<kInt8>::KCMAX / 64;
+  return a.p.KC == Geo<kInt8>::KCMAX ? launch_steps<kInt8, NB, full>(a, st) : launch_steps<kInt8, NB, full / 2>(a, st);
 }
 
 template <bool kInt8>
 w8a8_status launch_typed(const StreamArgs& a, cudaStream_t st) {
   switch (a.p.NB) {
-    case 1: return launch_nb<kInt8, 1, 4>(a, st);
-    case 2: return launch_nb<kInt8, 2, 4>(a, st);
-    case 4: return launch_nb<kInt8, 4, 2>(a, st);
-    default: return launch_nb<kInt8, 8, 1>(a, st);
+    case 1: return launch_nb<kInt8, 1>(a, st);
+    case 2: return launch_nb<kInt8, 2>(a, st);
+    case 4: return launch_nb<kInt8, 4>(a, st);
+    default: return launch_nb<kInt8, 8>(a, st);
   }
+}
+
+// ---------------------------------------------------------------------------------------------
+// INT8 GEMV for M <= 4 tokens: dp4a on the INT8 codes of both operands (exact INT32 sums, no
+// widening), the activation codes resident in shared memory for the whole kernel.  Same producer,
+// unit decomposition, partial-tile protocol and epilogues as the MMA kernel.  Lane l of consumer
+// warp w reads, in pass i, 16 bytes of tile row 16w + (l & 7) + 8 (i & 1) at logical chunk
+// (l >> 3) + 4 (i >> 1): the 8 lanes of a shared-memory phase read one logical chunk of 8 rows
+// whose swizzle keys differ, so the phase touches every bank once.
+template <int MT, int NCH>
+__global__ void __launch_bounds__(kThreads, 2)
+    gemv_dp4a_kernel(const __grid_constant__ CUtensorMap tmW, const StreamArgs a) {
+  constexpr int KC = NCH * 16;  // k bytes (= elements) per unit
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ int s_flag;
+  __shared__ unsigned long long s_best[kConsumerWarps][MT];
+
+  const StreamPlan& p = a.p;
+  const int S = p.stages, SB = p.stage_bytes;
+  const uint32_t raw_u32 = smem_u32(smem_raw);
+  const uint32_t ring = (raw_u32 + 1023u) & ~1023u;
+  const uint32_t xs = ring + (uint32_t)S * SB;                      // X codes [MT][K] (+ zero tail)
+  const uint32_t xbytes = (uint32_t)((MT * a.K + KC + 15) / 16 * 16);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (ring - raw_u32) + (size_t)S * SB + xbytes);
+  uint64_t* empty = full + S;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = p.G, C = p.C;
+  const long long U = (long long)G * C;
+  const int P = gridDim.x, cta = blockIdx.x;
+  const long long u0 = p.whole ? (long long)cta * G / P * C : (long long)cta * U / P;
+  const long long u1 = p.whole ? (long long)(cta + 1) * G / P * C : (long long)(cta + 1) * U / P;
+  auto cta_of = [&](long long u) -> int { return (int)(((u + 1) * P + U - 1) / U - 1); };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(full + s), 1);
+      mbar_init(smem_u32(empty + s), kConsumerWarps);
+    }
+    fence_mbar_init();
+  }
+  // activation codes -> shared memory (tokens >= M and the tail past K are zero)
+  {
+    const int8_t* X = reinterpret_cast<const int8_t*>(a.X);
+    uint8_t* xsp = smem_raw + (xs - raw_u32);
+    for (uint32_t i = threadIdx.x; i < xbytes / 16; i += blockDim.x) {
+      const uint32_t byte = i * 16;
+      const int m = (int)(byte / (uint32_t)a.K), k = (int)(byte % (uint32_t)a.K);
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (m < a.M) v = *reinterpret_cast<const uint4*>(X + (size_t)m * a.K + k);
+      *reinterpret_cast<uint4*>(xsp + byte) = v;
+    }
+  }
+  __syncthreads();
+  if (u0 >= u1) return;
+
+  if (warp == kConsumerWarps) {  // ---------------------------------------------- producer thread
+    if (lane != 0) return;
+    constexpr int nw = KC / 128;
+    bool ok = true;
+    long long it = 0;
+    for (long long u = u0; u < u1; ++u, ++it) {
+      const int s = (int)(it % S);
+      const uint32_t ph = (uint32_t)((it / S) & 1);
+      if (!mbar_wait_bounded(smem_u32(empty + s), ph ^ 1u, kWaitBudgetCycles)) {
+        ok = false;
+        break;
+      }
+      const int g = (int)(u / C), ch = (int)(u % C);
+      const uint32_t bar = smem_u32(full + s);
+      mbar_arrive_expect_tx(bar, (uint32_t)(nw * kBox));
+      for (int b = 0; b < nw; ++b) tma_load_2d(ring + (uint32_t)s * SB + b * kBox, &tmW, ch * KC + b * 128, g * 128, bar);
+    }
+    if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
+    for (long long j = it > S ? it - S : 0; j < it; ++j) {
+      if (!mbar_wait_bounded(smem_u32(full + (int)(j % S)), (uint32_t)((j / S) & 1), kWaitBudgetCycles)) {
+        atomicOr(a.err, DEVERR_DRAIN_WAIT);
+        break;
+      }
+    }
+    return;
+  }
+
+  // ------------------------------------------------------------------------ consumer warps
+  const int w = warp, rl = lane & 7, cq = lane >> 3;
+  const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
+  int acc[2][MT];
+  bool ok = true;
+  if (want_top)
+    for (int i = lane; i < MT; i += 32) s_best[w][i] = 0ull;
+  __syncwarp();
+
+  auto zero_acc = [&]() {
+#pragma unroll
+    for (int q = 0; q < 2; ++q)
+#pragma unroll
+      for (int m = 0; m < MT; ++m) acc[q][m] = 0;
+  };
+
+  auto epilogue = [&](int g, int (&v)[2][MT]) {  // lanes 0..7 hold rows 16w + rl and 16w + rl + 8
+    const int ra = g * 128 + 16 * w + rl, rb = ra + 8;
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      unsigned long long best = 0ull;
+      if (lane < 8 && m < a.M) {
+        if (a.kind == EPI_GEGLU) {
+          if (rb < a.N) {
+            float gv = __fmul_rn(__fmul_rn(a.s_x[m], a.s_w[ra]), __int2float_rn(v[0][m]));
+            float uv = __fmul_rn(__fmul_rn(a.s_x[m], a.s_w[rb]), __int2float_rn(v[1][m]));
+            if (a.bias) {
+              gv = __fadd_rn(gv, a.bias[ra]);
+              uv = __fadd_rn(uv, a.bias[rb]);
+            }
+            if (a.acc_dbg) {
+              a.acc_dbg[(size_t)m * a.N + ra] = v[0][m];
+              a.acc_dbg[(size_t)m * a.N + rb] = v[1][m];
+            }
+            a.y[(size_t)m * (a.N >> 1) + ((g * 128 + 16 * w) >> 1) + rl] = f32_to_bf16_bits(geglu_recipe(gv, uv));
+          }
+        } else {
+#pragma unroll
+          for (int side = 0; side < 2; ++side) {
+            const int i = side ? rb : ra;
+            if (i >= a.N) continue;
+            float y = __fmul_rn(__fmul_rn(a.s_x[m], a.s_w[i]), __int2float_rn(v[side][m]));
+            if (a.bias) y = __fadd_rn(y, a.bias[i]);
+            if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + i] = v[side][m];
+            if (a.kind == EPI_BF16) {
+              a.y[(size_t)m * a.N + i] = f32_to_bf16_bits(y);
+            } else {
+              if (a.logits) a.logits[(size_t)m * a.N + i] = y;
+              const unsigned long long key =
+                  ((unsigned long long)float_order_key(y) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)i);
+              best = key > best ? key : best;
+            }
+          }
+        }
+      }
+      if (want_top) {
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1) {
+          const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+          best = other > best ? other : best;
+        }
+        if (lane == 0 && best > s_best[w][m]) s_best[w][m] = best;
+      }
+    }
+  };
+
+  auto flush = [&](int g, int chf, int chl) {
+    int v[2][MT];
+#pragma unroll
+    for (int q = 0; q < 2; ++q)
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        int x = acc[q][m];
+        x += __shfl_xor_sync(0xffffffffu, x, 8);
+        x += __shfl_xor_sync(0xffffffffu, x, 16);
+        v[q][m] = x;
+      }
+    if (!(chf == 0 && chl == C - 1)) {
+      const long long ub = (long long)g * C;
+      const int f = cta_of(ub), l = cta_of(ub + C - 1);
+      int* part = reinterpret_cast<int*>(a.partials);
+      auto slot_base = [&](int c) -> int* {
+        const long long cu0 = (long long)c * U / P;
+        const int slot = (g == (int)(cu0 / C)) ? 0 : 1;
+        return part + ((size_t)(c * 2 + slot) * 128) * MT;
+      };
+      if (lane < 8) {
+        int* mine = slot_base(cta);
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+#pragma unroll
+          for (int m = 0; m < MT; ++m) mine[(16 * w + rl + 8 * q) * MT + m] = v[q][m];
+      }
+      __threadfence();
+      named_bar_sync(1, kConsumerWarps * 32);
+      if (threadIdx.x == 0) {
+        const unsigned int prev = atomicAdd(a.tile_counters + f, 1u);
+        const int is_last = prev == (unsigned int)(l - f);
+        if (is_last) a.tile_counters[f] = 0u;
+        s_flag = is_last;
+      }
+      named_bar_sync(1, kConsumerWarps * 32);
+      if (!s_flag) return;
+      __threadfence();
+      if (lane < 8) {
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+#pragma unroll
+          for (int m = 0; m < MT; ++m) v[q][m] = 0;
+        for (int c = f; c <= l; ++c) {
+          const int* src = slot_base(c);
+#pragma unroll
+          for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int m = 0; m < MT; ++m) v[q][m] += __ldcg(src + (16 * w + rl + 8 * q) * MT + m);
+        }
+      }
+    }
+    epilogue(g, v);
+  };
+
+  zero_acc();
+  int cur = -1, chf = 0, chl = 0;
+  long long it = 0;
+  for (long long u = u0; u < u1; ++u, ++it) {
+    const int g = (int)(u / C), ch = (int)(u % C);
+    if (g != cur) {
+      if (cur >= 0) flush(cur, chf, chl);
+      cur = g;
+      chf = ch;
+      zero_acc();
+    }
+    chl = ch;
+    const int s = (int)(it % S);
+    const uint32_t ph = (uint32_t)((it / S) & 1);
+    if (ok) {
+      bool got = true;
+      if (lane == 0) got = mbar_wait_bounded(smem_u32(full + s), ph, kWaitBudgetCycles);
+      got = __shfl_sync(0xffffffffu, got, 0);
+      if (!got) {
+        ok = false;
+        if (lane == 0) atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+      }
+    }
+    if (!ok) continue;
+    const uint32_t wbase = ring + (uint32_t)s * SB + (uint32_t)(16 * w + rl) * 128u;
+    const uint32_t xk = xs + (uint32_t)(ch * KC);
+#pragma unroll
+    for (int i = 0; i < NCH / 2; ++i) {
+      const int q = i & 1, c = cq + 4 * (i >> 1);
+      const uint4 wv = lds128(wbase + (uint32_t)q * 8u * 128u + (uint32_t)(c >> 3) * kBox + (uint32_t)(((c & 7) ^ rl) << 4));
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        const uint4 xv = lds128(xk + (uint32_t)(m * a.K + 16 * c));
+        int r = acc[q][m];
+        r = __dp4a((int)wv.x, (int)xv.x, r);
+        r = __dp4a((int)wv.y, (int)xv.y, r);
+        r = __dp4a((int)wv.z, (int)xv.z, r);
+        r = __dp4a((int)wv.w, (int)xv.w, r);
+        acc[q][m] = r;
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(empty + s));
+  }
+  if (cur >= 0) flush(cur, chf, chl);
+  if (!want_top) return;
+  __syncwarp();
+  if (lane < MT && lane < a.M && s_best[w][lane] != 0ull) atomicMax(a.top_keys + lane, s_best[w][lane]);
+  __threadfence();
+  named_bar_sync(1, kConsumerWarps * 32);
+  if (threadIdx.x == 0) {
+    const unsigned int prev = atomicAdd(a.grid_counter, 1u);
+    s_flag = prev == (unsigned int)(P - 1);
+    if (s_flag) *a.grid_counter = 0u;
+  }
+  named_bar_sync(1, kConsumerWarps * 32);
+  if (!s_flag) return;
+  __threadfence();
+  for (int tk = threadIdx.x; tk < a.M; tk += kConsumerWarps * 32) {
+    const unsigned long long key = atomicExch(a.top_keys + tk, 0ull);
+    a.top1[tk] = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+  }
+}
+
+template <int MT, int NCH>
+w8a8_status launch_dp4a(const StreamArgs& a, cudaStream_t st) {
+  static bool attr_set[64] = {};
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    W8A8_CUDA(cudaFuncSetAttribute(gemv_dp4a_kernel<MT, NCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemLimit / 2 - kStaticReserve));
+    attr_set[dev] = true;
+  }
+  CUtensorMap tw;
+  W8A8_TRY(make_tmap_2d(&tw, a.W, 1, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K, 128, 128));
+  gemv_dp4a_kernel<MT, NCH><<<a.p.P, kThreads, a.p.smem_bytes, st>>>(tw, a);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+template <int MT>
+w8a8_status launch_dp4a_mt(const StreamArgs& a, cudaStream_t st) {
+  return a.p.KC == 256 ? launch_dp4a<MT, 16>(a, st) : launch_dp4a<MT, 8>(a, st);
 }
 
 }  // namespace
 
-StreamPlan make_stream_plan(int M, int N, int K, int sm_count) {
+StreamPlan make_stream_plan(bool int8_weights, int M, int N, int K, int sm_count) {
   StreamPlan p{};
+  if (int8_weights && M <= 4 && (size_t)4 * K <= 32768) {
+    // INT8 GEMV with dp4a: X codes resident, two CTAs per SM, a stage = up to 2 weight boxes
+    p.dp4a = 1;
+    p.MT = M <= 1 ? 1 : M <= 2 ? 2 : 4;
+    p.NB = 1;
+    p.TOK = p.MT;
+    p.Z = 1;
+    p.G = std::max(1, (N + 127) / 128);
+    p.KC = 256;
+    while (p.KC > 128 && (long long)p.G * ((K + p.KC - 1) / p.KC) < 2 * sm_count) p.KC >>= 1;
+    p.C = std::max(1, (K + p.KC - 1) / p.KC);
+    p.P = (int)std::max(1LL, std::min<long long>(std::min(2 * sm_count, kTileCounterSlots), (long long)p.G * p.C));
+    p.whole = p.G >= p.P;
+    if (p.whole) p.KC = 256, p.C = std::max(1, (K + 255) / 256);
+    p.stage_bytes = 2 * kBox;
+    const int xbytes = (p.MT * K + p.KC + 15) / 16 * 16;
+    p.stages = std::max(2, std::min(8, (kSmemLimit / 2 - kStaticReserve - 2048 - xbytes) / p.stage_bytes));
+    p.smem_bytes = p.stages * p.stage_bytes + xbytes + 16 * p.stages + 1024;
+    p.partial_bytes = (size_t)p.P * 2 * 128 * p.MT * 4;
+    return p;
+  }
   p.NB = M <= 8 ? 1 : M <= 16 ? 2 : M <= 32 ? 4 : 8;
-  const int TOK = 8 * p.NB;
-  p.zgroups = M > 0 ? (M + TOK - 1) / TOK : 1;
-  p.RT = (N + 15) / 16;
-  p.KS = std::max(1, (K + 63) / 64);
-  const long target = std::max(1L, (long)sm_count * 16 / p.zgroups);
-  long S = (target + p.RT - 1) / std::max(1, p.RT);
-  S = std::max(1L, std::min((long)p.KS, S));
-  p.sps = (p.KS + (int)S - 1) / (int)S;
-  p.S = (p.KS + p.sps - 1) / p.sps;
-  p.WS = std::min(p.S, 8);
-  p.CS = (p.S + p.WS - 1) / p.WS;
-  p.RPC = std::max(1, std::min(8 / p.WS, p.RT));
-  p.groups = (p.RT + p.RPC - 1) / p.RPC;
-  p.partial_bytes = p.CS > 1 ? (size_t)p.zgroups * p.CS * p.RT * 16 * TOK * 4 : 0;
+  p.TOK = 8 * p.NB;
+  p.Z = std::max(1, (M + p.TOK - 1) / p.TOK);
+  p.G = std::max(1, (N + 127) / 128);
+  // Largest chunk (256, 128 or 64 k elements; the stage holds up to Geo::KC) that still gives every
+  // SM a unit; the grid never exceeds the number of units, so every CTA contributes.
+  const int kcmax = int8_weights ? Geo<true>::KCMAX : Geo<false>::KCMAX;
+  const int kcmin = int8_weights ? 128 : 64;  // one weight box
+  p.KC = kcmax;
+  while (p.KC > kcmin && (long long)p.Z * p.G * ((K + p.KC - 1) / p.KC) < sm_count) p.KC >>= 1;
+  p.C = std::max(1, (K + p.KC - 1) / p.KC);
+  const long long units = (long long)p.Z * p.G * p.C;
+  const int cps = p.NB == 1 ? 2 : 1;  // CTAs per SM (matches Cps<NB>)
+  p.P = (int)std::max(1LL, std::min<long long>(std::min(cps * sm_count, kTileCounterSlots), units));
+  p.whole = (long long)p.Z * p.G >= p.P;
+  if (p.whole) {
+    p.KC = kcmax;
+    p.C = std::max(1, (K + p.KC - 1) / p.KC);
+  }
+  p.stage_bytes = stage_bytes_for(int8_weights, p.TOK);
+  p.stages = std::max(2, std::min(8, (kSmemLimit / cps - kStaticReserve - 2048) / p.stage_bytes));
+  p.smem_bytes = p.stages * p.stage_bytes + 16 * p.stages + 1024;  // + alignment slack for the ring
+  p.partial_bytes = (size_t)p.P * 2 * 128 * p.TOK * 4;
   return p;
 }
 
+static thread_local cudaEvent_t g_ev_start = nullptr, g_ev_stop = nullptr;
+
+void set_kernel_events(void* start, void* stop) {
+  g_ev_start = reinterpret_cast<cudaEvent_t>(start);
+  g_ev_stop = reinterpret_cast<cudaEvent_t>(stop);
+}
+
+static w8a8_status dispatch_stream_gemm(bool int8_weights, const StreamArgs& a, cudaStream_t st);
+
 w8a8_status launch_stream_gemm(bool int8_weights, const StreamArgs& a, cudaStream_t st) {
   if (a.M == 0 || a.N == 0) return W8A8_OK;
-  const StreamPlan& p = a.p;
-  W8A8_CHECK_ARG(p.CS == 1 || p.zgroups * p.groups <= kTileCounterSlots, W8A8_ERR_SHAPE,
-                 "stream GEMM: %d split tiles exceed the %d counter slots", p.zgroups * p.groups, kTileCounterSlots);
+  cudaEvent_t e0 = g_ev_start, e1 = g_ev_stop;
+  g_ev_start = g_ev_stop = nullptr;
+  if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
+  const w8a8_status s = dispatch_stream_gemm(int8_weights, a, st);
+  if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
+  return s;
+}
+
+static w8a8_status dispatch_stream_gemm(bool int8_weights, const StreamArgs& a, cudaStream_t st) {
   W8A8_CHECK_ARG(!(a.kind == EPI_F32 && a.top1) || a.M <= kMaxTopKeys, W8A8_ERR_SHAPE,
                  "top-1: M=%d exceeds %d tokens per call", a.M, kMaxTopKeys);
+  W8A8_CHECK_ARG(a.p.smem_bytes <= kSmemLimit / (a.p.NB == 1 ? 2 : 1) - kStaticReserve, W8A8_ERR_SHAPE,
+                 "stream GEMM: stage does not fit in shared memory");
+  if (a.p.dp4a) {
+    W8A8_CHECK_ARG(int8_weights, W8A8_ERR_INVALID_ARG, "dp4a plan for bf16 weights");
+    switch (a.p.MT) {
+      case 1: return launch_dp4a_mt<1>(a, st);
+      case 2: return launch_dp4a_mt<2>(a, st);
+      default: return launch_dp4a_mt<4>(a, st);
+    }
+  }
   return int8_weights ? launch_typed<true>(a, st) : launch_typed<false>(a, st);
 }
 
-// Workspace carve-up shared by the entry points.
 void attach_reserved(StreamArgs& a, void* ws) {
   char* base = reinterpret_cast<char*>(ws);
   a.tile_counters = reinterpret_cast<unsigned int*>(base);
   a.grid_counter = reinterpret_cast<unsigned int*>(base + kGridCounterOffset);
   a.top_keys = reinterpret_cast<unsigned long long*>(base + kTopKeysOffset);
+  a.err = reinterpret_cast<unsigned int*>(base + kErrWordOffset);
 }
 
 int max_top_keys() { return kMaxTopKeys; }

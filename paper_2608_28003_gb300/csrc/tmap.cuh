@@ -1,0 +1,17 @@
+// Host helper: 2-D TMA tensor maps (cuTensorMapEncodeTiled reached through the runtime's driver
+// entry-point query, so the library does not link libcuda).
+#pragma once
+
+#include <cuda.h>
+
+#include "common.cuh"
+
+namespace w8a8 {
+
+// Row-major [rows, inner] tensor of `elem_bytes`-byte elements with a row pitch of `pitch_bytes`;
+// the box is [box_rows, box_inner] with 128-byte swizzle (box_inner * elem_bytes <= 128) and zero
+// fill outside the tensor.
+w8a8_status make_tmap_2d(CUtensorMap* map, const void* base, int elem_bytes, uint64_t inner, uint64_t rows,
+                         uint64_t pitch_bytes, uint32_t box_inner, uint32_t box_rows);
+
+}  // namespace w8a8

@@ -117,6 +117,7 @@ LINEAR_SHAPES = [
     (16, 6912, 1152),   # the single-linear workload (gate_proj shape, M = 16)
     (1, 1000, 1152),    # ragged N
     (3, 24, 64),
+    (2, 700, 2048),     # dp4a GEMV with two token slots
     (9, 4112, 1040),    # ragged K (not a multiple of 64)
     (17, 200, 6912),    # K-split across CTAs
     (33, 520, 1152),
