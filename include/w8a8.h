@@ -154,6 +154,25 @@ w8a8_status w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const f
                         uint16_t* Y, const w8a8_debug* dbg, void* workspace, size_t ws_bytes,
                         void* stream);
 
+/* The W8A8 linear of w8a8_linear for callers that cannot allocate device memory (no counterpart in
+ * the paper: it exists for integration).  Callers that run where cudaMalloc is not allowed, such
+ * as code inside a framework that owns all device memory or a path with a memory budget fixed at
+ * start-up, cannot provide a workspace; this entry point uses a scratch array built into the
+ * library instead (w8a8_linear_noalloc_capacity() bytes, 8 MiB, held by every GPU that loads the
+ * library until the process exits) and allocates nothing.
+ *   - Same arguments and results as w8a8_linear without the debug outputs and the workspace.
+ *   - Returns W8A8_ERR_SHAPE when M, N, K need more scratch than the array holds (about 32 tokens
+ *     for the Gemma-3-1B shapes); w8a8_linear with a workspace has no such limit.
+ *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
+ *     that device current; make that first call before any stream capture.
+ *   - Every call on a device shares the one array and clears its counter region with a
+ *     cudaMemsetAsync on `stream` before launching, so calls whose execution overlaps on the GPU
+ *     (different streams, or concurrent host threads) race and give undefined results; serialise
+ *     them.  Device-side timeouts are not reported by this entry point. */
+size_t w8a8_linear_noalloc_capacity(void);
+w8a8_status w8a8_linear_noalloc(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias,
+                                uint16_t* Y, void* stream);
+
 /* bf16 pass-through linear of a layer outside the INT8 set (FFN section: such layers keep the
  * original precision): Y = bf16(sum_j x_tj * w_ij (fp32 accumulation) + bias_i).
  * W [N, K] bf16. */

@@ -68,6 +68,8 @@ SIGNATURES = {
     "w8a8_quantize_activations": (_i32, [_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp]),
     "w8a8_linear_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
     "w8a8_linear": (_i32, [ctypes.POINTER(QWeightC), _vp, _i32, _vp, _vp, ctypes.POINTER(DebugC), _vp, _sz, _vp]),
+    "w8a8_linear_noalloc_capacity": (_sz, []),
+    "w8a8_linear_noalloc": (_i32, [ctypes.POINTER(QWeightC), _vp, _i32, _vp, _vp, _vp]),
     "w8a8_linear_bf16_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
     "w8a8_linear_bf16": (_i32, [_vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "w8a8_ffn_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
@@ -257,6 +259,18 @@ def linear(w: QWeight, X: torch.Tensor, bias: Optional[torch.Tensor] = None, deb
                                             buf.numel(), _stream(stream)))
     if debug:
         return Y, {"xq": dbg_t[0], "s_x": dbg_t[1], "acc": dbg_t[2]}
+    return Y
+
+
+def linear_noalloc(w: QWeight, X: torch.Tensor, bias: Optional[torch.Tensor] = None,
+                   out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """W8A8 linear on the library's built-in scratch array: for callers that cannot give a workspace.
+    Calls on one device must not overlap on the GPU (they share the array)."""
+    M = X.shape[0]
+    Y = out if out is not None else torch.empty(M, w.n, dtype=torch.bfloat16, device=X.device)
+    wc = w.c()
+    _check("w8a8_linear_noalloc", lib().w8a8_linear_noalloc(ctypes.byref(wc), _p(_bits(X)), M, _p(bias), _p(Y),
+                                                            _stream(stream)))
     return Y
 
 

@@ -161,6 +161,28 @@ static w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16
   return launch_stream_gemm(false, a, st);
 }
 
+// Internal: the W8A8 linear with its scratch at `scratch` (used by the no-allocation entry point).
+size_t linear_scratch_bytes(int M, int N, int K) { return linear_ws(M, N, K, true, device_sms()).total; }
+
+w8a8_status linear_on_scratch(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, uint16_t* Y,
+                              void* scratch, size_t scratch_bytes, cudaStream_t st) {
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));
+  W8A8_TRY(check_ws("w8a8_linear_noalloc", scratch, scratch_bytes, linear_ws(M, w->n, w->k, true, d.sms).total));
+  return run_w8a8_linear(w, X, M, bias, EPI_BF16, Y, nullptr, nullptr, nullptr, scratch, d.sms, st);
+}
+
+w8a8_status check_linear_args(const char* who, const w8a8_qweight* w, const uint16_t* X, int M, const float* bias,
+                              const uint16_t* Y) {
+  W8A8_TRY(check_qweight(who, w));
+  W8A8_CHECK_ARG(M >= 0, W8A8_ERR_INVALID_ARG, "%s: M=%d is negative", who, M);
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(X && Y, W8A8_ERR_INVALID_ARG, "%s: null X or Y", who);
+  W8A8_CHECK_ARG(aligned16(X) && aligned16(Y) && (!bias || aligned16(bias)), W8A8_ERR_ALIGN,
+                 "%s: X, Y and bias must be 16-byte aligned", who);
+  return W8A8_OK;
+}
+
 }  // namespace w8a8
 
 using namespace w8a8;
