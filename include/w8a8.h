@@ -220,6 +220,134 @@ w8a8_status w8a8_lm_head(const w8a8_head_weights* head, int precision, const uin
                          float* logits, int32_t* top1, void* workspace, size_t ws_bytes,
                          void* stream);
 
+/* ---------------------------------------------------------------------------- decoder
+ * A Gemma-3-1B-shaped decoder (Problem Statement: 26 layers, hidden 1152, 4 query heads sharing
+ * 1 key/value head of dim 256, FFN 6912, vocab 262144, lm_head tied to the embedding; Attention
+ * section: sliding window on local layers) under a per-layer precision mask: FFN layer l is W8A8
+ * when bit l of ffn_bits is set (the sets Q_FFN of Eq. ffn55, ffn1010, ffnall26), the attention
+ * projections of layer l when bit l of attn_bits is set (Q_ATT, Eq. attnffn55, attnffn1010), the
+ * lm_head when lm != 0 (LM Head section); everything else runs the bf16 pass-through.
+ *
+ * Per layer: a = bf16(rmsnorm(r) * ln_in); qkv = Linear(a); q, k = rope(rmsnorm_head(q|k) * q_norm|k_norm);
+ * K/V cache <- k, v; o = bf16(softmax(q k^T / sqrt(head_dim)) v) over keys p - window < j <= p
+ * (all j <= p on global layers); r += rmsnorm(Linear(o)) * ln_post_attn; a = bf16(rmsnorm(r) *
+ * ln_pre_ffn); r += rmsnorm(FFN(a)) * ln_post_ffn.  r starts as embed[token] * fl32(sqrt(hidden))
+ * (fp32 residual stream); logits = lm_head(bf16(rmsnorm(r) * final_norm)).
+ *
+ * The model object owns device buffers it allocates at creation and preparation (KV cache,
+ * activations, workspaces, the fused gate/up bf16 copy, prepared INT8 weights); forward and
+ * decode calls allocate nothing.  All pointers in the structs below are caller-owned device
+ * memory that must outlive the model. */
+typedef struct {
+  int32_t layers, hidden, inter, n_q, n_kv, head_dim, vocab;
+  float eps;                  /* RMSNorm epsilon */
+  float rope_local, rope_global; /* RoPE bases of local / global layers */
+  int32_t window;             /* sliding window of local layers */
+  int32_t n_global;           /* number of global layers listed in global_layers */
+  int32_t global_layers[32];
+  int32_t qk_norm;            /* 1: RMS-normalise q and k per head */
+  int32_t max_batch, max_seq; /* KV-cache capacity: sequences x positions */
+  int32_t max_tokens;         /* largest B * T of one forward call */
+} w8a8_model_cfg;
+
+typedef struct {
+  const uint16_t* wqkv;  /* [(n_q + 2 n_kv) * head_dim, hidden] bf16: q rows, then k, then v */
+  const uint16_t* wo;    /* [hidden, n_q * head_dim] */
+  const uint16_t* wgate; /* [inter, hidden] */
+  const uint16_t* wup;   /* [inter, hidden] */
+  const uint16_t* wdown; /* [hidden, inter] */
+  const float *ln_in, *ln_post_attn, *ln_pre_ffn, *ln_post_ffn; /* [hidden] RMSNorm multipliers */
+  const float *q_norm, *k_norm;                                 /* [head_dim] (used when qk_norm) */
+} w8a8_layer_bf16;
+
+typedef struct w8a8_model w8a8_model;
+
+enum { W8A8_SUB_FFN = 0, W8A8_SUB_ATTN = 1, W8A8_SUB_LM = 2 };
+
+/* layers: array of cfg->layers descriptors; embed [vocab, hidden] bf16 (also the lm_head);
+ * final_norm [hidden].  The mask starts all-bf16. */
+w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_layer_bf16* layers, const uint16_t* embed,
+                              const float* final_norm, w8a8_model** out);
+w8a8_status w8a8_model_destroy(w8a8_model* m);
+
+/* Calibration (LM Head section: max_t |X_tj| at every linear's input, collected over calibration
+ * tokens): runs the all-bf16 decoder over tokens [B, T] (device int32) from position 0 and folds
+ * each linear input's per-channel absolute maximum into the model's statistics.
+ * w8a8_model_reset_calibration zeroes them. */
+w8a8_status w8a8_model_calibrate(w8a8_model* m, const int32_t* tokens, int B, int T, void* stream);
+w8a8_status w8a8_model_reset_calibration(w8a8_model* m, void* stream);
+
+/* The statistics as one fp32 array of w8a8_model_stats_count() values: for each layer l,
+ * [hidden] at the qkv input, [n_q * head_dim] at the o input, [hidden] at the gate/up input and
+ * [inter] at the down input; then [hidden] at the lm_head input.  get / set copy to / from HOST
+ * memory and are synchronous (set replaces statistics gathered so far). */
+size_t w8a8_model_stats_count(const w8a8_model* m);
+w8a8_status w8a8_model_get_stats(const w8a8_model* m, float* host_out);
+w8a8_status w8a8_model_set_stats(w8a8_model* m, const float* host_in);
+
+/* Prepares the W8A8 weights of every linear (qkv, o, fused gate/up, down, lm_head) from the
+ * statistics (w8a8_prepare_weights / w8a8_prepare_gate_up semantics).  Required before a mask
+ * selects W8A8 for any sublayer. */
+w8a8_status w8a8_model_prepare(w8a8_model* m, float alpha, int smooth, void* stream);
+
+/* Host-side, synchronous.  layer in [0, layers) for FFN / ATTN; LM ignores layer. */
+w8a8_status w8a8_set_layer_precision(w8a8_model* m, int layer, int sublayer, int precision);
+w8a8_status w8a8_set_mask(w8a8_model* m, uint32_t ffn_bits, uint32_t attn_bits, int lm);
+w8a8_status w8a8_get_mask(const w8a8_model* m, uint32_t* ffn_bits, uint32_t* attn_bits, int* lm);
+
+/* Runs tokens [B, T] (device int32, row b * T + t at position start_pos + t) through the decoder,
+ * appending to the KV cache.  logits [B * T, vocab] fp32 (nullable), top1 [B * T] int32. */
+w8a8_status w8a8_decoder_forward(w8a8_model* m, const int32_t* tokens, int B, int T, int start_pos, float* logits,
+                                 int32_t* top1, void* stream);
+
+/* One decode step of B sequences (one token each, at position pos) replayed from a CUDA graph
+ * captured on first use for this (B, mask, logits wanted) and kept until the mask or the
+ * preparation changes.  tokens [B], logits [B, vocab] (nullable), top1 [B]: device memory. */
+w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* tokens, int B, int pos, float* logits,
+                                     int32_t* top1, void* stream);
+
+/* Negative log-likelihood of targets under softmax(logits) per row (LM Head section's
+ * perplexity): nll[i] = logsumexp(logits[i, :]) - logits[i, targets[i]], fp32. */
+w8a8_status w8a8_token_nll(const float* logits, const int32_t* targets, int M, int V, float* nll, void* stream);
+
+/* ------------------------------------------------------------------------ allocation
+ * The allocation rule (Problem Statement; Combined Configurations): among the candidates whose
+ * Top-1 agreement with the all-bf16 decoder is >= min_top1 and whose perplexity change is
+ * <= max_ppl_delta, the one with the smallest per-token latency; ties go to fewer INT8
+ * sublayers, then to the earlier candidate.  Host arrays of length n.  Returns the index, or -1
+ * if no candidate is feasible. */
+int w8a8_choose_mask(const float* latency, const float* top1, const float* ppl_delta, const int32_t* n_int8, int n,
+                     float min_top1, float max_ppl_delta);
+
+typedef struct {
+  uint32_t ffn_bits, attn_bits;
+  int32_t lm;
+} w8a8_mask;
+
+typedef struct {
+  const w8a8_mask* candidates; /* host array of n_candidates masks */
+  int32_t n_candidates;
+  const int32_t* eval_tokens;  /* device [eval_B, eval_T]: teacher-forced evaluation stream */
+  int32_t eval_B, eval_T;
+  int32_t decode_B;            /* latency: decode steps of decode_B sequences ... */
+  int32_t prefill_T;           /* ... after a prefill of prefill_T tokens ... */
+  int32_t decode_steps;        /* ... timed over decode_steps steps, median of reps runs */
+  int32_t reps;
+  float min_top1, max_ppl_delta;
+} w8a8_alloc_opts;
+
+typedef struct {
+  int32_t chosen;     /* index into candidates, -1 if none is feasible */
+  float* latency_ms;  /* host [n_candidates]: median ms per decode step */
+  float* top1;        /* host [n_candidates]: Top-1 agreement with the all-bf16 decoder */
+  float* ppl_delta;   /* host [n_candidates]: PPL / PPL(bf16) - 1 on the evaluation stream */
+} w8a8_alloc_report;
+
+/* The allocator: measures every candidate (latency with CUDA events; quality against the all-bf16
+ * decoder on the evaluation stream) and applies w8a8_choose_mask.  Leaves the chosen mask set
+ * (the all-bf16 mask if none is feasible).  Synchronous; requires w8a8_model_prepare. */
+w8a8_status w8a8_allocate_mask(w8a8_model* m, const w8a8_alloc_opts* opts, w8a8_alloc_report* report, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

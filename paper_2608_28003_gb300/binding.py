@@ -55,6 +55,38 @@ class HeadC(ctypes.Structure):
     _fields_ = [("vocab", ctypes.c_int32), ("hidden", ctypes.c_int32), ("q", QWeightC), ("bf16", _vp)]
 
 
+class ModelCfgC(ctypes.Structure):
+    _fields_ = [("layers", ctypes.c_int32), ("hidden", ctypes.c_int32), ("inter", ctypes.c_int32),
+                ("n_q", ctypes.c_int32), ("n_kv", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("vocab", ctypes.c_int32), ("eps", ctypes.c_float), ("rope_local", ctypes.c_float),
+                ("rope_global", ctypes.c_float), ("window", ctypes.c_int32), ("n_global", ctypes.c_int32),
+                ("global_layers", ctypes.c_int32 * 32), ("qk_norm", ctypes.c_int32), ("max_batch", ctypes.c_int32),
+                ("max_seq", ctypes.c_int32), ("max_tokens", ctypes.c_int32)]
+
+
+class LayerBf16C(ctypes.Structure):
+    _fields_ = [("wqkv", _vp), ("wo", _vp), ("wgate", _vp), ("wup", _vp), ("wdown", _vp), ("ln_in", _vp),
+                ("ln_post_attn", _vp), ("ln_pre_ffn", _vp), ("ln_post_ffn", _vp), ("q_norm", _vp), ("k_norm", _vp)]
+
+
+class MaskC(ctypes.Structure):
+    _fields_ = [("ffn_bits", ctypes.c_uint32), ("attn_bits", ctypes.c_uint32), ("lm", ctypes.c_int32)]
+
+
+class AllocOptsC(ctypes.Structure):
+    _fields_ = [("candidates", ctypes.POINTER(MaskC)), ("n_candidates", ctypes.c_int32), ("eval_tokens", _vp),
+                ("eval_B", ctypes.c_int32), ("eval_T", ctypes.c_int32), ("decode_B", ctypes.c_int32),
+                ("prefill_T", ctypes.c_int32), ("decode_steps", ctypes.c_int32), ("reps", ctypes.c_int32),
+                ("min_top1", ctypes.c_float), ("max_ppl_delta", ctypes.c_float)]
+
+
+class AllocReportC(ctypes.Structure):
+    _fields_ = [("chosen", ctypes.c_int32), ("latency_ms", ctypes.POINTER(ctypes.c_float)),
+                ("top1", ctypes.POINTER(ctypes.c_float)), ("ppl_delta", ctypes.POINTER(ctypes.c_float))]
+
+
+_fp = ctypes.POINTER(ctypes.c_float)
+
 # name -> (restype, argtypes)
 SIGNATURES = {
     "w8a8_abi_version": (_i32, []),
@@ -76,6 +108,24 @@ SIGNATURES = {
     "w8a8_ffn_block": (_i32, [ctypes.POINTER(FfnC), _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "w8a8_lm_head_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
     "w8a8_lm_head": (_i32, [ctypes.POINTER(HeadC), _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+    "w8a8_model_create": (_i32, [ctypes.POINTER(ModelCfgC), ctypes.POINTER(LayerBf16C), _vp, _vp,
+                                 ctypes.POINTER(_vp)]),
+    "w8a8_model_destroy": (_i32, [_vp]),
+    "w8a8_model_calibrate": (_i32, [_vp, _vp, _i32, _i32, _vp]),
+    "w8a8_model_reset_calibration": (_i32, [_vp, _vp]),
+    "w8a8_model_prepare": (_i32, [_vp, _f32, _i32, _vp]),
+    "w8a8_model_stats_count": (_sz, [_vp]),
+    "w8a8_model_get_stats": (_i32, [_vp, _fp]),
+    "w8a8_model_set_stats": (_i32, [_vp, _fp]),
+    "w8a8_set_layer_precision": (_i32, [_vp, _i32, _i32, _i32]),
+    "w8a8_set_mask": (_i32, [_vp, ctypes.c_uint32, ctypes.c_uint32, _i32]),
+    "w8a8_get_mask": (_i32, [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32),
+                             ctypes.POINTER(_i32)]),
+    "w8a8_decoder_forward": (_i32, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp]),
+    "w8a8_decoder_decode_step": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp, _vp]),
+    "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
+    "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
+    "w8a8_allocate_mask": (_i32, [_vp, ctypes.POINTER(AllocOptsC), ctypes.POINTER(AllocReportC), _vp]),
 }
 
 _LIB = None
@@ -344,3 +394,151 @@ def lm_head(hd: HeadWeights, precision: int, X: torch.Tensor, want_logits: bool 
                                               _p(logits) if want_logits else None, _p(top1), _p(buf), buf.numel(),
                                               _stream(stream)))
     return (logits if want_logits else None), top1
+
+
+# ------------------------------------------------------------------------------- decoder
+W8A8_SUB_FFN, W8A8_SUB_ATTN, W8A8_SUB_LM = 0, 1, 2
+
+
+def choose_mask(latency, top1, ppl_delta, n_int8, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> int:
+    """The library's allocation rule on host arrays (index, or -1 if nothing is feasible)."""
+    n = len(latency)
+    arr = lambda v, t: (t * n)(*v)  # noqa: E731
+    return lib().w8a8_choose_mask(arr(latency, ctypes.c_float), arr(top1, ctypes.c_float),
+                                  arr(ppl_delta, ctypes.c_float), arr(n_int8, ctypes.c_int32), n,
+                                  float(min_top1), float(max_ppl_delta))
+
+
+@dataclass
+class DecoderConfig:
+    layers: int = 26
+    hidden: int = 1152
+    inter: int = 6912
+    n_q: int = 4
+    n_kv: int = 1
+    head_dim: int = 256
+    vocab: int = 262144
+    eps: float = 1e-6
+    rope_local: float = 10000.0
+    rope_global: float = 1000000.0
+    window: int = 1024
+    global_layers: tuple = (0, 6, 12, 18)
+    qk_norm: bool = True
+    max_batch: int = 1
+    max_seq: int = 2048
+    max_tokens: int = 2048
+
+    def c(self) -> ModelCfgC:
+        g = (ctypes.c_int32 * 32)(*list(self.global_layers))
+        return ModelCfgC(self.layers, self.hidden, self.inter, self.n_q, self.n_kv, self.head_dim, self.vocab,
+                         self.eps, self.rope_local, self.rope_global, self.window, len(self.global_layers), g,
+                         int(self.qk_norm), self.max_batch, self.max_seq, self.max_tokens)
+
+
+class Decoder:
+    """Handle on a w8a8_model.  Keeps the caller-owned weight tensors alive while the model lives.
+
+    weights: dict of per-layer lists of bf16 CUDA tensors (wqkv, wo, wg, wu, wd) and "embed";
+    norms: dict of per-layer lists of fp32 CUDA tensors (ln_in, ln_post_attn, ln_pre_ffn,
+    ln_post_ffn, q_norm, k_norm) and "final_norm"."""
+
+    def __init__(self, cfg: DecoderConfig, weights: dict, norms: dict):
+        self.cfg = cfg
+        self._keep = (weights, norms)
+        layers = (LayerBf16C * cfg.layers)()
+        for l in range(cfg.layers):
+            layers[l] = LayerBf16C(*(t.data_ptr() for t in (
+                weights["wqkv"][l], weights["wo"][l], weights["wg"][l], weights["wu"][l], weights["wd"][l],
+                norms["ln_in"][l], norms["ln_post_attn"][l], norms["ln_pre_ffn"][l], norms["ln_post_ffn"][l],
+                norms["q_norm"][l], norms["k_norm"][l])))
+        h = ctypes.c_void_p()
+        cc = cfg.c()
+        _check("w8a8_model_create", lib().w8a8_model_create(ctypes.byref(cc), layers, _p(weights["embed"]),
+                                                            _p(norms["final_norm"]), ctypes.byref(h)))
+        self.h = h
+
+    def close(self):
+        if self.h:
+            _check("w8a8_model_destroy", lib().w8a8_model_destroy(self.h))
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def calibrate(self, tokens: torch.Tensor, stream=None):
+        B, T = tokens.shape
+        _check("w8a8_model_calibrate", lib().w8a8_model_calibrate(self.h, _p(_bits(tokens)), B, T, _stream(stream)))
+
+    def reset_calibration(self, stream=None):
+        _check("w8a8_model_reset_calibration", lib().w8a8_model_reset_calibration(self.h, _stream(stream)))
+
+    def get_stats(self):
+        """Calibration statistics (host numpy fp32; layout of w8a8_model_get_stats)."""
+        import numpy as np
+        n = lib().w8a8_model_stats_count(self.h)
+        out = np.zeros(n, dtype=np.float32)
+        _check("w8a8_model_get_stats", lib().w8a8_model_get_stats(self.h, out.ctypes.data_as(_fp)))
+        return out
+
+    def set_stats(self, stats):
+        import numpy as np
+        s = np.ascontiguousarray(stats, dtype=np.float32)
+        assert s.size == lib().w8a8_model_stats_count(self.h)
+        _check("w8a8_model_set_stats", lib().w8a8_model_set_stats(self.h, s.ctypes.data_as(_fp)))
+
+    def prepare(self, alpha: float = 0.5, smooth: bool = True, stream=None):
+        _check("w8a8_model_prepare", lib().w8a8_model_prepare(self.h, float(alpha), int(smooth), _stream(stream)))
+
+    def set_mask(self, ffn_bits: int = 0, attn_bits: int = 0, lm: bool = False):
+        _check("w8a8_set_mask", lib().w8a8_set_mask(self.h, ffn_bits, attn_bits, int(lm)))
+
+    def get_mask(self):
+        f, a, l = ctypes.c_uint32(), ctypes.c_uint32(), ctypes.c_int32()
+        _check("w8a8_get_mask", lib().w8a8_get_mask(self.h, ctypes.byref(f), ctypes.byref(a), ctypes.byref(l)))
+        return f.value, a.value, l.value
+
+    def set_layer_precision(self, layer: int, sublayer: int, precision: int):
+        _check("w8a8_set_layer_precision", lib().w8a8_set_layer_precision(self.h, layer, sublayer, precision))
+
+    def forward(self, tokens: torch.Tensor, start_pos: int = 0, want_logits: bool = True, stream=None):
+        B, T = tokens.shape
+        dev = tokens.device
+        logits = torch.empty(B * T, self.cfg.vocab, dtype=torch.float32, device=dev) if want_logits else None
+        top1 = torch.empty(B * T, dtype=torch.int32, device=dev)
+        _check("w8a8_decoder_forward", lib().w8a8_decoder_forward(self.h, _p(_bits(tokens)), B, T, int(start_pos),
+                                                                  _p(logits), _p(top1), _stream(stream)))
+        return logits, top1
+
+    def decode_step(self, tokens: torch.Tensor, pos: int, logits: Optional[torch.Tensor] = None,
+                    top1: Optional[torch.Tensor] = None, stream=None):
+        B = tokens.shape[0]
+        if top1 is None:
+            top1 = torch.empty(B, dtype=torch.int32, device=tokens.device)
+        _check("w8a8_decoder_decode_step", lib().w8a8_decoder_decode_step(self.h, _p(_bits(tokens)), B, int(pos),
+                                                                          _p(logits), _p(top1), _stream(stream)))
+        return logits, top1
+
+    def allocate(self, candidates, eval_tokens: torch.Tensor, decode_B: int, prefill_T: int, decode_steps: int,
+                 reps: int = 3, min_top1: float = 0.989, max_ppl_delta: float = 0.01, stream=None) -> dict:
+        """Run the allocator over candidate masks [(ffn_bits, attn_bits, lm), ...]."""
+        n = len(candidates)
+        masks = (MaskC * n)(*[MaskC(f, a, int(l)) for f, a, l in candidates])
+        eB, eT = eval_tokens.shape
+        opts = AllocOptsC(masks, n, _bits(eval_tokens).data_ptr(), eB, eT, decode_B, prefill_T, decode_steps, reps,
+                          float(min_top1), float(max_ppl_delta))
+        lat, t1, pd = (ctypes.c_float * n)(), (ctypes.c_float * n)(), (ctypes.c_float * n)()
+        rep = AllocReportC(-1, lat, t1, pd)
+        _check("w8a8_allocate_mask", lib().w8a8_allocate_mask(self.h, ctypes.byref(opts), ctypes.byref(rep),
+                                                              _stream(stream)))
+        return {"chosen": rep.chosen, "latency_ms": list(lat), "top1": list(t1), "ppl_delta": list(pd)}
+
+
+def token_nll(logits: torch.Tensor, targets: torch.Tensor, stream=None) -> torch.Tensor:
+    M, V = logits.shape
+    out = torch.empty(M, dtype=torch.float32, device=logits.device)
+    _check("w8a8_token_nll", lib().w8a8_token_nll(_p(_bits(logits)), _p(_bits(targets)), M, V, _p(out),
+                                                  _stream(stream)))
+    return out

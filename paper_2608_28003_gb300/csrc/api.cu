@@ -5,6 +5,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "ops.cuh"
 #include "stream_gemm.cuh"
 
 namespace w8a8 {
@@ -19,18 +20,10 @@ void set_error(const char* fmt, ...) {
 }
 const char* get_error() { return g_err; }
 
-w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* inv_delta, int8_t* xq,
-                                 uint16_t* xq_f16, float* s_x, cudaStream_t st);
-
-// Per-device facts, looked up once per device.
-struct DevInfo {
-  int ok = -1;  // -1 unknown, 0 unsupported, 1 sm_103
-  int sms = 0;
-};
 static DevInfo g_dev[64];
 static std::mutex g_dev_mu;
 
-static w8a8_status dev_info(DevInfo* out) {
+w8a8_status dev_info(DevInfo* out) {
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   W8A8_CHECK_ARG(dev >= 0 && dev < 64, W8A8_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
@@ -60,12 +53,9 @@ int device_sms() {
 }
 
 // ------------------------------------------------------------------------ workspace plans
-// Layout: [reserved counters | x codes fp16 [M,K] | s_x [M] | partials]
-struct LinearWs {
-  size_t xf16, sx, part, total;
-};
+// Layout: [reserved counters | x codes [M,K] | s_x [M] | partials]
 
-static LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
+LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
   LinearWs w{};
   size_t off = W8A8_WS_RESERVED;
   w.xf16 = off;
@@ -110,7 +100,7 @@ static w8a8_status quantize_for(const StreamPlan& p, const uint16_t* X, int M, i
 }
 
 // One W8A8 linear: K1 then the streaming GEMM.  s_x and the codes live in the workspace.
-static w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
+w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
                                    uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
                                    int sms, cudaStream_t st) {
   const int N = w->n, K = w->k;
@@ -140,7 +130,7 @@ static w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int
   return launch_stream_gemm(true, a, st);
 }
 
-static w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias,
+w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias,
                                    int kind, uint16_t* Y, float* logits, int32_t* top1, void* ws, int sms,
                                    cudaStream_t st) {
   LinearWs L = linear_ws(M, N, K, false, sms);
@@ -260,10 +250,10 @@ extern "C" w8a8_status w8a8_linear_bf16(const uint16_t* W, int N, int K, const u
 
 // ------------------------------------------------------------------------------- FFN
 // Layout: [reserved | h bf16 [M,F] | gate/up linear scratch | down linear scratch]
-struct FfnWs {
-  size_t h, gu, dn, total;
-};
-static FfnWs ffn_ws(int M, int H, int F, int sms) {
+
+namespace w8a8 {
+
+FfnWs ffn_ws(int M, int H, int F, int sms) {
   FfnWs w{};
   size_t off = W8A8_WS_RESERVED;
   w.h = off;
@@ -277,6 +267,92 @@ static FfnWs ffn_ws(int M, int H, int F, int sms) {
   w.total = off;
   return w;
 }
+
+w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y, uint16_t* h_dbg,
+                    void* workspace, int sms, cudaStream_t st) {
+  const int H = f->hidden, F = f->inter;
+  const FfnWs L = ffn_ws(M, H, F, sms);
+  char* base = reinterpret_cast<char*>(workspace);
+  uint16_t* h = h_dbg ? h_dbg : reinterpret_cast<uint16_t*>(base + L.h);
+  // The two linears run one after the other on `stream` and share the FFN workspace's reserved
+  // counters (each leaves them zero); their scratch regions are disjoint.
+  if (precision == W8A8_PREC_W8A8) {
+    // gate/up: scratch at L.gu
+    {
+      const LinearWs A = linear_ws(M, 2 * F, H, true, sms);
+      void* codes = base + L.gu + (A.xf16 - W8A8_WS_RESERVED);
+      float* s_x = reinterpret_cast<float*>(base + L.gu + (A.sx - W8A8_WS_RESERVED));
+      StreamArgs a{};
+      a.p = make_stream_plan(true, M, 2 * F, H, sms);
+      W8A8_TRY(quantize_for(a.p, X, M, H, f->gate_up.inv_delta, codes, nullptr, s_x, st));
+      a.W = f->gate_up.wq;
+      a.X = codes;
+      a.M = M;
+      a.N = 2 * F;
+      a.K = H;
+      a.kind = EPI_GEGLU;
+      a.s_x = s_x;
+      a.s_w = f->gate_up.s_w;
+      a.y = h;
+      a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(true, a, st));
+    }
+    {
+      const LinearWs B = linear_ws(M, H, F, true, sms);
+      void* codes = base + L.dn + (B.xf16 - W8A8_WS_RESERVED);
+      float* s_x = reinterpret_cast<float*>(base + L.dn + (B.sx - W8A8_WS_RESERVED));
+      StreamArgs a{};
+      a.p = make_stream_plan(true, M, H, F, sms);
+      W8A8_TRY(quantize_for(a.p, h, M, F, f->down.inv_delta, codes, nullptr, s_x, st));
+      a.W = f->down.wq;
+      a.X = codes;
+      a.M = M;
+      a.N = H;
+      a.K = F;
+      a.kind = EPI_BF16;
+      a.s_x = s_x;
+      a.s_w = f->down.s_w;
+      a.y = Y;
+      a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(true, a, st));
+    }
+  } else {
+    {
+      const LinearWs A = linear_ws(M, 2 * F, H, false, sms);
+      StreamArgs a{};
+      a.W = f->gate_up_bf16;
+      a.X = X;
+      a.M = M;
+      a.N = 2 * F;
+      a.K = H;
+      a.p = make_stream_plan(false, M, 2 * F, H, sms);
+      a.kind = EPI_GEGLU;
+      a.y = h;
+      a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(false, a, st));
+    }
+    {
+      const LinearWs B = linear_ws(M, H, F, false, sms);
+      StreamArgs a{};
+      a.W = f->down_bf16;
+      a.X = h;
+      a.M = M;
+      a.N = H;
+      a.K = F;
+      a.p = make_stream_plan(false, M, H, F, sms);
+      a.kind = EPI_BF16;
+      a.y = Y;
+      a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);
+      attach_reserved(a, workspace);
+      W8A8_TRY(launch_stream_gemm(false, a, st));
+    }
+  }
+  return W8A8_OK;
+}
+}  // namespace w8a8
 
 extern "C" w8a8_status w8a8_ffn_workspace_size(int M, int hidden, int inter, size_t* bytes) {
   W8A8_CHECK_ARG(bytes && M >= 0 && hidden >= 0 && inter >= 0, W8A8_ERR_INVALID_ARG, "w8a8_ffn_workspace_size: bad argument");
@@ -311,86 +387,7 @@ extern "C" w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* f, int precision, 
   W8A8_TRY(dev_info(&d));
   const FfnWs L = ffn_ws(M, H, F, d.sms);
   W8A8_TRY(check_ws("w8a8_ffn_block", workspace, ws_bytes, L.total));
-  cudaStream_t st = as_stream(stream);
-  char* base = reinterpret_cast<char*>(workspace);
-  uint16_t* h = h_dbg ? h_dbg : reinterpret_cast<uint16_t*>(base + L.h);
-  // The two linears run one after the other on `stream` and share the FFN workspace's reserved
-  // counters (each leaves them zero); their scratch regions are disjoint.
-  if (precision == W8A8_PREC_W8A8) {
-    // gate/up: scratch at L.gu
-    {
-      const LinearWs A = linear_ws(M, 2 * F, H, true, d.sms);
-      void* codes = base + L.gu + (A.xf16 - W8A8_WS_RESERVED);
-      float* s_x = reinterpret_cast<float*>(base + L.gu + (A.sx - W8A8_WS_RESERVED));
-      StreamArgs a{};
-      a.p = make_stream_plan(true, M, 2 * F, H, d.sms);
-      W8A8_TRY(quantize_for(a.p, X, M, H, f->gate_up.inv_delta, codes, nullptr, s_x, st));
-      a.W = f->gate_up.wq;
-      a.X = codes;
-      a.M = M;
-      a.N = 2 * F;
-      a.K = H;
-      a.kind = EPI_GEGLU;
-      a.s_x = s_x;
-      a.s_w = f->gate_up.s_w;
-      a.y = h;
-      a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
-      attach_reserved(a, workspace);
-      W8A8_TRY(launch_stream_gemm(true, a, st));
-    }
-    {
-      const LinearWs B = linear_ws(M, H, F, true, d.sms);
-      void* codes = base + L.dn + (B.xf16 - W8A8_WS_RESERVED);
-      float* s_x = reinterpret_cast<float*>(base + L.dn + (B.sx - W8A8_WS_RESERVED));
-      StreamArgs a{};
-      a.p = make_stream_plan(true, M, H, F, d.sms);
-      W8A8_TRY(quantize_for(a.p, h, M, F, f->down.inv_delta, codes, nullptr, s_x, st));
-      a.W = f->down.wq;
-      a.X = codes;
-      a.M = M;
-      a.N = H;
-      a.K = F;
-      a.kind = EPI_BF16;
-      a.s_x = s_x;
-      a.s_w = f->down.s_w;
-      a.y = Y;
-      a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);
-      attach_reserved(a, workspace);
-      W8A8_TRY(launch_stream_gemm(true, a, st));
-    }
-  } else {
-    {
-      const LinearWs A = linear_ws(M, 2 * F, H, false, d.sms);
-      StreamArgs a{};
-      a.W = f->gate_up_bf16;
-      a.X = X;
-      a.M = M;
-      a.N = 2 * F;
-      a.K = H;
-      a.p = make_stream_plan(false, M, 2 * F, H, d.sms);
-      a.kind = EPI_GEGLU;
-      a.y = h;
-      a.partials = base + L.gu + (A.part - W8A8_WS_RESERVED);
-      attach_reserved(a, workspace);
-      W8A8_TRY(launch_stream_gemm(false, a, st));
-    }
-    {
-      const LinearWs B = linear_ws(M, H, F, false, d.sms);
-      StreamArgs a{};
-      a.W = f->down_bf16;
-      a.X = h;
-      a.M = M;
-      a.N = H;
-      a.K = F;
-      a.p = make_stream_plan(false, M, H, F, d.sms);
-      a.kind = EPI_BF16;
-      a.y = Y;
-      a.partials = base + L.dn + (B.part - W8A8_WS_RESERVED);
-      attach_reserved(a, workspace);
-      W8A8_TRY(launch_stream_gemm(false, a, st));
-    }
-  }
-  return W8A8_OK;
+  return run_ffn(f, precision, X, M, Y, h_dbg, workspace, d.sms, as_stream(stream));
 }
 
 // --------------------------------------------------------------------------- lm_head

@@ -1,0 +1,412 @@
+// Supporting kernels of the Gemma-3-1B-shaped decoder: embedding + RMSNorm, residual + sandwich
+// RMSNorms, QK-norm + RoPE + KV-cache write, and causal (sliding-window) GQA attention.
+// bf16 activations between kernels, an fp32 residual stream, fp32 arithmetic inside.
+#include <cmath>
+
+#include "decoder_kernels.cuh"
+
+namespace w8a8 {
+
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum over the block (blockDim.x a multiple of 32, at most 1024); every thread gets the result.
+__device__ float block_sum(float v, float* red) {
+  v = warp_sum(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float s = 0.0f;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
+  return s;
+}
+
+constexpr int kRowThreads = 128;
+constexpr int kRowVec = 4;  // 8-element vectors per thread: H <= 4096
+
+__device__ __forceinline__ void unpack8(const uint4& w, float (&x)[8]) {
+  x[0] = bf16_lo(w.x); x[1] = bf16_hi(w.x); x[2] = bf16_lo(w.y); x[3] = bf16_hi(w.y);
+  x[4] = bf16_lo(w.z); x[5] = bf16_hi(w.z); x[6] = bf16_lo(w.w); x[7] = bf16_hi(w.w);
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&x)[8]) {
+  uint4 w;
+  w.x = (uint32_t)f32_to_bf16_bits(x[0]) | ((uint32_t)f32_to_bf16_bits(x[1]) << 16);
+  w.y = (uint32_t)f32_to_bf16_bits(x[2]) | ((uint32_t)f32_to_bf16_bits(x[3]) << 16);
+  w.z = (uint32_t)f32_to_bf16_bits(x[4]) | ((uint32_t)f32_to_bf16_bits(x[5]) << 16);
+  w.w = (uint32_t)f32_to_bf16_bits(x[6]) | ((uint32_t)f32_to_bf16_bits(x[7]) << 16);
+  return w;
+}
+
+__global__ void __launch_bounds__(kRowThreads) embed_norm_kernel(const int32_t* __restrict__ tokens, int vocab,
+                                                                 const uint16_t* __restrict__ embed, int H, float scale,
+                                                                 const float* __restrict__ w, float eps,
+                                                                 float* __restrict__ r, uint16_t* __restrict__ a) {
+  __shared__ float red[32];
+  const int row = blockIdx.x;
+  int tok = tokens[row];
+  if (tok < 0 || tok >= vocab) tok = 0;  // an invalid id reads row 0 instead of faulting
+  const int nv = H >> 3;
+  const uint4* src = reinterpret_cast<const uint4*>(embed + (size_t)tok * H);
+  float x[kRowVec][8];
+  float ss = 0.0f;
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      unpack8(src[vi], x[v]);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        x[v][e] *= scale;
+        ss += x[v][e] * x[v][e];
+      }
+    }
+  }
+  const float inv = 1.0f / sqrtf(block_sum(ss, red) / (float)H + eps);
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      float4* rp = reinterpret_cast<float4*>(r + (size_t)row * H + vi * 8);
+      rp[0] = make_float4(x[v][0], x[v][1], x[v][2], x[v][3]);
+      rp[1] = make_float4(x[v][4], x[v][5], x[v][6], x[v][7]);
+      float y[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) y[e] = x[v][e] * inv * w[vi * 8 + e];
+      reinterpret_cast<uint4*>(a + (size_t)row * H)[vi] = pack8(y);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kRowThreads) residual_norm_kernel(const uint16_t* __restrict__ y, int H,
+                                                                    const float* __restrict__ w_post,
+                                                                    const float* __restrict__ w_next, float eps,
+                                                                    float* __restrict__ r, uint16_t* __restrict__ a) {
+  __shared__ float red[32];
+  const int row = blockIdx.x;
+  const int nv = H >> 3;
+  float yv[kRowVec][8];
+  float ss = 0.0f;
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      unpack8(reinterpret_cast<const uint4*>(y + (size_t)row * H)[vi], yv[v]);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) ss += yv[v][e] * yv[v][e];
+    }
+  }
+  const float inv_y = 1.0f / sqrtf(block_sum(ss, red) / (float)H + eps);
+  float ss2 = 0.0f;
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      float4* rp = reinterpret_cast<float4*>(r + (size_t)row * H + vi * 8);
+      const float4 r0 = rp[0], r1 = rp[1];
+      float rv[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        rv[e] += yv[v][e] * inv_y * w_post[vi * 8 + e];
+        yv[v][e] = rv[e];  // keep the new residual
+        ss2 += rv[e] * rv[e];
+      }
+      rp[0] = make_float4(rv[0], rv[1], rv[2], rv[3]);
+      rp[1] = make_float4(rv[4], rv[5], rv[6], rv[7]);
+    }
+  }
+  const float inv_r = 1.0f / sqrtf(block_sum(ss2, red) / (float)H + eps);
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      float o[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) o[e] = yv[v][e] * inv_r * w_next[vi * 8 + e];
+      reinterpret_cast<uint4*>(a + (size_t)row * H)[vi] = pack8(o);
+    }
+  }
+}
+
+// One warp per head of a row (q heads, then k heads, then v heads).  hd == 256: lane l holds
+// dims 4l..4l+3 and 128+4l..128+4l+3, i.e. the four RoPE pairs (i, i + 128), i = 4l..4l+3.
+__global__ void qk_rope_kernel(const uint16_t* __restrict__ qkv, AttnShape s, const int* __restrict__ pos0,
+                               const float* __restrict__ qn, const float* __restrict__ kn, float eps,
+                               const float* __restrict__ rope_cos, const float* __restrict__ rope_sin,
+                               float* __restrict__ q, uint16_t* __restrict__ kcache, uint16_t* __restrict__ vcache) {
+  const int row = blockIdx.x;
+  const int b = row / s.T, t = row - (row / s.T) * s.T;
+  const int pos = *pos0 + t;
+  const int head = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int hd = s.hd, half = hd >> 1;
+  const int qkv_dim = (s.n_q + 2 * s.n_kv) * hd;
+  const uint16_t* src = qkv + (size_t)row * qkv_dim + (size_t)head * hd;
+  float x1[4], x2[4];
+  {
+    const uint2 a = *reinterpret_cast<const uint2*>(src + 4 * lane);
+    const uint2 c = *reinterpret_cast<const uint2*>(src + half + 4 * lane);
+    x1[0] = bf16_lo(a.x); x1[1] = bf16_hi(a.x); x1[2] = bf16_lo(a.y); x1[3] = bf16_hi(a.y);
+    x2[0] = bf16_lo(c.x); x2[1] = bf16_hi(c.x); x2[2] = bf16_lo(c.y); x2[3] = bf16_hi(c.y);
+  }
+  const bool is_q = head < s.n_q, is_k = !is_q && head < s.n_q + s.n_kv;
+  const size_t cache_row = ((size_t)b * s.max_seq + pos) * (size_t)(s.n_kv * hd);
+  if (!is_q && !is_k) {  // v: straight into the cache
+    const int vh = head - s.n_q - s.n_kv;
+    uint16_t* dst = vcache + cache_row + (size_t)vh * hd;
+    *reinterpret_cast<uint2*>(dst + 4 * lane) = *reinterpret_cast<const uint2*>(src + 4 * lane);
+    *reinterpret_cast<uint2*>(dst + half + 4 * lane) = *reinterpret_cast<const uint2*>(src + half + 4 * lane);
+    return;
+  }
+  const float* nw = is_q ? qn : kn;
+  if (nw) {
+    float ss = 0.0f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) ss += x1[e] * x1[e] + x2[e] * x2[e];
+    const float inv = 1.0f / sqrtf(warp_sum(ss) / (float)hd + eps);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x1[e] = x1[e] * inv * nw[4 * lane + e];
+      x2[e] = x2[e] * inv * nw[half + 4 * lane + e];
+    }
+  }
+  float y1[4], y2[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float c = rope_cos[(size_t)pos * half + 4 * lane + e], sn = rope_sin[(size_t)pos * half + 4 * lane + e];
+    y1[e] = x1[e] * c - x2[e] * sn;
+    y2[e] = x2[e] * c + x1[e] * sn;
+  }
+  if (is_q) {
+    float* dst = q + (size_t)row * (s.n_q * hd) + (size_t)head * hd;
+    *reinterpret_cast<float4*>(dst + 4 * lane) = make_float4(y1[0], y1[1], y1[2], y1[3]);
+    *reinterpret_cast<float4*>(dst + half + 4 * lane) = make_float4(y2[0], y2[1], y2[2], y2[3]);
+  } else {
+    const int kh = head - s.n_q;
+    uint16_t* dst = kcache + cache_row + (size_t)kh * hd;
+    uint2 u1, u2;
+    u1.x = (uint32_t)f32_to_bf16_bits(y1[0]) | ((uint32_t)f32_to_bf16_bits(y1[1]) << 16);
+    u1.y = (uint32_t)f32_to_bf16_bits(y1[2]) | ((uint32_t)f32_to_bf16_bits(y1[3]) << 16);
+    u2.x = (uint32_t)f32_to_bf16_bits(y2[0]) | ((uint32_t)f32_to_bf16_bits(y2[1]) << 16);
+    u2.y = (uint32_t)f32_to_bf16_bits(y2[2]) | ((uint32_t)f32_to_bf16_bits(y2[3]) << 16);
+    *reinterpret_cast<uint2*>(dst + 4 * lane) = u1;
+    *reinterpret_cast<uint2*>(dst + half + 4 * lane) = u2;
+  }
+}
+
+// ---------------------------------------------------------------------------------- attention
+constexpr int kKeyTile = 32;
+constexpr int kHd = 256;
+constexpr int kPartStride = kHd + 4;  // floats per split partial: o[256], m, l, 2 pad (16-byte multiple)
+
+// grid (splits, rows, n_kv), block 32 * G (G = n_q / n_kv query heads sharing one key/value head).
+// Warp h handles query head kvh * G + h; lane l holds dims 8l .. 8l+7 of q and of its output.
+__global__ void __launch_bounds__(256) attention_kernel(const float* __restrict__ q, const uint16_t* __restrict__ kcache,
+                                                        const uint16_t* __restrict__ vcache, AttnShape s,
+                                                        const int* __restrict__ pos0, uint16_t* __restrict__ o,
+                                                        float* __restrict__ part, unsigned int* __restrict__ ctr) {
+  __shared__ __align__(16) uint16_t ks[kKeyTile][kHd];
+  __shared__ __align__(16) uint16_t vs[kKeyTile][kHd];
+  __shared__ int s_last;
+  const int S = gridDim.x, split = blockIdx.x, row = blockIdx.y, kvh = blockIdx.z;
+  const int G = blockDim.x >> 5;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int head = kvh * G + warp;
+  const int b = row / s.T, t = row - (row / s.T) * s.T;
+  const int pos = *pos0 + t;
+  const int lo = s.window > 0 ? max(0, pos - s.window + 1) : 0;
+  const int len = pos - lo + 1;
+  const int chunk = (len + S - 1) / S;
+  const int kb = lo + split * chunk, ke = min(pos + 1, kb + chunk);
+
+  float qv[8];
+  {
+    const float4* qp = reinterpret_cast<const float4*>(q + (size_t)row * (s.n_q * kHd) + (size_t)head * kHd + 8 * lane);
+    const float4 a = qp[0], c = qp[1];
+    qv[0] = a.x * s.scale; qv[1] = a.y * s.scale; qv[2] = a.z * s.scale; qv[3] = a.w * s.scale;
+    qv[4] = c.x * s.scale; qv[5] = c.y * s.scale; qv[6] = c.z * s.scale; qv[7] = c.w * s.scale;
+  }
+  float m = -INFINITY, l = 0.0f, acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  const size_t seq_base = ((size_t)b * s.max_seq) * (size_t)(s.n_kv * kHd) + (size_t)kvh * kHd;
+  for (int j0 = kb; j0 < ke; j0 += kKeyTile) {
+    const int nk = min(kKeyTile, ke - j0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nk * (kHd / 8); i += blockDim.x) {
+      const int jj = i / (kHd / 8), c = i - jj * (kHd / 8);
+      const size_t off = seq_base + (size_t)(j0 + jj) * (s.n_kv * kHd) + 8 * c;
+      reinterpret_cast<uint4*>(&ks[jj][0])[c] = *reinterpret_cast<const uint4*>(kcache + off);
+      reinterpret_cast<uint4*>(&vs[jj][0])[c] = *reinterpret_cast<const uint4*>(vcache + off);
+    }
+    __syncthreads();
+    float sc = -INFINITY;  // lane jj keeps the score of key jj
+    for (int jj = 0; jj < nk; ++jj) {
+      float kx[8];
+      unpack8(reinterpret_cast<const uint4*>(&ks[jj][0])[lane], kx);
+      float d = 0.0f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) d += qv[e] * kx[e];
+      d = warp_sum(d);
+      if (lane == jj) sc = d;
+    }
+    float tmax = sc;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, off));
+    const float m_new = fmaxf(m, tmax);
+    const float corr = expf(m - m_new);  // 0 on the first tile (m = -inf)
+    const float p = lane < nk ? expf(sc - m_new) : 0.0f;
+    l = l * corr + warp_sum(p);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] *= corr;
+    for (int jj = 0; jj < nk; ++jj) {
+      const float pj = __shfl_sync(0xffffffffu, p, jj);
+      float vx[8];
+      unpack8(reinterpret_cast<const uint4*>(&vs[jj][0])[lane], vx);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] += pj * vx[e];
+    }
+    m = m_new;
+  }
+
+  uint16_t* out = o + (size_t)row * (s.n_q * kHd) + (size_t)head * kHd + 8 * lane;
+  if (S == 1) {
+    float y[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) y[e] = acc[e] / l;
+    *reinterpret_cast<uint4*>(out) = pack8(y);
+    return;
+  }
+  // partial (m, l, acc) of this split; the last CTA of (row, kvh) combines
+  float* pp = part + (((size_t)row * s.n_q + head) * S + split) * kPartStride;
+  reinterpret_cast<float4*>(pp + 8 * lane)[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  reinterpret_cast<float4*>(pp + 8 * lane)[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+  if (lane == 0) {
+    pp[kHd] = m;
+    pp[kHd + 1] = l;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned int* c = ctr + (size_t)row * s.n_kv + kvh;
+    const unsigned int prev = atomicAdd(c, 1u);
+    s_last = prev == (unsigned int)(S - 1);
+    if (s_last) *c = 0u;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const float* base = part + ((size_t)row * s.n_q + head) * S * kPartStride;
+  float mx = -INFINITY;
+  for (int sp = 0; sp < S; ++sp) mx = fmaxf(mx, __ldcg(base + (size_t)sp * kPartStride + kHd));
+  float L = 0.0f, y[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  for (int sp = 0; sp < S; ++sp) {
+    const float* ps = base + (size_t)sp * kPartStride;
+    const float ms = __ldcg(ps + kHd);
+    if (ms == -INFINITY) continue;  // an empty split
+    const float f = expf(ms - mx);
+    L += __ldcg(ps + kHd + 1) * f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) y[e] += __ldcg(ps + 8 * lane + e) * f;
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) y[e] /= L;
+  *reinterpret_cast<uint4*>(out) = pack8(y);
+}
+
+__global__ void rope_table_kernel(float* cos_t, float* sin_t, int max_seq, int half, int hd, double base) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= max_seq * half) return;
+  const int pos = idx / half, i = idx - (idx / half) * half;
+  const double inv_freq = pow(base, -2.0 * (double)i / (double)hd);
+  const double ang = (double)pos * inv_freq;
+  cos_t[idx] = (float)cos(ang);
+  sin_t[idx] = (float)sin(ang);
+}
+
+__global__ void set_int_kernel(int* dst, int v) { *dst = v; }
+
+int attention_splits(const AttnShape& s, int sm_count) {
+  const int rows = s.B * s.T * s.n_kv;
+  if (rows >= 2 * sm_count) return 1;
+  const int want = (2 * sm_count + rows - 1) / rows;
+  return std::max(1, std::min(32, want));
+}
+
+}  // namespace
+
+w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embed, int vocab, int H, float embed_scale,
+                              const float* w, float eps, float* r, uint16_t* a, cudaStream_t st) {
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "embed: hidden %d unsupported", H);
+  embed_norm_kernel<<<M, kRowThreads, 0, st>>>(tokens, vocab, embed, H, embed_scale, w, eps, r, a);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w_post, const float* w_next, float eps,
+                                 float* r, uint16_t* a, cudaStream_t st) {
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "residual norm: hidden %d unsupported", H);
+  residual_norm_kernel<<<M, kRowThreads, 0, st>>>(y, H, w_post, w_next, eps, r, a);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+w8a8_status launch_qk_rope(const uint16_t* qkv, const AttnShape& s, const int* pos0, const float* qn, const float* kn,
+                           float eps, const float* rope_cos, const float* rope_sin, float* q, uint16_t* kcache,
+                           uint16_t* vcache, cudaStream_t st) {
+  const int M = s.B * s.T;
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(s.hd == kHd && s.n_q + 2 * s.n_kv <= 32, W8A8_ERR_SHAPE, "qk_rope: head_dim %d / heads unsupported", s.hd);
+  qk_rope_kernel<<<M, 32 * (s.n_q + 2 * s.n_kv), 0, st>>>(qkv, s, pos0, qn, kn, eps, rope_cos, rope_sin, q, kcache,
+                                                           vcache);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+// Workspace: [kAttnCounterBytes of per-(row, kv head) arrival counters, zero between calls | partials]
+constexpr size_t kAttnCounterBytes = 65536;
+
+size_t attention_workspace_bytes(const AttnShape& s, int sm_count) {
+  const size_t rows = (size_t)s.B * s.T;
+  const int S = attention_splits(s, sm_count);
+  const size_t partial = S > 1 ? rows * s.n_q * S * kPartStride * 4 : 0;
+  return kAttnCounterBytes + partial;
+}
+
+w8a8_status launch_attention(const float* q, const uint16_t* kcache, const uint16_t* vcache, const AttnShape& s,
+                             const int* pos0, int max_pos_hint, uint16_t* o, void* ws, int sm_count, cudaStream_t st) {
+  (void)max_pos_hint;
+  const int M = s.B * s.T;
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(s.hd == kHd && s.n_kv > 0 && s.n_q % s.n_kv == 0 && s.n_q / s.n_kv <= 8, W8A8_ERR_SHAPE,
+                 "attention: head layout unsupported");
+  W8A8_CHECK_ARG((size_t)M * s.n_kv * 4 <= kAttnCounterBytes, W8A8_ERR_SHAPE, "attention: %d rows exceed the counters",
+                 M);
+  const int S = attention_splits(s, sm_count);
+  unsigned int* ctr = reinterpret_cast<unsigned int*>(ws);
+  float* part = reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + kAttnCounterBytes);
+  dim3 grid(S, M, s.n_kv);
+  attention_kernel<<<grid, 32 * (s.n_q / s.n_kv), 0, st>>>(q, kcache, vcache, s, pos0, o, part, ctr);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+w8a8_status launch_rope_table(float* cos_t, float* sin_t, int max_seq, int hd, double base, cudaStream_t st) {
+  const int half = hd / 2;
+  const int n = max_seq * half;
+  rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(cos_t, sin_t, max_seq, half, hd, base);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+w8a8_status launch_set_int(int* dst, int value, cudaStream_t st) {
+  set_int_kernel<<<1, 1, 0, st>>>(dst, value);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+}  // namespace w8a8

@@ -1,0 +1,42 @@
+// Supporting kernels of the Gemma-3-1B-shaped decoder (bf16 activations, fp32 residual stream).
+#pragma once
+
+#include "common.cuh"
+
+namespace w8a8 {
+
+struct AttnShape {
+  int B, T;            // sequences, new tokens per sequence (rows are b * T + t)
+  int n_q, n_kv, hd;   // query heads, key/value heads, head dim (hd == 256 supported)
+  int max_seq;         // KV-cache capacity per sequence
+  int window;          // sliding window (keys p - window < j <= p), or 0 for global attention
+  float scale;         // attention scale
+};
+
+// r = fp32(embed[token]) * embed_scale; a = bf16(rmsnorm(r) * w) (token ids outside [0, vocab) read row 0)
+w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embed, int vocab, int H, float embed_scale,
+                              const float* w, float eps, float* r, uint16_t* a, cudaStream_t st);
+
+// r += rmsnorm(y) * w_post;  a = bf16(rmsnorm(r) * w_next)
+w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w_post, const float* w_next, float eps,
+                                 float* r, uint16_t* a, cudaStream_t st);
+
+// Per row: q heads and k head RMS-normalised (weights qn, kn; skipped when null), RoPE at position
+// *pos0 + t, q -> fp32 [M, n_q*hd], k and v -> bf16 KV cache [B][max_seq][n_kv*hd] of this layer.
+w8a8_status launch_qk_rope(const uint16_t* qkv, const AttnShape& s, const int* pos0, const float* qn, const float* kn,
+                           float eps, const float* rope_cos, const float* rope_sin, float* q, uint16_t* kcache,
+                           uint16_t* vcache, cudaStream_t st);
+
+// Causal softmax attention over the cache; o bf16 [M, n_q*hd].  Long key ranges are split across
+// CTAs; the last CTA of a row combines the splits (workspace: partials + per-row counters, the
+// counters zero before and after).
+size_t attention_workspace_bytes(const AttnShape& s, int sm_count);
+w8a8_status launch_attention(const float* q, const uint16_t* kcache, const uint16_t* vcache, const AttnShape& s,
+                             const int* pos0, int max_pos_hint, uint16_t* o, void* ws, int sm_count, cudaStream_t st);
+
+// cos/sin tables [max_seq][hd/2] of RoPE with the given base, computed in fp64
+w8a8_status launch_rope_table(float* cos_t, float* sin_t, int max_seq, int hd, double base, cudaStream_t st);
+
+w8a8_status launch_set_int(int* dst, int value, cudaStream_t st);
+
+}  // namespace w8a8

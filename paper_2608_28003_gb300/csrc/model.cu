@@ -1,0 +1,661 @@
+// The Gemma-3-1B-shaped decoder under a per-layer precision mask, its calibration and weight
+// preparation, CUDA-graph decode steps, the token NLL, and the mask allocator (host C++ driving
+// the library's kernels).
+#include <algorithm>
+#include <chrono>
+#include <cmath>
+#include <map>
+#include <tuple>
+#include <vector>
+
+#include "decoder_kernels.cuh"
+#include "ops.cuh"
+#include "stream_gemm.cuh"
+
+using namespace w8a8;
+
+namespace {
+
+struct QW {
+  int8_t* wq = nullptr;
+  float* s_w = nullptr;
+  float* delta = nullptr;
+  float* inv_delta = nullptr;
+};
+
+constexpr int kHeadChunk = 2048;  // lm_head rows per launch (top-1 keys per call)
+
+}  // namespace
+
+struct w8a8_model {
+  w8a8_model_cfg cfg{};
+  int sms = 152;
+  std::vector<w8a8_layer_bf16> L;
+  const uint16_t* embed = nullptr;
+  const float* final_norm = nullptr;
+  int q_dim = 0, kv_dim = 0, qkv_dim = 0;
+  float embed_scale = 1.0f;
+
+  uint16_t* gu_bf16 = nullptr;  // [layers][2F][H] bf16, 8-row gate/up interleave
+  std::vector<QW> q_qkv, q_o, q_gu, q_down;
+  QW q_lm;
+  bool prepared = false;
+  int prep_version = 0;
+  float* stats = nullptr;  // per layer: [H] qkv input, [q_dim] o input, [H] gate/up input, [F] down input; then [H] lm
+
+  uint32_t ffn_bits = 0, attn_bits = 0;
+  int lm = 0;
+
+  float* r = nullptr;
+  uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *y = nullptr, *h = nullptr;
+  float* q = nullptr;
+  uint16_t *kc = nullptr, *vc = nullptr;
+  float *cos_l = nullptr, *sin_l = nullptr, *cos_g = nullptr, *sin_g = nullptr;
+  int* d_pos = nullptr;
+  int32_t* d_tokens = nullptr;
+  float* d_logits = nullptr;
+  int32_t* d_top1 = nullptr;
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  void* attn_ws = nullptr;
+  size_t attn_ws_bytes = 0;
+
+  cudaStream_t st = nullptr;  // private stream for graph capture / replay
+  cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+  std::map<std::tuple<int, uint32_t, uint32_t, int, int, int>, cudaGraphExec_t> graphs;
+  std::vector<void*> allocs;
+
+  size_t stats_stride() const { return (size_t)2 * cfg.hidden + q_dim + cfg.inter; }
+  float* stat_qkv(int l) const { return stats + l * stats_stride(); }
+  float* stat_o(int l) const { return stat_qkv(l) + cfg.hidden; }
+  float* stat_gu(int l) const { return stat_o(l) + q_dim; }
+  float* stat_down(int l) const { return stat_gu(l) + cfg.hidden; }
+  float* stat_lm() const { return stats + (size_t)cfg.layers * stats_stride(); }
+  size_t cache_layer_elems() const { return (size_t)cfg.max_batch * cfg.max_seq * kv_dim; }
+  bool is_global(int l) const {
+    for (int i = 0; i < cfg.n_global; ++i)
+      if (cfg.global_layers[i] == l) return true;
+    return false;
+  }
+};
+
+namespace {
+
+template <class T>
+w8a8_status dalloc(w8a8_model* m, T** p, size_t count) {
+  void* v = nullptr;
+  W8A8_CUDA(cudaMalloc(&v, std::max<size_t>(count * sizeof(T), 16)));
+  m->allocs.push_back(v);
+  *p = reinterpret_cast<T*>(v);
+  return W8A8_OK;
+}
+
+void free_all(w8a8_model* m) {
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  m->graphs.clear();
+  for (void* p : m->allocs) cudaFree(p);
+  m->allocs.clear();
+  if (m->ev_in) cudaEventDestroy(m->ev_in);
+  if (m->ev_out) cudaEventDestroy(m->ev_out);
+  if (m->st) cudaStreamDestroy(m->st);
+}
+
+w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, nullptr}; }
+
+w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
+                   uint16_t* Y, cudaStream_t st) {
+  if (int8) {
+    const w8a8_qweight w = qdesc(qw, N, K);
+    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st);
+  }
+  return run_bf16_linear(Wbf, N, K, X, M, nullptr, 0, Y, nullptr, nullptr, m->ws, m->sms, st);
+}
+
+// The decoder over M = B * T rows whose positions start at *m->d_pos (set by the caller).
+w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, float* logits, int32_t* top1, bool calib,
+                         cudaStream_t st) {
+  const w8a8_model_cfg& c = m->cfg;
+  const int M = B * T, H = c.hidden, F = c.inter;
+  W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, m->r, m->a, st));
+  for (int l = 0; l < c.layers; ++l) {
+    const w8a8_layer_bf16& W = m->L[l];
+    const bool att8 = !calib && m->prepared && ((m->attn_bits >> l) & 1u);
+    const bool ffn8 = !calib && m->prepared && ((m->ffn_bits >> l) & 1u);
+    const bool glob = m->is_global(l);
+    if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_qkv(l), st));
+    W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st));
+    AttnShape s{B, T, c.n_q, c.n_kv, c.head_dim, c.max_seq, glob ? 0 : c.window,
+                (float)(1.0 / std::sqrt((double)c.head_dim))};
+    uint16_t* kc = m->kc + (size_t)l * m->cache_layer_elems();
+    uint16_t* vc = m->vc + (size_t)l * m->cache_layer_elems();
+    W8A8_TRY(launch_qk_rope(m->qkv, s, m->d_pos, c.qk_norm ? W.q_norm : nullptr, c.qk_norm ? W.k_norm : nullptr, c.eps,
+                            glob ? m->cos_g : m->cos_l, glob ? m->sin_g : m->sin_l, m->q, kc, vc, st));
+    W8A8_TRY(launch_attention(m->q, kc, vc, s, m->d_pos, 0, m->o, m->attn_ws, m->sms, st));
+    if (calib) W8A8_TRY(launch_act_absmax(m->o, M, m->q_dim, m->stat_o(l), st));
+    W8A8_TRY(linear(m, att8, m->q_o[l], W.wo, H, m->q_dim, m->o, M, m->y, st));
+    W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, m->r, m->a, st));
+    if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
+    w8a8_ffn_weights f{H,
+                       F,
+                       qdesc(m->q_gu[l], 2 * F, H),
+                       qdesc(m->q_down[l], H, F),
+                       m->gu_bf16 + (size_t)l * 2 * F * H,
+                       W.wdown};
+    W8A8_TRY(run_ffn(&f, ffn8 ? W8A8_PREC_W8A8 : W8A8_PREC_BF16, m->a, M, m->y, calib ? m->h : nullptr, m->ws, m->sms,
+                     st));
+    if (calib) W8A8_TRY(launch_act_absmax(m->h, M, F, m->stat_down(l), st));
+    const float* next = l + 1 < c.layers ? m->L[l + 1].ln_in : m->final_norm;
+    W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, m->r, m->a, st));
+  }
+  if (calib) return launch_act_absmax(m->a, M, H, m->stat_lm(), st);
+  const bool lm8 = m->prepared && m->lm;
+  for (int r0 = 0; r0 < M; r0 += kHeadChunk) {
+    const int rows = std::min(kHeadChunk, M - r0);
+    const uint16_t* X = m->a + (size_t)r0 * H;
+    float* lg = logits ? logits + (size_t)r0 * c.vocab : nullptr;
+    int32_t* tp = top1 + r0;
+    if (lm8) {
+      const w8a8_qweight w = qdesc(m->q_lm, c.vocab, H);
+      W8A8_TRY(run_w8a8_linear(&w, X, rows, nullptr, 2, nullptr, lg, tp, nullptr, m->ws, m->sms, st));
+    } else {
+      W8A8_TRY(run_bf16_linear(m->embed, c.vocab, H, X, rows, nullptr, 2, nullptr, lg, tp, m->ws, m->sms, st));
+    }
+  }
+  return W8A8_OK;
+}
+
+w8a8_status check_call(w8a8_model* m, int B, int T, int start_pos) {
+  W8A8_CHECK_ARG(m != nullptr, W8A8_ERR_INVALID_ARG, "null model");
+  W8A8_CHECK_ARG(B > 0 && T > 0 && B <= m->cfg.max_batch && B * T <= m->cfg.max_tokens, W8A8_ERR_SHAPE,
+                 "B=%d T=%d exceeds the model's capacity (max_batch %d, max_tokens %d)", B, T, m->cfg.max_batch,
+                 m->cfg.max_tokens);
+  W8A8_CHECK_ARG(start_pos >= 0 && start_pos + T <= m->cfg.max_seq, W8A8_ERR_SHAPE,
+                 "positions %d..%d exceed max_seq %d", start_pos, start_pos + T - 1, m->cfg.max_seq);
+  return W8A8_OK;
+}
+
+// ------------------------------------------------------------------------------ NLL kernel
+__global__ void nll_kernel(const float* __restrict__ logits, const int32_t* __restrict__ targets, int V,
+                           float* __restrict__ nll) {
+  __shared__ double red[32];
+  __shared__ float s_max;
+  const int row = blockIdx.x;
+  const float* z = logits + (size_t)row * V;
+  float mx = -INFINITY;
+  for (int i = threadIdx.x; i < V; i += blockDim.x) mx = fmaxf(mx, z[i]);
+  mx = warp_max(mx);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float v = -INFINITY;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) v = fmaxf(v, (float)red[i]);
+    s_max = v;
+  }
+  __syncthreads();
+  const float m = s_max;
+  double sum = 0.0;
+  for (int i = threadIdx.x; i < V; i += blockDim.x) sum += exp((double)(z[i] - m));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sum;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
+    const int tg = targets[row];
+    nll[row] = (float)(log(s) + (double)m - (double)z[tg]);
+  }
+}
+
+__global__ void shift_targets_kernel(const int32_t* tokens, int B, int T, int32_t* targets) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * T) return;
+  const int t = i % T;
+  targets[i] = t + 1 < T ? tokens[i + 1] : tokens[i];
+}
+
+__global__ void fill_tokens_kernel(int32_t* tokens, int n, int vocab) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) tokens[i] = (int32_t)(((long long)i * 7919 + 13) % vocab);
+}
+
+}  // namespace
+
+// ====================================================================================== ABI
+extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_layer_bf16* layers,
+                                         const uint16_t* embed, const float* final_norm, w8a8_model** out) {
+  W8A8_CHECK_ARG(cfg && layers && embed && final_norm && out, W8A8_ERR_INVALID_ARG, "w8a8_model_create: null argument");
+  const w8a8_model_cfg& c = *cfg;
+  W8A8_CHECK_ARG(c.layers > 0 && c.layers <= 32 && c.hidden > 0 && c.hidden % 16 == 0 && c.hidden <= 4096 &&
+                     c.inter > 0 && c.inter % 16 == 0 && c.head_dim == 256 && c.n_kv > 0 && c.n_q % c.n_kv == 0 &&
+                     c.n_q / c.n_kv <= 8 && c.n_q + 2 * c.n_kv <= 32 && c.vocab > 0 && c.max_batch > 0 &&
+                     c.max_seq > 0 && c.max_tokens > 0 && c.n_global >= 0 && c.n_global <= 32,
+                 W8A8_ERR_SHAPE, "w8a8_model_create: unsupported configuration");
+  W8A8_CHECK_ARG(aligned16(embed) && aligned16(final_norm), W8A8_ERR_ALIGN, "w8a8_model_create: unaligned pointer");
+  for (int l = 0; l < c.layers; ++l) {
+    const w8a8_layer_bf16& W = layers[l];
+    W8A8_CHECK_ARG(W.wqkv && W.wo && W.wgate && W.wup && W.wdown && W.ln_in && W.ln_post_attn && W.ln_pre_ffn &&
+                       W.ln_post_ffn && (!c.qk_norm || (W.q_norm && W.k_norm)),
+                   W8A8_ERR_INVALID_ARG, "w8a8_model_create: layer %d has a null pointer", l);
+    W8A8_CHECK_ARG(aligned16(W.wqkv) && aligned16(W.wo) && aligned16(W.wgate) && aligned16(W.wup) &&
+                       aligned16(W.wdown),
+                   W8A8_ERR_ALIGN, "w8a8_model_create: layer %d weight not 16-byte aligned", l);
+  }
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));
+  w8a8_model* m = new w8a8_model();
+  m->cfg = c;
+  m->sms = d.sms;
+  m->L.assign(layers, layers + c.layers);
+  m->embed = embed;
+  m->final_norm = final_norm;
+  m->q_dim = c.n_q * c.head_dim;
+  m->kv_dim = c.n_kv * c.head_dim;
+  m->qkv_dim = m->q_dim + 2 * m->kv_dim;
+  m->embed_scale = (float)std::sqrt((double)c.hidden);
+  m->q_qkv.resize(c.layers);
+  m->q_o.resize(c.layers);
+  m->q_gu.resize(c.layers);
+  m->q_down.resize(c.layers);
+  auto fail = [&](w8a8_status s) {
+    free_all(m);
+    delete m;
+    return s;
+  };
+#define W8A8_MTRY(expr)             \
+  do {                              \
+    w8a8_status s_ = (expr);        \
+    if (s_ != W8A8_OK) return fail(s_); \
+  } while (0)
+  const int H = c.hidden, F = c.inter, Mx = c.max_tokens;
+  W8A8_MTRY(cudaStreamCreateWithFlags(&m->st, cudaStreamNonBlocking) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+  W8A8_MTRY(cudaEventCreateWithFlags(&m->ev_in, cudaEventDisableTiming) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+  W8A8_MTRY(cudaEventCreateWithFlags(&m->ev_out, cudaEventDisableTiming) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+  W8A8_MTRY(dalloc(m, &m->gu_bf16, (size_t)c.layers * 2 * F * H));
+  W8A8_MTRY(dalloc(m, &m->stats, (size_t)c.layers * m->stats_stride() + H));
+  W8A8_MTRY(dalloc(m, &m->r, (size_t)Mx * H));
+  W8A8_MTRY(dalloc(m, &m->a, (size_t)Mx * H));
+  W8A8_MTRY(dalloc(m, &m->qkv, (size_t)Mx * m->qkv_dim));
+  W8A8_MTRY(dalloc(m, &m->q, (size_t)Mx * m->q_dim));
+  W8A8_MTRY(dalloc(m, &m->o, (size_t)Mx * m->q_dim));
+  W8A8_MTRY(dalloc(m, &m->y, (size_t)Mx * H));
+  W8A8_MTRY(dalloc(m, &m->h, (size_t)Mx * F));
+  W8A8_MTRY(dalloc(m, &m->kc, (size_t)c.layers * m->cache_layer_elems()));
+  W8A8_MTRY(dalloc(m, &m->vc, (size_t)c.layers * m->cache_layer_elems()));
+  const size_t rope = (size_t)c.max_seq * (c.head_dim / 2);
+  W8A8_MTRY(dalloc(m, &m->cos_l, rope));
+  W8A8_MTRY(dalloc(m, &m->sin_l, rope));
+  W8A8_MTRY(dalloc(m, &m->cos_g, rope));
+  W8A8_MTRY(dalloc(m, &m->sin_g, rope));
+  W8A8_MTRY(dalloc(m, &m->d_pos, 4));
+  W8A8_MTRY(dalloc(m, &m->d_tokens, (size_t)c.max_batch));
+  W8A8_MTRY(dalloc(m, &m->d_logits, (size_t)c.max_batch * c.vocab));
+  W8A8_MTRY(dalloc(m, &m->d_top1, (size_t)c.max_batch));
+  // GEMM workspace: the largest of the model's linears at max_tokens rows (lm_head in chunks)
+  size_t ws = 0;
+  const int Mh = std::min(Mx, kHeadChunk);
+  ws = std::max(ws, linear_ws(Mx, m->qkv_dim, H, true, d.sms).total);
+  ws = std::max(ws, linear_ws(Mx, m->qkv_dim, H, false, d.sms).total);
+  ws = std::max(ws, linear_ws(Mx, H, m->q_dim, true, d.sms).total);
+  ws = std::max(ws, linear_ws(Mx, H, m->q_dim, false, d.sms).total);
+  ws = std::max(ws, ffn_ws(Mx, H, F, d.sms).total);
+  ws = std::max(ws, linear_ws(Mh, c.vocab, H, true, d.sms).total);
+  ws = std::max(ws, linear_ws(Mh, c.vocab, H, false, d.sms).total);
+  m->ws_bytes = ws;
+  W8A8_MTRY(dalloc(m, reinterpret_cast<char**>(&m->ws), ws));
+  W8A8_MTRY((size_t)Mx * c.n_kv * 4 <= 65536 ? W8A8_OK : W8A8_ERR_SHAPE);  // attention counters
+  size_t aws = 0;
+  for (int rows = 1; rows <= Mx; ++rows) {  // the split count depends on the row count: take the maximum
+    AttnShape s{1, rows, c.n_q, c.n_kv, c.head_dim, c.max_seq, 0, 1.0f};
+    aws = std::max(aws, attention_workspace_bytes(s, d.sms));
+  }
+  m->attn_ws_bytes = aws;
+  W8A8_MTRY(dalloc(m, reinterpret_cast<char**>(&m->attn_ws), aws));
+  cudaStream_t st = m->st;
+  W8A8_MTRY(cudaMemsetAsync(m->ws, 0, W8A8_WS_RESERVED, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+  W8A8_MTRY(cudaMemsetAsync(m->attn_ws, 0, aws, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+  W8A8_MTRY(cudaMemsetAsync(m->stats, 0, ((size_t)c.layers * m->stats_stride() + H) * 4, st) == cudaSuccess
+                ? W8A8_OK
+                : W8A8_ERR_CUDA);
+  W8A8_MTRY(launch_rope_table(m->cos_l, m->sin_l, c.max_seq, c.head_dim, c.rope_local, st));
+  W8A8_MTRY(launch_rope_table(m->cos_g, m->sin_g, c.max_seq, c.head_dim, c.rope_global, st));
+  for (int l = 0; l < c.layers; ++l)
+    W8A8_MTRY(w8a8_interleave_gate_up(layers[l].wgate, layers[l].wup, F, H, m->gu_bf16 + (size_t)l * 2 * F * H, st));
+  W8A8_MTRY(cudaStreamSynchronize(st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+#undef W8A8_MTRY
+  *out = m;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_model_destroy(w8a8_model* m) {
+  if (!m) return W8A8_OK;
+  cudaStreamSynchronize(m->st);
+  free_all(m);
+  delete m;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_model_reset_calibration(w8a8_model* m, void* stream) {
+  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "null model");
+  W8A8_CUDA(cudaMemsetAsync(m->stats, 0, ((size_t)m->cfg.layers * m->stats_stride() + m->cfg.hidden) * 4,
+                            as_stream(stream)));
+  return W8A8_OK;
+}
+
+extern "C" size_t w8a8_model_stats_count(const w8a8_model* m) {
+  return m ? (size_t)m->cfg.layers * m->stats_stride() + m->cfg.hidden : 0;
+}
+
+extern "C" w8a8_status w8a8_model_get_stats(const w8a8_model* m, float* host_out) {
+  W8A8_CHECK_ARG(m && host_out, W8A8_ERR_INVALID_ARG, "w8a8_model_get_stats: null argument");
+  W8A8_CUDA(cudaDeviceSynchronize());
+  W8A8_CUDA(cudaMemcpy(host_out, m->stats, w8a8_model_stats_count(m) * 4, cudaMemcpyDeviceToHost));
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_model_set_stats(w8a8_model* m, const float* host_in) {
+  W8A8_CHECK_ARG(m && host_in, W8A8_ERR_INVALID_ARG, "w8a8_model_set_stats: null argument");
+  W8A8_CUDA(cudaDeviceSynchronize());
+  W8A8_CUDA(cudaMemcpy(m->stats, host_in, w8a8_model_stats_count(m) * 4, cudaMemcpyHostToDevice));
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_model_calibrate(w8a8_model* m, const int32_t* tokens, int B, int T, void* stream) {
+  W8A8_TRY(check_call(m, B, T, 0));
+  W8A8_CHECK_ARG(tokens && aligned16(tokens), W8A8_ERR_INVALID_ARG, "w8a8_model_calibrate: null or unaligned tokens");
+  cudaStream_t st = as_stream(stream);
+  W8A8_TRY(launch_set_int(m->d_pos, 0, st));
+  return forward_core(m, tokens, B, T, nullptr, nullptr, true, st);
+}
+
+extern "C" w8a8_status w8a8_model_prepare(w8a8_model* m, float alpha, int smooth, void* stream) {
+  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "null model");
+  const w8a8_model_cfg& c = m->cfg;
+  const int H = c.hidden, F = c.inter;
+  auto ensure = [&](QW& q, int n, int k) -> w8a8_status {
+    if (q.wq) return W8A8_OK;
+    W8A8_TRY(dalloc(m, &q.wq, (size_t)n * k));
+    W8A8_TRY(dalloc(m, &q.s_w, (size_t)n));
+    W8A8_TRY(dalloc(m, &q.delta, (size_t)k));
+    W8A8_TRY(dalloc(m, &q.inv_delta, (size_t)k));
+    return W8A8_OK;
+  };
+  for (int l = 0; l < c.layers; ++l) {
+    W8A8_TRY(ensure(m->q_qkv[l], m->qkv_dim, H));
+    W8A8_TRY(ensure(m->q_o[l], H, m->q_dim));
+    W8A8_TRY(ensure(m->q_gu[l], 2 * F, H));
+    W8A8_TRY(ensure(m->q_down[l], H, F));
+  }
+  W8A8_TRY(ensure(m->q_lm, c.vocab, H));
+  for (int l = 0; l < c.layers; ++l) {
+    const w8a8_layer_bf16& W = m->L[l];
+    QW* q = &m->q_qkv[l];
+    W8A8_TRY(w8a8_prepare_weights(W.wqkv, m->qkv_dim, H, m->stat_qkv(l), alpha, smooth, q->wq, q->s_w, q->delta,
+                                  q->inv_delta, nullptr, stream));
+    q = &m->q_o[l];
+    W8A8_TRY(w8a8_prepare_weights(W.wo, H, m->q_dim, m->stat_o(l), alpha, smooth, q->wq, q->s_w, q->delta,
+                                  q->inv_delta, nullptr, stream));
+    q = &m->q_gu[l];
+    W8A8_TRY(w8a8_prepare_gate_up(W.wgate, W.wup, F, H, m->stat_gu(l), alpha, smooth, q->wq, q->s_w, q->delta,
+                                  q->inv_delta, nullptr, stream));
+    q = &m->q_down[l];
+    W8A8_TRY(w8a8_prepare_weights(W.wdown, H, F, m->stat_down(l), alpha, smooth, q->wq, q->s_w, q->delta,
+                                  q->inv_delta, nullptr, stream));
+  }
+  W8A8_TRY(w8a8_prepare_weights(m->embed, c.vocab, H, m->stat_lm(), alpha, smooth, m->q_lm.wq, m->q_lm.s_w,
+                                m->q_lm.delta, m->q_lm.inv_delta, nullptr, stream));
+  m->prepared = true;
+  ++m->prep_version;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_set_layer_precision(w8a8_model* m, int layer, int sublayer, int precision) {
+  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "null model");
+  W8A8_CHECK_ARG(precision == W8A8_PREC_BF16 || precision == W8A8_PREC_W8A8, W8A8_ERR_INVALID_ARG,
+                 "w8a8_set_layer_precision: precision %d", precision);
+  W8A8_CHECK_ARG(precision == W8A8_PREC_BF16 || m->prepared, W8A8_ERR_INVALID_ARG,
+                 "w8a8_set_layer_precision: W8A8 needs w8a8_model_prepare first");
+  if (sublayer == W8A8_SUB_LM) {
+    m->lm = precision;
+    return W8A8_OK;
+  }
+  W8A8_CHECK_ARG(sublayer == W8A8_SUB_FFN || sublayer == W8A8_SUB_ATTN, W8A8_ERR_INVALID_ARG,
+                 "w8a8_set_layer_precision: sublayer %d", sublayer);
+  W8A8_CHECK_ARG(layer >= 0 && layer < m->cfg.layers, W8A8_ERR_INVALID_ARG, "w8a8_set_layer_precision: layer %d", layer);
+  uint32_t& bits = sublayer == W8A8_SUB_FFN ? m->ffn_bits : m->attn_bits;
+  if (precision == W8A8_PREC_W8A8)
+    bits |= 1u << layer;
+  else
+    bits &= ~(1u << layer);
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_set_mask(w8a8_model* m, uint32_t ffn_bits, uint32_t attn_bits, int lm) {
+  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "null model");
+  const uint32_t all = m->cfg.layers >= 32 ? 0xFFFFFFFFu : ((1u << m->cfg.layers) - 1u);
+  W8A8_CHECK_ARG((ffn_bits & ~all) == 0 && (attn_bits & ~all) == 0, W8A8_ERR_INVALID_ARG,
+                 "w8a8_set_mask: bits beyond layer %d", m->cfg.layers - 1);
+  W8A8_CHECK_ARG(m->prepared || (ffn_bits == 0 && attn_bits == 0 && lm == 0), W8A8_ERR_INVALID_ARG,
+                 "w8a8_set_mask: W8A8 needs w8a8_model_prepare first");
+  m->ffn_bits = ffn_bits;
+  m->attn_bits = attn_bits;
+  m->lm = lm ? 1 : 0;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_get_mask(const w8a8_model* m, uint32_t* ffn_bits, uint32_t* attn_bits, int* lm) {
+  W8A8_CHECK_ARG(m && ffn_bits && attn_bits && lm, W8A8_ERR_INVALID_ARG, "w8a8_get_mask: null argument");
+  *ffn_bits = m->ffn_bits;
+  *attn_bits = m->attn_bits;
+  *lm = m->lm;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_decoder_forward(w8a8_model* m, const int32_t* tokens, int B, int T, int start_pos,
+                                            float* logits, int32_t* top1, void* stream) {
+  W8A8_TRY(check_call(m, B, T, start_pos));
+  W8A8_CHECK_ARG(tokens && top1, W8A8_ERR_INVALID_ARG, "w8a8_decoder_forward: null tokens or top1");
+  W8A8_CHECK_ARG(aligned16(tokens) && aligned16(top1) && (!logits || aligned16(logits)), W8A8_ERR_ALIGN,
+                 "w8a8_decoder_forward: pointers must be 16-byte aligned");
+  cudaStream_t st = as_stream(stream);
+  W8A8_TRY(launch_set_int(m->d_pos, start_pos, st));
+  return forward_core(m, tokens, B, T, logits, top1, false, st);
+}
+
+extern "C" w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* tokens, int B, int pos, float* logits,
+                                                int32_t* top1, void* stream) {
+  W8A8_TRY(check_call(m, B, 1, pos));
+  W8A8_CHECK_ARG(tokens && top1, W8A8_ERR_INVALID_ARG, "w8a8_decoder_decode_step: null tokens or top1");
+  cudaStream_t user = as_stream(stream), st = m->st;
+  W8A8_CUDA(cudaEventRecord(m->ev_in, user));
+  W8A8_CUDA(cudaStreamWaitEvent(st, m->ev_in, 0));
+  W8A8_CUDA(cudaMemcpyAsync(m->d_tokens, tokens, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice, st));
+  W8A8_TRY(launch_set_int(m->d_pos, pos, st));
+  const int want_logits = logits != nullptr;
+  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0), m->prep_version,
+                                   want_logits);
+  auto it = m->graphs.find(key);
+  if (it == m->graphs.end()) {
+    // one eager step first: every lazily set kernel attribute exists before capture; it computes
+    // exactly what the graph computes (same cache position, same outputs)
+    W8A8_TRY(forward_core(m, m->d_tokens, B, 1, want_logits ? m->d_logits : nullptr, m->d_top1, false, st));
+    cudaGraph_t g = nullptr;
+    W8A8_CUDA(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+    const w8a8_status s = forward_core(m, m->d_tokens, B, 1, want_logits ? m->d_logits : nullptr, m->d_top1, false, st);
+    const cudaError_t e = cudaStreamEndCapture(st, &g);
+    W8A8_TRY(s);
+    W8A8_CUDA(e);
+    cudaGraphExec_t exec = nullptr;
+    const cudaError_t ei = cudaGraphInstantiate(&exec, g, 0);
+    cudaGraphDestroy(g);
+    W8A8_CUDA(ei);
+    it = m->graphs.emplace(key, exec).first;
+  }
+  W8A8_CUDA(cudaGraphLaunch(it->second, st));
+  W8A8_CUDA(cudaMemcpyAsync(top1, m->d_top1, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice, st));
+  if (logits)
+    W8A8_CUDA(cudaMemcpyAsync(logits, m->d_logits, sizeof(float) * B * (size_t)m->cfg.vocab, cudaMemcpyDeviceToDevice,
+                              st));
+  W8A8_CUDA(cudaEventRecord(m->ev_out, st));
+  W8A8_CUDA(cudaStreamWaitEvent(user, m->ev_out, 0));
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_token_nll(const float* logits, const int32_t* targets, int M, int V, float* nll,
+                                      void* stream) {
+  W8A8_CHECK_ARG(M >= 0 && V > 0, W8A8_ERR_INVALID_ARG, "w8a8_token_nll: bad size");
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(logits && targets && nll, W8A8_ERR_INVALID_ARG, "w8a8_token_nll: null pointer");
+  W8A8_TRY(check_device());
+  nll_kernel<<<M, 256, 0, as_stream(stream)>>>(logits, targets, V, nll);
+  W8A8_LAUNCH_CHECK();
+  return W8A8_OK;
+}
+
+extern "C" int w8a8_choose_mask(const float* latency, const float* top1, const float* ppl_delta, const int32_t* n_int8,
+                                int n, float min_top1, float max_ppl_delta) {
+  int best = -1;
+  for (int i = 0; i < n; ++i) {
+    if (!(top1[i] >= min_top1 && ppl_delta[i] <= max_ppl_delta)) continue;
+    if (best < 0 || latency[i] < latency[best] || (latency[i] == latency[best] && n_int8[i] < n_int8[best])) best = i;
+  }
+  return best;
+}
+
+extern "C" w8a8_status w8a8_allocate_mask(w8a8_model* m, const w8a8_alloc_opts* o, w8a8_alloc_report* rep,
+                                          void* stream) {
+  W8A8_CHECK_ARG(m && o && rep && o->candidates && o->n_candidates > 0 && o->eval_tokens && rep->latency_ms &&
+                     rep->top1 && rep->ppl_delta,
+                 W8A8_ERR_INVALID_ARG, "w8a8_allocate_mask: null argument");
+  W8A8_CHECK_ARG(m->prepared, W8A8_ERR_INVALID_ARG, "w8a8_allocate_mask: w8a8_model_prepare first");
+  W8A8_TRY(check_call(m, o->eval_B, o->eval_T, 0));
+  W8A8_CHECK_ARG(o->decode_B > 0 && o->decode_B <= m->cfg.max_batch && o->prefill_T > 0, W8A8_ERR_SHAPE,
+                 "w8a8_allocate_mask: decode_B %d / prefill_T %d", o->decode_B, o->prefill_T);
+  W8A8_TRY(check_call(m, o->decode_B, 1, o->prefill_T + o->decode_steps - 1));
+  W8A8_CHECK_ARG(o->eval_T >= 2 && o->decode_steps > 0 && o->reps > 0, W8A8_ERR_INVALID_ARG,
+                 "w8a8_allocate_mask: eval_T >= 2, decode_steps > 0, reps > 0");
+  cudaStream_t st = as_stream(stream);
+  const int V = m->cfg.vocab, Me = o->eval_B * o->eval_T, Mp = o->decode_B * o->prefill_T;
+  // offline sweep: temporary buffers
+  float *logits = nullptr, *nll = nullptr;
+  int32_t *targets = nullptr, *top_ref = nullptr, *top_c = nullptr, *ptok = nullptr, *dtok = nullptr;
+  std::vector<void*> tmp;
+  auto talloc = [&](void** p, size_t bytes) -> w8a8_status {
+    W8A8_CUDA(cudaMalloc(p, std::max<size_t>(bytes, 16)));
+    tmp.push_back(*p);
+    return W8A8_OK;
+  };
+  auto cleanup = [&]() {
+    cudaStreamSynchronize(st);
+    for (void* p : tmp) cudaFree(p);
+  };
+  w8a8_status status = W8A8_OK;
+  do {
+    if ((status = talloc((void**)&logits, (size_t)Me * V * 4)) != W8A8_OK) break;
+    if ((status = talloc((void**)&nll, (size_t)Me * 4)) != W8A8_OK) break;
+    if ((status = talloc((void**)&targets, (size_t)Me * 4)) != W8A8_OK) break;
+    if ((status = talloc((void**)&top_ref, (size_t)Me * 4)) != W8A8_OK) break;
+    if ((status = talloc((void**)&top_c, (size_t)std::max(Me, m->cfg.max_tokens) * 4)) != W8A8_OK) break;
+    if ((status = talloc((void**)&ptok, (size_t)Mp * 4)) != W8A8_OK) break;
+    if ((status = talloc((void**)&dtok, (size_t)o->decode_B * 4)) != W8A8_OK) break;
+  } while (0);
+  if (status != W8A8_OK) {
+    cleanup();
+    return status;
+  }
+  shift_targets_kernel<<<(Me + 255) / 256, 256, 0, st>>>(o->eval_tokens, o->eval_B, o->eval_T, targets);
+  fill_tokens_kernel<<<(Mp + 255) / 256, 256, 0, st>>>(ptok, Mp, V);
+  std::vector<float> nll_h(Me);
+  std::vector<int32_t> top_h(Me), ref_h(Me);
+  auto mean_nll = [&](const std::vector<float>& v) {
+    double s = 0.0;
+    int n = 0;
+    for (int b = 0; b < o->eval_B; ++b)
+      for (int t = 0; t + 1 < o->eval_T; ++t, ++n) s += v[b * o->eval_T + t];
+    return s / n;
+  };
+  auto evaluate = [&](int32_t* top_out, double* mnll) -> w8a8_status {
+    W8A8_TRY(w8a8_decoder_forward(m, o->eval_tokens, o->eval_B, o->eval_T, 0, logits, top_out, stream));
+    W8A8_TRY(w8a8_token_nll(logits, targets, Me, V, nll, stream));
+    W8A8_CUDA(cudaMemcpyAsync(nll_h.data(), nll, (size_t)Me * 4, cudaMemcpyDeviceToHost, st));
+    W8A8_CUDA(cudaStreamSynchronize(st));
+    *mnll = mean_nll(nll_h);
+    return W8A8_OK;
+  };
+  const uint32_t saved_ffn = m->ffn_bits, saved_attn = m->attn_bits;
+  const int saved_lm = m->lm;
+  double ref_nll = 0.0;
+  m->ffn_bits = m->attn_bits = 0;
+  m->lm = 0;
+  status = evaluate(top_ref, &ref_nll);
+  if (status == W8A8_OK) status = cudaMemcpy(ref_h.data(), top_ref, (size_t)Me * 4, cudaMemcpyDeviceToHost) == cudaSuccess
+                                      ? W8A8_OK
+                                      : W8A8_ERR_CUDA;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  cudaEventCreate(&e0);
+  cudaEventCreate(&e1);
+  std::vector<int32_t> n8(o->n_candidates);
+  for (int i = 0; i < o->n_candidates && status == W8A8_OK; ++i) {
+    const w8a8_mask& c = o->candidates[i];
+    status = w8a8_set_mask(m, c.ffn_bits, c.attn_bits, c.lm);
+    if (status != W8A8_OK) break;
+    n8[i] = __builtin_popcount(c.ffn_bits) + __builtin_popcount(c.attn_bits) + (c.lm ? 1 : 0);
+    double cn = 0.0;
+    if ((status = evaluate(top_c, &cn)) != W8A8_OK) break;
+    if (cudaMemcpy(top_h.data(), top_c, (size_t)Me * 4, cudaMemcpyDeviceToHost) != cudaSuccess) {
+      status = W8A8_ERR_CUDA;
+      break;
+    }
+    int agree = 0, cnt = 0;
+    for (int b = 0; b < o->eval_B; ++b)
+      for (int t = 0; t + 1 < o->eval_T; ++t, ++cnt) agree += top_h[b * o->eval_T + t] == ref_h[b * o->eval_T + t];
+    rep->top1[i] = (float)agree / (float)cnt;
+    rep->ppl_delta[i] = (float)(std::exp(cn) / std::exp(ref_nll) - 1.0);
+    // latency: prefill, then decode steps from CUDA graphs fed by their own top-1 (greedy)
+    std::vector<float> runs;
+    for (int r = 0; r < o->reps && status == W8A8_OK; ++r) {
+      // prefill in chunks of at most max_tokens rows (the KV cache carries the earlier chunks)
+      const int chunk = std::max(1, m->cfg.max_tokens / o->decode_B);
+      for (int t0 = 0; t0 < o->prefill_T && status == W8A8_OK; t0 += chunk) {
+        const int tl = std::min(chunk, o->prefill_T - t0);
+        status = w8a8_decoder_forward(m, ptok + (size_t)o->decode_B * t0, o->decode_B, tl, t0, nullptr, top_c, stream);
+      }
+      if (status != W8A8_OK) break;
+      if (cudaMemcpyAsync(dtok, top_c, 4 * (size_t)o->decode_B, cudaMemcpyDeviceToDevice, st) != cudaSuccess) {
+        status = W8A8_ERR_CUDA;
+        break;
+      }
+      // warm the graph of this mask outside the timed region
+      if ((status = w8a8_decoder_decode_step(m, dtok, o->decode_B, o->prefill_T, nullptr, dtok, stream)) != W8A8_OK)
+        break;
+      cudaEventRecord(e0, st);
+      for (int s = 0; s < o->decode_steps && status == W8A8_OK; ++s)
+        status = w8a8_decoder_decode_step(m, dtok, o->decode_B, o->prefill_T + s, nullptr, dtok, stream);
+      cudaEventRecord(e1, st);
+      cudaEventSynchronize(e1);
+      float ms = 0.0f;
+      cudaEventElapsedTime(&ms, e0, e1);
+      runs.push_back(ms / (float)o->decode_steps);
+    }
+    if (status != W8A8_OK) break;
+    std::sort(runs.begin(), runs.end());
+    rep->latency_ms[i] = runs[runs.size() / 2];
+  }
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  cleanup();
+  if (status != W8A8_OK) {
+    m->ffn_bits = saved_ffn;
+    m->attn_bits = saved_attn;
+    m->lm = saved_lm;
+    return status;
+  }
+  rep->chosen = w8a8_choose_mask(rep->latency_ms, rep->top1, rep->ppl_delta, n8.data(), o->n_candidates, o->min_top1,
+                                 o->max_ppl_delta);
+  if (rep->chosen >= 0) {
+    const w8a8_mask& c = o->candidates[rep->chosen];
+    return w8a8_set_mask(m, c.ffn_bits, c.attn_bits, c.lm);
+  }
+  return w8a8_set_mask(m, 0, 0, 0);
+}

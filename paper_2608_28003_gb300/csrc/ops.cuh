@@ -1,0 +1,36 @@
+// Internal entry points shared by the C-ABI functions and the decoder (no argument checks).
+#pragma once
+
+#include "common.cuh"
+
+namespace w8a8 {
+
+struct DevInfo {
+  int ok = -1;  // -1 unknown, 0 unsupported, 1 sm_103
+  int sms = 0;
+};
+w8a8_status dev_info(DevInfo* out);
+int device_sms();
+
+struct LinearWs {
+  size_t xf16, sx, part, total;
+};
+struct FfnWs {
+  size_t h, gu, dn, total;
+};
+LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms);
+FfnWs ffn_ws(int M, int H, int F, int sms);
+
+w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* inv_delta, int8_t* xq,
+                                 uint16_t* xq_f16, float* s_x, cudaStream_t st);
+w8a8_status launch_act_absmax(const uint16_t* X, int T, int K, float* absmax, cudaStream_t st);
+
+// kind: 0 bf16 output, 1 GeGLU, 2 fp32 logits (+ top-1)
+w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind, uint16_t* Y,
+                            float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws, int sms, cudaStream_t st);
+w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias, int kind,
+                            uint16_t* Y, float* logits, int32_t* top1, void* ws, int sms, cudaStream_t st);
+w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y, uint16_t* h_dbg,
+                    void* workspace, int sms, cudaStream_t st);
+
+}  // namespace w8a8
