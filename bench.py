@@ -1,23 +1,31 @@
 #!/usr/bin/env python3
 """Benchmark of the W8A8 SmoothQuant hot path on GB300.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--quick]
 
-Prints ONE JSON line (rank 0).  The headline workload is the lm_head of a Gemma-3-1B-shaped
-model at decode (1152 -> 262144, W8A8, M = 1 token, fp32 logits + top-1), the paper's largest
-single operation.  A step is one lm_head call on a fresh token; L2 is flushed (a 512 MiB
-write) before every timed step, and each step is timed on the device with CUDA events.
-``value`` = ms per token (max over ranks; replicas only, every rank runs the same workload).
+Prints ONE JSON line (rank 0).  The headline workload is decode of a 26-layer Gemma-3-1B-shaped
+decoder (random-init bf16 weights, hidden 1152, 4 query / 1 KV heads of 256, FFN 6912, vocab
+262144) under the precision mask "FFN 5+5 + lm_head" (the FFN blocks of the five outermost
+layers at each end and lm_head in W8A8, everything else bf16), batch 1: a 128-token prefill,
+then one step = one decode token (a CUDA-graph replay of the whole decoder, fp32 logits' top-1
+included).  Tokens are seeded uniform ids, teacher-forced.  Every step streams about 1.46 GB of
+weights, far more than the 129 MB L2, so no flush is needed between steps.  ``value`` = ms per
+decoded token of the whole job (time, max over ranks, / tokens all ranks decoded; replicas only).
 
 The same line carries:
-  * ``kernels``: per-call time, TOPS and algorithmic GB/s of the single W8A8 linear
-    (M = 16, 1152 -> 6912), the FFN block (M in 1, 8, 64, 512, 2048) and lm_head
-    (M in 1, 16, 128, 512), W8A8 and bf16, with the fraction of the measured HBM peak;
-  * ``roofline`` of the headline kernel against the measured HBM copy bandwidth;
-  * ``e2e``: the same metric through the public API from pinned host buffers (input copy in,
-    top-1 copy out, host wall clock);
-  * ``cpu_baseline``: the oracle on this host's cores for a bounded sample.
-``--impl reference`` times the oracle (CPU) on the same workload and metric.
+  * ``masks``: per-mask decode ms/token, the latency change against the all-bf16 mask, Top-1
+    agreement and perplexity change, for the 16 candidate masks, and the mask the library's
+    allocator picks (Top-1 >= 98.9 %, perplexity change <= 1 %);
+  * ``batches``: decode ms/step at batch 1, 8 and 32 and prefill of 128 and 2048 tokens for four
+    masks;
+  * ``kernels``: per-call time, TOPS and algorithmic GB/s of the single W8A8 linear (M = 16,
+    1152 -> 6912), the FFN block (M in 1, 8, 64, 512, 2048) and lm_head (M in 1, 16, 128, 512),
+    W8A8 and bf16 (L2 flushed before each call);
+  * ``roofline`` of the decode step's largest kernel against the measured HBM copy bandwidth;
+  * ``e2e``: decode through the public API with the token copied in from pinned host memory
+    and the top-1 copied back every step (host wall clock);
+  * ``cpu_baseline``: the oracle on this host's cores for a bounded sample of the same decode.
+``--impl reference`` times the oracle (CPU) decoding the same model under the same mask.
 """
 from __future__ import annotations
 
@@ -36,18 +44,21 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "W8A8 linear TOPS & HBM GB/s vs GB300 roofline; decode ms/token per mask vs bf16"
-HIDDEN, INTER, VOCAB = 1152, 6912, 262144
+HIDDEN, INTER, VOCAB, LAYERS = 1152, 6912, 262144, 26
+PREFILL = 128
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
+WORKLOAD = ("decode, 26-layer Gemma-3-1B-shaped decoder (H 1152, 4q/1kv x 256, FFN 6912, V 262144), mask FFN 5+5 + "
+            "lm_head W8A8, batch 1, prefill 128 then one token per step (teacher-forced)")
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=128)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--no-sweep", action="store_true", help="skip the per-kernel sweep")
+    ap.add_argument("--quick", action="store_true", help="headline only: skip the mask sweep and the tables")
     return ap.parse_args()
 
 
@@ -63,6 +74,8 @@ def load_peaks():
 
 # ----------------------------------------------------------------------------- distributed
 class Dist:
+    """Replicas: every rank runs the same workload on its own GPU; only timings are reduced."""
+
     def __init__(self, backend):
         self.world = int(os.environ.get("WORLD_SIZE", "1"))
         self.rank = int(os.environ.get("RANK", "0"))
@@ -89,6 +102,11 @@ class Dist:
     def close(self):
         if self.pg:
             self.pg.destroy_process_group()
+
+
+def whole_job_ms_per_token(max_ms_total: float, tokens_per_rank: int, world: int) -> float:
+    """Time-like whole-job figure: the slowest rank's time over the tokens all ranks decoded."""
+    return max_ms_total / (tokens_per_rank * world)
 
 
 # ------------------------------------------------------------------------------ clocks
@@ -131,23 +149,34 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------------------- GPU timing
+def _events(n):
+    import torch
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+    s = torch.cuda.current_stream()
+    for e in ev:  # torch creates CUDA events lazily: record once so that their handles exist
+        e.record(s)
+    return ev
+
+
+def gpu_sleep_for(steps: int, ms_per_step: float):
+    """Queue a GPU-side sleep long enough for the host to enqueue every timed step before the
+    GPU reaches them, so that the events time device work only, not host launch gaps."""
+    import torch
+    torch.cuda._sleep(int(2e6 * (20 + steps * max(ms_per_step, 0.05) * 1.5)))  # ~2e6 cycles per ms
+
+
 def timed_steps(fn, steps: int, warmup: int, flush, stream, kernel_events=None):
-    """Run `warmup` untimed calls, then `steps` calls each preceded by an L2 flush; return the
-    per-step device times (ms) from CUDA events recorded on `stream`.  A GPU-side sleep is queued
-    first so that the host enqueues every step before the GPU reaches them: the events then time
-    device work only, not host launch gaps."""
+    """`warmup` untimed calls, then `steps` calls each preceded by an L2 flush; per-step device
+    times (ms) from CUDA events on `stream`."""
     import torch
     for _ in range(warmup):
         fn()
     torch.cuda.synchronize()
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-    for ka, kb in kev:  # torch creates CUDA events lazily: record once so that their handles exist
-        ka.record(stream)
-        kb.record(stream)
+    ev = [(a, b) for a, b in zip(_events(steps), _events(steps))]
+    kev = [(a, b) for a, b in zip(_events(steps), _events(steps))]
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
-        torch.cuda._sleep(int(4e7 + 2e6 * steps))  # ~20 ms + 1 ms per step at 2 GHz
+        gpu_sleep_for(steps, 1.0)
         for (a, b), (ka, kb) in zip(ev, kev):
             flush()
             a.record(stream)
@@ -177,6 +206,54 @@ def ffn_bytes(M, int8):
     return (2 * F * H + H * F) * 2 + M * H * 2 + 2 * M * F * 2 + M * H * 2
 
 
+def decode_weight_bytes(ffn_bits: int, attn_bits: int, lm: int) -> int:
+    """Weight bytes one decode token streams under a mask (INT8 = 1 byte, bf16 = 2 bytes)."""
+    qkv, o = (4 + 2) * 256 * HIDDEN, HIDDEN * 4 * 256
+    ffn = 3 * INTER * HIDDEN
+    total = 0
+    for l in range(LAYERS):
+        total += (qkv + o) * (1 if (attn_bits >> l) & 1 else 2)
+        total += ffn * (1 if (ffn_bits >> l) & 1 else 2)
+    return total + VOCAB * HIDDEN * (1 if lm else 2)
+
+
+# -------------------------------------------------------------------------- the decoder
+def make_decoder(B, dev, bf, norms, max_batch, max_seq, max_tokens):
+    import torch
+    w = {k: [t.to(dev) for t in v] if isinstance(v, list) else v.to(dev) for k, v in bf.items()}
+    n = {k: [torch.from_numpy(a).to(dev) for a in v] if isinstance(v, list) else torch.from_numpy(v).to(dev)
+         for k, v in norms.items()}
+    cfg = B.DecoderConfig(layers=LAYERS, max_batch=max_batch, max_seq=max_seq, max_tokens=max_tokens)
+    return B.Decoder(cfg, w, n), w
+
+
+def prefill(dec, toks, max_tokens):
+    """Prefill tokens [B, T] from position 0 in chunks of at most max_tokens rows."""
+    Bn, T = toks.shape
+    chunk = max(1, max_tokens // Bn)
+    for t0 in range(0, T, chunk):
+        dec.forward(toks[:, t0:t0 + chunk].contiguous(), t0, want_logits=False)
+
+
+def decode_ms(dec, Bn, steps, warmup, pos0):
+    """Greedy decode of Bn sequences after a prefill ending at pos0: per-step device time (ms)."""
+    import torch
+    dev = torch.device("cuda", torch.cuda.current_device())
+    tok = torch.zeros(max(4, Bn), dtype=torch.int32, device=dev)
+    for s in range(warmup):
+        dec.decode_step(tok[:Bn], pos0 + s, top1=tok[:Bn])
+    torch.cuda.synchronize()
+    e0, e1 = _events(2)
+    torch.cuda.synchronize()
+    gpu_sleep_for(steps, 1.0)
+    e0.record()
+    for s in range(steps):
+        dec.decode_step(tok[:Bn], pos0 + warmup + s, top1=tok[:Bn])
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
 def run_ours(args, dist: Dist):
     import torch
     import synth
@@ -188,78 +265,182 @@ def run_ours(args, dist: Dist):
     dev = torch.device("cuda", dist.local)
     stream = torch.cuda.current_stream()
     peaks = load_peaks()
+    K, W = args.steps, args.warmup
+    want_cpu = dist.rank == 0 and args.gpus == 1
+
+    # ---- weights (seeded), calibration (5 x 128 tokens of stream seed 1), preparation
+    t_setup = time.time()
+    f32, bf, norms = synth.decoder_weights(LAYERS, seed=0, want_f32=want_cpu)
+    max_seq = max(2304, PREFILL + 2 * (W + K) + 8)
+    dec, wdev = make_decoder(B, dev, bf, norms, max_batch=32, max_seq=max_seq, max_tokens=2048)
+    calib = torch.from_numpy(synth.tokens(5 * PREFILL, VOCAB, seed=1).reshape(5, PREFILL)).to(dev)
+    dec.calibrate(calib)
+    dec.prepare()
+    torch.cuda.synchronize()
+    setup_s = time.time() - t_setup
+
+    g = B.GROUP_BITS
+    head_mask = (g["5+5"], 0, 1)
+    dec.set_mask(*head_mask)
+    stream_toks = synth.tokens(PREFILL + 2 * (W + K) + 8, VOCAB, seed=2)
+    toks_dev = torch.from_numpy(stream_toks).to(dev)
+    prefill(dec, toks_dev[:PREFILL].view(1, PREFILL), 2048)
+    top = torch.zeros(W + K + 4, dtype=torch.int32, device=dev)
+
+    def step(s):  # token s of the stream after the prefill, at position PREFILL + s
+        dec.decode_step(toks_dev[PREFILL + s:PREFILL + s + 1], PREFILL + s, top1=top[s:s + 1])
+
+    # ---- headline: K decode tokens, device-timed
+    for s in range(W):
+        step(s)
+    torch.cuda.synchronize()
+    kernels_per_step = dec.decode_kernels(1)
+    ev = _events(K + 1)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(dist.local)
+    clocks.start()
+    dist.barrier()
+    torch.cuda.synchronize()
+    gpu_sleep_for(K, 1.0)
+    for s in range(K):
+        ev[s].record(stream)
+        step(W + s)
+    ev[K].record(stream)
+    torch.cuda.synchronize()
+    dist.barrier()
+    clk = clocks.stop()
+    total_ms = ev[0].elapsed_time(ev[K])
+    per_step = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
+    ms = whole_job_ms_per_token(dist.max(total_ms), K, dist.world)
+    wbytes = decode_weight_bytes(*head_mask)
+
+    # ---- e2e: token from pinned host memory in, top-1 back to pinned host memory, every step
+    host_tok = torch.from_numpy(stream_toks).pin_memory()
+    host_top = torch.zeros(1, dtype=torch.int32).pin_memory()
+    tok_in = torch.zeros(4, dtype=torch.int32, device=dev)
+    top_out = torch.zeros(4, dtype=torch.int32, device=dev)
+    p0 = PREFILL + W + K
+    e2e = []
+    for s in range(W + K):
+        i = p0 + s
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        tok_in[:1].copy_(host_tok[i:i + 1], non_blocking=True)
+        dec.decode_step(tok_in[:1], i, top1=top_out[:1])
+        host_top.copy_(top_out[:1], non_blocking=True)
+        stream.synchronize()
+        if s >= W:
+            e2e.append((time.perf_counter() - t0) * 1e3)
+    e2e_ms = whole_job_ms_per_token(dist.max(sum(e2e)), K, dist.world)
+
+    # ---- roofline: the decode step's largest kernel (lm_head W8A8 GEMV, M = 1), same launch
+    # configuration, timed alone with events around the kernel, L2 flushed before each launch
     flush_buf = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     flush = lambda: flush_buf.zero_()  # noqa: E731  (512 MiB > 129 MB L2)
-
-    # ---- lm_head weights (tied table) and its calibration statistic
-    hc = synth.lm_head_case(512, seed=0)
-    head_w = hc["w"].to(dev)
-    q = B.prepare_weights(head_w, B.act_absmax(hc["calib"].to(dev)))
-    head = B.HeadWeights(VOCAB, HIDDEN, q, head_w)
-    x_all = hc["x"].to(dev)
+    stats = torch.from_numpy(dec.get_stats()).to(dev)
+    lm_stat = stats[-HIDDEN:].contiguous()
+    q_lm = B.prepare_weights(wdev["embed"], lm_stat)
+    head = B.HeadWeights(VOCAB, HIDDEN, q_lm, wdev["embed"])
+    _, xh = synth.normed_rows(512, HIDDEN, seed=0)
+    xh = xh.to(dev)
     logits = torch.empty(512, VOCAB, dtype=torch.float32, device=dev)
     top1 = torch.empty(512 * 4, dtype=torch.int32, device=dev)  # slot i at 16 * i bytes (16-byte aligned)
     ws = B.Workspace(dev)
+    ctr = [0]
 
-    # ---- headline: lm_head W8A8, M = 1, a different token row per step
-    counter = [0]
+    def head_call():
+        i = ctr[0] % 512
+        ctr[0] += 1
+        B.lm_head(head, B.W8A8_PREC_W8A8, xh[i:i + 1], logits=logits[i:i + 1], top1=top1[4 * i:4 * i + 1], ws=ws)
 
-    def head_step():
-        i = counter[0] % 512
-        counter[0] += 1
-        B.lm_head(head, B.W8A8_PREC_W8A8, x_all[i:i + 1], logits=logits[i:i + 1], top1=top1[4 * i:4 * i + 1], ws=ws)
-
-    head_step()
-    torch.cuda.synchronize()
-    clocks = ClockSampler(dist.local)
-    dist.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    per_step = timed_steps(head_step, args.steps, args.warmup, flush, stream, kernel_events=B.set_kernel_events)
+    timed_steps(head_call, max(K, 20), 3, flush, stream, kernel_events=B.set_kernel_events)
     kernel_ms = statistics.mean(timed_steps.kernel_ms)
-    clk = clocks.stop()
-    torch.cuda.synchronize()
-    dist.barrier()
-    ms_local = statistics.mean(per_step)
-    ms = dist.max(ms_local)
-    launches_per_step = 2  # per-token quantiser + weight-streaming GEMV
-
     hb = w8a8_bytes(1, VOCAB, HIDDEN, out_bytes=4)
     achieved = hb / (kernel_ms * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None,
-                "peak_source": peaks["source"], "kernel": "gemv_dp4a_kernel<1,16> (W8A8 lm_head GEMV, M=1)",
-                "kernel_us": round(kernel_ms * 1e3, 2), "algorithmic_bytes_per_launch": hb}
+                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None, "peak_source": peaks["source"],
+                "kernel": "gemv_dp4a_kernel<1,16> (lm_head W8A8 GEMV, M=1, 1152 -> 262144)",
+                "kernel_us": round(kernel_ms * 1e3, 2), "algorithmic_bytes_per_launch": hb,
+                "timing": "CUDA events around the kernel on its stream, same launch as in the decode step, "
+                          "L2 flushed before each launch"}
 
-    # ---- e2e through the public API from pinned host memory
-    x_host = hc["x"][:64].pin_memory()
-    top_host = torch.empty(1, dtype=torch.int32).pin_memory()
-    x_dev = torch.empty(1, HIDDEN, dtype=torch.bfloat16, device=dev)
-    e2e_times = []
-    for s in range(args.warmup + args.steps):
-        flush()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        x_dev.copy_(x_host[s % 64:s % 64 + 1], non_blocking=True)
-        B.lm_head(head, B.W8A8_PREC_W8A8, x_dev, logits=logits[:1], top1=top1[:1], ws=ws)
-        top_host.copy_(top1[:1], non_blocking=True)
-        torch.cuda.current_stream().synchronize()
-        if s >= args.warmup:
-            e2e_times.append((time.perf_counter() - t0) * 1e3)
-    e2e_ms = dist.max(statistics.mean(e2e_times))
+    out = {"ms": ms, "total_ms": total_ms, "per_step": per_step, "clocks": clk, "roofline": roofline,
+           "launches": kernels_per_step * K, "kernels_per_step": kernels_per_step,
+           "e2e": {"value": round(e2e_ms, 5), "unit": "ms/token", "h2d_bytes_per_step": 4, "d2h_bytes_per_step": 4,
+                   "clock": "host wall clock per step: pinned H2D token copy, decode step, D2H top-1 copy, sync"},
+           "weight_gb_per_token": round(wbytes / 1e9, 4),
+           "weight_gbps": round(wbytes / (statistics.median(per_step) * 1e-3) / 1e9, 1),
+           "setup_s": round(setup_s, 1), "peaks": peaks, "f32": f32, "norms": norms}
 
-    kernels = {} if args.no_sweep else sweep(B, dev, head, hc, flush, stream, peaks)
-
-    return {
-        "ms": ms, "per_step": per_step, "clocks": clk, "roofline": roofline, "launches": launches_per_step * args.steps,
-        "e2e": {"value": round(e2e_ms, 4), "unit": "ms/token", "h2d_bytes_per_step": HIDDEN * 2,
-                "d2h_bytes_per_step": 4, "clock": "host wall clock incl. copies and stream sync"},
-        "kernels": kernels, "peaks": peaks,
-    }
+    if not args.quick:
+        out["masks"] = mask_sweep(B, dec, dev)
+        out["batches"] = batch_table(B, dec, dev)
+        out["kernels"] = sweep(B, dev, head, xh, flush, stream, peaks)
+    dec.close()
+    return out
 
 
-def sweep(B, dev, head, hc, flush, stream, peaks):
-    """Per-call device time of every workload shape, W8A8 and bf16 (3 warm-up, 10 timed)."""
+def mask_sweep(B, dec, dev):
+    """The library's allocator over the 16 candidate masks: Top-1 agreement and perplexity change
+    against the all-bf16 decoder on 4 x 128 eval tokens (stream seed 2), decode ms/token at
+    batch 1 after a 128-token prefill (median of 3 runs of 64 greedy steps)."""
+    import torch
+    import synth
+    names, cands = zip(*B.candidate_masks())
+    ev = torch.from_numpy(synth.tokens(4 * PREFILL, VOCAB, seed=2, stream=1).reshape(4, PREFILL)).to(dev)
+    t0 = time.time()
+    rep = dec.allocate(list(cands), ev, decode_B=1, prefill_T=PREFILL, decode_steps=64, reps=3)
+    base = rep["latency_ms"][0]  # candidate 0: all bf16
+    rows = []
+    for i, (n, (f, a, l)) in enumerate(zip(names, cands)):
+        t = rep["latency_ms"][i]
+        rows.append({"mask": n, "ms_per_token": round(t, 5), "latency_change_pct": round(100 * (t / base - 1), 2),
+                     "speedup_vs_bf16": round(base / t, 4), "top1": round(rep["top1"][i], 5),
+                     "ppl_delta": round(rep["ppl_delta"][i], 5), "weight_gb": round(decode_weight_bytes(f, a, l) / 1e9, 4)})
+    ch = rep["chosen"]
+    return {"rows": rows, "chosen": names[ch] if ch >= 0 else None, "rule": "Top-1 >= 0.989, ppl change <= 0.01",
+            "seconds": round(time.time() - t0, 1)}
+
+
+def batch_table(B, dec, dev):
+    """Decode ms/step at batch 1, 8, 32 (prefill 128, 16 greedy steps after 3 warm-ups) and prefill
+    time of 128 and 2048 tokens (batch 1), for four masks."""
+    import torch
+    import synth
+    g = B.GROUP_BITS
+    masks = {"bf16": (0, 0, 0), "ffn 5+5 + lm": (g["5+5"], 0, 1), "ffn all26 + lm": (g["all26"], 0, 1),
+             "ffn all26 + att all26 + lm": (g["all26"], g["all26"], 1)}
+    out = {}
+    pre = torch.from_numpy(synth.tokens(32 * 2048, VOCAB, seed=3).reshape(32, 2048)).to(dev)
+    for name, m in masks.items():
+        dec.set_mask(*m)
+        r = {}
+        for Bn in (1, 8, 32):
+            prefill(dec, pre[:Bn, :PREFILL], 2048)
+            t = decode_ms(dec, Bn, 16, 3, PREFILL)
+            r[f"decode_B{Bn}_ms_per_step"] = round(t, 4)
+            r[f"decode_B{Bn}_tok_s"] = round(Bn * 1e3 / t, 1)
+        for T in (PREFILL, 2048):
+            x = pre[:1, :T].contiguous()
+            dec.forward(x, 0, want_logits=False)
+            e0, e1 = _events(2)
+            torch.cuda.synchronize()
+            e0.record()
+            for _ in range(3):
+                dec.forward(x, 0, want_logits=False)
+            e1.record()
+            torch.cuda.synchronize()
+            t = e0.elapsed_time(e1) / 3
+            r[f"prefill_T{T}_ms"] = round(t, 3)
+            r[f"prefill_T{T}_tok_s"] = round(T * 1e3 / t, 1)
+        out[name] = r
+    dec.set_mask(g["5+5"], 0, 1)
+    return out
+
+
+def sweep(B, dev, head, xh, flush, stream, peaks):
+    """Per-call device time of the single linear, FFN block and lm_head shapes, W8A8 and bf16
+    (3 warm-up, 10 timed, L2 flushed before each call)."""
     import torch
     import synth
     out = {}
@@ -278,7 +459,6 @@ def sweep(B, dev, head, hc, flush, stream, peaks):
     kev = B.set_kernel_events
 
     ws = B.Workspace(dev)
-    # single linear (M = 16, 1152 -> 6912)
     c = synth.linear_case()
     q = B.prepare_weights(c["w"].to(dev), B.act_absmax(c["calib"].to(dev)))
     x = c["x"].to(dev)
@@ -288,7 +468,6 @@ def sweep(B, dev, head, hc, flush, stream, peaks):
     rec("linear_w8a8_M16", t, 2 * 16 * INTER * HIDDEN, w8a8_bytes(16, INTER, HIDDEN), True)
     t = statistics.mean(timed_steps(lambda: B.linear_bf16(w, x, out=y, ws=ws), 10, 3, flush, stream, kev))
     rec("linear_bf16_M16", t, 2 * 16 * INTER * HIDDEN, bf16_bytes(16, INTER, HIDDEN), True)
-    # FFN block
     fc = synth.ffn_case(2048, seed=0)
     gu = B.prepare_gate_up(fc["wg"].to(dev), fc["wu"].to(dev), B.act_absmax(fc["calib"].to(dev)))
     dn = B.prepare_weights(fc["wd"].to(dev), torch.from_numpy(fc["stat_h"]).to(dev))
@@ -298,10 +477,9 @@ def sweep(B, dev, head, hc, flush, stream, peaks):
     for M in (1, 8, 64, 512, 2048):
         flops = 2 * M * 3 * INTER * HIDDEN
         for prec, tag in ((B.W8A8_PREC_W8A8, "w8a8"), (B.W8A8_PREC_BF16, "bf16")):
-            t = statistics.mean(timed_steps(lambda: B.ffn_block(f, prec, xf[:M], out=yf[:M], ws=ws), 10, 3, flush, stream))
+            t = statistics.mean(timed_steps(lambda: B.ffn_block(f, prec, xf[:M], out=yf[:M], ws=ws), 10, 3, flush,
+                                            stream))
             rec(f"ffn_{tag}_M{M}", t, flops, ffn_bytes(M, prec == B.W8A8_PREC_W8A8))
-    # lm_head
-    xh = hc["x"].to(dev)
     lg = torch.empty(512, VOCAB, dtype=torch.float32, device=dev)
     tp = torch.empty(512, dtype=torch.int32, device=dev)
     for M in (1, 16, 128, 512):
@@ -327,20 +505,48 @@ def oracle_threads():
     return os.cpu_count()
 
 
-def oracle_lm_head_sample(n_tokens: int):
-    """Time the oracle's W8A8 lm_head (quantise, exact INT8 GEMM, dequantise, top-1) for
-    `n_tokens` single-token calls.  Returns (ms per token, description)."""
+def oracle_decode_sample(f32, norms, n_tokens: int, warmup: int = 1, prefill_T: int = 16):
+    """The oracle decoder (26 layers, full Gemma-3-1B shapes, the bench's weights) under the
+    FFN 5+5 + lm_head mask: statistics from 16 calibration tokens (stream seed 1), a prefill of
+    `prefill_T` tokens, then `warmup` untimed and `n_tokens` timed single-token decode steps.
+    Returns per-token times (ms)."""
     import synth
-    from oracle import blocks as OB
-    from oracle import w8a8 as OW
-    hc = synth.lm_head_case(n_tokens, seed=0)
-    prep = OW.prepare_weights(hc["w32"], OW.act_absmax(hc["calib32"]))
+    from oracle import decoder as OD
+    from oracle import masks as OM
+    if f32 is None:
+        f32, _, norms = synth.decoder_weights(LAYERS, seed=0)
+    ow = dict(f32)
+    ow.update(norms)
+    cfg = OD.DecoderConfig(layers=LAYERS)
+    od = OD.OracleDecoder(cfg, ow, batch=1, max_len=prefill_T + warmup + n_tokens + 1)
+    od.calibrate([synth.tokens(16, VOCAB, seed=1).reshape(1, 16)])
+    od.prepare()
+    mask = OM.make_mask("5+5", "none", True)
+    toks = synth.tokens(prefill_T + warmup + n_tokens, VOCAB, seed=2)
+    od.forward(toks[None, :prefill_T], 0, mask=mask, want_logits=False)
     times = []
-    for i in range(n_tokens):
+    for s in range(warmup + n_tokens):
+        p = prefill_T + s
         t0 = time.perf_counter()
-        OB.lm_head_w8a8(hc["x32"][i:i + 1], prep)
-        times.append((time.perf_counter() - t0) * 1e3)
-    return statistics.mean(times), times
+        od.forward(toks[None, p:p + 1], p, mask=mask)
+        if s >= warmup:
+            times.append((time.perf_counter() - t0) * 1e3)
+    return times
+
+
+def reference_line(args, times, n):
+    ms = statistics.mean(times)
+    cores = oracle_threads()
+    sample = (f"oracle decoder, 26 layers at full shapes, mask FFN 5+5 + lm_head: prefill 16 tokens, "
+              f"{min(args.warmup, 1)} untimed + {n} timed decode tokens")
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(ms, 3), "unit": "ms/token", "n_gpus": args.gpus,
+        "steps": n, "warmup": min(args.warmup, 1), "ms_per_step": round(ms, 3), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8/fp32 (f64 exact sums)", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "global_batch": 1, "seq_len": 1, "parallelism": "replicas"},
+        "cpu_baseline": {"value": round(ms, 3), "unit": "ms/token", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(ms, 3), "unit": "ms/token", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
 
 
 def main():
@@ -350,22 +556,9 @@ def main():
         if dist.rank != 0:
             dist.close()
             return
-        n = max(1, min(args.steps, 8))
-        for _ in range(min(args.warmup, 1)):
-            oracle_lm_head_sample(1)
-        ms, times = oracle_lm_head_sample(n)
-        cores = oracle_threads()
-        line = {
-            "impl": "reference", "metric": METRIC, "value": round(ms, 3), "unit": "ms/token", "n_gpus": args.gpus,
-            "steps": n, "warmup": args.warmup, "ms_per_step": round(ms, 3), "higher_is_better": False,
-            "scaling": "weak", "vs_baseline": None, "dtype": "int8/fp32 (f64 exact sums)", "data": "synthetic",
-            "config": {"workload": "lm_head 1152->262144 W8A8 decode, M=1 (fp32 logits + top-1)", "global_batch": 1,
-                       "seq_len": 1, "parallelism": "replicas"},
-            "cpu_baseline": {"value": round(ms, 3), "unit": "ms/token", "cores": cores, "kind": "oracle",
-                             "sample": f"{n} single-token lm_head calls of the numpy oracle"},
-            "e2e": {"value": round(ms, 3), "unit": "ms/token", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-        }
-        print(json.dumps(line))
+        n = max(1, min(args.steps, 16))
+        times = oracle_decode_sample(None, None, n, warmup=min(args.warmup, 1))
+        print(json.dumps(reference_line(args, times, n)))
         dist.close()
         return
 
@@ -373,21 +566,29 @@ def main():
     res = run_ours(args, dist)
     cpu = None
     if dist.rank == 0 and args.gpus == 1:
-        ms_cpu, _ = oracle_lm_head_sample(4)
-        cpu = {"value": round(ms_cpu, 3), "unit": "ms/token", "cores": oracle_threads(), "kind": "oracle",
-               "sample": "4 single-token W8A8 lm_head calls (1152 -> 262144) of the numpy oracle"}
+        times = oracle_decode_sample(res["f32"], res["norms"], 4)
+        cpu = {"value": round(statistics.mean(times), 3), "unit": "ms/token", "cores": oracle_threads(),
+               "kind": "oracle",
+               "sample": "oracle decoder, 26 layers at full shapes, same weights and mask: prefill 16 tokens, "
+                         "1 untimed + 4 timed decode tokens"}
     if dist.rank == 0:
         ms = res["ms"]
         line = {
             "metric": METRIC, "value": round(ms, 5), "unit": "ms/token", "n_gpus": args.gpus, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": round(ms, 5), "higher_is_better": False, "scaling": "weak",
-            "vs_baseline": None, "dtype": "int8 (fp16-coded operands, fp32->int32 exact accumulation)",
+            "warmup": args.warmup, "ms_per_step": round(res["total_ms"] / args.steps, 5), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": "int8 W8A8 (exact int32 sums) on the masked sublayers, bf16 (fp32 sums) elsewhere",
             "data": "synthetic",
-            "config": {"workload": "lm_head 1152->262144 W8A8 decode, M=1 (fp32 logits + top-1)", "global_batch": 1,
-                       "seq_len": 1, "parallelism": f"replicas x{args.gpus}", "l2": "flushed (512 MiB write) before every step"},
-            "aggregate_tok_s": round(args.gpus * 1e3 / ms, 1),
+            "config": {"workload": WORKLOAD, "global_batch": args.gpus, "seq_len": 1, "prefill": PREFILL,
+                       "parallelism": f"replicas x{args.gpus}",
+                       "l2": "not flushed: each step streams the mask's weights (1.46 GB) through the 129 MB L2",
+                       "weights": "random-init bf16 N(0, 0.02), seed 0; calibration 5 x 128 tokens (seed 1)"},
+            "median_step_ms": round(statistics.median(res["per_step"]), 5),
+            "weight_gb_per_token": res["weight_gb_per_token"], "weight_gbps_median_step": res["weight_gbps"],
             "clocks": res["clocks"], "roofline": res["roofline"], "e2e": res["e2e"], "gpu_launches": res["launches"],
-            "cpu_baseline": cpu, "kernels": res["kernels"],
+            "kernels_per_step": res["kernels_per_step"], "cpu_baseline": cpu,
+            "masks": res.get("masks"), "batches": res.get("batches"), "kernels": res.get("kernels"),
+            "setup_s": res["setup_s"],
         }
         print(json.dumps(line))
     dist.close()

@@ -306,6 +306,12 @@ w8a8_status w8a8_decoder_forward(w8a8_model* m, const int32_t* tokens, int B, in
 w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* tokens, int B, int pos, float* logits,
                                      int32_t* top1, void* stream);
 
+/* Measurement aid with no counterpart in the paper: *kernels = the number of kernel launches
+ * one w8a8_decoder_decode_step of B sequences makes under the current mask (the kernel nodes of
+ * its CUDA graph plus the position update launched beside it; copies are not counted).  The
+ * graph must exist: W8A8_ERR_INVALID_ARG before the first decode step of this (B, mask). */
+w8a8_status w8a8_model_decode_kernels(const w8a8_model* m, int B, int want_logits, int* kernels);
+
 /* Negative log-likelihood of targets under softmax(logits) per row (LM Head section's
  * perplexity): nll[i] = logsumexp(logits[i, :]) - logits[i, targets[i]], fp32. */
 w8a8_status w8a8_token_nll(const float* logits, const int32_t* targets, int M, int V, float* nll, void* stream);

@@ -123,6 +123,7 @@ SIGNATURES = {
                              ctypes.POINTER(_i32)]),
     "w8a8_decoder_forward": (_i32, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_decoder_decode_step": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp, _vp]),
+    "w8a8_model_decode_kernels": (_i32, [_vp, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
     "w8a8_allocate_mask": (_i32, [_vp, ctypes.POINTER(AllocOptsC), ctypes.POINTER(AllocReportC), _vp]),
@@ -400,6 +401,32 @@ def lm_head(hd: HeadWeights, precision: int, X: torch.Tensor, want_logits: bool 
 W8A8_SUB_FFN, W8A8_SUB_ATTN, W8A8_SUB_LM = 0, 1, 2
 
 
+def _layer_bits(layers) -> int:
+    return sum(1 << l for l in layers)
+
+
+# Layer groups of the paper's precision masks (bit l = layer l of the 26): outer 5 + 5 layers,
+# outer 10 + 10 layers, all 26 layers.
+GROUP_BITS = {
+    "none": 0,
+    "5+5": _layer_bits(list(range(0, 5)) + list(range(21, 26))),
+    "10+10": _layer_bits(list(range(0, 10)) + list(range(16, 26))),
+    "all26": _layer_bits(range(26)),
+}
+
+
+def candidate_masks():
+    """The 16 candidate masks of the allocation sweep: FFN group x attention group (none / all26)
+    x lm_head (bf16 / W8A8), as (name, (ffn_bits, attn_bits, lm))."""
+    out = []
+    for ffn in ("none", "5+5", "10+10", "all26"):
+        for att in ("none", "all26"):
+            for lm in (0, 1):
+                name = f"ffn={ffn} att={att} lm={'int8' if lm else 'bf16'}"
+                out.append((name, (GROUP_BITS[ffn], GROUP_BITS[att], lm)))
+    return out
+
+
 def choose_mask(latency, top1, ppl_delta, n_int8, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> int:
     """The library's allocation rule on host arrays (index, or -1 if nothing is feasible)."""
     n = len(latency)
@@ -520,6 +547,13 @@ class Decoder:
         _check("w8a8_decoder_decode_step", lib().w8a8_decoder_decode_step(self.h, _p(_bits(tokens)), B, int(pos),
                                                                           _p(logits), _p(top1), _stream(stream)))
         return logits, top1
+
+    def decode_kernels(self, B: int, want_logits: bool = False) -> int:
+        """Kernel launches of one decode step of B sequences under the current mask."""
+        n = ctypes.c_int32()
+        _check("w8a8_model_decode_kernels", lib().w8a8_model_decode_kernels(self.h, int(B), int(want_logits),
+                                                                            ctypes.byref(n)))
+        return n.value
 
     def allocate(self, candidates, eval_tokens: torch.Tensor, decode_B: int, prefill_T: int, decode_steps: int,
                  reps: int = 3, min_top1: float = 0.989, max_ppl_delta: float = 0.01, stream=None) -> dict:

@@ -5,6 +5,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "gemv_small.cuh"
 #include "ops.cuh"
 #include "stream_gemm.cuh"
 
@@ -99,11 +100,49 @@ static w8a8_status quantize_for(const StreamPlan& p, const uint16_t* X, int M, i
   return launch_quantize_rows(X, M, K, inv_delta, xq_dbg, reinterpret_cast<uint16_t*>(codes), s_x, st);
 }
 
+static unsigned int* err_word(void* ws) {
+  return reinterpret_cast<unsigned int*>(reinterpret_cast<char*>(ws) + kErrWordOffset);
+}
+
+// Decode-sized calls whose CTAs can own whole weight rows go to the row-owning GEMV (K1 fused
+// into it on the W8A8 path); returns false when the shape is left to the streaming kernel.
+static bool small_gemv(bool int8, const void* W, const float* inv_delta, const float* s_w, const uint16_t* X, int M,
+                       int N, int K, const float* bias, int kind, uint16_t* Y, const w8a8_debug* dbg, void* ws,
+                       const void* prefetch, size_t prefetch_bytes, int sms, cudaStream_t st, w8a8_status* status) {
+  if (kind != EPI_BF16 && kind != EPI_GEGLU) return false;
+  SmallArgs a{};
+  a.p = make_small_plan(int8, M, N, K, kind, sms);
+  if (!a.p.ok) return false;
+  a.W = W;
+  a.X = X;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.kind = kind;
+  a.inv_delta = inv_delta;
+  a.s_w = s_w;
+  a.bias = bias;
+  a.y = Y;
+  a.xq_dbg = dbg ? dbg->xq : nullptr;
+  a.s_x_dbg = dbg ? dbg->s_x : nullptr;
+  a.acc_dbg = dbg ? dbg->acc : nullptr;
+  a.prefetch = prefetch;
+  a.prefetch_bytes = prefetch ? prefetch_bytes / 16 * 16 : 0;
+  a.err = err_word(ws);
+  *status = launch_small_gemv(int8, a, st);
+  return true;
+}
+
 // One W8A8 linear: K1 then the streaming GEMM.  s_x and the codes live in the workspace.
 w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
                                    uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
-                                   int sms, cudaStream_t st) {
+                                   int sms, cudaStream_t st, const L2Prefetch* pf) {
   const int N = w->n, K = w->k;
+  w8a8_status small_status = W8A8_OK;
+  if (!logits && !top1 &&
+      small_gemv(true, w->wq, w->inv_delta, w->s_w, X, M, N, K, bias, kind, Y, dbg, ws, pf ? pf->ptr : nullptr,
+                 pf ? pf->bytes : 0, sms, st, &small_status))
+    return small_status;
   LinearWs L = linear_ws(M, N, K, true, sms);
   char* base = reinterpret_cast<char*>(ws);
   void* codes = base + L.xf16;
@@ -132,7 +171,12 @@ w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, con
 
 w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias,
                                    int kind, uint16_t* Y, float* logits, int32_t* top1, void* ws, int sms,
-                                   cudaStream_t st) {
+                                   cudaStream_t st, const L2Prefetch* pf) {
+  w8a8_status small_status = W8A8_OK;
+  if (!logits && !top1 &&
+      small_gemv(false, W, nullptr, nullptr, X, M, N, K, bias, kind, Y, nullptr, ws, pf ? pf->ptr : nullptr,
+                 pf ? pf->bytes : 0, sms, st, &small_status))
+    return small_status;
   LinearWs L = linear_ws(M, N, K, false, sms);
   StreamArgs a{};
   a.W = W;
@@ -269,7 +313,12 @@ FfnWs ffn_ws(int M, int H, int F, int sms) {
 }
 
 w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y, uint16_t* h_dbg,
-                    void* workspace, int sms, cudaStream_t st) {
+                    void* workspace, int sms, cudaStream_t st, const L2Prefetch* pf_gate_up,
+                    const L2Prefetch* pf_down) {
+  const void* pgu = pf_gate_up ? pf_gate_up->ptr : nullptr;
+  const size_t bgu = pf_gate_up ? pf_gate_up->bytes : 0;
+  const void* pdn = pf_down ? pf_down->ptr : nullptr;
+  const size_t bdn = pf_down ? pf_down->bytes : 0;
   const int H = f->hidden, F = f->inter;
   const FfnWs L = ffn_ws(M, H, F, sms);
   char* base = reinterpret_cast<char*>(workspace);
@@ -278,7 +327,11 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
   // counters (each leaves them zero); their scratch regions are disjoint.
   if (precision == W8A8_PREC_W8A8) {
     // gate/up: scratch at L.gu
-    {
+    w8a8_status ss = W8A8_OK;
+    if (small_gemv(true, f->gate_up.wq, f->gate_up.inv_delta, f->gate_up.s_w, X, M, 2 * F, H, nullptr, EPI_GEGLU, h,
+                   nullptr, workspace, pgu, bgu, sms, st, &ss)) {
+      W8A8_TRY(ss);
+    } else {
       const LinearWs A = linear_ws(M, 2 * F, H, true, sms);
       void* codes = base + L.gu + (A.xf16 - W8A8_WS_RESERVED);
       float* s_x = reinterpret_cast<float*>(base + L.gu + (A.sx - W8A8_WS_RESERVED));
@@ -298,7 +351,10 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
       attach_reserved(a, workspace);
       W8A8_TRY(launch_stream_gemm(true, a, st));
     }
-    {
+    if (small_gemv(true, f->down.wq, f->down.inv_delta, f->down.s_w, h, M, H, F, nullptr, EPI_BF16, Y, nullptr,
+                   workspace, pdn, bdn, sms, st, &ss)) {
+      W8A8_TRY(ss);
+    } else {
       const LinearWs B = linear_ws(M, H, F, true, sms);
       void* codes = base + L.dn + (B.xf16 - W8A8_WS_RESERVED);
       float* s_x = reinterpret_cast<float*>(base + L.dn + (B.sx - W8A8_WS_RESERVED));
@@ -319,7 +375,11 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
       W8A8_TRY(launch_stream_gemm(true, a, st));
     }
   } else {
-    {
+    w8a8_status ss = W8A8_OK;
+    if (small_gemv(false, f->gate_up_bf16, nullptr, nullptr, X, M, 2 * F, H, nullptr, EPI_GEGLU, h, nullptr,
+                   workspace, pgu, bgu, sms, st, &ss)) {
+      W8A8_TRY(ss);
+    } else {
       const LinearWs A = linear_ws(M, 2 * F, H, false, sms);
       StreamArgs a{};
       a.W = f->gate_up_bf16;
@@ -334,7 +394,10 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
       attach_reserved(a, workspace);
       W8A8_TRY(launch_stream_gemm(false, a, st));
     }
-    {
+    if (small_gemv(false, f->down_bf16, nullptr, nullptr, h, M, H, F, nullptr, EPI_BF16, Y, nullptr, workspace,
+                   pdn, bdn, sms, st, &ss)) {
+      W8A8_TRY(ss);
+    } else {
       const LinearWs B = linear_ws(M, H, F, false, sms);
       StreamArgs a{};
       a.W = f->down_bf16;

@@ -1,0 +1,381 @@
+// Decode attention fused with QK-norm, RoPE and the KV-cache write (one new token per sequence).
+//
+// At decode the attention of a layer reads a few hundred cached key/value rows and one new row;
+// split over separate kernels (QK-norm + RoPE, then attention with a cross-CTA combine through
+// global memory) it costs several dependent round trips.  Here one launch does it all:
+//  * grid (kSplits, B, n_kv) in clusters of kSplits CTAs along x: CTA r of a cluster takes an
+//    equal share of the key positions of (sequence b, key/value head kvh); shares are at least
+//    kMinKeys long, so short contexts leave the trailing CTAs idle;
+//  * before waiting for the preceding kernel (the q/k/v projection), each CTA starts copying its
+//    cached key/value rows (positions before the new one, written by earlier steps) into shared
+//    memory with cp.async, in tiles of 64 positions (one buffer: a share longer than a tile loads
+//    the next tile after using the current one);
+//  * then every working CTA applies RMSNorm (q_norm / k_norm) and RoPE to the new row with the
+//    arithmetic of the prefill path (one warp per head, lane l holding the RoPE pairs
+//    (4l + e, 128 + 4l + e)); the CTA whose share ends at the new position also writes its key
+//    (bf16) and value to the cache and uses them from shared memory;
+//  * warp w handles query head w mod G and key group w / G of each tile: lane j computes the dot
+//    product of the scaled query (broadcast from shared memory) with key j (rows padded to 528
+//    bytes: the lanes of a shared-memory phase hit different bank groups), then the warp updates
+//    its running max, sum and output (lane l: dims 8l .. 8l+7) over its keys;
+//  * the warps of a head combine their partial (m, l, o) inside the CTA; each CTA then stores its
+//    per-head partials into CTA 0's shared memory (distributed shared memory stores, released by
+//    one cluster barrier), and CTA 0 combines them and writes the output row.
+#include <cmath>
+
+#include "decoder_kernels.cuh"
+
+namespace w8a8 {
+
+namespace {
+
+constexpr int kHd = 256;
+constexpr int kSplits = 8;        // CTAs per cluster (portable cluster size)
+constexpr int kMinKeys = 64;      // positions per working CTA, at least
+constexpr int kTile = 64;         // positions per shared-memory tile
+constexpr int kKRow = 528;        // bytes per key row in shared memory (256 bf16 + 16 bytes of padding)
+constexpr int kVRow = 512;
+constexpr int kBuf = kTile * (kKRow + kVRow);
+constexpr int kWarps = 8;
+constexpr int kPartFloats = kHd + 4;  // o[256], m, l, pad
+// dynamic shared memory (about 111 KB, so that a CTA fits beside the q/k/v projection's CTAs and
+// starts its copies early): queries [G][256] fp32 | new key row | new value row | one tile buffer |
+// partials of the 8 warps | inbox of CTA 0 (the CTAs' per-head partials)
+constexpr int kMaxG = 4;  // query heads per key/value head (the inbox is sized for this many)
+constexpr int kOffQ = 0;
+constexpr int kOffKNew = kOffQ + kMaxG * kHd * 4;
+constexpr int kOffVNew = kOffKNew + kKRow;
+constexpr int kOffBuf = kOffVNew + kVRow;
+constexpr int kOffPart = kOffBuf + kBuf;
+constexpr int kOffInbox = kOffPart + kWarps * kPartFloats * 4;           // CTA 0: one partial per (CTA, head)
+constexpr int kSmem = kOffInbox + kSplits * kMaxG * kPartFloats * 4;
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;\n" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void st_cluster_f32x4(uint32_t addr, float a, float b, float c, float d) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
+               : "memory");
+}
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ void unpack8_bf16(const uint4& w, float (&x)[8]) {
+  x[0] = bf16_lo(w.x); x[1] = bf16_hi(w.x); x[2] = bf16_lo(w.y); x[3] = bf16_hi(w.y);
+  x[4] = bf16_lo(w.z); x[5] = bf16_hi(w.z); x[6] = bf16_lo(w.w); x[7] = bf16_hi(w.w);
+}
+
+// The constants one warp needs for RMSNorm + RoPE of a head (lane l: pairs (4l + e, 128 + 4l + e)).
+struct RopeConsts {
+  float w1[4], w2[4], c[4], s[4];
+};
+__device__ __forceinline__ void load_rope_consts(RopeConsts& k, const float* nw, const float* cos_row,
+                                                 const float* sin_row, int lane) {
+  const float4 c = *reinterpret_cast<const float4*>(cos_row + 4 * lane);
+  const float4 sn = *reinterpret_cast<const float4*>(sin_row + 4 * lane);
+  k.c[0] = c.x; k.c[1] = c.y; k.c[2] = c.z; k.c[3] = c.w;
+  k.s[0] = sn.x; k.s[1] = sn.y; k.s[2] = sn.z; k.s[3] = sn.w;
+  if (nw) {
+    const float4 a = *reinterpret_cast<const float4*>(nw + 4 * lane);
+    const float4 b = *reinterpret_cast<const float4*>(nw + kHd / 2 + 4 * lane);
+    k.w1[0] = a.x; k.w1[1] = a.y; k.w1[2] = a.z; k.w1[3] = a.w;
+    k.w2[0] = b.x; k.w2[1] = b.y; k.w2[2] = b.z; k.w2[3] = b.w;
+  }
+}
+
+// RMSNorm (when has_norm) and RoPE of one head held as lane l's pairs (4l + e, 128 + 4l + e).
+__device__ __forceinline__ void norm_rope(float (&x1)[4], float (&x2)[4], bool has_norm, const RopeConsts& k,
+                                          float eps) {
+  if (has_norm) {
+    float ss = 0.0f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) ss += x1[e] * x1[e] + x2[e] * x2[e];
+    const float inv = 1.0f / sqrtf(warp_sum_f(ss) / (float)kHd + eps);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x1[e] = x1[e] * inv * k.w1[e];
+      x2[e] = x2[e] * inv * k.w2[e];
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float y1 = x1[e] * k.c[e] - x2[e] * k.s[e];
+    const float y2 = x2[e] * k.c[e] + x1[e] * k.s[e];
+    x1[e] = y1;
+    x2[e] = y2;
+  }
+}
+
+__global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
+    attn_decode_kernel(const uint16_t* __restrict__ qkv, AttnShape s, const int* __restrict__ pos0,
+                       const float* __restrict__ qn, const float* __restrict__ kn, float eps,
+                       const float* __restrict__ rope_cos, const float* __restrict__ rope_sin,
+                       uint16_t* __restrict__ kcache, uint16_t* __restrict__ vcache, uint16_t* __restrict__ o) {
+  extern __shared__ __align__(16) uint8_t sm[];
+  pdl_trigger();
+  const int r = blockIdx.x, b = blockIdx.y, kvh = blockIdx.z;
+  const int G = s.n_q / s.n_kv, KG = kWarps / G;  // heads per key/value head; key groups per tile
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int hw = warp % G, gw = warp / G;         // this warp's head (within the group) and key group
+  const int kpw = kTile / KG;                     // keys of a tile per warp
+  // The position was set before this launch's chain began, and cached rows before it were
+  // written by earlier launches: both may be read before waiting for the preceding kernel.
+  const int pos = *pos0;
+  const int lo = s.window > 0 ? max(0, pos - s.window + 1) : 0;
+  const int len = pos - lo + 1;
+  const int used = max(1, min(kSplits, (len + kMinKeys - 1) / kMinKeys));
+  const int chunk = (len + used - 1) / used;
+  const int kb = lo + r * chunk, ke = r < used ? min(pos + 1, kb + chunk) : kb;  // [kb, ke)
+  const bool owns_new = r < used && ke == pos + 1;
+  const int kc_end = owns_new ? pos : ke;  // cached rows [kb, kc_end)
+  const int ntiles = (ke - kb + kTile - 1) / kTile;
+  const size_t row_stride = (size_t)s.n_kv * kHd;
+  const size_t seq_base = (size_t)b * s.max_seq * row_stride + (size_t)kvh * kHd;
+  const uint32_t sbase = smem_u32(sm);
+
+  auto stage = [&](int t) {  // cached rows of tile t into the buffer
+    const int j0 = kb + t * kTile, n = min(kTile, kc_end - j0);
+    const uint32_t kd = sbase + kOffBuf, vd = kd + kTile * kKRow;
+    for (int i = threadIdx.x; i < n * (kHd / 8); i += kWarps * 32) {
+      const int jj = i >> 5, c = i & 31;
+      const size_t off = seq_base + (size_t)(j0 + jj) * row_stride + 8 * c;
+      cp_async16(kd + (uint32_t)(jj * kKRow + 16 * c), kcache + off);
+      cp_async16(vd + (uint32_t)(jj * kVRow + 16 * c), vcache + off);
+    }
+    cp_async_commit();
+  };
+  if (ntiles > 0) stage(0);
+  // norm weights and the RoPE row of this position: constants, read before the wait as well
+  const float* cos_row = rope_cos + (size_t)pos * (kHd / 2);
+  const float* sin_row = rope_sin + (size_t)pos * (kHd / 2);
+  const int kwarp = G;  // the warp that rotates the new key (G < 8 warps)
+  RopeConsts qc, kc2;
+  if (r < used && warp < G) load_rope_consts(qc, qn, cos_row, sin_row, lane);
+  if (owns_new && warp == kwarp) load_rope_consts(kc2, kn, cos_row, sin_row, lane);
+
+  pdl_wait();
+  // ---- the new row: q heads (scaled, fp32, to shared memory), and k / v for the owning CTA
+  const int qkv_dim = (s.n_q + 2 * s.n_kv) * kHd;
+  const uint16_t* src_row = qkv + (size_t)b * qkv_dim;
+  if (r < used) {
+    if (warp < G) {
+      const uint16_t* src = src_row + (size_t)(kvh * G + warp) * kHd;
+      const uint2 a = *reinterpret_cast<const uint2*>(src + 4 * lane);
+      const uint2 c = *reinterpret_cast<const uint2*>(src + kHd / 2 + 4 * lane);
+      float x1[4] = {bf16_lo(a.x), bf16_hi(a.x), bf16_lo(a.y), bf16_hi(a.y)};
+      float x2[4] = {bf16_lo(c.x), bf16_hi(c.x), bf16_lo(c.y), bf16_hi(c.y)};
+      norm_rope(x1, x2, qn != nullptr, qc, eps);
+      float* qd = reinterpret_cast<float*>(sm + kOffQ) + warp * kHd;
+      *reinterpret_cast<float4*>(qd + 4 * lane) = make_float4(x1[0] * s.scale, x1[1] * s.scale, x1[2] * s.scale,
+                                                              x1[3] * s.scale);
+      *reinterpret_cast<float4*>(qd + kHd / 2 + 4 * lane) =
+          make_float4(x2[0] * s.scale, x2[1] * s.scale, x2[2] * s.scale, x2[3] * s.scale);
+    }
+    if (owns_new && warp == kwarp) {  // key head kvh
+      const uint16_t* src = src_row + (size_t)(s.n_q + kvh) * kHd;
+      const uint2 a = *reinterpret_cast<const uint2*>(src + 4 * lane);
+      const uint2 c = *reinterpret_cast<const uint2*>(src + kHd / 2 + 4 * lane);
+      float x1[4] = {bf16_lo(a.x), bf16_hi(a.x), bf16_lo(a.y), bf16_hi(a.y)};
+      float x2[4] = {bf16_lo(c.x), bf16_hi(c.x), bf16_lo(c.y), bf16_hi(c.y)};
+      norm_rope(x1, x2, kn != nullptr, kc2, eps);
+      uint2 u1, u2;
+      u1.x = (uint32_t)f32_to_bf16_bits(x1[0]) | ((uint32_t)f32_to_bf16_bits(x1[1]) << 16);
+      u1.y = (uint32_t)f32_to_bf16_bits(x1[2]) | ((uint32_t)f32_to_bf16_bits(x1[3]) << 16);
+      u2.x = (uint32_t)f32_to_bf16_bits(x2[0]) | ((uint32_t)f32_to_bf16_bits(x2[1]) << 16);
+      u2.y = (uint32_t)f32_to_bf16_bits(x2[2]) | ((uint32_t)f32_to_bf16_bits(x2[3]) << 16);
+      uint16_t* kd = kcache + seq_base + (size_t)pos * row_stride;
+      *reinterpret_cast<uint2*>(kd + 4 * lane) = u1;
+      *reinterpret_cast<uint2*>(kd + kHd / 2 + 4 * lane) = u2;
+      *reinterpret_cast<uint2*>(sm + kOffKNew + 8 * lane) = u1;
+      *reinterpret_cast<uint2*>(sm + kOffKNew + kHd + 8 * lane) = u2;
+    }
+    if (owns_new && warp == kWarps - 1) {  // value head kvh: straight copy
+      const uint16_t* src = src_row + (size_t)(s.n_q + s.n_kv + kvh) * kHd;
+      const uint4 v = *reinterpret_cast<const uint4*>(src + 8 * lane);
+      *reinterpret_cast<uint4*>(vcache + seq_base + (size_t)pos * row_stride + 8 * lane) = v;
+      *reinterpret_cast<uint4*>(sm + kOffVNew + 16 * lane) = v;
+    }
+  }
+  __syncthreads();
+
+  // ---- this warp's keys of every tile
+  const float* qs = reinterpret_cast<const float*>(sm + kOffQ) + hw * kHd;
+  float m = -INFINITY, l = 0.0f, acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  for (int t = 0; t < ntiles; ++t) {
+    cp_async_wait<0>();
+    __syncthreads();
+    const int j0 = kb + t * kTile;
+    const uint8_t* kt = sm + kOffBuf;
+    const uint8_t* vt = kt + kTile * kKRow;
+    for (int base = gw * kpw; base < (gw + 1) * kpw; base += 32) {
+      const int j = base + lane;          // key index within the tile
+      const int p = j0 + j;               // its position
+      const int nk = min(32, min((gw + 1) * kpw, ke - j0) - base);  // valid keys of this block
+      if (nk <= 0) break;
+      float sc = -INFINITY;
+      if (lane < nk) {
+        const uint4* kr = reinterpret_cast<const uint4*>(p == pos ? sm + kOffKNew : kt + j * kKRow);
+        float d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll 8
+        for (int c = 0; c < kHd / 8; ++c) {
+          float kx[8];
+          unpack8_bf16(kr[c], kx);
+          const float4 q0 = reinterpret_cast<const float4*>(qs + 8 * c)[0];
+          const float4 q1 = reinterpret_cast<const float4*>(qs + 8 * c)[1];
+          float& dd = d[c & 3];
+          dd = fmaf(q0.x, kx[0], dd);
+          dd = fmaf(q0.y, kx[1], dd);
+          dd = fmaf(q0.z, kx[2], dd);
+          dd = fmaf(q0.w, kx[3], dd);
+          dd = fmaf(q1.x, kx[4], dd);
+          dd = fmaf(q1.y, kx[5], dd);
+          dd = fmaf(q1.z, kx[6], dd);
+          dd = fmaf(q1.w, kx[7], dd);
+        }
+        sc = (d[0] + d[1]) + (d[2] + d[3]);
+      }
+      const float m_new = fmaxf(m, warp_max_f(sc));
+      const float corr = expf(m - m_new);  // 0 on the first block (m = -inf)
+      const float pr = lane < nk ? expf(sc - m_new) : 0.0f;
+      l = l * corr + warp_sum_f(pr);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] *= corr;
+      for (int jj0 = 0; jj0 < nk; jj0 += 4) {  // four keys' loads in flight
+        float pj[4];
+        uint4 vv[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int jj = jj0 + u < nk ? jj0 + u : 0;  // past the block: key 0 with weight 0
+          pj[u] = __shfl_sync(0xffffffffu, pr, jj);
+          if (jj0 + u >= nk) pj[u] = 0.0f;
+          const uint8_t* vrow = (j0 + base + jj == pos) ? sm + kOffVNew : vt + (base + jj) * kVRow;
+          vv[u] = reinterpret_cast<const uint4*>(vrow)[lane];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          float vx[8];
+          unpack8_bf16(vv[u], vx);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[e] = fmaf(pj[u], vx[e], acc[e]);
+        }
+      }
+      m = m_new;
+    }
+    __syncthreads();  // the buffer is refilled for tile t + 1
+    if (t + 1 < ntiles) stage(t + 1);
+  }
+
+  // ---- partials: the warps of a head combine inside the CTA, the CTA pushes the result into CTA
+  // 0's inbox (distributed shared memory stores), and CTA 0 combines the inbox after one barrier
+  float* part = reinterpret_cast<float*>(sm + kOffPart) + warp * kPartFloats;
+  *reinterpret_cast<float4*>(part + 8 * lane) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  *reinterpret_cast<float4*>(part + 8 * lane + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
+  if (lane == 0) {
+    part[kHd] = m;
+    part[kHd + 1] = l;
+  }
+  __syncthreads();
+  if (warp < G) {
+    const float* p0 = reinterpret_cast<const float*>(sm + kOffPart);
+    float M = -INFINITY;
+    for (int g = 0; g < KG; ++g) M = fmaxf(M, p0[(g * G + warp) * kPartFloats + kHd]);
+    float Lc = 0.0f, y[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int g = 0; g < KG; ++g) {
+      const float* pg = p0 + (g * G + warp) * kPartFloats;
+      const float mg = pg[kHd];
+      const float f = mg == -INFINITY ? 0.0f : expf(mg - M);  // empty partials weigh nothing
+      Lc += pg[kHd + 1] * f;
+      const float4 a = reinterpret_cast<const float4*>(pg + 8 * lane)[0];
+      const float4 c = reinterpret_cast<const float4*>(pg + 8 * lane)[1];
+      y[0] = fmaf(a.x, f, y[0]); y[1] = fmaf(a.y, f, y[1]); y[2] = fmaf(a.z, f, y[2]); y[3] = fmaf(a.w, f, y[3]);
+      y[4] = fmaf(c.x, f, y[4]); y[5] = fmaf(c.y, f, y[5]); y[6] = fmaf(c.z, f, y[6]); y[7] = fmaf(c.w, f, y[7]);
+    }
+    const uint32_t dst = map_to_rank(sbase + kOffInbox + (uint32_t)((r * kMaxG + warp) * kPartFloats * 4), 0);
+    st_cluster_f32x4(dst + 32 * lane, y[0], y[1], y[2], y[3]);
+    st_cluster_f32x4(dst + 32 * lane + 16, y[4], y[5], y[6], y[7]);
+    if (lane == 0) {
+      st_cluster_f32(dst + kHd * 4, M);
+      st_cluster_f32(dst + (kHd + 1) * 4, Lc);
+    }
+  }
+  cluster_sync_all();  // release the pushes / acquire them in CTA 0
+  if (r == 0 && warp < G) {
+    const float* in = reinterpret_cast<const float*>(sm + kOffInbox);
+    const float mi = lane < kSplits ? in[(lane * kMaxG + warp) * kPartFloats + kHd] : -INFINITY;
+    const float li = lane < kSplits ? in[(lane * kMaxG + warp) * kPartFloats + kHd + 1] : 0.0f;
+    const float mx = warp_max_f(mi);
+    const float fi = mi == -INFINITY ? 0.0f : expf(mi - mx);
+    const float L = warp_sum_f(li * fi);
+    float y[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+    for (int i = 0; i < kSplits; ++i) {
+      const float f = __shfl_sync(0xffffffffu, fi, i);
+      const float* pi = in + (i * kMaxG + warp) * kPartFloats + 8 * lane;
+      const float4 a = reinterpret_cast<const float4*>(pi)[0];
+      const float4 c = reinterpret_cast<const float4*>(pi)[1];
+      y[0] = fmaf(a.x, f, y[0]); y[1] = fmaf(a.y, f, y[1]); y[2] = fmaf(a.z, f, y[2]); y[3] = fmaf(a.w, f, y[3]);
+      y[4] = fmaf(c.x, f, y[4]); y[5] = fmaf(c.y, f, y[5]); y[6] = fmaf(c.z, f, y[6]); y[7] = fmaf(c.w, f, y[7]);
+    }
+    uint4 w;
+    float z[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) z[e] = y[e] / L;
+    w.x = (uint32_t)f32_to_bf16_bits(z[0]) | ((uint32_t)f32_to_bf16_bits(z[1]) << 16);
+    w.y = (uint32_t)f32_to_bf16_bits(z[2]) | ((uint32_t)f32_to_bf16_bits(z[3]) << 16);
+    w.z = (uint32_t)f32_to_bf16_bits(z[4]) | ((uint32_t)f32_to_bf16_bits(z[5]) << 16);
+    w.w = (uint32_t)f32_to_bf16_bits(z[6]) | ((uint32_t)f32_to_bf16_bits(z[7]) << 16);
+    *reinterpret_cast<uint4*>(o + (size_t)b * (s.n_q * kHd) + (size_t)(kvh * G + warp) * kHd + 8 * lane) = w;
+  }
+}
+
+}  // namespace
+
+bool attn_decode_supported(const AttnShape& s) {
+  if (s.T != 1 || s.hd != kHd || s.n_kv <= 0 || s.n_q % s.n_kv != 0) return false;
+  const int G = s.n_q / s.n_kv;
+  return G == 2 || G == 4;
+}
+
+w8a8_status launch_attn_decode(const uint16_t* qkv, const AttnShape& s, const int* pos0, const float* qn,
+                               const float* kn, float eps, const float* rope_cos, const float* rope_sin,
+                               uint16_t* kcache, uint16_t* vcache, uint16_t* o, cudaStream_t st) {
+  if (s.B == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(attn_decode_supported(s), W8A8_ERR_SHAPE,
+                 "decode attention: needs one token per sequence, head_dim 256 and 2 or 4 query heads per kv head");
+  static bool attr_set[64] = {};
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    W8A8_CUDA(cudaFuncSetAttribute(attn_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem));
+    attr_set[dev] = true;
+  }
+  W8A8_CUDA(launch_pdl(attn_decode_kernel, dim3(kSplits, s.B, s.n_kv), dim3(kWarps * 32), (size_t)kSmem, st, qkv, s,
+                       pos0, qn, kn, eps, rope_cos, rope_sin, kcache, vcache, o));
+  return W8A8_OK;
+}
+
+}  // namespace w8a8

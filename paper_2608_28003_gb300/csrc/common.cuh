@@ -1,6 +1,8 @@
 // Shared device/host helpers of libw8a8 (sm_103a).
 #pragma once
 
+#include <utility>
+
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
 #include <cuda_bf16.h>
@@ -33,6 +35,33 @@ const char* get_error();
   } while (0)
 
 #define W8A8_LAUNCH_CHECK() W8A8_CUDA(cudaGetLastError())
+
+// Programmatic dependent launch.  Kernels of the decoder path are launched with programmatic
+// stream serialization: the next kernel in the stream may start while this one runs, so that it
+// can set up and stream its weights (immutable) early.  Every such kernel calls pdl_wait() before
+// its first read of data an earlier kernel wrote and before its first global write; pdl_wait()
+// returns once the preceding grid has completed and its writes are visible (at once when the
+// launch allowed no overlap).  Because every kernel waits before it can finish, completion is
+// ordered along the whole stream.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+// Let the next kernel in the stream begin launching (its CTAs start as resources free up).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 #define W8A8_TRY(expr)            \
   do {                            \

@@ -26,8 +26,8 @@ __device__ float block_sum(float v, float* red) {
   return s;
 }
 
-constexpr int kRowThreads = 128;
-constexpr int kRowVec = 4;  // 8-element vectors per thread: H <= 4096
+constexpr int kRowThreads = 256;
+constexpr int kRowVec = 2;  // 8-element vectors per thread: H <= 4096
 
 __device__ __forceinline__ void unpack8(const uint4& w, float (&x)[8]) {
   x[0] = bf16_lo(w.x); x[1] = bf16_hi(w.x); x[2] = bf16_lo(w.y); x[3] = bf16_hi(w.y);
@@ -47,6 +47,8 @@ __global__ void __launch_bounds__(kRowThreads) embed_norm_kernel(const int32_t* 
                                                                  const uint16_t* __restrict__ embed, int H, float scale,
                                                                  const float* __restrict__ w, float eps,
                                                                  float* __restrict__ r, uint16_t* __restrict__ a) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
   const int row = blockIdx.x;
   int tok = tokens[row];
@@ -87,16 +89,37 @@ __global__ void __launch_bounds__(kRowThreads) residual_norm_kernel(const uint16
                                                                     const float* __restrict__ w_post,
                                                                     const float* __restrict__ w_next, float eps,
                                                                     float* __restrict__ r, uint16_t* __restrict__ a) {
+  pdl_trigger();
   __shared__ float red[32];
   const int row = blockIdx.x;
   const int nv = H >> 3;
-  float yv[kRowVec][8];
+  // the norm weights are constants: read them before the preceding kernel has finished
+  float wp[kRowVec][8], wn[kRowVec][8];
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      const float4* p0 = reinterpret_cast<const float4*>(w_post + vi * 8);
+      const float4* p1 = reinterpret_cast<const float4*>(w_next + vi * 8);
+      const float4 a0 = p0[0], a1 = p0[1], b0 = p1[0], b1 = p1[1];
+      wp[v][0] = a0.x; wp[v][1] = a0.y; wp[v][2] = a0.z; wp[v][3] = a0.w;
+      wp[v][4] = a1.x; wp[v][5] = a1.y; wp[v][6] = a1.z; wp[v][7] = a1.w;
+      wn[v][0] = b0.x; wn[v][1] = b0.y; wn[v][2] = b0.z; wn[v][3] = b0.w;
+      wn[v][4] = b1.x; wn[v][5] = b1.y; wn[v][6] = b1.z; wn[v][7] = b1.w;
+    }
+  }
+  pdl_wait();
+  float yv[kRowVec][8], rv[kRowVec][8];
   float ss = 0.0f;
 #pragma unroll
   for (int v = 0; v < kRowVec; ++v) {
     const int vi = threadIdx.x + v * kRowThreads;
     if (vi < nv) {
       unpack8(reinterpret_cast<const uint4*>(y + (size_t)row * H)[vi], yv[v]);
+      const float4* rp = reinterpret_cast<const float4*>(r + (size_t)row * H + vi * 8);
+      const float4 r0 = rp[0], r1 = rp[1];
+      rv[v][0] = r0.x; rv[v][1] = r0.y; rv[v][2] = r0.z; rv[v][3] = r0.w;
+      rv[v][4] = r1.x; rv[v][5] = r1.y; rv[v][6] = r1.z; rv[v][7] = r1.w;
 #pragma unroll
       for (int e = 0; e < 8; ++e) ss += yv[v][e] * yv[v][e];
     }
@@ -107,17 +130,14 @@ __global__ void __launch_bounds__(kRowThreads) residual_norm_kernel(const uint16
   for (int v = 0; v < kRowVec; ++v) {
     const int vi = threadIdx.x + v * kRowThreads;
     if (vi < nv) {
-      float4* rp = reinterpret_cast<float4*>(r + (size_t)row * H + vi * 8);
-      const float4 r0 = rp[0], r1 = rp[1];
-      float rv[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
-        rv[e] += yv[v][e] * inv_y * w_post[vi * 8 + e];
-        yv[v][e] = rv[e];  // keep the new residual
-        ss2 += rv[e] * rv[e];
+        rv[v][e] += yv[v][e] * inv_y * wp[v][e];
+        ss2 += rv[v][e] * rv[v][e];
       }
-      rp[0] = make_float4(rv[0], rv[1], rv[2], rv[3]);
-      rp[1] = make_float4(rv[4], rv[5], rv[6], rv[7]);
+      float4* rp = reinterpret_cast<float4*>(r + (size_t)row * H + vi * 8);
+      rp[0] = make_float4(rv[v][0], rv[v][1], rv[v][2], rv[v][3]);
+      rp[1] = make_float4(rv[v][4], rv[v][5], rv[v][6], rv[v][7]);
     }
   }
   const float inv_r = 1.0f / sqrtf(block_sum(ss2, red) / (float)H + eps);
@@ -125,10 +145,10 @@ __global__ void __launch_bounds__(kRowThreads) residual_norm_kernel(const uint16
   for (int v = 0; v < kRowVec; ++v) {
     const int vi = threadIdx.x + v * kRowThreads;
     if (vi < nv) {
-      float o[8];
+      float out[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) o[e] = yv[v][e] * inv_r * w_next[vi * 8 + e];
-      reinterpret_cast<uint4*>(a + (size_t)row * H)[vi] = pack8(o);
+      for (int e = 0; e < 8; ++e) out[e] = rv[v][e] * inv_r * wn[v][e];
+      reinterpret_cast<uint4*>(a + (size_t)row * H)[vi] = pack8(out);
     }
   }
 }
@@ -139,6 +159,8 @@ __global__ void qk_rope_kernel(const uint16_t* __restrict__ qkv, AttnShape s, co
                                const float* __restrict__ qn, const float* __restrict__ kn, float eps,
                                const float* __restrict__ rope_cos, const float* __restrict__ rope_sin,
                                float* __restrict__ q, uint16_t* __restrict__ kcache, uint16_t* __restrict__ vcache) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x;
   const int b = row / s.T, t = row - (row / s.T) * s.T;
   const int pos = *pos0 + t;
@@ -201,18 +223,40 @@ __global__ void qk_rope_kernel(const uint16_t* __restrict__ qkv, AttnShape s, co
 // ---------------------------------------------------------------------------------- attention
 constexpr int kKeyTile = 32;
 constexpr int kHd = 256;
+constexpr int kKStride = kHd + 8;                           // key rows padded to 528 bytes (see below)
+constexpr int kKTileBytes = kKeyTile * kKStride * 2;        // one key tile, bf16
+constexpr int kVTileBytes = kKeyTile * kHd * 2;             // one value tile, bf16
+constexpr int kBufBytes = kKTileBytes + kVTileBytes;
+constexpr int kMaxGroup = 8;                                // query heads per key/value head
+constexpr int kAttnSmem = 2 * kBufBytes + kMaxGroup * kHd * 4;  // two buffers + the scaled queries
 constexpr int kPartStride = kHd + 4;  // floats per split partial: o[256], m, l, 2 pad (16-byte multiple)
+constexpr int kMinSplitKeys = 64;     // a key-range split covers at least this many keys
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
 
 // grid (splits, rows, n_kv), block 32 * G (G = n_q / n_kv query heads sharing one key/value head).
-// Warp h handles query head kvh * G + h; lane l holds dims 8l .. 8l+7 of q and of its output.
+// Warp h handles query head kvh * G + h.  Key/value tiles of 32 positions are copied into shared
+// memory asynchronously, two buffers deep (the next tile's copies are in flight while the current
+// one is used).  Scores: lane j computes the whole dot product of the query with key j of the
+// tile (the query, scaled, is read from shared memory as a broadcast; key rows are padded to 528
+// bytes so that the 8 lanes of a shared-memory phase read 8 different 16-byte bank groups).
+// Output: lane l accumulates dims 8l .. 8l+7 over the tile's keys.
 __global__ void __launch_bounds__(256) attention_kernel(const float* __restrict__ q, const uint16_t* __restrict__ kcache,
                                                         const uint16_t* __restrict__ vcache, AttnShape s,
                                                         const int* __restrict__ pos0, uint16_t* __restrict__ o,
                                                         float* __restrict__ part, unsigned int* __restrict__ ctr) {
-  __shared__ __align__(16) uint16_t ks[kKeyTile][kHd];
-  __shared__ __align__(16) uint16_t vs[kKeyTile][kHd];
+  extern __shared__ __align__(16) uint8_t att_smem[];
   __shared__ int s_last;
-  const int S = gridDim.x, split = blockIdx.x, row = blockIdx.y, kvh = blockIdx.z;
+  pdl_trigger();
+  pdl_wait();
+  const int split = blockIdx.x, row = blockIdx.y, kvh = blockIdx.z;
   const int G = blockDim.x >> 5;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int head = kvh * G + warp;
@@ -220,37 +264,71 @@ __global__ void __launch_bounds__(256) attention_kernel(const float* __restrict_
   const int pos = *pos0 + t;
   const int lo = s.window > 0 ? max(0, pos - s.window + 1) : 0;
   const int len = pos - lo + 1;
+  // Splits actually used by this row: at least kMinSplitKeys keys each, at most the grid's; the
+  // rest of the grid's CTAs for this row have nothing to do.
+  const int S = max(1, min((int)gridDim.x, (len + kMinSplitKeys - 1) / kMinSplitKeys));
+  if (split >= S) return;
   const int chunk = (len + S - 1) / S;
   const int kb = lo + split * chunk, ke = min(pos + 1, kb + chunk);
-
-  float qv[8];
-  {
-    const float4* qp = reinterpret_cast<const float4*>(q + (size_t)row * (s.n_q * kHd) + (size_t)head * kHd + 8 * lane);
-    const float4 a = qp[0], c = qp[1];
-    qv[0] = a.x * s.scale; qv[1] = a.y * s.scale; qv[2] = a.z * s.scale; qv[3] = a.w * s.scale;
-    qv[4] = c.x * s.scale; qv[5] = c.y * s.scale; qv[6] = c.z * s.scale; qv[7] = c.w * s.scale;
-  }
-  float m = -INFINITY, l = 0.0f, acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   const size_t seq_base = ((size_t)b * s.max_seq) * (size_t)(s.n_kv * kHd) + (size_t)kvh * kHd;
-  for (int j0 = kb; j0 < ke; j0 += kKeyTile) {
+  const uint32_t sbase = smem_u32(att_smem);
+  auto stage = [&](int buf, int j0) {
     const int nk = min(kKeyTile, ke - j0);
-    __syncthreads();
+    const uint32_t kd = sbase + (uint32_t)(buf * kBufBytes), vd = kd + kKTileBytes;
     for (int i = threadIdx.x; i < nk * (kHd / 8); i += blockDim.x) {
       const int jj = i / (kHd / 8), c = i - jj * (kHd / 8);
       const size_t off = seq_base + (size_t)(j0 + jj) * (s.n_kv * kHd) + 8 * c;
-      reinterpret_cast<uint4*>(&ks[jj][0])[c] = *reinterpret_cast<const uint4*>(kcache + off);
-      reinterpret_cast<uint4*>(&vs[jj][0])[c] = *reinterpret_cast<const uint4*>(vcache + off);
+      cp_async16(kd + (uint32_t)((jj * kKStride + 8 * c) * 2), kcache + off);
+      cp_async16(vd + (uint32_t)((jj * kHd + 8 * c) * 2), vcache + off);
+    }
+    cp_async_commit();
+  };
+  if (kb < ke) stage(0, kb);
+
+  // this warp's query, scaled, in shared memory (read back as a broadcast)
+  float* qs = reinterpret_cast<float*>(att_smem + 2 * kBufBytes) + warp * kHd;
+  {
+    const float4* qp = reinterpret_cast<const float4*>(q + (size_t)row * (s.n_q * kHd) + (size_t)head * kHd + 8 * lane);
+    const float4 a = qp[0], c = qp[1];
+    reinterpret_cast<float4*>(qs + 8 * lane)[0] = make_float4(a.x * s.scale, a.y * s.scale, a.z * s.scale, a.w * s.scale);
+    reinterpret_cast<float4*>(qs + 8 * lane)[1] = make_float4(c.x * s.scale, c.y * s.scale, c.z * s.scale, c.w * s.scale);
+  }
+  __syncwarp();
+  float m = -INFINITY, l = 0.0f, acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  int tile = 0;
+  for (int j0 = kb; j0 < ke; j0 += kKeyTile, ++tile) {
+    const int nk = min(kKeyTile, ke - j0);
+    if (j0 + kKeyTile < ke) {
+      stage((tile + 1) & 1, j0 + kKeyTile);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
     __syncthreads();
-    float sc = -INFINITY;  // lane jj keeps the score of key jj
-    for (int jj = 0; jj < nk; ++jj) {
-      float kx[8];
-      unpack8(reinterpret_cast<const uint4*>(&ks[jj][0])[lane], kx);
-      float d = 0.0f;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) d += qv[e] * kx[e];
-      d = warp_sum(d);
-      if (lane == jj) sc = d;
+    const uint8_t* buf = att_smem + (tile & 1) * kBufBytes;
+    const uint16_t* ks = reinterpret_cast<const uint16_t*>(buf);
+    const uint16_t* vs = reinterpret_cast<const uint16_t*>(buf + kKTileBytes);
+    float sc = -INFINITY;  // lane j: the score of key j
+    if (lane < nk) {
+      const uint4* kr = reinterpret_cast<const uint4*>(ks + lane * kKStride);
+      float d[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // four partial sums, added in a fixed order
+#pragma unroll 8
+      for (int c = 0; c < kHd / 8; ++c) {
+        float kx[8];
+        unpack8(kr[c], kx);
+        const float4 q0 = reinterpret_cast<const float4*>(qs + 8 * c)[0];
+        const float4 q1 = reinterpret_cast<const float4*>(qs + 8 * c)[1];
+        float& dd = d[c & 3];
+        dd = fmaf(q0.x, kx[0], dd);
+        dd = fmaf(q0.y, kx[1], dd);
+        dd = fmaf(q0.z, kx[2], dd);
+        dd = fmaf(q0.w, kx[3], dd);
+        dd = fmaf(q1.x, kx[4], dd);
+        dd = fmaf(q1.y, kx[5], dd);
+        dd = fmaf(q1.z, kx[6], dd);
+        dd = fmaf(q1.w, kx[7], dd);
+      }
+      sc = (d[0] + d[1]) + (d[2] + d[3]);
     }
     float tmax = sc;
 #pragma unroll
@@ -261,14 +339,16 @@ __global__ void __launch_bounds__(256) attention_kernel(const float* __restrict_
     l = l * corr + warp_sum(p);
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] *= corr;
+#pragma unroll 4
     for (int jj = 0; jj < nk; ++jj) {
       const float pj = __shfl_sync(0xffffffffu, p, jj);
       float vx[8];
-      unpack8(reinterpret_cast<const uint4*>(&vs[jj][0])[lane], vx);
+      unpack8(reinterpret_cast<const uint4*>(vs + jj * kHd)[lane], vx);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] += pj * vx[e];
+      for (int e = 0; e < 8; ++e) acc[e] = fmaf(pj, vx[e], acc[e]);
     }
     m = m_new;
+    __syncthreads();  // this buffer is refilled two tiles later
   }
 
   uint16_t* out = o + (size_t)row * (s.n_q * kHd) + (size_t)head * kHd + 8 * lane;
@@ -280,7 +360,7 @@ __global__ void __launch_bounds__(256) attention_kernel(const float* __restrict_
     return;
   }
   // partial (m, l, acc) of this split; the last CTA of (row, kvh) combines
-  float* pp = part + (((size_t)row * s.n_q + head) * S + split) * kPartStride;
+  float* pp = part + (((size_t)row * s.n_q + head) * gridDim.x + split) * kPartStride;
   reinterpret_cast<float4*>(pp + 8 * lane)[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
   reinterpret_cast<float4*>(pp + 8 * lane)[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   if (lane == 0) {
@@ -298,18 +378,34 @@ __global__ void __launch_bounds__(256) attention_kernel(const float* __restrict_
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  const float* base = part + ((size_t)row * s.n_q + head) * S * kPartStride;
-  float mx = -INFINITY;
-  for (int sp = 0; sp < S; ++sp) mx = fmaxf(mx, __ldcg(base + (size_t)sp * kPartStride + kHd));
-  float L = 0.0f, y[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-  for (int sp = 0; sp < S; ++sp) {
-    const float* ps = base + (size_t)sp * kPartStride;
-    const float ms = __ldcg(ps + kHd);
-    if (ms == -INFINITY) continue;  // an empty split
-    const float f = expf(ms - mx);
-    L += __ldcg(ps + kHd + 1) * f;
+  // Combine: lane sp reads split sp's (m, l); every lane then reads its 8 outputs of all splits,
+  // four splits' loads in flight at a time.
+  const float* base = part + ((size_t)row * s.n_q + head) * gridDim.x * kPartStride;
+  const float ms = lane < S ? __ldcg(base + (size_t)lane * kPartStride + kHd) : -INFINITY;
+  const float ls = lane < S ? __ldcg(base + (size_t)lane * kPartStride + kHd + 1) : 0.0f;
+  float mx = ms;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) y[e] += __ldcg(ps + 8 * lane + e) * f;
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  const float fs = ms == -INFINITY ? 0.0f : expf(ms - mx);  // an empty split weighs nothing
+  const float L = warp_sum(ls * fs);
+  float y[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  for (int s0 = 0; s0 < S; s0 += 4) {
+    float4 va[4], vb[4];
+    float f[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int sp = min(s0 + j, S - 1);
+      const float4* ps = reinterpret_cast<const float4*>(base + (size_t)sp * kPartStride + 8 * lane);
+      va[j] = __ldcg(ps);
+      vb[j] = __ldcg(ps + 1);
+      f[j] = __shfl_sync(0xffffffffu, fs, sp);
+      if (s0 + j >= S) f[j] = 0.0f;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      y[0] += va[j].x * f[j]; y[1] += va[j].y * f[j]; y[2] += va[j].z * f[j]; y[3] += va[j].w * f[j];
+      y[4] += vb[j].x * f[j]; y[5] += vb[j].y * f[j]; y[6] += vb[j].z * f[j]; y[7] += vb[j].w * f[j];
+    }
   }
 #pragma unroll
   for (int e = 0; e < 8; ++e) y[e] /= L;
@@ -341,8 +437,8 @@ w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embe
                               const float* w, float eps, float* r, uint16_t* a, cudaStream_t st) {
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "embed: hidden %d unsupported", H);
-  embed_norm_kernel<<<M, kRowThreads, 0, st>>>(tokens, vocab, embed, H, embed_scale, w, eps, r, a);
-  W8A8_LAUNCH_CHECK();
+  W8A8_CUDA(launch_pdl(embed_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, tokens, vocab, embed, H, embed_scale, w,
+                       eps, r, a));
   return W8A8_OK;
 }
 
@@ -350,8 +446,7 @@ w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w
                                  float* r, uint16_t* a, cudaStream_t st) {
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "residual norm: hidden %d unsupported", H);
-  residual_norm_kernel<<<M, kRowThreads, 0, st>>>(y, H, w_post, w_next, eps, r, a);
-  W8A8_LAUNCH_CHECK();
+  W8A8_CUDA(launch_pdl(residual_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, y, H, w_post, w_next, eps, r, a));
   return W8A8_OK;
 }
 
@@ -361,9 +456,8 @@ w8a8_status launch_qk_rope(const uint16_t* qkv, const AttnShape& s, const int* p
   const int M = s.B * s.T;
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(s.hd == kHd && s.n_q + 2 * s.n_kv <= 32, W8A8_ERR_SHAPE, "qk_rope: head_dim %d / heads unsupported", s.hd);
-  qk_rope_kernel<<<M, 32 * (s.n_q + 2 * s.n_kv), 0, st>>>(qkv, s, pos0, qn, kn, eps, rope_cos, rope_sin, q, kcache,
-                                                           vcache);
-  W8A8_LAUNCH_CHECK();
+  W8A8_CUDA(launch_pdl(qk_rope_kernel, dim3(M), dim3(32 * (s.n_q + 2 * s.n_kv)), 0, st, qkv, s, pos0, qn, kn, eps,
+                       rope_cos, rope_sin, q, kcache, vcache));
   return W8A8_OK;
 }
 
@@ -382,7 +476,7 @@ w8a8_status launch_attention(const float* q, const uint16_t* kcache, const uint1
   (void)max_pos_hint;
   const int M = s.B * s.T;
   if (M == 0) return W8A8_OK;
-  W8A8_CHECK_ARG(s.hd == kHd && s.n_kv > 0 && s.n_q % s.n_kv == 0 && s.n_q / s.n_kv <= 8, W8A8_ERR_SHAPE,
+  W8A8_CHECK_ARG(s.hd == kHd && s.n_kv > 0 && s.n_q % s.n_kv == 0 && s.n_q / s.n_kv <= kMaxGroup, W8A8_ERR_SHAPE,
                  "attention: head layout unsupported");
   W8A8_CHECK_ARG((size_t)M * s.n_kv * 4 <= kAttnCounterBytes, W8A8_ERR_SHAPE, "attention: %d rows exceed the counters",
                  M);
@@ -390,8 +484,15 @@ w8a8_status launch_attention(const float* q, const uint16_t* kcache, const uint1
   unsigned int* ctr = reinterpret_cast<unsigned int*>(ws);
   float* part = reinterpret_cast<float*>(reinterpret_cast<char*>(ws) + kAttnCounterBytes);
   dim3 grid(S, M, s.n_kv);
-  attention_kernel<<<grid, 32 * (s.n_q / s.n_kv), 0, st>>>(q, kcache, vcache, s, pos0, o, part, ctr);
-  W8A8_LAUNCH_CHECK();
+  static bool attr_set[64] = {};
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    W8A8_CUDA(cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem));
+    attr_set[dev] = true;
+  }
+  W8A8_CUDA(launch_pdl(attention_kernel, grid, dim3(32 * (s.n_q / s.n_kv)), (size_t)kAttnSmem, st, q, kcache, vcache, s,
+                       pos0, o, part, ctr));
   return W8A8_OK;
 }
 

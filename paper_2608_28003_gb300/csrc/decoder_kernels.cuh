@@ -34,6 +34,14 @@ size_t attention_workspace_bytes(const AttnShape& s, int sm_count);
 w8a8_status launch_attention(const float* q, const uint16_t* kcache, const uint16_t* vcache, const AttnShape& s,
                              const int* pos0, int max_pos_hint, uint16_t* o, void* ws, int sm_count, cudaStream_t st);
 
+// Decode (T == 1): QK-norm + RoPE of the new row, its key/value into the cache, and attention over
+// the cache, in one launch (clusters of 8 CTAs combine their key ranges in distributed shared
+// memory).  Same results as launch_qk_rope followed by launch_attention up to fp32 summation order.
+bool attn_decode_supported(const AttnShape& s);
+w8a8_status launch_attn_decode(const uint16_t* qkv, const AttnShape& s, const int* pos0, const float* qn,
+                               const float* kn, float eps, const float* rope_cos, const float* rope_sin,
+                               uint16_t* kcache, uint16_t* vcache, uint16_t* o, cudaStream_t st);
+
 // cos/sin tables [max_seq][hd/2] of RoPE with the given base, computed in fp64
 w8a8_status launch_rope_table(float* cos_t, float* sin_t, int max_seq, int hd, double base, cudaStream_t st);
 

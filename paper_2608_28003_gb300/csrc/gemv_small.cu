@@ -1,0 +1,470 @@
+// Decode GEMV whose CTAs own whole weight rows (K3 for small layers, and the bf16 pass-through).
+//
+// At one to eight tokens a decoder layer's linears are small (2.4 to 32 MB) and each one sits on
+// the critical path of the next, so their cost is latency more than bandwidth.  The
+// weight-streaming kernel splits such a layer's k sum over many CTAs and finishes it with a
+// partial-tile protocol through global memory; here every CTA owns R = 8 RW consecutive weight
+// rows over the full k range, so each sum ends inside its CTA:
+//  * one producer thread streams the CTA's rows through a shared-memory ring with 2-D TMA, starting
+//    before the preceding kernel has finished (weights do not depend on it), and can ask L2 to
+//    fetch a later kernel's weights.  A stage holds KS sub-slices of 512 bytes per row (each one or
+//    two unswizzled boxes of R rows x 256 elements), so that small-R calls still move enough bytes
+//    per pipeline round trip;
+//  * the 8 consumer warps wait for the preceding kernel and stage the activations in shared
+//    memory.  The W8A8 path quantises them there, with the arithmetic of the stand-alone per-token
+//    quantiser (Eq. stx / xint8, smoothing of Eq. xhat-lmhead), so one launch does K1 and K3;
+//  * warp w takes rows w, w + 8, ...; in every sub-slice lane l reads bytes 16 l .. 16 l + 15 of
+//    a row's 512 bytes (consecutive lanes read consecutive bytes: no bank conflicts);
+//  * INT8: four dp4a per 16 bytes and token, exact INT32 sums (Eq. gemm-final); bf16: fp32 FMAs,
+//    sub-slice u of a stage feeding accumulator u mod NA, summed in a fixed order at the end;
+//  * the lanes' sums meet in a butterfly (every lane ends with the same value) and lane 0 runs the
+//    epilogue: dequantisation fl(fl(s_x s_w) acc) (Eq. gemm-final), bias, GeGLU of the FFN section
+//    on interleaved gate/up rows (blocks of 8: rows 16q .. 16q+7 are gate rows 8q .. 8q+7, the next
+//    8 the matching up rows; warp w holds both rows of a pair).
+// Waits are bounded as in the weight-streaming kernel (error word, no hang).
+#include <algorithm>
+#include <type_traits>
+
+#include "gemv_small.cuh"
+#include "stream_gemm.cuh"
+#include "tmap.cuh"
+
+namespace w8a8 {
+
+namespace {
+
+constexpr int kCW = 8;  // consumer warps
+constexpr int kThreads = (kCW + 1) * 32;
+constexpr int kSmemLimit = 227 * 1024;
+constexpr int kStatic = 2048;       // static shared memory of the kernel (reduction slots, scales) + slack
+constexpr int kSliceBytes = 512;    // bytes of one weight row per sub-slice
+constexpr int kMaxInt8K = 8 * 256 * 4;  // K1 keeps a token's smoothed row in registers: 4 vectors of 8 per thread
+
+__device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(ptr), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
+  x[0] = bf16_lo(v.x); x[1] = bf16_hi(v.x); x[2] = bf16_lo(v.y); x[3] = bf16_hi(v.y);
+  x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
+}
+
+template <bool kInt8, int MT, int RW>
+__global__ void __launch_bounds__(kThreads, 2)
+    gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
+  constexpr int R = 8 * RW;
+  using Acc = typename std::conditional<kInt8, int, float>::type;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ float s_red[kCW];
+  __shared__ float s_sx[MT];
+
+  const SmallPlan& p = a.p;
+  const int S = p.stages, SB = p.stage_bytes, nst = p.nst, kpad = p.kpad, KS = p.ks, nsub = p.nsub;
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t ring = (raw + 1023u) & ~1023u;
+  const uint32_t xs = ring + (uint32_t)(S * SB);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (ring - raw) + (size_t)S * SB + p.xbytes);
+  uint64_t* empty = full + S;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row0 = blockIdx.x * R;
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(full + s), 1);
+      mbar_init(smem_u32(empty + s), kCW);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  // ------------------------------------------------------------------------ producer thread
+  if (warp == kCW) {
+    if (lane != 0) return;
+    bool ok = true;
+    int it = 0, s = 0;
+    uint32_t ph = 0;
+    const int first_fill = S < nst ? S : nst;
+    for (; it < nst; ++it) {
+      if (!mbar_wait_bounded(smem_u32(empty + s), ph ^ 1u, kWaitBudgetCycles)) {
+        ok = false;
+        break;
+      }
+      const int u0 = it * KS, cnt = min(KS, nsub - u0);
+      const uint32_t bar = smem_u32(full + s), dst = ring + (uint32_t)(s * SB);
+      mbar_arrive_expect_tx(bar, (uint32_t)(cnt * R * kSliceBytes));
+      for (int u = 0; u < cnt; ++u) {
+        const uint32_t d = dst + (uint32_t)(u * R * kSliceBytes);
+        if constexpr (kInt8) {
+          tma_load_2d(d, &tmW, (u0 + u) * 512, row0, bar);
+          tma_load_2d(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar);
+        } else {
+          tma_load_2d(d, &tmW, (u0 + u) * 256, row0, bar);
+        }
+      }
+      if (it + 1 == first_fill && a.prefetch) {  // this CTA's share of a later kernel's weights
+        const size_t per = ((a.prefetch_bytes + gridDim.x - 1) / gridDim.x + 15) / 16 * 16;
+        const size_t beg = per * blockIdx.x;
+        const size_t end = beg + per < a.prefetch_bytes ? beg + per : a.prefetch_bytes;
+        for (size_t off = beg; off < end; off += 65536) {
+          const size_t n = end - off < 65536 ? end - off : 65536;
+          prefetch_l2(reinterpret_cast<const char*>(a.prefetch) + off, (uint32_t)n);
+        }
+      }
+      if (++s == S) {
+        s = 0;
+        ph ^= 1u;
+      }
+    }
+    if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
+    for (int j = it > S ? it - S : 0; j < it; ++j) {
+      if (!mbar_wait_bounded(smem_u32(full + j % S), (uint32_t)((j / S) & 1), kWaitBudgetCycles)) {
+        atomicOr(a.err, DEVERR_DRAIN_WAIT);
+        break;
+      }
+    }
+    return;
+  }
+
+  // ------------------------------------------------------------------------ consumer warps
+  const int tid = threadIdx.x;  // 0 .. 255
+  // Constants of this warp's rows (per-channel scales, bias) and of K1 (1 / delta): read before
+  // waiting for the preceding kernel, so that their latency is off the critical path.
+  float swr[RW], bir[RW];
+#pragma unroll
+  for (int i = 0; i < RW; ++i) {
+    const int row = row0 + warp + 8 * i;
+    swr[i] = kInt8 && row < a.N ? a.s_w[row] : 0.0f;
+    bir[i] = a.bias && row < a.N ? a.bias[row] : 0.0f;
+  }
+  float4 idr[4][2];
+  if constexpr (kInt8) {
+    const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const int vi = tid + v * kCW * 32;
+      if (vi < (a.K >> 3)) {
+        idr[v][0] = idl[2 * vi];
+        idr[v][1] = idl[2 * vi + 1];
+      }
+    }
+  }
+  pdl_wait();
+  uint8_t* xsp = smem_raw + (xs - raw);
+  if constexpr (kInt8) {
+    // K1 for every token slot: x_hat = x * (1 / delta), m = max |x_hat|, s = m / 127,
+    // q = clamp(rint(x_hat * (127 / m)), -127, 127); slots >= M and the tail past K hold zeros.
+    const int nvec = a.K >> 3;
+    for (int m = 0; m < MT; ++m) {
+      float xh[4][8];
+      float amax = 0.0f;
+      const bool live = m < a.M;
+      if (live) {
+        const uint4* src = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K);
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          const int vi = tid + v * kCW * 32;
+          if (vi < nvec) {
+            const uint4 w = src[vi];
+            const float4 d0 = idr[v][0], d1 = idr[v][1];
+            xh[v][0] = __fmul_rn(bf16_lo(w.x), d0.x);
+            xh[v][1] = __fmul_rn(bf16_hi(w.x), d0.y);
+            xh[v][2] = __fmul_rn(bf16_lo(w.y), d0.z);
+            xh[v][3] = __fmul_rn(bf16_hi(w.y), d0.w);
+            xh[v][4] = __fmul_rn(bf16_lo(w.z), d1.x);
+            xh[v][5] = __fmul_rn(bf16_hi(w.z), d1.y);
+            xh[v][6] = __fmul_rn(bf16_lo(w.w), d1.z);
+            xh[v][7] = __fmul_rn(bf16_hi(w.w), d1.w);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(xh[v][e]));
+          }
+        }
+      }
+      amax = warp_max(amax);
+      if (lane == 0) s_red[warp] = amax;
+      named_bar_sync(1, kCW * 32);
+      float mx = 0.0f;
+#pragma unroll
+      for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red[i]);
+      named_bar_sync(1, kCW * 32);  // s_red is reused by the next slot
+      const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
+      if (tid == 0) {
+        const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127)
+        s_sx[m] = sx;
+        if (live && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
+      }
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int vi = tid + v * kCW * 32;
+        if (vi < nvec) {
+          uint2 packed = make_uint2(0u, 0u);
+          if (live) {
+            int q[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][e], r))));
+            packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                       ((uint32_t)(q[3] & 0xff) << 24);
+            packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                       ((uint32_t)(q[7] & 0xff) << 24);
+            if (a.xq_dbg && blockIdx.x == 0) *reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K + 8 * vi) = packed;
+          }
+          *reinterpret_cast<uint2*>(xsp + (size_t)m * kpad + 8 * vi) = packed;
+        }
+      }
+    }
+    const int tail16 = (kpad - a.K) >> 4;
+    for (int i = tid; i < MT * tail16; i += kCW * 32) {
+      const int m = i / tail16, c = i - m * tail16;
+      *reinterpret_cast<uint4*>(xsp + (size_t)m * kpad + a.K + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
+    }
+  } else {
+    const int vpr = kpad >> 3;  // 16-byte vectors per slot
+    const int total = MT * vpr;
+    for (int i0 = tid; i0 < total; i0 += 4 * kCW * 32) {  // four loads in flight per thread
+      uint4 val[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kCW * 32;
+        const int m = i / vpr, v = i - m * vpr;
+        val[u] = make_uint4(0u, 0u, 0u, 0u);
+        if (i < total && m < a.M && 8 * v < a.K) val[u] = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K)[v];
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kCW * 32;
+        if (i < total) *reinterpret_cast<uint4*>(xsp + (size_t)i * 16) = val[u];
+      }
+    }
+  }
+  named_bar_sync(1, kCW * 32);
+
+  // NA independent accumulators per (row, token) keep the FMA / dp4a chains short when a warp has
+  // few rows and tokens; sub-slice u of every stage feeds accumulator u mod NA.
+  constexpr int NA = RW * MT <= 2 ? 4 : (RW * MT <= 8 ? 2 : 1);
+  Acc acc[NA][RW][MT];
+#pragma unroll
+  for (int c = 0; c < NA; ++c)
+#pragma unroll
+    for (int i = 0; i < RW; ++i)
+#pragma unroll
+      for (int m = 0; m < MT; ++m) acc[c][i][m] = 0;
+  bool ok = true;
+  // INT8 sub-slice: two boxes [R][256 B]; lane l reads box l / 16 at byte 16 (l % 16) of the row
+  const uint32_t wlane = kInt8 ? (uint32_t)((lane >> 4) * R * 256 + 16 * (lane & 15)) : (uint32_t)(16 * lane);
+  int s = 0;
+  uint32_t ph = 0;
+  for (int it = 0; it < nst; ++it) {
+    if (ok) {
+      bool got = true;
+      if (lane == 0) got = mbar_wait_bounded(smem_u32(full + s), ph, kWaitBudgetCycles);
+      got = __shfl_sync(0xffffffffu, got, 0);
+      if (!got) {
+        ok = false;
+        if (lane == 0) atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+      }
+    }
+    if (ok) {
+      const uint32_t sb = ring + (uint32_t)(s * SB);
+      const int u0 = it * KS, cnt = min(KS, nsub - u0);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (u >= cnt) break;
+        const uint32_t sub = sb + (uint32_t)(u * R * kSliceBytes);
+        if constexpr (kInt8) {
+          uint4 xv[MT];
+#pragma unroll
+          for (int m = 0; m < MT; ++m) xv[m] = lds128(xs + (uint32_t)(m * kpad + (u0 + u) * 512 + 16 * lane));
+#pragma unroll
+          for (int i = 0; i < RW; ++i) {
+            const uint4 wv = lds128(sub + wlane + (uint32_t)((warp + 8 * i) * 256));
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+              int t = acc[u % NA][i][m];
+              t = __dp4a((int)wv.x, (int)xv[m].x, t);
+              t = __dp4a((int)wv.y, (int)xv[m].y, t);
+              t = __dp4a((int)wv.z, (int)xv[m].z, t);
+              t = __dp4a((int)wv.w, (int)xv[m].w, t);
+              acc[u % NA][i][m] = t;
+            }
+          }
+        } else {
+          uint4 wv[RW];
+#pragma unroll
+          for (int i = 0; i < RW; ++i) wv[i] = lds128(sub + wlane + (uint32_t)((warp + 8 * i) * kSliceBytes));
+#pragma unroll
+          for (int m = 0; m < MT; ++m) {
+            float x[8];
+            unpack_bf16x8(lds128(xs + (uint32_t)((m * kpad + (u0 + u) * 256 + 8 * lane) * 2)), x);
+#pragma unroll
+            for (int i = 0; i < RW; ++i) {
+              float w[8];
+              unpack_bf16x8(wv[i], w);
+              float t = acc[u % NA][i][m];
+#pragma unroll
+              for (int e = 0; e < 8; ++e) t = fmaf(w[e], x[e], t);
+              acc[u % NA][i][m] = t;
+            }
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(empty + s));
+    }
+    if (++s == S) {
+      s = 0;
+      ph ^= 1u;
+    }
+  }
+  if (!ok) return;
+#pragma unroll
+  for (int c = 1; c < NA; ++c)  // fixed order: ((a0 + a1) + a2) + a3
+#pragma unroll
+    for (int i = 0; i < RW; ++i)
+#pragma unroll
+      for (int m = 0; m < MT; ++m) acc[0][i][m] += acc[c][i][m];
+
+  // butterfly: every lane ends with the full sum (a + b == b + a, so partners agree bit for bit)
+#pragma unroll
+  for (int i = 0; i < RW; ++i)
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[0][i][m] += __shfl_xor_sync(0xffffffffu, acc[0][i][m], o);
+    }
+  if (lane != 0) return;
+
+  auto value = [&](Acc v, int i, int row, int m) -> float {  // i: the warp's row slot of `row`
+    float y;
+    if constexpr (kInt8) {
+      y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), __int2float_rn(v));
+      if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row] = v;
+    } else {
+      y = v;
+    }
+    return a.bias ? __fadd_rn(y, bir[i]) : y;
+  };
+  if (a.kind == EPI_GEGLU) {
+#pragma unroll
+    for (int j = 0; j < RW / 2; ++j) {
+      const int gi = row0 + 16 * j + warp, ui = gi + 8;
+      if (ui >= a.N) continue;
+      const int hid = ((row0 + 16 * j) >> 1) + warp;
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        if (m >= a.M) break;
+        const float g = value(acc[0][2 * j][m], 2 * j, gi, m), u = value(acc[0][2 * j + 1][m], 2 * j + 1, ui, m);
+        a.y[(size_t)m * (a.N >> 1) + hid] = f32_to_bf16_bits(geglu_recipe(g, u));
+      }
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < RW; ++i) {
+      const int row = row0 + warp + 8 * i;
+      if (row >= a.N) continue;
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        if (m >= a.M) break;
+        a.y[(size_t)m * a.N + row] = f32_to_bf16_bits(value(acc[0][i][m], i, row, m));
+      }
+    }
+  }
+}
+
+template <bool kInt8, int MT, int RW>
+w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
+  static bool attr_set[64] = {};
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kInt8, MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemLimit - kStatic));
+    attr_set[dev] = true;
+  }
+  constexpr int EB = kInt8 ? 1 : 2;
+  CUtensorMap tw;
+  W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, false));
+  W8A8_CUDA(launch_pdl(gemv_small_kernel<kInt8, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
+                       a));
+  return W8A8_OK;
+}
+
+template <bool kInt8, int MT>
+w8a8_status launch_mt(const SmallArgs& a, cudaStream_t st) {
+  switch (a.p.RW) {
+    case 1: return launch_t<kInt8, MT, 1>(a, st);
+    case 2: return launch_t<kInt8, MT, 2>(a, st);
+    case 4: return launch_t<kInt8, MT, 4>(a, st);
+    default: return launch_t<kInt8, MT, 6>(a, st);
+  }
+}
+
+template <bool kInt8>
+w8a8_status launch_typed(const SmallArgs& a, cudaStream_t st) {
+  switch (a.p.MT) {
+    case 1: return launch_mt<kInt8, 1>(a, st);
+    case 2: return launch_mt<kInt8, 2>(a, st);
+    case 4: return launch_mt<kInt8, 4>(a, st);
+    default: return launch_mt<kInt8, 8>(a, st);
+  }
+}
+
+}  // namespace
+
+SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count) {
+  SmallPlan p{};
+  if (M < 1 || M > 8 || N < 1 || K < 16 || K % 16 != 0) return p;
+  if (kind != EPI_BF16 && kind != EPI_GEGLU) return p;
+  if (kind == EPI_GEGLU && N % 16 != 0) return p;
+  if (int8_weights && K > kMaxInt8K) return p;
+  p.MT = M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
+  // fewest rows per CTA (more CTAs) that still fit in two CTAs per SM
+  static const int kRw[] = {1, 2, 4, 6};
+  for (int rw : kRw) {
+    if (kind == EPI_GEGLU && (rw & 1)) continue;
+    if ((long long)(N + 8 * rw - 1) / (8 * rw) <= 2LL * sm_count) {
+      p.RW = rw;
+      break;
+    }
+  }
+  if (p.RW == 0) return p;
+  if (!int8_weights && p.MT == 8 && p.RW == 6) return p;  // would spill registers: streaming kernel
+  const int R = 8 * p.RW;
+  p.P = (N + R - 1) / R;
+  const int cps = p.P > sm_count ? 2 : 1;
+  p.sub = int8_weights ? 512 : 256;
+  p.nsub = (K + p.sub - 1) / p.sub;
+  p.kpad = p.nsub * p.sub;
+  p.xbytes = p.MT * p.kpad * (int8_weights ? 1 : 2);
+  const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - 16 * 16;
+  // sub-slices per stage: 4 for warps with one or two rows, fewer for wider CTAs; each stage must
+  // fit twice in the ring unless one stage covers everything
+  for (int ks = p.RW <= 2 ? 4 : p.RW == 4 ? 2 : 1; ks >= 1; ks >>= 1) {
+    const int nst = (p.nsub + ks - 1) / ks, sb = ks * R * kSliceBytes;
+    const int stages = std::min(std::min(16, nst), budget / sb);
+    if (stages >= std::min(nst, 2)) {
+      p.ks = ks;
+      p.nst = nst;
+      p.stage_bytes = sb;
+      p.stages = stages;
+      break;
+    }
+  }
+  if (p.ks == 0) return p;
+  p.smem_bytes = 1024 + p.stages * p.stage_bytes + p.xbytes + 16 * p.stages;
+  p.ok = 1;
+  return p;
+}
+
+w8a8_status launch_small_gemv(bool int8_weights, const SmallArgs& a, cudaStream_t st) {
+  if (a.M == 0 || a.N == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(a.p.ok, W8A8_ERR_SHAPE, "small GEMV: no plan for M=%d N=%d K=%d", a.M, a.N, a.K);
+  void *v0, *v1;
+  take_kernel_events(&v0, &v1);
+  cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
+  if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
+  const w8a8_status s = int8_weights ? launch_typed<true>(a, st) : launch_typed<false>(a, st);
+  if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
+  return s;
+}
+
+}  // namespace w8a8

@@ -1,0 +1,47 @@
+// Decode GEMV for up to 8 tokens whose CTAs own whole weight rows (no split of the k sum across
+// CTAs): the W8A8 path with the per-token quantiser (K1) fused into its prologue, and the bf16
+// pass-through.
+#pragma once
+
+#include "common.cuh"
+
+namespace w8a8 {
+
+struct SmallPlan {
+  int ok;           // 0: this shape is left to the weight-streaming kernel
+  int MT;           // token slots: 1, 2, 4 or 8
+  int RW;           // weight rows per consumer warp: 1, 2, 4 or 6 (R = 8 RW rows per CTA)
+  int P;            // CTAs
+  int sub;          // k elements per 512-byte sub-slice of a row (256 bf16, 512 INT8)
+  int nsub;         // sub-slices covering K
+  int kpad;         // nsub * sub
+  int ks;           // sub-slices per pipeline stage (1, 2 or 4)
+  int nst;          // pipeline steps per CTA (nsub / ks, rounded up)
+  int stages;       // ring depth
+  int stage_bytes;  // ks x R rows x 512 bytes
+  int xbytes;       // activations in shared memory: MT x kpad bf16 or INT8 codes
+  int smem_bytes;
+};
+
+struct SmallArgs {
+  const void* W;           // [N, K] INT8 codes or bf16, row = output channel
+  const uint16_t* X;       // [M, K] bf16 activations
+  int M, N, K;
+  int kind;                // EPI_BF16 or EPI_GEGLU (gate/up rows interleaved in blocks of 8)
+  const float* inv_delta;  // [K] INT8 path: 1 / delta_j
+  const float* s_w;        // [N] INT8 path
+  const float* bias;       // [N] nullable
+  uint16_t* y;             // [M, N] bf16 or [M, N / 2] for GeGLU
+  int8_t* xq_dbg;          // [M, K] nullable: the INT8 activation codes
+  float* s_x_dbg;          // [M] nullable: the per-token scales
+  int32_t* acc_dbg;        // [M, N] nullable: the INT32 sums
+  const void* prefetch;    // nullable: bytes to pull into L2 for a later kernel (16-byte aligned)
+  size_t prefetch_bytes;   // a multiple of 16
+  unsigned int* err;       // device error word
+  SmallPlan p;
+};
+
+SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count);
+w8a8_status launch_small_gemv(bool int8_weights, const SmallArgs& a, cudaStream_t st);
+
+}  // namespace w8a8

@@ -62,7 +62,11 @@ struct w8a8_model {
 
   cudaStream_t st = nullptr;  // private stream for graph capture / replay
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
-  std::map<std::tuple<int, uint32_t, uint32_t, int, int, int>, cudaGraphExec_t> graphs;
+  struct Graph {
+    cudaGraphExec_t exec;
+    int kernels;  // kernel nodes
+  };
+  std::map<std::tuple<int, uint32_t, uint32_t, int, int, int>, Graph> graphs;
   std::vector<void*> allocs;
 
   size_t stats_stride() const { return (size_t)2 * cfg.hidden + q_dim + cfg.inter; }
@@ -91,7 +95,7 @@ w8a8_status dalloc(w8a8_model* m, T** p, size_t count) {
 }
 
 void free_all(w8a8_model* m) {
-  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second.exec);
   m->graphs.clear();
   for (void* p : m->allocs) cudaFree(p);
   m->allocs.clear();
@@ -103,12 +107,12 @@ void free_all(w8a8_model* m) {
 w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, nullptr}; }
 
 w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
-                   uint16_t* Y, cudaStream_t st) {
+                   uint16_t* Y, cudaStream_t st, const L2Prefetch* pf) {
   if (int8) {
     const w8a8_qweight w = qdesc(qw, N, K);
-    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st);
+    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st, pf);
   }
-  return run_bf16_linear(Wbf, N, K, X, M, nullptr, 0, Y, nullptr, nullptr, m->ws, m->sms, st);
+  return run_bf16_linear(Wbf, N, K, X, M, nullptr, 0, Y, nullptr, nullptr, m->ws, m->sms, st, pf);
 }
 
 // The decoder over M = B * T rows whose positions start at *m->d_pos (set by the caller).
@@ -123,16 +127,23 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     const bool ffn8 = !calib && m->prepared && ((m->ffn_bits >> l) & 1u);
     const bool glob = m->is_global(l);
     if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_qkv(l), st));
-    W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st));
+    W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
     AttnShape s{B, T, c.n_q, c.n_kv, c.head_dim, c.max_seq, glob ? 0 : c.window,
                 (float)(1.0 / std::sqrt((double)c.head_dim))};
     uint16_t* kc = m->kc + (size_t)l * m->cache_layer_elems();
     uint16_t* vc = m->vc + (size_t)l * m->cache_layer_elems();
-    W8A8_TRY(launch_qk_rope(m->qkv, s, m->d_pos, c.qk_norm ? W.q_norm : nullptr, c.qk_norm ? W.k_norm : nullptr, c.eps,
-                            glob ? m->cos_g : m->cos_l, glob ? m->sin_g : m->sin_l, m->q, kc, vc, st));
-    W8A8_TRY(launch_attention(m->q, kc, vc, s, m->d_pos, 0, m->o, m->attn_ws, m->sms, st));
+    const float* qn = c.qk_norm ? W.q_norm : nullptr;
+    const float* kn = c.qk_norm ? W.k_norm : nullptr;
+    const float* cs = glob ? m->cos_g : m->cos_l;
+    const float* sn = glob ? m->sin_g : m->sin_l;
+    if (attn_decode_supported(s)) {
+      W8A8_TRY(launch_attn_decode(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, kc, vc, m->o, st));
+    } else {
+      W8A8_TRY(launch_qk_rope(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, m->q, kc, vc, st));
+      W8A8_TRY(launch_attention(m->q, kc, vc, s, m->d_pos, 0, m->o, m->attn_ws, m->sms, st));
+    }
     if (calib) W8A8_TRY(launch_act_absmax(m->o, M, m->q_dim, m->stat_o(l), st));
-    W8A8_TRY(linear(m, att8, m->q_o[l], W.wo, H, m->q_dim, m->o, M, m->y, st));
+    W8A8_TRY(linear(m, att8, m->q_o[l], W.wo, H, m->q_dim, m->o, M, m->y, st, nullptr));
     W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, m->r, m->a, st));
     if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
     w8a8_ffn_weights f{H,
@@ -486,19 +497,40 @@ extern "C" w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* to
     const cudaError_t e = cudaStreamEndCapture(st, &g);
     W8A8_TRY(s);
     W8A8_CUDA(e);
+    int kernels = 0;
+    size_t n_nodes = 0;
+    if (cudaGraphGetNodes(g, nullptr, &n_nodes) == cudaSuccess) {
+      std::vector<cudaGraphNode_t> nodes(n_nodes);
+      if (cudaGraphGetNodes(g, nodes.data(), &n_nodes) == cudaSuccess)
+        for (cudaGraphNode_t nd : nodes) {
+          cudaGraphNodeType t;
+          if (cudaGraphNodeGetType(nd, &t) == cudaSuccess && t == cudaGraphNodeTypeKernel) ++kernels;
+        }
+    }
     cudaGraphExec_t exec = nullptr;
     const cudaError_t ei = cudaGraphInstantiate(&exec, g, 0);
     cudaGraphDestroy(g);
     W8A8_CUDA(ei);
-    it = m->graphs.emplace(key, exec).first;
+    it = m->graphs.emplace(key, w8a8_model::Graph{exec, kernels}).first;
   }
-  W8A8_CUDA(cudaGraphLaunch(it->second, st));
+  W8A8_CUDA(cudaGraphLaunch(it->second.exec, st));
   W8A8_CUDA(cudaMemcpyAsync(top1, m->d_top1, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice, st));
   if (logits)
     W8A8_CUDA(cudaMemcpyAsync(logits, m->d_logits, sizeof(float) * B * (size_t)m->cfg.vocab, cudaMemcpyDeviceToDevice,
                               st));
   W8A8_CUDA(cudaEventRecord(m->ev_out, st));
   W8A8_CUDA(cudaStreamWaitEvent(user, m->ev_out, 0));
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_model_decode_kernels(const w8a8_model* m, int B, int want_logits, int* kernels) {
+  W8A8_CHECK_ARG(m && kernels, W8A8_ERR_INVALID_ARG, "w8a8_model_decode_kernels: null argument");
+  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0), m->prep_version,
+                                   want_logits ? 1 : 0);
+  const auto it = m->graphs.find(key);
+  W8A8_CHECK_ARG(it != m->graphs.end(), W8A8_ERR_INVALID_ARG,
+                 "w8a8_model_decode_kernels: no decode step of B=%d under this mask yet", B);
+  *kernels = it->second.kernels + 1;  // + the position update launched beside the graph
   return W8A8_OK;
 }
 

@@ -22,6 +22,8 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __re
                                                            int8_t* __restrict__ xq,
                                                            uint16_t* __restrict__ xq_f16,
                                                            float* __restrict__ s_x) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x;
   const int nvec = K >> 3;
   const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)row * K);
@@ -121,8 +123,7 @@ w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* i
   if (M == 0) return W8A8_OK;
   const int nvec = K / 8;
   const int threads = nvec <= 4 * 128 ? 128 : 256;
-  quantize_rows_kernel<4><<<M, threads, 0, st>>>(X, K, inv_delta, xq, xq_f16, s_x);
-  W8A8_LAUNCH_CHECK();
+  W8A8_CUDA(launch_pdl(quantize_rows_kernel<4>, dim3(M), dim3(threads), 0, st, X, K, inv_delta, xq, xq_f16, s_x));
   return W8A8_OK;
 }
 

@@ -110,6 +110,7 @@ __global__ void __launch_bounds__(kThreads, Cps<NB>::value)
   const long long u1 = p.whole ? (long long)(cta + 1) * ZG / P * C : (long long)(cta + 1) * U / P;
   auto cta_of = [&](long long u) -> int { return (int)(((u + 1) * P + U - 1) / U - 1); };
 
+  pdl_trigger();
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(full + s), 1);
@@ -118,7 +119,10 @@ __global__ void __launch_bounds__(kThreads, Cps<NB>::value)
     fence_mbar_init();
   }
   __syncthreads();
-  if (u0 >= u1) return;
+  if (u0 >= u1) {
+    pdl_wait();
+    return;
+  }
 
   // ------------------------------------------------------------------------ producer thread
   if (warp == kConsumerWarps) {
@@ -127,7 +131,28 @@ __global__ void __launch_bounds__(kThreads, Cps<NB>::value)
     const uint32_t tx = (uint32_t)(nw * kBox + nx * XBOX);
     bool ok = true;
     long long it = 0;
-    for (long long u = u0; u < u1; ++u, ++it) {
+    // The weights of the first stages do not depend on the preceding kernel: request them before
+    // waiting for it, then add the token rows of X to the same stages.
+    const long long npre = (long long)S < u1 - u0 ? (long long)S : u1 - u0;
+    for (; it < npre; ++it) {
+      const long long u = u0 + it;
+      const int zg = (int)(u / C), ch = (int)(u % C);
+      const int g = zg % G;
+      const uint32_t bar = smem_u32(full + (int)it);
+      mbar_arrive_expect_tx(bar, tx);
+      for (int b = 0; b < nw; ++b)
+        tma_load_2d(ring + (uint32_t)it * SB + b * kBox, &tmW, ch * KC + b * BOXK, g * 128, bar);
+    }
+    pdl_wait();
+    for (long long j = 0; j < npre; ++j) {
+      const long long u = u0 + j;
+      const int zg = (int)(u / C), ch = (int)(u % C);
+      const int z = zg / G;
+      const uint32_t bar = smem_u32(full + (int)j);
+      for (int b = 0; b < nx; ++b)
+        tma_load_2d(ring + (uint32_t)j * SB + 2 * kBox + b * XBOX, &tmX, ch * KC + b * 64, z * TOK, bar);
+    }
+    for (long long u = u0 + npre; u < u1; ++u, ++it) {
       const int s = (int)(it % S);
       const uint32_t ph = (uint32_t)((it / S) & 1);
       if (!mbar_wait_bounded(smem_u32(empty + s), ph ^ 1u, kWaitBudgetCycles)) {
@@ -154,6 +179,7 @@ __global__ void __launch_bounds__(kThreads, Cps<NB>::value)
   }
 
   // ----------------------------------------------------------------------- consumer warps
+  pdl_wait();
   const int w = warp;
   const int gl = lane >> 2, t = lane & 3;
   const int pr = row_perm<kInt8>(gl);  // tile row (within 16) of MMA row gl; MMA row gl+8 -> pr+8
@@ -309,21 +335,45 @@ __global__ void __launch_bounds__(kThreads, Cps<NB>::value)
       named_bar_sync(1, kConsumerWarps * 32);
       if (!s_flag) return;
       __threadfence();
+      // Sum the contributors' partial tiles with RU loads in flight per value: accumulator j takes
+      // contributors f + j, f + j + RU, ... in order, then the RU accumulators are added pairwise.
+      // The order depends only on (f, l), so the fp32 result is the same on every run.
+      constexpr int RU = NB >= 8 ? 1 : 8 / NB;
+      uint32_t ra[RU][NB][4];
 #pragma unroll
-      for (int nb = 0; nb < NB; ++nb)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) v[nb][e] = 0u;
-      for (int c = f; c <= l; ++c) {
-        const uint32_t* src = slot_base(c);
+      for (int j = 0; j < RU; ++j)
 #pragma unroll
         for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const uint32_t x = __ldcg(src + (16 * w + pr + (e >> 1) * 8) * TOK + nb * 8 + 2 * t + (e & 1));
-            v[nb][e] = kInt8 ? (uint32_t)((int)v[nb][e] + (int)x)
-                             : __float_as_uint(__uint_as_float(v[nb][e]) + __uint_as_float(x));
-          }
+          for (int e = 0; e < 4; ++e) ra[j][nb][e] = 0u;
+      auto add = [](uint32_t x, uint32_t y) -> uint32_t {
+        return kInt8 ? (uint32_t)((int)x + (int)y) : __float_as_uint(__uint_as_float(x) + __uint_as_float(y));
+      };
+      for (int c0 = f; c0 <= l; c0 += RU) {
+#pragma unroll
+        for (int j = 0; j < RU; ++j) {
+          if (c0 + j > l) break;
+          const uint32_t* src = slot_base(c0 + j);
+#pragma unroll
+          for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              ra[j][nb][e] = add(ra[j][nb][e],
+                                 __ldcg(src + (16 * w + pr + (e >> 1) * 8) * TOK + nb * 8 + 2 * t + (e & 1)));
+        }
       }
+#pragma unroll
+      for (int span = 1; span < RU; span <<= 1)
+#pragma unroll
+        for (int j = 0; j + span < RU; j += 2 * span)
+#pragma unroll
+          for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) ra[j][nb][e] = add(ra[j][nb][e], ra[j + span][nb][e]);
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) v[nb][e] = ra[0][nb][e];
     }
     epilogue(z, g, v);
   };
@@ -459,8 +509,8 @@ w8a8_status launch_steps(const StreamArgs& a, cudaStream_t st) {
   CUtensorMap tw, tx;
   W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 128));
   W8A8_TRY(make_tmap_2d(&tx, a.X, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, 64, 8 * NB));
-  stream_gemm_kernel<kInt8, NB, STEPS><<<a.p.P, kThreads, a.p.smem_bytes, st>>>(tw, tx, a);
-  W8A8_LAUNCH_CHECK();
+  W8A8_CUDA(launch_pdl(stream_gemm_kernel<kInt8, NB, STEPS>, dim3(a.p.P), dim3(kThreads), a.p.smem_bytes, st, tw, tx,
+                       a));
   return W8A8_OK;
 }
 
@@ -512,6 +562,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   const long long u1 = p.whole ? (long long)(cta + 1) * G / P * C : (long long)(cta + 1) * U / P;
   auto cta_of = [&](long long u) -> int { return (int)(((u + 1) * P + U - 1) / U - 1); };
 
+  pdl_trigger();
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(full + s), 1);
@@ -519,21 +570,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     fence_mbar_init();
   }
-  // activation codes -> shared memory (tokens >= M and the tail past K are zero)
-  {
-    const int8_t* X = reinterpret_cast<const int8_t*>(a.X);
-    uint8_t* xsp = smem_raw + (xs - raw_u32);
-    for (uint32_t i = threadIdx.x; i < xbytes / 16; i += blockDim.x) {
-      const uint32_t byte = i * 16;
-      const int m = (int)(byte / (uint32_t)a.K), k = (int)(byte % (uint32_t)a.K);
-      uint4 v = make_uint4(0, 0, 0, 0);
-      if (m < a.M) v = *reinterpret_cast<const uint4*>(X + (size_t)m * a.K + k);
-      *reinterpret_cast<uint4*>(xsp + byte) = v;
-    }
-  }
   __syncthreads();
-  if (u0 >= u1) return;
+  if (u0 >= u1) {
+    pdl_wait();
+    return;
+  }
 
+  // The producer streams weights only (independent of the preceding kernel) and starts at once;
+  // the consumers wait for the preceding kernel, then stage the activation codes.
   if (warp == kConsumerWarps) {  // ---------------------------------------------- producer thread
     if (lane != 0) return;
     constexpr int nw = KC / 128;
@@ -562,6 +606,19 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 
   // ------------------------------------------------------------------------ consumer warps
+  pdl_wait();
+  {  // activation codes -> shared memory (tokens >= M and the tail past K are zero)
+    const int8_t* X = reinterpret_cast<const int8_t*>(a.X);
+    uint8_t* xsp = smem_raw + (xs - raw_u32);
+    for (uint32_t i = threadIdx.x; i < xbytes / 16; i += kConsumerWarps * 32) {
+      const uint32_t byte = i * 16;
+      const int m = (int)(byte / (uint32_t)a.K), k = (int)(byte % (uint32_t)a.K);
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (m < a.M) v = *reinterpret_cast<const uint4*>(X + (size_t)m * a.K + k);
+      *reinterpret_cast<uint4*>(xsp + byte) = v;
+    }
+  }
+  named_bar_sync(1, kConsumerWarps * 32);
   const int w = warp, rl = lane & 7, cq = lane >> 3;
   const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
   int acc[2][MT];
@@ -665,19 +722,36 @@ __global__ void __launch_bounds__(kThreads, 2)
       named_bar_sync(1, kConsumerWarps * 32);
       if (!s_flag) return;
       __threadfence();
-      if (lane < 8) {
+      // All 32 lanes sum: lane rl + 8 cq takes contributors f + cq, f + cq + 4, ..., four at a time
+      // (16 loads in flight per lane), then the four lane groups are added (INT32: any order).
 #pragma unroll
-        for (int q = 0; q < 2; ++q)
+      for (int q = 0; q < 2; ++q)
 #pragma unroll
-          for (int m = 0; m < MT; ++m) v[q][m] = 0;
-        for (int c = f; c <= l; ++c) {
-          const int* src = slot_base(c);
+        for (int m = 0; m < MT; ++m) v[q][m] = 0;
+      for (int c0 = f + cq; c0 <= l; c0 += 16) {
+        int x[4][2][MT];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int c = c0 + 4 * j;
 #pragma unroll
           for (int q = 0; q < 2; ++q)
 #pragma unroll
-            for (int m = 0; m < MT; ++m) v[q][m] += __ldcg(src + (16 * w + rl + 8 * q) * MT + m);
+            for (int m = 0; m < MT; ++m) x[j][q][m] = c <= l ? __ldcg(slot_base(c) + (16 * w + rl + 8 * q) * MT + m) : 0;
         }
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+          for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int m = 0; m < MT; ++m) v[q][m] += x[j][q][m];
       }
+#pragma unroll
+      for (int q = 0; q < 2; ++q)
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+          v[q][m] += __shfl_xor_sync(0xffffffffu, v[q][m], 8);
+          v[q][m] += __shfl_xor_sync(0xffffffffu, v[q][m], 16);
+        }
     }
     epilogue(g, v);
   };
@@ -758,8 +832,7 @@ w8a8_status launch_dp4a(const StreamArgs& a, cudaStream_t st) {
   }
   CUtensorMap tw;
   W8A8_TRY(make_tmap_2d(&tw, a.W, 1, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K, 128, 128));
-  gemv_dp4a_kernel<MT, NCH><<<a.p.P, kThreads, a.p.smem_bytes, st>>>(tw, a);
-  W8A8_LAUNCH_CHECK();
+  W8A8_CUDA(launch_pdl(gemv_dp4a_kernel<MT, NCH>, dim3(a.p.P), dim3(kThreads), a.p.smem_bytes, st, tw, a));
   return W8A8_OK;
 }
 
@@ -826,12 +899,19 @@ void set_kernel_events(void* start, void* stop) {
   g_ev_stop = reinterpret_cast<cudaEvent_t>(stop);
 }
 
+void take_kernel_events(void** start, void** stop) {
+  *start = g_ev_start;
+  *stop = g_ev_stop;
+  g_ev_start = g_ev_stop = nullptr;
+}
+
 static w8a8_status dispatch_stream_gemm(bool int8_weights, const StreamArgs& a, cudaStream_t st);
 
 w8a8_status launch_stream_gemm(bool int8_weights, const StreamArgs& a, cudaStream_t st) {
   if (a.M == 0 || a.N == 0) return W8A8_OK;
-  cudaEvent_t e0 = g_ev_start, e1 = g_ev_stop;
-  g_ev_start = g_ev_stop = nullptr;
+  void *v0, *v1;
+  take_kernel_events(&v0, &v1);
+  cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
   const w8a8_status s = dispatch_stream_gemm(int8_weights, a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));

@@ -51,6 +51,7 @@ StreamPlan make_stream_plan(bool int8_weights, int M, int N, int K, int sm_count
 void attach_reserved(StreamArgs& a, void* ws);  // counters, top-1 keys and error word in the reserved region
 int max_top_keys();
 void set_kernel_events(void* start, void* stop);  // next launch on this thread records them around the kernel
+void take_kernel_events(void** start, void** stop);  // the pending pair (or nulls), cleared
 w8a8_status launch_stream_gemm(bool int8_weights, const StreamArgs& a, cudaStream_t st);
 
 }  // namespace w8a8

@@ -45,3 +45,10 @@ def test_library_rule_matches_oracle_on_random_sets(B):
         want = allocator.choose(cands, min_top1=float(np.float32(0.989)), max_ppl_delta=float(np.float32(0.01)))
         got = B.choose_mask(lat.tolist(), t1.tolist(), pd.tolist(), n8.tolist(), 0.989, 0.01)
         assert got == (-1 if want is None else want), trial
+
+
+def test_library_candidate_masks_equal_paper_groups(B):
+    ours = B.candidate_masks()
+    ref = list(masks.candidate_masks().items())
+    assert [n for n, _ in ours] == [n for n, _ in ref]
+    assert [bits for _, bits in ours] == [m.bits() for _, m in ref]

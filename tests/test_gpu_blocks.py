@@ -43,7 +43,7 @@ def ffn(B):
     return c, f, prep
 
 
-@pytest.mark.parametrize("M", [1, 8, 13, 64])
+@pytest.mark.parametrize("M", [1, 3, 8, 13, 64])
 def test_ffn_w8a8_bit_exact(B, ffn, M):
     c, f, prep = ffn
     x = c["x"][:M]
@@ -53,7 +53,7 @@ def test_ffn_w8a8_bit_exact(B, ffn, M):
     assert np.array_equal(f32_of_bf16(Y), r["y"])
 
 
-@pytest.mark.parametrize("M", [1, 8, 64])
+@pytest.mark.parametrize("M", [1, 5, 8, 64])
 def test_ffn_bf16_within_tolerance(B, ffn, M):
     c, f, _ = ffn
     Y, h = B.ffn_block(f, B.W8A8_PREC_BF16, cu(c["x"][:M]), want_h=True)

@@ -141,6 +141,26 @@ def test_decode_step_graph_equals_eager_forward(B, setup):
     assert torch.equal(lg3, lg) and torch.equal(t3, t1)
 
 
+def test_decode_kernel_count(B, setup):
+    """A decode step launches the position update, embedding + norm, per layer q/k/v, attention
+    (QK-norm, RoPE and the cache write fused in), o, residual + norms, gate/up + GeGLU, down,
+    residual + norms, then lm_head.
+    At decode the W8A8 linears of the layers fuse their per-token quantiser into the GEMV, so a
+    W8A8 FFN or attention block costs no extra launch; W8A8 lm_head adds its quantiser."""
+    dec, _, toks = setup[:3]
+    col = torch.from_numpy(toks[:, 21].copy()).cuda()
+    buf = torch.empty(2, V, dtype=torch.float32, device="cuda")
+    counts = {}
+    for m in [(0, 0, 0), (0b1001, 0b0010, 1)]:
+        dec.set_mask(*m)
+        with pytest.raises(B.W8A8Error):
+            dec.decode_kernels(2, want_logits=False)  # no graph of this (B, mask) without logits yet
+        dec.decode_step(col, 21, logits=buf)
+        counts[m] = dec.decode_kernels(2, want_logits=True)
+    assert counts[(0, 0, 0)] == 2 + 7 * L + 1
+    assert counts[(0b1001, 0b0010, 1)] - counts[(0, 0, 0)] == 1
+
+
 def test_mask_controls(B, setup):
     dec = setup[0]
     dec.set_mask(0, 0, 0)

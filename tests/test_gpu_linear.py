@@ -123,6 +123,11 @@ LINEAR_SHAPES = [
     (33, 520, 1152),
     (64, 1152, 6912),   # down_proj shape
     (130, 300, 256),    # several token groups with a ragged tail
+    (5, 1536, 1152),    # row-owning decode GEMV, 8 token slots (qkv shape)
+    (8, 1152, 6912),    # row-owning decode GEMV, K past one stage ring (down_proj shape)
+    (4, 1152, 1024),    # o_proj shape
+    (7, 9, 16),         # fewer rows than one CTA's eight, K of one vector
+    (2, 64, 9216),      # K too long for the fused quantiser: K1 + streaming kernel
 ]
 
 
@@ -189,7 +194,8 @@ def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarr
     assert np.all(np.abs(y_gpu.astype(np.float64) - y_ref) <= bound)
 
 
-@pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040)])
+@pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040),
+                                   (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152)])
 def test_bf16_linear_within_tolerance(B, M, N, K):
     x32, x, w32, w, _, _ = _case(M, N, K, seed=11 + M)
     Y = B.linear_bf16(cu(w), cu(x))
