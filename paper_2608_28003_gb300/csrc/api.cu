@@ -5,6 +5,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "gemm_tc.cuh"
 #include "gemv_small.cuh"
 #include "ops.cuh"
 #include "stream_gemm.cuh"
@@ -133,6 +134,52 @@ static bool small_gemv(bool int8, const void* W, const float* inv_delta, const f
   return true;
 }
 
+// Calls with more tokens than the decode GEMV takes go to the tensor-core GEMM when its shape
+// rules hold (W8A8: the weights' fp16 code copy must exist); false leaves them to the streaming
+// kernel.
+constexpr int kTcMinTokens = 64;
+
+static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N, int K, const float* bias, int kind,
+                    const float* inv_delta, const float* s_w, uint16_t* Y, float* logits, int32_t* top1,
+                    const w8a8_debug* dbg, void* ws, void* codes, float* s_x, cudaStream_t st, w8a8_status* status) {
+  if (M < kTcMinTokens || !W16 || !tc_gemm_supported(M, N, K, kind, top1 != nullptr, max_top_keys())) return false;
+  TcArgs a{};
+  if (int8) {
+    w8a8_status q = launch_quantize_rows(X, M, K, inv_delta, dbg ? dbg->xq : nullptr,
+                                         reinterpret_cast<uint16_t*>(codes), s_x, st);
+    if (q == W8A8_OK && dbg && dbg->s_x)
+      q = cudaMemcpyAsync(dbg->s_x, s_x, sizeof(float) * M, cudaMemcpyDeviceToDevice, st) == cudaSuccess
+              ? W8A8_OK
+              : W8A8_ERR_CUDA;
+    if (q != W8A8_OK) {
+      *status = q;
+      return true;
+    }
+    a.A = codes;
+    a.s_x = s_x;
+    a.s_w = s_w;
+    a.acc_dbg = dbg ? dbg->acc : nullptr;
+  } else {
+    a.A = X;
+  }
+  a.B = W16;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.kind = kind;
+  a.bias = bias;
+  a.y = Y;
+  a.logits = logits;
+  a.top1 = top1;
+  StreamArgs r{};
+  attach_reserved(r, ws);
+  a.grid_counter = r.grid_counter;
+  a.top_keys = r.top_keys;
+  a.err = r.err;
+  *status = launch_tc_gemm(int8, a, st);
+  return true;
+}
+
 // One W8A8 linear: K1 then the streaming GEMM.  s_x and the codes live in the workspace.
 w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
                                    uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
@@ -147,6 +194,9 @@ w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, con
   char* base = reinterpret_cast<char*>(ws);
   void* codes = base + L.xf16;
   float* s_x = reinterpret_cast<float*>(base + L.sx);
+  if (tc_path(true, w->wq_f16, X, M, N, K, bias, kind, w->inv_delta, w->s_w, Y, logits, top1, dbg, ws, codes, s_x, st,
+              &small_status))
+    return small_status;
   StreamArgs a{};
   a.p = make_stream_plan(true, M, N, K, sms);
   W8A8_TRY(quantize_for(a.p, X, M, K, w->inv_delta, codes, dbg ? dbg->xq : nullptr, s_x, st));
@@ -176,6 +226,9 @@ w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, 
   if (!logits && !top1 &&
       small_gemv(false, W, nullptr, nullptr, X, M, N, K, bias, kind, Y, nullptr, ws, pf ? pf->ptr : nullptr,
                  pf ? pf->bytes : 0, sms, st, &small_status))
+    return small_status;
+  if (tc_path(false, W, X, M, N, K, bias, kind, nullptr, nullptr, Y, logits, top1, nullptr, ws, nullptr, nullptr, st,
+              &small_status))
     return small_status;
   LinearWs L = linear_ws(M, N, K, false, sms);
   StreamArgs a{};
@@ -331,6 +384,12 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     if (small_gemv(true, f->gate_up.wq, f->gate_up.inv_delta, f->gate_up.s_w, X, M, 2 * F, H, nullptr, EPI_GEGLU, h,
                    nullptr, workspace, pgu, bgu, sms, st, &ss)) {
       W8A8_TRY(ss);
+    } else if (tc_path(true, f->gate_up.wq_f16, X, M, 2 * F, H, nullptr, EPI_GEGLU, f->gate_up.inv_delta,
+                       f->gate_up.s_w, h, nullptr, nullptr, nullptr, workspace,
+                       base + L.gu + (linear_ws(M, 2 * F, H, true, sms).xf16 - W8A8_WS_RESERVED),
+                       reinterpret_cast<float*>(base + L.gu + (linear_ws(M, 2 * F, H, true, sms).sx - W8A8_WS_RESERVED)),
+                       st, &ss)) {
+      W8A8_TRY(ss);
     } else {
       const LinearWs A = linear_ws(M, 2 * F, H, true, sms);
       void* codes = base + L.gu + (A.xf16 - W8A8_WS_RESERVED);
@@ -353,6 +412,12 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     }
     if (small_gemv(true, f->down.wq, f->down.inv_delta, f->down.s_w, h, M, H, F, nullptr, EPI_BF16, Y, nullptr,
                    workspace, pdn, bdn, sms, st, &ss)) {
+      W8A8_TRY(ss);
+    } else if (tc_path(true, f->down.wq_f16, h, M, H, F, nullptr, EPI_BF16, f->down.inv_delta, f->down.s_w, Y,
+                       nullptr, nullptr, nullptr, workspace,
+                       base + L.dn + (linear_ws(M, H, F, true, sms).xf16 - W8A8_WS_RESERVED),
+                       reinterpret_cast<float*>(base + L.dn + (linear_ws(M, H, F, true, sms).sx - W8A8_WS_RESERVED)), st,
+                       &ss)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs B = linear_ws(M, H, F, true, sms);
@@ -379,6 +444,9 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     if (small_gemv(false, f->gate_up_bf16, nullptr, nullptr, X, M, 2 * F, H, nullptr, EPI_GEGLU, h, nullptr,
                    workspace, pgu, bgu, sms, st, &ss)) {
       W8A8_TRY(ss);
+    } else if (tc_path(false, f->gate_up_bf16, X, M, 2 * F, H, nullptr, EPI_GEGLU, nullptr, nullptr, h, nullptr,
+                       nullptr, nullptr, workspace, nullptr, nullptr, st, &ss)) {
+      W8A8_TRY(ss);
     } else {
       const LinearWs A = linear_ws(M, 2 * F, H, false, sms);
       StreamArgs a{};
@@ -396,6 +464,9 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     }
     if (small_gemv(false, f->down_bf16, nullptr, nullptr, h, M, H, F, nullptr, EPI_BF16, Y, nullptr, workspace,
                    pdn, bdn, sms, st, &ss)) {
+      W8A8_TRY(ss);
+    } else if (tc_path(false, f->down_bf16, h, M, H, F, nullptr, EPI_BF16, nullptr, nullptr, Y, nullptr, nullptr,
+                       nullptr, workspace, nullptr, nullptr, st, &ss)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs B = linear_ws(M, H, F, false, sms);

@@ -1,0 +1,31 @@
+// Tensor-core GEMM for prefill-sized token counts on the 5th-generation tensor cores (tcgen05):
+// the W8A8 path (INT8 codes carried as fp16, exact) and the bf16 pass-through.
+#pragma once
+
+#include "common.cuh"
+
+namespace w8a8 {
+
+struct TcArgs {
+  const void* A;        // [M, K] activations: fp16 INT8 codes (W8A8) or bf16, row-major
+  const void* B;        // [N, K] weights: fp16 INT8 codes (W8A8) or bf16, row = output channel
+  int M, N, K;
+  int kind;             // EPI_BF16, EPI_GEGLU or EPI_F32
+  const float* s_x;     // [M] W8A8: per-token scales
+  const float* s_w;     // [N] W8A8: per-channel scales
+  const float* bias;    // [N] nullable
+  uint16_t* y;          // bf16 [M, N] (EPI_BF16) or [M, N / 2] (EPI_GEGLU)
+  float* logits;        // [M, N] nullable (EPI_F32)
+  int32_t* top1;        // [M] nullable (EPI_F32)
+  int32_t* acc_dbg;     // [M, N] nullable (W8A8): the INT32 sums
+  unsigned int* grid_counter;     // top-1: one counter, zero between calls
+  unsigned long long* top_keys;   // top-1: [M] keys, zero between calls
+  unsigned int* err;              // device error word
+};
+
+// Shapes the tensor-core GEMM takes: K a multiple of 16, N a multiple of 16, top-1 for at most
+// max_top rows.
+bool tc_gemm_supported(int M, int N, int K, int kind, bool want_top, int max_top);
+w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st);
+
+}  // namespace w8a8

@@ -18,6 +18,7 @@ namespace {
 
 struct QW {
   int8_t* wq = nullptr;
+  uint16_t* wq_f16 = nullptr;  // the same codes as fp16, for the tensor-core GEMM of prefill
   float* s_w = nullptr;
   float* delta = nullptr;
   float* inv_delta = nullptr;
@@ -104,7 +105,7 @@ void free_all(w8a8_model* m) {
   if (m->st) cudaStreamDestroy(m->st);
 }
 
-w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, nullptr}; }
+w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, q.wq_f16}; }
 
 w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
                    uint16_t* Y, cudaStream_t st, const L2Prefetch* pf) {
@@ -387,6 +388,7 @@ extern "C" w8a8_status w8a8_model_prepare(w8a8_model* m, float alpha, int smooth
   auto ensure = [&](QW& q, int n, int k) -> w8a8_status {
     if (q.wq) return W8A8_OK;
     W8A8_TRY(dalloc(m, &q.wq, (size_t)n * k));
+    W8A8_TRY(dalloc(m, &q.wq_f16, (size_t)n * k));
     W8A8_TRY(dalloc(m, &q.s_w, (size_t)n));
     W8A8_TRY(dalloc(m, &q.delta, (size_t)k));
     W8A8_TRY(dalloc(m, &q.inv_delta, (size_t)k));
@@ -403,19 +405,19 @@ extern "C" w8a8_status w8a8_model_prepare(w8a8_model* m, float alpha, int smooth
     const w8a8_layer_bf16& W = m->L[l];
     QW* q = &m->q_qkv[l];
     W8A8_TRY(w8a8_prepare_weights(W.wqkv, m->qkv_dim, H, m->stat_qkv(l), alpha, smooth, q->wq, q->s_w, q->delta,
-                                  q->inv_delta, nullptr, stream));
+                                  q->inv_delta, q->wq_f16, stream));
     q = &m->q_o[l];
     W8A8_TRY(w8a8_prepare_weights(W.wo, H, m->q_dim, m->stat_o(l), alpha, smooth, q->wq, q->s_w, q->delta,
-                                  q->inv_delta, nullptr, stream));
+                                  q->inv_delta, q->wq_f16, stream));
     q = &m->q_gu[l];
     W8A8_TRY(w8a8_prepare_gate_up(W.wgate, W.wup, F, H, m->stat_gu(l), alpha, smooth, q->wq, q->s_w, q->delta,
-                                  q->inv_delta, nullptr, stream));
+                                  q->inv_delta, q->wq_f16, stream));
     q = &m->q_down[l];
     W8A8_TRY(w8a8_prepare_weights(W.wdown, H, F, m->stat_down(l), alpha, smooth, q->wq, q->s_w, q->delta,
-                                  q->inv_delta, nullptr, stream));
+                                  q->inv_delta, q->wq_f16, stream));
   }
   W8A8_TRY(w8a8_prepare_weights(m->embed, c.vocab, H, m->stat_lm(), alpha, smooth, m->q_lm.wq, m->q_lm.s_w,
-                                m->q_lm.delta, m->q_lm.inv_delta, nullptr, stream));
+                                m->q_lm.delta, m->q_lm.inv_delta, m->q_lm.wq_f16, stream));
   m->prepared = true;
   ++m->prep_version;
   return W8A8_OK;

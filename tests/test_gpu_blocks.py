@@ -36,8 +36,9 @@ def f32_of_bf16(t):
 def ffn(B):
     c = synth.ffn_case(64, seed=0)
     stat_in = OW.act_absmax(c["calib32"])
-    gu = B.prepare_gate_up(cu(c["wg"]), cu(c["wu"]), cu(torch.from_numpy(stat_in)))
-    dn = B.prepare_weights(cu(c["wd"]), cu(torch.from_numpy(c["stat_h"])))
+    # fp16 code copies too: 64 tokens take the tensor-core GEMM
+    gu = B.prepare_gate_up(cu(c["wg"]), cu(c["wu"]), cu(torch.from_numpy(stat_in)), want_f16=True)
+    dn = B.prepare_weights(cu(c["wd"]), cu(torch.from_numpy(c["stat_h"])), want_f16=True)
     f = B.FfnWeights(1152, 6912, gu, dn, B.interleave_gate_up(cu(c["wg"]), cu(c["wu"])), cu(c["wd"]))
     prep = OB.prepare_ffn(c["wg32"], c["wu32"], c["wd32"], stat_in, c["stat_h"])
     return c, f, prep
@@ -122,6 +123,43 @@ def test_lm_head_bf16_within_tolerance(B, head, M):
     clear = (srt[:, -1] - srt[:, -2]) > 2 * bound.max(axis=1)
     t = top1.cpu().numpy()
     assert np.array_equal(t[clear], r["top1"][clear])
+    assert np.all(lg[np.arange(M), t] == lg.max(axis=1))
+
+
+@pytest.fixture(scope="module")
+def head16(B, head):
+    """The same lm_head with the fp16 copy of the codes (the tensor-core GEMM's operand)."""
+    c, hd, prep = head
+    q = hd.q
+    q16 = B.prepare_weights(cu(c["w"]), q.delta.new_tensor(OW.act_absmax(c["calib32"])), want_f16=True)
+    assert torch.equal(q16.wq, q.wq)
+    return c, B.HeadWeights(262144, 1152, q16, hd.bf16), prep
+
+
+@pytest.mark.parametrize("M", [128, 512])
+def test_lm_head_w8a8_tensor_core_sampled(B, head16, M):
+    c, hd, prep = head16
+    x32, x = synth.normed_rows(M, 1152, seed=M + 7)
+    logits, top1 = B.lm_head(hd, B.W8A8_PREC_W8A8, cu(x))
+    idx = np.array([0, 1, 77, M // 2, M - 1])
+    r = OB.lm_head_w8a8(x32[idx], prep)
+    assert np.array_equal(logits.cpu().numpy()[idx].view(np.uint32), r["logits"].view(np.uint32))
+    assert np.array_equal(top1.cpu().numpy()[idx], r["top1"])
+    lg = logits.cpu().numpy()
+    assert np.array_equal(top1.cpu().numpy(), np.argmax(lg, axis=1))
+
+
+def test_lm_head_bf16_tensor_core_sampled(B, head):
+    c, hd, _ = head
+    M = 128
+    x32, x = synth.normed_rows(M, 1152, seed=3)
+    logits, top1 = B.lm_head(hd, B.W8A8_PREC_BF16, cu(x))
+    idx = np.array([0, 5, 64, 127])
+    r = OB.lm_head_bf16(x32[idx], c["w32"])
+    mag = np.abs(x32[idx]).astype(np.float64) @ np.abs(c["w32"]).astype(np.float64).T
+    lg = logits.cpu().numpy()
+    assert np.all(np.abs(lg[idx] - r["logits"]) <= 1152 * 2.0 ** -24 * mag + 1e-30)
+    t = top1.cpu().numpy()
     assert np.all(lg[np.arange(M), t] == lg.max(axis=1))
 
 

@@ -148,6 +148,29 @@ def test_w8a8_linear_bit_exact(B, M, N, K):
     assert np.array_equal(f32_of_bf16(Y), r["y"])
 
 
+TC_SHAPES = [
+    (64, 1152, 6912),    # seven 1024-k chunks folded into INT32
+    (130, 4112, 1040),   # ragged M, K not a multiple of the 64-wide stage
+    (256, 1536, 1152),
+    (200, 13824, 1152),  # gate/up shape, ragged M
+]
+
+
+@pytest.mark.parametrize("M,N,K", TC_SHAPES)
+def test_w8a8_linear_tensor_core_bit_exact(B, M, N, K):
+    """Prefill-sized calls with the fp16 code copy take the tcgen05 GEMM: codes, scales and INT32
+    sums bit for bit, bf16 outputs bit for bit."""
+    x32, x, w32, w, c32, c = _case(M, N, K, seed=M * 3 + K)
+    stat = OW.act_absmax(np.concatenate([c32, x32]))
+    q = B.prepare_weights(cu(w), cu(torch.from_numpy(stat)), want_f16=True)
+    Y, dbg = B.linear(q, cu(x), debug=True)
+    r = OW.w8a8_linear(x32, OW.prepare_weights(w32, stat), out="bf16")
+    assert np.array_equal(dbg["xq"].cpu().numpy(), r["xq"])
+    assert np.array_equal(dbg["s_x"].cpu().numpy(), r["s_x"])
+    assert np.array_equal(dbg["acc"].cpu().numpy().astype(np.int64), r["acc"])
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+
+
 def test_single_linear_workload_calibrated_on_its_input(B):
     """M = 16, K = 1152, N = 6912, 8 outlier channels x20, delta from X itself (seed 0)."""
     c = synth.linear_case()
@@ -195,7 +218,8 @@ def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarr
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040),
-                                   (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152)])
+                                   (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152),
+                                   (128, 6912, 1152), (70, 1152, 6912), (300, 256, 64)])
 def test_bf16_linear_within_tolerance(B, M, N, K):
     x32, x, w32, w, _, _ = _case(M, N, K, seed=11 + M)
     Y = B.linear_bf16(cu(w), cu(x))
