@@ -21,7 +21,8 @@ The same line carries:
   * ``kernels``: per-call time, TOPS and algorithmic GB/s of the single W8A8 linear (M = 16,
     1152 -> 6912), the FFN block (M in 1, 8, 64, 512, 2048) and lm_head (M in 1, 16, 128, 512),
     W8A8 and bf16 (L2 flushed before each call);
-  * ``roofline`` of the decode step's largest kernel against the measured HBM copy bandwidth;
+  * ``roofline`` of the decode step's dominant kernel (the row-owning GEMV on bf16 weights, by
+    share of device time) against the measured HBM copy bandwidth, with the lm_head GEMV beside it;
   * ``e2e``: decode through the public API with the token copied in from pinned host memory
     and the top-1 copied back every step (host wall clock);
   * ``cpu_baseline``: the oracle on this host's cores for a bounded sample of the same decode.
@@ -333,19 +334,50 @@ def run_ours(args, dist: Dist):
             e2e.append((time.perf_counter() - t0) * 1e3)
     e2e_ms = whole_job_ms_per_token(dist.max(sum(e2e)), K, dist.world)
 
-    # ---- roofline: the decode step's largest kernel (lm_head W8A8 GEMV, M = 1), same launch
-    # configuration, timed alone with events around the kernel, L2 flushed before each launch
+    # ---- roofline: the decode step's dominant kernel by share of device time (the ncu launch list),
+    # the row-owning decode GEMV on bf16 weights at one token: per step 26 q/k/v (1152 -> 1536),
+    # 26 o (1024 -> 1152) and 16 down (6912 -> 1152, the bf16 FFN layers of the mask).  Each shape
+    # is launched as in the decode step, timed alone with events around the kernel, L2 flushed
+    # before each launch; achieved = the mix's algorithmic bytes / its kernel time.
     flush_buf = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     flush = lambda: flush_buf.zero_()  # noqa: E731  (512 MiB > 129 MB L2)
+    ws = B.Workspace(dev)
+    mix = [("qkv", 26, wdev["wqkv"][5], 1536, HIDDEN), ("o", 26, wdev["wo"][5], HIDDEN, 1024),
+           ("down", 16, wdev["wd"][5], HIDDEN, INTER)]
+    parts, tot_bytes, tot_us = {}, 0.0, 0.0
+    for name, count, wmat, N, Kd in mix:
+        xin = torch.from_numpy(synth.activations(1, Kd, 8, seed=N)[0]).to(torch.bfloat16).to(dev)
+        yout = torch.empty(1, N, dtype=torch.bfloat16, device=dev)
+        timed_steps(lambda: B.linear_bf16(wmat, xin, out=yout, ws=ws), max(K, 20), 3, flush, stream,
+                    kernel_events=B.set_kernel_events)
+        us = statistics.mean(timed_steps.kernel_ms) * 1e3
+        nbytes = bf16_bytes(1, N, Kd)
+        parts[name] = {"launches_per_step": count, "kernel_us": round(us, 2), "bytes": nbytes,
+                       "GBps": round(nbytes / (us * 1e-6) / 1e9, 1)}
+        tot_bytes += count * nbytes
+        tot_us += count * us
+    achieved = tot_bytes / (tot_us * 1e-6) / 1e9
+    # DRAM bytes read + written per launch of the same mix from one ncu capture of this kernel inside
+    # the decode step (q/k/v 3,564,544 + o 2,384,128 + down 15,961,856 bytes, weighted 26 : 26 : 16)
+    traffic = (26 * 3564544 + 26 * 2384128 + 16 * 15961856) / 68
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": round(traffic),
+                "peak_source": peaks["source"],
+                "kernel": "gemv_small_kernel<bf16, 1 token, 1 row/warp> (decode row-owning GEMV)",
+                "kernel_us": round(tot_us / 68, 2), "algorithmic_bytes_per_launch": round(tot_bytes / 68),
+                "launch_mix": parts,
+                "timing": "CUDA events around the kernel on its stream, launches as in the decode step, "
+                          "L2 flushed before each launch; per-launch figures are the mix's averages"}
+
+    # the lm_head GEMV (W8A8, one token) on the same terms, for comparison
     stats = torch.from_numpy(dec.get_stats()).to(dev)
     lm_stat = stats[-HIDDEN:].contiguous()
-    q_lm = B.prepare_weights(wdev["embed"], lm_stat)
+    q_lm = B.prepare_weights(wdev["embed"], lm_stat, want_f16=True)
     head = B.HeadWeights(VOCAB, HIDDEN, q_lm, wdev["embed"])
     _, xh = synth.normed_rows(512, HIDDEN, seed=0)
     xh = xh.to(dev)
     logits = torch.empty(512, VOCAB, dtype=torch.float32, device=dev)
     top1 = torch.empty(512 * 4, dtype=torch.int32, device=dev)  # slot i at 16 * i bytes (16-byte aligned)
-    ws = B.Workspace(dev)
     ctr = [0]
 
     def head_call():
@@ -356,13 +388,10 @@ def run_ours(args, dist: Dist):
     timed_steps(head_call, max(K, 20), 3, flush, stream, kernel_events=B.set_kernel_events)
     kernel_ms = statistics.mean(timed_steps.kernel_ms)
     hb = w8a8_bytes(1, VOCAB, HIDDEN, out_bytes=4)
-    achieved = hb / (kernel_ms * 1e-3) / 1e9
-    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None, "peak_source": peaks["source"],
-                "kernel": "gemv_dp4a_kernel<1,16> (lm_head W8A8 GEMV, M=1, 1152 -> 262144)",
-                "kernel_us": round(kernel_ms * 1e3, 2), "algorithmic_bytes_per_launch": hb,
-                "timing": "CUDA events around the kernel on its stream, same launch as in the decode step, "
-                          "L2 flushed before each launch"}
+    roofline["lm_head_gemv"] = {"kernel": "gemv_dp4a_kernel<1,16> (lm_head W8A8, M=1, 1152 -> 262144)",
+                                "kernel_us": round(kernel_ms * 1e3, 2), "bytes": hb,
+                                "GBps": round(hb / (kernel_ms * 1e-3) / 1e9, 1),
+                                "frac": round(hb / (kernel_ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4)}
 
     out = {"ms": ms, "total_ms": total_ms, "per_step": per_step, "clocks": clk, "roofline": roofline,
            "launches": kernels_per_step * K, "kernels_per_step": kernels_per_step,
@@ -460,7 +489,7 @@ def sweep(B, dev, head, xh, flush, stream, peaks):
 
     ws = B.Workspace(dev)
     c = synth.linear_case()
-    q = B.prepare_weights(c["w"].to(dev), B.act_absmax(c["calib"].to(dev)))
+    q = B.prepare_weights(c["w"].to(dev), B.act_absmax(c["calib"].to(dev)), want_f16=True)
     x = c["x"].to(dev)
     w = c["w"].to(dev)
     y = torch.empty(16, INTER, dtype=torch.bfloat16, device=dev)
@@ -469,8 +498,8 @@ def sweep(B, dev, head, xh, flush, stream, peaks):
     t = statistics.mean(timed_steps(lambda: B.linear_bf16(w, x, out=y, ws=ws), 10, 3, flush, stream, kev))
     rec("linear_bf16_M16", t, 2 * 16 * INTER * HIDDEN, bf16_bytes(16, INTER, HIDDEN), True)
     fc = synth.ffn_case(2048, seed=0)
-    gu = B.prepare_gate_up(fc["wg"].to(dev), fc["wu"].to(dev), B.act_absmax(fc["calib"].to(dev)))
-    dn = B.prepare_weights(fc["wd"].to(dev), torch.from_numpy(fc["stat_h"]).to(dev))
+    gu = B.prepare_gate_up(fc["wg"].to(dev), fc["wu"].to(dev), B.act_absmax(fc["calib"].to(dev)), want_f16=True)
+    dn = B.prepare_weights(fc["wd"].to(dev), torch.from_numpy(fc["stat_h"]).to(dev), want_f16=True)
     f = B.FfnWeights(HIDDEN, INTER, gu, dn, B.interleave_gate_up(fc["wg"].to(dev), fc["wu"].to(dev)), fc["wd"].to(dev))
     xf = fc["x"].to(dev)
     yf = torch.empty(2048, HIDDEN, dtype=torch.bfloat16, device=dev)

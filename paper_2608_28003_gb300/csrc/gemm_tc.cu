@@ -1,17 +1,21 @@
 // Tensor-core GEMM (tcgen05, TMEM accumulators, TMA) for prefill-sized token counts.
 //
-// D[128 tokens x BN channels] of one CTA lives in tensor memory; A (tokens x K) and B (channels x
-// K) tiles of 64 k arrive by 2-D TMA into 128-byte-swizzled shared memory, S stages deep.
+// A persistent grid (one CTA per SM) walks the output tiles of 128 tokens x BN channels.  A
+// (tokens x K) and B (channels x K) tiles of 64 k arrive by 2-D TMA into 128-byte-swizzled shared
+// memory, S stages deep, continuously across tiles.  Accumulators live in tensor memory (all 512
+// columns), as a ring of BN-column slots, so the epilogue of one tile overlaps the MMAs of the next.
 //  * warp 4 (one thread) issues the TMA copies; warp 5 allocates tensor memory and one of its
-//    threads issues tcgen05.mma (M = 128, N = BN, K = 16, fp32 accumulation) for each stage and
-//    commits the stage back to the producer; warps 0-3 are the epilogue, warp w reading TMEM lanes
-//    32w .. 32w+31 (its tokens) with tcgen05.ld.
-//  * W8A8 path: both operands are INT8 codes stored as fp16 (exact).  Every product is an integer
-//    below 2^14, so a fp32 sum of at most 1024 of them is exact; the accumulator is therefore
-//    restarted every 1024 k (16 stages) in one of two TMEM buffers while the epilogue warps fold the
-//    other into INT32 registers, and the INT32 result is exact in any order (Eq. gemm-final).  The
-//    epilogue then dequantises fl(fl(s_x s_w) acc) (+ bias).
-//  * bf16 path: one accumulator over the whole k range, N = 256.
+//    threads issues tcgen05.mma (M = 128, N = BN, K = 16, fp32 accumulation) for each stage,
+//    commits the stage back to the producer and each finished slot to the epilogue; warps 0-3 are
+//    the epilogue, warp w reading TMEM lanes 32w .. 32w+31 (its tokens) with tcgen05.ld and
+//    handing the slot back.
+//  * W8A8 path (BN = 128, four slots): both operands are INT8 codes stored as fp16 (exact).  Every
+//    product is an integer below 2^14, so a fp32 sum of at most 1024 of them is exact; the
+//    accumulator is therefore restarted every 1024 k (16 stages) in the next slot while the
+//    epilogue folds the finished one into INT32 registers, and the INT32 result is exact in any
+//    order (Eq. gemm-final).  The epilogue then dequantises fl(fl(s_x s_w) acc) (+ bias).
+//  * bf16 path (BN = 256 and two slots, or BN = 128 and four when 256-wide tiles would leave SMs
+//    idle): one accumulator per tile over the whole k range.
 //  * epilogues: bf16 output, GeGLU of interleaved gate/up columns (16-column blocks: 8 gate, then
 //    the 8 matching up channels), or fp32 logits with the top-1 index (keys reduced with atomicMax,
 //    the last CTA to finish decodes them).
@@ -20,6 +24,7 @@
 #include <algorithm>
 
 #include "gemm_tc.cuh"
+#include "ops.cuh"
 #include "stream_gemm.cuh"
 #include "tmap.cuh"
 
@@ -28,17 +33,18 @@ namespace w8a8 {
 namespace {
 
 constexpr int kBM = 128;
-constexpr int kBK = 64;                  // one 128-byte swizzle atom of fp16 per row
-constexpr int kKbPerChunk = 16;          // 1024 k per exact fp32 chunk
+constexpr int kSwz = 128;                // swizzle span in bytes (TMA and the MMA descriptors agree)
+constexpr int kBK = kSwz / 2;            // k per stage: one swizzle span of fp16 per row
+constexpr int kKbPerChunk = 1024 / kBK;  // stages per exact fp32 chunk of 1024 k
 constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kTmemCols = 512;  // all of an SM's tensor memory: 2 (bf16) or 4 (W8A8) accumulator slots
 constexpr uint32_t kABytes = kBM * kBK * 2;
 
-template <bool kInt8>
+template <bool kInt8, int kBN>
 struct TcGeo {
-  static constexpr int BN = kInt8 ? 128 : 256;
-  static constexpr int S = kInt8 ? 6 : 4;
+  static constexpr int BN = kBN;
   static constexpr uint32_t BBytes = BN * kBK * 2;
+  static constexpr int S = (192 * 1024) / (int)(kABytes + BBytes);
   static constexpr int Smem = S * (kABytes + BBytes) + 1024;
 };
 
@@ -46,15 +52,16 @@ struct TcGeo {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
 
-// Shared-memory matrix descriptor of a K-major tile with 128-byte swizzle: rows of 128 bytes,
-// 8-row groups 1024 bytes apart (stride byte offset), descriptor version 1, layout SWIZZLE_128B.
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+// Shared-memory matrix descriptor of a K-major tile swizzled over kSwz bytes: rows of kSwz bytes,
+// 8-row groups 8 kSwz bytes apart (stride byte offset), descriptor version 1, layout SWIZZLE_128B
+// (2) or SWIZZLE_64B (4).
+__device__ __forceinline__ uint64_t sdesc_swz(uint32_t saddr) {
   uint64_t d = 0;
   d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)1 << 16;              // leading byte offset (unused by swizzled K-major layouts)
-  d |= (uint64_t)(1024 >> 4) << 32;    // stride byte offset
-  d |= (uint64_t)1 << 46;              // version
-  d |= (uint64_t)2 << 61;              // SWIZZLE_128B
+  d |= (uint64_t)1 << 16;                       // leading byte offset (unused by swizzled K-major layouts)
+  d |= (uint64_t)((8 * kSwz) >> 4) << 32;       // stride byte offset
+  d |= (uint64_t)1 << 46;                       // version
+  d |= (uint64_t)(kSwz == 128 ? 2 : 4) << 61;   // layout
   return d;
 }
 
@@ -91,13 +98,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return (uint32_t)f32_to_bf16_bits(a) | ((uint32_t)f32_to_bf16_bits(b) << 16);
 }
 
-template <bool kInt8>
+template <bool kInt8, int kBN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const TcArgs a) {
-  using GG = TcGeo<kInt8>;
+  using GG = TcGeo<kInt8, kBN>;
   constexpr int BN = GG::BN, S = GG::S;
+  constexpr int NSLOT = (int)kTmemCols / BN;  // accumulator slots in tensor memory
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t bars[2 * S + 5];
+  __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
   __shared__ uint32_t tmem_slot;
   __shared__ int s_flag;
 
@@ -105,11 +113,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t base = (raw + 1023u) & ~1023u;
   const uint32_t sA = base, sB = base + (uint32_t)S * kABytes;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
+  const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + kBM - 1) / kBM);
   const int nkb = (a.K + kBK - 1) / kBK;
   const int nchunks = kInt8 ? (nkb + kKbPerChunk - 1) / kKbPerChunk : 1;
-  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 16,
-                 done = acce0 + 16;
+  const int kb_per_chunk = kInt8 ? kKbPerChunk : nkb;
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
+                 done = acce0 + 8 * NSLOT;
 
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -117,7 +126,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < NSLOT; ++b) {
       mbar_init(accf0 + 8 * b, 1);
       mbar_init(acce0 + 8 * b, 128);
     }
@@ -136,25 +145,29 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = tmem_slot;
   pdl_wait();  // activations and outputs belong to the preceding kernels
 
+  // Persistent: CTA b takes tiles b, b + grid, ...; tile t covers channels (t mod NT) * BN and
+  // tokens (t / NT) * 128, so neighbouring CTAs share the activation rows.
   if (warp == 4) {
     // ---------------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
-      int kb = 0;
-      for (; kb < nkb; ++kb) {
-        const int s = kb % S;
-        const uint32_t ph = (uint32_t)((kb / S) & 1);
-        if (!mbar_wait_bounded(empty0 + 8 * s, ph ^ 1u, kWaitBudgetCycles)) {
-          ok = false;
-          break;
+      int g = 0;  // stages issued
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        const int n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
+        for (int kb = 0; kb < nkb; ++kb, ++g) {
+          const int s = g % S;
+          if (!mbar_wait_bounded(empty0 + 8 * s, (uint32_t)(((g / S) & 1) ^ 1), kWaitBudgetCycles)) {
+            ok = false;
+            break;
+          }
+          const uint32_t bar = full0 + 8 * s;
+          mbar_arrive_expect_tx(bar, kABytes + GG::BBytes);
+          tma_load_2d(sA + (uint32_t)s * kABytes, &tmA, kb * kBK, m0, bar);
+          tma_load_2d(sB + (uint32_t)s * GG::BBytes, &tmB, kb * kBK, n0, bar);
         }
-        const uint32_t bar = full0 + 8 * s;
-        mbar_arrive_expect_tx(bar, kABytes + GG::BBytes);
-        tma_load_2d(sA + (uint32_t)s * kABytes, &tmA, kb * kBK, m0, bar);
-        tma_load_2d(sB + (uint32_t)s * GG::BBytes, &tmB, kb * kBK, n0, bar);
       }
       if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
-      for (int j = kb > S ? kb - S : 0; j < kb; ++j) {  // let the last copies land before exit
+      for (int j = g > S ? g - S : 0; j < g; ++j) {  // let the last copies land before exit
         if (!mbar_wait_bounded(full0 + 8 * (j % S), (uint32_t)((j / S) & 1), kWaitBudgetCycles)) {
           atomicOr(a.err, DEVERR_DRAIN_WAIT);
           break;
@@ -166,32 +179,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16(kInt8 ? 0u : 1u, BN, kBM);
       bool ok = true;
-      for (int kb = 0; kb < nkb && ok; ++kb) {
-        const int c = kInt8 ? kb / kKbPerChunk : 0;
-        const int buf = c & 1;
-        const bool first = kInt8 ? (kb % kKbPerChunk == 0) : (kb == 0);
-        const bool last = kInt8 ? (kb % kKbPerChunk == kKbPerChunk - 1 || kb == nkb - 1) : (kb == nkb - 1);
-        if (kInt8 && first && c >= 2) {  // the epilogue has folded this buffer's previous chunk
-          if (!mbar_wait_bounded(acce0 + 8 * buf, (uint32_t)(((c >> 1) - 1) & 1), kWaitBudgetCycles)) {
+      int g = 0, q = 0;  // stages consumed, accumulator chunks produced
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        for (int c = 0; c < nchunks && ok; ++c, ++q) {
+          const int slot = q % NSLOT;
+          if (q >= NSLOT &&  // the epilogue has drained this slot's previous chunk
+              !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
             ok = false;
             break;
           }
-        }
-        const int s = kb % S;
-        if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((kb / S) & 1), kWaitBudgetCycles)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(buf * BN);
+          tc_fence_after();
+          const uint32_t d = tmem + (uint32_t)(slot * BN);
+          const int kb0 = c * kb_per_chunk, kb1 = min(nkb, kb0 + kb_per_chunk);
+          for (int kb = kb0; kb < kb1; ++kb, ++g) {
+            const int s = g % S;
+            if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
 #pragma unroll
-        for (int k16 = 0; k16 < kBK / 16; ++k16) {
-          const uint64_t ad = sdesc_sw128(sA + (uint32_t)s * kABytes + 32u * k16);
-          const uint64_t bd = sdesc_sw128(sB + (uint32_t)s * GG::BBytes + 32u * k16);
-          tc_mma(d, ad, bd, idesc, (first && k16 == 0) ? 0u : 1u);
+            for (int k16 = 0; k16 < kBK / 16; ++k16) {
+              const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
+              const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BBytes + 32u * k16);
+              tc_mma(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
+            }
+            tc_commit(empty0 + 8 * s);
+          }
+          if (ok) tc_commit(accf0 + 8 * slot);
         }
-        tc_commit(empty0 + 8 * s);
-        if (last) tc_commit(accf0 + 8 * buf);
       }
       if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
       tc_commit(done);  // completes once every MMA issued above has completed
@@ -199,87 +215,90 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------------------------------------------------------------- epilogue warps 0-3
-    const int row = m0 + 32 * warp + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
     const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
-    unsigned long long best = 0ull;
     bool ok = true;
-    // apply the epilogue to 32 consecutive columns c0 .. c0+31 of this thread's row
-    auto emit32 = [&](int c0, const float (&v)[32]) {
-      if (row >= a.M) return;
-      const int col0 = n0 + c0;
-      if (a.kind == EPI_GEGLU) {
+    int q = 0;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      const int n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
+      const int row = m0 + 32 * warp + lane;
+      unsigned long long best = 0ull;
+      // the epilogue of 32 consecutive columns c0 .. c0+31 of this thread's row
+      auto emit32 = [&](int c0, const float (&v)[32]) {
+        if (row >= a.M) return;
+        const int col0 = n0 + c0;
+        if (a.kind == EPI_GEGLU) {
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {  // two 16-column blocks: gate 0..7, up 8..15
-          const int cb = col0 + 16 * q;
-          if (cb + 16 > a.N) continue;
-          float h[8];
+          for (int hq = 0; hq < 2; ++hq) {  // two 16-column blocks: gate 0..7, up 8..15
+            const int cb = col0 + 16 * hq;
+            if (cb + 16 > a.N) continue;
+            float h[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) h[j] = geglu_recipe(v[16 * q + j], v[16 * q + 8 + j]);
-          uint4 w;
-          w.x = pack_bf16x2(h[0], h[1]);
-          w.y = pack_bf16x2(h[2], h[3]);
-          w.z = pack_bf16x2(h[4], h[5]);
-          w.w = pack_bf16x2(h[6], h[7]);
-          *reinterpret_cast<uint4*>(a.y + (size_t)row * (a.N >> 1) + (cb >> 1)) = w;
-        }
-      } else if (a.kind == EPI_BF16) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int cb = col0 + 8 * q;
-          if (cb + 8 <= a.N) {
+            for (int j = 0; j < 8; ++j) h[j] = geglu_recipe(v[16 * hq + j], v[16 * hq + 8 + j]);
             uint4 w;
-            w.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
-            w.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
-            w.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
-            w.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
-            *reinterpret_cast<uint4*>(a.y + (size_t)row * a.N + cb) = w;
+            w.x = pack_bf16x2(h[0], h[1]);
+            w.y = pack_bf16x2(h[2], h[3]);
+            w.z = pack_bf16x2(h[4], h[5]);
+            w.w = pack_bf16x2(h[6], h[7]);
+            *reinterpret_cast<uint4*>(a.y + (size_t)row * (a.N >> 1) + (cb >> 1)) = w;
           }
-        }
-      } else {
+        } else if (a.kind == EPI_BF16) {
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const int cb = col0 + 4 * q;
-          if (cb + 4 <= a.N && a.logits)
-            *reinterpret_cast<float4*>(a.logits + (size_t)row * a.N + cb) =
-                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-        }
-        if (want_top) {
+          for (int j8 = 0; j8 < 4; ++j8) {
+            const int cb = col0 + 8 * j8;
+            if (cb + 8 <= a.N) {
+              uint4 w;
+              w.x = pack_bf16x2(v[8 * j8 + 0], v[8 * j8 + 1]);
+              w.y = pack_bf16x2(v[8 * j8 + 2], v[8 * j8 + 3]);
+              w.z = pack_bf16x2(v[8 * j8 + 4], v[8 * j8 + 5]);
+              w.w = pack_bf16x2(v[8 * j8 + 6], v[8 * j8 + 7]);
+              *reinterpret_cast<uint4*>(a.y + (size_t)row * a.N + cb) = w;
+            }
+          }
+        } else {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int col = col0 + j;
-            if (col < a.N) {
-              const unsigned long long key = ((unsigned long long)float_order_key(v[j]) << 32) |
-                                             (unsigned long long)(0xFFFFFFFFu - (uint32_t)col);
-              best = key > best ? key : best;
+          for (int j4 = 0; j4 < 8; ++j4) {
+            const int cb = col0 + 4 * j4;
+            if (cb + 4 <= a.N && a.logits)
+              *reinterpret_cast<float4*>(a.logits + (size_t)row * a.N + cb) =
+                  make_float4(v[4 * j4], v[4 * j4 + 1], v[4 * j4 + 2], v[4 * j4 + 3]);
+          }
+          if (want_top) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const int col = col0 + j;
+              if (col < a.N) {
+                const unsigned long long key = ((unsigned long long)float_order_key(v[j]) << 32) |
+                                               (unsigned long long)(0xFFFFFFFFu - (uint32_t)col);
+                best = key > best ? key : best;
+              }
             }
           }
         }
-      }
-    };
-    if constexpr (kInt8) {
-      int isum[BN];
+      };
+      if constexpr (kInt8) {
+        int isum[BN];
 #pragma unroll
-      for (int j = 0; j < BN; ++j) isum[j] = 0;
-      for (int c = 0; c < nchunks && ok; ++c) {
-        const int buf = c & 1;
-        if (!mbar_wait_bounded(accf0 + 8 * buf, (uint32_t)((c >> 1) & 1), kWaitBudgetCycles)) {
-          ok = false;
-          atomicOr(a.err, DEVERR_CONSUMER_WAIT);
-          break;
+        for (int j = 0; j < BN; ++j) isum[j] = 0;
+        for (int c = 0; c < nchunks; ++c, ++q) {
+          const int slot = q % NSLOT;
+          if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
+            ok = false;
+            atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int g = 0; g < BN / 32; ++g) {
+            uint32_t r[32];
+            tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) isum[32 * g + j] += __float2int_rn(__uint_as_float(r[j]));
+          }
+          tc_fence_before();
+          mbar_arrive(acce0 + 8 * slot);
         }
-        tc_fence_after();
-#pragma unroll
-        for (int g = 0; g < BN / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(lane_base + (uint32_t)(buf * BN + 32 * g), r);
-#pragma unroll
-          for (int j = 0; j < 32; ++j) isum[32 * g + j] += __float2int_rn(__uint_as_float(r[j]));
-        }
-        tc_fence_before();
-        mbar_arrive(acce0 + 8 * buf);
-      }
-      if (ok) {
+        if (!ok) break;
         const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
         for (int g = 0; g < BN / 32; ++g) {
@@ -297,18 +316,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           emit32(32 * g, v);
         }
-      }
-    } else {
-      if (!mbar_wait_bounded(accf0, 0u, kWaitBudgetCycles)) {
-        ok = false;
-        atomicOr(a.err, DEVERR_CONSUMER_WAIT);
-      }
-      if (ok) {
+      } else {
+        const int slot = q % NSLOT;
+        if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
+          ok = false;
+          atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+          break;
+        }
         tc_fence_after();
 #pragma unroll 1
         for (int g = 0; g < BN / 32; ++g) {
           uint32_t r[32];
-          tmem_ld32(lane_base + (uint32_t)(32 * g), r);
+          tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -319,16 +338,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           emit32(32 * g, v);
         }
+        tc_fence_before();
+        mbar_arrive(acce0 + 8 * slot);
+        ++q;
       }
+      if (want_top && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
     }
-    // top-1 across the grid: per-row maxima by atomicMax, the last CTA decodes and clears them
+    // top-1 across the grid: the last CTA to finish decodes the per-row keys and clears them
     if (want_top) {
-      if (ok && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
       __threadfence();
       named_bar_sync(1, 128);
       if (threadIdx.x == 0) {
         const unsigned int prev = atomicAdd(a.grid_counter, 1u);
-        s_flag = prev == gridDim.x * gridDim.y - 1;
+        s_flag = prev == gridDim.x - 1;
         if (s_flag) *a.grid_counter = 0u;
       }
       named_bar_sync(1, 128);
@@ -349,21 +371,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <bool kInt8>
+template <bool kInt8, int kBN>
 w8a8_status launch_t(const TcArgs& a, cudaStream_t st) {
-  using GG = TcGeo<kInt8>;
+  using GG = TcGeo<kInt8, kBN>;
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<kInt8>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
+    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<kInt8, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
     attr_set[dev] = true;
   }
   CUtensorMap ta, tb;
-  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, kBM, true));
-  W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN, true));
-  const dim3 grid((a.N + GG::BN - 1) / GG::BN, (a.M + kBM - 1) / kBM);
-  W8A8_CUDA(launch_pdl(gemm_tc_kernel<kInt8>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, a));
+  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, kBM, kSwz));
+  W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN, kSwz));
+  const long long tiles = (long long)((a.N + GG::BN - 1) / GG::BN) * ((a.M + kBM - 1) / kBM);
+  const dim3 grid((unsigned)std::min<long long>(tiles, device_sms()));
+  W8A8_CUDA(launch_pdl(gemm_tc_kernel<kInt8, kBN>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, a));
   return W8A8_OK;
 }
 
@@ -382,7 +405,11 @@ w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st) {
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  const w8a8_status s = int8_codes ? launch_t<true>(a, st) : launch_t<false>(a, st);
+  // bf16: 256-channel tiles unless that leaves SMs without a tile
+  const long long tiles256 = (long long)((a.N + 255) / 256) * ((a.M + kBM - 1) / kBM);
+  const w8a8_status s = int8_codes                    ? launch_t<true, 128>(a, st)
+                        : tiles256 >= device_sms() ? launch_t<false, 256>(a, st)
+                                                   : launch_t<false, 128>(a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }

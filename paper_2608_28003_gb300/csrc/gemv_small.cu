@@ -155,60 +155,113 @@ __global__ void __launch_bounds__(kThreads, 2)
     // K1 for every token slot: x_hat = x * (1 / delta), m = max |x_hat|, s = m / 127,
     // q = clamp(rint(x_hat * (127 / m)), -127, 127); slots >= M and the tail past K hold zeros.
     const int nvec = a.K >> 3;
-    for (int m = 0; m < MT; ++m) {
-      float xh[4][8];
-      float amax = 0.0f;
-      const bool live = m < a.M;
-      if (live) {
-        const uint4* src = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K);
-#pragma unroll
+    if constexpr (MT <= 4) {  // one token at a time, all consumer warps on its row
+      for (int m = 0; m < MT; ++m) {
+        float xh[4][8];
+        float amax = 0.0f;
+        const bool live = m < a.M;
+        if (live) {
+          const uint4* src = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K);
+  #pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            const int vi = tid + v * kCW * 32;
+            if (vi < nvec) {
+              const uint4 w = src[vi];
+              const float4 d0 = idr[v][0], d1 = idr[v][1];
+              xh[v][0] = __fmul_rn(bf16_lo(w.x), d0.x);
+              xh[v][1] = __fmul_rn(bf16_hi(w.x), d0.y);
+              xh[v][2] = __fmul_rn(bf16_lo(w.y), d0.z);
+              xh[v][3] = __fmul_rn(bf16_hi(w.y), d0.w);
+              xh[v][4] = __fmul_rn(bf16_lo(w.z), d1.x);
+              xh[v][5] = __fmul_rn(bf16_hi(w.z), d1.y);
+              xh[v][6] = __fmul_rn(bf16_lo(w.w), d1.z);
+              xh[v][7] = __fmul_rn(bf16_hi(w.w), d1.w);
+  #pragma unroll
+              for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(xh[v][e]));
+            }
+          }
+        }
+        amax = warp_max(amax);
+        if (lane == 0) s_red[warp] = amax;
+        named_bar_sync(1, kCW * 32);
+        float mx = 0.0f;
+  #pragma unroll
+        for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red[i]);
+        named_bar_sync(1, kCW * 32);  // s_red is reused by the next slot
+        const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
+        if (tid == 0) {
+          const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127)
+          s_sx[m] = sx;
+          if (live && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
+        }
+  #pragma unroll
         for (int v = 0; v < 4; ++v) {
           const int vi = tid + v * kCW * 32;
           if (vi < nvec) {
-            const uint4 w = src[vi];
-            const float4 d0 = idr[v][0], d1 = idr[v][1];
-            xh[v][0] = __fmul_rn(bf16_lo(w.x), d0.x);
-            xh[v][1] = __fmul_rn(bf16_hi(w.x), d0.y);
-            xh[v][2] = __fmul_rn(bf16_lo(w.y), d0.z);
-            xh[v][3] = __fmul_rn(bf16_hi(w.y), d0.w);
-            xh[v][4] = __fmul_rn(bf16_lo(w.z), d1.x);
-            xh[v][5] = __fmul_rn(bf16_hi(w.z), d1.y);
-            xh[v][6] = __fmul_rn(bf16_lo(w.w), d1.z);
-            xh[v][7] = __fmul_rn(bf16_hi(w.w), d1.w);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(xh[v][e]));
+            uint2 packed = make_uint2(0u, 0u);
+            if (live) {
+              int q[8];
+  #pragma unroll
+              for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][e], r))));
+              packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                         ((uint32_t)(q[3] & 0xff) << 24);
+              packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                         ((uint32_t)(q[7] & 0xff) << 24);
+              if (a.xq_dbg && blockIdx.x == 0) *reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K + 8 * vi) = packed;
+            }
+            *reinterpret_cast<uint2*>(xsp + (size_t)m * kpad + 8 * vi) = packed;
           }
         }
       }
-      amax = warp_max(amax);
-      if (lane == 0) s_red[warp] = amax;
-      named_bar_sync(1, kCW * 32);
-      float mx = 0.0f;
+    } else {  // warp w quantises token w on its own (no block-wide barrier per token)
+      for (int m = warp; m < MT; m += kCW) {
+        uint2* dst = reinterpret_cast<uint2*>(xsp + (size_t)m * kpad);
+        if (m >= a.M) {
+          for (int vi = lane; vi < nvec; vi += 32) dst[vi] = make_uint2(0u, 0u);
+          if (lane == 0) s_sx[m] = 0.0f;
+          continue;
+        }
+        const uint4* src = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K);
+        const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
+        auto smooth8 = [&](int vi, float (&xh)[8]) {
+          const uint4 w = src[vi];
+          const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
+          xh[0] = __fmul_rn(bf16_lo(w.x), d0.x);
+          xh[1] = __fmul_rn(bf16_hi(w.x), d0.y);
+          xh[2] = __fmul_rn(bf16_lo(w.y), d0.z);
+          xh[3] = __fmul_rn(bf16_hi(w.y), d0.w);
+          xh[4] = __fmul_rn(bf16_lo(w.z), d1.x);
+          xh[5] = __fmul_rn(bf16_hi(w.z), d1.y);
+          xh[6] = __fmul_rn(bf16_lo(w.w), d1.z);
+          xh[7] = __fmul_rn(bf16_hi(w.w), d1.w);
+        };
+        float amax = 0.0f;
+        for (int vi = lane; vi < nvec; vi += 32) {
+          float xh[8];
+          smooth8(vi, xh);
 #pragma unroll
-      for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red[i]);
-      named_bar_sync(1, kCW * 32);  // s_red is reused by the next slot
-      const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
-      if (tid == 0) {
-        const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127)
-        s_sx[m] = sx;
-        if (live && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
-      }
+          for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(xh[e]));
+        }
+        const float mx = warp_max(amax);
+        const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
+        if (lane == 0) {
+          const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127)
+          s_sx[m] = sx;
+          if (a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
+        }
+        for (int vi = lane; vi < nvec; vi += 32) {  // second pass: the row again (L1 / L2)
+          float xh[8];
+          smooth8(vi, xh);
+          int q[8];
 #pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        const int vi = tid + v * kCW * 32;
-        if (vi < nvec) {
-          uint2 packed = make_uint2(0u, 0u);
-          if (live) {
-            int q[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][e], r))));
-            packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
-                       ((uint32_t)(q[3] & 0xff) << 24);
-            packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
-                       ((uint32_t)(q[7] & 0xff) << 24);
-            if (a.xq_dbg && blockIdx.x == 0) *reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K + 8 * vi) = packed;
-          }
-          *reinterpret_cast<uint2*>(xsp + (size_t)m * kpad + 8 * vi) = packed;
+          for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[e], r))));
+          uint2 packed;
+          packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                     ((uint32_t)(q[3] & 0xff) << 24);
+          packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                     ((uint32_t)(q[7] & 0xff) << 24);
+          dst[vi] = packed;
+          if (a.xq_dbg && blockIdx.x == 0) reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] = packed;
         }
       }
     }
@@ -271,19 +324,19 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (u >= cnt) break;
         const uint32_t sub = sb + (uint32_t)(u * R * kSliceBytes);
         if constexpr (kInt8) {
-          uint4 xv[MT];
+          uint4 wv[RW];
 #pragma unroll
-          for (int m = 0; m < MT; ++m) xv[m] = lds128(xs + (uint32_t)(m * kpad + (u0 + u) * 512 + 16 * lane));
+          for (int i = 0; i < RW; ++i) wv[i] = lds128(sub + wlane + (uint32_t)((warp + 8 * i) * 256));
 #pragma unroll
-          for (int i = 0; i < RW; ++i) {
-            const uint4 wv = lds128(sub + wlane + (uint32_t)((warp + 8 * i) * 256));
+          for (int m = 0; m < MT; ++m) {
+            const uint4 xv = lds128(xs + (uint32_t)(m * kpad + (u0 + u) * 512 + 16 * lane));
 #pragma unroll
-            for (int m = 0; m < MT; ++m) {
+            for (int i = 0; i < RW; ++i) {
               int t = acc[u % NA][i][m];
-              t = __dp4a((int)wv.x, (int)xv[m].x, t);
-              t = __dp4a((int)wv.y, (int)xv[m].y, t);
-              t = __dp4a((int)wv.z, (int)xv[m].z, t);
-              t = __dp4a((int)wv.w, (int)xv[m].w, t);
+              t = __dp4a((int)wv[i].x, (int)xv.x, t);
+              t = __dp4a((int)wv[i].y, (int)xv.y, t);
+              t = __dp4a((int)wv[i].z, (int)xv.z, t);
+              t = __dp4a((int)wv[i].w, (int)xv.w, t);
               acc[u % NA][i][m] = t;
             }
           }
@@ -382,19 +435,34 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   }
   constexpr int EB = kInt8 ? 1 : 2;
   CUtensorMap tw;
-  W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, false));
+  W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
   W8A8_CUDA(launch_pdl(gemv_small_kernel<kInt8, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
                        a));
   return W8A8_OK;
 }
 
+// accumulator registers a warp may hold (tokens x rows): larger products spill
+template <bool kInt8>
+constexpr int max_slots() {
+  return kInt8 ? 48 : 32;
+}
+
+template <bool kInt8, int MT, int RW>
+w8a8_status launch_checked(const SmallArgs& a, cudaStream_t st) {
+  if constexpr (MT * RW <= max_slots<kInt8>()) {
+    return launch_t<kInt8, MT, RW>(a, st);
+  } else {
+    W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "small GEMV: %d tokens x %d rows per warp not built", MT, RW);
+  }
+}
+
 template <bool kInt8, int MT>
 w8a8_status launch_mt(const SmallArgs& a, cudaStream_t st) {
   switch (a.p.RW) {
-    case 1: return launch_t<kInt8, MT, 1>(a, st);
-    case 2: return launch_t<kInt8, MT, 2>(a, st);
-    case 4: return launch_t<kInt8, MT, 4>(a, st);
-    default: return launch_t<kInt8, MT, 6>(a, st);
+    case 1: return launch_checked<kInt8, MT, 1>(a, st);
+    case 2: return launch_checked<kInt8, MT, 2>(a, st);
+    case 4: return launch_checked<kInt8, MT, 4>(a, st);
+    default: return launch_checked<kInt8, MT, 6>(a, st);
   }
 }
 
@@ -415,8 +483,8 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
   if (M < 1 || M > 8 || N < 1 || K < 16 || K % 16 != 0) return p;
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return p;
   if (kind == EPI_GEGLU && N % 16 != 0) return p;
-  if (int8_weights && K > kMaxInt8K) return p;
   p.MT = M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
+  if (int8_weights && p.MT <= 4 && K > kMaxInt8K) return p;
   // fewest rows per CTA (more CTAs) that still fit in two CTAs per SM
   static const int kRw[] = {1, 2, 4, 6};
   for (int rw : kRw) {
@@ -427,7 +495,7 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
     }
   }
   if (p.RW == 0) return p;
-  if (!int8_weights && p.MT == 8 && p.RW == 6) return p;  // would spill registers: streaming kernel
+  if (p.MT * p.RW > (int8_weights ? max_slots<true>() : max_slots<false>())) return p;  // registers
   const int R = 8 * p.RW;
   p.P = (N + R - 1) / R;
   const int cps = p.P > sm_count ? 2 : 1;

@@ -27,7 +27,7 @@ EncodeTiledFn encode_fn() {
 }  // namespace
 
 w8a8_status make_tmap_2d(CUtensorMap* map, const void* base, int elem_bytes, uint64_t inner, uint64_t rows,
-                         uint64_t pitch_bytes, uint32_t box_inner, uint32_t box_rows, bool swizzle128) {
+                         uint64_t pitch_bytes, uint32_t box_inner, uint32_t box_rows, int swizzle_bytes) {
   EncodeTiledFn fn = encode_fn();
   W8A8_CHECK_ARG(fn != nullptr, W8A8_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
   const CUtensorMapDataType dt = elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
@@ -36,7 +36,10 @@ w8a8_status make_tmap_2d(CUtensorMap* map, const void* base, int elem_bytes, uin
   const cuuint32_t box[2] = {box_inner, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   const CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                        swizzle_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                        : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                              : CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   W8A8_CHECK_ARG(r == CUDA_SUCCESS, W8A8_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d) for [%llu x %llu] box [%u x %u]",
                  (int)r, (unsigned long long)rows, (unsigned long long)inner, box_rows, box_inner);
   return W8A8_OK;
