@@ -109,11 +109,15 @@ static unsigned int* err_word(void* ws) {
 // into it on the W8A8 path); returns false when the shape is left to the streaming kernel.
 static bool small_gemv(bool int8, const void* W, const float* inv_delta, const float* s_w, const uint16_t* X, int M,
                        int N, int K, const float* bias, int kind, uint16_t* Y, const w8a8_debug* dbg, void* ws,
-                       const void* prefetch, size_t prefetch_bytes, int sms, cudaStream_t st, w8a8_status* status) {
+                       const ResNorm* rn, int sms, cudaStream_t st, w8a8_status* status) {
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return false;
   SmallArgs a{};
-  a.p = make_small_plan(int8, M, N, K, kind, sms);
+  a.p = make_small_plan(int8, M, N, K, kind, sms, rn != nullptr);
   if (!a.p.ok) return false;
+  if (rn) {
+    a.has_rn = 1;
+    a.rn = *rn;
+  }
   a.W = W;
   a.X = X;
   a.M = M;
@@ -127,11 +131,13 @@ static bool small_gemv(bool int8, const void* W, const float* inv_delta, const f
   a.xq_dbg = dbg ? dbg->xq : nullptr;
   a.s_x_dbg = dbg ? dbg->s_x : nullptr;
   a.acc_dbg = dbg ? dbg->acc : nullptr;
-  a.prefetch = prefetch;
-  a.prefetch_bytes = prefetch ? prefetch_bytes / 16 * 16 : 0;
   a.err = err_word(ws);
   *status = launch_small_gemv(int8, a, st);
   return true;
+}
+
+bool decode_gemv_takes(bool int8, int M, int N, int K, bool geglu, int sms) {
+  return make_small_plan(int8, M, N, K, geglu ? EPI_GEGLU : EPI_BF16, sms, true).ok != 0;
 }
 
 // Calls with more tokens than the decode GEMV takes go to the tensor-core GEMM when its shape
@@ -183,13 +189,13 @@ static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N,
 // One W8A8 linear: K1 then the streaming GEMM.  s_x and the codes live in the workspace.
 w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
                                    uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
-                                   int sms, cudaStream_t st, const L2Prefetch* pf) {
+                                   int sms, cudaStream_t st, const ResNorm* rn) {
   const int N = w->n, K = w->k;
   w8a8_status small_status = W8A8_OK;
   if (!logits && !top1 &&
-      small_gemv(true, w->wq, w->inv_delta, w->s_w, X, M, N, K, bias, kind, Y, dbg, ws, pf ? pf->ptr : nullptr,
-                 pf ? pf->bytes : 0, sms, st, &small_status))
+      small_gemv(true, w->wq, w->inv_delta, w->s_w, X, M, N, K, bias, kind, Y, dbg, ws, rn, sms, st, &small_status))
     return small_status;
+  W8A8_CHECK_ARG(!rn, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take M=%d N=%d K=%d", M, N, K);
   LinearWs L = linear_ws(M, N, K, true, sms);
   char* base = reinterpret_cast<char*>(ws);
   void* codes = base + L.xf16;
@@ -221,12 +227,12 @@ w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, con
 
 w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias,
                                    int kind, uint16_t* Y, float* logits, int32_t* top1, void* ws, int sms,
-                                   cudaStream_t st, const L2Prefetch* pf) {
+                                   cudaStream_t st, const ResNorm* rn) {
   w8a8_status small_status = W8A8_OK;
   if (!logits && !top1 &&
-      small_gemv(false, W, nullptr, nullptr, X, M, N, K, bias, kind, Y, nullptr, ws, pf ? pf->ptr : nullptr,
-                 pf ? pf->bytes : 0, sms, st, &small_status))
+      small_gemv(false, W, nullptr, nullptr, X, M, N, K, bias, kind, Y, nullptr, ws, rn, sms, st, &small_status))
     return small_status;
+  W8A8_CHECK_ARG(!rn, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take M=%d N=%d K=%d", M, N, K);
   if (tc_path(false, W, X, M, N, K, bias, kind, nullptr, nullptr, Y, logits, top1, nullptr, ws, nullptr, nullptr, st,
               &small_status))
     return small_status;
@@ -366,12 +372,7 @@ FfnWs ffn_ws(int M, int H, int F, int sms) {
 }
 
 w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y, uint16_t* h_dbg,
-                    void* workspace, int sms, cudaStream_t st, const L2Prefetch* pf_gate_up,
-                    const L2Prefetch* pf_down) {
-  const void* pgu = pf_gate_up ? pf_gate_up->ptr : nullptr;
-  const size_t bgu = pf_gate_up ? pf_gate_up->bytes : 0;
-  const void* pdn = pf_down ? pf_down->ptr : nullptr;
-  const size_t bdn = pf_down ? pf_down->bytes : 0;
+                    void* workspace, int sms, cudaStream_t st, const ResNorm* rn_gate_up) {
   const int H = f->hidden, F = f->inter;
   const FfnWs L = ffn_ws(M, H, F, sms);
   char* base = reinterpret_cast<char*>(workspace);
@@ -382,8 +383,10 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     // gate/up: scratch at L.gu
     w8a8_status ss = W8A8_OK;
     if (small_gemv(true, f->gate_up.wq, f->gate_up.inv_delta, f->gate_up.s_w, X, M, 2 * F, H, nullptr, EPI_GEGLU, h,
-                   nullptr, workspace, pgu, bgu, sms, st, &ss)) {
+                   nullptr, workspace, rn_gate_up, sms, st, &ss)) {
       W8A8_TRY(ss);
+    } else if (rn_gate_up) {
+      W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take gate/up at M=%d", M);
     } else if (tc_path(true, f->gate_up.wq_f16, X, M, 2 * F, H, nullptr, EPI_GEGLU, f->gate_up.inv_delta,
                        f->gate_up.s_w, h, nullptr, nullptr, nullptr, workspace,
                        base + L.gu + (linear_ws(M, 2 * F, H, true, sms).xf16 - W8A8_WS_RESERVED),
@@ -411,7 +414,7 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
       W8A8_TRY(launch_stream_gemm(true, a, st));
     }
     if (small_gemv(true, f->down.wq, f->down.inv_delta, f->down.s_w, h, M, H, F, nullptr, EPI_BF16, Y, nullptr,
-                   workspace, pdn, bdn, sms, st, &ss)) {
+                   workspace, nullptr, sms, st, &ss)) {
       W8A8_TRY(ss);
     } else if (tc_path(true, f->down.wq_f16, h, M, H, F, nullptr, EPI_BF16, f->down.inv_delta, f->down.s_w, Y,
                        nullptr, nullptr, nullptr, workspace,
@@ -442,8 +445,10 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
   } else {
     w8a8_status ss = W8A8_OK;
     if (small_gemv(false, f->gate_up_bf16, nullptr, nullptr, X, M, 2 * F, H, nullptr, EPI_GEGLU, h, nullptr,
-                   workspace, pgu, bgu, sms, st, &ss)) {
+                   workspace, rn_gate_up, sms, st, &ss)) {
       W8A8_TRY(ss);
+    } else if (rn_gate_up) {
+      W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take gate/up at M=%d", M);
     } else if (tc_path(false, f->gate_up_bf16, X, M, 2 * F, H, nullptr, EPI_GEGLU, nullptr, nullptr, h, nullptr,
                        nullptr, nullptr, workspace, nullptr, nullptr, st, &ss)) {
       W8A8_TRY(ss);
@@ -463,7 +468,7 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
       W8A8_TRY(launch_stream_gemm(false, a, st));
     }
     if (small_gemv(false, f->down_bf16, nullptr, nullptr, h, M, H, F, nullptr, EPI_BF16, Y, nullptr, workspace,
-                   pdn, bdn, sms, st, &ss)) {
+                   nullptr, sms, st, &ss)) {
       W8A8_TRY(ss);
     } else if (tc_path(false, f->down_bf16, h, M, H, F, nullptr, EPI_BF16, nullptr, nullptr, Y, nullptr, nullptr,
                        nullptr, workspace, nullptr, nullptr, st, &ss)) {

@@ -6,13 +6,15 @@
 // partial-tile protocol through global memory; here every CTA owns R = 8 RW consecutive weight
 // rows over the full k range, so each sum ends inside its CTA:
 //  * one producer thread streams the CTA's rows through a shared-memory ring with 2-D TMA, starting
-//    before the preceding kernel has finished (weights do not depend on it), and can ask L2 to
-//    fetch a later kernel's weights.  A stage holds KS sub-slices of 512 bytes per row (each one or
+//    before the preceding kernel has finished (weights do not depend on it).  A stage holds KS
+//    sub-slices of 512 bytes per row (each one or
 //    two unswizzled boxes of R rows x 256 elements), so that small-R calls still move enough bytes
 //    per pipeline round trip;
 //  * the 8 consumer warps wait for the preceding kernel and stage the activations in shared
-//    memory.  The W8A8 path quantises them there, with the arithmetic of the stand-alone per-token
-//    quantiser (Eq. stx / xint8, smoothing of Eq. xhat-lmhead), so one launch does K1 and K3;
+//    memory, optionally computing them first from the decoder's residual step (residual add and
+//    the two RMSNorms, fused here instead of a separate launch).  The W8A8 path quantises them
+//    there, with the arithmetic of the stand-alone per-token quantiser (Eq. stx / xint8,
+//    smoothing of Eq. xhat-lmhead), so one launch does K1 and K3;
 //  * warp w takes rows w, w + 8, ...; in every sub-slice lane l reads bytes 16 l .. 16 l + 15 of
 //    a row's 512 bytes (consecutive lanes read consecutive bytes: no bank conflicts);
 //  * INT8: four dp4a per 16 bytes and token, exact INT32 sums (Eq. gemm-final); bf16: fp32 FMAs,
@@ -40,8 +42,23 @@ constexpr int kStatic = 2048;       // static shared memory of the kernel (reduc
 constexpr int kSliceBytes = 512;    // bytes of one weight row per sub-slice
 constexpr int kMaxInt8K = 8 * 256 * 4;  // K1 keeps a token's smoothed row in registers: 4 vectors of 8 per thread
 
-__device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(ptr), "r"(bytes) : "memory");
+__device__ __forceinline__ float warp_sum32(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum over the 256 consumer threads in the residual-norm kernel's order (lane tree, then warps
+// 0..7 in turn); every consumer thread gets the result.
+__device__ __forceinline__ float consumer_sum(float v, float* red, int warp, int lane) {
+  v = warp_sum32(v);
+  named_bar_sync(1, 256);
+  if (lane == 0) red[warp] = v;
+  named_bar_sync(1, 256);
+  float t = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) t += red[i];
+  return t;
 }
 
 __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
@@ -63,7 +80,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t ring = (raw + 1023u) & ~1023u;
   const uint32_t xs = ring + (uint32_t)(S * SB);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (ring - raw) + (size_t)S * SB + p.xbytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (ring - raw) + (size_t)S * SB + p.xbytes + p.abytes);
   uint64_t* empty = full + S;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row0 = blockIdx.x * R;
@@ -84,7 +101,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     bool ok = true;
     int it = 0, s = 0;
     uint32_t ph = 0;
-    const int first_fill = S < nst ? S : nst;
     for (; it < nst; ++it) {
       if (!mbar_wait_bounded(smem_u32(empty + s), ph ^ 1u, kWaitBudgetCycles)) {
         ok = false;
@@ -100,15 +116,6 @@ __global__ void __launch_bounds__(kThreads, 2)
           tma_load_2d(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar);
         } else {
           tma_load_2d(d, &tmW, (u0 + u) * 256, row0, bar);
-        }
-      }
-      if (it + 1 == first_fill && a.prefetch) {  // this CTA's share of a later kernel's weights
-        const size_t per = ((a.prefetch_bytes + gridDim.x - 1) / gridDim.x + 15) / 16 * 16;
-        const size_t beg = per * blockIdx.x;
-        const size_t end = beg + per < a.prefetch_bytes ? beg + per : a.prefetch_bytes;
-        for (size_t off = beg; off < end; off += 65536) {
-          const size_t n = end - off < 65536 ? end - off : 65536;
-          prefetch_l2(reinterpret_cast<const char*>(a.prefetch) + off, (uint32_t)n);
         }
       }
       if (++s == S) {
@@ -149,8 +156,70 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
     }
   }
+  // weights of the fused residual norm (constants): this thread's 8 channels
+  const int nvk = a.K >> 3;
+  float wp[8], wn[8];
+  if (a.has_rn && tid < nvk) {
+    const float4* p0 = reinterpret_cast<const float4*>(a.rn.w_post + 8 * tid);
+    const float4* p1 = reinterpret_cast<const float4*>(a.rn.w_next + 8 * tid);
+    const float4 a0 = p0[0], a1 = p0[1], b0 = p1[0], b1 = p1[1];
+    wp[0] = a0.x; wp[1] = a0.y; wp[2] = a0.z; wp[3] = a0.w; wp[4] = a1.x; wp[5] = a1.y; wp[6] = a1.z; wp[7] = a1.w;
+    wn[0] = b0.x; wn[1] = b0.y; wn[2] = b0.z; wn[3] = b0.w; wn[4] = b1.x; wn[5] = b1.y; wn[6] = b1.z; wn[7] = b1.w;
+  }
   pdl_wait();
   uint8_t* xsp = smem_raw + (xs - raw);
+  // The bf16 rows behind the activations: the caller's X, or the fused residual norm's output
+  // (thread t < K / 8 owns channels 8t .. 8t+7 of every token, as in the residual-norm kernel).
+  const uint16_t* xrows = a.X;
+  int xstride = a.K;
+  if (a.has_rn) {
+    uint16_t* as = kInt8 ? reinterpret_cast<uint16_t*>(xsp + p.xbytes) : reinterpret_cast<uint16_t*>(xsp);
+    for (int m = 0; m < MT; ++m) {
+      const bool mine = m < a.M && tid < nvk;
+      float yv[8], rv[8];
+      float ss = 0.0f;
+      if (mine) {
+        const uint4 yw = reinterpret_cast<const uint4*>(a.rn.y + (size_t)m * a.K)[tid];
+        unpack_bf16x8(yw, yv);
+        const float4* rp = reinterpret_cast<const float4*>(a.rn.r_in + (size_t)m * a.K + 8 * tid);
+        const float4 r0 = rp[0], r1 = rp[1];
+        rv[0] = r0.x; rv[1] = r0.y; rv[2] = r0.z; rv[3] = r0.w; rv[4] = r1.x; rv[5] = r1.y; rv[6] = r1.z; rv[7] = r1.w;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) ss += yv[e] * yv[e];
+      }
+      const float inv_y = 1.0f / sqrtf(consumer_sum(ss, s_red, warp, lane) / (float)a.K + a.rn.eps);
+      float ss2 = 0.0f;
+      if (mine) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          rv[e] += yv[e] * inv_y * wp[e];
+          ss2 += rv[e] * rv[e];
+        }
+        if (blockIdx.x == 0) {
+          float4* ro = reinterpret_cast<float4*>(a.rn.r_out + (size_t)m * a.K + 8 * tid);
+          ro[0] = make_float4(rv[0], rv[1], rv[2], rv[3]);
+          ro[1] = make_float4(rv[4], rv[5], rv[6], rv[7]);
+        }
+      }
+      const float inv_r = 1.0f / sqrtf(consumer_sum(ss2, s_red, warp, lane) / (float)a.K + a.rn.eps);
+      if (tid < (kpad >> 3)) {  // the padded row: zeros past K and in slots >= M
+        uint4 w = make_uint4(0u, 0u, 0u, 0u);
+        if (mine) {
+          float o[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) o[e] = rv[e] * inv_r * wn[e];
+          w.x = (uint32_t)f32_to_bf16_bits(o[0]) | ((uint32_t)f32_to_bf16_bits(o[1]) << 16);
+          w.y = (uint32_t)f32_to_bf16_bits(o[2]) | ((uint32_t)f32_to_bf16_bits(o[3]) << 16);
+          w.z = (uint32_t)f32_to_bf16_bits(o[4]) | ((uint32_t)f32_to_bf16_bits(o[5]) << 16);
+          w.w = (uint32_t)f32_to_bf16_bits(o[6]) | ((uint32_t)f32_to_bf16_bits(o[7]) << 16);
+        }
+        *reinterpret_cast<uint4*>(as + (size_t)m * kpad + 8 * tid) = w;
+      }
+    }
+    named_bar_sync(1, kCW * 32);
+    xrows = as;
+    xstride = kpad;
+  }
   if constexpr (kInt8) {
     // K1 for every token slot: x_hat = x * (1 / delta), m = max |x_hat|, s = m / 127,
     // q = clamp(rint(x_hat * (127 / m)), -127, 127); slots >= M and the tail past K hold zeros.
@@ -161,8 +230,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         float amax = 0.0f;
         const bool live = m < a.M;
         if (live) {
-          const uint4* src = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K);
-  #pragma unroll
+          const uint4* src = reinterpret_cast<const uint4*>(xrows + (size_t)m * xstride);
+#pragma unroll
           for (int v = 0; v < 4; ++v) {
             const int vi = tid + v * kCW * 32;
             if (vi < nvec) {
@@ -176,7 +245,7 @@ __global__ void __launch_bounds__(kThreads, 2)
               xh[v][5] = __fmul_rn(bf16_hi(w.z), d1.y);
               xh[v][6] = __fmul_rn(bf16_lo(w.w), d1.z);
               xh[v][7] = __fmul_rn(bf16_hi(w.w), d1.w);
-  #pragma unroll
+#pragma unroll
               for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(xh[v][e]));
             }
           }
@@ -185,7 +254,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (lane == 0) s_red[warp] = amax;
         named_bar_sync(1, kCW * 32);
         float mx = 0.0f;
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red[i]);
         named_bar_sync(1, kCW * 32);  // s_red is reused by the next slot
         const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
@@ -194,14 +263,14 @@ __global__ void __launch_bounds__(kThreads, 2)
           s_sx[m] = sx;
           if (live && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
         }
-  #pragma unroll
+#pragma unroll
         for (int v = 0; v < 4; ++v) {
           const int vi = tid + v * kCW * 32;
           if (vi < nvec) {
             uint2 packed = make_uint2(0u, 0u);
             if (live) {
               int q[8];
-  #pragma unroll
+#pragma unroll
               for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][e], r))));
               packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
                          ((uint32_t)(q[3] & 0xff) << 24);
@@ -221,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 2)
           if (lane == 0) s_sx[m] = 0.0f;
           continue;
         }
-        const uint4* src = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K);
+        const uint4* src = reinterpret_cast<const uint4*>(xrows + (size_t)m * xstride);
         const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
         auto smooth8 = [&](int vi, float (&xh)[8]) {
           const uint4 w = src[vi];
@@ -270,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       const int m = i / tail16, c = i - m * tail16;
       *reinterpret_cast<uint4*>(xsp + (size_t)m * kpad + a.K + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
     }
-  } else {
+  } else if (!a.has_rn) {
     const int vpr = kpad >> 3;  // 16-byte vectors per slot
     const int total = MT * vpr;
     for (int i0 = tid; i0 < total; i0 += 4 * kCW * 32) {  // four loads in flight per thread
@@ -478,8 +547,9 @@ w8a8_status launch_typed(const SmallArgs& a, cudaStream_t st) {
 
 }  // namespace
 
-SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count) {
+SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count, bool fused_norm) {
   SmallPlan p{};
+  if (fused_norm && K > 2048) return p;  // one 8-channel vector per consumer thread
   if (M < 1 || M > 8 || N < 1 || K < 16 || K % 16 != 0) return p;
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return p;
   if (kind == EPI_GEGLU && N % 16 != 0) return p;
@@ -503,7 +573,8 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
   p.nsub = (K + p.sub - 1) / p.sub;
   p.kpad = p.nsub * p.sub;
   p.xbytes = p.MT * p.kpad * (int8_weights ? 1 : 2);
-  const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - 16 * 16;
+  p.abytes = fused_norm && int8_weights ? p.MT * p.kpad * 2 : 0;
+  const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - p.abytes - 16 * 16;
   // sub-slices per stage: 4 for warps with one or two rows, fewer for wider CTAs; each stage must
   // fit twice in the ring unless one stage covers everything
   for (int ks = p.RW <= 2 ? 4 : p.RW == 4 ? 2 : 1; ks >= 1; ks >>= 1) {
@@ -518,7 +589,7 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
     }
   }
   if (p.ks == 0) return p;
-  p.smem_bytes = 1024 + p.stages * p.stage_bytes + p.xbytes + 16 * p.stages;
+  p.smem_bytes = 1024 + p.stages * p.stage_bytes + p.xbytes + p.abytes + 16 * p.stages;
   p.ok = 1;
   return p;
 }

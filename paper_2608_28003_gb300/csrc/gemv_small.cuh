@@ -20,7 +20,21 @@ struct SmallPlan {
   int stages;       // ring depth
   int stage_bytes;  // ks x R rows x 512 bytes
   int xbytes;       // activations in shared memory: MT x kpad bf16 or INT8 codes
+  int abytes;       // W8A8 with a fused residual norm: the bf16 rows it produces, before K1
   int smem_bytes;
+};
+
+// The decoder's residual step in front of a decode linear, fused into the GEMV's prologue:
+// r_out = r_in + rmsnorm(y) * w_post, and the linear's input X = bf16(rmsnorm(r_out) * w_next),
+// with the arithmetic of the stand-alone residual-norm kernel (bit-identical results).  Every CTA
+// computes the rows it needs; the first CTA writes r_out, so r_out must not alias r_in.
+struct ResNorm {
+  const uint16_t* y;    // [M, K] bf16: the previous linear's output
+  const float* r_in;    // [M, K] fp32 residual stream before
+  float* r_out;         // [M, K] fp32 residual stream after
+  const float* w_post;  // [K] weights of the norm of y
+  const float* w_next;  // [K] weights of the norm of the new residual (this linear's input norm)
+  float eps;
 };
 
 struct SmallArgs {
@@ -35,13 +49,14 @@ struct SmallArgs {
   int8_t* xq_dbg;          // [M, K] nullable: the INT8 activation codes
   float* s_x_dbg;          // [M] nullable: the per-token scales
   int32_t* acc_dbg;        // [M, N] nullable: the INT32 sums
-  const void* prefetch;    // nullable: bytes to pull into L2 for a later kernel (16-byte aligned)
-  size_t prefetch_bytes;   // a multiple of 16
+  int has_rn;              // 1: X is computed from rn (X unused)
+  ResNorm rn;
   unsigned int* err;       // device error word
   SmallPlan p;
 };
 
-SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count);
+// fused_norm: the call computes its input with a ResNorm (needs K <= 2048)
+SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count, bool fused_norm = false);
 w8a8_status launch_small_gemv(bool int8_weights, const SmallArgs& a, cudaStream_t st);
 
 }  // namespace w8a8

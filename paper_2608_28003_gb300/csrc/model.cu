@@ -6,6 +6,7 @@
 #include <cmath>
 #include <map>
 #include <tuple>
+#include <utility>
 #include <vector>
 
 #include "decoder_kernels.cuh"
@@ -48,6 +49,7 @@ struct w8a8_model {
   int lm = 0;
 
   float* r = nullptr;
+  float* r2 = nullptr;  // the residual stream ping-pongs between r and r2 when its update is fused
   uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *y = nullptr, *h = nullptr;
   float* q = nullptr;
   uint16_t *kc = nullptr, *vc = nullptr;
@@ -108,12 +110,27 @@ void free_all(w8a8_model* m) {
 w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, q.wq_f16}; }
 
 w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
-                   uint16_t* Y, cudaStream_t st, const L2Prefetch* pf) {
+                   uint16_t* Y, cudaStream_t st, const ResNorm* rn) {
   if (int8) {
     const w8a8_qweight w = qdesc(qw, N, K);
-    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st, pf);
+    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st, rn);
   }
-  return run_bf16_linear(Wbf, N, K, X, M, nullptr, 0, Y, nullptr, nullptr, m->ws, m->sms, st, pf);
+  return run_bf16_linear(Wbf, N, K, X, M, nullptr, 0, Y, nullptr, nullptr, m->ws, m->sms, st, rn);
+}
+
+// At decode the residual step (residual add + the two RMSNorms) runs inside the next linear's
+// decode GEMV: q/k/v takes the step after the previous layer's FFN, gate/up the step after o.
+// It needs the decode GEMV to take both linears of every layer under the current mask.
+bool fuse_residual(const w8a8_model* m, int M, bool calib) {
+  if (calib || M > 8) return false;
+  const int H = m->cfg.hidden, F = m->cfg.inter;
+  for (int l = 0; l < m->cfg.layers; ++l) {
+    const bool att8 = m->prepared && ((m->attn_bits >> l) & 1u);
+    const bool ffn8 = m->prepared && ((m->ffn_bits >> l) & 1u);
+    if (!decode_gemv_takes(att8, M, m->qkv_dim, H, false, m->sms)) return false;
+    if (!decode_gemv_takes(ffn8, M, 2 * F, H, true, m->sms)) return false;
+  }
+  return true;
 }
 
 // The decoder over M = B * T rows whose positions start at *m->d_pos (set by the caller).
@@ -121,14 +138,23 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
                          cudaStream_t st) {
   const w8a8_model_cfg& c = m->cfg;
   const int M = B * T, H = c.hidden, F = c.inter;
-  W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, m->r, m->a, st));
+  const bool fuse = fuse_residual(m, M, calib);
+  float* rc = m->r;   // the residual stream as of now
+  float* rn = m->r2;  // where a fused update writes the next one
+  W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st));
   for (int l = 0; l < c.layers; ++l) {
     const w8a8_layer_bf16& W = m->L[l];
     const bool att8 = !calib && m->prepared && ((m->attn_bits >> l) & 1u);
     const bool ffn8 = !calib && m->prepared && ((m->ffn_bits >> l) & 1u);
     const bool glob = m->is_global(l);
     if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_qkv(l), st));
-    W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
+    if (fuse && l > 0) {  // the previous layer's post-FFN step, then q/k/v
+      const ResNorm R{m->y, rc, rn, m->L[l - 1].ln_post_ffn, W.ln_in, c.eps};
+      W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, nullptr, M, m->qkv, st, &R));
+      std::swap(rc, rn);
+    } else {
+      W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
+    }
     AttnShape s{B, T, c.n_q, c.n_kv, c.head_dim, c.max_seq, glob ? 0 : c.window,
                 (float)(1.0 / std::sqrt((double)c.head_dim))};
     uint16_t* kc = m->kc + (size_t)l * m->cache_layer_elems();
@@ -145,19 +171,27 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     }
     if (calib) W8A8_TRY(launch_act_absmax(m->o, M, m->q_dim, m->stat_o(l), st));
     W8A8_TRY(linear(m, att8, m->q_o[l], W.wo, H, m->q_dim, m->o, M, m->y, st, nullptr));
-    W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, m->r, m->a, st));
-    if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
     w8a8_ffn_weights f{H,
                        F,
                        qdesc(m->q_gu[l], 2 * F, H),
                        qdesc(m->q_down[l], H, F),
                        m->gu_bf16 + (size_t)l * 2 * F * H,
                        W.wdown};
-    W8A8_TRY(run_ffn(&f, ffn8 ? W8A8_PREC_W8A8 : W8A8_PREC_BF16, m->a, M, m->y, calib ? m->h : nullptr, m->ws, m->sms,
-                     st));
+    const int prec = ffn8 ? W8A8_PREC_W8A8 : W8A8_PREC_BF16;
+    if (fuse) {  // the post-attention step inside gate/up
+      const ResNorm R{m->y, rc, rn, W.ln_post_attn, W.ln_pre_ffn, c.eps};
+      W8A8_TRY(run_ffn(&f, prec, nullptr, M, m->y, nullptr, m->ws, m->sms, st, &R));
+      std::swap(rc, rn);
+    } else {
+      W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, rc, m->a, st));
+      if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
+      W8A8_TRY(run_ffn(&f, prec, m->a, M, m->y, calib ? m->h : nullptr, m->ws, m->sms, st));
+    }
     if (calib) W8A8_TRY(launch_act_absmax(m->h, M, F, m->stat_down(l), st));
-    const float* next = l + 1 < c.layers ? m->L[l + 1].ln_in : m->final_norm;
-    W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, m->r, m->a, st));
+    if (!fuse || l + 1 == c.layers) {
+      const float* next = l + 1 < c.layers ? m->L[l + 1].ln_in : m->final_norm;
+      W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, rc, m->a, st));
+    }
   }
   if (calib) return launch_act_absmax(m->a, M, H, m->stat_lm(), st);
   const bool lm8 = m->prepared && m->lm;
@@ -287,6 +321,7 @@ extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_l
   W8A8_MTRY(dalloc(m, &m->gu_bf16, (size_t)c.layers * 2 * F * H));
   W8A8_MTRY(dalloc(m, &m->stats, (size_t)c.layers * m->stats_stride() + H));
   W8A8_MTRY(dalloc(m, &m->r, (size_t)Mx * H));
+  W8A8_MTRY(dalloc(m, &m->r2, (size_t)Mx * H));
   W8A8_MTRY(dalloc(m, &m->a, (size_t)Mx * H));
   W8A8_MTRY(dalloc(m, &m->qkv, (size_t)Mx * m->qkv_dim));
   W8A8_MTRY(dalloc(m, &m->q, (size_t)Mx * m->q_dim));

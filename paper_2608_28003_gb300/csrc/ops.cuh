@@ -2,6 +2,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "gemv_small.cuh"
 
 namespace w8a8 {
 
@@ -25,23 +26,17 @@ w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* i
                                  uint16_t* xq_f16, float* s_x, cudaStream_t st);
 w8a8_status launch_act_absmax(const uint16_t* X, int T, int K, float* absmax, cudaStream_t st);
 
-// Bytes a decode GEMV asks L2 to fetch for a later kernel (the next linears' weights), so that
-// their HBM traffic overlaps the latency-bound kernels in between.  Only the row-owning decode
-// GEMV issues it; elsewhere it is ignored.
-struct L2Prefetch {
-  const void* ptr;
-  size_t bytes;
-};
-
 // kind: 0 bf16 output, 1 GeGLU, 2 fp32 logits (+ top-1)
 w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind, uint16_t* Y,
                             float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws, int sms, cudaStream_t st,
-                            const L2Prefetch* pf = nullptr);
+                            const ResNorm* rn = nullptr);
 w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, int M, const float* bias, int kind,
                             uint16_t* Y, float* logits, int32_t* top1, void* ws, int sms, cudaStream_t st,
-                            const L2Prefetch* pf = nullptr);
+                            const ResNorm* rn = nullptr);
 w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y, uint16_t* h_dbg,
-                    void* workspace, int sms, cudaStream_t st, const L2Prefetch* pf_gate_up = nullptr,
-                    const L2Prefetch* pf_down = nullptr);
+                    void* workspace, int sms, cudaStream_t st, const ResNorm* rn_gate_up = nullptr);
+// rn (decode only): the call's input is computed from the decoder's residual step inside the
+// decode GEMV (X is ignored); W8A8_ERR_SHAPE when the decode GEMV does not take the call.
+bool decode_gemv_takes(bool int8, int M, int N, int K, bool geglu, int sms);
 
 }  // namespace w8a8

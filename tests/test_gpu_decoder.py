@@ -142,9 +142,10 @@ def test_decode_step_graph_equals_eager_forward(B, setup):
 
 
 def test_decode_kernel_count(B, setup):
-    """A decode step launches the position update, embedding + norm, per layer q/k/v, attention
-    (QK-norm, RoPE and the cache write fused in), o, residual + norms, gate/up + GeGLU, down,
-    residual + norms, then lm_head.
+    """A decode step launches the position update, embedding + norm, per layer q/k/v (with the
+    previous layer's residual step fused in), attention (QK-norm, RoPE and the cache write fused
+    in), o, gate/up + GeGLU (with the post-attention residual step fused in) and down, then the
+    last residual step and lm_head.
     At decode the W8A8 linears of the layers fuse their per-token quantiser into the GEMV, so a
     W8A8 FFN or attention block costs no extra launch; W8A8 lm_head adds its quantiser."""
     dec, _, toks = setup[:3]
@@ -157,7 +158,7 @@ def test_decode_kernel_count(B, setup):
             dec.decode_kernels(2, want_logits=False)  # no graph of this (B, mask) without logits yet
         dec.decode_step(col, 21, logits=buf)
         counts[m] = dec.decode_kernels(2, want_logits=True)
-    assert counts[(0, 0, 0)] == 2 + 7 * L + 1
+    assert counts[(0, 0, 0)] == 2 + 5 * L + 2
     assert counts[(0b1001, 0b0010, 1)] - counts[(0, 0, 0)] == 1
 
 
