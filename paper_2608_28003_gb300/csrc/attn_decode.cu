@@ -14,10 +14,11 @@
 //    arithmetic of the prefill path (one warp per head, lane l holding the RoPE pairs
 //    (4l + e, 128 + 4l + e)); the CTA whose share ends at the new position also writes its key
 //    (bf16) and value to the cache and uses them from shared memory;
-//  * warp w handles query head w mod G and key group w / G of each tile: lane j computes the dot
-//    product of the scaled query (broadcast from shared memory) with key j (rows padded to 528
-//    bytes: the lanes of a shared-memory phase hit different bank groups), then the warp updates
-//    its running max, sum and output (lane l: dims 8l .. 8l+7) over its keys;
+//  * warp w handles query head w mod G and an even share (key group w / G) of each tile: one, two
+//    or four lanes per key compute its dot product with the scaled query (read from shared
+//    memory; key rows padded to 528 bytes, chunks rotated per lane so that the lanes of a
+//    shared-memory phase hit different bank groups), then the warp updates its running max, sum
+//    and output (lane l: dims 8l .. 8l+7) over its keys;
 //  * the warps of a head combine their partial (m, l, o) inside the CTA; each CTA then stores its
 //    per-head partials into CTA 0's shared memory (distributed shared memory stores, released by
 //    one cluster barrier), and CTA 0 combines them and writes the output row.
@@ -31,7 +32,7 @@ namespace {
 
 constexpr int kHd = 256;
 constexpr int kSplits = 8;        // CTAs per cluster (portable cluster size)
-constexpr int kMinKeys = 64;      // positions per working CTA, at least
+constexpr int kMinKeys = 16;      // positions per working CTA, at least
 constexpr int kTile = 64;         // positions per shared-memory tile
 constexpr int kKRow = 528;        // bytes per key row in shared memory (256 bf16 + 16 bytes of padding)
 constexpr int kVRow = 512;
@@ -141,7 +142,6 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
   const int G = s.n_q / s.n_kv, KG = kWarps / G;  // heads per key/value head; key groups per tile
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hw = warp % G, gw = warp / G;         // this warp's head (within the group) and key group
-  const int kpw = kTile / KG;                     // keys of a tile per warp
   // The position was set before this launch's chain began, and cached rows before it were
   // written by earlier launches: both may be read before waiting for the preceding kernel.
   const int pos = *pos0;
@@ -231,22 +231,30 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     const int j0 = kb + t * kTile;
     const uint8_t* kt = sm + kOffBuf;
     const uint8_t* vt = kt + kTile * kKRow;
-    for (int base = gw * kpw; base < (gw + 1) * kpw; base += 32) {
-      const int j = base + lane;          // key index within the tile
-      const int p = j0 + j;               // its position
-      const int nk = min(32, min((gw + 1) * kpw, ke - j0) - base);  // valid keys of this block
-      if (nk <= 0) break;
-      float sc = -INFINITY;
-      if (lane < nk) {
-        const uint4* kr = reinterpret_cast<const uint4*>(p == pos ? sm + kOffKNew : kt + j * kKRow);
+    // this warp's keys of the tile: an even share of the tile among the KG warps of its head
+    const int nt = min(kTile, ke - j0), per = (nt + KG - 1) / KG;
+    const int wk0 = gw * per, nkw = min(per, nt - wk0);
+    // lanes per key: 1 for 17-32 keys, 2 for 9-16, 4 for up to 8, so that short shares split each
+    // dot product over more lanes (lane = key slot * lpk + part; part p takes its own quarter /
+    // half of the 32 chunks, rotated so that a shared-memory phase hits 8 different bank groups)
+    const int lpk = nkw > 16 ? 1 : nkw > 8 ? 2 : 4;
+    const int nc = 32 / lpk, rot = lpk == 2 ? 4 : lpk == 4 ? 2 : 0;
+    const int kl = lane / lpk, part = lane % lpk;
+    for (int base = wk0; base < wk0 + nkw; base += 32 / lpk) {
+      const int nk = min(32 / lpk, wk0 + nkw - base);  // keys of this pass
+      const int j = base + kl;                          // key index within the tile
+      float dsum = 0.0f;
+      if (kl < nk) {
+        const uint4* kr = reinterpret_cast<const uint4*>(j0 + j == pos ? sm + kOffKNew : kt + j * kKRow);
         float d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll 8
-        for (int c = 0; c < kHd / 8; ++c) {
+        for (int it = 0; it < nc; ++it) {
+          const int c = part * nc + ((it + part * rot) & (nc - 1));
           float kx[8];
           unpack8_bf16(kr[c], kx);
           const float4 q0 = reinterpret_cast<const float4*>(qs + 8 * c)[0];
           const float4 q1 = reinterpret_cast<const float4*>(qs + 8 * c)[1];
-          float& dd = d[c & 3];
+          float& dd = d[it & 3];
           dd = fmaf(q0.x, kx[0], dd);
           dd = fmaf(q0.y, kx[1], dd);
           dd = fmaf(q0.z, kx[2], dd);
@@ -256,12 +264,14 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
           dd = fmaf(q1.z, kx[6], dd);
           dd = fmaf(q1.w, kx[7], dd);
         }
-        sc = (d[0] + d[1]) + (d[2] + d[3]);
+        dsum = (d[0] + d[1]) + (d[2] + d[3]);
       }
+      for (int o = 1; o < lpk; o <<= 1) dsum += __shfl_xor_sync(0xffffffffu, dsum, o);  // the key's parts
+      const float sc = kl < nk ? dsum : -INFINITY;
       const float m_new = fmaxf(m, warp_max_f(sc));
       const float corr = expf(m - m_new);  // 0 on the first block (m = -inf)
-      const float pr = lane < nk ? expf(sc - m_new) : 0.0f;
-      l = l * corr + warp_sum_f(pr);
+      const float pr = kl < nk ? expf(sc - m_new) : 0.0f;
+      l = l * corr + warp_sum_f(part == 0 ? pr : 0.0f);
 #pragma unroll
       for (int e = 0; e < 8; ++e) acc[e] *= corr;
       for (int jj0 = 0; jj0 < nk; jj0 += 4) {  // four keys' loads in flight
@@ -269,8 +279,8 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
         uint4 vv[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const int jj = jj0 + u < nk ? jj0 + u : 0;  // past the block: key 0 with weight 0
-          pj[u] = __shfl_sync(0xffffffffu, pr, jj);
+          const int jj = jj0 + u < nk ? jj0 + u : 0;  // past the pass: key 0 with weight 0
+          pj[u] = __shfl_sync(0xffffffffu, pr, jj * lpk);
           if (jj0 + u >= nk) pj[u] = 0.0f;
           const uint8_t* vrow = (j0 + base + jj == pos) ? sm + kOffVNew : vt + (base + jj) * kVRow;
           vv[u] = reinterpret_cast<const uint4*>(vrow)[lane];
