@@ -4,11 +4,12 @@
 // (tokens x K) and B (channels x K) tiles of 64 k arrive by 2-D TMA into 128-byte-swizzled shared
 // memory, S stages deep, continuously across tiles.  Accumulators live in tensor memory (all 512
 // columns), as a ring of BN-column slots, so the epilogue of one tile overlaps the MMAs of the next.
-//  * warp 4 (one thread) issues the TMA copies; warp 5 allocates tensor memory and one of its
+//  * warp 8 (one thread) issues the TMA copies; warp 9 allocates tensor memory and one of its
 //    threads issues tcgen05.mma (M = 128, N = BN, K = 16, fp32 accumulation) for each stage,
-//    commits the stage back to the producer and each finished slot to the epilogue; warps 0-3 are
-//    the epilogue, warp w reading TMEM lanes 32w .. 32w+31 (its tokens) with tcgen05.ld and
-//    handing the slot back.
+//    commits the stage back to the producer and each finished slot to the epilogue; warps 0-7 are
+//    the epilogue, warp w reading TMEM lanes 32 (w mod 4) .. +31 (its tokens) and column half
+//    w / 4 of the slot with tcgen05.ld, then handing the slot back.  Two epilogue warps per SM
+//    sub-partition keep its issue slots busy while the other waits on a dependency.
 //  * W8A8 path (BN = 128, four slots): both operands are INT8 codes stored as fp16 (exact).  Every
 //    product is an integer below 2^14, so a fp32 sum of at most 1024 of them is exact; the
 //    accumulator is therefore restarted every 1024 k (16 stages) in the next slot while the
@@ -18,7 +19,8 @@
 //    idle): one accumulator per tile over the whole k range.
 //  * epilogues: bf16 output, GeGLU of interleaved gate/up columns (16-column blocks: 8 gate, then
 //    the 8 matching up channels), or fp32 logits with the top-1 index (keys reduced with atomicMax,
-//    the last CTA to finish decodes them).
+//    the last CTA to finish decodes them); outputs leave through 32 x 32 shared-memory blocks and
+//    2-D TMA stores.
 // Every mbarrier wait is bounded: on timeout the kernel sets a bit of the error word, stops, waits
 // (bounded) for its own copies and MMAs in flight and frees its tensor memory.
 #include <algorithm>
@@ -36,16 +38,20 @@ constexpr int kBM = 128;
 constexpr int kSwz = 128;                // swizzle span in bytes (TMA and the MMA descriptors agree)
 constexpr int kBK = kSwz / 2;            // k per stage: one swizzle span of fp16 per row
 constexpr int kKbPerChunk = 1024 / kBK;  // stages per exact fp32 chunk of 1024 k
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;                    // two per TMEM lane quarter: one per column half
+constexpr int kProdWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1;
+constexpr int kThreads = 32 * (kEpiWarps + 2);
 constexpr uint32_t kTmemCols = 512;  // all of an SM's tensor memory: 2 (bf16) or 4 (W8A8) accumulator slots
 constexpr uint32_t kABytes = kBM * kBK * 2;
+constexpr int kStageBufBytes = 32 * 64;                  // one epilogue block: 32 rows of 64 bytes
+constexpr int kEpiSmem = kEpiWarps * 2 * kStageBufBytes;  // two blocks per epilogue warp
 
 template <bool kInt8, int kBN>
 struct TcGeo {
   static constexpr int BN = kBN;
   static constexpr uint32_t BBytes = BN * kBK * 2;
   static constexpr int S = (192 * 1024) / (int)(kABytes + BBytes);
-  static constexpr int Smem = S * (kABytes + BBytes) + 1024;
+  static constexpr int Smem = S * (kABytes + BBytes) + kEpiSmem + 1024;
 };
 
 // ---------------------------------------------------------------------------- tcgen05 helpers
@@ -82,25 +88,129 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar) : "memory");
 }
+// 32 consecutive accumulator columns of this thread's lane; the wait sits in the same statement, so
+// no use of r can be scheduled before the load has completed.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
       "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
         "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
         "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
         "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+      : "r"(taddr)
+      : "memory");
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return (uint32_t)f32_to_bf16_bits(a) | ((uint32_t)f32_to_bf16_bits(b) << 16);
 }
 
+// ------------------------------------------------------------------ epilogue through TMA stores
+// Each epilogue warp stages 32 rows x 32 columns of output (its rows, one 32-column group) in one of
+// its two shared-memory buffers and one lane stores the block with a 2-D TMA store (rows past M and
+// columns past N are clipped by the tensor map), so the global writes are whole rows, not one
+// 16-byte piece per thread and row.  A staged row is 64 bytes (32 bf16 or 16 fp32: fp32 output goes
+// out as two blocks of 16 columns) or 32 (GeGLU); the block is kept in the tensor map's swizzled
+// layout of that width (16-byte chunk c of row r at chunk c ^ ((r >> 1) & 3), or c ^ ((r >> 2) & 1)),
+// so the 16-byte stores of eight consecutive rows fall in eight different bank groups.
+
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const void* tmap, uint32_t src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];\n" ::"l"(
+                   reinterpret_cast<uint64_t>(tmap)),
+               "r"(src), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
+
+// The epilogue of 32 consecutive columns col0 .. col0+31 of this thread's row (lane of the warp
+// whose rows start at row0): bf16 output, GeGLU of the interleaved gate/up columns (two 16-column
+// blocks: 8 gate, then the 8 matching up channels), or fp32 logits with the row's running top-1 key.
+__device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap* tmY, uint32_t bufs, int& which,
+                                             int row0, int col0, int lane, const float (&v)[32], bool want_top,
+                                             unsigned long long& best) {
+  const int row = row0 + lane;
+  if (a.kind == EPI_F32 && want_top && row < a.M) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int col = col0 + j;
+      if (col < a.N) {
+        const unsigned long long key =
+            ((unsigned long long)float_order_key(v[j]) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)col);
+        best = key > best ? key : best;
+      }
+    }
+  }
+  if (a.kind == EPI_F32) {
+    if (!a.logits) return;  // top-1 only
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      if (lane == 0) bulk_wait_read1();  // the buffer's previous store has read it
+      __syncwarp();
+      const uint32_t buf = bufs + (uint32_t)(which * kStageBufBytes);
+      const uint32_t dst = buf + (uint32_t)(lane * 64), sw = (uint32_t)((lane >> 1) & 3);
+#pragma unroll
+      for (int j4 = 0; j4 < 4; ++j4)
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst + 16 * ((uint32_t)j4 ^ sw)),
+                     "f"(v[16 * h + 4 * j4]), "f"(v[16 * h + 4 * j4 + 1]), "f"(v[16 * h + 4 * j4 + 2]),
+                     "f"(v[16 * h + 4 * j4 + 3])
+                     : "memory");
+      fence_proxy_async_shared();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(tmY, buf, col0 + 16 * h, row0);
+        bulk_commit();
+      }
+      which ^= 1;
+    }
+    return;
+  }
+  if (lane == 0) bulk_wait_read1();  // the buffer's previous store has read it
+  __syncwarp();
+  const uint32_t buf = bufs + (uint32_t)(which * kStageBufBytes);
+  if (a.kind == EPI_GEGLU) {
+    uint32_t w[8];
+#pragma unroll
+    for (int hq = 0; hq < 2; ++hq)
+#pragma unroll
+      for (int j = 0; j < 8; j += 2)
+        w[4 * hq + j / 2] = pack_bf16x2(geglu_recipe(v[16 * hq + j], v[16 * hq + 8 + j]),
+                                        geglu_recipe(v[16 * hq + j + 1], v[16 * hq + 9 + j]));
+    const uint32_t dst = buf + (uint32_t)(lane * 32), sw = (uint32_t)((lane >> 2) & 1);
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst + 16 * sw), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+                 "r"(w[3])
+                 : "memory");
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst + 16 * (1u ^ sw)), "r"(w[4]), "r"(w[5]),
+                 "r"(w[6]), "r"(w[7])
+                 : "memory");
+  } else {
+    const uint32_t dst = buf + (uint32_t)(lane * 64), sw = (uint32_t)((lane >> 1) & 3);
+#pragma unroll
+    for (int j8 = 0; j8 < 4; ++j8)
+      asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst + 16 * ((uint32_t)j8 ^ sw)),
+                   "r"(pack_bf16x2(v[8 * j8], v[8 * j8 + 1])), "r"(pack_bf16x2(v[8 * j8 + 2], v[8 * j8 + 3])),
+                   "r"(pack_bf16x2(v[8 * j8 + 4], v[8 * j8 + 5])), "r"(pack_bf16x2(v[8 * j8 + 6], v[8 * j8 + 7]))
+                   : "memory");
+  }
+  fence_proxy_async_shared();
+  __syncwarp();
+  if (lane == 0) {
+    tma_store_2d(tmY, buf, a.kind == EPI_GEGLU ? col0 >> 1 : col0, row0);
+    bulk_commit();
+  }
+  which ^= 1;
+}
+
 template <bool kInt8, int kBN>
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const TcArgs a) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmY, const TcArgs a) {
   using GG = TcGeo<kInt8, kBN>;
   constexpr int BN = GG::BN, S = GG::S;
   constexpr int NSLOT = (int)kTmemCols / BN;  // accumulator slots in tensor memory
@@ -111,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t sA = base, sB = base + (uint32_t)S * kABytes;
+  const uint32_t sA = base, sB = base + (uint32_t)S * kABytes, stg = sB + (uint32_t)S * GG::BBytes;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + kBM - 1) / kBM);
   const int nkb = (a.K + kBK - 1) / kBK;
@@ -128,12 +238,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < NSLOT; ++b) {
       mbar_init(accf0 + 8 * b, 1);
-      mbar_init(acce0 + 8 * b, 128);
+      mbar_init(acce0 + 8 * b, 32 * kEpiWarps);
     }
     mbar_init(done, 1);
     fence_mbar_init();
   }
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(&tmem_slot)),
                  "r"(kTmemCols)
                  : "memory");
@@ -147,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // Persistent: CTA b takes tiles b, b + grid, ...; tile t covers channels (t mod NT) * BN and
   // tokens (t / NT) * 128, so neighbouring CTAs share the activation rows.
-  if (warp == 4) {
+  if (warp == kProdWarp) {
     // ---------------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
@@ -174,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16(kInt8 ? 0u : 1u, BN, kBM);
@@ -214,72 +324,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait_bounded(done, 0u, kWaitBudgetCycles)) atomicOr(a.err, DEVERR_DRAIN_WAIT);
     }
   } else {
-    // ---------------------------------------------------------------------- epilogue warps 0-3
-    const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
+    // ---------------------------------------------------------------------- epilogue warps 0-7
+    const int quad = warp & 3, half = warp >> 2;  // TMEM lane quarter (tokens), column half
+    const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
     const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
+    const uint32_t bufs = stg + (uint32_t)(warp * 2 * kStageBufBytes);
+    int which = 0;
     bool ok = true;
     int q = 0;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
       const int n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
-      const int row = m0 + 32 * warp + lane;
+      const int row = m0 + 32 * quad + lane;
       unsigned long long best = 0ull;
-      // the epilogue of 32 consecutive columns c0 .. c0+31 of this thread's row
       auto emit32 = [&](int c0, const float (&v)[32]) {
-        if (row >= a.M) return;
-        const int col0 = n0 + c0;
-        if (a.kind == EPI_GEGLU) {
-#pragma unroll
-          for (int hq = 0; hq < 2; ++hq) {  // two 16-column blocks: gate 0..7, up 8..15
-            const int cb = col0 + 16 * hq;
-            if (cb + 16 > a.N) continue;
-            float h[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) h[j] = geglu_recipe(v[16 * hq + j], v[16 * hq + 8 + j]);
-            uint4 w;
-            w.x = pack_bf16x2(h[0], h[1]);
-            w.y = pack_bf16x2(h[2], h[3]);
-            w.z = pack_bf16x2(h[4], h[5]);
-            w.w = pack_bf16x2(h[6], h[7]);
-            *reinterpret_cast<uint4*>(a.y + (size_t)row * (a.N >> 1) + (cb >> 1)) = w;
-          }
-        } else if (a.kind == EPI_BF16) {
-#pragma unroll
-          for (int j8 = 0; j8 < 4; ++j8) {
-            const int cb = col0 + 8 * j8;
-            if (cb + 8 <= a.N) {
-              uint4 w;
-              w.x = pack_bf16x2(v[8 * j8 + 0], v[8 * j8 + 1]);
-              w.y = pack_bf16x2(v[8 * j8 + 2], v[8 * j8 + 3]);
-              w.z = pack_bf16x2(v[8 * j8 + 4], v[8 * j8 + 5]);
-              w.w = pack_bf16x2(v[8 * j8 + 6], v[8 * j8 + 7]);
-              *reinterpret_cast<uint4*>(a.y + (size_t)row * a.N + cb) = w;
-            }
-          }
-        } else {
-#pragma unroll
-          for (int j4 = 0; j4 < 8; ++j4) {
-            const int cb = col0 + 4 * j4;
-            if (cb + 4 <= a.N && a.logits)
-              *reinterpret_cast<float4*>(a.logits + (size_t)row * a.N + cb) =
-                  make_float4(v[4 * j4], v[4 * j4 + 1], v[4 * j4 + 2], v[4 * j4 + 3]);
-          }
-          if (want_top) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const int col = col0 + j;
-              if (col < a.N) {
-                const unsigned long long key = ((unsigned long long)float_order_key(v[j]) << 32) |
-                                               (unsigned long long)(0xFFFFFFFFu - (uint32_t)col);
-                best = key > best ? key : best;
-              }
-            }
-          }
-        }
+        stage_cols32(a, &tmY, bufs, which, m0 + 32 * quad, n0 + c0, lane, v, want_top, best);
       };
       if constexpr (kInt8) {
-        int isum[BN];
+        constexpr int HC = BN / 2;  // this warp's columns: half * HC .. + HC - 1
+        int isum[HC];
 #pragma unroll
-        for (int j = 0; j < BN; ++j) isum[j] = 0;
+        for (int j = 0; j < HC; ++j) isum[j] = 0;
         for (int c = 0; c < nchunks; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
@@ -289,9 +353,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
 #pragma unroll
-          for (int g = 0; g < BN / 32; ++g) {
+          for (int g = 0; g < HC / 32; ++g) {
             uint32_t r[32];
-            tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
+            tmem_ld32(lane_base + (uint32_t)(slot * BN + half * HC + 32 * g), r);
 #pragma unroll
             for (int j = 0; j < 32; ++j) isum[32 * g + j] += __float2int_rn(__uint_as_float(r[j]));
           }
@@ -301,11 +365,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
-        for (int g = 0; g < BN / 32; ++g) {
+        for (int g = 0; g < HC / 32; ++g) {
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            const int col = n0 + 32 * g + j;
+            const int col = n0 + half * HC + 32 * g + j;
             float y = 0.0f;
             if (col < a.N) {
               y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * g + j]));
@@ -314,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             v[j] = y;
           }
-          emit32(32 * g, v);
+          emit32(half * HC + 32 * g, v);
         }
       } else {
         const int slot = q % NSLOT;
@@ -325,7 +389,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
 #pragma unroll 1
-        for (int g = 0; g < BN / 32; ++g) {
+        for (int g = half * (BN / 64); g < (half + 1) * (BN / 64); ++g) {
           uint32_t r[32];
           tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
           float v[32];
@@ -344,19 +408,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (want_top && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
     }
+    if (lane == 0) bulk_wait_all();  // this warp's output stores have completed
+    __syncwarp();
     // top-1 across the grid: the last CTA to finish decodes the per-row keys and clears them
     if (want_top) {
       __threadfence();
-      named_bar_sync(1, 128);
+      named_bar_sync(1, 32 * kEpiWarps);
       if (threadIdx.x == 0) {
         const unsigned int prev = atomicAdd(a.grid_counter, 1u);
         s_flag = prev == gridDim.x - 1;
         if (s_flag) *a.grid_counter = 0u;
       }
-      named_bar_sync(1, 128);
+      named_bar_sync(1, 32 * kEpiWarps);
       if (s_flag) {
         __threadfence();
-        for (int t = threadIdx.x; t < a.M; t += 128) {
+        for (int t = threadIdx.x; t < a.M; t += 32 * kEpiWarps) {
           const unsigned long long key = atomicExch(a.top_keys + t, 0ull);
           a.top1[t] = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
         }
@@ -365,10 +431,315 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
   }
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(kTmemCols) : "memory");
   }
+}
+
+// ------------------------------------------------------------------------- 2-CTA variant
+// The same GEMM on CTA pairs (clusters of 2) with tcgen05.mma.cta_group::2: a pair computes a tile
+// of 256 tokens x BN channels; CTA r holds tokens m0 + 128 r .. +127 of A and channels
+// n0 + r BN/2 .. + BN/2 - 1 of B in its shared memory, so each SM loads half of the B tile, and its
+// tensor memory receives its 128 rows of D.  CTA 0 of the pair issues the MMAs; both CTAs' TMA
+// copies complete on CTA 0's stage barrier; the stage and accumulator barriers of both CTAs are
+// signalled by multicast commits; both CTAs' epilogue threads hand the slot back to CTA 0.
+template <bool kInt8, int kBN>
+struct Tc2Geo {
+  static constexpr int BN = kBN;
+  static constexpr uint32_t BHalf = (kBN / 2) * kBK * 2;
+  static constexpr int S = (192 * 1024) / (int)(kABytes + BHalf);
+  static constexpr int Smem = S * (kABytes + BHalf) + kEpiSmem + 1024;
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];\n" ::"r"(cluster_addr) : "memory");
+}
+// 2-D TMA load into this CTA's shared memory whose completion is counted on an mbarrier of either
+// CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap, int c0, int c1, uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+      "[%4];\n" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void tc2_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                        uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// arrive on the barrier at this shared-memory offset in both CTAs of the pair once the MMAs issued
+// so far have completed
+__device__ __forceinline__ void tc2_commit_both(uint32_t bar) {
+  const uint16_t mask = 0x3;
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n" ::"r"(bar),
+      "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ void tc2_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar) : "memory");
+}
+
+template <bool kInt8, int kBN>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmY, const TcArgs a) {
+  using GG = Tc2Geo<kInt8, kBN>;
+  constexpr int BN = GG::BN, S = GG::S;
+  constexpr int NSLOT = (int)kTmemCols / BN;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
+  __shared__ uint32_t tmem_slot;
+  __shared__ int s_flag;
+
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const uint32_t sA = base, sB = base + (uint32_t)S * kABytes, stg = sB + (uint32_t)S * GG::BHalf;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + 2 * kBM - 1) / (2 * kBM));
+  const int nkb = (a.K + kBK - 1) / kBK;
+  const int nchunks = kInt8 ? (nkb + kKbPerChunk - 1) / kKbPerChunk : 1;
+  const int kb_per_chunk = kInt8 ? kKbPerChunk : nkb;
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
+                 done = acce0 + 8 * NSLOT;
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int b = 0; b < NSLOT; ++b) {
+      mbar_init(accf0 + 8 * b, 1);
+      mbar_init(acce0 + 8 * b, 2 * 32 * kEpiWarps);  // both CTAs' epilogue threads
+    }
+    mbar_init(done, 1);
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;\n" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers exist before either signals the other
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+  const uint32_t full_lead = map_to_rank(full0, 0), acce_lead = map_to_rank(acce0, 0);
+  pdl_wait();
+
+  if (warp == kProdWarp) {
+    // ---------------------------------------------------------------------- TMA producers (both CTAs)
+    if (lane == 0) {
+      bool ok = true;
+      int g = 0;
+      for (int t = pair; t < tiles && ok; t += npairs) {
+        const int n0 = (t % NT) * BN, m0 = (t / NT) * 2 * kBM;
+        for (int kb = 0; kb < nkb; ++kb, ++g) {
+          const int s = g % S;
+          if (!mbar_wait_bounded(empty0 + 8 * s, (uint32_t)(((g / S) & 1) ^ 1), kWaitBudgetCycles)) {
+            ok = false;
+            break;
+          }
+          if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * s, 2 * (kABytes + GG::BHalf));
+          tma_load_2d_pair(sA + (uint32_t)s * kABytes, &tmA, kb * kBK, m0 + kBM * (int)rank, full_lead + 8 * s);
+          tma_load_2d_pair(sB + (uint32_t)s * GG::BHalf, &tmB, kb * kBK, n0 + (BN / 2) * (int)rank, full_lead + 8 * s);
+        }
+      }
+      if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
+      // the last stages are consumed (so their copies have landed) before this CTA can exit
+      for (int j = g > S ? g - S : 0; j < g; ++j) {
+        if (!mbar_wait_bounded(empty0 + 8 * (j % S), (uint32_t)((j / S) & 1), kWaitBudgetCycles)) {
+          atomicOr(a.err, DEVERR_DRAIN_WAIT);
+          break;
+        }
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------------- MMA issuer (CTA 0)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_f16(kInt8 ? 0u : 1u, BN, 2 * kBM);
+      bool ok = true;
+      int g = 0, q = 0;
+      for (int t = pair; t < tiles && ok; t += npairs) {
+        for (int c = 0; c < nchunks && ok; ++c, ++q) {
+          const int slot = q % NSLOT;
+          if (q >= NSLOT &&
+              !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + (uint32_t)(slot * BN);
+          const int kb0 = c * kb_per_chunk, kb1 = min(nkb, kb0 + kb_per_chunk);
+          for (int kb = kb0; kb < kb1; ++kb, ++g) {
+            const int s = g % S;
+            if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int k16 = 0; k16 < kBK / 16; ++k16) {
+              const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
+              const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BHalf + 32u * k16);
+              tc2_mma(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
+            }
+            tc2_commit_both(empty0 + 8 * s);
+          }
+          if (ok) tc2_commit_both(accf0 + 8 * slot);
+        }
+      }
+      if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
+      tc2_commit(done);
+      if (!mbar_wait_bounded(done, 0u, kWaitBudgetCycles)) atomicOr(a.err, DEVERR_DRAIN_WAIT);
+    }
+  } else {
+    // ---------------------------------------------------------------------- epilogue warps 0-7 (both CTAs)
+    const int quad = warp & 3, half = warp >> 2;
+    const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
+    const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
+    const uint32_t bufs = stg + (uint32_t)(warp * 2 * kStageBufBytes);
+    int which = 0;
+    bool ok = true;
+    int q = 0;
+    for (int t = pair; t < tiles && ok; t += npairs) {
+      const int n0 = (t % NT) * BN, m0 = (t / NT) * 2 * kBM;
+      const int row = m0 + kBM * (int)rank + 32 * quad + lane;
+      unsigned long long best = 0ull;
+      auto emit = [&](int c0, const float (&v)[32]) {
+        stage_cols32(a, &tmY, bufs, which, m0 + kBM * (int)rank + 32 * quad, n0 + c0, lane, v, want_top, best);
+      };
+      if constexpr (kInt8) {
+        constexpr int HC = BN / 2;  // this warp's columns: half * HC .. + HC - 1
+        int isum[HC];
+#pragma unroll
+        for (int j = 0; j < HC; ++j) isum[j] = 0;
+        for (int c = 0; c < nchunks; ++c, ++q) {
+          const int slot = q % NSLOT;
+          if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
+            ok = false;
+            atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int g = 0; g < HC / 32; ++g) {
+            uint32_t r[32];
+            tmem_ld32(lane_base + (uint32_t)(slot * BN + half * HC + 32 * g), r);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) isum[32 * g + j] += __float2int_rn(__uint_as_float(r[j]));
+          }
+          tc_fence_before();
+          mbar_arrive_cluster(acce_lead + 8 * slot);
+        }
+        if (!ok) break;
+        const float sx = row < a.M ? a.s_x[row] : 0.0f;
+#pragma unroll
+        for (int g = 0; g < HC / 32; ++g) {
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int col = n0 + half * HC + 32 * g + j;
+            float y = 0.0f;
+            if (col < a.N) {
+              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * g + j]));
+              if (a.bias) y = __fadd_rn(y, a.bias[col]);
+              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * g + j];
+            }
+            v[j] = y;
+          }
+          emit(half * HC + 32 * g, v);
+        }
+      } else {
+        const int slot = q % NSLOT;
+        if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
+          ok = false;
+          atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+          break;
+        }
+        tc_fence_after();
+#pragma unroll 1
+        for (int g = half * (BN / 64); g < (half + 1) * (BN / 64); ++g) {
+          uint32_t r[32];
+          tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int col = n0 + 32 * g + j;
+            float y = __uint_as_float(r[j]);
+            if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
+            v[j] = y;
+          }
+          emit(32 * g, v);
+        }
+        tc_fence_before();
+        mbar_arrive_cluster(acce_lead + 8 * slot);
+        ++q;
+      }
+      if (want_top && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
+    }
+    if (lane == 0) bulk_wait_all();  // this warp's output stores have completed
+    __syncwarp();
+    if (want_top) {
+      __threadfence();
+      named_bar_sync(1, 32 * kEpiWarps);
+      if (threadIdx.x == 0) {
+        const unsigned int prev = atomicAdd(a.grid_counter, 1u);
+        s_flag = prev == gridDim.x - 1;
+        if (s_flag) *a.grid_counter = 0u;
+      }
+      named_bar_sync(1, 32 * kEpiWarps);
+      if (s_flag) {
+        __threadfence();
+        for (int t = threadIdx.x; t < a.M; t += 32 * kEpiWarps) {
+          const unsigned long long key = atomicExch(a.top_keys + t, 0ull);
+          a.top1[t] = (int32_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+        }
+      }
+    }
+    tc_fence_before();
+  }
+  __syncthreads();
+  cluster_sync_all();  // neither CTA leaves while the other may still signal its barriers
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(kTmemCols) : "memory");
+  }
+}
+
+// The output's tensor map for the epilogue's TMA stores: 32 rows x 32 bf16 columns, or 16 (GeGLU
+// output, fp32 logits), swizzled over the staged row's width.
+w8a8_status make_out_map(const TcArgs& a, CUtensorMap* ty, const CUtensorMap& unused) {
+  if (a.kind == EPI_BF16) return make_tmap_2d(ty, a.y, 2, (uint64_t)a.N, (uint64_t)a.M, (uint64_t)a.N * 2, 32, 32, 64);
+  if (a.kind == EPI_GEGLU)
+    return make_tmap_2d(ty, a.y, 2, (uint64_t)(a.N / 2), (uint64_t)a.M, (uint64_t)a.N, 16, 32, 32);
+  if (a.logits) return make_tmap_2d(ty, a.logits, 4, (uint64_t)a.N, (uint64_t)a.M, (uint64_t)a.N * 4, 16, 32, 64);
+  *ty = unused;  // top-1 only: nothing is stored
+  return W8A8_OK;
 }
 
 template <bool kInt8, int kBN>
@@ -384,9 +755,33 @@ w8a8_status launch_t(const TcArgs& a, cudaStream_t st) {
   CUtensorMap ta, tb;
   W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, kBM, kSwz));
   W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN, kSwz));
+  CUtensorMap ty;
+  W8A8_TRY(make_out_map(a, &ty, ta));
   const long long tiles = (long long)((a.N + GG::BN - 1) / GG::BN) * ((a.M + kBM - 1) / kBM);
   const dim3 grid((unsigned)std::min<long long>(tiles, device_sms()));
-  W8A8_CUDA(launch_pdl(gemm_tc_kernel<kInt8, kBN>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, a));
+  W8A8_CUDA(launch_pdl(gemm_tc_kernel<kInt8, kBN>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, ty, a));
+  return W8A8_OK;
+}
+
+template <bool kInt8, int kBN>
+w8a8_status launch_t2(const TcArgs& a, cudaStream_t st) {
+  using GG = Tc2Geo<kInt8, kBN>;
+  static bool attr_set[64] = {};
+  int dev = 0;
+  W8A8_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc2_kernel<kInt8, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
+    attr_set[dev] = true;
+  }
+  CUtensorMap ta, tb;
+  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, kBM, kSwz));
+  W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN / 2, kSwz));
+  CUtensorMap ty;
+  W8A8_TRY(make_out_map(a, &ty, ta));
+  const long long tiles = (long long)((a.N + GG::BN - 1) / GG::BN) * ((a.M + 2 * kBM - 1) / (2 * kBM));
+  const long long pairs = std::min<long long>(tiles, device_sms() / 2);
+  W8A8_CUDA(launch_pdl(gemm_tc2_kernel<kInt8, kBN>, dim3((unsigned)(2 * pairs)), dim3(kThreads), (size_t)GG::Smem, st,
+                       ta, tb, ty, a));
   return W8A8_OK;
 }
 
@@ -405,11 +800,20 @@ w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st) {
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  // bf16: 256-channel tiles unless that leaves SMs without a tile
+  // bf16: CTA pairs on 256 x 256 tiles when they fill the SMs, else single CTAs on 256- or
+  // 128-channel tiles
+  const int sms = device_sms();
+  const long long pair_tiles = (long long)((a.N + 255) / 256) * ((a.M + 2 * kBM - 1) / (2 * kBM));
   const long long tiles256 = (long long)((a.N + 255) / 256) * ((a.M + kBM - 1) / kBM);
-  const w8a8_status s = int8_codes                    ? launch_t<true, 128>(a, st)
-                        : tiles256 >= device_sms() ? launch_t<false, 256>(a, st)
-                                                   : launch_t<false, 128>(a, st);
+  w8a8_status s;
+  if (int8_codes)
+    s = launch_t<true, 128>(a, st);
+  else if (pair_tiles >= sms / 2)
+    s = launch_t2<false, 256>(a, st);
+  else if (tiles256 >= sms)
+    s = launch_t<false, 256>(a, st);
+  else
+    s = launch_t<false, 128>(a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }
