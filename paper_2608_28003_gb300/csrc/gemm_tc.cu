@@ -3,20 +3,22 @@
 // A persistent grid (one CTA per SM) walks the output tiles of 128 tokens x BN channels.  A
 // (tokens x K) and B (channels x K) tiles of 64 k arrive by 2-D TMA into 128-byte-swizzled shared
 // memory, S stages deep, continuously across tiles.  Accumulators live in tensor memory (all 512
-// columns), as a ring of BN-column slots, so the epilogue of one tile overlaps the MMAs of the next.
-//  * warp 8 (one thread) issues the TMA copies; warp 9 allocates tensor memory and one of its
+// columns), as a ring of slots (BN rounded up to 128 or 256 columns), so the epilogue of one tile
+// overlaps the MMAs of the next.
+//  * warp 16 (one thread) issues the TMA copies; warp 17 allocates tensor memory and one of its
 //    threads issues tcgen05.mma (M = 128, N = BN, K = 16, fp32 accumulation) for each stage,
-//    commits the stage back to the producer and each finished slot to the epilogue; warps 0-7 are
-//    the epilogue, warp w reading TMEM lanes 32 (w mod 4) .. +31 (its tokens) and column half
-//    w / 4 of the slot with tcgen05.ld, then handing the slot back.  Two epilogue warps per SM
-//    sub-partition keep its issue slots busy while the other waits on a dependency.
-//  * W8A8 path (BN = 128, four slots): both operands are INT8 codes stored as fp16 (exact).  Every
-//    product is an integer below 2^14, so a fp32 sum of at most 1024 of them is exact; the
-//    accumulator is therefore restarted every 1024 k (16 stages) in the next slot while the
-//    epilogue folds the finished one into INT32 registers, and the INT32 result is exact in any
-//    order (Eq. gemm-final).  The epilogue then dequantises fl(fl(s_x s_w) acc) (+ bias).
-//  * bf16 path (BN = 256 and two slots, or BN = 128 and four when 256-wide tiles would leave SMs
-//    idle): one accumulator per tile over the whole k range.
+//    commits the stage back to the producer and each finished slot to the epilogue; warps 0-15 are
+//    the epilogue, warp w reading TMEM lanes 32 (w mod 4) .. +31 (its tokens) and column quarter
+//    w / 4 of the slot with tcgen05.ld, then handing the slot back.  Four epilogue warps per SM
+//    sub-partition keep its issue slots busy while one waits on a dependency.
+//  * tiles: BN = 128 (four slots) on single CTAs, or BN = 192 / 256 (two slots) on CTA pairs of
+//    256 tokens (cta_group::2, below), chosen by a cost model of the waves.
+//  * W8A8 path: both operands are INT8 codes stored as fp16 (exact).  Every product is an integer
+//    below 2^14, so a fp32 sum of at most 1024 of them is exact; the accumulator is therefore
+//    restarted every 1024 k (16 stages) in the next slot while the epilogue folds the finished one
+//    into INT32 registers, and the INT32 result is exact in any order (Eq. gemm-final).  The
+//    epilogue then dequantises fl(fl(s_x s_w) acc) (+ bias).
+//  * bf16 path: one accumulator per tile over the whole k range.
 //  * epilogues: bf16 output, GeGLU of interleaved gate/up columns (16-column blocks: 8 gate, then
 //    the 8 matching up channels), or fp32 logits with the top-1 index (keys reduced with atomicMax,
 //    the last CTA to finish decodes them); outputs leave through 32 x 32 shared-memory blocks and
@@ -38,13 +40,18 @@ constexpr int kBM = 128;
 constexpr int kSwz = 128;                // swizzle span in bytes (TMA and the MMA descriptors agree)
 constexpr int kBK = kSwz / 2;            // k per stage: one swizzle span of fp16 per row
 constexpr int kKbPerChunk = 1024 / kBK;  // stages per exact fp32 chunk of 1024 k
-constexpr int kEpiWarps = 8;                    // two per TMEM lane quarter: one per column half
+constexpr int kEpiWarps = 16;                   // four per TMEM lane quarter: one per column quarter
+constexpr int kParts = kEpiWarps / 4;
 constexpr int kProdWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1;
 constexpr int kThreads = 32 * (kEpiWarps + 2);
 constexpr uint32_t kTmemCols = 512;  // all of an SM's tensor memory: 2 (bf16) or 4 (W8A8) accumulator slots
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kStageBufBytes = 32 * 64;                  // one epilogue block: 32 rows of 64 bytes
-constexpr int kEpiSmem = kEpiWarps * 2 * kStageBufBytes;  // two blocks per epilogue warp
+constexpr int kEpiSmem = kEpiWarps * kStageBufBytes;  // one block per epilogue warp
+
+// Tensor-memory columns of one accumulator slot: BN rounded up to a power of two, so every slot
+// starts on a 128-column boundary.
+__host__ __device__ constexpr int slot_cols(int bn) { return bn <= 128 ? 128 : bn <= 256 ? 256 : 512; }
 
 template <bool kInt8, int kBN>
 struct TcGeo {
@@ -108,10 +115,11 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 }
 
 // ------------------------------------------------------------------ epilogue through TMA stores
-// Each epilogue warp stages 32 rows x 32 columns of output (its rows, one 32-column group) in one of
-// its two shared-memory buffers and one lane stores the block with a 2-D TMA store (rows past M and
+// Each epilogue warp stages 32 rows x 32 columns of output (its rows, one 32-column group) in its
+// 2 KB shared-memory block and one lane stores the block with a 2-D TMA store (rows past M and
 // columns past N are clipped by the tensor map), so the global writes are whole rows, not one
-// 16-byte piece per thread and row.  A staged row is 64 bytes (32 bf16 or 16 fp32: fp32 output goes
+// 16-byte piece per thread and row; the warp waits for the store to have read the block before it
+// refills it (the other warps of its sub-partition issue meanwhile).  A staged row is 64 bytes (32 bf16 or 16 fp32: fp32 output goes
 // out as two blocks of 16 columns) or 32 (GeGLU); the block is kept in the tensor map's swizzled
 // layout of that width (16-byte chunk c of row r at chunk c ^ ((r >> 1) & 3), or c ^ ((r >> 2) & 1)),
 // so the 16-byte stores of eight consecutive rows fall in eight different bank groups.
@@ -126,13 +134,13 @@ __device__ __forceinline__ void tma_store_2d(const void* tmap, uint32_t src, int
                : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
 
 // The epilogue of 32 consecutive columns col0 .. col0+31 of this thread's row (lane of the warp
 // whose rows start at row0): bf16 output, GeGLU of the interleaved gate/up columns (two 16-column
 // blocks: 8 gate, then the 8 matching up channels), or fp32 logits with the row's running top-1 key.
-__device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap* tmY, uint32_t bufs, int& which,
+__device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap* tmY, uint32_t buf,
                                              int row0, int col0, int lane, const float (&v)[32], bool want_top,
                                              unsigned long long& best) {
   const int row = row0 + lane;
@@ -151,9 +159,8 @@ __device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap*
     if (!a.logits) return;  // top-1 only
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      if (lane == 0) bulk_wait_read1();  // the buffer's previous store has read it
+      if (lane == 0) bulk_wait_read0();  // the previous store has read the block
       __syncwarp();
-      const uint32_t buf = bufs + (uint32_t)(which * kStageBufBytes);
       const uint32_t dst = buf + (uint32_t)(lane * 64), sw = (uint32_t)((lane >> 1) & 3);
 #pragma unroll
       for (int j4 = 0; j4 < 4; ++j4)
@@ -167,13 +174,11 @@ __device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap*
         tma_store_2d(tmY, buf, col0 + 16 * h, row0);
         bulk_commit();
       }
-      which ^= 1;
     }
     return;
   }
-  if (lane == 0) bulk_wait_read1();  // the buffer's previous store has read it
+  if (lane == 0) bulk_wait_read0();  // the previous store has read the block
   __syncwarp();
-  const uint32_t buf = bufs + (uint32_t)(which * kStageBufBytes);
   if (a.kind == EPI_GEGLU) {
     uint32_t w[8];
 #pragma unroll
@@ -204,7 +209,6 @@ __device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap*
     tma_store_2d(tmY, buf, a.kind == EPI_GEGLU ? col0 >> 1 : col0, row0);
     bulk_commit();
   }
-  which ^= 1;
 }
 
 template <bool kInt8, int kBN>
@@ -213,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ CUtensorMap tmY, const TcArgs a) {
   using GG = TcGeo<kInt8, kBN>;
   constexpr int BN = GG::BN, S = GG::S;
-  constexpr int NSLOT = (int)kTmemCols / BN;  // accumulator slots in tensor memory
+  constexpr int SC = slot_cols(BN), NSLOT = (int)kTmemCols / SC;  // accumulator slots in tensor memory
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
   __shared__ uint32_t tmem_slot;
@@ -299,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d = tmem + (uint32_t)(slot * BN);
+          const uint32_t d = tmem + (uint32_t)(slot * SC);
           const int kb0 = c * kb_per_chunk, kb1 = min(nkb, kb0 + kb_per_chunk);
           for (int kb = kb0; kb < kb1; ++kb, ++g) {
             const int s = g % S;
@@ -324,12 +328,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait_bounded(done, 0u, kWaitBudgetCycles)) atomicOr(a.err, DEVERR_DRAIN_WAIT);
     }
   } else {
-    // ---------------------------------------------------------------------- epilogue warps 0-7
-    const int quad = warp & 3, half = warp >> 2;  // TMEM lane quarter (tokens), column half
+    // ---------------------------------------------------------------------- epilogue warps 0-15
+    const int quad = warp & 3, part = warp >> 2;  // TMEM lane quarter (tokens), column quarter
     const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
     const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
-    const uint32_t bufs = stg + (uint32_t)(warp * 2 * kStageBufBytes);
-    int which = 0;
+    const uint32_t buf = stg + (uint32_t)(warp * kStageBufBytes);
     bool ok = true;
     int q = 0;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
@@ -337,13 +340,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row = m0 + 32 * quad + lane;
       unsigned long long best = 0ull;
       auto emit32 = [&](int c0, const float (&v)[32]) {
-        stage_cols32(a, &tmY, bufs, which, m0 + 32 * quad, n0 + c0, lane, v, want_top, best);
+        stage_cols32(a, &tmY, buf, m0 + 32 * quad, n0 + c0, lane, v, want_top, best);
       };
       if constexpr (kInt8) {
-        constexpr int HC = BN / 2;  // this warp's columns: half * HC .. + HC - 1
-        int isum[HC];
+        constexpr int NG = (BN / 32 + kParts - 1) / kParts;  // this warp's 32-column groups: part + kParts i
+        int isum[32 * NG];
 #pragma unroll
-        for (int j = 0; j < HC; ++j) isum[j] = 0;
+        for (int j = 0; j < 32 * NG; ++j) isum[j] = 0;
         for (int c = 0; c < nchunks; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
@@ -353,11 +356,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
 #pragma unroll
-          for (int g = 0; g < HC / 32; ++g) {
+          for (int i = 0; i < NG; ++i) {
+            const int g = part + kParts * i;
+            if (g >= BN / 32) break;
             uint32_t r[32];
-            tmem_ld32(lane_base + (uint32_t)(slot * BN + half * HC + 32 * g), r);
+            tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) isum[32 * g + j] += __float2int_rn(__uint_as_float(r[j]));
+            for (int j = 0; j < 32; ++j) isum[32 * i + j] += __float2int_rn(__uint_as_float(r[j]));
           }
           tc_fence_before();
           mbar_arrive(acce0 + 8 * slot);
@@ -365,20 +370,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
-        for (int g = 0; g < HC / 32; ++g) {
+        for (int i = 0; i < NG; ++i) {
+          const int g = part + kParts * i;
+          if (g >= BN / 32) break;
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            const int col = n0 + half * HC + 32 * g + j;
+            const int col = n0 + 32 * g + j;
             float y = 0.0f;
             if (col < a.N) {
-              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * g + j]));
+              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * i + j]));
               if (a.bias) y = __fadd_rn(y, a.bias[col]);
-              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * g + j];
+              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * i + j];
             }
             v[j] = y;
           }
-          emit32(half * HC + 32 * g, v);
+          emit32(32 * g, v);
         }
       } else {
         const int slot = q % NSLOT;
@@ -389,9 +396,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
 #pragma unroll 1
-        for (int g = half * (BN / 64); g < (half + 1) * (BN / 64); ++g) {
+        for (int g = part; g < BN / 32; g += kParts) {
           uint32_t r[32];
-          tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
+          tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -505,7 +512,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     const __grid_constant__ CUtensorMap tmY, const TcArgs a) {
   using GG = Tc2Geo<kInt8, kBN>;
   constexpr int BN = GG::BN, S = GG::S;
-  constexpr int NSLOT = (int)kTmemCols / BN;
+  constexpr int SC = slot_cols(BN), NSLOT = (int)kTmemCols / SC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
   __shared__ uint32_t tmem_slot;
@@ -593,7 +600,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d = tmem + (uint32_t)(slot * BN);
+          const uint32_t d = tmem + (uint32_t)(slot * SC);
           const int kb0 = c * kb_per_chunk, kb1 = min(nkb, kb0 + kb_per_chunk);
           for (int kb = kb0; kb < kb1; ++kb, ++g) {
             const int s = g % S;
@@ -618,12 +625,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (!mbar_wait_bounded(done, 0u, kWaitBudgetCycles)) atomicOr(a.err, DEVERR_DRAIN_WAIT);
     }
   } else {
-    // ---------------------------------------------------------------------- epilogue warps 0-7 (both CTAs)
-    const int quad = warp & 3, half = warp >> 2;
+    // ---------------------------------------------------------------------- epilogue warps 0-15 (both CTAs)
+    const int quad = warp & 3, part = warp >> 2;
     const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
     const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
-    const uint32_t bufs = stg + (uint32_t)(warp * 2 * kStageBufBytes);
-    int which = 0;
+    const uint32_t buf = stg + (uint32_t)(warp * kStageBufBytes);
     bool ok = true;
     int q = 0;
     for (int t = pair; t < tiles && ok; t += npairs) {
@@ -631,13 +637,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int row = m0 + kBM * (int)rank + 32 * quad + lane;
       unsigned long long best = 0ull;
       auto emit = [&](int c0, const float (&v)[32]) {
-        stage_cols32(a, &tmY, bufs, which, m0 + kBM * (int)rank + 32 * quad, n0 + c0, lane, v, want_top, best);
+        stage_cols32(a, &tmY, buf, m0 + kBM * (int)rank + 32 * quad, n0 + c0, lane, v, want_top, best);
       };
       if constexpr (kInt8) {
-        constexpr int HC = BN / 2;  // this warp's columns: half * HC .. + HC - 1
-        int isum[HC];
+        constexpr int NG = (BN / 32 + kParts - 1) / kParts;  // this warp's 32-column groups: part + kParts i
+        int isum[32 * NG];
 #pragma unroll
-        for (int j = 0; j < HC; ++j) isum[j] = 0;
+        for (int j = 0; j < 32 * NG; ++j) isum[j] = 0;
         for (int c = 0; c < nchunks; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
@@ -647,11 +653,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
 #pragma unroll
-          for (int g = 0; g < HC / 32; ++g) {
+          for (int i = 0; i < NG; ++i) {
+            const int g = part + kParts * i;
+            if (g >= BN / 32) break;
             uint32_t r[32];
-            tmem_ld32(lane_base + (uint32_t)(slot * BN + half * HC + 32 * g), r);
+            tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) isum[32 * g + j] += __float2int_rn(__uint_as_float(r[j]));
+            for (int j = 0; j < 32; ++j) isum[32 * i + j] += __float2int_rn(__uint_as_float(r[j]));
           }
           tc_fence_before();
           mbar_arrive_cluster(acce_lead + 8 * slot);
@@ -659,20 +667,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (!ok) break;
         const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
-        for (int g = 0; g < HC / 32; ++g) {
+        for (int i = 0; i < NG; ++i) {
+          const int g = part + kParts * i;
+          if (g >= BN / 32) break;
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            const int col = n0 + half * HC + 32 * g + j;
+            const int col = n0 + 32 * g + j;
             float y = 0.0f;
             if (col < a.N) {
-              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * g + j]));
+              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * i + j]));
               if (a.bias) y = __fadd_rn(y, a.bias[col]);
-              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * g + j];
+              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * i + j];
             }
             v[j] = y;
           }
-          emit(half * HC + 32 * g, v);
+          emit(32 * g, v);
         }
       } else {
         const int slot = q % NSLOT;
@@ -683,9 +693,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
 #pragma unroll 1
-        for (int g = half * (BN / 64); g < (half + 1) * (BN / 64); ++g) {
+        for (int g = part; g < BN / 32; g += kParts) {
           uint32_t r[32];
-          tmem_ld32(lane_base + (uint32_t)(slot * BN + 32 * g), r);
+          tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -785,6 +795,25 @@ w8a8_status launch_t2(const TcArgs& a, cudaStream_t st) {
   return W8A8_OK;
 }
 
+// Tile choice: CTA pairs on 256 tokens x 256 or 192 channels, or single CTAs on 128 x 128.  A
+// persistent grid's time is taken as waves x the time of one SM's share of a tile (128 tokens x BN
+// channels), that share costing BN x {1, 1.32, 1.81} for the three shapes (fitted to one-wave timings
+// on K = 6912, where a narrower tile spends relatively more of each k step on operand traffic
+// through shared memory).  Narrow tiles win where the wide ones would leave SMs idle.
+template <bool kInt8>
+w8a8_status dispatch(const TcArgs& a, cudaStream_t st) {
+  const long long pairs = device_sms() / 2;
+  auto cost = [&](int bm, int bn, double unit, long long slots) {
+    const long long t = (long long)((a.N + bn - 1) / bn) * ((a.M + bm - 1) / bm);
+    return (double)((t + slots - 1) / slots) * bn * unit;
+  };
+  const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
+               c128 = cost(kBM, 128, 1.81, 2 * pairs);
+  if (c256 <= c192 && c256 <= c128) return launch_t2<kInt8, 256>(a, st);
+  if (c192 <= c128) return launch_t2<kInt8, 192>(a, st);
+  return launch_t<kInt8, 128>(a, st);
+}
+
 }  // namespace
 
 bool tc_gemm_supported(int M, int N, int K, int kind, bool want_top, int max_top) {
@@ -800,20 +829,7 @@ w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st) {
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  // bf16: CTA pairs on 256 x 256 tiles when they fill the SMs, else single CTAs on 256- or
-  // 128-channel tiles
-  const int sms = device_sms();
-  const long long pair_tiles = (long long)((a.N + 255) / 256) * ((a.M + 2 * kBM - 1) / (2 * kBM));
-  const long long tiles256 = (long long)((a.N + 255) / 256) * ((a.M + kBM - 1) / kBM);
-  w8a8_status s;
-  if (int8_codes)
-    s = launch_t<true, 128>(a, st);
-  else if (pair_tiles >= sms / 2)
-    s = launch_t2<false, 256>(a, st);
-  else if (tiles256 >= sms)
-    s = launch_t<false, 256>(a, st);
-  else
-    s = launch_t<false, 128>(a, st);
+  const w8a8_status s = int8_codes ? dispatch<true>(a, st) : dispatch<false>(a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }

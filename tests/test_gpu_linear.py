@@ -152,7 +152,10 @@ TC_SHAPES = [
     (64, 1152, 6912),    # seven 1024-k chunks folded into INT32
     (130, 4112, 1040),   # ragged M, K not a multiple of the 64-wide stage
     (256, 1536, 1152),
-    (200, 13824, 1152),  # gate/up shape, ragged M
+    (200, 13824, 1152),  # gate/up shape, ragged M: CTA pairs on 256 x 192 tiles
+    (300, 4608, 2176),   # ragged M, three k chunks
+    (512, 13824, 1152),  # CTA pairs on 256 x 192 tiles, two k chunks
+    (1024, 13824, 1152), # CTA pairs on 256 x 256 tiles
 ]
 
 
@@ -220,7 +223,8 @@ def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarr
 @pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040),
                                    (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152),
                                    (128, 6912, 1152), (70, 1152, 6912), (300, 256, 64),
-                                   (300, 19472, 1152)])  # CTA pairs (2-SM tcgen05), ragged M and N
+                                   (300, 19472, 1152),   # CTA pairs on 256 x 192 tiles, ragged M and N
+                                   (1024, 13824, 1152)])  # CTA pairs on 256 x 256 tiles
 def test_bf16_linear_within_tolerance(B, M, N, K):
     x32, x, w32, w, _, _ = _case(M, N, K, seed=11 + M)
     Y = B.linear_bf16(cu(w), cu(x))
