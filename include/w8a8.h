@@ -306,6 +306,16 @@ w8a8_status w8a8_decoder_forward(w8a8_model* m, const int32_t* tokens, int B, in
 w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* tokens, int B, int pos, float* logits,
                                      int32_t* top1, void* stream);
 
+/* How a decode step of one sequence runs (no counterpart in the paper; results agree up to fp32
+ * summation order): W8A8_DECODE_PER_STEP (default) launches one kernel per step of each layer
+ * (programmatic dependent launch overlaps each kernel's weight reads with its predecessor),
+ * W8A8_DECODE_PERSISTENT runs every decoder layer in one cooperative launch of one CTA per SM
+ * whose phases wait on each other through global counters (when the shapes allow: head dim 256,
+ * hidden <= 2048, intermediate <= 7168).  Other batch sizes always take the per-step kernels.
+ * W8A8_ERR_INVALID_ARG for another value. */
+enum { W8A8_DECODE_PER_STEP = 0, W8A8_DECODE_PERSISTENT = 1 };
+w8a8_status w8a8_model_set_decode_path(w8a8_model* m, int path);
+
 /* Measurement aid with no counterpart in the paper: *kernels = the number of kernel launches
  * one w8a8_decoder_decode_step of B sequences makes under the current mask (the kernel nodes of
  * its CUDA graph plus the position update launched beside it; copies are not counted).  The

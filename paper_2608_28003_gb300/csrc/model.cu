@@ -9,6 +9,7 @@
 #include <utility>
 #include <vector>
 
+#include "decode_mega.cuh"
 #include "decoder_kernels.cuh"
 #include "ops.cuh"
 #include "stream_gemm.cuh"
@@ -62,6 +63,14 @@ struct w8a8_model {
   size_t ws_bytes = 0;
   void* attn_ws = nullptr;
   size_t attn_ws_bytes = 0;
+  // persistent decode kernel: per-layer descriptors (host copy kept for the asynchronous upload),
+  // phase counters, attention partials; decode_path: W8A8_DECODE_PER_STEP or W8A8_DECODE_PERSISTENT
+  std::vector<MegaLayer> mega_host;
+  MegaLayer* d_mega = nullptr;
+  unsigned int* mega_sync = nullptr;
+  float* mega_part = nullptr;
+  bool mega_ok = false;
+  int decode_path = 0;
 
   cudaStream_t st = nullptr;  // private stream for graph capture / replay
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
@@ -109,6 +118,40 @@ void free_all(w8a8_model* m) {
 
 w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, q.wq_f16}; }
 
+// The persistent decode kernel's per-layer descriptors (INT8 pointers once prepared), uploaded on st.
+w8a8_status upload_mega(w8a8_model* m, cudaStream_t st) {
+  const w8a8_model_cfg& c = m->cfg;
+  m->mega_host.assign(c.layers, MegaLayer{});
+  for (int l = 0; l < c.layers; ++l) {
+    const w8a8_layer_bf16& W = m->L[l];
+    MegaLayer& g = m->mega_host[l];
+    g.w16[0] = W.wqkv;
+    g.w16[1] = W.wo;
+    g.w16[2] = m->gu_bf16 + (size_t)l * 2 * c.inter * c.hidden;
+    g.w16[3] = W.wdown;
+    const QW* q[4] = {&m->q_qkv[l], &m->q_o[l], &m->q_gu[l], &m->q_down[l]};
+    for (int j = 0; j < 4; ++j) {
+      g.w8[j] = q[j]->wq;
+      g.s_w[j] = q[j]->s_w;
+      g.inv_delta[j] = q[j]->inv_delta;
+    }
+    g.ln_in = W.ln_in;
+    g.ln_post_attn = W.ln_post_attn;
+    g.ln_pre_ffn = W.ln_pre_ffn;
+    g.ln_post_ffn = W.ln_post_ffn;
+    g.q_norm = c.qk_norm ? W.q_norm : nullptr;
+    g.k_norm = c.qk_norm ? W.k_norm : nullptr;
+    const bool glob = m->is_global(l);
+    g.rope_cos = glob ? m->cos_g : m->cos_l;
+    g.rope_sin = glob ? m->sin_g : m->sin_l;
+    g.window = glob ? 0 : c.window;
+    g.kc = m->kc + (size_t)l * m->cache_layer_elems();
+    g.vc = m->vc + (size_t)l * m->cache_layer_elems();
+  }
+  W8A8_CUDA(cudaMemcpyAsync(m->d_mega, m->mega_host.data(), sizeof(MegaLayer) * c.layers, cudaMemcpyHostToDevice, st));
+  return W8A8_OK;
+}
+
 w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
                    uint16_t* Y, cudaStream_t st, const ResNorm* rn) {
   if (int8) {
@@ -142,7 +185,36 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
   float* rc = m->r;   // the residual stream as of now
   float* rn = m->r2;  // where a fused update writes the next one
   W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st));
-  for (int l = 0; l < c.layers; ++l) {
+  const bool mega = !calib && B == 1 && T == 1 && m->mega_ok && m->decode_path == W8A8_DECODE_PERSISTENT;
+  if (mega) {  // every layer in one persistent launch, then the final residual step
+    W8A8_CUDA(cudaMemsetAsync(m->mega_sync, 0, mega_sync_words(c.layers, c.n_q) * sizeof(unsigned int), st));
+    MegaArgs g{};
+    g.layers = m->d_mega;
+    g.L = c.layers;
+    g.H = H;
+    g.F = F;
+    g.n_q = c.n_q;
+    g.n_kv = c.n_kv;
+    g.max_seq = c.max_seq;
+    g.eps = c.eps;
+    g.scale = (float)(1.0 / std::sqrt((double)c.head_dim));
+    g.attn_bits = m->prepared ? m->attn_bits : 0u;
+    g.ffn_bits = m->prepared ? m->ffn_bits : 0u;
+    g.pos = m->d_pos;
+    g.a0 = m->a;
+    g.r0 = m->r;
+    g.r1 = m->r2;
+    g.qkv = m->qkv;
+    g.att = m->o;
+    g.y = m->y;
+    g.h = m->h;
+    g.part = m->mega_part;
+    g.sync = m->mega_sync;
+    g.err = reinterpret_cast<unsigned int*>(reinterpret_cast<char*>(m->ws) + kErrWordOffset);
+    W8A8_TRY(launch_decode_mega(g, st));
+    W8A8_TRY(launch_residual_norm(m->y, M, H, m->L[c.layers - 1].ln_post_ffn, m->final_norm, c.eps, m->r2, m->a, st));
+  }
+  for (int l = 0; l < (mega ? 0 : c.layers); ++l) {
     const w8a8_layer_bf16& W = m->L[l];
     const bool att8 = !calib && m->prepared && ((m->attn_bits >> l) & 1u);
     const bool ffn8 = !calib && m->prepared && ((m->ffn_bits >> l) & 1u);
@@ -369,6 +441,13 @@ extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_l
   W8A8_MTRY(launch_rope_table(m->cos_g, m->sin_g, c.max_seq, c.head_dim, c.rope_global, st));
   for (int l = 0; l < c.layers; ++l)
     W8A8_MTRY(w8a8_interleave_gate_up(layers[l].wgate, layers[l].wup, F, H, m->gu_bf16 + (size_t)l * 2 * F * H, st));
+  m->mega_ok = decode_mega_supported(H, F, c.n_q, c.n_kv, c.head_dim, d.sms);
+  if (m->mega_ok) {
+    W8A8_MTRY(dalloc(m, &m->d_mega, (size_t)c.layers));
+    W8A8_MTRY(dalloc(m, &m->mega_sync, mega_sync_words(c.layers, c.n_q)));
+    W8A8_MTRY(dalloc(m, &m->mega_part, mega_part_floats(c.n_q)));
+    W8A8_MTRY(upload_mega(m, st));
+  }
   W8A8_MTRY(cudaStreamSynchronize(st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
 #undef W8A8_MTRY
   *out = m;
@@ -455,6 +534,10 @@ extern "C" w8a8_status w8a8_model_prepare(w8a8_model* m, float alpha, int smooth
                                 m->q_lm.delta, m->q_lm.inv_delta, m->q_lm.wq_f16, stream));
   m->prepared = true;
   ++m->prep_version;
+  if (m->mega_ok) {
+    W8A8_TRY(upload_mega(m, as_stream(stream)));
+    W8A8_CUDA(cudaStreamSynchronize(as_stream(stream)));  // the host copy may be rewritten next time
+  }
   return W8A8_OK;
 }
 
@@ -521,8 +604,8 @@ extern "C" w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* to
   W8A8_CUDA(cudaMemcpyAsync(m->d_tokens, tokens, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice, st));
   W8A8_TRY(launch_set_int(m->d_pos, pos, st));
   const int want_logits = logits != nullptr;
-  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0), m->prep_version,
-                                   want_logits);
+  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0) | (m->decode_path << 2),
+                                   m->prep_version, want_logits);
   auto it = m->graphs.find(key);
   if (it == m->graphs.end()) {
     // one eager step first: every lazily set kernel attribute exists before capture; it computes
@@ -560,10 +643,18 @@ extern "C" w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* to
   return W8A8_OK;
 }
 
+extern "C" w8a8_status w8a8_model_set_decode_path(w8a8_model* m, int path) {
+  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "null model");
+  W8A8_CHECK_ARG(path == W8A8_DECODE_PERSISTENT || path == W8A8_DECODE_PER_STEP, W8A8_ERR_INVALID_ARG,
+                 "w8a8_model_set_decode_path: path %d", path);
+  m->decode_path = path;
+  return W8A8_OK;
+}
+
 extern "C" w8a8_status w8a8_model_decode_kernels(const w8a8_model* m, int B, int want_logits, int* kernels) {
   W8A8_CHECK_ARG(m && kernels, W8A8_ERR_INVALID_ARG, "w8a8_model_decode_kernels: null argument");
-  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0), m->prep_version,
-                                   want_logits ? 1 : 0);
+  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0) | (m->decode_path << 2),
+                                   m->prep_version, want_logits ? 1 : 0);
   const auto it = m->graphs.find(key);
   W8A8_CHECK_ARG(it != m->graphs.end(), W8A8_ERR_INVALID_ARG,
                  "w8a8_model_decode_kernels: no decode step of B=%d under this mask yet", B);
