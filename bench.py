@@ -47,6 +47,9 @@ sys.path.insert(0, ROOT)
 METRIC = "W8A8 linear TOPS & HBM GB/s vs GB300 roofline; decode ms/token per mask vs bf16"
 HIDDEN, INTER, VOCAB, LAYERS = 1152, 6912, 262144, 26
 PREFILL = 128
+# DRAM bytes read + written per launch of the decode GEMV, averaged over the roofline mix's launches
+# (ncu over one decode step of `--profile-workload decode4`, the same shapes)
+GEMV_MIX_TRAFFIC = 11170455
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 WORKLOAD = ("decode, 26-layer Gemma-3-1B-shaped decoder (H 1152, 4q/1kv x 256, FFN 6912, V 262144), mask FFN 5+5 + "
@@ -60,7 +63,73 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--quick", action="store_true", help="headline only: skip the mask sweep and the tables")
+    ap.add_argument("--profile-workload", choices=["decode4", "gemm", "linear16"], default=None,
+                    help="run a small fixed workload for a profiler and exit (no JSON line): 'decode4' = five "
+                         "batch-1 decode steps of a 4-layer decoder with the full shapes (FFN layers 0-1 and "
+                         "lm_head W8A8); 'gemm' = three bf16 and three W8A8 prefill linears, 2048 x 1152 -> 13824; "
+                         "'linear16' = three W8A8 linears of the single-linear workload (M 16, 1152 -> 6912) and "
+                         "three W8A8 FFN blocks at M 8")
     return ap.parse_args()
+
+
+def profile_workload(name):
+    """Small fixed workloads for ncu captures (a few GB on the device at most)."""
+    import torch
+    import synth
+    from paper_2608_28003_gb300 import build
+    build.build()
+    from paper_2608_28003_gb300 import binding as B
+    dev = torch.device("cuda", 0)
+    if name == "decode4":
+        global LAYERS
+        LAYERS = 4
+        f32, bf, norms = synth.decoder_weights(4, seed=0, want_f32=False)
+        dec, _ = make_decoder(B, dev, bf, norms, max_batch=1, max_seq=512, max_tokens=256)
+        dec.calibrate(torch.from_numpy(synth.tokens(64, VOCAB, seed=1).reshape(1, 64)).to(dev))
+        dec.prepare()
+        dec.set_mask(0b0011, 0, 1)
+        toks = torch.from_numpy(synth.tokens(300, VOCAB, seed=2)).to(dev)
+        prefill(dec, toks[:PREFILL].view(1, PREFILL), 256)
+        top = torch.zeros(16, dtype=torch.int32, device=dev)
+        for s in range(5):
+            dec.decode_step(toks[PREFILL + s:PREFILL + s + 1], PREFILL + s, top1=top[s:s + 1])
+        torch.cuda.synchronize()
+        dec.close()
+    elif name == "linear16":
+        c = synth.linear_case()
+        stat = torch.from_numpy(c["calib32"]).abs().amax(0).to(dev)
+        q = B.prepare_weights(c["w"].to(dev), stat)
+        x = c["x"].to(dev)
+        ws = B.Workspace(dev)
+        y = torch.empty(x.shape[0], q.n, dtype=torch.bfloat16, device=dev)
+        for _ in range(3):
+            B.linear(q, x, out=y, ws=ws)
+        _, wg = synth.weight(INTER, HIDDEN, seed=3)
+        _, wu = synth.weight(INTER, HIDDEN, seed=4)
+        _, wd = synth.weight(HIDDEN, INTER, seed=5)
+        _, x8, _ = synth.activations(8, HIDDEN, 8, seed=6)
+        x8 = x8.to(dev)
+        ones_h, ones_f = torch.ones(HIDDEN, device=dev), torch.ones(INTER, device=dev)
+        f = B.FfnWeights(HIDDEN, INTER, gate_up=B.prepare_gate_up(wg.to(dev), wu.to(dev), ones_h),
+                         down=B.prepare_weights(wd.to(dev), ones_f))
+        y8 = torch.empty(8, HIDDEN, dtype=torch.bfloat16, device=dev)
+        for _ in range(3):
+            B.ffn_block(f, B.W8A8_PREC_W8A8, x8, out=y8, ws=ws)
+        torch.cuda.synchronize()
+    else:
+        M, N, K = 2048, 2 * INTER, HIDDEN
+        _, w = synth.weight(N, K, seed=1)
+        _, x, _ = synth.activations(M, K, 8, seed=2)
+        w, x = w.to(dev), x.to(dev)
+        ws = B.Workspace(dev)
+        y = torch.empty(M, N, dtype=torch.bfloat16, device=dev)
+        q = B.prepare_weights(w, B.act_absmax(x), want_f16=True)
+        for _ in range(3):
+            B.linear_bf16(w, x, out=y, ws=ws)
+        for _ in range(3):
+            B.linear(q, x, out=y, ws=ws)
+        torch.cuda.synchronize()
+    print("ok")
 
 
 def load_peaks():
@@ -335,42 +404,72 @@ def run_ours(args, dist: Dist):
     e2e_ms = whole_job_ms_per_token(dist.max(sum(e2e)), K, dist.world)
 
     # ---- roofline: the decode step's dominant kernel by share of device time (the ncu launch list),
-    # the row-owning decode GEMV on bf16 weights at one token: per step 26 q/k/v (1152 -> 1536),
-    # 26 o (1024 -> 1152) and 16 down (6912 -> 1152, the bf16 FFN layers of the mask).  Each shape
-    # is launched as in the decode step, timed alone with events around the kernel, L2 flushed
-    # before each launch; achieved = the mix's algorithmic bytes / its kernel time.
+    # the row-owning decode GEMV, over every one of its launches in a step under the headline mask:
+    # 26 q/k/v (1152 -> 1536) and 26 o (1024 -> 1152) on bf16 weights, gate/up + GeGLU (1152 ->
+    # 2 x 6912) and down (6912 -> 1152) on the 16 bf16 and the 10 W8A8 FFN layers (K1 fused into the
+    # W8A8 ones).  Each shape is launched as in the decode step, timed alone with events around the
+    # kernel, L2 flushed before each launch; achieved = the mix's algorithmic bytes / its kernel time.
+    # L2 flush: write 512 MiB (> 129 MB L2), then read another 512 MiB so that the write-backs of the
+    # dirty lines happen before the timed kernel, not during it
     flush_buf = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
-    flush = lambda: flush_buf.zero_()  # noqa: E731  (512 MiB > 129 MB L2)
+    flush_rd = torch.ones(128 << 20, dtype=torch.float32, device=dev)
+    flush_sum = torch.empty((), dtype=torch.float32, device=dev)
+
+    def flush():
+        flush_buf.zero_()
+        torch.sum(flush_rd, dim=0, out=flush_sum)
+
     ws = B.Workspace(dev)
-    mix = [("qkv", 26, wdev["wqkv"][5], 1536, HIDDEN), ("o", 26, wdev["wo"][5], HIDDEN, 1024),
-           ("down", 16, wdev["wd"][5], HIDDEN, INTER)]
-    parts, tot_bytes, tot_us = {}, 0.0, 0.0
-    for name, count, wmat, N, Kd in mix:
-        xin = torch.from_numpy(synth.activations(1, Kd, 8, seed=N)[0]).to(torch.bfloat16).to(dev)
-        yout = torch.empty(1, N, dtype=torch.bfloat16, device=dev)
-        timed_steps(lambda: B.linear_bf16(wmat, xin, out=yout, ws=ws), max(K, 20), 3, flush, stream,
-                    kernel_events=B.set_kernel_events)
+    stats = torch.from_numpy(dec.get_stats()).to(dev)
+    stride = 2 * HIDDEN + 1024 + INTER  # per layer: q/k/v, o, gate/up, down input statistics
+    st5 = stats[5 * stride:6 * stride]
+    gu_stat, down_stat = st5[HIDDEN + 1024:2 * HIDDEN + 1024].contiguous(), st5[2 * HIDDEN + 1024:].contiguous()
+    wg, wu, wd = wdev["wg"][5], wdev["wu"][5], wdev["wd"][5]
+    f_bf = B.FfnWeights(HIDDEN, INTER, gate_up_bf16=B.interleave_gate_up(wg, wu), down_bf16=wd)
+    f_i8 = B.FfnWeights(HIDDEN, INTER, gate_up=B.prepare_gate_up(wg, wu, gu_stat), down=B.prepare_weights(wd, down_stat))
+    n_i8 = bin(head_mask[0]).count("1")
+    n_bf = LAYERS - n_i8
+
+    def xrow(k, seed):
+        return torch.from_numpy(synth.activations(1, k, 8, seed=seed)[0]).to(torch.bfloat16).to(dev)
+
+    x_h, x_q, x_f = xrow(HIDDEN, 1), xrow(1024, 2), xrow(INTER, 3)
+    y_h, y_qkv = torch.empty(1, HIDDEN, dtype=torch.bfloat16, device=dev), torch.empty(1, 1536, dtype=torch.bfloat16,
+                                                                                       device=dev)
+    wq5, wo5 = wdev["wqkv"][5], wdev["wo"][5]
+    mix = [("qkv bf16", 26, lambda: B.linear_bf16(wq5, x_h, out=y_qkv, ws=ws), bf16_bytes(1, 1536, HIDDEN)),
+           ("o bf16", 26, lambda: B.linear_bf16(wo5, x_q, out=y_h, ws=ws), bf16_bytes(1, HIDDEN, 1024)),
+           ("gate/up bf16", n_bf, lambda: B.ffn_block(f_bf, B.W8A8_PREC_BF16, x_h, out=y_h, ws=ws),
+            bf16_bytes(1, 2 * INTER, HIDDEN, out_bytes=1)),
+           ("down bf16", n_bf, lambda: B.linear_bf16(wd, x_f, out=y_h, ws=ws), bf16_bytes(1, HIDDEN, INTER)),
+           ("gate/up W8A8", n_i8, lambda: B.ffn_block(f_i8, B.W8A8_PREC_W8A8, x_h, out=y_h, ws=ws),
+            w8a8_bytes(1, 2 * INTER, HIDDEN, out_bytes=1)),
+           ("down W8A8", n_i8, lambda: B.linear(f_i8.down, x_f, out=y_h, ws=ws), w8a8_bytes(1, HIDDEN, INTER))]
+    parts, tot_bytes, tot_us, n_launch = {}, 0.0, 0.0, 0
+    for name, count, fn, nbytes in mix:
+        if count == 0:
+            continue
+        # the hook's events bracket the next library launch: the GEMV itself (for the FFN block, its
+        # first launch, gate/up + GeGLU)
+        timed_steps(fn, max(K, 20), 3, flush, stream, kernel_events=B.set_kernel_events)
         us = statistics.mean(timed_steps.kernel_ms) * 1e3
-        nbytes = bf16_bytes(1, N, Kd)
         parts[name] = {"launches_per_step": count, "kernel_us": round(us, 2), "bytes": nbytes,
                        "GBps": round(nbytes / (us * 1e-6) / 1e9, 1)}
         tot_bytes += count * nbytes
         tot_us += count * us
+        n_launch += count
     achieved = tot_bytes / (tot_us * 1e-6) / 1e9
-    # DRAM bytes read + written per launch of the same mix from one ncu capture of this kernel inside
-    # the decode step (q/k/v 3,564,544 + o 2,384,128 + down 15,961,856 bytes, weighted 26 : 26 : 16)
-    traffic = (26 * 3564544 + 26 * 2384128 + 16 * 15961856) / 68
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": round(traffic),
+                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": GEMV_MIX_TRAFFIC,
                 "peak_source": peaks["source"],
-                "kernel": "gemv_small_kernel<bf16, 1 token, 1 row/warp> (decode row-owning GEMV)",
-                "kernel_us": round(tot_us / 68, 2), "algorithmic_bytes_per_launch": round(tot_bytes / 68),
+                "kernel": "gemv_small_kernel (decode row-owning GEMV, all %d launches of a step)" % n_launch,
+                "kernel_us": round(tot_us / n_launch, 2), "algorithmic_bytes_per_launch": round(tot_bytes / n_launch),
                 "launch_mix": parts,
-                "timing": "CUDA events around the kernel on its stream, launches as in the decode step, "
-                          "L2 flushed before each launch; per-launch figures are the mix's averages"}
+                "timing": "CUDA events around the kernel on its stream, each shape launched alone as in the "
+                          "decode step, L2 flushed (512 MiB written, then 512 MiB read) before each launch; "
+                          "per-launch figures are the mix's averages"}
 
     # the lm_head GEMV (W8A8, one token) on the same terms, for comparison
-    stats = torch.from_numpy(dec.get_stats()).to(dev)
     lm_stat = stats[-HIDDEN:].contiguous()
     q_lm = B.prepare_weights(wdev["embed"], lm_stat, want_f16=True)
     head = B.HeadWeights(VOCAB, HIDDEN, q_lm, wdev["embed"])
@@ -580,6 +679,9 @@ def reference_line(args, times, n):
 
 def main():
     args = parse()
+    if args.profile_workload:
+        profile_workload(args.profile_workload)
+        return
     if args.impl == "reference":
         dist = Dist("gloo")
         if dist.rank != 0:
