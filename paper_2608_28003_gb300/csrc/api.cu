@@ -142,13 +142,18 @@ bool decode_gemv_takes(bool int8, int M, int N, int K, bool geglu, int sms) {
 
 // Calls with more tokens than the decode GEMV takes go to the tensor-core GEMM when its shape
 // rules hold (W8A8: the weights' fp16 code copy must exist); false leaves them to the streaming
-// kernel.
-constexpr int kTcMinTokens = 64;
+// kernel.  Below 64 tokens a 128-token tile is mostly padding; it still beats the streaming kernel
+// on the decoder's linears (one wave of 128 x 64 tiles, measured 12-15 us against 20 us at M 16),
+// but not on lm_head-sized outputs, where the streaming kernel's INT8 reads (half the bytes of the
+// fp16 code copy) win.
+constexpr int kTcMinTokens = 64, kTcMinTokensNarrow = 9, kTcNarrowMaxN = 16384;
 
 static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N, int K, const float* bias, int kind,
                     const float* inv_delta, const float* s_w, uint16_t* Y, float* logits, int32_t* top1,
                     const w8a8_debug* dbg, void* ws, void* codes, float* s_x, cudaStream_t st, w8a8_status* status) {
-  if (M < kTcMinTokens || !W16 || !tc_gemm_supported(M, N, K, kind, top1 != nullptr, max_top_keys())) return false;
+  if (M < (N <= kTcNarrowMaxN ? kTcMinTokensNarrow : kTcMinTokens) || !W16 ||
+      !tc_gemm_supported(M, N, K, kind, top1 != nullptr, max_top_keys()))
+    return false;
   TcArgs a{};
   if (int8) {
     w8a8_status q = launch_quantize_rows(X, M, K, inv_delta, dbg ? dbg->xq : nullptr,

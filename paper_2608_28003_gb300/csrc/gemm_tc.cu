@@ -11,8 +11,8 @@
 //    the epilogue, warp w reading TMEM lanes 32 (w mod 4) .. +31 (its tokens) and column quarter
 //    w / 4 of the slot with tcgen05.ld, then handing the slot back.  Four epilogue warps per SM
 //    sub-partition keep its issue slots busy while one waits on a dependency.
-//  * tiles: BN = 128 (four slots) on single CTAs, or BN = 192 / 256 (two slots) on CTA pairs of
-//    256 tokens (cta_group::2, below), chosen by a cost model of the waves.
+//  * tiles: BN = 64 / 128 (four slots) on single CTAs, or BN = 192 / 256 (two slots) on CTA pairs
+//    of 256 tokens (cta_group::2, below), chosen by a cost model of the waves.
 //  * W8A8 path: both operands are INT8 codes stored as fp16 (exact).  Every product is an integer
 //    below 2^14, so a fp32 sum of at most 1024 of them is exact; the accumulator is therefore
 //    restarted every 1024 k (16 stages) in the next slot while the epilogue folds the finished one
@@ -48,6 +48,12 @@ constexpr uint32_t kTmemCols = 512;  // all of an SM's tensor memory: 2 (bf16) o
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kStageBufBytes = 32 * 64;                  // one epilogue block: 32 rows of 64 bytes
 constexpr int kEpiSmem = kEpiWarps * kStageBufBytes;  // one block per epilogue warp
+
+// Rows of the activation box a stage loads: with fewer than 128 tokens only the rows that exist
+// (rounded up to 8) are copied; the MMA still reads 128 rows, but rows past M only feed output
+// rows that are never stored, so the rest of the tile is left as it is (a zero fill would cost as
+// much TMA time as real data).
+__host__ __device__ constexpr int a_box_rows(int M) { return M < kBM ? (M + 7) / 8 * 8 : kBM; }
 
 // Tensor-memory columns of one accumulator slot: BN rounded up to a power of two, so every slot
 // starts on a 128-column boundary.
@@ -275,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           const uint32_t bar = full0 + 8 * s;
-          mbar_arrive_expect_tx(bar, kABytes + GG::BBytes);
+          mbar_arrive_expect_tx(bar, (uint32_t)(a_box_rows(a.M) * kBK * 2) + GG::BBytes);
           tma_load_2d(sA + (uint32_t)s * kABytes, &tmA, kb * kBK, m0, bar);
           tma_load_2d(sB + (uint32_t)s * GG::BBytes, &tmB, kb * kBK, n0, bar);
         }
@@ -763,7 +769,8 @@ w8a8_status launch_t(const TcArgs& a, cudaStream_t st) {
     attr_set[dev] = true;
   }
   CUtensorMap ta, tb;
-  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, kBM, kSwz));
+  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, (uint32_t)a_box_rows(a.M),
+                        kSwz));
   W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN, kSwz));
   CUtensorMap ty;
   W8A8_TRY(make_out_map(a, &ty, ta));
@@ -795,11 +802,12 @@ w8a8_status launch_t2(const TcArgs& a, cudaStream_t st) {
   return W8A8_OK;
 }
 
-// Tile choice: CTA pairs on 256 tokens x 256 or 192 channels, or single CTAs on 128 x 128.  A
-// persistent grid's time is taken as waves x the time of one SM's share of a tile (128 tokens x BN
-// channels), that share costing BN x {1, 1.32, 1.81} for the three shapes (fitted to one-wave timings
-// on K = 6912, where a narrower tile spends relatively more of each k step on operand traffic
-// through shared memory).  Narrow tiles win where the wide ones would leave SMs idle.
+// Tile choice: CTA pairs on 256 tokens x 256 or 192 channels, or single CTAs on 128 x 128 or
+// 128 x 64.  A persistent grid's time is taken as waves x the time of one SM's share of a tile (128
+// tokens x BN channels), that share costing BN x {1, 1.32, 1.81, 2.7} for the four shapes (fitted
+// to one-wave timings on K = 6912, where a narrower tile spends relatively more of each k step on
+// operand traffic through shared memory; the last estimated from its operand bytes per MMA).
+// Narrow tiles win where the wide ones would leave SMs idle, as at decode-sized token counts.
 template <bool kInt8>
 w8a8_status dispatch(const TcArgs& a, cudaStream_t st) {
   const long long pairs = device_sms() / 2;
@@ -808,10 +816,11 @@ w8a8_status dispatch(const TcArgs& a, cudaStream_t st) {
     return (double)((t + slots - 1) / slots) * bn * unit;
   };
   const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
-               c128 = cost(kBM, 128, 1.81, 2 * pairs);
-  if (c256 <= c192 && c256 <= c128) return launch_t2<kInt8, 256>(a, st);
-  if (c192 <= c128) return launch_t2<kInt8, 192>(a, st);
-  return launch_t<kInt8, 128>(a, st);
+               c128 = cost(kBM, 128, 1.81, 2 * pairs), c64 = cost(kBM, 64, 2.7, 2 * pairs);
+  if (c256 <= c192 && c256 <= c128 && c256 <= c64) return launch_t2<kInt8, 256>(a, st);
+  if (c192 <= c128 && c192 <= c64) return launch_t2<kInt8, 192>(a, st);
+  if (c128 <= c64) return launch_t<kInt8, 128>(a, st);
+  return launch_t<kInt8, 64>(a, st);  // few tokens: spread the weight stream over more SMs
 }
 
 }  // namespace

@@ -149,6 +149,9 @@ def test_w8a8_linear_bit_exact(B, M, N, K):
 
 
 TC_SHAPES = [
+    (16, 6912, 1152),    # the single-linear workload: 128 x 64 tiles, 15/16 of each tile padding
+    (9, 1536, 1152),     # fewest tokens the tensor-core path takes
+    (40, 1152, 6912),    # ragged M, seven k chunks
     (64, 1152, 6912),    # seven 1024-k chunks folded into INT32
     (130, 4112, 1040),   # ragged M, K not a multiple of the 64-wide stage
     (256, 1536, 1152),
