@@ -67,8 +67,8 @@ def parse():
                     help="run a small fixed workload for a profiler and exit (no JSON line): 'decode4' = five "
                          "batch-1 decode steps of a 4-layer decoder with the full shapes (FFN layers 0-1 and "
                          "lm_head W8A8); 'gemm' = three bf16 and three W8A8 prefill linears, 2048 x 1152 -> 13824; "
-                         "'linear16' = three W8A8 linears of the single-linear workload (M 16, 1152 -> 6912) and "
-                         "three W8A8 FFN blocks at M 8")
+                         "'linear16' = the single-linear workload (M 16, 1152 -> 6912) three times each as W8A8 "
+                         "on INT8 codes, W8A8 with the fp16 code copy and bf16, then three W8A8 FFN blocks at M 8")
     return ap.parse_args()
 
 
@@ -99,11 +99,16 @@ def profile_workload(name):
         c = synth.linear_case()
         stat = torch.from_numpy(c["calib32"]).abs().amax(0).to(dev)
         q = B.prepare_weights(c["w"].to(dev), stat)
+        q16 = B.prepare_weights(c["w"].to(dev), stat, want_f16=True)
         x = c["x"].to(dev)
         ws = B.Workspace(dev)
         y = torch.empty(x.shape[0], q.n, dtype=torch.bfloat16, device=dev)
         for _ in range(3):
-            B.linear(q, x, out=y, ws=ws)
+            B.linear(q, x, out=y, ws=ws)  # INT8 codes only: the streaming kernel
+        for _ in range(3):
+            B.linear(q16, x, out=y, ws=ws)  # with the fp16 code copy: the tensor-core GEMM
+        for _ in range(3):
+            B.linear_bf16(c["w"].to(dev), x, out=y, ws=ws)
         _, wg = synth.weight(INTER, HIDDEN, seed=3)
         _, wu = synth.weight(INTER, HIDDEN, seed=4)
         _, wd = synth.weight(HIDDEN, INTER, seed=5)
@@ -458,16 +463,73 @@ def run_ours(args, dist: Dist):
         tot_bytes += count * nbytes
         tot_us += count * us
         n_launch += count
-    achieved = tot_bytes / (tot_us * 1e-6) / 1e9
-    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": GEMV_MIX_TRAFFIC,
-                "peak_source": peaks["source"],
-                "kernel": "gemv_small_kernel (decode row-owning GEMV, all %d launches of a step)" % n_launch,
-                "kernel_us": round(tot_us / n_launch, 2), "algorithmic_bytes_per_launch": round(tot_bytes / n_launch),
+    isolated = {"GBps": round(tot_bytes / (tot_us * 1e-6) / 1e9, 1), "kernel_us": round(tot_us / n_launch, 2),
                 "launch_mix": parts,
                 "timing": "CUDA events around the kernel on its stream, each shape launched alone as in the "
                           "decode step, L2 flushed (512 MiB written, then 512 MiB read) before each launch; "
                           "per-launch figures are the mix's averages"}
+
+    # The same 104 launches chained as in the decode step: every layer's q/k/v, o and FFN (gate/up +
+    # GeGLU, down) on that layer's own weights (bf16, or W8A8 on the mask's FFN layers), recorded
+    # once as a CUDA graph (programmatic dependent launch between the kernels, nothing else in
+    # between) and replayed back to back; 1.15 GB of weights per replay stream through the 129 MB
+    # L2.  Average launch duration = replay time / 104.
+    f_layers = []
+    for l in range(LAYERS):
+        wgl, wul, wdl = wdev["wg"][l], wdev["wu"][l], wdev["wd"][l]
+        if (head_mask[0] >> l) & 1:
+            stl = stats[l * stride:(l + 1) * stride]
+            f_layers.append(B.FfnWeights(
+                HIDDEN, INTER, gate_up=B.prepare_gate_up(wgl, wul, stl[HIDDEN + 1024:2 * HIDDEN + 1024].contiguous()),
+                down=B.prepare_weights(wdl, stl[2 * HIDDEN + 1024:].contiguous())))
+        else:
+            f_layers.append(B.FfnWeights(HIDDEN, INTER, gate_up_bf16=B.interleave_gate_up(wgl, wul), down_bf16=wdl))
+    chain_bytes = 0
+    for l in range(LAYERS):
+        i8 = (head_mask[0] >> l) & 1
+        chain_bytes += bf16_bytes(1, 1536, HIDDEN) + bf16_bytes(1, HIDDEN, 1024)
+        chain_bytes += (w8a8_bytes(1, 2 * INTER, HIDDEN, out_bytes=1) + w8a8_bytes(1, HIDDEN, INTER) if i8 else
+                        bf16_bytes(1, 2 * INTER, HIDDEN, out_bytes=1) + bf16_bytes(1, HIDDEN, INTER))
+
+    def chain():
+        for l in range(LAYERS):
+            B.linear_bf16(wdev["wqkv"][l], x_h, out=y_qkv, ws=ws)
+            B.linear_bf16(wdev["wo"][l], x_q, out=y_h, ws=ws)
+            B.ffn_block(f_layers[l], B.W8A8_PREC_W8A8 if (head_mask[0] >> l) & 1 else B.W8A8_PREC_BF16, x_h, out=y_h,
+                        ws=ws)
+
+    cap = torch.cuda.Stream()  # graphs are captured on a side stream
+    with torch.cuda.stream(cap):
+        chain()  # every kernel's attributes set before capture
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=cap):
+        chain()
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    reps = max(K, 20)
+    c0, c1 = _events(2)
+    with torch.cuda.stream(stream):
+        gpu_sleep_for(reps, 1.0)
+        c0.record(stream)
+        for _ in range(reps):
+            graph.replay()
+        c1.record(stream)
+    torch.cuda.synchronize()
+    chain_us = c0.elapsed_time(c1) * 1e3 / reps
+    del graph
+    achieved = chain_bytes / (chain_us * 1e-6) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": GEMV_MIX_TRAFFIC,
+                "peak_source": peaks["source"],
+                "kernel": "gemv_small_kernel (decode row-owning GEMV, all %d launches of a step)" % n_launch,
+                "kernel_us": round(chain_us / n_launch, 2), "algorithmic_bytes_per_launch": round(chain_bytes / n_launch),
+                "timing": "the step's %d GEMV launches chained as in the decode step (each layer's own weights, "
+                          "programmatic dependent launch, one CUDA graph) and replayed %d times back to back; CUDA "
+                          "events on the launching stream around the replays; average launch duration = replay "
+                          "time / %d" % (n_launch, reps, n_launch),
+                "isolated_launches": isolated}
 
     # the lm_head GEMV (W8A8, one token) on the same terms, for comparison
     lm_stat = stats[-HIDDEN:].contiguous()
