@@ -63,12 +63,14 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--quick", action="store_true", help="headline only: skip the mask sweep and the tables")
-    ap.add_argument("--profile-workload", choices=["decode4", "gemm", "linear16"], default=None,
+    ap.add_argument("--profile-workload", choices=["decode4", "gemm", "linear16", "prefill4", "ffn2048"], default=None,
                     help="run a small fixed workload for a profiler and exit (no JSON line): 'decode4' = five "
                          "batch-1 decode steps of a 4-layer decoder with the full shapes (FFN layers 0-1 and "
                          "lm_head W8A8); 'gemm' = three bf16 and three W8A8 prefill linears, 2048 x 1152 -> 13824; "
                          "'linear16' = the single-linear workload (M 16, 1152 -> 6912) three times each as W8A8 "
-                         "on INT8 codes, W8A8 with the fp16 code copy and bf16, then three W8A8 FFN blocks at M 8")
+                         "on INT8 codes, W8A8 with the fp16 code copy and bf16, then three W8A8 FFN blocks at M 8; "
+                         "'prefill4' = a 2048-token prefill of a 4-layer decoder with the full shapes (bf16); "
+                         "'ffn2048' = three W8A8 and three bf16 FFN blocks at M 2048")
     return ap.parse_args()
 
 
@@ -80,8 +82,17 @@ def profile_workload(name):
     build.build()
     from paper_2608_28003_gb300 import binding as B
     dev = torch.device("cuda", 0)
-    if name == "decode4":
-        global LAYERS
+    global LAYERS
+    if name == "prefill4":
+        LAYERS = 4
+        f32, bf, norms = synth.decoder_weights(4, seed=0, want_f32=False)
+        dec, _ = make_decoder(B, dev, bf, norms, max_batch=1, max_seq=2048, max_tokens=2048)
+        toks = torch.from_numpy(synth.tokens(2048, VOCAB, seed=2)).to(dev).view(1, 2048)
+        for _ in range(2):
+            dec.forward(toks, 0, want_logits=False)
+        torch.cuda.synchronize()
+        dec.close()
+    elif name == "decode4":
         LAYERS = 4
         f32, bf, norms = synth.decoder_weights(4, seed=0, want_f32=False)
         dec, _ = make_decoder(B, dev, bf, norms, max_batch=1, max_seq=512, max_tokens=256)
@@ -95,6 +106,19 @@ def profile_workload(name):
             dec.decode_step(toks[PREFILL + s:PREFILL + s + 1], PREFILL + s, top1=top[s:s + 1])
         torch.cuda.synchronize()
         dec.close()
+    elif name == "ffn2048":
+        fc = synth.ffn_case(2048, seed=0)
+        gu = B.prepare_gate_up(fc["wg"].to(dev), fc["wu"].to(dev), B.act_absmax(fc["calib"].to(dev)), want_f16=True)
+        dn = B.prepare_weights(fc["wd"].to(dev), torch.from_numpy(fc["stat_h"]).to(dev), want_f16=True)
+        f = B.FfnWeights(HIDDEN, INTER, gu, dn, B.interleave_gate_up(fc["wg"].to(dev), fc["wu"].to(dev)),
+                         fc["wd"].to(dev))
+        x = fc["x"].to(dev)
+        ws = B.Workspace(dev)
+        y = torch.empty(2048, HIDDEN, dtype=torch.bfloat16, device=dev)
+        for prec in (B.W8A8_PREC_W8A8, B.W8A8_PREC_BF16):
+            for _ in range(3):
+                B.ffn_block(f, prec, x, out=y, ws=ws)
+        torch.cuda.synchronize()
     elif name == "linear16":
         c = synth.linear_case()
         stat = torch.from_numpy(c["calib32"]).abs().amax(0).to(dev)

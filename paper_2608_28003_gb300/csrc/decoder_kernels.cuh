@@ -42,6 +42,12 @@ w8a8_status launch_attn_decode(const uint16_t* qkv, const AttnShape& s, const in
                                const float* kn, float eps, const float* rope_cos, const float* rope_sin,
                                uint16_t* kcache, uint16_t* vcache, uint16_t* o, cudaStream_t st);
 
+// Prefill (T > 1): flash-attention-style attention of q (fp32, after QK-norm and RoPE) over the
+// cache on the tensor cores (fp16 operands, fp32 accumulation and softmax); o bf16 [M, n_q*hd].
+bool attention_prefill_supported(const AttnShape& s);
+w8a8_status launch_attention_prefill(const float* q, const uint16_t* kcache, const uint16_t* vcache, const AttnShape& s,
+                                     const int* pos0, uint16_t* o, cudaStream_t st);
+
 // cos/sin tables [max_seq][hd/2] of RoPE with the given base, computed in fp64
 w8a8_status launch_rope_table(float* cos_t, float* sin_t, int max_seq, int hd, double base, cudaStream_t st);
 

@@ -239,7 +239,10 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
       W8A8_TRY(launch_attn_decode(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, kc, vc, m->o, st));
     } else {
       W8A8_TRY(launch_qk_rope(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, m->q, kc, vc, st));
-      W8A8_TRY(launch_attention(m->q, kc, vc, s, m->d_pos, 0, m->o, m->attn_ws, m->sms, st));
+      if (attention_prefill_supported(s))
+        W8A8_TRY(launch_attention_prefill(m->q, kc, vc, s, m->d_pos, m->o, st));
+      else
+        W8A8_TRY(launch_attention(m->q, kc, vc, s, m->d_pos, 0, m->o, m->attn_ws, m->sms, st));
     }
     if (calib) W8A8_TRY(launch_act_absmax(m->o, M, m->q_dim, m->stat_o(l), st));
     W8A8_TRY(linear(m, att8, m->q_o[l], W.wo, H, m->q_dim, m->o, M, m->y, st, nullptr));
