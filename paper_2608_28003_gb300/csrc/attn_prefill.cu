@@ -3,13 +3,15 @@
 // The query-row kernel (attention_kernel) reads a row's keys and values from L2 for every query
 // row, so a 2048-token prefill moves about 2 GB per layer through L2 and the arithmetic runs on
 // the CUDA cores.  Here a CTA takes a block of 64 queries of one head and walks the keys in tiles
-// of 64 positions that all of its queries share:
-//  * grid (query blocks, query heads, sequences), 4 warps; warp w owns query rows 16w .. 16w+15
-//    of the block.  The block's queries (after QK-norm and RoPE, fp32) are scaled by the
+// of 32 positions that all of its queries share:
+//  * grid (query blocks, query heads, sequences), 8 warps in two groups of four; warp w of a group
+//    owns query rows 16w .. 16w+15 of the block, group 0 takes the even key tiles and group 1 the
+//    odd ones (two warps per SM sub-partition, each with half of the serial MMA chain), and at the
+//    end group 0 merges group 1's (m, l, O) through shared memory.  The block's queries (after QK-norm and RoPE, fp32) are scaled by the
 //    attention scale and rounded to fp16 into shared memory once (fp16, not bf16: 11 mantissa
 //    bits keep the scores and probabilities close to the fp32 arithmetic of the other paths);
 //  * key/value tiles (bf16 rows of 512 bytes straight from the cache) arrive by cp.async, two
-//    tiles deep, into shared memory whose 16-byte chunks are XOR-swizzled by (row mod 8), so the
+//    tiles deep per group, into shared memory whose 16-byte chunks are XOR-swizzled by (row mod 8), so the
 //    8 row addresses of an ldmatrix phase hit 8 different bank groups; each landed tile is
 //    converted to fp16 in place (exact for the cache's bf16 values in the fp16 normal range);
 //  * S = Q K^T with mma.sync m16n8k16 (fp16 in, fp32 accumulation): Q fragments by ldmatrix, K
@@ -29,13 +31,17 @@ namespace {
 
 constexpr int kHd = 256;
 constexpr int kBq = 64;             // queries per CTA
-constexpr int kBk = 64;             // keys per tile
-constexpr int kWarps = kBq / 16;
+constexpr int kBk = 32;             // keys per tile
+constexpr int kGW = kBq / 16;       // warps per group (one per 16 query rows)
+constexpr int kWarps = 2 * kGW;     // two groups: even and odd key tiles
+constexpr int kGT = kGW * 32;       // threads per group
 constexpr int kRowBytes = kHd * 2;  // one bf16 row of 256
 constexpr int kTileBytes = kBk * kRowBytes;
 constexpr int kOffQ = 0;
-constexpr int kOffKV = kBq * kRowBytes;                 // two buffers of (K tile, V tile)
-constexpr int kSmem = kOffKV + 2 * 2 * kTileBytes;      // 32 KB + 128 KB
+constexpr int kOffKV = kBq * kRowBytes;                 // per group two buffers of (K tile, V tile)
+constexpr int kGroupKV = 2 * 2 * kTileBytes;
+constexpr int kSmem = kOffKV + 2 * kGroupKV;            // 32 KB + 128 KB
+static_assert(kGW * 32 * 132 * 4 <= 2 * kGroupKV, "the merge area must fit in the key/value buffers");
 
 __device__ __forceinline__ uint32_t swz(int row, int chunk) {  // byte offset of a 16-byte chunk
   return (uint32_t)(row * kRowBytes + ((chunk ^ (row & 7)) << 4));
@@ -78,7 +84,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_prefill_kernel(const float* 
   pdl_wait();
   const int qb = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int G = s.n_q / s.n_kv, kvh = head / G;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int warp_all = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int grp = warp_all / kGW, warp = warp_all % kGW, gt = threadIdx.x % kGT;
   const int g = lane >> 2, t4 = lane & 3;
   const int p0 = *pos0;
   const int t0 = qb * kBq;                           // first query (token index within the call)
@@ -89,10 +96,10 @@ __global__ void __launch_bounds__(kWarps * 32) attn_prefill_kernel(const float* 
   const size_t row_stride = (size_t)s.n_kv * kHd;
   const size_t seq_base = (size_t)b * s.max_seq * row_stride + (size_t)kvh * kHd;
 
-  // key/value tile starting at key j0 into buffer buf (keys past hi: zeros)
+  // key/value tile starting at key j0 into this group's buffer buf (keys past hi: zeros)
   auto stage = [&](int buf, int j0) {
-    const uint32_t kd = sb + kOffKV + (uint32_t)(buf * 2 * kTileBytes), vd = kd + kTileBytes;
-    for (int i = threadIdx.x; i < kBk * (kHd / 8); i += kWarps * 32) {
+    const uint32_t kd = sb + kOffKV + (uint32_t)(grp * kGroupKV + buf * 2 * kTileBytes), vd = kd + kTileBytes;
+    for (int i = gt; i < kBk * (kHd / 8); i += kGT) {
       const int r = i >> 5, c = i & 31, j = j0 + r;
       if (j <= hi) {
         const size_t off = seq_base + (size_t)j * row_stride + 8 * c;
@@ -105,8 +112,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_prefill_kernel(const float* 
     }
     asm volatile("cp.async.commit_group;\n" ::: "memory");
   };
-  const int jt0 = lo & ~(kBk - 1);  // tiles aligned to 64 keys
-  stage(0, jt0);
+  const int jt0 = lo & ~(kBk - 1);  // tiles aligned to 32 keys; group grp takes tiles grp, grp + 2, ...
+  if (jt0 + grp * kBk <= hi) stage(0, jt0 + grp * kBk);
 
   // the block's queries, scaled, as fp16 (rows past the call's tokens: zeros)
   for (int i = threadIdx.x; i < kBq * (kHd / 8); i += kWarps * 32) {
@@ -134,20 +141,22 @@ __global__ void __launch_bounds__(kWarps * 32) attn_prefill_kernel(const float* 
   for (int n = 0; n < kHd / 8; ++n) O[n][0] = O[n][1] = O[n][2] = O[n][3] = 0.0f;
   float ma = -INFINITY, mb = -INFINITY, la = 0.0f, lb = 0.0f;
   const uint32_t qbase = sb + kOffQ;
+  __syncthreads();  // the queries are in shared memory
+  auto group_sync = [&]() { named_bar_sync(1 + grp, kGT); };
 
   int buf = 0;
-  for (int j0 = jt0; j0 <= hi; j0 += kBk, buf ^= 1) {
-    if (j0 + kBk <= hi) {
-      stage(buf ^ 1, j0 + kBk);
+  for (int j0 = jt0 + grp * kBk; j0 <= hi; j0 += 2 * kBk, buf ^= 1) {
+    if (j0 + 2 * kBk <= hi) {
+      stage(buf ^ 1, j0 + 2 * kBk);
       asm volatile("cp.async.wait_group 1;\n" ::: "memory");
     } else {
       asm volatile("cp.async.wait_group 0;\n" ::: "memory");
     }
-    __syncthreads();
-    const uint32_t kbase = sb + kOffKV + (uint32_t)(buf * 2 * kTileBytes), vbase = kbase + kTileBytes;
+    group_sync();
+    const uint32_t kbase = sb + kOffKV + (uint32_t)(grp * kGroupKV + buf * 2 * kTileBytes), vbase = kbase + kTileBytes;
     {  // the landed K and V tiles, bf16 -> fp16 in place
-      uint8_t* kv = smem + kOffKV + buf * 2 * kTileBytes;
-      for (int i = threadIdx.x; i < 2 * kTileBytes / 16; i += kWarps * 32) {
+      uint8_t* kv = smem + kOffKV + grp * kGroupKV + buf * 2 * kTileBytes;
+      for (int i = gt; i < 2 * kTileBytes / 16; i += kGT) {
         uint4* pchunk = reinterpret_cast<uint4*>(kv + 16 * i);
         uint4 w = *pchunk;
         w.x = bf16x2_to_f16x2(w.x);
@@ -156,10 +165,10 @@ __global__ void __launch_bounds__(kWarps * 32) attn_prefill_kernel(const float* 
         w.w = bf16x2_to_f16x2(w.w);
         *pchunk = w;
       }
-      __syncthreads();
+      group_sync();
     }
 
-    // S = Q K^T for the warp's 16 rows x 64 keys (8 n-tiles of 8 keys)
+    // S = Q K^T for the warp's 16 rows x 32 keys (4 n-tiles of 8 keys)
     float S[kBk / 8][4];
 #pragma unroll
     for (int n = 0; n < kBk / 8; ++n) S[n][0] = S[n][1] = S[n][2] = S[n][3] = 0.0f;
@@ -240,7 +249,41 @@ __global__ void __launch_bounds__(kWarps * 32) attn_prefill_kernel(const float* 
         mma_f16_16816(O[2 * d + 1], a0, a1, a2, a3, b2, b3);
       }
     }
-    __syncthreads();  // the buffer is refilled two tiles on
+    group_sync();  // the buffer is refilled two of this group's tiles on
+  }
+
+  // group 1 hands its (m, l, O) to group 0 through the key/value area (now free), laid out
+  // [value][warp][lane] so that a warp's accesses are consecutive words
+  __syncthreads();
+  float* xo = reinterpret_cast<float*>(smem + kOffKV);
+  const int slot = warp * 32 + lane;
+  if (grp == 1) {
+#pragma unroll
+    for (int n = 0; n < kHd / 8; ++n)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) xo[(4 * n + e) * kGT + slot] = O[n][e];
+    xo[128 * kGT + slot] = ma;
+    xo[129 * kGT + slot] = mb;
+    xo[130 * kGT + slot] = la;
+    xo[131 * kGT + slot] = lb;
+  }
+  __syncthreads();
+  if (grp == 1) return;
+  {
+    const float ma1 = xo[128 * kGT + slot], mb1 = xo[129 * kGT + slot];
+    const float la1 = xo[130 * kGT + slot], lb1 = xo[131 * kGT + slot];
+    const float na = fmaxf(ma, ma1), nb = fmaxf(mb, mb1);
+    const float fa0 = ma == -INFINITY ? 0.0f : expf(ma - na), fa1 = ma1 == -INFINITY ? 0.0f : expf(ma1 - na);
+    const float fb0 = mb == -INFINITY ? 0.0f : expf(mb - nb), fb1 = mb1 == -INFINITY ? 0.0f : expf(mb1 - nb);
+    la = la * fa0 + la1 * fa1;
+    lb = lb * fb0 + lb1 * fb1;
+#pragma unroll
+    for (int n = 0; n < kHd / 8; ++n) {
+      O[n][0] = O[n][0] * fa0 + xo[(4 * n + 0) * kGT + slot] * fa1;
+      O[n][1] = O[n][1] * fa0 + xo[(4 * n + 1) * kGT + slot] * fa1;
+      O[n][2] = O[n][2] * fb0 + xo[(4 * n + 2) * kGT + slot] * fb1;
+      O[n][3] = O[n][3] * fb0 + xo[(4 * n + 3) * kGT + slot] * fb1;
+    }
   }
 
   // o = O / l (rows past the call's tokens are not stored)
