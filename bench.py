@@ -63,14 +63,16 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--quick", action="store_true", help="headline only: skip the mask sweep and the tables")
-    ap.add_argument("--profile-workload", choices=["decode4", "gemm", "linear16", "prefill4", "ffn2048"], default=None,
+    ap.add_argument("--profile-workload", choices=["decode4", "gemm", "linear16", "prefill4", "ffn2048", "mid4"], default=None,
                     help="run a small fixed workload for a profiler and exit (no JSON line): 'decode4' = five "
                          "batch-1 decode steps of a 4-layer decoder with the full shapes (FFN layers 0-1 and "
                          "lm_head W8A8); 'gemm' = three bf16 and three W8A8 prefill linears, 2048 x 1152 -> 13824; "
                          "'linear16' = the single-linear workload (M 16, 1152 -> 6912) three times each as W8A8 "
                          "on INT8 codes, W8A8 with the fp16 code copy and bf16, then three W8A8 FFN blocks at M 8; "
                          "'prefill4' = a 2048-token prefill of a 4-layer decoder with the full shapes (bf16); "
-                         "'ffn2048' = three W8A8 and three bf16 FFN blocks at M 2048")
+                         "'ffn2048' = three W8A8 and three bf16 FFN blocks at M 2048; 'mid4' = two 128-token "
+                         "prefills (batch 1) and three batch-32 decode steps of a 4-layer decoder with the full "
+                         "shapes (bf16)")
     return ap.parse_args()
 
 
@@ -90,6 +92,19 @@ def profile_workload(name):
         toks = torch.from_numpy(synth.tokens(2048, VOCAB, seed=2)).to(dev).view(1, 2048)
         for _ in range(2):
             dec.forward(toks, 0, want_logits=False)
+        torch.cuda.synchronize()
+        dec.close()
+    elif name == "mid4":
+        LAYERS = 4
+        f32, bf, norms = synth.decoder_weights(4, seed=0, want_f32=False)
+        dec, _ = make_decoder(B, dev, bf, norms, max_batch=32, max_seq=512, max_tokens=2048)
+        toks = torch.from_numpy(synth.tokens(32 * 128, VOCAB, seed=2)).to(dev).view(32, 128)
+        for _ in range(2):
+            dec.forward(toks[:1].contiguous(), 0, want_logits=False)
+        prefill(dec, toks, 2048)
+        top = torch.zeros(32, dtype=torch.int32, device=dev)
+        for s in range(3):
+            dec.decode_step(top, 128 + s, top1=top)
         torch.cuda.synchronize()
         dec.close()
     elif name == "decode4":

@@ -65,7 +65,7 @@ LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
   w.sx = off;
   if (int8_path) off += round_up((size_t)M * 4, 256);
   w.part = off;
-  off += round_up(make_stream_plan(int8_path, M, N, K, sms).partial_bytes, 256);
+  off += round_up(std::max(make_stream_plan(int8_path, M, N, K, sms).partial_bytes, tc_split_partial_bytes(M, sms)), 256);
   w.total = off;
   return w;
 }
@@ -150,7 +150,8 @@ constexpr int kTcMinTokens = 64, kTcMinTokensNarrow = 9, kTcNarrowMaxN = 16384;
 
 static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N, int K, const float* bias, int kind,
                     const float* inv_delta, const float* s_w, uint16_t* Y, float* logits, int32_t* top1,
-                    const w8a8_debug* dbg, void* ws, void* codes, float* s_x, cudaStream_t st, w8a8_status* status) {
+                    const w8a8_debug* dbg, void* ws, void* codes, float* s_x, void* part, cudaStream_t st,
+                    w8a8_status* status) {
   if (M < (N <= kTcNarrowMaxN ? kTcMinTokensNarrow : kTcMinTokens) || !W16 ||
       !tc_gemm_supported(M, N, K, kind, top1 != nullptr, max_top_keys()))
     return false;
@@ -187,6 +188,8 @@ static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N,
   a.grid_counter = r.grid_counter;
   a.top_keys = r.top_keys;
   a.err = r.err;
+  a.partials = part;
+  a.tile_counters = r.tile_counters;
   *status = launch_tc_gemm(int8, a, st);
   return true;
 }
@@ -205,8 +208,8 @@ w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, con
   char* base = reinterpret_cast<char*>(ws);
   void* codes = base + L.xf16;
   float* s_x = reinterpret_cast<float*>(base + L.sx);
-  if (tc_path(true, w->wq_f16, X, M, N, K, bias, kind, w->inv_delta, w->s_w, Y, logits, top1, dbg, ws, codes, s_x, st,
-              &small_status))
+  if (tc_path(true, w->wq_f16, X, M, N, K, bias, kind, w->inv_delta, w->s_w, Y, logits, top1, dbg, ws, codes, s_x,
+              base + L.part, st, &small_status))
     return small_status;
   StreamArgs a{};
   a.p = make_stream_plan(true, M, N, K, sms);
@@ -238,10 +241,10 @@ w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, 
       small_gemv(false, W, nullptr, nullptr, X, M, N, K, bias, kind, Y, nullptr, ws, rn, sms, st, &small_status))
     return small_status;
   W8A8_CHECK_ARG(!rn, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take M=%d N=%d K=%d", M, N, K);
-  if (tc_path(false, W, X, M, N, K, bias, kind, nullptr, nullptr, Y, logits, top1, nullptr, ws, nullptr, nullptr, st,
-              &small_status))
-    return small_status;
   LinearWs L = linear_ws(M, N, K, false, sms);
+  if (tc_path(false, W, X, M, N, K, bias, kind, nullptr, nullptr, Y, logits, top1, nullptr, ws, nullptr, nullptr,
+              reinterpret_cast<char*>(ws) + L.part, st, &small_status))
+    return small_status;
   StreamArgs a{};
   a.W = W;
   a.X = X;
@@ -396,7 +399,7 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
                        f->gate_up.s_w, h, nullptr, nullptr, nullptr, workspace,
                        base + L.gu + (linear_ws(M, 2 * F, H, true, sms).xf16 - W8A8_WS_RESERVED),
                        reinterpret_cast<float*>(base + L.gu + (linear_ws(M, 2 * F, H, true, sms).sx - W8A8_WS_RESERVED)),
-                       st, &ss)) {
+                       base + L.gu + (linear_ws(M, 2 * F, H, true, sms).part - W8A8_WS_RESERVED), st, &ss)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs A = linear_ws(M, 2 * F, H, true, sms);
@@ -424,8 +427,8 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     } else if (tc_path(true, f->down.wq_f16, h, M, H, F, nullptr, EPI_BF16, f->down.inv_delta, f->down.s_w, Y,
                        nullptr, nullptr, nullptr, workspace,
                        base + L.dn + (linear_ws(M, H, F, true, sms).xf16 - W8A8_WS_RESERVED),
-                       reinterpret_cast<float*>(base + L.dn + (linear_ws(M, H, F, true, sms).sx - W8A8_WS_RESERVED)), st,
-                       &ss)) {
+                       reinterpret_cast<float*>(base + L.dn + (linear_ws(M, H, F, true, sms).sx - W8A8_WS_RESERVED)),
+                       base + L.dn + (linear_ws(M, H, F, true, sms).part - W8A8_WS_RESERVED), st, &ss)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs B = linear_ws(M, H, F, true, sms);
@@ -455,7 +458,8 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
     } else if (rn_gate_up) {
       W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take gate/up at M=%d", M);
     } else if (tc_path(false, f->gate_up_bf16, X, M, 2 * F, H, nullptr, EPI_GEGLU, nullptr, nullptr, h, nullptr,
-                       nullptr, nullptr, workspace, nullptr, nullptr, st, &ss)) {
+                       nullptr, nullptr, workspace, nullptr, nullptr,
+                       base + L.gu + (linear_ws(M, 2 * F, H, false, sms).part - W8A8_WS_RESERVED), st, &ss)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs A = linear_ws(M, 2 * F, H, false, sms);
@@ -476,7 +480,8 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
                    nullptr, sms, st, &ss)) {
       W8A8_TRY(ss);
     } else if (tc_path(false, f->down_bf16, h, M, H, F, nullptr, EPI_BF16, nullptr, nullptr, Y, nullptr, nullptr,
-                       nullptr, workspace, nullptr, nullptr, st, &ss)) {
+                       nullptr, workspace, nullptr, nullptr,
+                       base + L.dn + (linear_ws(M, H, F, false, sms).part - W8A8_WS_RESERVED), st, &ss)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs B = linear_ws(M, H, F, false, sms);

@@ -217,6 +217,53 @@ __device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap*
   }
 }
 
+// The last unit of a split tile: the 512 epilogue threads sum the tile's KS partials (units u0 ..
+// u0 + KS - 1) in part order, four columns per thread with every part's load in flight, and write
+// the bf16 outputs (W8A8: the INT32 sums dequantised exactly as the tile epilogue does it).
+template <bool kInt8, int BN>
+__device__ __forceinline__ void split_reduce(const TcArgs& a, int u0, int KS, int R, int m0, int n0) {
+  const uint4* part = reinterpret_cast<const uint4*>(a.partials) + (size_t)u0 * R * (BN / 4);
+  const size_t pstride = (size_t)R * (BN / 4);
+  for (int e = threadIdx.x; e < R * (BN / 4); e += 32 * kEpiWarps) {
+    const int r = e / (BN / 4), c = 4 * (e % (BN / 4));
+    const int row = m0 + r, col = n0 + c;
+    if (row >= a.M || col >= a.N) continue;  // N is a multiple of 16: four columns are all in or out
+    const uint4* p = part + e;
+    float y[4];
+    if constexpr (kInt8) {
+      int s[4] = {0, 0, 0, 0};
+#pragma unroll 8
+      for (int sp = 0; sp < KS; ++sp) {
+        const uint4 v = __ldcg(p + sp * pstride);
+        s[0] += (int)v.x;
+        s[1] += (int)v.y;
+        s[2] += (int)v.z;
+        s[3] += (int)v.w;
+      }
+      const float sx = a.s_x[row];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) y[k] = __fmul_rn(__fmul_rn(sx, a.s_w[col + k]), __int2float_rn(s[k]));
+      if (a.acc_dbg)
+        *reinterpret_cast<int4*>(a.acc_dbg + (size_t)row * a.N + col) = make_int4(s[0], s[1], s[2], s[3]);
+    } else {
+      y[0] = y[1] = y[2] = y[3] = 0.0f;
+#pragma unroll 8
+      for (int sp = 0; sp < KS; ++sp) {
+        const uint4 v = __ldcg(p + sp * pstride);
+        y[0] = __fadd_rn(y[0], __uint_as_float(v.x));
+        y[1] = __fadd_rn(y[1], __uint_as_float(v.y));
+        y[2] = __fadd_rn(y[2], __uint_as_float(v.z));
+        y[3] = __fadd_rn(y[3], __uint_as_float(v.w));
+      }
+    }
+    if (a.bias) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) y[k] = __fadd_rn(y[k], a.bias[col + k]);
+    }
+    *reinterpret_cast<uint2*>(a.y + (size_t)row * a.N + col) = make_uint2(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]));
+  }
+}
+
 template <bool kInt8, int kBN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -227,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
   __shared__ uint32_t tmem_slot;
-  __shared__ int s_flag;
+  __shared__ int s_flag, s_last;
 
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -235,12 +282,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + kBM - 1) / kBM);
   const int nkb = (a.K + kBK - 1) / kBK;
-  const int nchunks = kInt8 ? (nkb + kKbPerChunk - 1) / kKbPerChunk : 1;
-  const int kb_per_chunk = kInt8 ? kKbPerChunk : nkb;
+  // work units: (tile, k part); unit u is part u mod KS of tile u / KS, stages [kb_lo, kb_hi)
+  const int KS = a.ksplit > 1 ? a.ksplit : 1, units = tiles * KS;
+  auto kb_lo = [&](int u) { return (int)((long long)(u % KS) * nkb / KS); };
+  auto kb_hi = [&](int u) { return (int)((long long)(u % KS + 1) * nkb / KS); };
+  // accumulator chunks of a unit: W8A8 restarts every 1024 k counted from the unit's first stage
+  auto chunks_of = [&](int u) { return kInt8 ? (kb_hi(u) - kb_lo(u) + kKbPerChunk - 1) / kKbPerChunk : 1; };
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
                  done = acce0 + 8 * NSLOT;
 
   pdl_trigger();
+  if (warp == kProdWarp && lane == 0) {
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+    prefetch_tmap(&tmY);
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full0 + 8 * s, 1);
@@ -265,16 +321,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = tmem_slot;
   pdl_wait();  // activations and outputs belong to the preceding kernels
 
-  // Persistent: CTA b takes tiles b, b + grid, ...; tile t covers channels (t mod NT) * BN and
+  // Persistent: CTA b takes units b, b + grid, ...; tile t covers channels (t mod NT) * BN and
   // tokens (t / NT) * 128, so neighbouring CTAs share the activation rows.
   if (warp == kProdWarp) {
     // ---------------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
       int g = 0;  // stages issued
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        const int n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
-        for (int kb = 0; kb < nkb; ++kb, ++g) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const int t = u / KS, n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
+        const int kb_end = kb_hi(u);
+        for (int kb = kb_lo(u); kb < kb_end; ++kb, ++g) {
           const int s = g % S;
           if (!mbar_wait_bounded(empty0 + 8 * s, (uint32_t)(((g / S) & 1) ^ 1), kWaitBudgetCycles)) {
             ok = false;
@@ -300,8 +357,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc = idesc_f16(kInt8 ? 0u : 1u, BN, kBM);
       bool ok = true;
       int g = 0, q = 0;  // stages consumed, accumulator chunks produced
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        for (int c = 0; c < nchunks && ok; ++c, ++q) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const int nch = chunks_of(u), ulo = kb_lo(u), uhi = kb_hi(u);
+        for (int c = 0; c < nch && ok; ++c, ++q) {
           const int slot = q % NSLOT;
           if (q >= NSLOT &&  // the epilogue has drained this slot's previous chunk
               !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
@@ -310,7 +368,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(slot * SC);
-          const int kb0 = c * kb_per_chunk, kb1 = min(nkb, kb0 + kb_per_chunk);
+          const int kb0 = kInt8 ? ulo + c * kKbPerChunk : ulo, kb1 = kInt8 ? min(uhi, kb0 + kKbPerChunk) : uhi;
           for (int kb = kb0; kb < kb1; ++kb, ++g) {
             const int s = g % S;
             if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
@@ -341,19 +399,49 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t buf = stg + (uint32_t)(warp * kStageBufBytes);
     bool ok = true;
     int q = 0;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-      const int n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
-      const int row = m0 + 32 * quad + lane;
+    // split-K partials (bf16 outputs only): unit u's block of R rows x BN columns, row-major; a
+    // thread stores its row's 32 sums of a column group as 16-byte vectors (W8A8: the INT32 sums,
+    // bf16: the fp32 ones)
+    const int R = a_box_rows(a.M), rloc = 32 * quad + lane;
+    const bool has_row = rloc < R;
+    auto store_part32 = [&](int u, int g, const uint32_t (&w)[32]) {
+      uint32_t* p = reinterpret_cast<uint32_t*>(a.partials) + ((size_t)u * R + rloc) * BN + 32 * g;
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        __stcg(reinterpret_cast<uint4*>(p) + k, make_uint4(w[4 * k], w[4 * k + 1], w[4 * k + 2], w[4 * k + 3]));
+    };
+    for (int u = blockIdx.x; u < units; u += gridDim.x) {
+      const int t = u / KS, n0 = (t % NT) * BN, m0 = (t / NT) * kBM;
+      const int row = m0 + rloc;
       unsigned long long best = 0ull;
       auto emit32 = [&](int c0, const float (&v)[32]) {
         stage_cols32(a, &tmY, buf, m0 + 32 * quad, n0 + c0, lane, v, want_top, best);
+      };
+      // After this unit's partials are stored: true when the unit is the tile's last to arrive (it
+      // then sums all parts in part order); false, or a failed wait anywhere in the epilogue, ends it.
+      auto arrive_last = [&]() -> bool {
+        __threadfence();
+        if (!named_bar_all(2, 32 * kEpiWarps, ok)) {
+          ok = false;
+          return false;
+        }
+        if (threadIdx.x == 0) {
+          const unsigned int prev = atomicAdd(a.tile_counters + t, 1u);
+          s_last = prev == (unsigned int)(KS - 1);
+          if (s_last) a.tile_counters[t] = 0u;
+        }
+        named_bar_sync(2, 32 * kEpiWarps);
+        if (!s_last) return false;
+        __threadfence();
+        return true;
       };
       if constexpr (kInt8) {
         constexpr int NG = (BN / 32 + kParts - 1) / kParts;  // this warp's 32-column groups: part + kParts i
         int isum[32 * NG];
 #pragma unroll
         for (int j = 0; j < 32 * NG; ++j) isum[j] = 0;
-        for (int c = 0; c < nchunks; ++c, ++q) {
+        const int nch = chunks_of(u);
+        for (int c = 0; c < nch; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
             ok = false;
@@ -373,7 +461,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
           mbar_arrive(acce0 + 8 * slot);
         }
-        if (!ok) break;
+        if (KS > 1) {
+          if (ok && has_row) {
+#pragma unroll
+            for (int i = 0; i < NG; ++i) {
+              const int g = part + kParts * i;
+              if (g >= BN / 32) break;
+              store_part32(u, g, reinterpret_cast<const uint32_t(&)[32]>(isum[32 * i]));
+            }
+          }
+          if (arrive_last()) split_reduce<true, BN>(a, t * KS, KS, R, m0, n0);
+          if (!ok) break;
+          continue;
+        } else if (!ok) {
+          break;
+        }
         const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
         for (int i = 0; i < NG; ++i) {
@@ -398,26 +500,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
           ok = false;
           atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+        } else {
+          tc_fence_after();
+#pragma unroll 1
+          for (int g = part; g < BN / 32; g += kParts) {
+            uint32_t r[32];
+            tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
+            if (KS > 1) {  // this part's fp32 sums go to the partials
+              if (has_row) store_part32(u, g, r);
+              continue;
+            }
+            float v[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const int col = n0 + 32 * g + j;
+              float y = __uint_as_float(r[j]);
+              if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
+              v[j] = y;
+            }
+            emit32(32 * g, v);
+          }
+          tc_fence_before();
+          mbar_arrive(acce0 + 8 * slot);
+        }
+        ++q;
+        if (KS > 1) {
+          if (arrive_last()) split_reduce<false, BN>(a, t * KS, KS, R, m0, n0);
+          if (!ok) break;
+          continue;
+        } else if (!ok) {
           break;
         }
-        tc_fence_after();
-#pragma unroll 1
-        for (int g = part; g < BN / 32; g += kParts) {
-          uint32_t r[32];
-          tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
-          float v[32];
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int col = n0 + 32 * g + j;
-            float y = __uint_as_float(r[j]);
-            if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
-            v[j] = y;
-          }
-          emit32(32 * g, v);
-        }
-        tc_fence_before();
-        mbar_arrive(acce0 + 8 * slot);
-        ++q;
       }
       if (want_top && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
     }
@@ -538,6 +651,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                  done = acce0 + 8 * NSLOT;
 
   pdl_trigger();
+  if (warp == kProdWarp && lane == 0) {
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+    prefetch_tmap(&tmY);
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full0 + 8 * s, 1);
@@ -775,7 +893,7 @@ w8a8_status launch_t(const TcArgs& a, cudaStream_t st) {
   CUtensorMap ty;
   W8A8_TRY(make_out_map(a, &ty, ta));
   const long long tiles = (long long)((a.N + GG::BN - 1) / GG::BN) * ((a.M + kBM - 1) / kBM);
-  const dim3 grid((unsigned)std::min<long long>(tiles, device_sms()));
+  const dim3 grid((unsigned)std::min<long long>(tiles * std::max(a.ksplit, 1), device_sms()));
   W8A8_CUDA(launch_pdl(gemm_tc_kernel<kInt8, kBN>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, ty, a));
   return W8A8_OK;
 }
@@ -808,8 +926,36 @@ w8a8_status launch_t2(const TcArgs& a, cudaStream_t st) {
 // to one-wave timings on K = 6912, where a narrower tile spends relatively more of each k step on
 // operand traffic through shared memory; the last estimated from its operand bytes per MMA).
 // Narrow tiles win where the wide ones would leave SMs idle, as at decode-sized token counts.
+//
+// Split-K: where a single-CTA bf16-output shape leaves more than half of the SMs without a tile
+// (few tokens and a narrow output, as the attention projections and the down projection at decode
+// batch sizes), the k range of every tile is cut into parts on different CTAs (at most one unit per
+// SM, at least kMinKbPerPart stages per part).  Each CTA streams its part of the weights at the
+// per-SM copy rate, so the spread is what reaches HBM bandwidth.
+constexpr int kMinKbPerPart = 2;
+
+// The parts are also capped at K / (4 R), so that the partials a tile's last unit reads back (KS R
+// BN fp32) stay below half of the tile's weight bytes (BN K bf16), and fewer than kMinParts parts
+// are not worth the arrival protocol.  Measured: 6-8 parts on q/k/v and o at 32 tokens save 1.5 us
+// of 10-11, the down projection drops from 34 to 12-16 us, and q/k/v and o at 128 tokens (2 parts
+// under the cap) would lose.
+constexpr int kMinParts = 4;
+
+template <bool kInt8, int kBN>
+w8a8_status launch_split(TcArgs a, cudaStream_t st) {
+  const int sms = device_sms(), nkb = (a.K + kBK - 1) / kBK;
+  const long long tiles = (long long)((a.N + kBN - 1) / kBN) * ((a.M + kBM - 1) / kBM);
+  a.ksplit = 1;
+  if (a.kind == EPI_BF16 && a.partials && a.tile_counters && 2 * tiles <= sms) {
+    const int ks = std::min({(int)(sms / tiles), nkb / kMinKbPerPart, a.K / (4 * a_box_rows(a.M))});
+    if (ks >= kMinParts) a.ksplit = ks;
+  }
+  return launch_t<kInt8, kBN>(a, st);
+}
+
 template <bool kInt8>
-w8a8_status dispatch(const TcArgs& a, cudaStream_t st) {
+w8a8_status dispatch(TcArgs a, cudaStream_t st) {
+  a.ksplit = 1;
   const long long pairs = device_sms() / 2;
   auto cost = [&](int bm, int bn, double unit, long long slots) {
     const long long t = (long long)((a.N + bn - 1) / bn) * ((a.M + bm - 1) / bm);
@@ -819,8 +965,8 @@ w8a8_status dispatch(const TcArgs& a, cudaStream_t st) {
                c128 = cost(kBM, 128, 1.81, 2 * pairs), c64 = cost(kBM, 64, 2.7, 2 * pairs);
   if (c256 <= c192 && c256 <= c128 && c256 <= c64) return launch_t2<kInt8, 256>(a, st);
   if (c192 <= c128 && c192 <= c64) return launch_t2<kInt8, 192>(a, st);
-  if (c128 <= c64) return launch_t<kInt8, 128>(a, st);
-  return launch_t<kInt8, 64>(a, st);  // few tokens: spread the weight stream over more SMs
+  if (c128 <= c64) return launch_split<kInt8, 128>(a, st);
+  return launch_split<kInt8, 64>(a, st);  // few tokens: spread the weight stream over more SMs
 }
 
 }  // namespace
@@ -830,6 +976,11 @@ bool tc_gemm_supported(int M, int N, int K, int kind, bool want_top, int max_top
   if (kind != EPI_BF16 && kind != EPI_GEGLU && kind != EPI_F32) return false;
   if (want_top && M > max_top) return false;
   return true;
+}
+
+size_t tc_split_partial_bytes(int M, int sms) {
+  // at most one unit per SM, BN <= 128 on the single-CTA kernel, R = a_box_rows(M) rows per unit
+  return (size_t)std::max(sms, 1) * 128 * (size_t)a_box_rows(std::max(M, 1)) * 4;
 }
 
 w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st) {

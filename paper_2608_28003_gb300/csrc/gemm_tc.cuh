@@ -21,11 +21,18 @@ struct TcArgs {
   unsigned int* grid_counter;     // top-1: one counter, zero between calls
   unsigned long long* top_keys;   // top-1: [M] keys, zero between calls
   unsigned int* err;              // device error word
+  // split-K (few output tiles): the k range of a tile is cut into ksplit parts on different CTAs
+  int ksplit;                     // set by the launcher (1: no split)
+  void* partials;                 // tc_split_partial_bytes(M) bytes of workspace
+  unsigned int* tile_counters;    // one per output tile, zero between calls
 };
 
 // Shapes the tensor-core GEMM takes: K a multiple of 16, N a multiple of 16, top-1 for at most
 // max_top rows.
 bool tc_gemm_supported(int M, int N, int K, int kind, bool want_top, int max_top);
+// Workspace bytes the split-K partials of an M-token call may take (an upper bound over N and K,
+// non-decreasing in M).
+size_t tc_split_partial_bytes(int M, int sms);
 w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st);
 
 }  // namespace w8a8

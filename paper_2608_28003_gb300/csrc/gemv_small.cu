@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     bool ok = true;
     int it = 0, s = 0;
     uint32_t ph = 0;
+    const uint64_t wpol = l2_evict_first_policy();  // each weight row is read once per call
     for (; it < nst; ++it) {
       if (!mbar_wait_bounded(smem_u32(empty + s), ph ^ 1u, kWaitBudgetCycles)) {
         ok = false;
@@ -112,10 +113,10 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int u = 0; u < cnt; ++u) {
         const uint32_t d = dst + (uint32_t)(u * R * kSliceBytes);
         if constexpr (kInt8) {
-          tma_load_2d(d, &tmW, (u0 + u) * 512, row0, bar);
-          tma_load_2d(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar);
+          tma_load_2d_policy(d, &tmW, (u0 + u) * 512, row0, bar, wpol);
+          tma_load_2d_policy(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar, wpol);
         } else {
-          tma_load_2d(d, &tmW, (u0 + u) * 256, row0, bar);
+          tma_load_2d_policy(d, &tmW, (u0 + u) * 256, row0, bar, wpol);
         }
       }
       if (++s == S) {

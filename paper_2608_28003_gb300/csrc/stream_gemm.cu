@@ -583,6 +583,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     constexpr int nw = KC / 128;
     bool ok = true;
     long long it = 0;
+    const uint64_t wpol = l2_evict_first_policy();  // every weight box is read once per call
     for (long long u = u0; u < u1; ++u, ++it) {
       const int s = (int)(it % S);
       const uint32_t ph = (uint32_t)((it / S) & 1);
@@ -593,7 +594,8 @@ __global__ void __launch_bounds__(kThreads, 2)
       const int g = (int)(u / C), ch = (int)(u % C);
       const uint32_t bar = smem_u32(full + s);
       mbar_arrive_expect_tx(bar, (uint32_t)(nw * kBox));
-      for (int b = 0; b < nw; ++b) tma_load_2d(ring + (uint32_t)s * SB + b * kBox, &tmW, ch * KC + b * 128, g * 128, bar);
+      for (int b = 0; b < nw; ++b)
+        tma_load_2d_policy(ring + (uint32_t)s * SB + b * kBox, &tmW, ch * KC + b * 128, g * 128, bar, wpol);
     }
     if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
     for (long long j = it > S ? it - S : 0; j < it; ++j) {

@@ -153,6 +153,9 @@ TC_SHAPES = [
     (9, 1536, 1152),     # fewest tokens the tensor-core path takes
     (40, 1152, 6912),    # ragged M, seven k chunks
     (64, 1152, 6912),    # seven 1024-k chunks folded into INT32
+    (32, 1152, 6912),    # split-K: 18 tiles of 128 x 64, k cut into 8 parts on 144 CTAs
+    (200, 1152, 6912),   # split-K over two row blocks of a ragged M, parts of 27 stages
+    (24, 1040, 4096),    # split-K with a bias added once, after the parts are summed
     (130, 4112, 1040),   # ragged M, K not a multiple of the 64-wide stage
     (256, 1536, 1152),
     (200, 13824, 1152),  # gate/up shape, ragged M: CTA pairs on 256 x 192 tiles
@@ -169,8 +172,9 @@ def test_w8a8_linear_tensor_core_bit_exact(B, M, N, K):
     x32, x, w32, w, c32, c = _case(M, N, K, seed=M * 3 + K)
     stat = OW.act_absmax(np.concatenate([c32, x32]))
     q = B.prepare_weights(cu(w), cu(torch.from_numpy(stat)), want_f16=True)
-    Y, dbg = B.linear(q, cu(x), debug=True)
-    r = OW.w8a8_linear(x32, OW.prepare_weights(w32, stat), out="bf16")
+    bias = np.random.default_rng(2).standard_normal(N).astype(np.float32) if N == 1040 else None
+    Y, dbg = B.linear(q, cu(x), bias=cu(torch.from_numpy(bias)) if bias is not None else None, debug=True)
+    r = OW.w8a8_linear(x32, OW.prepare_weights(w32, stat), bias=bias, out="bf16")
     assert np.array_equal(dbg["xq"].cpu().numpy(), r["xq"])
     assert np.array_equal(dbg["s_x"].cpu().numpy(), r["s_x"])
     assert np.array_equal(dbg["acc"].cpu().numpy().astype(np.int64), r["acc"])
@@ -226,10 +230,13 @@ def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarr
 @pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040),
                                    (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152),
                                    (128, 6912, 1152), (70, 1152, 6912), (300, 256, 64),
+                                   (32, 1152, 4608),     # split-K: 18 tiles, k cut into 8 parts
+                                   (200, 1152, 6912),    # split-K over two row blocks
                                    (300, 19472, 1152),   # CTA pairs on 256 x 192 tiles, ragged M and N
                                    (1024, 13824, 1152)])  # CTA pairs on 256 x 256 tiles
 def test_bf16_linear_within_tolerance(B, M, N, K):
     x32, x, w32, w, _, _ = _case(M, N, K, seed=11 + M)
-    Y = B.linear_bf16(cu(w), cu(x))
-    ref = OW.bf16_linear(x32, w32, out="bf16")
+    bias = np.random.default_rng(3).standard_normal(N).astype(np.float32) if M == 32 else None
+    Y = B.linear_bf16(cu(w), cu(x), bias=cu(torch.from_numpy(bias)) if bias is not None else None)
+    ref = OW.bf16_linear(x32, w32, bias=bias, out="bf16")
     _bf16_close(f32_of_bf16(Y), x32, w32, ref)
