@@ -61,6 +61,15 @@ __device__ __forceinline__ float consumer_sum(float v, float* red, int warp, int
   return t;
 }
 
+__device__ __forceinline__ void ldm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];\n" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+__device__ __forceinline__ void ldm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
 __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
   x[0] = bf16_lo(v.x); x[1] = bf16_hi(v.x); x[2] = bf16_lo(v.y); x[3] = bf16_hi(v.y);
   x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
@@ -70,6 +79,11 @@ template <bool kInt8, int MT, int RW>
 __global__ void __launch_bounds__(kThreads, 2)
     gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
   constexpr int R = 8 * RW;
+  // bf16 at 5-8 tokens: the products run on the tensor cores (mma.sync m16n8k16, the activations
+  // as the A operand with token rows 8-15 zero, each 8 weight rows an n-tile), the 8 consumer warps
+  // taking alternate k steps of every stage; the weights arrive as 128-byte-swizzled boxes of 64
+  // columns and the activation rows are padded by 16 bytes, so the fragment loads hit distinct banks
+  constexpr bool kMma = !kInt8 && MT == 8;
   using Acc = typename std::conditional<kInt8, int, float>::type;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ float s_red[kCW];
@@ -80,7 +94,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t ring = (raw + 1023u) & ~1023u;
   const uint32_t xs = ring + (uint32_t)(S * SB);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (ring - raw) + (size_t)S * SB + p.xbytes + p.abytes);
+  uint64_t* full =
+      reinterpret_cast<uint64_t*>(smem_raw + (ring - raw) + (size_t)S * SB + p.xbytes + p.abytes + p.rbytes);
   uint64_t* empty = full + S;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row0 = blockIdx.x * R;
@@ -115,6 +130,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         if constexpr (kInt8) {
           tma_load_2d_policy(d, &tmW, (u0 + u) * 512, row0, bar, wpol);
           tma_load_2d_policy(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar, wpol);
+        } else if constexpr (kMma) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) tma_load_2d_policy(d + j * R * 128, &tmW, (u0 + u) * 256 + 64 * j, row0, bar, wpol);
         } else {
           tma_load_2d_policy(d, &tmW, (u0 + u) * 256, row0, bar, wpol);
         }
@@ -173,6 +191,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   // (thread t < K / 8 owns channels 8t .. 8t+7 of every token, as in the residual-norm kernel).
   const uint16_t* xrows = a.X;
   int xstride = a.K;
+  const int xsb = kMma ? kpad + 8 : kpad;  // elements between the bf16 activation rows in shared memory
   if (a.has_rn) {
     uint16_t* as = kInt8 ? reinterpret_cast<uint16_t*>(xsp + p.xbytes) : reinterpret_cast<uint16_t*>(xsp);
     for (int m = 0; m < MT; ++m) {
@@ -214,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 2)
           w.z = (uint32_t)f32_to_bf16_bits(o[4]) | ((uint32_t)f32_to_bf16_bits(o[5]) << 16);
           w.w = (uint32_t)f32_to_bf16_bits(o[6]) | ((uint32_t)f32_to_bf16_bits(o[7]) << 16);
         }
-        *reinterpret_cast<uint4*>(as + (size_t)m * kpad + 8 * tid) = w;
+        *reinterpret_cast<uint4*>(as + (size_t)m * (kInt8 ? kpad : xsb) + 8 * tid) = w;
       }
     }
     named_bar_sync(1, kCW * 32);
@@ -355,7 +374,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const int i = i0 + u * kCW * 32;
-        if (i < total) *reinterpret_cast<uint4*>(xsp + (size_t)i * 16) = val[u];
+        const int m = i / vpr, v = i - m * vpr;
+        if (i < total) *reinterpret_cast<uint4*>(xsp + ((size_t)m * xsb + 8 * v) * 2) = val[u];
       }
     }
   }
@@ -371,6 +391,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int i = 0; i < RW; ++i)
 #pragma unroll
       for (int m = 0; m < MT; ++m) acc[c][i][m] = 0;
+  float mc[2][RW][4];  // MMA path: two accumulator sets (alternate k steps), per n-tile of 8 rows
+#pragma unroll
+  for (int c = 0; c < 2; ++c)
+#pragma unroll
+    for (int i = 0; i < RW; ++i) mc[c][i][0] = mc[c][i][1] = mc[c][i][2] = mc[c][i][3] = 0.0f;
   bool ok = true;
   // INT8 sub-slice: two boxes [R][256 B]; lane l reads box l / 16 at byte 16 (l % 16) of the row
   const uint32_t wlane = kInt8 ? (uint32_t)((lane >> 4) * R * 256 + 16 * (lane & 15)) : (uint32_t)(16 * lane);
@@ -386,7 +411,41 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (lane == 0) atomicOr(a.err, DEVERR_CONSUMER_WAIT);
       }
     }
-    if (ok) {
+    if (ok && kMma) {
+      // k steps of 16 of this stage: step q is sub-slice q / 16, 64-column box (q % 16) / 4,
+      // chunks 2 (q % 4) and 2 (q % 4) + 1 of its rows; warp w takes steps w, w + 8, ...
+      const uint32_t sb = ring + (uint32_t)(s * SB);
+      const int u0 = it * KS, cnt = min(KS, nsub - u0);
+      const int xr = lane & 7, xh = (lane >> 3) & 1;  // ldmatrix row addresses: token / half
+      auto step = [&](int q, float (&c)[RW][4]) {
+        const int u = q >> 4, kk = q & 15, c0 = 2 * (kk & 3);
+        const uint32_t box = sb + (uint32_t)(u * R * kSliceBytes + (kk >> 2) * R * 128);
+        const int kg = (u0 + u) * 256 + 16 * kk;
+        uint32_t a0, a2;
+        ldm_x2(xs + (uint32_t)((xr * xsb + kg + 8 * xh) * 2), a0, a2);
+#pragma unroll
+        for (int i = 0; i < RW; i += 2) {
+          if (i + 1 < RW) {  // n-tiles i and i + 1: matrices (i, k lo), (i, k hi), (i + 1, lo), (i + 1, hi)
+            const int mi = lane >> 3, r = 8 * (i + (mi >> 1)) + xr, ch = c0 + (mi & 1);
+            uint32_t b0, b1, b2, b3;
+            ldm_x4(box + (uint32_t)(r * 128 + ((ch ^ xr) << 4)), b0, b1, b2, b3);
+            mma_bf16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
+            mma_bf16_16816(c[i + 1], a0, 0u, a2, 0u, b2, b3);
+          } else {
+            const int r = 8 * i + xr, ch = c0 + xh;
+            uint32_t b0, b1;
+            ldm_x2(box + (uint32_t)(r * 128 + ((ch ^ xr) << 4)), b0, b1);
+            mma_bf16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
+          }
+        }
+      };
+      for (int q = warp; q < 16 * cnt; q += 2 * kCW) {  // alternate steps feed the two accumulator sets
+        step(q, mc[0]);
+        if (q + kCW < 16 * cnt) step(q + kCW, mc[1]);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(empty + s));
+    } else if (ok) {
       const uint32_t sb = ring + (uint32_t)(s * SB);
       const int u0 = it * KS, cnt = min(KS, nsub - u0);
 #pragma unroll
@@ -437,6 +496,42 @@ __global__ void __launch_bounds__(kThreads, 2)
       s = 0;
       ph ^= 1u;
     }
+  }
+  if constexpr (kMma) {
+    // Each warp's sums (accumulator c0 / c1 of n-tile i: token g, rows 8 i + 2 t and + 1) go to
+    // shared memory [warp][row][token]; then every output sums the 8 warps in warp order.
+    float* part = reinterpret_cast<float*>(xsp + p.xbytes + p.abytes);
+    const int g = lane >> 2, t = lane & 3;
+    if (ok) {
+#pragma unroll
+      for (int i = 0; i < RW; ++i) {
+        part[(warp * R + 8 * i + 2 * t) * 8 + g] = mc[0][i][0] + mc[1][i][0];
+        part[(warp * R + 8 * i + 2 * t + 1) * 8 + g] = mc[0][i][1] + mc[1][i][1];
+      }
+    }
+    if (!named_bar_all(1, kCW * 32, ok)) return;
+    auto total = [&](int r, int m) {
+      float v = 0.0f;
+#pragma unroll
+      for (int w = 0; w < kCW; ++w) v += part[(w * R + r) * 8 + m];
+      return a.bias ? __fadd_rn(v, a.bias[row0 + r]) : v;
+    };
+    if (a.kind == EPI_GEGLU) {  // pair b of block j: gate row 16 j + b, up row 16 j + 8 + b
+      for (int e = tid; e < (R / 2) * 8; e += kCW * 32) {
+        const int pr = e >> 3, m = e & 7, j = pr >> 3, b = pr & 7;
+        const int gr = 16 * j + b;
+        if (m >= a.M || row0 + gr + 8 >= a.N) continue;
+        a.y[(size_t)m * (a.N >> 1) + ((row0 + 16 * j) >> 1) + b] =
+            f32_to_bf16_bits(geglu_recipe(total(gr, m), total(gr + 8, m)));
+      }
+    } else {
+      for (int e = tid; e < R * 8; e += kCW * 32) {
+        const int r = e >> 3, m = e & 7;
+        if (m >= a.M || row0 + r >= a.N) continue;
+        a.y[(size_t)m * a.N + row0 + r] = f32_to_bf16_bits(total(r, m));
+      }
+    }
+    return;
   }
   if (!ok) return;
 #pragma unroll
@@ -505,21 +600,26 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   }
   constexpr int EB = kInt8 ? 1 : 2;
   CUtensorMap tw;
-  W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
+  if (!kInt8 && MT == 8)  // the tensor-core path: 64-column boxes, 128-byte swizzle
+    W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 64, 8 * RW, 128));
+  else
+    W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
   W8A8_CUDA(launch_pdl(gemv_small_kernel<kInt8, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
                        a));
   return W8A8_OK;
 }
 
-// accumulator registers a warp may hold (tokens x rows): larger products spill
+// accumulator registers a warp may hold (tokens x rows): larger products spill; the tensor-core path
+// (bf16, 8 token slots) holds 8 per n-tile of 8 rows whatever the token count
 template <bool kInt8>
 constexpr int max_slots() {
   return kInt8 ? 48 : 32;
 }
+constexpr bool slots_fit(bool int8, int MT, int RW) { return (!int8 && MT == 8) || MT * RW <= (int8 ? 48 : 32); }
 
 template <bool kInt8, int MT, int RW>
 w8a8_status launch_checked(const SmallArgs& a, cudaStream_t st) {
-  if constexpr (MT * RW <= max_slots<kInt8>()) {
+  if constexpr (slots_fit(kInt8, MT, RW)) {
     return launch_t<kInt8, MT, RW>(a, st);
   } else {
     W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "small GEMV: %d tokens x %d rows per warp not built", MT, RW);
@@ -566,16 +666,18 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
     }
   }
   if (p.RW == 0) return p;
-  if (p.MT * p.RW > (int8_weights ? max_slots<true>() : max_slots<false>())) return p;  // registers
+  if (!slots_fit(int8_weights, p.MT, p.RW)) return p;  // registers
   const int R = 8 * p.RW;
   p.P = (N + R - 1) / R;
   const int cps = p.P > sm_count ? 2 : 1;
   p.sub = int8_weights ? 512 : 256;
   p.nsub = (K + p.sub - 1) / p.sub;
   p.kpad = p.nsub * p.sub;
-  p.xbytes = p.MT * p.kpad * (int8_weights ? 1 : 2);
+  const bool mma = !int8_weights && p.MT == 8;  // the kernel's tensor-core path (same rule)
+  p.xbytes = int8_weights ? p.MT * p.kpad : p.MT * (p.kpad + (mma ? 8 : 0)) * 2;
   p.abytes = fused_norm && int8_weights ? p.MT * p.kpad * 2 : 0;
-  const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - p.abytes - 16 * 16;
+  p.rbytes = mma ? kCW * R * 8 * 4 : 0;  // the warps' partial sums
+  const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - p.abytes - p.rbytes - 16 * 16;
   // sub-slices per stage: 4 for warps with one or two rows, fewer for wider CTAs; each stage must
   // fit twice in the ring unless one stage covers everything
   for (int ks = p.RW <= 2 ? 4 : p.RW == 4 ? 2 : 1; ks >= 1; ks >>= 1) {
@@ -590,7 +692,7 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
     }
   }
   if (p.ks == 0) return p;
-  p.smem_bytes = 1024 + p.stages * p.stage_bytes + p.xbytes + p.abytes + 16 * p.stages;
+  p.smem_bytes = 1024 + p.stages * p.stage_bytes + p.xbytes + p.abytes + p.rbytes + 16 * p.stages;
   p.ok = 1;
   return p;
 }

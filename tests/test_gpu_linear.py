@@ -230,13 +230,16 @@ def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarr
 @pytest.mark.parametrize("M,N,K", [(1, 6912, 1152), (16, 6912, 1152), (5, 1152, 6912), (40, 300, 1040),
                                    (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152),
                                    (128, 6912, 1152), (70, 1152, 6912), (300, 256, 64),
+                                   (6, 1536, 1152),      # 8 token slots on the tensor cores, with a bias
+                                   (7, 200, 64),         # the same, ragged rows, one 64-column box of K
+                                   (8, 13824, 1152),     # the same, 48 rows per CTA
                                    (32, 1152, 4608),     # split-K: 18 tiles, k cut into 8 parts
                                    (200, 1152, 6912),    # split-K over two row blocks
                                    (300, 19472, 1152),   # CTA pairs on 256 x 192 tiles, ragged M and N
                                    (1024, 13824, 1152)])  # CTA pairs on 256 x 256 tiles
 def test_bf16_linear_within_tolerance(B, M, N, K):
     x32, x, w32, w, _, _ = _case(M, N, K, seed=11 + M)
-    bias = np.random.default_rng(3).standard_normal(N).astype(np.float32) if M == 32 else None
+    bias = np.random.default_rng(3).standard_normal(N).astype(np.float32) if M in (6, 32) else None
     Y = B.linear_bf16(cu(w), cu(x), bias=cu(torch.from_numpy(bias)) if bias is not None else None)
     ref = OW.bf16_linear(x32, w32, bias=bias, out="bf16")
     _bf16_close(f32_of_bf16(Y), x32, w32, ref)
