@@ -61,6 +61,24 @@ __device__ __forceinline__ float consumer_sum(float v, float* red, int warp, int
   return t;
 }
 
+__device__ __forceinline__ uint32_t f16x2_of(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+// Four signed INT8 codes (bytes 0..3 of w) as two fp16 pairs (bytes 0, 1) and (2, 3), exactly:
+// byte b + 128 is placed under the exponent bits 0x64 (the half 1024 + b + 128), then 1152 is
+// subtracted.
+__device__ __forceinline__ void i8x4_to_f16x2x2(uint32_t w, uint32_t& lo, uint32_t& hi) {
+  const uint32_t u = w ^ 0x80808080u;
+  uint32_t p0, p1;
+  asm("prmt.b32 %0, %1, %2, 0x4140;\n" : "=r"(p0) : "r"(u), "r"(0x64646464u));
+  asm("prmt.b32 %0, %1, %2, 0x4342;\n" : "=r"(p1) : "r"(u), "r"(0x64646464u));
+  const uint32_t k1152 = 0x64806480u;  // (1152, 1152) as fp16
+  asm("sub.rn.f16x2 %0, %1, %2;\n" : "=r"(lo) : "r"(p0), "r"(k1152));
+  asm("sub.rn.f16x2 %0, %1, %2;\n" : "=r"(hi) : "r"(p1), "r"(k1152));
+}
+
 __device__ __forceinline__ void ldm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];\n" : "=r"(r0), "=r"(r1) : "r"(addr));
 }
@@ -83,10 +101,17 @@ __global__ void __launch_bounds__(kThreads, 2)
   // as the A operand with token rows 8-15 zero, each 8 weight rows an n-tile), the 8 consumer warps
   // taking alternate k steps of every stage; the weights arrive as 128-byte-swizzled boxes of 64
   // columns and the activation rows are padded by 16 bytes, so the fragment loads hit distinct banks
-  constexpr bool kMma = !kInt8 && MT == 8;
+  constexpr bool kMma = MT == 8;
+  // W8A8 at 5-8 tokens: the same on INT8 codes carried as fp16 (exact): K1 writes the activation
+  // codes to shared memory as fp16, each thread widens four consecutive weight bytes (one 32-bit
+  // load from 128-byte-swizzled boxes of 128 columns) into two fp16 pairs, and the k order inside
+  // an MMA is permuted alike on both operands (thread t's pairs (2t, 2t+1) and (2t+8, 2t+9) hold
+  // k 4t .. 4t+3), which leaves the sum unchanged; the fp32 accumulators (at most 128 products per
+  // stage, exact) are folded into INT32 after every stage.
   using Acc = typename std::conditional<kInt8, int, float>::type;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ float s_red[kCW];
+  __shared__ float s_red8[MT > 4 ? MT : 1][kCW];  // eight-slot K1: per-token maxima of the warps
   __shared__ float s_sx[MT];
 
   const SmallPlan& p = a.p;
@@ -127,7 +152,10 @@ __global__ void __launch_bounds__(kThreads, 2)
       mbar_arrive_expect_tx(bar, (uint32_t)(cnt * R * kSliceBytes));
       for (int u = 0; u < cnt; ++u) {
         const uint32_t d = dst + (uint32_t)(u * R * kSliceBytes);
-        if constexpr (kInt8) {
+        if constexpr (kInt8 && kMma) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) tma_load_2d_policy(d + j * R * 128, &tmW, (u0 + u) * 512 + 128 * j, row0, bar, wpol);
+        } else if constexpr (kInt8) {
           tma_load_2d_policy(d, &tmW, (u0 + u) * 512, row0, bar, wpol);
           tma_load_2d_policy(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar, wpol);
         } else if constexpr (kMma) {
@@ -191,7 +219,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   // (thread t < K / 8 owns channels 8t .. 8t+7 of every token, as in the residual-norm kernel).
   const uint16_t* xrows = a.X;
   int xstride = a.K;
-  const int xsb = kMma ? kpad + 8 : kpad;  // elements between the bf16 activation rows in shared memory
+  // elements between the activation rows in shared memory (bf16, or the fp16 codes of the W8A8
+  // tensor-core path; INT8 codes otherwise): padded on the tensor-core paths against bank conflicts
+  const int xsb = kMma ? kpad + (kInt8 ? 16 : 8) : kpad;
   if (a.has_rn) {
     uint16_t* as = kInt8 ? reinterpret_cast<uint16_t*>(xsp + p.xbytes) : reinterpret_cast<uint16_t*>(xsp);
     for (int m = 0; m < MT; ++m) {
@@ -302,62 +332,100 @@ __global__ void __launch_bounds__(kThreads, 2)
           }
         }
       }
-    } else {  // warp w quantises token w on its own (no block-wide barrier per token)
-      for (int m = warp; m < MT; m += kCW) {
-        uint2* dst = reinterpret_cast<uint2*>(xsp + (size_t)m * kpad);
-        if (m >= a.M) {
-          for (int vi = lane; vi < nvec; vi += 32) dst[vi] = make_uint2(0u, 0u);
-          if (lane == 0) s_sx[m] = 0.0f;
-          continue;
-        }
-        const uint4* src = reinterpret_cast<const uint4*>(xrows + (size_t)m * xstride);
-        const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
-        auto smooth8 = [&](int vi, float (&xh)[8]) {
-          const uint4 w = src[vi];
-          const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
-          xh[0] = __fmul_rn(bf16_lo(w.x), d0.x);
-          xh[1] = __fmul_rn(bf16_hi(w.x), d0.y);
-          xh[2] = __fmul_rn(bf16_lo(w.y), d0.z);
-          xh[3] = __fmul_rn(bf16_hi(w.y), d0.w);
-          xh[4] = __fmul_rn(bf16_lo(w.z), d1.x);
-          xh[5] = __fmul_rn(bf16_hi(w.z), d1.y);
-          xh[6] = __fmul_rn(bf16_lo(w.w), d1.z);
-          xh[7] = __fmul_rn(bf16_hi(w.w), d1.w);
-        };
-        float amax = 0.0f;
-        for (int vi = lane; vi < nvec; vi += 32) {
-          float xh[8];
-          smooth8(vi, xh);
+    } else {  // eight token slots: the whole block on all tokens at once, two passes over the rows
+      // pass 1: thread t smooths vectors t, t + 256, ... of every token (eight loads in flight) and
+      // keeps each token's running max |x_hat|; one block reduction gives m_t for all tokens
+      const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
+      auto smooth8 = [&](const uint4& w, const float4& d0, const float4& d1, float (&xh)[8]) {
+        xh[0] = __fmul_rn(bf16_lo(w.x), d0.x);
+        xh[1] = __fmul_rn(bf16_hi(w.x), d0.y);
+        xh[2] = __fmul_rn(bf16_lo(w.y), d0.z);
+        xh[3] = __fmul_rn(bf16_hi(w.y), d0.w);
+        xh[4] = __fmul_rn(bf16_lo(w.z), d1.x);
+        xh[5] = __fmul_rn(bf16_hi(w.z), d1.y);
+        xh[6] = __fmul_rn(bf16_lo(w.w), d1.z);
+        xh[7] = __fmul_rn(bf16_hi(w.w), d1.w);
+      };
+      auto load_tokens = [&](int vi, uint4 (&w)[MT]) {
 #pragma unroll
-          for (int e = 0; e < 8; ++e) amax = fmaxf(amax, fabsf(xh[e]));
-        }
-        const float mx = warp_max(amax);
-        const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
-        if (lane == 0) {
-          const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127)
-          s_sx[m] = sx;
-          if (a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
-        }
-        for (int vi = lane; vi < nvec; vi += 32) {  // second pass: the row again (L1 / L2)
+        for (int m = 0; m < MT; ++m)
+          w[m] = m < a.M ? reinterpret_cast<const uint4*>(xrows + (size_t)m * xstride)[vi] : make_uint4(0u, 0u, 0u, 0u);
+      };
+      float am[MT];
+#pragma unroll
+      for (int m = 0; m < MT; ++m) am[m] = 0.0f;
+      for (int vi = tid; vi < nvec; vi += kCW * 32) {
+        uint4 w[MT];
+        load_tokens(vi, w);
+        const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
           float xh[8];
-          smooth8(vi, xh);
+          smooth8(w[m], d0, d1, xh);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) am[m] = fmaxf(am[m], fabsf(xh[e]));
+        }
+      }
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        const float v = warp_max(am[m]);
+        if (lane == 0) s_red8[m][warp] = v;
+      }
+      named_bar_sync(1, kCW * 32);
+      float rr[MT];
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        float mx = 0.0f;
+#pragma unroll
+        for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red8[m][i]);
+        rr[m] = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
+        if (tid == m) {
+          const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127); 0 for slots >= M
+          s_sx[m] = sx;
+          if (m < a.M && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
+        }
+      }
+      // pass 2: the rows again (L1), quantised; codes of slots >= M are zeros
+      for (int vi = tid; vi < nvec; vi += kCW * 32) {
+        uint4 w[MT];
+        load_tokens(vi, w);
+        const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+          float xh[8];
+          smooth8(w[m], d0, d1, xh);
           int q[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[e], r))));
-          uint2 packed;
-          packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
-                     ((uint32_t)(q[3] & 0xff) << 24);
-          packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
-                     ((uint32_t)(q[7] & 0xff) << 24);
-          dst[vi] = packed;
-          if (a.xq_dbg && blockIdx.x == 0) reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] = packed;
+          for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[e], rr[m]))));
+          if constexpr (kMma) {
+            reinterpret_cast<uint4*>(xsp + (size_t)m * xsb * 2)[vi] =
+                make_uint4(f16x2_of((float)q[0], (float)q[1]), f16x2_of((float)q[2], (float)q[3]),
+                           f16x2_of((float)q[4], (float)q[5]), f16x2_of((float)q[6], (float)q[7]));
+          }
+          if (!kMma || (a.xq_dbg && blockIdx.x == 0 && m < a.M)) {
+            uint2 packed;
+            packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                       ((uint32_t)(q[3] & 0xff) << 24);
+            packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                       ((uint32_t)(q[7] & 0xff) << 24);
+            if (!kMma) reinterpret_cast<uint2*>(xsp + (size_t)m * kpad)[vi] = packed;
+            if (a.xq_dbg && blockIdx.x == 0 && m < a.M) reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] = packed;
+          }
         }
       }
     }
-    const int tail16 = (kpad - a.K) >> 4;
-    for (int i = tid; i < MT * tail16; i += kCW * 32) {
-      const int m = i / tail16, c = i - m * tail16;
-      *reinterpret_cast<uint4*>(xsp + (size_t)m * kpad + a.K + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
+    if constexpr (kMma) {  // fp16 codes: zeros from K to the padded length
+      const int t8 = (kpad - a.K) >> 3;
+      for (int i = tid; i < MT * t8; i += kCW * 32) {
+        const int m = i / t8, c = i - m * t8;
+        *reinterpret_cast<uint4*>(xsp + ((size_t)m * xsb + a.K + 8 * c) * 2) = make_uint4(0u, 0u, 0u, 0u);
+      }
+    } else {  // INT8 codes: zeros from K to the padded length
+      const int tail16 = (kpad - a.K) >> 4;
+      for (int i = tid; i < MT * tail16; i += kCW * 32) {
+        const int m = i / tail16, c = i - m * tail16;
+        *reinterpret_cast<uint4*>(xsp + (size_t)m * kpad + a.K + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
+      }
     }
   } else if (!a.has_rn) {
     const int vpr = kpad >> 3;  // 16-byte vectors per slot
@@ -392,6 +460,9 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
       for (int m = 0; m < MT; ++m) acc[c][i][m] = 0;
   float mc[2][RW][4];  // MMA path: two accumulator sets (alternate k steps), per n-tile of 8 rows
+  int mi32[RW][2];     // W8A8 MMA path: the folded INT32 sums (token g, rows 8 i + 2 t and + 1)
+#pragma unroll
+  for (int i = 0; i < RW; ++i) mi32[i][0] = mi32[i][1] = 0;
 #pragma unroll
   for (int c = 0; c < 2; ++c)
 #pragma unroll
@@ -417,6 +488,38 @@ __global__ void __launch_bounds__(kThreads, 2)
       const uint32_t sb = ring + (uint32_t)(s * SB);
       const int u0 = it * KS, cnt = min(KS, nsub - u0);
       const int xr = lane & 7, xh = (lane >> 3) & 1;  // ldmatrix row addresses: token / half
+      if constexpr (kInt8) {
+        // k steps of 16 of this stage: step q is sub-slice q / 32, 128-column box (q % 32) / 8,
+        // 16-byte chunk q % 8 of its rows; thread (g, t) reads bytes 4 t .. 4 t + 3 of row g's chunk
+        // and of token g's codes
+        const int g = lane >> 2, t = lane & 3;
+        auto step8 = [&](int q, float (&c)[RW][4]) {
+          const int u = q >> 5, kk = q & 31, ch = kk & 7;
+          const uint32_t box = sb + (uint32_t)(u * R * kSliceBytes + (kk >> 3) * R * 128);
+          const int kg = (u0 + u) * 512 + 16 * kk;
+          uint32_t a0, a2;
+          asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];\n" : "=r"(a0), "=r"(a2) : "r"(xs + (uint32_t)((g * xsb + kg + 4 * t) * 2)));
+#pragma unroll
+          for (int i = 0; i < RW; ++i) {
+            uint32_t wb;
+            asm volatile("ld.shared.u32 %0, [%1];\n" : "=r"(wb) : "r"(box + (uint32_t)((8 * i + g) * 128 + ((ch ^ g) << 4) + 4 * t)));
+            uint32_t b0, b1;
+            i8x4_to_f16x2x2(wb, b0, b1);
+            mma_f16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
+          }
+        };
+        for (int q = warp; q < 32 * cnt; q += 2 * kCW) {
+          step8(q, mc[0]);
+          if (q + kCW < 32 * cnt) step8(q + kCW, mc[1]);
+        }
+#pragma unroll
+        for (int i = 0; i < RW; ++i) {  // fold: each set took at most 128 products per output this stage
+          mi32[i][0] += __float2int_rn(mc[0][i][0]) + __float2int_rn(mc[1][i][0]);
+          mi32[i][1] += __float2int_rn(mc[0][i][1]) + __float2int_rn(mc[1][i][1]);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) mc[0][i][e] = mc[1][i][e] = 0.0f;
+        }
+      } else {
       auto step = [&](int q, float (&c)[RW][4]) {
         const int u = q >> 4, kk = q & 15, c0 = 2 * (kk & 3);
         const uint32_t box = sb + (uint32_t)(u * R * kSliceBytes + (kk >> 2) * R * 128);
@@ -442,6 +545,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int q = warp; q < 16 * cnt; q += 2 * kCW) {  // alternate steps feed the two accumulator sets
         step(q, mc[0]);
         if (q + kCW < 16 * cnt) step(q + kCW, mc[1]);
+      }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(empty + s));
@@ -499,22 +603,35 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   if constexpr (kMma) {
     // Each warp's sums (accumulator c0 / c1 of n-tile i: token g, rows 8 i + 2 t and + 1) go to
-    // shared memory [warp][row][token]; then every output sums the 8 warps in warp order.
-    float* part = reinterpret_cast<float*>(xsp + p.xbytes + p.abytes);
+    // shared memory [warp][row][token]; then every output sums the 8 warps in warp order (W8A8:
+    // INT32, exact, then dequantised as fl(fl(s_x s_w) acc)).
+    Acc* part = reinterpret_cast<Acc*>(xsp + p.xbytes + p.abytes);
     const int g = lane >> 2, t = lane & 3;
     if (ok) {
 #pragma unroll
       for (int i = 0; i < RW; ++i) {
-        part[(warp * R + 8 * i + 2 * t) * 8 + g] = mc[0][i][0] + mc[1][i][0];
-        part[(warp * R + 8 * i + 2 * t + 1) * 8 + g] = mc[0][i][1] + mc[1][i][1];
+        if constexpr (kInt8) {
+          part[(warp * R + 8 * i + 2 * t) * 8 + g] = mi32[i][0];
+          part[(warp * R + 8 * i + 2 * t + 1) * 8 + g] = mi32[i][1];
+        } else {
+          part[(warp * R + 8 * i + 2 * t) * 8 + g] = mc[0][i][0] + mc[1][i][0];
+          part[(warp * R + 8 * i + 2 * t + 1) * 8 + g] = mc[0][i][1] + mc[1][i][1];
+        }
       }
     }
     if (!named_bar_all(1, kCW * 32, ok)) return;
     auto total = [&](int r, int m) {
-      float v = 0.0f;
+      Acc v = 0;
 #pragma unroll
       for (int w = 0; w < kCW; ++w) v += part[(w * R + r) * 8 + m];
-      return a.bias ? __fadd_rn(v, a.bias[row0 + r]) : v;
+      float y;
+      if constexpr (kInt8) {
+        y = __fmul_rn(__fmul_rn(s_sx[m], a.s_w[row0 + r]), __int2float_rn(v));
+        if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row0 + r] = v;
+      } else {
+        y = v;
+      }
+      return a.bias ? __fadd_rn(y, a.bias[row0 + r]) : y;
     };
     if (a.kind == EPI_GEGLU) {  // pair b of block j: gate row 16 j + b, up row 16 j + 8 + b
       for (int e = tid; e < (R / 2) * 8; e += kCW * 32) {
@@ -600,8 +717,8 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   }
   constexpr int EB = kInt8 ? 1 : 2;
   CUtensorMap tw;
-  if (!kInt8 && MT == 8)  // the tensor-core path: 64-column boxes, 128-byte swizzle
-    W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 64, 8 * RW, 128));
+  if (MT == 8)  // the tensor-core paths: 128-byte boxes (64 bf16 or 128 INT8 columns), 128-byte swizzle
+    W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 8 * RW, 128));
   else
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
   W8A8_CUDA(launch_pdl(gemv_small_kernel<kInt8, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
@@ -609,13 +726,13 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   return W8A8_OK;
 }
 
-// accumulator registers a warp may hold (tokens x rows): larger products spill; the tensor-core path
-// (bf16, 8 token slots) holds 8 per n-tile of 8 rows whatever the token count
+// accumulator registers a warp may hold (tokens x rows): larger products spill; the tensor-core paths
+// (8 token slots) hold 8 (+ 2 INT32) per n-tile of 8 rows whatever the token count
 template <bool kInt8>
 constexpr int max_slots() {
   return kInt8 ? 48 : 32;
 }
-constexpr bool slots_fit(bool int8, int MT, int RW) { return (!int8 && MT == 8) || MT * RW <= (int8 ? 48 : 32); }
+constexpr bool slots_fit(bool int8, int MT, int RW) { return MT == 8 || MT * RW <= (int8 ? 48 : 32); }
 
 template <bool kInt8, int MT, int RW>
 w8a8_status launch_checked(const SmallArgs& a, cudaStream_t st) {
@@ -673,8 +790,8 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
   p.sub = int8_weights ? 512 : 256;
   p.nsub = (K + p.sub - 1) / p.sub;
   p.kpad = p.nsub * p.sub;
-  const bool mma = !int8_weights && p.MT == 8;  // the kernel's tensor-core path (same rule)
-  p.xbytes = int8_weights ? p.MT * p.kpad : p.MT * (p.kpad + (mma ? 8 : 0)) * 2;
+  const bool mma = p.MT == 8;  // the kernel's tensor-core paths (same rule): padded bf16 / fp16 rows
+  p.xbytes = mma ? p.MT * (p.kpad + (int8_weights ? 16 : 8)) * 2 : p.MT * p.kpad * (int8_weights ? 1 : 2);
   p.abytes = fused_norm && int8_weights ? p.MT * p.kpad * 2 : 0;
   p.rbytes = mma ? kCW * R * 8 * 4 : 0;  // the warps' partial sums
   const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - p.abytes - p.rbytes - 16 * 16;

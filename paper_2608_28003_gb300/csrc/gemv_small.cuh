@@ -21,7 +21,7 @@ struct SmallPlan {
   int stage_bytes;  // ks x R rows x 512 bytes
   int xbytes;       // activations in shared memory: MT x kpad bf16 or INT8 codes
   int abytes;       // W8A8 with a fused residual norm: the bf16 rows it produces, before K1
-  int rbytes;       // bf16 at 5-8 tokens (tensor-core path): the consumer warps' partial sums
+  int rbytes;       // 5-8 tokens (tensor-core paths): the consumer warps' partial sums
   int smem_bytes;
 };
 
