@@ -612,7 +612,9 @@ def run_ours(args, dist: Dist):
 def mask_sweep(B, dec, dev):
     """The library's allocator over the 16 candidate masks: Top-1 agreement and perplexity change
     against the all-bf16 decoder on 4 x 128 eval tokens (stream seed 2), decode ms/token at
-    batch 1 after a 128-token prefill (median of 3 runs of 64 greedy steps)."""
+    batch 1 after a 128-token prefill (median of 3 runs of 64 greedy steps); then the
+    per-sublayer allocator (single-sublayer masks timed over 3 runs of 32 steps, greedy additions
+    under the same budget)."""
     import torch
     import synth
     names, cands = zip(*B.candidate_masks())
@@ -627,8 +629,20 @@ def mask_sweep(B, dec, dev):
                      "speedup_vs_bf16": round(base / t, 4), "top1": round(rep["top1"][i], 5),
                      "ppl_delta": round(rep["ppl_delta"][i], 5), "weight_gb": round(decode_weight_bytes(f, a, l) / 1e9, 4)})
     ch = rep["chosen"]
-    return {"rows": rows, "chosen": names[ch] if ch >= 0 else None, "rule": "Top-1 >= 0.989, ppl change <= 0.01",
-            "seconds": round(time.time() - t0, 1)}
+    out = {"rows": rows, "chosen": names[ch] if ch >= 0 else None, "rule": "Top-1 >= 0.989, ppl change <= 0.01",
+           "seconds": round(time.time() - t0, 1)}
+    # below the groups: the per-sublayer allocator on the same stream and budget
+    t0 = time.time()
+    lr = dec.allocate_layers(ev, decode_B=1, prefill_T=PREFILL, decode_steps=32, reps=3)
+    f, a, l = lr["chosen"]
+    out["per_sublayer"] = {
+        "ffn_layers": [i for i in range(LAYERS) if f >> i & 1], "attn_layers": [i for i in range(LAYERS) if a >> i & 1],
+        "lm_head": bool(l), "ranked": len(lr["order"]), "accepted": lr["n_accepted"],
+        "bf16_ms_per_token": round(lr["base_ms"], 5), "ms_per_token": round(lr["chosen_ms"], 5),
+        "speedup_vs_bf16": round(lr["base_ms"] / lr["chosen_ms"], 4), "top1": round(lr["chosen_top1"], 5),
+        "ppl_delta": round(lr["chosen_ppl_delta"], 5), "weight_gb": round(decode_weight_bytes(f, a, l) / 1e9, 4),
+        "seconds": round(time.time() - t0, 1)}
+    return out
 
 
 def batch_table(B, dec, dev):

@@ -364,6 +364,47 @@ typedef struct {
  * (the all-bf16 mask if none is feasible).  Synchronous; requires w8a8_model_prepare. */
 w8a8_status w8a8_allocate_mask(w8a8_model* m, const w8a8_alloc_opts* opts, w8a8_alloc_report* report, void* stream);
 
+/* Allocation per sublayer, below the groups of the Combined Configurations (the finer granularity
+ * the paper's title names; its own search stops at groups).  Sublayer i: 0 .. L-1 the FFN of
+ * layer i, L .. 2L-1 the attention projections of layer i - L, 2L the lm_head.
+ *
+ * The ranking rule (host code, exported for tests): the sublayers with a positive latency gain
+ * whose single-sublayer mask meets the budget by itself, in descending order of
+ * gain / (cost + 1e-3), where cost = max(0, 1 - top1) / max(1e-6, 1 - min_top1)
+ *                                  + max(0, ppl_delta) / max(1e-6, max_ppl_delta)
+ * (evaluated in double precision); ties go to the lower index.  Host arrays of length n; writes the
+ * ranked indices to order (length n) and returns how many there are. */
+int w8a8_greedy_order(const float* gain_ms, const float* top1, const float* ppl_delta, int n, float min_top1,
+                      float max_ppl_delta, int32_t* order);
+
+typedef struct {
+  const int32_t* eval_tokens;  /* device [eval_B, eval_T]: teacher-forced evaluation stream */
+  int32_t eval_B, eval_T;
+  int32_t decode_B, prefill_T, decode_steps, reps;  /* latency, as in w8a8_alloc_opts */
+  float min_top1, max_ppl_delta;
+} w8a8_layer_alloc_opts;
+
+typedef struct {
+  w8a8_mask chosen;        /* the accepted sublayers (all-bf16 if none) */
+  float base_ms;           /* decode ms per step of the all-bf16 mask */
+  float chosen_ms;         /* ... and of the chosen mask */
+  float chosen_top1, chosen_ppl_delta;
+  float* gain_ms;          /* host [2L + 1]: base_ms - ms of each single-sublayer mask */
+  float* top1;             /* host [2L + 1]: Top-1 agreement of each single-sublayer mask */
+  float* ppl_delta;        /* host [2L + 1]: its perplexity change */
+  int32_t* order;          /* host [2L + 1]: the ranked sublayers, n_order of them */
+  int32_t n_order;
+  int32_t n_accepted;      /* how many of them the chosen mask holds */
+} w8a8_layer_alloc_report;
+
+/* The per-sublayer allocator: measures every single-sublayer mask (quality and latency, as
+ * w8a8_allocate_mask does), ranks the sublayers with w8a8_greedy_order, then adds them one at a
+ * time in that order, keeping each one only if the cumulative mask still meets the budget (its
+ * quality measured again); finally times the chosen mask and leaves it set.  Synchronous; requires
+ * w8a8_model_prepare and at most 32 layers. */
+w8a8_status w8a8_allocate_layers(w8a8_model* m, const w8a8_layer_alloc_opts* opts, w8a8_layer_alloc_report* report,
+                                 void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -85,6 +85,20 @@ class AllocReportC(ctypes.Structure):
                 ("top1", ctypes.POINTER(ctypes.c_float)), ("ppl_delta", ctypes.POINTER(ctypes.c_float))]
 
 
+class LayerAllocOptsC(ctypes.Structure):
+    _fields_ = [("eval_tokens", _vp), ("eval_B", ctypes.c_int32), ("eval_T", ctypes.c_int32),
+                ("decode_B", ctypes.c_int32), ("prefill_T", ctypes.c_int32), ("decode_steps", ctypes.c_int32),
+                ("reps", ctypes.c_int32), ("min_top1", ctypes.c_float), ("max_ppl_delta", ctypes.c_float)]
+
+
+class LayerAllocReportC(ctypes.Structure):
+    _fields_ = [("chosen", MaskC), ("base_ms", ctypes.c_float), ("chosen_ms", ctypes.c_float),
+                ("chosen_top1", ctypes.c_float), ("chosen_ppl_delta", ctypes.c_float),
+                ("gain_ms", ctypes.POINTER(ctypes.c_float)), ("top1", ctypes.POINTER(ctypes.c_float)),
+                ("ppl_delta", ctypes.POINTER(ctypes.c_float)), ("order", ctypes.POINTER(ctypes.c_int32)),
+                ("n_order", ctypes.c_int32), ("n_accepted", ctypes.c_int32)]
+
+
 _fp = ctypes.POINTER(ctypes.c_float)
 
 # name -> (restype, argtypes)
@@ -128,6 +142,8 @@ SIGNATURES = {
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
     "w8a8_allocate_mask": (_i32, [_vp, ctypes.POINTER(AllocOptsC), ctypes.POINTER(AllocReportC), _vp]),
+    "w8a8_greedy_order": (_i32, [_fp, _fp, _fp, _i32, _f32, _f32, ctypes.POINTER(ctypes.c_int32)]),
+    "w8a8_allocate_layers": (_i32, [_vp, ctypes.POINTER(LayerAllocOptsC), ctypes.POINTER(LayerAllocReportC), _vp]),
 }
 
 _LIB = None
@@ -428,6 +444,16 @@ def candidate_masks():
     return out
 
 
+def greedy_order(gain_ms, top1, ppl_delta, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> list:
+    """The library's per-sublayer ranking rule on host arrays: the ranked sublayer indices."""
+    n = len(gain_ms)
+    arr = lambda v, t: (t * n)(*v)  # noqa: E731
+    order = (ctypes.c_int32 * max(n, 1))()
+    k = lib().w8a8_greedy_order(arr(gain_ms, ctypes.c_float), arr(top1, ctypes.c_float),
+                                arr(ppl_delta, ctypes.c_float), n, float(min_top1), float(max_ppl_delta), order)
+    return list(order[:k])
+
+
 def choose_mask(latency, top1, ppl_delta, n_int8, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> int:
     """The library's allocation rule on host arrays (index, or -1 if nothing is feasible)."""
     n = len(latency)
@@ -576,6 +602,25 @@ class Decoder:
         _check("w8a8_allocate_mask", lib().w8a8_allocate_mask(self.h, ctypes.byref(opts), ctypes.byref(rep),
                                                               _stream(stream)))
         return {"chosen": rep.chosen, "latency_ms": list(lat), "top1": list(t1), "ppl_delta": list(pd)}
+
+    def allocate_layers(self, eval_tokens: torch.Tensor, decode_B: int, prefill_T: int, decode_steps: int,
+                        reps: int = 3, min_top1: float = 0.989, max_ppl_delta: float = 0.01, stream=None) -> dict:
+        """Run the per-sublayer allocator (sublayer i: FFN of layer i for i < L, attention of layer
+        i - L for i < 2L, lm_head for i = 2L); leaves the chosen mask set."""
+        n = 2 * self.cfg.layers + 1
+        eB, eT = eval_tokens.shape
+        opts = LayerAllocOptsC(_bits(eval_tokens).data_ptr(), eB, eT, decode_B, prefill_T, decode_steps, reps,
+                               float(min_top1), float(max_ppl_delta))
+        gain, t1, pd = (ctypes.c_float * n)(), (ctypes.c_float * n)(), (ctypes.c_float * n)()
+        order = (ctypes.c_int32 * n)()
+        rep = LayerAllocReportC(MaskC(0, 0, 0), 0.0, 0.0, 0.0, 0.0, gain, t1, pd, order, 0, 0)
+        _check("w8a8_allocate_layers", lib().w8a8_allocate_layers(self.h, ctypes.byref(opts), ctypes.byref(rep),
+                                                                  _stream(stream)))
+        c = rep.chosen
+        return {"chosen": (c.ffn_bits, c.attn_bits, c.lm), "base_ms": rep.base_ms, "chosen_ms": rep.chosen_ms,
+                "chosen_top1": rep.chosen_top1, "chosen_ppl_delta": rep.chosen_ppl_delta, "gain_ms": list(gain),
+                "top1": list(t1), "ppl_delta": list(pd), "order": list(order[:rep.n_order]),
+                "n_accepted": rep.n_accepted}
 
 
 def token_nll(logits: torch.Tensor, targets: torch.Tensor, stream=None) -> torch.Tensor:

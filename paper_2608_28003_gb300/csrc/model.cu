@@ -686,128 +686,158 @@ extern "C" int w8a8_choose_mask(const float* latency, const float* top1, const f
   return best;
 }
 
-extern "C" w8a8_status w8a8_allocate_mask(w8a8_model* m, const w8a8_alloc_opts* o, w8a8_alloc_report* rep,
-                                          void* stream) {
-  W8A8_CHECK_ARG(m && o && rep && o->candidates && o->n_candidates > 0 && o->eval_tokens && rep->latency_ms &&
-                     rep->top1 && rep->ppl_delta,
-                 W8A8_ERR_INVALID_ARG, "w8a8_allocate_mask: null argument");
-  W8A8_CHECK_ARG(m->prepared, W8A8_ERR_INVALID_ARG, "w8a8_allocate_mask: w8a8_model_prepare first");
-  W8A8_TRY(check_call(m, o->eval_B, o->eval_T, 0));
-  W8A8_CHECK_ARG(o->decode_B > 0 && o->decode_B <= m->cfg.max_batch && o->prefill_T > 0, W8A8_ERR_SHAPE,
-                 "w8a8_allocate_mask: decode_B %d / prefill_T %d", o->decode_B, o->prefill_T);
-  W8A8_TRY(check_call(m, o->decode_B, 1, o->prefill_T + o->decode_steps - 1));
-  W8A8_CHECK_ARG(o->eval_T >= 2 && o->decode_steps > 0 && o->reps > 0, W8A8_ERR_INVALID_ARG,
-                 "w8a8_allocate_mask: eval_T >= 2, decode_steps > 0, reps > 0");
-  cudaStream_t st = as_stream(stream);
-  const int V = m->cfg.vocab, Me = o->eval_B * o->eval_T, Mp = o->decode_B * o->prefill_T;
-  // offline sweep: temporary buffers
+namespace {
+
+// The measurements both allocators make (Problem Statement; Combined Configurations): a mask's
+// quality against the all-bf16 decoder on a teacher-forced evaluation stream (Top-1 agreement over
+// the positions with a next token, and the perplexity ratio minus one), and its decode latency
+// (median over reps of the mean ms per step of decode_steps CUDA-graph steps after a prefill).
+// Buffers live from init() to the destructor; the model's mask is whatever was set last.
+struct AllocRun {
+  w8a8_model* m;
+  const int32_t* eval_tokens;
+  int eval_B, eval_T, decode_B, prefill_T, decode_steps, reps;
+  void* stream;
+  cudaStream_t st;
+  int V = 0, Me = 0, Mp = 0;
   float *logits = nullptr, *nll = nullptr;
   int32_t *targets = nullptr, *top_ref = nullptr, *top_c = nullptr, *ptok = nullptr, *dtok = nullptr;
   std::vector<void*> tmp;
-  auto talloc = [&](void** p, size_t bytes) -> w8a8_status {
+  std::vector<float> nll_h;
+  std::vector<int32_t> top_h, ref_h;
+  double ref_nll = 0.0;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+
+  ~AllocRun() {
+    cudaStreamSynchronize(st);
+    for (void* p : tmp) cudaFree(p);
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+  }
+  w8a8_status talloc(void** p, size_t bytes) {
     W8A8_CUDA(cudaMalloc(p, std::max<size_t>(bytes, 16)));
     tmp.push_back(*p);
     return W8A8_OK;
-  };
-  auto cleanup = [&]() {
-    cudaStreamSynchronize(st);
-    for (void* p : tmp) cudaFree(p);
-  };
-  w8a8_status status = W8A8_OK;
-  do {
-    if ((status = talloc((void**)&logits, (size_t)Me * V * 4)) != W8A8_OK) break;
-    if ((status = talloc((void**)&nll, (size_t)Me * 4)) != W8A8_OK) break;
-    if ((status = talloc((void**)&targets, (size_t)Me * 4)) != W8A8_OK) break;
-    if ((status = talloc((void**)&top_ref, (size_t)Me * 4)) != W8A8_OK) break;
-    if ((status = talloc((void**)&top_c, (size_t)std::max(Me, m->cfg.max_tokens) * 4)) != W8A8_OK) break;
-    if ((status = talloc((void**)&ptok, (size_t)Mp * 4)) != W8A8_OK) break;
-    if ((status = talloc((void**)&dtok, (size_t)o->decode_B * 4)) != W8A8_OK) break;
-  } while (0);
-  if (status != W8A8_OK) {
-    cleanup();
-    return status;
   }
-  shift_targets_kernel<<<(Me + 255) / 256, 256, 0, st>>>(o->eval_tokens, o->eval_B, o->eval_T, targets);
-  fill_tokens_kernel<<<(Mp + 255) / 256, 256, 0, st>>>(ptok, Mp, V);
-  std::vector<float> nll_h(Me);
-  std::vector<int32_t> top_h(Me), ref_h(Me);
-  auto mean_nll = [&](const std::vector<float>& v) {
-    double s = 0.0;
+  double mean_nll() const {
+    double sum = 0.0;
     int n = 0;
-    for (int b = 0; b < o->eval_B; ++b)
-      for (int t = 0; t + 1 < o->eval_T; ++t, ++n) s += v[b * o->eval_T + t];
-    return s / n;
-  };
-  auto evaluate = [&](int32_t* top_out, double* mnll) -> w8a8_status {
-    W8A8_TRY(w8a8_decoder_forward(m, o->eval_tokens, o->eval_B, o->eval_T, 0, logits, top_out, stream));
+    for (int b = 0; b < eval_B; ++b)
+      for (int t = 0; t + 1 < eval_T; ++t, ++n) sum += nll_h[b * eval_T + t];
+    return sum / n;
+  }
+  w8a8_status forward_eval(int32_t* top_out, double* mnll) {
+    W8A8_TRY(w8a8_decoder_forward(m, eval_tokens, eval_B, eval_T, 0, logits, top_out, stream));
     W8A8_TRY(w8a8_token_nll(logits, targets, Me, V, nll, stream));
     W8A8_CUDA(cudaMemcpyAsync(nll_h.data(), nll, (size_t)Me * 4, cudaMemcpyDeviceToHost, st));
     W8A8_CUDA(cudaStreamSynchronize(st));
-    *mnll = mean_nll(nll_h);
+    *mnll = mean_nll();
     return W8A8_OK;
-  };
+  }
+  // buffers, the shifted targets, the prefill tokens and the all-bf16 reference (sets that mask)
+  w8a8_status init() {
+    st = as_stream(stream);
+    V = m->cfg.vocab;
+    Me = eval_B * eval_T;
+    Mp = decode_B * prefill_T;
+    W8A8_TRY(talloc((void**)&logits, (size_t)Me * V * 4));
+    W8A8_TRY(talloc((void**)&nll, (size_t)Me * 4));
+    W8A8_TRY(talloc((void**)&targets, (size_t)Me * 4));
+    W8A8_TRY(talloc((void**)&top_ref, (size_t)Me * 4));
+    W8A8_TRY(talloc((void**)&top_c, (size_t)std::max(Me, m->cfg.max_tokens) * 4));
+    W8A8_TRY(talloc((void**)&ptok, (size_t)Mp * 4));
+    W8A8_TRY(talloc((void**)&dtok, (size_t)decode_B * 4));
+    W8A8_CUDA(cudaEventCreate(&e0));
+    W8A8_CUDA(cudaEventCreate(&e1));
+    nll_h.resize(Me);
+    top_h.resize(Me);
+    ref_h.resize(Me);
+    shift_targets_kernel<<<(Me + 255) / 256, 256, 0, st>>>(eval_tokens, eval_B, eval_T, targets);
+    W8A8_LAUNCH_CHECK();
+    fill_tokens_kernel<<<(Mp + 255) / 256, 256, 0, st>>>(ptok, Mp, V);
+    W8A8_LAUNCH_CHECK();
+    W8A8_TRY(w8a8_set_mask(m, 0, 0, 0));
+    W8A8_TRY(forward_eval(top_ref, &ref_nll));
+    W8A8_CUDA(cudaMemcpy(ref_h.data(), top_ref, (size_t)Me * 4, cudaMemcpyDeviceToHost));
+    return W8A8_OK;
+  }
+  w8a8_status quality(const w8a8_mask& c, float* top1, float* ppl_delta) {
+    W8A8_TRY(w8a8_set_mask(m, c.ffn_bits, c.attn_bits, c.lm));
+    double cn = 0.0;
+    W8A8_TRY(forward_eval(top_c, &cn));
+    W8A8_CUDA(cudaMemcpy(top_h.data(), top_c, (size_t)Me * 4, cudaMemcpyDeviceToHost));
+    int agree = 0, cnt = 0;
+    for (int b = 0; b < eval_B; ++b)
+      for (int t = 0; t + 1 < eval_T; ++t, ++cnt) agree += top_h[b * eval_T + t] == ref_h[b * eval_T + t];
+    *top1 = (float)agree / (float)cnt;
+    *ppl_delta = (float)(std::exp(cn) / std::exp(ref_nll) - 1.0);
+    return W8A8_OK;
+  }
+  // prefill, then decode steps from CUDA graphs fed by their own top-1 (greedy)
+  w8a8_status latency(const w8a8_mask& c, float* ms_per_step) {
+    W8A8_TRY(w8a8_set_mask(m, c.ffn_bits, c.attn_bits, c.lm));
+    std::vector<float> runs;
+    for (int r = 0; r < reps; ++r) {
+      // prefill in chunks of at most max_tokens rows (the KV cache carries the earlier chunks)
+      const int chunk = std::max(1, m->cfg.max_tokens / decode_B);
+      for (int t0 = 0; t0 < prefill_T; t0 += chunk) {
+        const int tl = std::min(chunk, prefill_T - t0);
+        W8A8_TRY(w8a8_decoder_forward(m, ptok + (size_t)decode_B * t0, decode_B, tl, t0, nullptr, top_c, stream));
+      }
+      W8A8_CUDA(cudaMemcpyAsync(dtok, top_c, 4 * (size_t)decode_B, cudaMemcpyDeviceToDevice, st));
+      // warm the graph of this mask outside the timed region
+      W8A8_TRY(w8a8_decoder_decode_step(m, dtok, decode_B, prefill_T, nullptr, dtok, stream));
+      W8A8_CUDA(cudaEventRecord(e0, st));
+      for (int s = 0; s < decode_steps; ++s)
+        W8A8_TRY(w8a8_decoder_decode_step(m, dtok, decode_B, prefill_T + s, nullptr, dtok, stream));
+      W8A8_CUDA(cudaEventRecord(e1, st));
+      W8A8_CUDA(cudaEventSynchronize(e1));
+      float ms = 0.0f;
+      W8A8_CUDA(cudaEventElapsedTime(&ms, e0, e1));
+      runs.push_back(ms / (float)decode_steps);
+    }
+    std::sort(runs.begin(), runs.end());
+    *ms_per_step = runs[runs.size() / 2];
+    return W8A8_OK;
+  }
+};
+
+w8a8_status check_alloc_args(w8a8_model* m, const int32_t* eval_tokens, int eval_B, int eval_T, int decode_B,
+                             int prefill_T, int decode_steps, int reps, const char* who) {
+  W8A8_CHECK_ARG(m && eval_tokens, W8A8_ERR_INVALID_ARG, "%s: null argument", who);
+  W8A8_CHECK_ARG(m->prepared, W8A8_ERR_INVALID_ARG, "%s: w8a8_model_prepare first", who);
+  W8A8_TRY(check_call(m, eval_B, eval_T, 0));
+  W8A8_CHECK_ARG(decode_B > 0 && decode_B <= m->cfg.max_batch && prefill_T > 0, W8A8_ERR_SHAPE,
+                 "%s: decode_B %d / prefill_T %d", who, decode_B, prefill_T);
+  W8A8_TRY(check_call(m, decode_B, 1, prefill_T + decode_steps - 1));
+  W8A8_CHECK_ARG(eval_T >= 2 && decode_steps > 0 && reps > 0, W8A8_ERR_INVALID_ARG,
+                 "%s: eval_T >= 2, decode_steps > 0, reps > 0", who);
+  return W8A8_OK;
+}
+
+}  // namespace
+
+extern "C" w8a8_status w8a8_allocate_mask(w8a8_model* m, const w8a8_alloc_opts* o, w8a8_alloc_report* rep,
+                                          void* stream) {
+  W8A8_CHECK_ARG(m && o && rep && o->candidates && o->n_candidates > 0 && rep->latency_ms && rep->top1 &&
+                     rep->ppl_delta,
+                 W8A8_ERR_INVALID_ARG, "w8a8_allocate_mask: null argument");
+  W8A8_TRY(check_alloc_args(m, o->eval_tokens, o->eval_B, o->eval_T, o->decode_B, o->prefill_T, o->decode_steps,
+                            o->reps, "w8a8_allocate_mask"));
   const uint32_t saved_ffn = m->ffn_bits, saved_attn = m->attn_bits;
   const int saved_lm = m->lm;
-  double ref_nll = 0.0;
-  m->ffn_bits = m->attn_bits = 0;
-  m->lm = 0;
-  status = evaluate(top_ref, &ref_nll);
-  if (status == W8A8_OK) status = cudaMemcpy(ref_h.data(), top_ref, (size_t)Me * 4, cudaMemcpyDeviceToHost) == cudaSuccess
-                                      ? W8A8_OK
-                                      : W8A8_ERR_CUDA;
-  cudaEvent_t e0 = nullptr, e1 = nullptr;
-  cudaEventCreate(&e0);
-  cudaEventCreate(&e1);
   std::vector<int32_t> n8(o->n_candidates);
-  for (int i = 0; i < o->n_candidates && status == W8A8_OK; ++i) {
-    const w8a8_mask& c = o->candidates[i];
-    status = w8a8_set_mask(m, c.ffn_bits, c.attn_bits, c.lm);
-    if (status != W8A8_OK) break;
-    n8[i] = __builtin_popcount(c.ffn_bits) + __builtin_popcount(c.attn_bits) + (c.lm ? 1 : 0);
-    double cn = 0.0;
-    if ((status = evaluate(top_c, &cn)) != W8A8_OK) break;
-    if (cudaMemcpy(top_h.data(), top_c, (size_t)Me * 4, cudaMemcpyDeviceToHost) != cudaSuccess) {
-      status = W8A8_ERR_CUDA;
-      break;
+  w8a8_status status = W8A8_OK;
+  {
+    AllocRun run{m, o->eval_tokens, o->eval_B, o->eval_T, o->decode_B, o->prefill_T, o->decode_steps, o->reps, stream};
+    status = run.init();
+    for (int i = 0; i < o->n_candidates && status == W8A8_OK; ++i) {
+      const w8a8_mask& c = o->candidates[i];
+      n8[i] = __builtin_popcount(c.ffn_bits) + __builtin_popcount(c.attn_bits) + (c.lm ? 1 : 0);
+      status = run.quality(c, &rep->top1[i], &rep->ppl_delta[i]);
+      if (status == W8A8_OK) status = run.latency(c, &rep->latency_ms[i]);
     }
-    int agree = 0, cnt = 0;
-    for (int b = 0; b < o->eval_B; ++b)
-      for (int t = 0; t + 1 < o->eval_T; ++t, ++cnt) agree += top_h[b * o->eval_T + t] == ref_h[b * o->eval_T + t];
-    rep->top1[i] = (float)agree / (float)cnt;
-    rep->ppl_delta[i] = (float)(std::exp(cn) / std::exp(ref_nll) - 1.0);
-    // latency: prefill, then decode steps from CUDA graphs fed by their own top-1 (greedy)
-    std::vector<float> runs;
-    for (int r = 0; r < o->reps && status == W8A8_OK; ++r) {
-      // prefill in chunks of at most max_tokens rows (the KV cache carries the earlier chunks)
-      const int chunk = std::max(1, m->cfg.max_tokens / o->decode_B);
-      for (int t0 = 0; t0 < o->prefill_T && status == W8A8_OK; t0 += chunk) {
-        const int tl = std::min(chunk, o->prefill_T - t0);
-        status = w8a8_decoder_forward(m, ptok + (size_t)o->decode_B * t0, o->decode_B, tl, t0, nullptr, top_c, stream);
-      }
-      if (status != W8A8_OK) break;
-      if (cudaMemcpyAsync(dtok, top_c, 4 * (size_t)o->decode_B, cudaMemcpyDeviceToDevice, st) != cudaSuccess) {
-        status = W8A8_ERR_CUDA;
-        break;
-      }
-      // warm the graph of this mask outside the timed region
-      if ((status = w8a8_decoder_decode_step(m, dtok, o->decode_B, o->prefill_T, nullptr, dtok, stream)) != W8A8_OK)
-        break;
-      cudaEventRecord(e0, st);
-      for (int s = 0; s < o->decode_steps && status == W8A8_OK; ++s)
-        status = w8a8_decoder_decode_step(m, dtok, o->decode_B, o->prefill_T + s, nullptr, dtok, stream);
-      cudaEventRecord(e1, st);
-      cudaEventSynchronize(e1);
-      float ms = 0.0f;
-      cudaEventElapsedTime(&ms, e0, e1);
-      runs.push_back(ms / (float)o->decode_steps);
-    }
-    if (status != W8A8_OK) break;
-    std::sort(runs.begin(), runs.end());
-    rep->latency_ms[i] = runs[runs.size() / 2];
   }
-  cudaEventDestroy(e0);
-  cudaEventDestroy(e1);
-  cleanup();
   if (status != W8A8_OK) {
     m->ffn_bits = saved_ffn;
     m->attn_bits = saved_attn;
@@ -821,4 +851,83 @@ extern "C" w8a8_status w8a8_allocate_mask(w8a8_model* m, const w8a8_alloc_opts* 
     return w8a8_set_mask(m, c.ffn_bits, c.attn_bits, c.lm);
   }
   return w8a8_set_mask(m, 0, 0, 0);
+}
+
+extern "C" int w8a8_greedy_order(const float* gain_ms, const float* top1, const float* ppl_delta, int n,
+                                 float min_top1, float max_ppl_delta, int32_t* order) {
+  if (!gain_ms || !top1 || !ppl_delta || !order || n <= 0) return 0;
+  const double t_scale = std::max(1e-6, 1.0 - (double)min_top1), p_scale = std::max(1e-6, (double)max_ppl_delta);
+  std::vector<std::pair<double, int>> keep;
+  for (int i = 0; i < n; ++i) {
+    if (!(gain_ms[i] > 0.0f) || !(top1[i] >= min_top1 && ppl_delta[i] <= max_ppl_delta)) continue;
+    const double cost = std::max(0.0, 1.0 - (double)top1[i]) / t_scale + std::max(0.0, (double)ppl_delta[i]) / p_scale;
+    keep.emplace_back((double)gain_ms[i] / (cost + 1e-3), i);
+  }
+  std::stable_sort(keep.begin(), keep.end(), [](const std::pair<double, int>& a, const std::pair<double, int>& b) {
+    return a.first > b.first;  // stable: equal scores keep the lower index first
+  });
+  for (size_t k = 0; k < keep.size(); ++k) order[k] = keep[k].second;
+  return (int)keep.size();
+}
+
+extern "C" w8a8_status w8a8_allocate_layers(w8a8_model* m, const w8a8_layer_alloc_opts* o,
+                                            w8a8_layer_alloc_report* rep, void* stream) {
+  W8A8_CHECK_ARG(m && o && rep && rep->gain_ms && rep->top1 && rep->ppl_delta && rep->order, W8A8_ERR_INVALID_ARG,
+                 "w8a8_allocate_layers: null argument");
+  W8A8_TRY(check_alloc_args(m, o->eval_tokens, o->eval_B, o->eval_T, o->decode_B, o->prefill_T, o->decode_steps,
+                            o->reps, "w8a8_allocate_layers"));
+  const int L = m->cfg.layers, n = 2 * L + 1;
+  auto single = [&](int i) {
+    w8a8_mask c{0u, 0u, 0};
+    if (i < L) c.ffn_bits = 1u << i;
+    else if (i < 2 * L) c.attn_bits = 1u << (i - L);
+    else c.lm = 1;
+    return c;
+  };
+  const uint32_t saved_ffn = m->ffn_bits, saved_attn = m->attn_bits;
+  const int saved_lm = m->lm;
+  w8a8_mask chosen{0u, 0u, 0};
+  w8a8_status status = W8A8_OK;
+  {
+    AllocRun run{m, o->eval_tokens, o->eval_B, o->eval_T, o->decode_B, o->prefill_T, o->decode_steps, o->reps, stream};
+    status = run.init();
+    if (status == W8A8_OK) status = run.latency(chosen, &rep->base_ms);
+    for (int i = 0; i < n && status == W8A8_OK; ++i) {
+      float ms = 0.0f;
+      status = run.quality(single(i), &rep->top1[i], &rep->ppl_delta[i]);
+      if (status == W8A8_OK) status = run.latency(single(i), &ms);
+      rep->gain_ms[i] = rep->base_ms - ms;
+    }
+    rep->n_order = 0;
+    rep->n_accepted = 0;
+    rep->chosen_top1 = 1.0f;
+    rep->chosen_ppl_delta = 0.0f;
+    if (status == W8A8_OK)
+      rep->n_order = w8a8_greedy_order(rep->gain_ms, rep->top1, rep->ppl_delta, n, o->min_top1, o->max_ppl_delta,
+                                       rep->order);
+    for (int k = 0; k < rep->n_order && status == W8A8_OK; ++k) {
+      const w8a8_mask s1 = single(rep->order[k]);
+      const w8a8_mask trial{chosen.ffn_bits | s1.ffn_bits, chosen.attn_bits | s1.attn_bits, chosen.lm | s1.lm};
+      float t1 = 0.0f, pd = 0.0f;
+      status = run.quality(trial, &t1, &pd);
+      if (status == W8A8_OK && t1 >= o->min_top1 && pd <= o->max_ppl_delta) {
+        chosen = trial;
+        rep->chosen_top1 = t1;
+        rep->chosen_ppl_delta = pd;
+        ++rep->n_accepted;
+      }
+    }
+    if (status == W8A8_OK) {
+      if (rep->n_accepted > 0) status = run.latency(chosen, &rep->chosen_ms);
+      else rep->chosen_ms = rep->base_ms;
+    }
+  }
+  if (status != W8A8_OK) {
+    m->ffn_bits = saved_ffn;
+    m->attn_bits = saved_attn;
+    m->lm = saved_lm;
+    return status;
+  }
+  rep->chosen = chosen;
+  return w8a8_set_mask(m, chosen.ffn_bits, chosen.attn_bits, chosen.lm);
 }

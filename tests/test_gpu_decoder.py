@@ -273,6 +273,39 @@ def test_token_nll_matches_oracle(B):
     assert np.allclose(got, OQ.nll(z, tg), rtol=1e-5, atol=1e-5)
 
 
+def test_allocate_layers_greedy(B, setup):
+    """The per-sublayer allocator on the 4-layer decoder: its ranking equals the library's rule on
+    its own single-sublayer measurements, and a replay of the greedy additions (each cumulative
+    mask's quality measured again through the group allocator, deterministic kernels) accepts
+    exactly the sublayers it chose."""
+    dec, _, toks = setup[:3]
+    ev = torch.from_numpy(toks[:, :16].copy()).cuda()
+    mt, mp = 0.9, 0.05
+    rep = dec.allocate_layers(ev, decode_B=1, prefill_T=8, decode_steps=4, reps=2, min_top1=mt, max_ppl_delta=mp)
+    n = 2 * L + 1
+    assert len(rep["gain_ms"]) == n and rep["base_ms"] > 0 and rep["chosen_ms"] > 0
+    assert rep["order"] == B.greedy_order(rep["gain_ms"], rep["top1"], rep["ppl_delta"], mt, mp)
+
+    def mask_of(ids):
+        f = sum(1 << i for i in ids if i < L)
+        a = sum(1 << (i - L) for i in ids if L <= i < 2 * L)
+        return (f, a, int(2 * L in ids))
+
+    chosen = []
+    for i in rep["order"]:
+        r = dec.allocate([mask_of(chosen + [i])], ev, decode_B=1, prefill_T=8, decode_steps=1, reps=1,
+                         min_top1=mt, max_ppl_delta=mp)
+        if r["top1"][0] >= np.float32(mt) and r["ppl_delta"][0] <= np.float32(mp):
+            chosen.append(i)
+    assert rep["n_accepted"] == len(chosen)
+    assert rep["chosen"] == mask_of(chosen)
+    if chosen:
+        assert rep["chosen_top1"] >= np.float32(mt) and rep["chosen_ppl_delta"] <= np.float32(mp)
+    else:
+        assert rep["chosen_ms"] == rep["base_ms"]
+    dec.set_mask(*rep["chosen"])
+
+
 def test_allocator_run(B, setup):
     dec, _, toks = setup[:3]
     cands = [(0, 0, 0), (0b1111, 0, 0), (0, 0, 1), (0b1001, 0, 1), (0b1111, 0b1111, 1)]
