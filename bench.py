@@ -605,6 +605,7 @@ def run_ours(args, dist: Dist):
         out["masks"] = mask_sweep(B, dec, dev)
         out["batches"] = batch_table(B, dec, dev)
         out["kernels"] = sweep(B, dev, head, xh, flush, stream, peaks)
+        out["sqnr"] = sqnr_table(B, dec, dev)
     dec.close()
     return out
 
@@ -642,6 +643,48 @@ def mask_sweep(B, dec, dev):
         "speedup_vs_bf16": round(lr["base_ms"] / lr["chosen_ms"], 4), "top1": round(lr["chosen_top1"], 5),
         "ppl_delta": round(lr["chosen_ppl_delta"], 5), "weight_gb": round(decode_weight_bytes(f, a, l) / 1e9, 4),
         "seconds": round(time.time() - t0, 1)}
+    return out
+
+
+def sqnr_table(B, dec, dev):
+    """SQNR diagnostics (Eq. sqnr-block per decoder layer, Eq. sqnr-ffn on the logits) of four
+    masks over a 4 x 128-token prefill of the evaluation stream, isolated and propagated, with
+    SmoothQuant (alpha 0.5) and with delta = 1 (no smoothing); the model is re-prepared with
+    smoothing afterwards."""
+    import torch
+    import synth
+    g = B.GROUP_BITS
+    masks = {"ffn 5+5 + lm": (g["5+5"], 0, 1), "ffn all26 + lm": (g["all26"], 0, 1),
+             "att all26": (0, g["all26"], 0), "ffn all26 + att all26 + lm": (g["all26"], g["all26"], 1)}
+    toks = torch.from_numpy(synth.tokens(4 * PREFILL, VOCAB, seed=2, stream=1).reshape(4, PREFILL)).to(dev)
+    t0 = time.time()
+    out = {}
+    r2 = lambda v: round(v, 2) if v != float("inf") else None  # noqa: E731  (None: layer left in bf16)
+    for smooth in (True, False):
+        dec.prepare(0.5, smooth)
+        rows = {}
+        for name, m in masks.items():
+            row = {}
+            for mode in ("isolated", "propagated"):
+                layer, lm = dec.sqnr_profile(toks, m, isolated=mode == "isolated")
+                fin = [v for v in layer if v != float("inf")]
+                row[mode] = {"layers_db": [r2(v) for v in layer], "min_db": r2(min(fin)) if fin else None,
+                             "lm_head_logits_db": r2(lm)}
+            rows[name] = row
+        out["smoothquant_alpha_0.5" if smooth else "delta_1"] = rows
+    dec.prepare(0.5, True)
+    # the single linear (M 16, 1152 -> 6912, 8 outlier channels x20, delta from its own input):
+    # the W8A8 output against the bf16 pass-through's, with and without smoothing
+    c = synth.linear_case()
+    x, w = c["x"].to(dev), c["w"].to(dev)
+    stat = torch.from_numpy(c["calib32"]).abs().amax(0).to(dev)
+    y_ref = B.linear_bf16(w, x).float()
+    lin = {}
+    for smooth in (True, False):
+        q = B.prepare_weights(w, stat, 0.5, smooth)
+        lin["smoothquant_alpha_0.5" if smooth else "delta_1"] = round(B.sqnr_db(y_ref, B.linear(q, x).float()), 2)
+    out["single_linear_db"] = lin
+    out["seconds"] = round(time.time() - t0, 1)
     return out
 
 
@@ -834,7 +877,7 @@ def main():
             "clocks": res["clocks"], "roofline": res["roofline"], "e2e": res["e2e"], "gpu_launches": res["launches"],
             "kernels_per_step": res["kernels_per_step"], "cpu_baseline": cpu,
             "masks": res.get("masks"), "batches": res.get("batches"), "kernels": res.get("kernels"),
-            "setup_s": res["setup_s"],
+            "sqnr": res.get("sqnr"), "setup_s": res["setup_s"],
         }
         print(json.dumps(line))
     dist.close()

@@ -405,6 +405,25 @@ typedef struct {
 w8a8_status w8a8_allocate_layers(w8a8_model* m, const w8a8_layer_alloc_opts* opts, w8a8_layer_alloc_report* report,
                                  void* stream);
 
+/* SQNR in dB (Eq. sqnr-ffn; Eq. sqnr-block is the same ratio of means):
+ * 10 log10(sum y_ref^2 / sum (y_ref - y_q)^2) over n device floats, the sums taken in fp64 in a
+ * fixed order (deterministic); +inf when the two arrays are equal.  Synchronous. */
+w8a8_status w8a8_sqnr_db(const float* y_ref, const float* y_q, size_t n, double* out_db, void* stream);
+
+/* SQNR diagnostics of a mask over a prefill of tokens [B, T] (device, T >= 2) from position 0,
+ * against the all-bf16 decoder (Combined Configurations: the isolated and propagated regimes).
+ * layer_db (host [L]): the SQNR of every decoder block's output (the residual stream after its
+ * post-FFN step, Eq. sqnr-block); lm_db (host [1]): of the lm_head's fp32 logits.
+ *   propagated (isolated = 0): one pass under the whole mask, so errors accumulate;
+ *   isolated (isolated = 1): for each layer a pass with only that layer's sublayers of the mask
+ *   quantised, so the layer takes the reference input (+inf where the mask quantises nothing in
+ *   the layer); the lm_head likewise alone (+inf if the mask leaves it in bf16).
+ * Leaves the model's mask as it was; overwrites the layers' KV cache rows [0, T).  Synchronous;
+ * requires w8a8_model_prepare (with or without smoothing: the delta = 1 ablation is a prepare
+ * with smooth = 0). */
+w8a8_status w8a8_sqnr_profile(w8a8_model* m, const int32_t* tokens, int B, int T, const w8a8_mask* mask, int isolated,
+                              float* layer_db, float* lm_db, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -143,6 +143,8 @@ SIGNATURES = {
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
     "w8a8_allocate_mask": (_i32, [_vp, ctypes.POINTER(AllocOptsC), ctypes.POINTER(AllocReportC), _vp]),
     "w8a8_greedy_order": (_i32, [_fp, _fp, _fp, _i32, _f32, _f32, ctypes.POINTER(ctypes.c_int32)]),
+    "w8a8_sqnr_db": (_i32, [_vp, _vp, ctypes.c_size_t, ctypes.POINTER(ctypes.c_double), _vp]),
+    "w8a8_sqnr_profile": (_i32, [_vp, _vp, _i32, _i32, ctypes.POINTER(MaskC), _i32, _fp, _fp, _vp]),
     "w8a8_allocate_layers": (_i32, [_vp, ctypes.POINTER(LayerAllocOptsC), ctypes.POINTER(LayerAllocReportC), _vp]),
 }
 
@@ -444,6 +446,15 @@ def candidate_masks():
     return out
 
 
+def sqnr_db(y_ref: torch.Tensor, y_q: torch.Tensor, stream=None) -> float:
+    """Eq. sqnr-ffn / sqnr-block of two fp32 device tensors of the same size (fp64 sums on the GPU)."""
+    assert y_ref.dtype == torch.float32 and y_q.dtype == torch.float32 and y_ref.numel() == y_q.numel()
+    out = ctypes.c_double()
+    _check("w8a8_sqnr_db", lib().w8a8_sqnr_db(_p(y_ref.contiguous()), _p(y_q.contiguous()), y_ref.numel(),
+                                              ctypes.byref(out), _stream(stream)))
+    return out.value
+
+
 def greedy_order(gain_ms, top1, ppl_delta, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> list:
     """The library's per-sublayer ranking rule on host arrays: the ranked sublayer indices."""
     n = len(gain_ms)
@@ -602,6 +613,17 @@ class Decoder:
         _check("w8a8_allocate_mask", lib().w8a8_allocate_mask(self.h, ctypes.byref(opts), ctypes.byref(rep),
                                                               _stream(stream)))
         return {"chosen": rep.chosen, "latency_ms": list(lat), "top1": list(t1), "ppl_delta": list(pd)}
+
+    def sqnr_profile(self, tokens: torch.Tensor, mask, isolated: bool, stream=None):
+        """Per-layer block-output SQNR (dB, length L) and the lm_head logits' SQNR of mask =
+        (ffn_bits, attn_bits, lm) over a prefill of tokens [B, T], isolated or propagated."""
+        B, T = tokens.shape
+        L = self.cfg.layers
+        layer, lm = (ctypes.c_float * L)(), (ctypes.c_float * 1)()
+        mk = MaskC(int(mask[0]), int(mask[1]), int(mask[2]))
+        _check("w8a8_sqnr_profile", lib().w8a8_sqnr_profile(self.h, _p(_bits(tokens)), B, T, ctypes.byref(mk),
+                                                            int(bool(isolated)), layer, lm, _stream(stream)))
+        return list(layer), lm[0]
 
     def allocate_layers(self, eval_tokens: torch.Tensor, decode_B: int, prefill_T: int, decode_steps: int,
                         reps: int = 3, min_top1: float = 0.989, max_ppl_delta: float = 0.01, stream=None) -> dict:

@@ -71,6 +71,9 @@ struct w8a8_model {
   float* mega_part = nullptr;
   bool mega_ok = false;
   int decode_path = 0;
+  // diagnostics: when set, a forward copies every layer's output (the residual stream after its
+  // post-FFN step, fp32 [M, H]) to capture + l M H
+  float* capture = nullptr;
 
   cudaStream_t st = nullptr;  // private stream for graph capture / replay
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
@@ -165,7 +168,7 @@ w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, 
 // decode GEMV: q/k/v takes the step after the previous layer's FFN, gate/up the step after o.
 // It needs the decode GEMV to take both linears of every layer under the current mask.
 bool fuse_residual(const w8a8_model* m, int M, bool calib) {
-  if (calib || M > 8) return false;
+  if (calib || M > 8 || m->capture) return false;
   const int H = m->cfg.hidden, F = m->cfg.inter;
   for (int l = 0; l < m->cfg.layers; ++l) {
     const bool att8 = m->prepared && ((m->attn_bits >> l) & 1u);
@@ -185,7 +188,8 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
   float* rc = m->r;   // the residual stream as of now
   float* rn = m->r2;  // where a fused update writes the next one
   W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st));
-  const bool mega = !calib && B == 1 && T == 1 && m->mega_ok && m->decode_path == W8A8_DECODE_PERSISTENT;
+  const bool mega =
+      !calib && !m->capture && B == 1 && T == 1 && m->mega_ok && m->decode_path == W8A8_DECODE_PERSISTENT;
   if (mega) {  // every layer in one persistent launch, then the final residual step
     W8A8_CUDA(cudaMemsetAsync(m->mega_sync, 0, mega_sync_words(c.layers, c.n_q) * sizeof(unsigned int), st));
     MegaArgs g{};
@@ -267,6 +271,8 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
       const float* next = l + 1 < c.layers ? m->L[l + 1].ln_in : m->final_norm;
       W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, rc, m->a, st));
     }
+    if (m->capture)
+      W8A8_CUDA(cudaMemcpyAsync(m->capture + (size_t)l * M * H, rc, sizeof(float) * M * H, cudaMemcpyDeviceToDevice, st));
   }
   if (calib) return launch_act_absmax(m->a, M, H, m->stat_lm(), st);
   const bool lm8 = m->prepared && m->lm;
@@ -296,6 +302,35 @@ w8a8_status check_call(w8a8_model* m, int B, int T, int start_pos) {
 }
 
 // ------------------------------------------------------------------------------ NLL kernel
+// Eq. sqnr-ffn / sqnr-block: the sums of y_ref^2 and (y_ref - y_q)^2 in fp64.  Each of the
+// kSqnrBlocks blocks strides over the elements and reduces its 256 threads in a fixed tree; the
+// host adds the blocks' partials in block order (deterministic).
+constexpr int kSqnrBlocks = 256;
+__global__ void sqnr_partial_kernel(const float* __restrict__ ref, const float* __restrict__ q, size_t n,
+                                    double* __restrict__ part) {
+  __shared__ double ss[256], se[256];
+  double s = 0.0, e = 0.0;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    const double r = ref[i], d = r - (double)q[i];
+    s += r * r;
+    e += d * d;
+  }
+  ss[threadIdx.x] = s;
+  se[threadIdx.x] = e;
+  __syncthreads();
+  for (int o = 128; o > 0; o >>= 1) {
+    if ((int)threadIdx.x < o) {
+      ss[threadIdx.x] += ss[threadIdx.x + o];
+      se[threadIdx.x] += se[threadIdx.x + o];
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    part[2 * blockIdx.x] = ss[0];
+    part[2 * blockIdx.x + 1] = se[0];
+  }
+}
+
 __global__ void nll_kernel(const float* __restrict__ logits, const int32_t* __restrict__ targets, int V,
                            float* __restrict__ nll) {
   __shared__ double red[32];
@@ -930,4 +965,98 @@ extern "C" w8a8_status w8a8_allocate_layers(w8a8_model* m, const w8a8_layer_allo
   }
   rep->chosen = chosen;
   return w8a8_set_mask(m, chosen.ffn_bits, chosen.attn_bits, chosen.lm);
+}
+
+extern "C" w8a8_status w8a8_sqnr_db(const float* y_ref, const float* y_q, size_t n, double* out_db, void* stream) {
+  W8A8_CHECK_ARG(y_ref && y_q && out_db, W8A8_ERR_INVALID_ARG, "w8a8_sqnr_db: null pointer");
+  W8A8_CHECK_ARG(n > 0, W8A8_ERR_INVALID_ARG, "w8a8_sqnr_db: no elements");
+  W8A8_TRY(check_device());
+  cudaStream_t st = as_stream(stream);
+  double* part = nullptr;
+  W8A8_CUDA(cudaMalloc(&part, sizeof(double) * 2 * kSqnrBlocks));
+  sqnr_partial_kernel<<<kSqnrBlocks, 256, 0, st>>>(y_ref, y_q, n, part);
+  std::vector<double> h(2 * kSqnrBlocks);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h.data(), part, sizeof(double) * h.size(), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(part);
+  W8A8_CUDA(e);
+  double sig = 0.0, err = 0.0;
+  for (int b = 0; b < kSqnrBlocks; ++b) {
+    sig += h[2 * b];
+    err += h[2 * b + 1];
+  }
+  *out_db = err > 0.0 ? 10.0 * std::log10(sig / err) : INFINITY;
+  return W8A8_OK;
+}
+
+extern "C" w8a8_status w8a8_sqnr_profile(w8a8_model* m, const int32_t* tokens, int B, int T, const w8a8_mask* mask,
+                                         int isolated, float* layer_db, float* lm_db, void* stream) {
+  W8A8_CHECK_ARG(m && tokens && mask && layer_db && lm_db, W8A8_ERR_INVALID_ARG, "w8a8_sqnr_profile: null argument");
+  W8A8_CHECK_ARG(m->prepared, W8A8_ERR_INVALID_ARG, "w8a8_sqnr_profile: w8a8_model_prepare first");
+  W8A8_CHECK_ARG(T >= 2, W8A8_ERR_SHAPE, "w8a8_sqnr_profile: T >= 2 (a prefill)");
+  W8A8_TRY(check_call(m, B, T, 0));
+  const int L = m->cfg.layers, M = B * T, H = m->cfg.hidden, V = m->cfg.vocab;
+  cudaStream_t st = as_stream(stream);
+  const uint32_t saved_ffn = m->ffn_bits, saved_attn = m->attn_bits;
+  const int saved_lm = m->lm;
+  std::vector<void*> tmp;
+  auto talloc = [&](void** p, size_t bytes) -> w8a8_status {
+    W8A8_CUDA(cudaMalloc(p, bytes));
+    tmp.push_back(*p);
+    return W8A8_OK;
+  };
+  float *h_ref = nullptr, *h_q = nullptr, *lg_ref = nullptr, *lg_q = nullptr;
+  int32_t* top = nullptr;
+  const size_t hl = (size_t)M * H;
+  auto run = [&](uint32_t f, uint32_t a, int l, float* hcap, float* lg) -> w8a8_status {
+    W8A8_TRY(w8a8_set_mask(m, f, a, l));
+    m->capture = hcap;
+    const w8a8_status s = w8a8_decoder_forward(m, tokens, B, T, 0, lg, top, stream);
+    m->capture = nullptr;
+    return s;
+  };
+  auto sqnr = [&](const float* r, const float* q, size_t n, float* out) -> w8a8_status {
+    double db = 0.0;
+    W8A8_TRY(w8a8_sqnr_db(r, q, n, &db, stream));
+    *out = (float)db;
+    return W8A8_OK;
+  };
+  w8a8_status s = W8A8_OK;
+  do {
+    if ((s = talloc((void**)&h_ref, sizeof(float) * hl * L)) != W8A8_OK) break;
+    if ((s = talloc((void**)&h_q, sizeof(float) * hl * L)) != W8A8_OK) break;
+    if ((s = talloc((void**)&lg_ref, sizeof(float) * (size_t)M * V)) != W8A8_OK) break;
+    if ((s = talloc((void**)&lg_q, sizeof(float) * (size_t)M * V)) != W8A8_OK) break;
+    if ((s = talloc((void**)&top, sizeof(int32_t) * (size_t)std::max(M, 4))) != W8A8_OK) break;
+    if ((s = run(0u, 0u, 0, h_ref, lg_ref)) != W8A8_OK) break;  // the reference: all bf16
+    if (!isolated) {  // one pass under the whole mask: errors accumulate
+      if ((s = run(mask->ffn_bits, mask->attn_bits, mask->lm, h_q, lg_q)) != W8A8_OK) break;
+      for (int l = 0; l < L && s == W8A8_OK; ++l) s = sqnr(h_ref + l * hl, h_q + l * hl, hl, &layer_db[l]);
+      if (s == W8A8_OK) s = sqnr(lg_ref, lg_q, (size_t)M * V, lm_db);
+      break;
+    }
+    // isolated: each layer's quantised sublayers alone, so the layer takes the reference input
+    for (int l = 0; l < L && s == W8A8_OK; ++l) {
+      const uint32_t f = mask->ffn_bits & (1u << l), a = mask->attn_bits & (1u << l);
+      if (!f && !a) {
+        layer_db[l] = INFINITY;  // nothing quantised: the reference output itself
+        continue;
+      }
+      if ((s = run(f, a, 0, h_q, nullptr)) == W8A8_OK) s = sqnr(h_ref + l * hl, h_q + l * hl, hl, &layer_db[l]);
+    }
+    if (s != W8A8_OK) break;
+    if (mask->lm) {
+      if ((s = run(0u, 0u, 1, h_q, lg_q)) == W8A8_OK) s = sqnr(lg_ref, lg_q, (size_t)M * V, lm_db);
+    } else {
+      *lm_db = INFINITY;
+    }
+  } while (0);
+  cudaStreamSynchronize(st);
+  for (void* p : tmp) cudaFree(p);
+  m->capture = nullptr;
+  m->ffn_bits = saved_ffn;
+  m->attn_bits = saved_attn;
+  m->lm = saved_lm;
+  return s;
 }

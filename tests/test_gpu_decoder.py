@@ -273,6 +273,41 @@ def test_token_nll_matches_oracle(B):
     assert np.allclose(got, OQ.nll(z, tg), rtol=1e-5, atol=1e-5)
 
 
+def test_sqnr_db_matches_oracle(B):
+    """The GPU reduction against the oracle's Eq. sqnr-ffn (both in double; only the summation order
+    differs), on values whose SQNR spans the paper's range; equal inputs give +inf."""
+    g = np.random.default_rng(4)
+    for noise in (1e-1, 1e-3, 1e-5):
+        ref = g.standard_normal(300_001).astype(np.float32)
+        q = (ref + noise * g.standard_normal(ref.size)).astype(np.float32)
+        got = B.sqnr_db(torch.from_numpy(ref).cuda(), torch.from_numpy(q).cuda())
+        want = OQ.sqnr_db(ref.astype(np.float64), q.astype(np.float64))
+        assert abs(got - want) < 1e-9, (noise, got, want)
+    x = torch.from_numpy(g.standard_normal(1000).astype(np.float32)).cuda()
+    assert B.sqnr_db(x, x.clone()) == float("inf")
+
+
+def test_sqnr_profile_isolated_and_propagated(B, setup):
+    """Isolated: a layer the mask leaves in bf16 reproduces the reference (+inf); the first quantised
+    layer sees the reference input in both regimes, so its SQNR is the same number; later layers
+    and the logits carry the accumulated error in the propagated regime.  The model's mask is left
+    as it was."""
+    dec, _, toks = setup[:3]
+    dec.set_mask(0b0010, 0b1000, 0)
+    before = dec.get_mask()
+    tt = torch.from_numpy(toks[:, :16].copy()).cuda()
+    mask = (0b0101, 0b0010, 1)  # FFN of layers 0 and 2, attention of layer 1, lm_head
+    iso, iso_lm = dec.sqnr_profile(tt, mask, isolated=True)
+    pro, pro_lm = dec.sqnr_profile(tt, mask, isolated=False)
+    assert dec.get_mask() == before
+    assert iso[3] == float("inf") and all(np.isfinite(iso[:3]))
+    assert iso[0] == pro[0]
+    assert all(np.isfinite(pro)) and np.isfinite(iso_lm) and np.isfinite(pro_lm)
+    assert pro[3] < 60.0 and pro_lm < iso_lm  # the error carried through layer 3 and into the logits
+    none, none_lm = dec.sqnr_profile(tt, (0, 0, 0), isolated=False)
+    assert all(v == float("inf") for v in none) and none_lm == float("inf")
+
+
 def test_allocate_layers_greedy(B, setup):
     """The per-sublayer allocator on the 4-layer decoder: its ranking equals the library's rule on
     its own single-sublayer measurements, and a replay of the greedy additions (each cumulative
