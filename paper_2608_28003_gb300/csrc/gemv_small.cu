@@ -126,6 +126,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int row0 = blockIdx.x * R;
 
   pdl_trigger();
+  if (threadIdx.x == kCW * 32) {  // the producer thread: fetch the tensor map before the first copy needs it
+    prefetch_tmap(&tmW);
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(full + s), 1);

@@ -111,6 +111,10 @@ __global__ void __launch_bounds__(kThreads, Cps<NB>::value)
   auto cta_of = [&](long long u) -> int { return (int)(((u + 1) * P + U - 1) / U - 1); };
 
   pdl_trigger();
+  if (threadIdx.x == kConsumerWarps * 32) {  // the producer thread: fetch the tensor maps before the first copy needs them
+    prefetch_tmap(&tmW);
+    prefetch_tmap(&tmX);
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(full + s), 1);
@@ -563,6 +567,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   auto cta_of = [&](long long u) -> int { return (int)(((u + 1) * P + U - 1) / U - 1); };
 
   pdl_trigger();
+  if (threadIdx.x == kConsumerWarps * 32) {  // the producer thread: fetch the tensor map before the first copy needs it
+    prefetch_tmap(&tmW);
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(full + s), 1);
