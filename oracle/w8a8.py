@@ -7,7 +7,7 @@ the precision the GPU path decides in and both sides must decide identically.  S
 the paper defines exactly (the INT8 dot products, the bf16 pass-through) are evaluated
 exactly or in fp64.
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open:
   * round() is round-half-to-even (np.rint); codes are clamped to [-127, 127]
     (2^(b-1) - 1 with b = 8, Eq. si), so -128 never occurs.
   * x / s with s = m / 127 is evaluated as x * (127 / m): one fp32 division per row or
