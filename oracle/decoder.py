@@ -181,9 +181,10 @@ class OracleDecoder:
                     out[b, t, h] = pr @ V
         return out
 
-    def forward(self, tokens, pos0, mask=None, stats=None, want_logits=True):
+    def forward(self, tokens, pos0, mask=None, stats=None, want_logits=True, want_layers=False):
         """tokens [B, T] at positions pos0 .. pos0+T-1; mask an oracle.masks.Mask or None
-        (all bf16).  Returns dict(logits fp32 [B, T, V], top1 [B, T], final bf16 hidden)."""
+        (all bf16).  Returns dict(logits fp32 [B, T, V], top1 [B, T], final bf16 hidden, and with
+        want_layers every layer's output: the residual stream after its post-FFN step, [L][M, H])."""
         c, w = self.cfg, self.w
         toks = np.asarray(tokens).reshape(self.B, -1)
         T = toks.shape[1]
@@ -194,6 +195,7 @@ class OracleDecoder:
         es = np.float32(c.embed_scale)
         r = (w["embed"][toks.reshape(-1)].astype(np.float32) * es).astype(np.float64)
         pos = np.arange(pos0, pos0 + T)
+        layers = []
         for l in range(c.layers):
             base = c.rope_global if l in c.global_layers else c.rope_local
             a = _w.round_to_bf16(rmsnorm(r, w["ln_in"][l], c.eps).astype(np.float32))
@@ -217,14 +219,51 @@ class OracleDecoder:
             a2 = _w.round_to_bf16(rmsnorm(r, w["ln_pre_ffn"][l], c.eps).astype(np.float32))
             f = self._ffn(a2, l, l in ffn_set, stats).astype(np.float64)
             r = r + rmsnorm(f, w["ln_post_ffn"][l], c.eps)
+            if want_layers:
+                layers.append(r.copy())
         fin = _w.round_to_bf16(rmsnorm(r, w["final_norm"], c.eps).astype(np.float32))
         if stats is not None:
             stats["lm"] = np.maximum(stats["lm"], _w.act_absmax(fin))
         if not want_logits:
-            return {"final": fin}
+            return {"final": fin, "layers": layers}
         if lm8:
             head = _b.lm_head_w8a8(fin, self.prep["lm"])
         else:
             head = _b.lm_head_bf16(fin, w["embed"])
         return {"logits": head["logits"].reshape(self.B, T, -1),
-                "top1": head["top1"].reshape(self.B, T), "final": fin}
+                "top1": head["top1"].reshape(self.B, T), "final": fin, "layers": layers}
+
+    def sqnr_profile(self, tokens, mask, isolated: bool):
+        """SQNR of every layer's output (Eq. sqnr-block) and of the logits (Eq. sqnr-ffn) under
+        mask against the all-bf16 model, over a prefill from position 0 (Combined Configurations):
+        propagated, one pass under the whole mask; isolated, a pass per layer with only that
+        layer's sublayers of the mask quantised (it then takes the reference input; +inf where the
+        mask quantises nothing in the layer), and the lm_head alone likewise."""
+        from . import masks as _m
+        from . import quality as _q
+        L = self.cfg.layers
+        self.reset()
+        ref = self.forward(tokens, 0, None, want_layers=True)
+        if not isolated:
+            self.reset()
+            q = self.forward(tokens, 0, mask, want_layers=True)
+            self.reset()
+            return ([_q.sqnr_block_db(ref["layers"][l], q["layers"][l]) for l in range(L)],
+                    _q.sqnr_db(ref["logits"].astype(np.float64), q["logits"].astype(np.float64)))
+        out = []
+        for l in range(L):
+            f = frozenset({l}) & mask.ffn
+            a = frozenset({l}) & mask.att
+            if not f and not a:
+                out.append(float("inf"))
+                continue
+            self.reset()
+            q = self.forward(tokens, 0, _m.Mask(f, a, False), want_layers=True, want_logits=False)
+            out.append(_q.sqnr_block_db(ref["layers"][l], q["layers"][l]))
+        lm = float("inf")
+        if mask.lm:
+            self.reset()
+            q = self.forward(tokens, 0, _m.Mask(frozenset(), frozenset(), True))
+            lm = _q.sqnr_db(ref["logits"].astype(np.float64), q["logits"].astype(np.float64))
+        self.reset()
+        return out, lm

@@ -43,17 +43,20 @@ def ppl_delta(ppl_q: float, ppl_ref: float) -> float:
 
 
 def sqnr_db(y_clean: np.ndarray, y_dirty: np.ndarray) -> float:
-    """Eq. sqnr-ffn: 10 log10(||y_clean||^2 / ||y_clean - y_dirty||^2)."""
+    """Eq. sqnr-ffn: 10 log10(||y_clean||^2 / ||y_clean - y_dirty||^2); +inf when the two are
+    equal (the noiseless limit)."""
     c = np.asarray(y_clean, np.float64)
     d = c - np.asarray(y_dirty, np.float64)
-    return float(10.0 * np.log10(np.sum(c * c) / np.sum(d * d)))
+    e = np.sum(d * d)
+    return float("inf") if e == 0 else float(10.0 * np.log10(np.sum(c * c) / e))
 
 
 def sqnr_block_db(h_ref: np.ndarray, h_q: np.ndarray) -> float:
-    """Eq. sqnr-block: 10 log10(E[h_ref^2] / E[(h_ref - h_q)^2])."""
+    """Eq. sqnr-block: 10 log10(E[h_ref^2] / E[(h_ref - h_q)^2]); +inf when the two are equal."""
     r = np.asarray(h_ref, np.float64)
     d = r - np.asarray(h_q, np.float64)
-    return float(10.0 * np.log10(np.mean(r * r) / np.mean(d * d)))
+    e = np.mean(d * d)
+    return float("inf") if e == 0 else float(10.0 * np.log10(np.mean(r * r) / e))
 
 
 def speedup(toks_per_s: float, toks_per_s_base: float) -> float:

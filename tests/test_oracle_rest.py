@@ -244,3 +244,23 @@ def test_ffn_block_stages_consistent():
     assert np.array_equal(xq, r["down"]["xq"])
     ref = blocks.ffn_bf16(c["x32"], c["wg32"], c["wu32"], c["wd32"])
     assert np.abs(r["y"] - ref["y"]).max() < 0.1 * np.abs(ref["y"]).max()
+
+
+def test_decoder_sqnr_profile_structure():
+    """The oracle's SQNR profile: nothing quantised gives +inf everywhere; in the propagated regime
+    the layers before the first quantised one are untouched (+inf: errors do not flow backwards),
+    and the first quantised layer has the same SQNR in both regimes (it sees the reference input
+    either way); in the isolated regime a layer the mask leaves in bf16 is +inf."""
+    cfg, w = _tiny_decoder(layers=4)
+    dec = decoder.OracleDecoder(cfg, w, batch=1, max_len=16)
+    dec.calibrate([np.random.default_rng(4).integers(0, cfg.vocab, (1, 12))])
+    dec.prepare()
+    toks = np.random.default_rng(5).integers(0, cfg.vocab, (1, 10))
+    none, none_lm = dec.sqnr_profile(toks, masks.Mask(frozenset(), frozenset(), False), isolated=False)
+    assert all(v == float("inf") for v in none) and none_lm == float("inf")
+    mask = masks.Mask(frozenset({1, 3}), frozenset({2}), True)
+    pro, pro_lm = dec.sqnr_profile(toks, mask, isolated=False)
+    iso, iso_lm = dec.sqnr_profile(toks, mask, isolated=True)
+    assert pro[0] == float("inf") and all(np.isfinite(pro[1:])) and np.isfinite(pro_lm)
+    assert iso[0] == float("inf") and all(np.isfinite(iso[1:])) and np.isfinite(iso_lm)
+    assert iso[1] == pro[1]
