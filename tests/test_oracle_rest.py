@@ -264,3 +264,55 @@ def test_decoder_sqnr_profile_structure():
     assert pro[0] == float("inf") and all(np.isfinite(pro[1:])) and np.isfinite(pro_lm)
     assert iso[0] == float("inf") and all(np.isfinite(iso[1:])) and np.isfinite(iso_lm)
     assert iso[1] == pro[1]
+
+
+def test_rope_frequencies_by_hand_and_relative_position():
+    """Rotate-half RoPE with angle pos * base^(-2i/d) for pair (i, i + d/2): checked element by
+    element at d = 4 (pair 0 turns by pos radians, pair 1 by pos / 100 with base 10^4), and the
+    defining property: the score of a rotated query and key depends on their positions' difference
+    only."""
+    x = np.array([[1.0, 2.0, 3.0, 4.0]])
+    r = decoder.rope(x, np.array([3]), 10000.0, 4)[0]
+    a0, a1 = 3.0, 3.0 / 100.0
+    want = [1 * np.cos(a0) - 3 * np.sin(a0), 2 * np.cos(a1) - 4 * np.sin(a1),
+            3 * np.cos(a0) + 1 * np.sin(a0), 4 * np.cos(a1) + 2 * np.sin(a1)]
+    assert np.allclose(r, want, rtol=0, atol=1e-12)
+    g = np.random.default_rng(6)
+    q, k = g.standard_normal((1, 256)), g.standard_normal((1, 256))
+    for base in (1e4, 1e6):
+        def score(m, n):
+            return (decoder.rope(q, np.array([m]), base, 256) @ decoder.rope(k, np.array([n]), base, 256).T).item()
+        for m, n, s in ((5, 2, 11), (100, 99, 1900), (0, 7, 1024)):
+            assert score(m, n) == pytest.approx(score(m + s, n + s), rel=1e-9, abs=1e-9)
+
+
+def test_rmsnorm_against_torch_and_scale_invariance():
+    g = np.random.default_rng(7)
+    x = g.standard_normal((9, 1152)) * 3.0
+    w = g.uniform(0.5, 1.5, 1152)
+    ref = torch.nn.functional.rms_norm(torch.from_numpy(x), (1152,), torch.from_numpy(w), eps=1e-6).numpy()
+    assert np.allclose(decoder.rmsnorm(x, w, 1e-6), ref, rtol=1e-12, atol=1e-12)
+    assert np.allclose(decoder.rmsnorm(5.0 * x, w, 0.0), decoder.rmsnorm(x, w, 0.0), rtol=1e-12, atol=0)
+
+
+@pytest.mark.parametrize("glob", [True, False])
+def test_attention_against_torch_sdpa(glob):
+    """The oracle's attention (scores q.k / sqrt(d), softmax over the allowed keys, 4 query heads
+    sharing one key/value head) against torch's scaled_dot_product_attention in fp64 with the causal
+    (global layer) or causal sliding-window (local layer) mask written out."""
+    cfg, w = _tiny_decoder(layers=1, window=3)
+    cfg.global_layers = (0,) if glob else ()
+    dec = decoder.OracleDecoder(cfg, w, batch=1, max_len=16)
+    g = np.random.default_rng(8)
+    T, d = 7, cfg.head_dim
+    dec.kc[0, 0, :T] = g.standard_normal((T, cfg.kv_dim))
+    dec.vc[0, 0, :T] = g.standard_normal((T, cfg.kv_dim))
+    q = g.standard_normal((1, T, cfg.n_q, d))
+    got = dec._attention(0, q, 0, T)[0]  # [T, n_q, d]
+    K = torch.from_numpy(dec.kc[0, 0, :T].copy()).view(1, 1, T, d).expand(1, cfg.n_q, T, d)
+    V = torch.from_numpy(dec.vc[0, 0, :T].copy()).view(1, 1, T, d).expand(1, cfg.n_q, T, d)
+    Q = torch.from_numpy(q.copy()).permute(0, 2, 1, 3)  # [1, n_q, T, d]
+    i = torch.arange(T)
+    allowed = (i[None, :] <= i[:, None]) & (glob | (i[None, :] > i[:, None] - cfg.window))
+    ref = torch.nn.functional.scaled_dot_product_attention(Q, K, V, attn_mask=allowed)[0].permute(1, 0, 2).numpy()
+    assert np.allclose(got, ref, rtol=1e-12, atol=1e-12)
