@@ -96,3 +96,25 @@ def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         binding.lib()
+
+
+def test_header_is_plain_c(tmp_path):
+    """The boundary is a C ABI: every header compiles as strict C99 (no C++ constructs), and its
+    structs are usable from C."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "use_header.c"
+    src.write_text('#include "w8a8.h"\n'
+                   "int main(void) {\n"
+                   "  w8a8_mask m = {0u, 0u, 0};\n"
+                   "  w8a8_layer_alloc_report r;\n"
+                   "  r.chosen = m;\n"
+                   "  return (int)r.chosen.lm;\n"
+                   "}\n")
+    out = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I",
+                          os.path.join(ROOT, "include"), "-c", str(src), "-o", str(tmp_path / "use_header.o")],
+                         capture_output=True, text=True)
+    assert out.returncode == 0, out.stderr
