@@ -316,3 +316,77 @@ def test_attention_against_torch_sdpa(glob):
     allowed = (i[None, :] <= i[:, None]) & (glob | (i[None, :] > i[:, None] - cfg.window))
     ref = torch.nn.functional.scaled_dot_product_attention(Q, K, V, attn_mask=allowed)[0].permute(1, 0, 2).numpy()
     assert np.allclose(got, ref, rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------------------------- decoder composition
+def _composition_decoder(seed=11):
+    """One layer, every matrix N(0, 0.2), the final norm's multiplier non-uniform."""
+    cfg = decoder.DecoderConfig(hidden=32, inter=48, layers=1, n_q=4, n_kv=1, head_dim=8, vocab=64,
+                                window=16, global_layers=(0,))
+    import synth
+    f32, _, norms = synth.decoder_weights(1, 32, 48, 64, 4, 1, 8, seed=seed, std=0.2)
+    w = dict(f32)
+    w.update(norms)
+    w["final_norm"] = np.linspace(0.5, 1.5, 32).astype(F32)
+    return cfg, w
+
+
+def _logits(cfg, w, toks):
+    dec = decoder.OracleDecoder(cfg, w, batch=1, max_len=8)
+    return dec.forward(toks, 0)["logits"][0].astype(np.float64)
+
+
+def test_decoder_closed_form_with_zero_post_norms():
+    """With the post-attention and post-FFN norm multipliers zero, a sublayer's output cannot reach
+    the residual stream whatever its weights (it enters only through those norms and the residual
+    adds), so the residual stream stays at the scaled embedding row.  For a row c * s (s_j = +-1)
+    the logits are then the closed form
+        logits_v = sum_j E_vj * bf16(s_j * kappa * f_j),  kappa = c S / sqrt(c^2 S^2 + eps),
+    S = fl32(sqrt(H)) the embedding scale and f the final norm's multiplier.  c^2 H is chosen
+    comparable to eps, where dropping the embedding scale moves kappa from 0.81 to 0.24."""
+    cfg, w = _composition_decoder()
+    H, eps = cfg.hidden, cfg.eps
+    c = 2.0 ** -12
+    signs = np.where(np.random.default_rng(12).random((2, H)) < 0.5, -1.0, 1.0)
+    w["embed"] = w["embed"].copy()
+    w["embed"][[3, 7]] = (c * signs).astype(F32)  # exactly representable in bf16
+    w["ln_post_attn"] = [np.zeros(H, F32)]
+    w["ln_post_ffn"] = [np.zeros(H, F32)]
+    got = _logits(cfg, w, np.array([[3, 7]]))
+    S = float(F32(math.sqrt(H)))
+    kappa = c * S / math.sqrt(c * c * S * S + eps)
+    assert 0.8 < kappa < 0.82 and abs(c / math.sqrt(c * c + eps) - 0.24) < 0.01
+    fin = W.round_to_bf16((signs * kappa * w["final_norm"].astype(np.float64)).astype(F32))
+    want = fin.astype(np.float64) @ w["embed"].astype(np.float64).T
+    assert np.allclose(got, want, rtol=1e-6, atol=1e-7)
+
+
+def test_decoder_sublayers_enter_through_their_post_norms():
+    """Each sublayer's output passes an RMSNorm before the residual add (the sandwich norms), and q
+    and k are RMS-normalised before the scores.  Scaling the value rows of W_qkv, W_o, W_up or
+    W_down by 4 scales that sublayer's output by exactly 4 (bf16 rounding commutes with powers of
+    two), and scaling the query or key rows by 2 leaves the normalised q and k unchanged, so the
+    logits move only through eps; doubling a post-norm multiplier or the gate rows does move them.
+    A composition that skipped a post-norm, normed the residual sum or left out the QK-norm fails."""
+    cfg, w = _composition_decoder()
+    toks = np.array([[5, 9, 33, 2]])
+    base = _logits(cfg, w, toks)
+    qd, kd = cfg.q_dim, cfg.kv_dim
+    rows = {"q": slice(0, qd), "k": slice(qd, qd + kd), "v": slice(qd + kd, qd + 2 * kd)}
+
+    def scaled(name, factor, part=None):
+        v = {k: (list(x) if isinstance(x, list) else x) for k, x in w.items()}
+        m = v[name][0].copy()
+        if part is None:
+            m = m * F32(factor)
+        else:
+            m[rows[part]] = m[rows[part]] * F32(factor)
+        v[name] = [m]
+        return _logits(cfg, v, toks)
+
+    scale = np.abs(base).max()
+    for name, factor, part in (("wqkv", 4, "v"), ("wo", 4, None), ("wu", 4, None), ("wd", 4, None),
+                               ("wqkv", 2, "q"), ("wqkv", 2, "k")):
+        assert np.abs(scaled(name, factor, part) - base).max() < 1e-3 * scale, (name, part)
+    for name, factor in (("ln_post_attn", 2), ("ln_post_ffn", 2), ("wg", 2)):
+        assert np.abs(scaled(name, factor) - base).max() > 0.05 * scale, name
