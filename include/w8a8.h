@@ -168,10 +168,16 @@ w8a8_status w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const f
  *   - Every call on a device shares the one array and clears its counter region with a
  *     cudaMemsetAsync on `stream` before launching, so calls whose execution overlaps on the GPU
  *     (different streams, or concurrent host threads) race and give undefined results; serialise
- *     them.  Device-side timeouts are not reported by this entry point. */
+ *     them.
+ *   - A bounded device-side wait that gives up sets the array's error word, which the next calls
+ *     leave set; w8a8_linear_noalloc_check reports it. */
 size_t w8a8_linear_noalloc_capacity(void);
 w8a8_status w8a8_linear_noalloc(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias,
                                 uint16_t* Y, void* stream);
+/* w8a8_workspace_check for the built-in scratch array of the current device: waits for `stream`,
+ * then reads and clears the array's device error word.  W8A8_ERR_TIMEOUT if a wait gave up in a
+ * w8a8_linear_noalloc call since the last check (their outputs are then undefined).  Synchronous. */
+w8a8_status w8a8_linear_noalloc_check(void* stream);
 
 /* bf16 pass-through linear of a layer outside the INT8 set (FFN section: such layers keep the
  * original precision): Y = bf16(sum_j x_tj * w_ij (fp32 accumulation) + bias_i).

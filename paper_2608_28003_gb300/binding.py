@@ -116,6 +116,7 @@ SIGNATURES = {
     "w8a8_linear": (_i32, [ctypes.POINTER(QWeightC), _vp, _i32, _vp, _vp, ctypes.POINTER(DebugC), _vp, _sz, _vp]),
     "w8a8_linear_noalloc_capacity": (_sz, []),
     "w8a8_linear_noalloc": (_i32, [ctypes.POINTER(QWeightC), _vp, _i32, _vp, _vp, _vp]),
+    "w8a8_linear_noalloc_check": (_i32, [_vp]),
     "w8a8_linear_bf16_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
     "w8a8_linear_bf16": (_i32, [_vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "w8a8_ffn_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),

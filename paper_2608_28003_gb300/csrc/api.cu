@@ -263,7 +263,7 @@ w8a8_status run_bf16_linear(const uint16_t* W, int N, int K, const uint16_t* X, 
 }
 
 // Internal: the W8A8 linear with its scratch at `scratch` (used by the no-allocation entry point).
-size_t linear_scratch_bytes(int M, int N, int K) { return linear_ws(M, N, K, true, device_sms()).total; }
+size_t linear_scratch_bytes(int M, int N, int K, int sms) { return linear_ws(M, N, K, true, sms).total; }
 
 w8a8_status linear_on_scratch(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, uint16_t* Y,
                               void* scratch, size_t scratch_bytes, cudaStream_t st) {

@@ -9,10 +9,11 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "ops.cuh"
 
 namespace w8a8 {
 
-size_t linear_scratch_bytes(int M, int N, int K);
+size_t linear_scratch_bytes(int M, int N, int K, int sms);
 w8a8_status linear_on_scratch(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, uint16_t* Y,
                               void* scratch, size_t scratch_bytes, cudaStream_t st);
 w8a8_status check_linear_args(const char* who, const w8a8_qweight* w, const uint16_t* X, int M, const float* bias,
@@ -57,17 +58,29 @@ extern "C" w8a8_status w8a8_linear_noalloc(const w8a8_qweight* w, const uint16_t
                                            uint16_t* Y, void* stream) {
   W8A8_TRY(check_linear_args("w8a8_linear_noalloc", w, X, M, bias, Y));
   if (M == 0) return W8A8_OK;
-  const size_t need = linear_scratch_bytes(M, w->n, w->k);
+  DevInfo d;
+  W8A8_TRY(dev_info(&d));  // an unsupported device is reported as such, before any sizing
+  const size_t need = linear_scratch_bytes(M, w->n, w->k, d.sms);
   W8A8_CHECK_ARG(need <= kNoAllocScratchBytes, W8A8_ERR_SHAPE,
                  "w8a8_linear_noalloc: M=%d, N=%d, K=%d needs %zu bytes of scratch; the built-in array holds %zu "
                  "(use w8a8_linear with a workspace)",
                  M, w->n, w->k, need, kNoAllocScratchBytes);
-  W8A8_TRY(check_device());
   void* scratch = nullptr;
   W8A8_TRY(scratch_for_current_device(&scratch));
   cudaStream_t st = as_stream(stream);
   // The counters and top-1 keys at the start of the scratch must be zero when a call begins; the
-  // array keeps whatever the previous call left, so clear them on every call (no allocation).
-  W8A8_CUDA(cudaMemsetAsync(scratch, 0, W8A8_WS_RESERVED, st));
+  // array keeps whatever the previous call left, so clear them on every call (no allocation).  The
+  // device error word between them is left alone: it stays set until w8a8_linear_noalloc_check
+  // reads it, as a workspace's word stays set until w8a8_workspace_check.
+  char* base = static_cast<char*>(scratch);
+  W8A8_CUDA(cudaMemsetAsync(base, 0, kErrWordOffset, st));
+  W8A8_CUDA(cudaMemsetAsync(base + kErrWordOffset + 16, 0, W8A8_WS_RESERVED - kErrWordOffset - 16, st));
   return linear_on_scratch(w, X, M, bias, Y, scratch, kNoAllocScratchBytes, st);
+}
+
+extern "C" w8a8_status w8a8_linear_noalloc_check(void* stream) {
+  W8A8_TRY(check_device());
+  void* scratch = nullptr;
+  W8A8_TRY(scratch_for_current_device(&scratch));
+  return w8a8_workspace_check(scratch, stream);
 }

@@ -34,7 +34,7 @@ def f32_of_bf16(t):
 
 @pytest.fixture(scope="module")
 def ffn(B):
-    c = synth.ffn_case(64, seed=0)
+    c = synth.ffn_case(2048, seed=0)  # rows 0..M-1 of this draw are the M-token inputs
     stat_in = OW.act_absmax(c["calib32"])
     # fp16 code copies too: 64 tokens take the tensor-core GEMM
     gu = B.prepare_gate_up(cu(c["wg"]), cu(c["wu"]), cu(torch.from_numpy(stat_in)), want_f16=True)
@@ -54,20 +54,54 @@ def test_ffn_w8a8_bit_exact(B, ffn, M):
     assert np.array_equal(f32_of_bf16(Y), r["y"])
 
 
+def _sample_rows(M):
+    """Rows on tile and pair-tile boundaries (128 / 256 tokens), the ragged tail and a few drawn at
+    random: the FFN is row-independent (per-token scales), so the oracle computes just these."""
+    idx = {0, 1, 127, 128, 255, 256, M // 2, M - 2, M - 1}
+    idx |= set(np.random.default_rng(M).integers(0, M, 7).tolist())
+    return np.array(sorted(i for i in idx if 0 <= i < M))
+
+
+@pytest.mark.parametrize("M", [300, 512, 2048])
+def test_ffn_w8a8_large_m_sampled_bit_exact(B, ffn, M):
+    """Prefill sizes: gate/up on the CTA-pair tensor-core GEMM with the GeGLU epilogue (16-column
+    gate/up blocks, swizzled staging, TMA stores of half-width rows), down on the tensor-core GEMM;
+    h and Y of sampled rows bit-exact, every column."""
+    c, f, prep = ffn
+    Y, h = B.ffn_block(f, B.W8A8_PREC_W8A8, cu(c["x"][:M]), want_h=True)
+    idx = _sample_rows(M)
+    r = OB.ffn_w8a8(c["x32"][idx], prep)
+    assert np.array_equal(f32_of_bf16(h)[idx], r["h"])
+    assert np.array_equal(f32_of_bf16(Y)[idx], r["y"])
+
+
+def _bf16_ffn_check(c, h, Y, rows):
+    """h within a few ulps of the oracle's; Y within 1 ulp + the fp32 bound of the oracle's down
+    projection fed the GPU's own h."""
+    r = OB.ffn_bf16(c["x32"][rows], c["wg32"], c["wu32"], c["wd32"])
+    hg, hr = f32_of_bf16(h)[rows], r["h"]
+    scale = np.maximum(np.abs(hr), 1e-3)
+    assert np.max(np.abs(hg - hr) / scale) < 2 ** -6
+    yref = OW.bf16_linear(hg, c["wd32"], out="bf16")
+    mag = np.abs(hg).astype(np.float64) @ np.abs(c["wd32"]).astype(np.float64).T
+    ulp = np.spacing(np.abs(yref).astype(np.float32)) * 2 ** 16
+    assert np.all(np.abs(f32_of_bf16(Y)[rows] - yref) <= ulp + 6912 * 2.0 ** -24 * mag)
+
+
+@pytest.mark.parametrize("M", [300, 512, 2048])
+def test_ffn_bf16_large_m_sampled(B, ffn, M):
+    c, f, _ = ffn
+    Y, h = B.ffn_block(f, B.W8A8_PREC_BF16, cu(c["x"][:M]), want_h=True)
+    _bf16_ffn_check(c, h, Y, _sample_rows(M))
+
+
 @pytest.mark.parametrize("M", [1, 5, 8, 64])
 def test_ffn_bf16_within_tolerance(B, ffn, M):
     c, f, _ = ffn
     Y, h = B.ffn_block(f, B.W8A8_PREC_BF16, cu(c["x"][:M]), want_h=True)
-    r = OB.ffn_bf16(c["x32"][:M], c["wg32"], c["wu32"], c["wd32"])
-    # h: g and u carry fp32 accumulation error before the activation; compare within a few ulps
-    hg, hr = f32_of_bf16(h), r["h"]
-    scale = np.maximum(np.abs(hr), 1e-3)
-    assert np.max(np.abs(hg - hr) / scale) < 2 ** -6
-    # down consumes the GPU's own h; check it against the oracle fed the same h
-    yref = OW.bf16_linear(hg, c["wd32"], out="bf16")
-    mag = np.abs(hg).astype(np.float64) @ np.abs(c["wd32"]).astype(np.float64).T
-    ulp = np.spacing(np.abs(yref).astype(np.float32)) * 2 ** 16
-    assert np.all(np.abs(f32_of_bf16(Y) - yref) <= ulp + 6912 * 2.0 ** -24 * mag)
+    # h: g and u carry fp32 accumulation error before the activation (a few ulps); down consumes
+    # the GPU's own h and is checked against the oracle fed the same h
+    _bf16_ffn_check(c, h, Y, np.arange(M))
 
 
 @pytest.fixture(scope="module")

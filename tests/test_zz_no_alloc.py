@@ -36,6 +36,9 @@ def _call_noalloc(B, q, x):
                                          ctypes.c_void_p(y.data_ptr()),
                                          ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     assert status == 0, B.lib().w8a8_last_error()
+    # no bounded wait gave up during the call
+    status = B.lib().w8a8_linear_noalloc_check(ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert status == 0, B.lib().w8a8_last_error()
     return y
 
 
