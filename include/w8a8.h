@@ -209,6 +209,59 @@ w8a8_status w8a8_ffn_block(const w8a8_ffn_weights* ffn, int precision, const uin
                            uint16_t* Y, uint16_t* h_dbg, void* workspace, size_t ws_bytes,
                            void* stream);
 
+/* ------------------------------------------------------------------ FP8 (e4m3) variant
+ * The paper's Future Work moves from INT8 to FP8 on Blackwell; it gives no scheme, so this variant
+ * keeps the INT8 path's SmoothQuant structure (Eq. delta-attn / delta-lmhead, what-lmhead,
+ * xhat-lmhead) and replaces the integer grid by e4m3 (1 sign, 4 exponent bits with bias 7, 3
+ * mantissa bits, subnormals down to 2^-9, largest value 448):
+ *   s_w_i = fl32(m_i / 448), wq_ij = e4m3(fl32(W_hat_ij * fl32(448 / m_i)))   (m_i = max_j |W_hat_ij|)
+ *   s_x_t = fl32(m_t / 448), xq_tj = e4m3(fl32(x_hat_tj * fl32(448 / m_t)))   (m_t = max_j |x_hat_tj|)
+ *   acc_ti = sum_j xq_tj * wq_ij in fp32 (every product exact; the sum's rounding depends on the
+ *            kernel's order: not bit-exact, within K * 2^-23 * sum_j |xq_tj wq_ij|)
+ *   y_ti   = fl32(fl32(s_x_t * s_w_i) * acc_ti), then + bias_i, then bf16 (RNE)
+ * e4m3(v): nearest e4m3 value, ties to even, saturating at +-448; an all-zero row or token has scale
+ * 0 and codes 0.  Codes are stored as bytes (sign | exponent | mantissa).
+ *   wq [n, k] e4m3 codes; s_w [n]; inv_delta [k] = fl32(1 / delta) as for INT8. */
+typedef struct {
+  int32_t n, k;
+  const uint8_t* wq;
+  const float* s_w;
+  const float* inv_delta;
+} w8a8_fp8_weight;
+
+/* Preparation of one linear (w8a8_prepare_weights with the e4m3 rule above), and of the fused
+ * gate/up pair with the 8-row interleave of w8a8_prepare_gate_up.  Outputs (caller-owned):
+ * wq [N, K] (or [2F, H]) codes, s_w, delta, inv_delta. */
+w8a8_status w8a8_fp8_prepare_weights(const uint16_t* W, int N, int K, const float* act_absmax, float alpha,
+                                     int smooth, uint8_t* wq, float* s_w, float* delta, float* inv_delta,
+                                     void* stream);
+w8a8_status w8a8_fp8_prepare_gate_up(const uint16_t* W_gate, const uint16_t* W_up, int F, int H,
+                                     const float* act_absmax, float alpha, int smooth, uint8_t* wq,
+                                     float* s_w, float* delta, float* inv_delta, void* stream);
+
+/* Per-token e4m3 quantisation of the smoothed input: X [M, K] bf16 -> xq [M, K] codes, s_x [M]. */
+w8a8_status w8a8_fp8_quantize_activations(const uint16_t* X, int M, int K, const float* inv_delta,
+                                          uint8_t* xq, float* s_x, void* stream);
+
+/* Y [M, N] bf16 = FP8 linear of X [M, K] bf16 (rule above).  N and K multiples of 16.
+ * xq_dbg [M, K] and s_x_dbg [M] (nullable) receive the activation codes and scales.  The workspace
+ * is sized by w8a8_linear_workspace_size. */
+w8a8_status w8a8_fp8_linear(const w8a8_fp8_weight* w, const uint16_t* X, int M, const float* bias,
+                            uint16_t* Y, uint8_t* xq_dbg, float* s_x_dbg, void* workspace, size_t ws_bytes,
+                            void* stream);
+
+/* The FFN block of w8a8_ffn_block with both linears in FP8: [g | u] = FP8 gate/up linear of X (fp32
+ * out of the epilogue), h = bf16(gelu_tanh(g) * u) (the same fp32 recipe), Y = FP8 down linear of h.
+ * The workspace is sized by w8a8_ffn_workspace_size; h_dbg [M, F] (nullable) receives h. */
+typedef struct {
+  int32_t hidden, inter;
+  w8a8_fp8_weight gate_up; /* n = 2*inter, k = hidden, 8-row interleave */
+  w8a8_fp8_weight down;    /* n = hidden, k = inter */
+} w8a8_fp8_ffn_weights;
+
+w8a8_status w8a8_fp8_ffn_block(const w8a8_fp8_ffn_weights* ffn, const uint16_t* X, int M, uint16_t* Y,
+                               uint16_t* h_dbg, void* workspace, size_t ws_bytes, void* stream);
+
 /* --------------------------------------------------------------------------- lm_head
  * Logits over the tied [V, d] table (LM Head section) and the top-1 index.
  *   W8A8: logits_tv = fl32(fl32(s_x_t * s_w_v) * fl32(acc_tv)) (fp32, not rounded further).

@@ -9,11 +9,16 @@ original precision").
 
 lm_head (LM Head section): logits = W8A8 linear of the final-norm hidden state with the tied
 [V, d] table, kept in fp32, and the top-1 index (ties to the lowest index).
+
+FP8 block (Future Work: e4m3 in place of INT8; the reading of oracle/fp8.py): the same block with
+both linears in the e4m3 variant, g and u in fp32 out of its epilogue, h rounded to bf16.  Parity
+against the paper unpinned (it prints no FP8 numbers).
 """
 from __future__ import annotations
 
 import numpy as np
 
+from . import fp8 as _fp8
 from . import geglu as _geglu
 from . import w8a8 as _w
 
@@ -62,3 +67,24 @@ def lm_head_bf16(X, W) -> dict:
     """bf16 pass-through lm_head: fp32 logits (fp64 sums rounded once) and top-1."""
     logits = _w.bf16_linear(X, W, out="f32")
     return {"logits": logits, "top1": _w.top1(logits)}
+
+
+def prepare_ffn_fp8(w_gate, w_up, w_down, stat_in, stat_h, alpha: float = 0.5, smooth: bool = True):
+    """prepare_ffn with the e4m3 rule: one delta over the fused [gate; up] rows, then e4m3 codes."""
+    gu = np.concatenate([np.asarray(w_gate, np.float32), np.asarray(w_up, np.float32)], axis=0)
+    return {
+        "F": int(np.asarray(w_gate).shape[0]),
+        "gu": _fp8.prepare_weights_fp8(gu, stat_in, alpha, smooth),
+        "down": _fp8.prepare_weights_fp8(w_down, stat_h, alpha, smooth),
+    }
+
+
+def ffn_fp8(X, prep) -> dict:
+    """FP8 FFN block: g, u (fp32) from the e4m3 gate/up linear, h = bf16(geglu(g, u)), y from the
+    e4m3 down linear (bf16)."""
+    F = prep["F"]
+    gu = _fp8.fp8_linear(X, prep["gu"], out="f32")
+    g, u = gu["y"][:, :F], gu["y"][:, F:]
+    h = _w.round_to_bf16(_geglu.geglu_f32(g, u))
+    dn = _fp8.fp8_linear(h, prep["down"], out="bf16")
+    return {"gu": gu, "g": g, "u": u, "h": h, "down": dn, "y": dn["y"]}

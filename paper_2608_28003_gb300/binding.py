@@ -51,6 +51,14 @@ class FfnC(ctypes.Structure):
                 ("gate_up_bf16", _vp), ("down_bf16", _vp)]
 
 
+class Fp8WeightC(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int32), ("k", ctypes.c_int32), ("wq", _vp), ("s_w", _vp), ("inv_delta", _vp)]
+
+
+class Fp8FfnC(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_int32), ("inter", ctypes.c_int32), ("gate_up", Fp8WeightC), ("down", Fp8WeightC)]
+
+
 class HeadC(ctypes.Structure):
     _fields_ = [("vocab", ctypes.c_int32), ("hidden", ctypes.c_int32), ("q", QWeightC), ("bf16", _vp)]
 
@@ -121,6 +129,11 @@ SIGNATURES = {
     "w8a8_linear_bf16": (_i32, [_vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "w8a8_ffn_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
     "w8a8_ffn_block": (_i32, [ctypes.POINTER(FfnC), _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+    "w8a8_fp8_prepare_weights": (_i32, [_vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp]),
+    "w8a8_fp8_prepare_gate_up": (_i32, [_vp, _vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp]),
+    "w8a8_fp8_quantize_activations": (_i32, [_vp, _i32, _i32, _vp, _vp, _vp, _vp]),
+    "w8a8_fp8_linear": (_i32, [ctypes.POINTER(Fp8WeightC), _vp, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "w8a8_fp8_ffn_block": (_i32, [ctypes.POINTER(Fp8FfnC), _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "w8a8_lm_head_workspace_size": (_i32, [_i32, _i32, _i32, ctypes.POINTER(_sz)]),
     "w8a8_lm_head": (_i32, [ctypes.POINTER(HeadC), _i32, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "w8a8_model_create": (_i32, [ctypes.POINTER(ModelCfgC), ctypes.POINTER(LayerBf16C), _vp, _vp,
@@ -384,6 +397,98 @@ def ffn_block(f: FfnWeights, precision: int, X: torch.Tensor, want_h: bool = Fal
     fc = f.c()
     _check("w8a8_ffn_block", lib().w8a8_ffn_block(ctypes.byref(fc), int(precision), _p(_bits(X)), M, _p(Y), _p(h),
                                                   _p(buf), buf.numel(), _stream(stream)))
+    return (Y, h) if want_h else Y
+
+
+# ------------------------------------------------------------------------ FP8 (e4m3) variant
+@dataclass
+class Fp8Weight:
+    """A prepared FP8 weight: e4m3 codes (uint8 bytes), per-channel scales, smoothing factors."""
+    wq: torch.Tensor
+    s_w: torch.Tensor
+    delta: torch.Tensor
+    inv_delta: torch.Tensor
+
+    @property
+    def n(self):
+        return self.wq.shape[0]
+
+    @property
+    def k(self):
+        return self.wq.shape[1]
+
+    def c(self) -> Fp8WeightC:
+        return Fp8WeightC(self.n, self.k, self.wq.data_ptr(), self.s_w.data_ptr(), self.inv_delta.data_ptr())
+
+
+def _fp8_weight(rows: int, K: int, dev) -> Fp8Weight:
+    return Fp8Weight(torch.empty(rows, K, dtype=torch.uint8, device=dev),
+                     torch.empty(rows, dtype=torch.float32, device=dev),
+                     torch.empty(K, dtype=torch.float32, device=dev), torch.empty(K, dtype=torch.float32, device=dev))
+
+
+def fp8_prepare_weights(W: torch.Tensor, act_stat: Optional[torch.Tensor], alpha: float = 0.5, smooth: bool = True,
+                        stream=None) -> Fp8Weight:
+    N, K = W.shape
+    q = _fp8_weight(N, K, W.device)
+    _check("w8a8_fp8_prepare_weights", lib().w8a8_fp8_prepare_weights(
+        _p(_bits(W)), N, K, _p(act_stat), float(alpha), int(smooth), _p(q.wq), _p(q.s_w), _p(q.delta),
+        _p(q.inv_delta), _stream(stream)))
+    return q
+
+
+def fp8_prepare_gate_up(W_gate: torch.Tensor, W_up: torch.Tensor, act_stat: Optional[torch.Tensor],
+                        alpha: float = 0.5, smooth: bool = True, stream=None) -> Fp8Weight:
+    F, H = W_gate.shape
+    q = _fp8_weight(2 * F, H, W_gate.device)
+    _check("w8a8_fp8_prepare_gate_up", lib().w8a8_fp8_prepare_gate_up(
+        _p(_bits(W_gate)), _p(_bits(W_up)), F, H, _p(act_stat), float(alpha), int(smooth), _p(q.wq), _p(q.s_w),
+        _p(q.delta), _p(q.inv_delta), _stream(stream)))
+    return q
+
+
+def fp8_quantize_activations(X: torch.Tensor, inv_delta: torch.Tensor, stream=None):
+    M, K = X.shape
+    xq = torch.empty(M, K, dtype=torch.uint8, device=X.device)
+    s_x = torch.empty(M, dtype=torch.float32, device=X.device)
+    _check("w8a8_fp8_quantize_activations", lib().w8a8_fp8_quantize_activations(
+        _p(_bits(X)), M, K, _p(inv_delta), _p(xq), _p(s_x), _stream(stream)))
+    return xq, s_x
+
+
+def fp8_linear(w: Fp8Weight, X: torch.Tensor, bias: Optional[torch.Tensor] = None, debug: bool = False,
+               out: Optional[torch.Tensor] = None, ws: Optional[Workspace] = None, stream=None):
+    M = X.shape[0]
+    Y = out if out is not None else torch.empty(M, w.n, dtype=torch.bfloat16, device=X.device)
+    buf = (ws or default_workspace()).get(_size("w8a8_linear_workspace_size", M, w.n, w.k))
+    xq = torch.empty(M, w.k, dtype=torch.uint8, device=X.device) if debug else None
+    s_x = torch.empty(M, dtype=torch.float32, device=X.device) if debug else None
+    wc = w.c()
+    _check("w8a8_fp8_linear", lib().w8a8_fp8_linear(ctypes.byref(wc), _p(_bits(X)), M, _p(bias), _p(Y), _p(xq),
+                                                    _p(s_x), _p(buf), buf.numel(), _stream(stream)))
+    return (Y, {"xq": xq, "s_x": s_x}) if debug else Y
+
+
+@dataclass
+class Fp8FfnWeights:
+    hidden: int
+    inter: int
+    gate_up: Fp8Weight
+    down: Fp8Weight
+
+    def c(self) -> Fp8FfnC:
+        return Fp8FfnC(self.hidden, self.inter, self.gate_up.c(), self.down.c())
+
+
+def fp8_ffn_block(f: Fp8FfnWeights, X: torch.Tensor, want_h: bool = False, out: Optional[torch.Tensor] = None,
+                  ws: Optional[Workspace] = None, stream=None):
+    M = X.shape[0]
+    Y = out if out is not None else torch.empty(M, f.hidden, dtype=torch.bfloat16, device=X.device)
+    h = torch.empty(M, f.inter, dtype=torch.bfloat16, device=X.device) if want_h else None
+    buf = (ws or default_workspace()).get(_size("w8a8_ffn_workspace_size", M, f.hidden, f.inter))
+    fc = f.c()
+    _check("w8a8_fp8_ffn_block", lib().w8a8_fp8_ffn_block(ctypes.byref(fc), _p(_bits(X)), M, _p(Y), _p(h), _p(buf),
+                                                          buf.numel(), _stream(stream)))
     return (Y, h) if want_h else Y
 
 

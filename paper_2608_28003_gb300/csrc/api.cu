@@ -190,7 +190,7 @@ static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N,
   a.err = r.err;
   a.partials = part;
   a.tile_counters = r.tile_counters;
-  *status = launch_tc_gemm(int8, a, st);
+  *status = launch_tc_gemm(int8 ? TC_I8 : TC_BF16, a, st);
   return true;
 }
 

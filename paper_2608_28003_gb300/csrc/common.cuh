@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
 #include <cuda_bf16.h>
+#include <cuda_fp8.h>
 #include <stdint.h>
 #include <stddef.h>
 
@@ -103,6 +104,18 @@ __device__ __forceinline__ void i8x4_to_f16x2x2(uint32_t w, uint32_t& lo, uint32
   __half2 b = __hsub2(*reinterpret_cast<const __half2*>(&phi), bias);
   lo = *reinterpret_cast<uint32_t*>(&a);
   hi = *reinterpret_cast<uint32_t*>(&b);
+}
+
+// Two fp32 values -> two e4m3 codes (lo in the low byte): round to nearest even, saturating at
+// +-448 (the hardware conversion with .satfinite).
+__device__ __forceinline__ uint32_t e4m3x2_of(float lo, float hi) {
+  return (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(lo, hi), __NV_SATFINITE, __NV_E4M3);
+}
+// Two e4m3 codes (low byte first) -> their values as an fp16 pair, low half first (exact: every
+// e4m3 value is an fp16 value).
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t codes16) {
+  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(codes16 & 0xFFFFu), __NV_E4M3);
+  return (uint32_t)h.x | ((uint32_t)h.y << 16);
 }
 
 // ------------------------------------------------------------------------- legacy MMA

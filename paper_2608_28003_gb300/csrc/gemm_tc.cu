@@ -19,6 +19,11 @@
 //    into INT32 registers, and the INT32 result is exact in any order (Eq. gemm-final).  The
 //    epilogue then dequantises fl(fl(s_x s_w) acc) (+ bias).
 //  * bf16 path: one accumulator per tile over the whole k range.
+//  * FP8 path (the e4m3 variant of the W8A8 linear): both operands are e4m3 codes, one byte each;
+//    tcgen05.mma kind::f8f6f4 (K = 32 per instruction) reads the same 128-byte swizzled rows, so a
+//    stage carries 128 k in the bytes a fp16 stage uses for 64, and the fp32 accumulator runs over
+//    the whole k range (fp32 sums of e4m3 products are not exact; no fold) before the epilogue
+//    dequantises fl(fl(s_x s_w) acc).
 //  * epilogues: bf16 output, GeGLU of interleaved gate/up columns (16-column blocks: 8 gate, then
 //    the 8 matching up channels), or fp32 logits with the top-1 index (keys reduced with atomicMax,
 //    the last CTA to finish decodes them); outputs leave through 32 x 32 shared-memory blocks and
@@ -39,6 +44,11 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kSwz = 128;                // swizzle span in bytes (TMA and the MMA descriptors agree)
 constexpr int kBK = kSwz / 2;            // k per stage: one swizzle span of fp16 per row
+// operand modes: bf16 pass-through, INT8 codes carried as fp16 (exact, folded), e4m3 codes
+constexpr int kModeBf16 = TC_BF16, kModeI8 = TC_I8, kModeFp8 = TC_FP8;
+// k elements per stage: one 128-byte swizzle span per row (64 two-byte or 128 one-byte elements)
+__host__ __device__ constexpr int bk_elems(int mode) { return mode == kModeFp8 ? kSwz : kSwz / 2; }
+__host__ __device__ constexpr int elem_bytes(int mode) { return mode == kModeFp8 ? 1 : 2; }
 constexpr int kKbPerChunk = 1024 / kBK;  // stages per exact fp32 chunk of 1024 k
 constexpr int kEpiWarps = 16;                   // four per TMEM lane quarter: one per column quarter
 constexpr int kParts = kEpiWarps / 4;
@@ -59,7 +69,7 @@ __host__ __device__ constexpr int a_box_rows(int M) { return M < kBM ? (M + 7) /
 // starts on a 128-column boundary.
 __host__ __device__ constexpr int slot_cols(int bn) { return bn <= 128 ? 128 : bn <= 256 ? 256 : 512; }
 
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 struct TcGeo {
   static constexpr int BN = kBN;
   static constexpr uint32_t BBytes = BN * kBK * 2;
@@ -84,7 +94,8 @@ __device__ __forceinline__ uint64_t sdesc_swz(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor of kind::f16: fp32 accumulator, A/B fp16 (0) or bf16 (1), both K-major,
+// Instruction descriptor of kind::f16 / kind::f8f6f4: fp32 accumulator (bits 4-5 = 1), A and B
+// format at bits 7-9 and 10-12 (kind::f16: fp16 0, bf16 1; kind::f8f6f4: e4m3 0), both K-major,
 // N >> 3 at bit 17, M >> 4 at bit 24.
 __host__ __device__ constexpr uint32_t idesc_f16(uint32_t ab_format, int n, int m) {
   return (1u << 4) | (ab_format << 7) | (ab_format << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
@@ -97,6 +108,22 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+__device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+template <int kMode>
+__device__ __forceinline__ void tc_mma_m(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  if constexpr (kMode == kModeFp8)
+    tc_mma_f8(d_tmem, a_desc, b_desc, idesc, accumulate);
+  else
+    tc_mma(d_tmem, a_desc, b_desc, idesc, accumulate);
 }
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar) : "memory");
@@ -220,7 +247,7 @@ __device__ __forceinline__ void stage_cols32(const TcArgs& a, const CUtensorMap*
 // The last unit of a split tile: the 512 epilogue threads sum the tile's KS partials (units u0 ..
 // u0 + KS - 1) in part order, four columns per thread with every part's load in flight, and write
 // the bf16 outputs (W8A8: the INT32 sums dequantised exactly as the tile epilogue does it).
-template <bool kInt8, int BN>
+template <int kMode, int BN>
 __device__ __forceinline__ void split_reduce(const TcArgs& a, int u0, int KS, int R, int m0, int n0) {
   const uint4* part = reinterpret_cast<const uint4*>(a.partials) + (size_t)u0 * R * (BN / 4);
   const size_t pstride = (size_t)R * (BN / 4);
@@ -230,7 +257,7 @@ __device__ __forceinline__ void split_reduce(const TcArgs& a, int u0, int KS, in
     if (row >= a.M || col >= a.N) continue;  // N is a multiple of 16: four columns are all in or out
     const uint4* p = part + e;
     float y[4];
-    if constexpr (kInt8) {
+    if constexpr (kMode == kModeI8) {
       int s[4] = {0, 0, 0, 0};
 #pragma unroll 8
       for (int sp = 0; sp < KS; ++sp) {
@@ -255,6 +282,11 @@ __device__ __forceinline__ void split_reduce(const TcArgs& a, int u0, int KS, in
         y[2] = __fadd_rn(y[2], __uint_as_float(v.z));
         y[3] = __fadd_rn(y[3], __uint_as_float(v.w));
       }
+      if constexpr (kMode == kModeFp8) {  // the fp32 sum of all parts, dequantised
+        const float sx = a.s_x[row];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] = __fmul_rn(__fmul_rn(sx, a.s_w[col + k]), y[k]);
+      }
     }
     if (a.bias) {
 #pragma unroll
@@ -264,11 +296,13 @@ __device__ __forceinline__ void split_reduce(const TcArgs& a, int u0, int KS, in
   }
 }
 
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmY, const TcArgs a) {
-  using GG = TcGeo<kInt8, kBN>;
+  using GG = TcGeo<kMode, kBN>;
+  constexpr bool kInt8 = kMode == kModeI8, kFp8 = kMode == kModeFp8;
+  constexpr int BKe = bk_elems(kMode);
   constexpr int BN = GG::BN, S = GG::S;
   constexpr int SC = slot_cols(BN), NSLOT = (int)kTmemCols / SC;  // accumulator slots in tensor memory
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -281,7 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sA = base, sB = base + (uint32_t)S * kABytes, stg = sB + (uint32_t)S * GG::BBytes;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + kBM - 1) / kBM);
-  const int nkb = (a.K + kBK - 1) / kBK;
+  const int nkb = (a.K + BKe - 1) / BKe;
   // work units: (tile, k part); unit u is part u mod KS of tile u / KS, stages [kb_lo, kb_hi)
   const int KS = a.ksplit > 1 ? a.ksplit : 1, units = tiles * KS;
   auto kb_lo = [&](int u) { return (int)((long long)(u % KS) * nkb / KS); };
@@ -338,9 +372,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           const uint32_t bar = full0 + 8 * s;
-          mbar_arrive_expect_tx(bar, (uint32_t)(a_box_rows(a.M) * kBK * 2) + GG::BBytes);
-          tma_load_2d(sA + (uint32_t)s * kABytes, &tmA, kb * kBK, m0, bar);
-          tma_load_2d(sB + (uint32_t)s * GG::BBytes, &tmB, kb * kBK, n0, bar);
+          mbar_arrive_expect_tx(bar, (uint32_t)(a_box_rows(a.M) * kSwz) + GG::BBytes);
+          tma_load_2d(sA + (uint32_t)s * kABytes, &tmA, kb * BKe, m0, bar);
+          tma_load_2d(sB + (uint32_t)s * GG::BBytes, &tmB, kb * BKe, n0, bar);
         }
       }
       if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
@@ -354,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_f16(kInt8 ? 0u : 1u, BN, kBM);
+      constexpr uint32_t idesc = idesc_f16(kMode == kModeBf16 ? 1u : 0u, BN, kBM);
       bool ok = true;
       int g = 0, q = 0;  // stages consumed, accumulator chunks produced
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
@@ -377,10 +411,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
 #pragma unroll
-            for (int k16 = 0; k16 < kBK / 16; ++k16) {
+            for (int k16 = 0; k16 < kSwz / 32; ++k16) {  // 32 bytes of k per instruction
               const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
               const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BBytes + 32u * k16);
-              tc_mma(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
+              tc_mma_m<kMode>(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
             }
             tc_commit(empty0 + 8 * s);
           }
@@ -470,7 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               store_part32(u, g, reinterpret_cast<const uint32_t(&)[32]>(isum[32 * i]));
             }
           }
-          if (arrive_last()) split_reduce<true, BN>(a, t * KS, KS, R, m0, n0);
+          if (arrive_last()) split_reduce<kModeI8, BN>(a, t * KS, KS, R, m0, n0);
           if (!ok) break;
           continue;
         } else if (!ok) {
@@ -511,10 +545,12 @@ __global__ void __launch_bounds__(kThreads, 1)
               continue;
             }
             float v[32];
+            const float sx = kFp8 && row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
               const int col = n0 + 32 * g + j;
               float y = __uint_as_float(r[j]);
+              if (kFp8) y = col < a.N ? __fmul_rn(__fmul_rn(sx, a.s_w[col]), y) : 0.0f;
               if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
               v[j] = y;
             }
@@ -525,7 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ++q;
         if (KS > 1) {
-          if (arrive_last()) split_reduce<false, BN>(a, t * KS, KS, R, m0, n0);
+          if (arrive_last()) split_reduce<kMode, BN>(a, t * KS, KS, R, m0, n0);
           if (!ok) break;
           continue;
         } else if (!ok) {
@@ -570,7 +606,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // tensor memory receives its 128 rows of D.  CTA 0 of the pair issues the MMAs; both CTAs' TMA
 // copies complete on CTA 0's stage barrier; the stage and accumulator barriers of both CTAs are
 // signalled by multicast commits; both CTAs' epilogue threads hand the slot back to CTA 0.
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 struct Tc2Geo {
   static constexpr int BN = kBN;
   static constexpr uint32_t BHalf = (kBN / 2) * kBK * 2;
@@ -612,6 +648,22 @@ __device__ __forceinline__ void tc2_mma(uint32_t d_tmem, uint64_t a_desc, uint64
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+__device__ __forceinline__ void tc2_mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+template <int kMode>
+__device__ __forceinline__ void tc2_mma_m(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  if constexpr (kMode == kModeFp8)
+    tc2_mma_f8(d_tmem, a_desc, b_desc, idesc, accumulate);
+  else
+    tc2_mma(d_tmem, a_desc, b_desc, idesc, accumulate);
+}
 // arrive on the barrier at this shared-memory offset in both CTAs of the pair once the MMAs issued
 // so far have completed
 __device__ __forceinline__ void tc2_commit_both(uint32_t bar) {
@@ -625,11 +677,13 @@ __device__ __forceinline__ void tc2_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar) : "memory");
 }
 
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmY, const TcArgs a) {
-  using GG = Tc2Geo<kInt8, kBN>;
+  using GG = Tc2Geo<kMode, kBN>;
+  constexpr bool kInt8 = kMode == kModeI8, kFp8 = kMode == kModeFp8;
+  constexpr int BKe = bk_elems(kMode);
   constexpr int BN = GG::BN, S = GG::S;
   constexpr int SC = slot_cols(BN), NSLOT = (int)kTmemCols / SC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -644,7 +698,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t rank = cluster_rank();
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + 2 * kBM - 1) / (2 * kBM));
-  const int nkb = (a.K + kBK - 1) / kBK;
+  const int nkb = (a.K + BKe - 1) / BKe;
   const int nchunks = kInt8 ? (nkb + kKbPerChunk - 1) / kKbPerChunk : 1;
   const int kb_per_chunk = kInt8 ? kKbPerChunk : nkb;
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
@@ -696,8 +750,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             break;
           }
           if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * s, 2 * (kABytes + GG::BHalf));
-          tma_load_2d_pair(sA + (uint32_t)s * kABytes, &tmA, kb * kBK, m0 + kBM * (int)rank, full_lead + 8 * s);
-          tma_load_2d_pair(sB + (uint32_t)s * GG::BHalf, &tmB, kb * kBK, n0 + (BN / 2) * (int)rank, full_lead + 8 * s);
+          tma_load_2d_pair(sA + (uint32_t)s * kABytes, &tmA, kb * BKe, m0 + kBM * (int)rank, full_lead + 8 * s);
+          tma_load_2d_pair(sB + (uint32_t)s * GG::BHalf, &tmB, kb * BKe, n0 + (BN / 2) * (int)rank, full_lead + 8 * s);
         }
       }
       if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
@@ -712,7 +766,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------------- MMA issuer (CTA 0)
     if (lane == 0 && rank == 0) {
-      constexpr uint32_t idesc = idesc_f16(kInt8 ? 0u : 1u, BN, 2 * kBM);
+      constexpr uint32_t idesc = idesc_f16(kMode == kModeBf16 ? 1u : 0u, BN, 2 * kBM);
       bool ok = true;
       int g = 0, q = 0;
       for (int t = pair; t < tiles && ok; t += npairs) {
@@ -734,10 +788,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
 #pragma unroll
-            for (int k16 = 0; k16 < kBK / 16; ++k16) {
+            for (int k16 = 0; k16 < kSwz / 32; ++k16) {  // 32 bytes of k per instruction
               const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
               const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BHalf + 32u * k16);
-              tc2_mma(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
+              tc2_mma_m<kMode>(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
             }
             tc2_commit_both(empty0 + 8 * s);
           }
@@ -821,10 +875,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           uint32_t r[32];
           tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
           float v[32];
+          const float sx = kFp8 && row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             const int col = n0 + 32 * g + j;
             float y = __uint_as_float(r[j]);
+            if (kFp8) y = col < a.N ? __fmul_rn(__fmul_rn(sx, a.s_w[col]), y) : 0.0f;
             if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
             v[j] = y;
           }
@@ -876,46 +932,48 @@ w8a8_status make_out_map(const TcArgs& a, CUtensorMap* ty, const CUtensorMap& un
   return W8A8_OK;
 }
 
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 w8a8_status launch_t(const TcArgs& a, cudaStream_t st) {
-  using GG = TcGeo<kInt8, kBN>;
+  using GG = TcGeo<kMode, kBN>;
+  constexpr int EB = elem_bytes(kMode), BKe = bk_elems(kMode);
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<kInt8, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
+    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<kMode, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
     attr_set[dev] = true;
   }
   CUtensorMap ta, tb;
-  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, (uint32_t)a_box_rows(a.M),
-                        kSwz));
-  W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN, kSwz));
+  W8A8_TRY(make_tmap_2d(&ta, a.A, EB, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * EB, BKe,
+                        (uint32_t)a_box_rows(a.M), kSwz));
+  W8A8_TRY(make_tmap_2d(&tb, a.B, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, BKe, GG::BN, kSwz));
   CUtensorMap ty;
   W8A8_TRY(make_out_map(a, &ty, ta));
   const long long tiles = (long long)((a.N + GG::BN - 1) / GG::BN) * ((a.M + kBM - 1) / kBM);
   const dim3 grid((unsigned)std::min<long long>(tiles * std::max(a.ksplit, 1), device_sms()));
-  W8A8_CUDA(launch_pdl(gemm_tc_kernel<kInt8, kBN>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, ty, a));
+  W8A8_CUDA(launch_pdl(gemm_tc_kernel<kMode, kBN>, grid, dim3(kThreads), (size_t)GG::Smem, st, ta, tb, ty, a));
   return W8A8_OK;
 }
 
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 w8a8_status launch_t2(const TcArgs& a, cudaStream_t st) {
-  using GG = Tc2Geo<kInt8, kBN>;
+  using GG = Tc2Geo<kMode, kBN>;
+  constexpr int EB = elem_bytes(kMode), BKe = bk_elems(kMode);
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc2_kernel<kInt8, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
+    W8A8_CUDA(cudaFuncSetAttribute(gemm_tc2_kernel<kMode, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GG::Smem));
     attr_set[dev] = true;
   }
   CUtensorMap ta, tb;
-  W8A8_TRY(make_tmap_2d(&ta, a.A, 2, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * 2, kBK, kBM, kSwz));
-  W8A8_TRY(make_tmap_2d(&tb, a.B, 2, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * 2, kBK, GG::BN / 2, kSwz));
+  W8A8_TRY(make_tmap_2d(&ta, a.A, EB, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K * EB, BKe, kBM, kSwz));
+  W8A8_TRY(make_tmap_2d(&tb, a.B, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, BKe, GG::BN / 2, kSwz));
   CUtensorMap ty;
   W8A8_TRY(make_out_map(a, &ty, ta));
   const long long tiles = (long long)((a.N + GG::BN - 1) / GG::BN) * ((a.M + 2 * kBM - 1) / (2 * kBM));
   const long long pairs = std::min<long long>(tiles, device_sms() / 2);
-  W8A8_CUDA(launch_pdl(gemm_tc2_kernel<kInt8, kBN>, dim3((unsigned)(2 * pairs)), dim3(kThreads), (size_t)GG::Smem, st,
+  W8A8_CUDA(launch_pdl(gemm_tc2_kernel<kMode, kBN>, dim3((unsigned)(2 * pairs)), dim3(kThreads), (size_t)GG::Smem, st,
                        ta, tb, ty, a));
   return W8A8_OK;
 }
@@ -941,19 +999,19 @@ constexpr int kMinKbPerPart = 2;
 // under the cap) would lose.
 constexpr int kMinParts = 4;
 
-template <bool kInt8, int kBN>
+template <int kMode, int kBN>
 w8a8_status launch_split(TcArgs a, cudaStream_t st) {
-  const int sms = device_sms(), nkb = (a.K + kBK - 1) / kBK;
+  const int sms = device_sms(), nkb = (a.K + bk_elems(kMode) - 1) / bk_elems(kMode);
   const long long tiles = (long long)((a.N + kBN - 1) / kBN) * ((a.M + kBM - 1) / kBM);
   a.ksplit = 1;
   if (a.kind == EPI_BF16 && a.partials && a.tile_counters && 2 * tiles <= sms) {
     const int ks = std::min({(int)(sms / tiles), nkb / kMinKbPerPart, a.K / (4 * a_box_rows(a.M))});
     if (ks >= kMinParts) a.ksplit = ks;
   }
-  return launch_t<kInt8, kBN>(a, st);
+  return launch_t<kMode, kBN>(a, st);
 }
 
-template <bool kInt8>
+template <int kMode>
 w8a8_status dispatch(TcArgs a, cudaStream_t st) {
   a.ksplit = 1;
   const long long pairs = device_sms() / 2;
@@ -963,10 +1021,10 @@ w8a8_status dispatch(TcArgs a, cudaStream_t st) {
   };
   const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
                c128 = cost(kBM, 128, 1.81, 2 * pairs), c64 = cost(kBM, 64, 2.7, 2 * pairs);
-  if (c256 <= c192 && c256 <= c128 && c256 <= c64) return launch_t2<kInt8, 256>(a, st);
-  if (c192 <= c128 && c192 <= c64) return launch_t2<kInt8, 192>(a, st);
-  if (c128 <= c64) return launch_split<kInt8, 128>(a, st);
-  return launch_split<kInt8, 64>(a, st);  // few tokens: spread the weight stream over more SMs
+  if (c256 <= c192 && c256 <= c128 && c256 <= c64) return launch_t2<kMode, 256>(a, st);
+  if (c192 <= c128 && c192 <= c64) return launch_t2<kMode, 192>(a, st);
+  if (c128 <= c64) return launch_split<kMode, 128>(a, st);
+  return launch_split<kMode, 64>(a, st);  // few tokens: spread the weight stream over more SMs
 }
 
 }  // namespace
@@ -983,13 +1041,15 @@ size_t tc_split_partial_bytes(int M, int sms) {
   return (size_t)std::max(sms, 1) * 128 * (size_t)a_box_rows(std::max(M, 1)) * 4;
 }
 
-w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st) {
+w8a8_status launch_tc_gemm(int mode, const TcArgs& a, cudaStream_t st) {
   if (a.M == 0 || a.N == 0) return W8A8_OK;
   void *v0, *v1;
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  const w8a8_status s = int8_codes ? dispatch<true>(a, st) : dispatch<false>(a, st);
+  const w8a8_status s = mode == TC_FP8 ? dispatch<kModeFp8>(a, st)
+                        : mode == TC_I8 ? dispatch<kModeI8>(a, st)
+                                        : dispatch<kModeBf16>(a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }

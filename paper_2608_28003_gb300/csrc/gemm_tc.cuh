@@ -1,18 +1,23 @@
 // Tensor-core GEMM for prefill-sized token counts on the 5th-generation tensor cores (tcgen05):
-// the W8A8 path (INT8 codes carried as fp16, exact) and the bf16 pass-through.
+// the W8A8 path (INT8 codes carried as fp16, exact), the FP8 variant (e4m3 codes) and the bf16
+// pass-through.
 #pragma once
 
 #include "common.cuh"
 
 namespace w8a8 {
 
+// Operand modes: bf16, INT8 codes carried as fp16 (kind::f16, exact INT32 by folding every 1024 k),
+// e4m3 codes (kind::f8f6f4, fp32 accumulation).
+enum { TC_BF16 = 0, TC_I8 = 1, TC_FP8 = 2 };
+
 struct TcArgs {
-  const void* A;        // [M, K] activations: fp16 INT8 codes (W8A8) or bf16, row-major
-  const void* B;        // [N, K] weights: fp16 INT8 codes (W8A8) or bf16, row = output channel
+  const void* A;        // [M, K] activations: fp16 INT8 codes (TC_I8), e4m3 codes (TC_FP8) or bf16, row-major
+  const void* B;        // [N, K] weights in the same type as A, row = output channel
   int M, N, K;
   int kind;             // EPI_BF16, EPI_GEGLU or EPI_F32
-  const float* s_x;     // [M] W8A8: per-token scales
-  const float* s_w;     // [N] W8A8: per-channel scales
+  const float* s_x;     // [M] W8A8 / FP8: per-token scales
+  const float* s_w;     // [N] W8A8 / FP8: per-channel scales
   const float* bias;    // [N] nullable
   uint16_t* y;          // bf16 [M, N] (EPI_BF16) or [M, N / 2] (EPI_GEGLU)
   float* logits;        // [M, N] nullable (EPI_F32)
@@ -33,6 +38,6 @@ bool tc_gemm_supported(int M, int N, int K, int kind, bool want_top, int max_top
 // Workspace bytes the split-K partials of an M-token call may take (an upper bound over N and K,
 // non-decreasing in M).
 size_t tc_split_partial_bytes(int M, int sms);
-w8a8_status launch_tc_gemm(bool int8_codes, const TcArgs& a, cudaStream_t st);
+w8a8_status launch_tc_gemm(int mode, const TcArgs& a, cudaStream_t st);
 
 }  // namespace w8a8

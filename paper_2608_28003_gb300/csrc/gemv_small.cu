@@ -93,9 +93,14 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
   x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
 }
 
-template <bool kInt8, int MT, int RW>
+template <int kW, int MT, int RW>
 __global__ void __launch_bounds__(kThreads, 2)
     gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
+  // kW: weights bf16 (SMALL_BF16), INT8 codes (SMALL_INT8) or e4m3 codes (SMALL_FP8, 8 slots only)
+  constexpr bool kInt8 = kW == SMALL_INT8, kFp8 = kW == SMALL_FP8;
+  constexpr bool kQ = kInt8 || kFp8;  // one-byte codes, per-token K1, dequantising epilogue
+  static_assert(!kFp8 || MT == 8, "the e4m3 path runs on the tensor cores (8 token slots)");
+  constexpr float kQmax = kFp8 ? 448.0f : 127.0f;  // largest code magnitude
   constexpr int R = 8 * RW;
   // bf16 at 5-8 tokens: the products run on the tensor cores (mma.sync m16n8k16, the activations
   // as the A operand with token rows 8-15 zero, each 8 weight rows an n-tile), the 8 consumer warps
@@ -107,7 +112,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   // load from 128-byte-swizzled boxes of 128 columns) into two fp16 pairs, and the k order inside
   // an MMA is permuted alike on both operands (thread t's pairs (2t, 2t+1) and (2t+8, 2t+9) hold
   // k 4t .. 4t+3), which leaves the sum unchanged; the fp32 accumulators (at most 128 products per
-  // stage, exact) are folded into INT32 after every stage.
+  // stage, exact) are folded into INT32 after every stage.  The e4m3 path (FP8 variant) does the
+  // same with e4m3 codes widened to fp16 by the hardware conversion (exact) and plain fp32
+  // accumulation (no fold).
   using Acc = typename std::conditional<kInt8, int, float>::type;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ float s_red[kCW];
@@ -155,10 +162,10 @@ __global__ void __launch_bounds__(kThreads, 2)
       mbar_arrive_expect_tx(bar, (uint32_t)(cnt * R * kSliceBytes));
       for (int u = 0; u < cnt; ++u) {
         const uint32_t d = dst + (uint32_t)(u * R * kSliceBytes);
-        if constexpr (kInt8 && kMma) {
+        if constexpr (kQ && kMma) {
 #pragma unroll
           for (int j = 0; j < 4; ++j) tma_load_2d_policy(d + j * R * 128, &tmW, (u0 + u) * 512 + 128 * j, row0, bar, wpol);
-        } else if constexpr (kInt8) {
+        } else if constexpr (kQ) {
           tma_load_2d_policy(d, &tmW, (u0 + u) * 512, row0, bar, wpol);
           tma_load_2d_policy(d + R * 256, &tmW, (u0 + u) * 512 + 256, row0, bar, wpol);
         } else if constexpr (kMma) {
@@ -191,11 +198,11 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
   for (int i = 0; i < RW; ++i) {
     const int row = row0 + warp + 8 * i;
-    swr[i] = kInt8 && row < a.N ? a.s_w[row] : 0.0f;
+    swr[i] = kQ && row < a.N ? a.s_w[row] : 0.0f;
     bir[i] = a.bias && row < a.N ? a.bias[row] : 0.0f;
   }
   float4 idr[4][2];
-  if constexpr (kInt8) {
+  if constexpr (kQ) {
     const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
@@ -224,9 +231,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   int xstride = a.K;
   // elements between the activation rows in shared memory (bf16, or the fp16 codes of the W8A8
   // tensor-core path; INT8 codes otherwise): padded on the tensor-core paths against bank conflicts
-  const int xsb = kMma ? kpad + (kInt8 ? 16 : 8) : kpad;
+  const int xsb = kMma ? kpad + (kQ ? 16 : 8) : kpad;
   if (a.has_rn) {
-    uint16_t* as = kInt8 ? reinterpret_cast<uint16_t*>(xsp + p.xbytes) : reinterpret_cast<uint16_t*>(xsp);
+    uint16_t* as = kQ ? reinterpret_cast<uint16_t*>(xsp + p.xbytes) : reinterpret_cast<uint16_t*>(xsp);
     for (int m = 0; m < MT; ++m) {
       const bool mine = m < a.M && tid < nvk;
       float yv[8], rv[8];
@@ -266,16 +273,17 @@ __global__ void __launch_bounds__(kThreads, 2)
           w.z = (uint32_t)f32_to_bf16_bits(o[4]) | ((uint32_t)f32_to_bf16_bits(o[5]) << 16);
           w.w = (uint32_t)f32_to_bf16_bits(o[6]) | ((uint32_t)f32_to_bf16_bits(o[7]) << 16);
         }
-        *reinterpret_cast<uint4*>(as + (size_t)m * (kInt8 ? kpad : xsb) + 8 * tid) = w;
+        *reinterpret_cast<uint4*>(as + (size_t)m * (kQ ? kpad : xsb) + 8 * tid) = w;
       }
     }
     named_bar_sync(1, kCW * 32);
     xrows = as;
     xstride = kpad;
   }
-  if constexpr (kInt8) {
+  if constexpr (kQ) {
     // K1 for every token slot: x_hat = x * (1 / delta), m = max |x_hat|, s = m / 127,
     // q = clamp(rint(x_hat * (127 / m)), -127, 127); slots >= M and the tail past K hold zeros.
+    // (e4m3: s = m / 448, q = e4m3(x_hat * (448 / m)), nearest even, saturating.)
     const int nvec = a.K >> 3;
     if constexpr (MT <= 4) {  // one token at a time, all consumer warps on its row
       for (int m = 0; m < MT; ++m) {
@@ -381,9 +389,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         float mx = 0.0f;
 #pragma unroll
         for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red8[m][i]);
-        rr[m] = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
+        rr[m] = mx > 0.0f ? __fdiv_rn(kQmax, mx) : 0.0f;  // fl32(127 / m_t)
         if (tid == m) {
-          const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127); 0 for slots >= M
+          const float sx = __fdiv_rn(mx, kQmax);  // s_t^x = fl32(m_t / 127); 0 for slots >= M
           s_sx[m] = sx;
           if (m < a.M && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
         }
@@ -397,22 +405,35 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int m = 0; m < MT; ++m) {
           float xh[8];
           smooth8(w[m], d0, d1, xh);
-          int q[8];
+          if constexpr (kFp8) {  // e4m3 codes: their fp16 values for the MMA, the bytes for debugging
+            uint32_t c[4];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[e], rr[m]))));
-          if constexpr (kMma) {
+            for (int e = 0; e < 4; ++e)
+              c[e] = e4m3x2_of(__fmul_rn(xh[2 * e], rr[m]), __fmul_rn(xh[2 * e + 1], rr[m]));
             reinterpret_cast<uint4*>(xsp + (size_t)m * xsb * 2)[vi] =
-                make_uint4(f16x2_of((float)q[0], (float)q[1]), f16x2_of((float)q[2], (float)q[3]),
-                           f16x2_of((float)q[4], (float)q[5]), f16x2_of((float)q[6], (float)q[7]));
-          }
-          if (!kMma || (a.xq_dbg && blockIdx.x == 0 && m < a.M)) {
-            uint2 packed;
-            packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
-                       ((uint32_t)(q[3] & 0xff) << 24);
-            packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
-                       ((uint32_t)(q[7] & 0xff) << 24);
-            if (!kMma) reinterpret_cast<uint2*>(xsp + (size_t)m * kpad)[vi] = packed;
-            if (a.xq_dbg && blockIdx.x == 0 && m < a.M) reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] = packed;
+                make_uint4(e4m3x2_to_f16x2(c[0]), e4m3x2_to_f16x2(c[1]), e4m3x2_to_f16x2(c[2]), e4m3x2_to_f16x2(c[3]));
+            if (a.xq_dbg && blockIdx.x == 0 && m < a.M)
+              reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] =
+                  make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
+          } else {
+            int q[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[e], rr[m]))));
+            if constexpr (kMma) {
+              reinterpret_cast<uint4*>(xsp + (size_t)m * xsb * 2)[vi] =
+                  make_uint4(f16x2_of((float)q[0], (float)q[1]), f16x2_of((float)q[2], (float)q[3]),
+                             f16x2_of((float)q[4], (float)q[5]), f16x2_of((float)q[6], (float)q[7]));
+            }
+            if (!kMma || (a.xq_dbg && blockIdx.x == 0 && m < a.M)) {
+              uint2 packed;
+              packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                         ((uint32_t)(q[3] & 0xff) << 24);
+              packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                         ((uint32_t)(q[7] & 0xff) << 24);
+              if (!kMma) reinterpret_cast<uint2*>(xsp + (size_t)m * kpad)[vi] = packed;
+              if (a.xq_dbg && blockIdx.x == 0 && m < a.M)
+                reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] = packed;
+            }
           }
         }
       }
@@ -472,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int i = 0; i < RW; ++i) mc[c][i][0] = mc[c][i][1] = mc[c][i][2] = mc[c][i][3] = 0.0f;
   bool ok = true;
   // INT8 sub-slice: two boxes [R][256 B]; lane l reads box l / 16 at byte 16 (l % 16) of the row
-  const uint32_t wlane = kInt8 ? (uint32_t)((lane >> 4) * R * 256 + 16 * (lane & 15)) : (uint32_t)(16 * lane);
+  const uint32_t wlane = kQ ? (uint32_t)((lane >> 4) * R * 256 + 16 * (lane & 15)) : (uint32_t)(16 * lane);
   int s = 0;
   uint32_t ph = 0;
   for (int it = 0; it < nst; ++it) {
@@ -491,7 +512,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       const uint32_t sb = ring + (uint32_t)(s * SB);
       const int u0 = it * KS, cnt = min(KS, nsub - u0);
       const int xr = lane & 7, xh = (lane >> 3) & 1;  // ldmatrix row addresses: token / half
-      if constexpr (kInt8) {
+      if constexpr (kQ) {
         // k steps of 16 of this stage: step q is sub-slice q / 32, 128-column box (q % 32) / 8,
         // 16-byte chunk q % 8 of its rows; thread (g, t) reads bytes 4 t .. 4 t + 3 of row g's chunk
         // and of token g's codes
@@ -507,7 +528,12 @@ __global__ void __launch_bounds__(kThreads, 2)
             uint32_t wb;
             asm volatile("ld.shared.u32 %0, [%1];\n" : "=r"(wb) : "r"(box + (uint32_t)((8 * i + g) * 128 + ((ch ^ g) << 4) + 4 * t)));
             uint32_t b0, b1;
-            i8x4_to_f16x2x2(wb, b0, b1);
+            if constexpr (kFp8) {
+              b0 = e4m3x2_to_f16x2(wb);
+              b1 = e4m3x2_to_f16x2(wb >> 16);
+            } else {
+              i8x4_to_f16x2x2(wb, b0, b1);
+            }
             mma_f16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
           }
         };
@@ -515,12 +541,14 @@ __global__ void __launch_bounds__(kThreads, 2)
           step8(q, mc[0]);
           if (q + kCW < 32 * cnt) step8(q + kCW, mc[1]);
         }
+        if constexpr (kInt8) {
 #pragma unroll
-        for (int i = 0; i < RW; ++i) {  // fold: each set took at most 128 products per output this stage
-          mi32[i][0] += __float2int_rn(mc[0][i][0]) + __float2int_rn(mc[1][i][0]);
-          mi32[i][1] += __float2int_rn(mc[0][i][1]) + __float2int_rn(mc[1][i][1]);
+          for (int i = 0; i < RW; ++i) {  // fold: each set took at most 128 products per output this stage
+            mi32[i][0] += __float2int_rn(mc[0][i][0]) + __float2int_rn(mc[1][i][0]);
+            mi32[i][1] += __float2int_rn(mc[0][i][1]) + __float2int_rn(mc[1][i][1]);
 #pragma unroll
-          for (int e = 0; e < 4; ++e) mc[0][i][e] = mc[1][i][e] = 0.0f;
+            for (int e = 0; e < 4; ++e) mc[0][i][e] = mc[1][i][e] = 0.0f;
+          }
         }
       } else {
       auto step = [&](int q, float (&c)[RW][4]) {
@@ -631,6 +659,8 @@ __global__ void __launch_bounds__(kThreads, 2)
       if constexpr (kInt8) {
         y = __fmul_rn(__fmul_rn(s_sx[m], a.s_w[row0 + r]), __int2float_rn(v));
         if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row0 + r] = v;
+      } else if constexpr (kFp8) {
+        y = __fmul_rn(__fmul_rn(s_sx[m], a.s_w[row0 + r]), v);
       } else {
         y = v;
       }
@@ -708,73 +738,76 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 }
 
-template <bool kInt8, int MT, int RW>
+template <int kW, int MT, int RW>
 w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kInt8, MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    kSmemLimit - kStatic));
     attr_set[dev] = true;
   }
-  constexpr int EB = kInt8 ? 1 : 2;
+  constexpr int EB = kW == SMALL_BF16 ? 2 : 1;
   CUtensorMap tw;
   if (MT == 8)  // the tensor-core paths: 128-byte boxes (64 bf16 or 128 INT8 columns), 128-byte swizzle
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 8 * RW, 128));
   else
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
-  W8A8_CUDA(launch_pdl(gemv_small_kernel<kInt8, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
+  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
                        a));
   return W8A8_OK;
 }
 
 // accumulator registers a warp may hold (tokens x rows): larger products spill; the tensor-core paths
 // (8 token slots) hold 8 (+ 2 INT32) per n-tile of 8 rows whatever the token count
-template <bool kInt8>
-constexpr int max_slots() {
-  return kInt8 ? 48 : 32;
+constexpr bool slots_fit(int kw, int MT, int RW) {
+  return MT == 8 || (kw != SMALL_FP8 && MT * RW <= (kw == SMALL_INT8 ? 48 : 32));
 }
-constexpr bool slots_fit(bool int8, int MT, int RW) { return MT == 8 || MT * RW <= (int8 ? 48 : 32); }
 
-template <bool kInt8, int MT, int RW>
+template <int kW, int MT, int RW>
 w8a8_status launch_checked(const SmallArgs& a, cudaStream_t st) {
-  if constexpr (slots_fit(kInt8, MT, RW)) {
-    return launch_t<kInt8, MT, RW>(a, st);
+  if constexpr (slots_fit(kW, MT, RW)) {
+    return launch_t<kW, MT, RW>(a, st);
   } else {
     W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "small GEMV: %d tokens x %d rows per warp not built", MT, RW);
   }
 }
 
-template <bool kInt8, int MT>
+template <int kW, int MT>
 w8a8_status launch_mt(const SmallArgs& a, cudaStream_t st) {
   switch (a.p.RW) {
-    case 1: return launch_checked<kInt8, MT, 1>(a, st);
-    case 2: return launch_checked<kInt8, MT, 2>(a, st);
-    case 4: return launch_checked<kInt8, MT, 4>(a, st);
-    default: return launch_checked<kInt8, MT, 6>(a, st);
+    case 1: return launch_checked<kW, MT, 1>(a, st);
+    case 2: return launch_checked<kW, MT, 2>(a, st);
+    case 4: return launch_checked<kW, MT, 4>(a, st);
+    default: return launch_checked<kW, MT, 6>(a, st);
   }
 }
 
-template <bool kInt8>
+template <int kW>
 w8a8_status launch_typed(const SmallArgs& a, cudaStream_t st) {
-  switch (a.p.MT) {
-    case 1: return launch_mt<kInt8, 1>(a, st);
-    case 2: return launch_mt<kInt8, 2>(a, st);
-    case 4: return launch_mt<kInt8, 4>(a, st);
-    default: return launch_mt<kInt8, 8>(a, st);
+  if constexpr (kW == SMALL_FP8) {
+    return launch_mt<kW, 8>(a, st);
+  } else {
+    switch (a.p.MT) {
+      case 1: return launch_mt<kW, 1>(a, st);
+      case 2: return launch_mt<kW, 2>(a, st);
+      case 4: return launch_mt<kW, 4>(a, st);
+      default: return launch_mt<kW, 8>(a, st);
+    }
   }
 }
 
 }  // namespace
 
-SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count, bool fused_norm) {
+SmallPlan make_small_plan(int wkind, int M, int N, int K, int kind, int sm_count, bool fused_norm) {
   SmallPlan p{};
+  const bool int8_weights = wkind != SMALL_BF16;  // one-byte codes (INT8 or e4m3)
   if (fused_norm && K > 2048) return p;  // one 8-channel vector per consumer thread
   if (M < 1 || M > 8 || N < 1 || K < 16 || K % 16 != 0) return p;
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return p;
   if (kind == EPI_GEGLU && N % 16 != 0) return p;
-  p.MT = M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
+  p.MT = wkind == SMALL_FP8 ? 8 : M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
   if (int8_weights && p.MT <= 4 && K > kMaxInt8K) return p;
   // fewest rows per CTA (more CTAs) that still fit in two CTAs per SM
   static const int kRw[] = {1, 2, 4, 6};
@@ -786,7 +819,7 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
     }
   }
   if (p.RW == 0) return p;
-  if (!slots_fit(int8_weights, p.MT, p.RW)) return p;  // registers
+  if (!slots_fit(wkind, p.MT, p.RW)) return p;  // registers
   const int R = 8 * p.RW;
   p.P = (N + R - 1) / R;
   const int cps = p.P > sm_count ? 2 : 1;
@@ -817,14 +850,16 @@ SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int 
   return p;
 }
 
-w8a8_status launch_small_gemv(bool int8_weights, const SmallArgs& a, cudaStream_t st) {
+w8a8_status launch_small_gemv(int wkind, const SmallArgs& a, cudaStream_t st) {
   if (a.M == 0 || a.N == 0) return W8A8_OK;
   W8A8_CHECK_ARG(a.p.ok, W8A8_ERR_SHAPE, "small GEMV: no plan for M=%d N=%d K=%d", a.M, a.N, a.K);
   void *v0, *v1;
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  const w8a8_status s = int8_weights ? launch_typed<true>(a, st) : launch_typed<false>(a, st);
+  const w8a8_status s = wkind == SMALL_FP8    ? launch_typed<SMALL_FP8>(a, st)
+                        : wkind == SMALL_INT8 ? launch_typed<SMALL_INT8>(a, st)
+                                              : launch_typed<SMALL_BF16>(a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }

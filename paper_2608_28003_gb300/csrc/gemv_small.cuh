@@ -1,11 +1,15 @@
 // Decode GEMV for up to 8 tokens whose CTAs own whole weight rows (no split of the k sum across
-// CTAs): the W8A8 path with the per-token quantiser (K1) fused into its prologue, and the bf16
-// pass-through.
+// CTAs): the W8A8 path with the per-token quantiser (K1) fused into its prologue, its e4m3 (FP8)
+// variant, and the bf16 pass-through.
 #pragma once
 
 #include "common.cuh"
 
 namespace w8a8 {
+
+// Weight kinds: bf16, INT8 codes (W8A8), e4m3 codes (the FP8 variant; always 8 token slots on the
+// tensor cores).
+enum { SMALL_BF16 = 0, SMALL_INT8 = 1, SMALL_FP8 = 2 };
 
 struct SmallPlan {
   int ok;           // 0: this shape is left to the weight-streaming kernel
@@ -39,7 +43,7 @@ struct ResNorm {
 };
 
 struct SmallArgs {
-  const void* W;           // [N, K] INT8 codes or bf16, row = output channel
+  const void* W;           // [N, K] INT8 codes, e4m3 codes or bf16, row = output channel
   const uint16_t* X;       // [M, K] bf16 activations
   int M, N, K;
   int kind;                // EPI_BF16 or EPI_GEGLU (gate/up rows interleaved in blocks of 8)
@@ -47,9 +51,9 @@ struct SmallArgs {
   const float* s_w;        // [N] INT8 path
   const float* bias;       // [N] nullable
   uint16_t* y;             // [M, N] bf16 or [M, N / 2] for GeGLU
-  int8_t* xq_dbg;          // [M, K] nullable: the INT8 activation codes
+  int8_t* xq_dbg;          // [M, K] nullable: the INT8 (or e4m3) activation codes
   float* s_x_dbg;          // [M] nullable: the per-token scales
-  int32_t* acc_dbg;        // [M, N] nullable: the INT32 sums
+  int32_t* acc_dbg;        // [M, N] nullable: the INT32 sums (INT8 codes only)
   int has_rn;              // 1: X is computed from rn (X unused)
   ResNorm rn;
   unsigned int* err;       // device error word
@@ -57,7 +61,7 @@ struct SmallArgs {
 };
 
 // fused_norm: the call computes its input with a ResNorm (needs K <= 2048)
-SmallPlan make_small_plan(bool int8_weights, int M, int N, int K, int kind, int sm_count, bool fused_norm = false);
-w8a8_status launch_small_gemv(bool int8_weights, const SmallArgs& a, cudaStream_t st);
+SmallPlan make_small_plan(int wkind, int M, int N, int K, int kind, int sm_count, bool fused_norm = false);
+w8a8_status launch_small_gemv(int wkind, const SmallArgs& a, cudaStream_t st);
 
 }  // namespace w8a8

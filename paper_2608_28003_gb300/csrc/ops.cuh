@@ -24,6 +24,8 @@ FfnWs ffn_ws(int M, int H, int F, int sms);
 
 w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* inv_delta, int8_t* xq,
                                  uint16_t* xq_f16, float* s_x, cudaStream_t st);
+w8a8_status launch_quantize_rows_fp8(const uint16_t* X, int M, int K, const float* inv_delta, uint8_t* xq,
+                                     float* s_x, cudaStream_t st);
 w8a8_status launch_act_absmax(const uint16_t* X, int T, int K, float* absmax, cudaStream_t st);
 
 // kind: 0 bf16 output, 1 GeGLU, 2 fp32 logits (+ top-1)

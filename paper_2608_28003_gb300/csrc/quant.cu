@@ -6,7 +6,9 @@
 //        si, what-ffn
 //
 // Every step that decides an INT8 code is one IEEE fp32 operation with round-to-nearest-even
-// (__fmul_rn, __fdiv_rn, __fsqrt_rn, __float2int_rn), in the order the header documents.
+// (__fmul_rn, __fdiv_rn, __fsqrt_rn, __float2int_rn), in the order the header documents.  The FP8
+// variant (Future Work: e4m3 in place of INT8) runs the same kernels with 448 in place of 127 and
+// the hardware's e4m3 conversion (nearest even, saturating) in place of rint and the clamp.
 #include <cmath>
 
 #include "common.cuh"
@@ -16,7 +18,7 @@ namespace w8a8 {
 // ------------------------------------------------------------------------------ K1
 // One CTA per row.  Each thread holds up to kVec 16-byte vectors (8 bf16 each) of the row in
 // registers between the max pass and the quantise pass; longer rows are re-read.
-template <int kVec>
+template <int kVec, bool kFp8>
 __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __restrict__ X, int K,
                                                            const float* __restrict__ inv_delta,
                                                            int8_t* __restrict__ xq,
@@ -75,28 +77,36 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __re
   }
   __syncthreads();
   const float m = red[0];
-  const float r = m > 0.0f ? __fdiv_rn(127.0f, m) : 0.0f;  // fl32(127 / m_t)
-  if (threadIdx.x == 0) s_x[row] = __fdiv_rn(m, 127.0f);  // s_t^x = fl32(m_t / 127)
+  constexpr float kQmax = kFp8 ? 448.0f : 127.0f;
+  const float r = m > 0.0f ? __fdiv_rn(kQmax, m) : 0.0f;  // fl32(127 / m_t)
+  if (threadIdx.x == 0) s_x[row] = __fdiv_rn(m, kQmax);  // s_t^x = fl32(m_t / 127)
 
   auto emit = [&](int vi, const float (&v8)[8]) {
-    int q[8];
+    if constexpr (kFp8) {  // e4m3 codes (xq receives the bytes)
+      uint32_t c[4];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(v8[e], r))));
-    if (xq) {
-      uint2 packed;
-      packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
-                 ((uint32_t)(q[3] & 0xff) << 24);
-      packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
-                 ((uint32_t)(q[7] & 0xff) << 24);
-      reinterpret_cast<uint2*>(xq + (size_t)row * K)[vi] = packed;
-    }
-    if (xq_f16) {
-      uint4 h;
-      h.x = (uint32_t)int_to_f16_bits(q[0]) | ((uint32_t)int_to_f16_bits(q[1]) << 16);
-      h.y = (uint32_t)int_to_f16_bits(q[2]) | ((uint32_t)int_to_f16_bits(q[3]) << 16);
-      h.z = (uint32_t)int_to_f16_bits(q[4]) | ((uint32_t)int_to_f16_bits(q[5]) << 16);
-      h.w = (uint32_t)int_to_f16_bits(q[6]) | ((uint32_t)int_to_f16_bits(q[7]) << 16);
-      reinterpret_cast<uint4*>(xq_f16 + (size_t)row * K)[vi] = h;
+      for (int e = 0; e < 4; ++e) c[e] = e4m3x2_of(__fmul_rn(v8[2 * e], r), __fmul_rn(v8[2 * e + 1], r));
+      reinterpret_cast<uint2*>(xq + (size_t)row * K)[vi] = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
+    } else {
+      int q[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(v8[e], r))));
+      if (xq) {
+        uint2 packed;
+        packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                   ((uint32_t)(q[3] & 0xff) << 24);
+        packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                   ((uint32_t)(q[7] & 0xff) << 24);
+        reinterpret_cast<uint2*>(xq + (size_t)row * K)[vi] = packed;
+      }
+      if (xq_f16) {
+        uint4 h;
+        h.x = (uint32_t)int_to_f16_bits(q[0]) | ((uint32_t)int_to_f16_bits(q[1]) << 16);
+        h.y = (uint32_t)int_to_f16_bits(q[2]) | ((uint32_t)int_to_f16_bits(q[3]) << 16);
+        h.z = (uint32_t)int_to_f16_bits(q[4]) | ((uint32_t)int_to_f16_bits(q[5]) << 16);
+        h.w = (uint32_t)int_to_f16_bits(q[6]) | ((uint32_t)int_to_f16_bits(q[7]) << 16);
+        reinterpret_cast<uint4*>(xq_f16 + (size_t)row * K)[vi] = h;
+      }
     }
   };
   if (in_regs) {
@@ -123,7 +133,18 @@ w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* i
   if (M == 0) return W8A8_OK;
   const int nvec = K / 8;
   const int threads = nvec <= 4 * 128 ? 128 : 256;
-  W8A8_CUDA(launch_pdl(quantize_rows_kernel<4>, dim3(M), dim3(threads), 0, st, X, K, inv_delta, xq, xq_f16, s_x));
+  W8A8_CUDA(launch_pdl(quantize_rows_kernel<4, false>, dim3(M), dim3(threads), 0, st, X, K, inv_delta, xq, xq_f16,
+                       s_x));
+  return W8A8_OK;
+}
+
+w8a8_status launch_quantize_rows_fp8(const uint16_t* X, int M, int K, const float* inv_delta, uint8_t* xq,
+                                     float* s_x, cudaStream_t st) {
+  if (M == 0) return W8A8_OK;
+  const int nvec = K / 8;
+  const int threads = nvec <= 4 * 128 ? 128 : 256;
+  W8A8_CUDA(launch_pdl(quantize_rows_kernel<4, true>, dim3(M), dim3(threads), 0, st, X, K, inv_delta,
+                       reinterpret_cast<int8_t*>(xq), static_cast<uint16_t*>(nullptr), s_x));
   return W8A8_OK;
 }
 
@@ -215,6 +236,7 @@ __global__ void smooth_factor_kernel(const float* __restrict__ ax, float* __rest
 // q = clamp(rint(fl32(W_hat * fl32(127 / m))), -127, 127) (Eq. si, what-ffn on Eq. what-lmhead).
 // The source row is W0 + p*K, or for the gate/up interleave (W1 != nullptr): block q = p / 16,
 // r = p % 16, r < 8 -> W0 row 8q + r, else W1 row 8q + r - 8.
+template <bool kFp8>
 __global__ void __launch_bounds__(256) quant_weight_rows_kernel(const uint16_t* __restrict__ W0,
                                                                const uint16_t* __restrict__ W1, int K,
                                                                const float* __restrict__ delta,
@@ -254,8 +276,9 @@ __global__ void __launch_bounds__(256) quant_weight_rows_kernel(const uint16_t* 
   }
   __syncthreads();
   const float m = red[0];
-  const float r = m > 0.0f ? __fdiv_rn(127.0f, m) : 0.0f;
-  if (threadIdx.x == 0) s_w[p] = __fdiv_rn(m, 127.0f);
+  constexpr float kQmax = kFp8 ? 448.0f : 127.0f;
+  const float r = m > 0.0f ? __fdiv_rn(kQmax, m) : 0.0f;
+  if (threadIdx.x == 0) s_w[p] = __fdiv_rn(m, kQmax);
   for (int vi = threadIdx.x; vi < nvec; vi += blockDim.x) {
     const uint4 w = reinterpret_cast<const uint4*>(src)[vi];
     const float4 d0 = reinterpret_cast<const float4*>(delta)[2 * vi];
@@ -264,22 +287,29 @@ __global__ void __launch_bounds__(256) quant_weight_rows_kernel(const uint16_t* 
                          __fmul_rn(bf16_lo(w.y), d0.z), __fmul_rn(bf16_hi(w.y), d0.w),
                          __fmul_rn(bf16_lo(w.z), d1.x), __fmul_rn(bf16_hi(w.z), d1.y),
                          __fmul_rn(bf16_lo(w.w), d1.z), __fmul_rn(bf16_hi(w.w), d1.w)};
-    int q[8];
+    if constexpr (kFp8) {  // e4m3 codes; an all-zero row has r = 0 and codes 0
+      uint32_t c[4];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) q[e] = m > 0.0f ? max(-127, min(127, __float2int_rn(__fmul_rn(v8[e], r)))) : 0;
-    uint2 packed;
-    packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
-               ((uint32_t)(q[3] & 0xff) << 24);
-    packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
-               ((uint32_t)(q[7] & 0xff) << 24);
-    reinterpret_cast<uint2*>(wq + (size_t)p * K)[vi] = packed;
-    if (wq_f16) {
-      uint4 h;
-      h.x = (uint32_t)int_to_f16_bits(q[0]) | ((uint32_t)int_to_f16_bits(q[1]) << 16);
-      h.y = (uint32_t)int_to_f16_bits(q[2]) | ((uint32_t)int_to_f16_bits(q[3]) << 16);
-      h.z = (uint32_t)int_to_f16_bits(q[4]) | ((uint32_t)int_to_f16_bits(q[5]) << 16);
-      h.w = (uint32_t)int_to_f16_bits(q[6]) | ((uint32_t)int_to_f16_bits(q[7]) << 16);
-      reinterpret_cast<uint4*>(wq_f16 + (size_t)p * K)[vi] = h;
+      for (int e = 0; e < 4; ++e) c[e] = e4m3x2_of(__fmul_rn(v8[2 * e], r), __fmul_rn(v8[2 * e + 1], r));
+      reinterpret_cast<uint2*>(wq + (size_t)p * K)[vi] = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
+    } else {
+      int q[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) q[e] = m > 0.0f ? max(-127, min(127, __float2int_rn(__fmul_rn(v8[e], r)))) : 0;
+      uint2 packed;
+      packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
+                 ((uint32_t)(q[3] & 0xff) << 24);
+      packed.y = (uint32_t)(q[4] & 0xff) | ((uint32_t)(q[5] & 0xff) << 8) | ((uint32_t)(q[6] & 0xff) << 16) |
+                 ((uint32_t)(q[7] & 0xff) << 24);
+      reinterpret_cast<uint2*>(wq + (size_t)p * K)[vi] = packed;
+      if (wq_f16) {
+        uint4 h;
+        h.x = (uint32_t)int_to_f16_bits(q[0]) | ((uint32_t)int_to_f16_bits(q[1]) << 16);
+        h.y = (uint32_t)int_to_f16_bits(q[2]) | ((uint32_t)int_to_f16_bits(q[3]) << 16);
+        h.z = (uint32_t)int_to_f16_bits(q[4]) | ((uint32_t)int_to_f16_bits(q[5]) << 16);
+        h.w = (uint32_t)int_to_f16_bits(q[6]) | ((uint32_t)int_to_f16_bits(q[7]) << 16);
+        reinterpret_cast<uint4*>(wq_f16 + (size_t)p * K)[vi] = h;
+      }
     }
   }
 }
@@ -305,7 +335,8 @@ static w8a8_status launch_colmax(const uint16_t* W, int N, int K, float* out, cu
 
 static w8a8_status prepare_common(const uint16_t* W0, const uint16_t* W1, int rows_each, int K,
                                   const float* act_absmax, float alpha, int smooth, int8_t* wq, float* s_w,
-                                  float* delta, float* inv_delta, uint16_t* wq_f16, cudaStream_t st) {
+                                  float* delta, float* inv_delta, uint16_t* wq_f16, cudaStream_t st,
+                                  bool fp8 = false) {
   const int N = W1 ? 2 * rows_each : rows_each;
   W8A8_CUDA(cudaMemsetAsync(delta, 0, sizeof(float) * K, st));
   if (smooth) {
@@ -319,7 +350,10 @@ static w8a8_status prepare_common(const uint16_t* W0, const uint16_t* W1, int ro
   smooth_factor_kernel<<<(K + 255) / 256, 256, 0, st>>>(act_absmax, delta, inv_delta, K, alpha, smooth);
   W8A8_LAUNCH_CHECK();
   if (N > 0) {
-    quant_weight_rows_kernel<<<N, 256, 0, st>>>(W0, W1, K, delta, wq, s_w, wq_f16);
+    if (fp8)
+      quant_weight_rows_kernel<true><<<N, 256, 0, st>>>(W0, W1, K, delta, wq, s_w, nullptr);
+    else
+      quant_weight_rows_kernel<false><<<N, 256, 0, st>>>(W0, W1, K, delta, wq, s_w, wq_f16);
     W8A8_LAUNCH_CHECK();
   }
   return W8A8_OK;
@@ -413,4 +447,53 @@ extern "C" w8a8_status w8a8_quantize_activations(const uint16_t* X, int M, int K
   w8a8_status s = check_device();
   if (s != W8A8_OK) return s;
   return launch_quantize_rows(X, M, K, inv_delta, xq, xq_f16, s_x, as_stream(stream));
+}
+
+// ------------------------------------------------------------------------ FP8 (e4m3) variant
+extern "C" w8a8_status w8a8_fp8_prepare_weights(const uint16_t* W, int N, int K, const float* act_absmax, float alpha,
+                                                int smooth, uint8_t* wq, float* s_w, float* delta, float* inv_delta,
+                                                void* stream) {
+  int8_t* codes = reinterpret_cast<int8_t*>(wq);
+  w8a8_status s =
+      check_prep_args("w8a8_fp8_prepare_weights", W, N, K, act_absmax, smooth, codes, s_w, delta, inv_delta, nullptr);
+  if (s != W8A8_OK) return s;
+  W8A8_CHECK_ARG(std::isfinite(alpha) && alpha >= 0.0f && alpha <= 1.0f, W8A8_ERR_INVALID_ARG,
+                 "w8a8_fp8_prepare_weights: alpha must be in [0, 1]");
+  if (K == 0) return W8A8_OK;
+  s = check_device();
+  if (s != W8A8_OK) return s;
+  return prepare_common(W, nullptr, N, K, act_absmax, alpha, smooth, codes, s_w, delta, inv_delta, nullptr,
+                        as_stream(stream), true);
+}
+
+extern "C" w8a8_status w8a8_fp8_prepare_gate_up(const uint16_t* W_gate, const uint16_t* W_up, int F, int H,
+                                                const float* act_absmax, float alpha, int smooth, uint8_t* wq,
+                                                float* s_w, float* delta, float* inv_delta, void* stream) {
+  int8_t* codes = reinterpret_cast<int8_t*>(wq);
+  w8a8_status s = check_prep_args("w8a8_fp8_prepare_gate_up", W_gate, F, H, act_absmax, smooth, codes, s_w, delta,
+                                  inv_delta, nullptr);
+  if (s != W8A8_OK) return s;
+  W8A8_CHECK_ARG(W_up && aligned16(W_up), W8A8_ERR_INVALID_ARG, "w8a8_fp8_prepare_gate_up: W_up null or unaligned");
+  W8A8_CHECK_ARG(F % 8 == 0, W8A8_ERR_SHAPE, "w8a8_fp8_prepare_gate_up: F=%d must be a multiple of 8", F);
+  W8A8_CHECK_ARG(std::isfinite(alpha) && alpha >= 0.0f && alpha <= 1.0f, W8A8_ERR_INVALID_ARG,
+                 "w8a8_fp8_prepare_gate_up: alpha must be in [0, 1]");
+  if (H == 0) return W8A8_OK;
+  s = check_device();
+  if (s != W8A8_OK) return s;
+  return prepare_common(W_gate, W_up, F, H, act_absmax, alpha, smooth, codes, s_w, delta, inv_delta, nullptr,
+                        as_stream(stream), true);
+}
+
+extern "C" w8a8_status w8a8_fp8_quantize_activations(const uint16_t* X, int M, int K, const float* inv_delta,
+                                                     uint8_t* xq, float* s_x, void* stream) {
+  W8A8_CHECK_ARG(M >= 0 && K >= 0, W8A8_ERR_INVALID_ARG, "w8a8_fp8_quantize_activations: negative size");
+  W8A8_CHECK_ARG(K % 16 == 0 && K <= W8A8_MAX_K, W8A8_ERR_SHAPE,
+                 "w8a8_fp8_quantize_activations: K=%d must be a multiple of 16 and <= %d", K, W8A8_MAX_K);
+  if (M == 0) return W8A8_OK;
+  W8A8_CHECK_ARG(X && inv_delta && s_x && xq, W8A8_ERR_INVALID_ARG, "w8a8_fp8_quantize_activations: null pointer");
+  W8A8_CHECK_ARG(aligned16(X) && aligned16(inv_delta) && aligned16(s_x) && aligned16(xq), W8A8_ERR_ALIGN,
+                 "w8a8_fp8_quantize_activations: pointers must be 16-byte aligned");
+  w8a8_status s = check_device();
+  if (s != W8A8_OK) return s;
+  return launch_quantize_rows_fp8(X, M, K, inv_delta, xq, s_x, as_stream(stream));
 }

@@ -110,3 +110,19 @@ def test_linear_error_bound(smooth):
     assert np.all(np.abs(r["y"] - exact) <= bound)
     # and the bound is not vacuous: the error is a visible fraction of it somewhere
     assert np.max(np.abs(r["y"] - exact) / bound) > 0.01
+
+
+def test_fp8_ffn_block_stages_chain():
+    """The FP8 block's stages chain: h is bf16(geglu(g, u)) of the fp32 gate/up outputs, down's
+    codes are those of that h, and the block stays within the quantisation error of the bf16 block."""
+    import synth
+    from oracle import blocks, geglu
+    from oracle import w8a8 as W
+    c = synth.ffn_case(3, seed=0, hidden=64, inter=96, calib_rows=16)
+    prep = blocks.prepare_ffn_fp8(c["wg32"], c["wu32"], c["wd32"], W.act_absmax(c["calib32"]), c["stat_h"])
+    r = blocks.ffn_fp8(c["x32"], prep)
+    assert np.array_equal(r["h"], W.round_to_bf16(geglu.geglu_f32(r["g"], r["u"])))
+    xq, _ = fp8.quantize_rows_fp8(W.smooth_activations(r["h"], prep["down"]["inv_delta"]))
+    assert np.array_equal(xq, r["down"]["xq"])
+    ref = blocks.ffn_bf16(c["x32"], c["wg32"], c["wu32"], c["wd32"])
+    assert np.abs(r["y"] - ref["y"]).max() < 0.1 * np.abs(ref["y"]).max()
