@@ -66,7 +66,7 @@ def parse():
     ap.add_argument("--profile-workload", choices=["decode4", "gemm", "linear16", "prefill4", "ffn2048", "mid4"], default=None,
                     help="run a small fixed workload for a profiler and exit (no JSON line): 'decode4' = five "
                          "batch-1 decode steps of a 4-layer decoder with the full shapes (FFN layers 0-1 and "
-                         "lm_head W8A8); 'gemm' = three bf16 and three W8A8 prefill linears, 2048 x 1152 -> 13824; "
+                         "lm_head W8A8); 'gemm' = three bf16, three W8A8 and three FP8 prefill linears, 2048 x 1152 -> 13824; "
                          "'linear16' = the single-linear workload (M 16, 1152 -> 6912) three times each as W8A8 "
                          "on INT8 codes, W8A8 with the fp16 code copy and bf16, then three W8A8 FFN blocks at M 8; "
                          "'prefill4' = a 2048-token prefill of a 4-layer decoder with the full shapes (bf16); "
@@ -168,10 +168,13 @@ def profile_workload(name):
         ws = B.Workspace(dev)
         y = torch.empty(M, N, dtype=torch.bfloat16, device=dev)
         q = B.prepare_weights(w, B.act_absmax(x), want_f16=True)
+        q8 = B.fp8_prepare_weights(w, B.act_absmax(x))
         for _ in range(3):
             B.linear_bf16(w, x, out=y, ws=ws)
         for _ in range(3):
             B.linear(q, x, out=y, ws=ws)
+        for _ in range(3):
+            B.fp8_linear(q8, x, out=y, ws=ws)
         torch.cuda.synchronize()
     print("ok")
 
@@ -754,18 +757,32 @@ def sweep(B, dev, head, xh, flush, stream, peaks):
     rec("linear_w8a8_M16", t, 2 * 16 * INTER * HIDDEN, w8a8_bytes(16, INTER, HIDDEN), True)
     t = statistics.mean(timed_steps(lambda: B.linear_bf16(w, x, out=y, ws=ws), 10, 3, flush, stream, kev))
     rec("linear_bf16_M16", t, 2 * 16 * INTER * HIDDEN, bf16_bytes(16, INTER, HIDDEN), True)
+    q8 = B.fp8_prepare_weights(w, B.act_absmax(c["calib"].to(dev)))
+    t = statistics.mean(timed_steps(lambda: B.fp8_linear(q8, x, out=y, ws=ws), 10, 3, flush, stream, kev))
+    rec("linear_fp8_M16", t, 2 * 16 * INTER * HIDDEN, w8a8_bytes(16, INTER, HIDDEN), True)
     fc = synth.ffn_case(2048, seed=0)
     gu = B.prepare_gate_up(fc["wg"].to(dev), fc["wu"].to(dev), B.act_absmax(fc["calib"].to(dev)), want_f16=True)
     dn = B.prepare_weights(fc["wd"].to(dev), torch.from_numpy(fc["stat_h"]).to(dev), want_f16=True)
     f = B.FfnWeights(HIDDEN, INTER, gu, dn, B.interleave_gate_up(fc["wg"].to(dev), fc["wu"].to(dev)), fc["wd"].to(dev))
     xf = fc["x"].to(dev)
     yf = torch.empty(2048, HIDDEN, dtype=torch.bfloat16, device=dev)
+    stat_in = B.act_absmax(fc["calib"].to(dev))
+    f8 = B.Fp8FfnWeights(HIDDEN, INTER, B.fp8_prepare_gate_up(fc["wg"].to(dev), fc["wu"].to(dev), stat_in),
+                         B.fp8_prepare_weights(fc["wd"].to(dev), torch.from_numpy(fc["stat_h"]).to(dev)))
+    cmp = {}
     for M in (1, 8, 64, 512, 2048):
         flops = 2 * M * 3 * INTER * HIDDEN
-        for prec, tag in ((B.W8A8_PREC_W8A8, "w8a8"), (B.W8A8_PREC_BF16, "bf16")):
-            t = statistics.mean(timed_steps(lambda: B.ffn_block(f, prec, xf[:M], out=yf[:M], ws=ws), 10, 3, flush,
-                                            stream))
-            rec(f"ffn_{tag}_M{M}", t, flops, ffn_bytes(M, prec == B.W8A8_PREC_W8A8))
+        row = {}
+        for tag, fn in (("w8a8", lambda: B.ffn_block(f, B.W8A8_PREC_W8A8, xf[:M], out=yf[:M], ws=ws)),
+                        ("bf16", lambda: B.ffn_block(f, B.W8A8_PREC_BF16, xf[:M], out=yf[:M], ws=ws)),
+                        ("fp8", lambda: B.fp8_ffn_block(f8, xf[:M], out=yf[:M], ws=ws))):
+            t = statistics.mean(timed_steps(fn, 10, 3, flush, stream))
+            rec(f"ffn_{tag}_M{M}", t, flops, ffn_bytes(M, tag != "bf16"))
+            row[f"{tag}_us"] = out[f"ffn_{tag}_M{M}"]["us"]
+        row["w8a8_vs_bf16"] = round(row["bf16_us"] / row["w8a8_us"], 3)
+        row["fp8_vs_bf16"] = round(row["bf16_us"] / row["fp8_us"], 3)
+        cmp[f"M{M}"] = row
+    out["ffn_fp8_int8_bf16"] = cmp
     lg = torch.empty(512, VOCAB, dtype=torch.float32, device=dev)
     tp = torch.empty(512, dtype=torch.int32, device=dev)
     for M in (1, 16, 128, 512):

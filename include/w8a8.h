@@ -365,15 +365,29 @@ w8a8_status w8a8_decoder_forward(w8a8_model* m, const int32_t* tokens, int B, in
 w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* tokens, int B, int pos, float* logits,
                                      int32_t* top1, void* stream);
 
-/* How a decode step of one sequence runs (no counterpart in the paper; results agree up to fp32
- * summation order): W8A8_DECODE_PER_STEP (default) launches one kernel per step of each layer
- * (programmatic dependent launch overlaps each kernel's weight reads with its predecessor),
- * W8A8_DECODE_PERSISTENT runs every decoder layer in one cooperative launch of one CTA per SM
- * whose phases wait on each other through global counters (when the shapes allow: head dim 256,
- * hidden <= 2048, intermediate <= 7168).  Other batch sizes always take the per-step kernels.
- * W8A8_ERR_INVALID_ARG for another value. */
-enum { W8A8_DECODE_PER_STEP = 0, W8A8_DECODE_PERSISTENT = 1 };
-w8a8_status w8a8_model_set_decode_path(w8a8_model* m, int path);
+/* Diagnostic trace (no counterpart in the paper; it lets a reference check every step of every
+ * layer on the GPU's own inputs): while set, each w8a8_decoder_forward and w8a8_decoder_decode_step
+ * of M = B * T <= max_rows rows copies, for every layer l, these tensors into caller-owned DEVICE
+ * buffers laid out [layers][max_rows][width] (rows [0, M) of slice l are written; each pointer
+ * nullable):
+ *   a_in  bf16 [., ., hidden]    the q/k/v input bf16(rmsnorm(r) * ln_in)
+ *   qkv   bf16 [., ., (n_q + 2 n_kv) head_dim]
+ *   attn  bf16 [., ., n_q head_dim]   the attention output (the o projection's input)
+ *   y_o   bf16 [., ., hidden]    the o projection's output
+ *   a_ffn bf16 [., ., hidden]    the FFN block's input
+ *   h     bf16 [., ., inter]     the GeGLU output (the down projection's input)
+ *   y_f   bf16 [., ., hidden]    the FFN block's output
+ *   r     fp32 [., ., hidden]    the residual stream after the layer
+ * and a_fin bf16 [max_rows][hidden], the lm_head's input.  Tracing turns off the fusion of the
+ * residual step into the decode GEMV (the traced path computes the same values through the
+ * stand-alone residual-norm kernel).  NULL clears the trace.  Host-side, synchronous. */
+typedef struct {
+  uint16_t *a_in, *qkv, *attn, *y_o, *a_ffn, *h, *y_f;
+  float* r;
+  uint16_t* a_fin;
+  int32_t max_rows;
+} w8a8_trace;
+w8a8_status w8a8_model_set_trace(w8a8_model* m, const w8a8_trace* t);
 
 /* Measurement aid with no counterpart in the paper: *kernels = the number of kernel launches
  * one w8a8_decoder_decode_step of B sequences makes under the current mask (the kernel nodes of

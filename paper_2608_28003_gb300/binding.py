@@ -152,7 +152,6 @@ SIGNATURES = {
     "w8a8_decoder_forward": (_i32, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_decoder_decode_step": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_model_decode_kernels": (_i32, [_vp, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
-    "w8a8_model_set_decode_path": (_i32, [_vp, _i32]),
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
     "w8a8_allocate_mask": (_i32, [_vp, ctypes.POINTER(AllocOptsC), ctypes.POINTER(AllocReportC), _vp]),
@@ -691,13 +690,6 @@ class Decoder:
         _check("w8a8_decoder_decode_step", lib().w8a8_decoder_decode_step(self.h, _p(_bits(tokens)), B, int(pos),
                                                                           _p(logits), _p(top1), _stream(stream)))
         return logits, top1
-
-    DECODE_PER_STEP, DECODE_PERSISTENT = 0, 1
-
-    def set_decode_path(self, path: int) -> None:
-        """Decode steps of one sequence: one kernel per step (0, default) or the persistent all-layer
-        kernel (1)."""
-        _check("w8a8_model_set_decode_path", lib().w8a8_model_set_decode_path(self.h, int(path)))
 
     def decode_kernels(self, B: int, want_logits: bool = False) -> int:
         """Kernel launches of one decode step of B sequences under the current mask."""

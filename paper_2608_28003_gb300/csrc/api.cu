@@ -288,7 +288,7 @@ w8a8_status check_linear_args(const char* who, const w8a8_qweight* w, const uint
 
 using namespace w8a8;
 
-extern "C" int w8a8_abi_version(void) { return 1; }
+extern "C" int w8a8_abi_version(void) { return 2; }
 
 extern "C" w8a8_status w8a8_set_kernel_events(void* start_event, void* stop_event) {
   W8A8_CHECK_ARG((start_event == nullptr) == (stop_event == nullptr), W8A8_ERR_INVALID_ARG,

@@ -143,8 +143,54 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
       : "memory");
 }
 
+// Two fp32 values -> bf16x2 (a in the low half), each rounded to nearest even: one instruction.
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
-  return (uint32_t)f32_to_bf16_bits(a) | ((uint32_t)f32_to_bf16_bits(b) << 16);
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(b), "f"(a));
+  return r;
+}
+
+// 32 consecutive fp32 values p[c0 .. c0 + 31] into w, 0 past n (c0 a multiple of 32, p 16-byte
+// aligned): eight 16-byte loads when the group lies inside n.  Every lane of a warp reads the same
+// addresses (a broadcast).
+__device__ __forceinline__ void ld_cols32(const float* p, int c0, int n, float (&w)[32]) {
+  if (c0 + 32 <= n) {
+    const float4* q = reinterpret_cast<const float4*>(p + c0);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float4 t = __ldg(q + k);
+      w[4 * k] = t.x;
+      w[4 * k + 1] = t.y;
+      w[4 * k + 2] = t.z;
+      w[4 * k + 3] = t.w;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) w[j] = c0 + j < n ? __ldg(p + c0 + j) : 0.0f;
+  }
+}
+
+// The dequantising epilogue of one 32-column group: w holds s_w of the columns on entry and
+// fl(fl(s_x s_w) acc) (+ bias) on exit (Eq. gemm-final); acc is the INT32 sum (W8A8) or the fp32
+// one (FP8).
+template <typename T>
+__device__ __forceinline__ float acc_as_f32(T v);
+template <>
+__device__ __forceinline__ float acc_as_f32<int>(int v) { return __int2float_rn(v); }
+template <>
+__device__ __forceinline__ float acc_as_f32<uint32_t>(uint32_t v) { return __uint_as_float(v); }
+
+template <typename T>
+__device__ __forceinline__ void dequant32(const TcArgs& a, float sx, int c0, const T* acc, float (&w)[32]) {
+  ld_cols32(a.s_w, c0, a.N, w);
+#pragma unroll
+  for (int j = 0; j < 32; ++j) w[j] = __fmul_rn(__fmul_rn(sx, w[j]), acc_as_f32<T>(acc[j]));
+  if (a.bias) {
+    float b[32];
+    ld_cols32(a.bias, c0, a.N, b);
+#pragma unroll
+    for (int j = 0; j < 32; ++j) w[j] = __fadd_rn(w[j], b[j]);
+  }
 }
 
 // ------------------------------------------------------------------ epilogue through TMA stores
@@ -515,18 +561,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < NG; ++i) {
           const int g = part + kParts * i;
           if (g >= BN / 32) break;
-          float v[32];
+          if (a.acc_dbg && row < a.M) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int col = n0 + 32 * g + j;
-            float y = 0.0f;
-            if (col < a.N) {
-              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * i + j]));
-              if (a.bias) y = __fadd_rn(y, a.bias[col]);
-              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * i + j];
-            }
-            v[j] = y;
+            for (int j = 0; j < 32; ++j)
+              if (n0 + 32 * g + j < a.N) a.acc_dbg[(size_t)row * a.N + n0 + 32 * g + j] = isum[32 * i + j];
           }
+          float v[32];
+          dequant32(a, sx, n0 + 32 * g, &isum[32 * i], v);
           emit32(32 * g, v);
         }
       } else {
@@ -545,14 +586,17 @@ __global__ void __launch_bounds__(kThreads, 1)
               continue;
             }
             float v[32];
-            const float sx = kFp8 && row < a.M ? a.s_x[row] : 0.0f;
+            if constexpr (kFp8) {
+              dequant32(a, row < a.M ? a.s_x[row] : 0.0f, n0 + 32 * g, r, v);
+            } else {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const int col = n0 + 32 * g + j;
-              float y = __uint_as_float(r[j]);
-              if (kFp8) y = col < a.N ? __fmul_rn(__fmul_rn(sx, a.s_w[col]), y) : 0.0f;
-              if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
-              v[j] = y;
+              for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+              if (a.bias) {
+                float b[32];
+                ld_cols32(a.bias, n0 + 32 * g, a.N, b);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = __fadd_rn(v[j], b[j]);
+              }
             }
             emit32(32 * g, v);
           }
@@ -848,18 +892,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int i = 0; i < NG; ++i) {
           const int g = part + kParts * i;
           if (g >= BN / 32) break;
-          float v[32];
+          if (a.acc_dbg && row < a.M) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int col = n0 + 32 * g + j;
-            float y = 0.0f;
-            if (col < a.N) {
-              y = __fmul_rn(__fmul_rn(sx, a.s_w[col]), __int2float_rn(isum[32 * i + j]));
-              if (a.bias) y = __fadd_rn(y, a.bias[col]);
-              if (a.acc_dbg && row < a.M) a.acc_dbg[(size_t)row * a.N + col] = isum[32 * i + j];
-            }
-            v[j] = y;
+            for (int j = 0; j < 32; ++j)
+              if (n0 + 32 * g + j < a.N) a.acc_dbg[(size_t)row * a.N + n0 + 32 * g + j] = isum[32 * i + j];
           }
+          float v[32];
+          dequant32(a, sx, n0 + 32 * g, &isum[32 * i], v);
           emit(32 * g, v);
         }
       } else {
@@ -875,14 +914,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           uint32_t r[32];
           tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
           float v[32];
-          const float sx = kFp8 && row < a.M ? a.s_x[row] : 0.0f;
+          if constexpr (kFp8) {
+            dequant32(a, row < a.M ? a.s_x[row] : 0.0f, n0 + 32 * g, r, v);
+          } else {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int col = n0 + 32 * g + j;
-            float y = __uint_as_float(r[j]);
-            if (kFp8) y = col < a.N ? __fmul_rn(__fmul_rn(sx, a.s_w[col]), y) : 0.0f;
-            if (a.bias && col < a.N) y = __fadd_rn(y, a.bias[col]);
-            v[j] = y;
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+            if (a.bias) {
+              float b[32];
+              ld_cols32(a.bias, n0 + 32 * g, a.N, b);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) v[j] = __fadd_rn(v[j], b[j]);
+            }
           }
           emit(32 * g, v);
         }

@@ -9,7 +9,6 @@
 #include <utility>
 #include <vector>
 
-#include "decode_mega.cuh"
 #include "decoder_kernels.cuh"
 #include "ops.cuh"
 #include "stream_gemm.cuh"
@@ -63,17 +62,13 @@ struct w8a8_model {
   size_t ws_bytes = 0;
   void* attn_ws = nullptr;
   size_t attn_ws_bytes = 0;
-  // persistent decode kernel: per-layer descriptors (host copy kept for the asynchronous upload),
-  // phase counters, attention partials; decode_path: W8A8_DECODE_PER_STEP or W8A8_DECODE_PERSISTENT
-  std::vector<MegaLayer> mega_host;
-  MegaLayer* d_mega = nullptr;
-  unsigned int* mega_sync = nullptr;
-  float* mega_part = nullptr;
-  bool mega_ok = false;
-  int decode_path = 0;
   // diagnostics: when set, a forward copies every layer's output (the residual stream after its
   // post-FFN step, fp32 [M, H]) to capture + l M H
   float* capture = nullptr;
+  // diagnostics: when trace_on, a forward copies every layer's intermediate tensors into the
+  // caller's trace buffers (w8a8_model_set_trace)
+  bool trace_on = false;
+  w8a8_trace trace{};
 
   cudaStream_t st = nullptr;  // private stream for graph capture / replay
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
@@ -121,40 +116,6 @@ void free_all(w8a8_model* m) {
 
 w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, q.wq_f16}; }
 
-// The persistent decode kernel's per-layer descriptors (INT8 pointers once prepared), uploaded on st.
-w8a8_status upload_mega(w8a8_model* m, cudaStream_t st) {
-  const w8a8_model_cfg& c = m->cfg;
-  m->mega_host.assign(c.layers, MegaLayer{});
-  for (int l = 0; l < c.layers; ++l) {
-    const w8a8_layer_bf16& W = m->L[l];
-    MegaLayer& g = m->mega_host[l];
-    g.w16[0] = W.wqkv;
-    g.w16[1] = W.wo;
-    g.w16[2] = m->gu_bf16 + (size_t)l * 2 * c.inter * c.hidden;
-    g.w16[3] = W.wdown;
-    const QW* q[4] = {&m->q_qkv[l], &m->q_o[l], &m->q_gu[l], &m->q_down[l]};
-    for (int j = 0; j < 4; ++j) {
-      g.w8[j] = q[j]->wq;
-      g.s_w[j] = q[j]->s_w;
-      g.inv_delta[j] = q[j]->inv_delta;
-    }
-    g.ln_in = W.ln_in;
-    g.ln_post_attn = W.ln_post_attn;
-    g.ln_pre_ffn = W.ln_pre_ffn;
-    g.ln_post_ffn = W.ln_post_ffn;
-    g.q_norm = c.qk_norm ? W.q_norm : nullptr;
-    g.k_norm = c.qk_norm ? W.k_norm : nullptr;
-    const bool glob = m->is_global(l);
-    g.rope_cos = glob ? m->cos_g : m->cos_l;
-    g.rope_sin = glob ? m->sin_g : m->sin_l;
-    g.window = glob ? 0 : c.window;
-    g.kc = m->kc + (size_t)l * m->cache_layer_elems();
-    g.vc = m->vc + (size_t)l * m->cache_layer_elems();
-  }
-  W8A8_CUDA(cudaMemcpyAsync(m->d_mega, m->mega_host.data(), sizeof(MegaLayer) * c.layers, cudaMemcpyHostToDevice, st));
-  return W8A8_OK;
-}
-
 w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
                    uint16_t* Y, cudaStream_t st, const ResNorm* rn) {
   if (int8) {
@@ -168,7 +129,7 @@ w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, 
 // decode GEMV: q/k/v takes the step after the previous layer's FFN, gate/up the step after o.
 // It needs the decode GEMV to take both linears of every layer under the current mask.
 bool fuse_residual(const w8a8_model* m, int M, bool calib) {
-  if (calib || M > 8 || m->capture) return false;
+  if (calib || M > 8 || m->capture || m->trace_on) return false;
   const int H = m->cfg.hidden, F = m->cfg.inter;
   for (int l = 0; l < m->cfg.layers; ++l) {
     const bool att8 = m->prepared && ((m->attn_bits >> l) & 1u);
@@ -188,37 +149,16 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
   float* rc = m->r;   // the residual stream as of now
   float* rn = m->r2;  // where a fused update writes the next one
   W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st));
-  const bool mega =
-      !calib && !m->capture && B == 1 && T == 1 && m->mega_ok && m->decode_path == W8A8_DECODE_PERSISTENT;
-  if (mega) {  // every layer in one persistent launch, then the final residual step
-    W8A8_CUDA(cudaMemsetAsync(m->mega_sync, 0, mega_sync_words(c.layers, c.n_q) * sizeof(unsigned int), st));
-    MegaArgs g{};
-    g.layers = m->d_mega;
-    g.L = c.layers;
-    g.H = H;
-    g.F = F;
-    g.n_q = c.n_q;
-    g.n_kv = c.n_kv;
-    g.max_seq = c.max_seq;
-    g.eps = c.eps;
-    g.scale = (float)(1.0 / std::sqrt((double)c.head_dim));
-    g.attn_bits = m->prepared ? m->attn_bits : 0u;
-    g.ffn_bits = m->prepared ? m->ffn_bits : 0u;
-    g.pos = m->d_pos;
-    g.a0 = m->a;
-    g.r0 = m->r;
-    g.r1 = m->r2;
-    g.qkv = m->qkv;
-    g.att = m->o;
-    g.y = m->y;
-    g.h = m->h;
-    g.part = m->mega_part;
-    g.sync = m->mega_sync;
-    g.err = reinterpret_cast<unsigned int*>(reinterpret_cast<char*>(m->ws) + kErrWordOffset);
-    W8A8_TRY(launch_decode_mega(g, st));
-    W8A8_TRY(launch_residual_norm(m->y, M, H, m->L[c.layers - 1].ln_post_ffn, m->final_norm, c.eps, m->r2, m->a, st));
-  }
-  for (int l = 0; l < (mega ? 0 : c.layers); ++l) {
+  const w8a8_trace* tr = m->trace_on && !calib ? &m->trace : nullptr;
+  W8A8_CHECK_ARG(!tr || M <= tr->max_rows, W8A8_ERR_SHAPE, "trace: %d rows exceed the trace's %d", M, tr ? tr->max_rows : 0);
+  // copy this call's M rows of a [rows, width] tensor into slice l of a [L][max_rows][width] trace buffer
+  auto trace_copy = [&](void* base, int l, const void* src, int width, size_t elem) -> w8a8_status {
+    if (!base) return W8A8_OK;
+    char* dst = static_cast<char*>(base) + ((size_t)l * tr->max_rows) * width * elem;
+    W8A8_CUDA(cudaMemcpyAsync(dst, src, (size_t)M * width * elem, cudaMemcpyDeviceToDevice, st));
+    return W8A8_OK;
+  };
+  for (int l = 0; l < c.layers; ++l) {
     const w8a8_layer_bf16& W = m->L[l];
     const bool att8 = !calib && m->prepared && ((m->attn_bits >> l) & 1u);
     const bool ffn8 = !calib && m->prepared && ((m->ffn_bits >> l) & 1u);
@@ -229,7 +169,9 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
       W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, nullptr, M, m->qkv, st, &R));
       std::swap(rc, rn);
     } else {
+      if (tr) W8A8_TRY(trace_copy(tr->a_in, l, m->a, H, 2));
       W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
+      if (tr) W8A8_TRY(trace_copy(tr->qkv, l, m->qkv, m->qkv_dim, 2));
     }
     AttnShape s{B, T, c.n_q, c.n_kv, c.head_dim, c.max_seq, glob ? 0 : c.window,
                 (float)(1.0 / std::sqrt((double)c.head_dim))};
@@ -249,7 +191,9 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
         W8A8_TRY(launch_attention(m->q, kc, vc, s, m->d_pos, 0, m->o, m->attn_ws, m->sms, st));
     }
     if (calib) W8A8_TRY(launch_act_absmax(m->o, M, m->q_dim, m->stat_o(l), st));
+    if (tr) W8A8_TRY(trace_copy(tr->attn, l, m->o, m->q_dim, 2));
     W8A8_TRY(linear(m, att8, m->q_o[l], W.wo, H, m->q_dim, m->o, M, m->y, st, nullptr));
+    if (tr) W8A8_TRY(trace_copy(tr->y_o, l, m->y, H, 2));
     w8a8_ffn_weights f{H,
                        F,
                        qdesc(m->q_gu[l], 2 * F, H),
@@ -264,7 +208,11 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     } else {
       W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, rc, m->a, st));
       if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
-      W8A8_TRY(run_ffn(&f, prec, m->a, M, m->y, calib ? m->h : nullptr, m->ws, m->sms, st));
+      if (tr) W8A8_TRY(trace_copy(tr->a_ffn, l, m->a, H, 2));
+      uint16_t* h_out = calib ? m->h : nullptr;
+      if (tr && tr->h) h_out = tr->h + (size_t)l * tr->max_rows * F;  // the block writes h there
+      W8A8_TRY(run_ffn(&f, prec, m->a, M, m->y, h_out, m->ws, m->sms, st));
+      if (tr) W8A8_TRY(trace_copy(tr->y_f, l, m->y, H, 2));
     }
     if (calib) W8A8_TRY(launch_act_absmax(m->h, M, F, m->stat_down(l), st));
     if (!fuse || l + 1 == c.layers) {
@@ -273,7 +221,9 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     }
     if (m->capture)
       W8A8_CUDA(cudaMemcpyAsync(m->capture + (size_t)l * M * H, rc, sizeof(float) * M * H, cudaMemcpyDeviceToDevice, st));
+    if (tr) W8A8_TRY(trace_copy(tr->r, l, rc, H, 4));
   }
+  if (tr) W8A8_TRY(trace_copy(tr->a_fin, 0, m->a, H, 2));
   if (calib) return launch_act_absmax(m->a, M, H, m->stat_lm(), st);
   const bool lm8 = m->prepared && m->lm;
   for (int r0 = 0; r0 < M; r0 += kHeadChunk) {
@@ -479,13 +429,6 @@ extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_l
   W8A8_MTRY(launch_rope_table(m->cos_g, m->sin_g, c.max_seq, c.head_dim, c.rope_global, st));
   for (int l = 0; l < c.layers; ++l)
     W8A8_MTRY(w8a8_interleave_gate_up(layers[l].wgate, layers[l].wup, F, H, m->gu_bf16 + (size_t)l * 2 * F * H, st));
-  m->mega_ok = decode_mega_supported(H, F, c.n_q, c.n_kv, c.head_dim, d.sms);
-  if (m->mega_ok) {
-    W8A8_MTRY(dalloc(m, &m->d_mega, (size_t)c.layers));
-    W8A8_MTRY(dalloc(m, &m->mega_sync, mega_sync_words(c.layers, c.n_q)));
-    W8A8_MTRY(dalloc(m, &m->mega_part, mega_part_floats(c.n_q)));
-    W8A8_MTRY(upload_mega(m, st));
-  }
   W8A8_MTRY(cudaStreamSynchronize(st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
 #undef W8A8_MTRY
   *out = m;
@@ -572,10 +515,6 @@ extern "C" w8a8_status w8a8_model_prepare(w8a8_model* m, float alpha, int smooth
                                 m->q_lm.delta, m->q_lm.inv_delta, m->q_lm.wq_f16, stream));
   m->prepared = true;
   ++m->prep_version;
-  if (m->mega_ok) {
-    W8A8_TRY(upload_mega(m, as_stream(stream)));
-    W8A8_CUDA(cudaStreamSynchronize(as_stream(stream)));  // the host copy may be rewritten next time
-  }
   return W8A8_OK;
 }
 
@@ -642,7 +581,17 @@ extern "C" w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* to
   W8A8_CUDA(cudaMemcpyAsync(m->d_tokens, tokens, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice, st));
   W8A8_TRY(launch_set_int(m->d_pos, pos, st));
   const int want_logits = logits != nullptr;
-  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0) | (m->decode_path << 2),
+  if (m->trace_on) {  // traced steps run eagerly (a cached graph holds no trace copies)
+    W8A8_TRY(forward_core(m, m->d_tokens, B, 1, want_logits ? m->d_logits : nullptr, m->d_top1, false, st));
+    W8A8_CUDA(cudaMemcpyAsync(top1, m->d_top1, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice, st));
+    if (logits)
+      W8A8_CUDA(cudaMemcpyAsync(logits, m->d_logits, sizeof(float) * B * (size_t)m->cfg.vocab,
+                                cudaMemcpyDeviceToDevice, st));
+    W8A8_CUDA(cudaEventRecord(m->ev_out, st));
+    W8A8_CUDA(cudaStreamWaitEvent(user, m->ev_out, 0));
+    return W8A8_OK;
+  }
+  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0),
                                    m->prep_version, want_logits);
   auto it = m->graphs.find(key);
   if (it == m->graphs.end()) {
@@ -681,17 +630,25 @@ extern "C" w8a8_status w8a8_decoder_decode_step(w8a8_model* m, const int32_t* to
   return W8A8_OK;
 }
 
-extern "C" w8a8_status w8a8_model_set_decode_path(w8a8_model* m, int path) {
-  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "null model");
-  W8A8_CHECK_ARG(path == W8A8_DECODE_PERSISTENT || path == W8A8_DECODE_PER_STEP, W8A8_ERR_INVALID_ARG,
-                 "w8a8_model_set_decode_path: path %d", path);
-  m->decode_path = path;
+extern "C" w8a8_status w8a8_model_set_trace(w8a8_model* m, const w8a8_trace* t) {
+  W8A8_CHECK_ARG(m, W8A8_ERR_INVALID_ARG, "w8a8_model_set_trace: null model");
+  if (!t) {
+    m->trace_on = false;
+    m->trace = w8a8_trace{};
+    return W8A8_OK;
+  }
+  W8A8_CHECK_ARG(t->max_rows > 0, W8A8_ERR_INVALID_ARG, "w8a8_model_set_trace: max_rows must be positive");
+  const void* ptrs[] = {t->a_in, t->qkv, t->attn, t->y_o, t->a_ffn, t->h, t->y_f, t->r, t->a_fin};
+  for (const void* p : ptrs)
+    W8A8_CHECK_ARG(!p || aligned16(p), W8A8_ERR_ALIGN, "w8a8_model_set_trace: buffers must be 16-byte aligned");
+  m->trace = *t;
+  m->trace_on = true;
   return W8A8_OK;
 }
 
 extern "C" w8a8_status w8a8_model_decode_kernels(const w8a8_model* m, int B, int want_logits, int* kernels) {
   W8A8_CHECK_ARG(m && kernels, W8A8_ERR_INVALID_ARG, "w8a8_model_decode_kernels: null argument");
-  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0) | (m->decode_path << 2),
+  const auto key = std::make_tuple(B, m->ffn_bits, m->attn_bits, m->lm | (m->prepared ? 2 : 0),
                                    m->prep_version, want_logits ? 1 : 0);
   const auto it = m->graphs.find(key);
   W8A8_CHECK_ARG(it != m->graphs.end(), W8A8_ERR_INVALID_ARG,

@@ -40,7 +40,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_error_channel(lib):
-    assert lib.abi_version() == 1
+    assert lib.abi_version() == 2
     assert isinstance(lib.lib().w8a8_last_error(), bytes)
 
 

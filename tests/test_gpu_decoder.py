@@ -199,57 +199,6 @@ def test_decode_kernel_count(B, setup):
     assert counts[(0b1001, 0b0010, 1)] - counts[(0, 0, 0)] == 1
 
 
-@pytest.mark.parametrize("mask", [OM.make_mask(), OM.Mask(frozenset({0, 3}), frozenset({1}), True)],
-                         ids=["bf16", "mixed"])
-def test_persistent_decode_matches_oracle(B, setup, mask):
-    """One sequence: decode steps through the persistent all-layer kernel and through the per-step
-    kernels, both against the oracle (batch 1, the same prepared weights) at positions 24..27,
-    which cross the sliding window of 8 on layers 1..3."""
-    dec, od, toks = setup[:3]
-    od1 = OD.OracleDecoder(od.cfg, od.w, batch=1, max_len=64)
-    od1.prep, od1.stats = od.prep, od.stats
-    fb, ab, lm = mask.bits()
-    dec.set_mask(fb, ab, lm)
-    t1 = np.ascontiguousarray(toks[:1])
-    ref_all, sens = _sensitivity(od1, t1, 28, mask)
-    tt = torch.from_numpy(t1).cuda()
-    buf = torch.empty(1, V, dtype=torch.float32, device="cuda")
-    outs = {}
-    try:
-        for path in (dec.DECODE_PER_STEP, dec.DECODE_PERSISTENT):
-            dec.set_decode_path(path)
-            dec.forward(tt[:, :24].contiguous(), 0, want_logits=False)
-            rows = []
-            for s in range(4):
-                lg, t = dec.decode_step(tt[:, 24 + s].contiguous(), 24 + s, logits=buf)
-                rows.append(lg.cpu().numpy()[0])
-                assert int(t.item()) == int(np.argmax(rows[-1]))
-            outs[path] = np.stack(rows)
-    finally:
-        dec.set_decode_path(dec.DECODE_PER_STEP)
-    for path in outs:
-        _close(outs[path], ref_all[0, 24:28], sens[0, 24:28])
-
-
-def test_persistent_decode_kernel_count(B, setup):
-    """Batch 1 on the persistent path: the position update, embedding + norm, the persistent kernel
-    for all layers, the last residual step and lm_head (W8A8 lm_head adds its quantiser)."""
-    dec, _, toks = setup[:3]
-    col = torch.from_numpy(toks[:1, 21].copy()).cuda()
-    buf = torch.empty(1, V, dtype=torch.float32, device="cuda")
-    counts = {}
-    dec.set_decode_path(dec.DECODE_PERSISTENT)
-    try:
-        for m in [(0, 0, 0), (0b1001, 0b0010, 1)]:
-            dec.set_mask(*m)
-            dec.decode_step(col, 21, logits=buf)
-            counts[m] = dec.decode_kernels(1, want_logits=True)
-    finally:
-        dec.set_decode_path(dec.DECODE_PER_STEP)
-    assert counts[(0, 0, 0)] == 5
-    assert counts[(0b1001, 0b0010, 1)] == 6
-
-
 def test_mask_controls(B, setup):
     dec = setup[0]
     dec.set_mask(0, 0, 0)
