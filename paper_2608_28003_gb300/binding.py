@@ -77,6 +77,11 @@ class LayerBf16C(ctypes.Structure):
                 ("ln_post_attn", _vp), ("ln_pre_ffn", _vp), ("ln_post_ffn", _vp), ("q_norm", _vp), ("k_norm", _vp)]
 
 
+class TraceC(ctypes.Structure):
+    _fields_ = [("a_in", _vp), ("qkv", _vp), ("attn", _vp), ("y_o", _vp), ("a_ffn", _vp), ("h", _vp), ("y_f", _vp),
+                ("r", _vp), ("a_fin", _vp), ("max_rows", ctypes.c_int32)]
+
+
 class MaskC(ctypes.Structure):
     _fields_ = [("ffn_bits", ctypes.c_uint32), ("attn_bits", ctypes.c_uint32), ("lm", ctypes.c_int32)]
 
@@ -152,6 +157,7 @@ SIGNATURES = {
     "w8a8_decoder_forward": (_i32, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_decoder_decode_step": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_model_decode_kernels": (_i32, [_vp, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
+    "w8a8_model_set_trace": (_i32, [_vp, ctypes.POINTER(TraceC)]),
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
     "w8a8_allocate_mask": (_i32, [_vp, ctypes.POINTER(AllocOptsC), ctypes.POINTER(AllocReportC), _vp]),
@@ -690,6 +696,28 @@ class Decoder:
         _check("w8a8_decoder_decode_step", lib().w8a8_decoder_decode_step(self.h, _p(_bits(tokens)), B, int(pos),
                                                                           _p(logits), _p(top1), _stream(stream)))
         return logits, top1
+
+    TRACE_FIELDS = ("a_in", "qkv", "attn", "y_o", "a_ffn", "h", "y_f", "r", "a_fin")
+
+    def set_trace(self, max_rows: Optional[int]):
+        """Start tracing every layer's intermediate tensors of the following forward / decode calls
+        (rows [0, M) of each call) into fresh device tensors, returned as a dict; None stops."""
+        if max_rows is None:
+            _check("w8a8_model_set_trace", lib().w8a8_model_set_trace(self.h, None))
+            self._trace = None
+            return None
+        c, L, R = self.cfg, self.cfg.layers, int(max_rows)
+        qkv = (c.n_q + 2 * c.n_kv) * c.head_dim
+        dev = self._keep[0]["embed"].device
+        bf = lambda w: torch.empty(L, R, w, dtype=torch.bfloat16, device=dev)  # noqa: E731
+        t = {"a_in": bf(c.hidden), "qkv": bf(qkv), "attn": bf(c.n_q * c.head_dim), "y_o": bf(c.hidden),
+             "a_ffn": bf(c.hidden), "h": bf(c.inter), "y_f": bf(c.hidden),
+             "r": torch.empty(L, R, c.hidden, dtype=torch.float32, device=dev),
+             "a_fin": torch.empty(R, c.hidden, dtype=torch.bfloat16, device=dev)}
+        tc = TraceC(*(t[k].data_ptr() for k in self.TRACE_FIELDS), R)
+        _check("w8a8_model_set_trace", lib().w8a8_model_set_trace(self.h, ctypes.byref(tc)))
+        self._trace = t
+        return t
 
     def decode_kernels(self, B: int, want_logits: bool = False) -> int:
         """Kernel launches of one decode step of B sequences under the current mask."""

@@ -136,6 +136,39 @@ static bool small_gemv(bool int8, const void* W, const float* inv_delta, const f
   return true;
 }
 
+// The one-token q/k/v projection with the decode attention of its sequence as the GEMV's tail
+// (W8A8_ERR_SHAPE when the decode GEMV's plan for this shape cannot carry the tail).
+w8a8_status run_qkv_attention(bool int8, const void* W, const float* inv_delta, const float* s_w, int N, int K,
+                              const ResNorm* rn, const uint16_t* X, uint16_t* Y, const AttnTail& tail, void* ws,
+                              int sms, cudaStream_t st) {
+  SmallArgs a{};
+  a.p = make_small_plan(int8 ? SMALL_INT8 : SMALL_BF16, 1, N, K, EPI_BF16, sms, rn != nullptr);
+  W8A8_CHECK_ARG(a.p.ok && a.p.MT == 1 && a.p.RW == 1, W8A8_ERR_SHAPE, "q/k/v with attention: no plan for N=%d K=%d",
+                 N, K);
+  if (rn) {
+    a.has_rn = 1;
+    a.rn = *rn;
+  }
+  a.W = W;
+  a.X = X;
+  a.M = 1;
+  a.N = N;
+  a.K = K;
+  a.kind = EPI_BF16;
+  a.inv_delta = inv_delta;
+  a.s_w = s_w;
+  a.y = Y;
+  a.err = err_word(ws);
+  a.has_tail = 1;
+  a.tail = tail;
+  return launch_small_gemv(int8 ? SMALL_INT8 : SMALL_BF16, a, st);
+}
+
+bool qkv_attention_takes(bool int8, int N, int K, int sms) {
+  const SmallPlan p = make_small_plan(int8 ? SMALL_INT8 : SMALL_BF16, 1, N, K, EPI_BF16, sms, true);
+  return p.ok && p.MT == 1 && p.RW == 1;
+}
+
 bool decode_gemv_takes(bool int8, int M, int N, int K, bool geglu, int sms) {
   return make_small_plan(int8, M, N, K, geglu ? EPI_GEGLU : EPI_BF16, sms, true).ok != 0;
 }

@@ -93,9 +93,10 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
   x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
 }
 
-template <int kW, int MT, int RW>
+template <int kW, int MT, int RW, bool kTail = false>
 __global__ void __launch_bounds__(kThreads, 2)
     gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
+  static_assert(!kTail || (MT == 1 && RW == 1), "the attention tail follows the one-token q/k/v projection");
   // kW: weights bf16 (SMALL_BF16), INT8 codes (SMALL_INT8) or e4m3 codes (SMALL_FP8, 8 slots only)
   constexpr bool kInt8 = kW == SMALL_INT8, kFp8 = kW == SMALL_FP8;
   constexpr bool kQ = kInt8 || kFp8;  // one-byte codes, per-token K1, dequantising epilogue
@@ -683,7 +684,10 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     return;
   }
-  if (!ok) return;
+  if (!ok) {
+    if constexpr (kTail) attn_tail(a.tail, a.y, smem_raw + a.p.smem_bytes, 1, a.err);  // keeps the tickets whole
+    return;
+  }
 #pragma unroll
   for (int c = 1; c < NA; ++c)  // fixed order: ((a0 + a1) + a2) + a3
 #pragma unroll
@@ -699,52 +703,59 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) acc[0][i][m] += __shfl_xor_sync(0xffffffffu, acc[0][i][m], o);
     }
-  if (lane != 0) return;
-
-  auto value = [&](Acc v, int i, int row, int m) -> float {  // i: the warp's row slot of `row`
-    float y;
-    if constexpr (kInt8) {
-      y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), __int2float_rn(v));
-      if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row] = v;
-    } else {
-      y = v;
-    }
-    return a.bias ? __fadd_rn(y, bir[i]) : y;
-  };
-  if (a.kind == EPI_GEGLU) {
-#pragma unroll
-    for (int j = 0; j < RW / 2; ++j) {
-      const int gi = row0 + 16 * j + warp, ui = gi + 8;
-      if (ui >= a.N) continue;
-      const int hid = ((row0 + 16 * j) >> 1) + warp;
-#pragma unroll
-      for (int m = 0; m < MT; ++m) {
-        if (m >= a.M) break;
-        const float g = value(acc[0][2 * j][m], 2 * j, gi, m), u = value(acc[0][2 * j + 1][m], 2 * j + 1, ui, m);
-        a.y[(size_t)m * (a.N >> 1) + hid] = f32_to_bf16_bits(geglu_recipe(g, u));
+  if constexpr (!kTail) {
+    if (lane != 0) return;
+  }
+  if (lane == 0) {  // the epilogue (the whole warp reaches the attention tail after it)
+    auto value = [&](Acc v, int i, int row, int m) -> float {  // i: the warp's row slot of `row`
+      float y;
+      if constexpr (kInt8) {
+        y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), __int2float_rn(v));
+        if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row] = v;
+      } else {
+        y = v;
       }
-    }
-  } else {
+      return a.bias ? __fadd_rn(y, bir[i]) : y;
+    };
+    if (a.kind == EPI_GEGLU) {
 #pragma unroll
-    for (int i = 0; i < RW; ++i) {
-      const int row = row0 + warp + 8 * i;
-      if (row >= a.N) continue;
+      for (int j = 0; j < RW / 2; ++j) {
+        const int gi = row0 + 16 * j + warp, ui = gi + 8;
+        if (ui >= a.N) continue;
+        const int hid = ((row0 + 16 * j) >> 1) + warp;
 #pragma unroll
-      for (int m = 0; m < MT; ++m) {
-        if (m >= a.M) break;
-        a.y[(size_t)m * a.N + row] = f32_to_bf16_bits(value(acc[0][i][m], i, row, m));
+        for (int m = 0; m < MT; ++m) {
+          if (m >= a.M) break;
+          const float g = value(acc[0][2 * j][m], 2 * j, gi, m), u = value(acc[0][2 * j + 1][m], 2 * j + 1, ui, m);
+          a.y[(size_t)m * (a.N >> 1) + hid] = f32_to_bf16_bits(geglu_recipe(g, u));
+        }
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < RW; ++i) {
+        const int row = row0 + warp + 8 * i;
+        if (row >= a.N) continue;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+          if (m >= a.M) break;
+          a.y[(size_t)m * a.N + row] = f32_to_bf16_bits(value(acc[0][i][m], i, row, m));
+        }
       }
     }
   }
+  if constexpr (kTail) {
+    __syncwarp();
+    attn_tail(a.tail, a.y, smem_raw + a.p.smem_bytes, 1, a.err);
+  }
 }
 
-template <int kW, int MT, int RW>
+template <int kW, int MT, int RW, bool kTail = false>
 w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW, kTail>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    kSmemLimit - kStatic));
     attr_set[dev] = true;
   }
@@ -754,7 +765,9 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 8 * RW, 128));
   else
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
-  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
+  const size_t smem = (size_t)a.p.smem_bytes + (kTail ? (size_t)kTailSmem : 0);  // the tail's region follows
+  W8A8_CHECK_ARG(smem <= (size_t)(kSmemLimit - kStatic), W8A8_ERR_SHAPE, "small GEMV: %zu bytes of shared memory", smem);
+  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW, kTail>, dim3(a.p.P), dim3(kThreads), smem, st, tw,
                        a));
   return W8A8_OK;
 }
@@ -857,9 +870,17 @@ w8a8_status launch_small_gemv(int wkind, const SmallArgs& a, cudaStream_t st) {
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  const w8a8_status s = wkind == SMALL_FP8    ? launch_typed<SMALL_FP8>(a, st)
-                        : wkind == SMALL_INT8 ? launch_typed<SMALL_INT8>(a, st)
-                                              : launch_typed<SMALL_BF16>(a, st);
+  w8a8_status s;
+  if (a.has_tail) {
+    W8A8_CHECK_ARG(wkind != SMALL_FP8 && a.M == 1 && a.p.MT == 1 && a.p.RW == 1 && a.tail.n_q >= 1 &&
+                       a.tail.n_q <= kTailMaxG && 8 % a.tail.n_q == 0,
+                   W8A8_ERR_SHAPE, "small GEMV: the attention tail needs one token, one row per warp, 1-4 heads");
+    s = wkind == SMALL_INT8 ? launch_t<SMALL_INT8, 1, 1, true>(a, st) : launch_t<SMALL_BF16, 1, 1, true>(a, st);
+  } else {
+    s = wkind == SMALL_FP8    ? launch_typed<SMALL_FP8>(a, st)
+        : wkind == SMALL_INT8 ? launch_typed<SMALL_INT8>(a, st)
+                              : launch_typed<SMALL_BF16>(a, st);
+  }
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }

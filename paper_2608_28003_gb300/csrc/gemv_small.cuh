@@ -3,6 +3,7 @@
 // variant, and the bf16 pass-through.
 #pragma once
 
+#include "attn_tail.cuh"
 #include "common.cuh"
 
 namespace w8a8 {
@@ -58,6 +59,8 @@ struct SmallArgs {
   ResNorm rn;
   unsigned int* err;       // device error word
   SmallPlan p;
+  int has_tail;            // 1: the decode attention of one sequence runs as this GEMV's tail (q/k/v
+  AttnTail tail;           //    projection at one token; the plan must have one token slot, one row per warp)
 };
 
 // fused_norm: the call computes its input with a ResNorm (needs K <= 2048)

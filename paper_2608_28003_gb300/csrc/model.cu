@@ -62,6 +62,9 @@ struct w8a8_model {
   size_t ws_bytes = 0;
   void* attn_ws = nullptr;
   size_t attn_ws_bytes = 0;
+  // decode attention of one sequence as the tail of the q/k/v GEMV: two tickets (zero between
+  // launches), then the attention CTAs' partials
+  unsigned char* tail_ws = nullptr;
   // diagnostics: when set, a forward copies every layer's output (the residual stream after its
   // post-FFN step, fp32 [M, H]) to capture + l M H
   float* capture = nullptr;
@@ -140,6 +143,16 @@ bool fuse_residual(const w8a8_model* m, int M, bool calib) {
   return true;
 }
 
+// Whether the decode attention of this call can run as the q/k/v GEMV's tail: one sequence at one
+// token, one key/value head of 256 shared by 1, 2 or 4 query heads, and a decode-GEMV plan for q/k/v
+// with one row per warp.
+bool attn_tail_ok(const w8a8_model* m, bool att8, int B, int T) {
+  const w8a8_model_cfg& c = m->cfg;
+  if (B != 1 || T != 1 || c.n_kv != 1 || c.head_dim != kAttnHd) return false;
+  if (c.n_q != 1 && c.n_q != 2 && c.n_q != 4) return false;
+  return qkv_attention_takes(att8, m->qkv_dim, c.hidden, m->sms);
+}
+
 // The decoder over M = B * T rows whose positions start at *m->d_pos (set by the caller).
 w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, float* logits, int32_t* top1, bool calib,
                          cudaStream_t st) {
@@ -164,15 +177,6 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     const bool ffn8 = !calib && m->prepared && ((m->ffn_bits >> l) & 1u);
     const bool glob = m->is_global(l);
     if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_qkv(l), st));
-    if (fuse && l > 0) {  // the previous layer's post-FFN step, then q/k/v
-      const ResNorm R{m->y, rc, rn, m->L[l - 1].ln_post_ffn, W.ln_in, c.eps};
-      W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, nullptr, M, m->qkv, st, &R));
-      std::swap(rc, rn);
-    } else {
-      if (tr) W8A8_TRY(trace_copy(tr->a_in, l, m->a, H, 2));
-      W8A8_TRY(linear(m, att8, m->q_qkv[l], W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
-      if (tr) W8A8_TRY(trace_copy(tr->qkv, l, m->qkv, m->qkv_dim, 2));
-    }
     AttnShape s{B, T, c.n_q, c.n_kv, c.head_dim, c.max_seq, glob ? 0 : c.window,
                 (float)(1.0 / std::sqrt((double)c.head_dim))};
     uint16_t* kc = m->kc + (size_t)l * m->cache_layer_elems();
@@ -181,7 +185,31 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     const float* kn = c.qk_norm ? W.k_norm : nullptr;
     const float* cs = glob ? m->cos_g : m->cos_l;
     const float* sn = glob ? m->sin_g : m->sin_l;
-    if (attn_decode_supported(s)) {
+    // one sequence at one token: the attention runs as the q/k/v GEMV's tail (no separate launch)
+    const bool tail = !calib && attn_tail_ok(m, att8, B, T);
+    const AttnTail at{c.n_q, glob ? 0 : c.window, c.max_seq, s.scale, c.eps, m->d_pos, qn, kn, cs, sn, kc, vc, m->o,
+                      reinterpret_cast<float*>(m->tail_ws + 256), reinterpret_cast<unsigned int*>(m->tail_ws)};
+    const QW& qq = m->q_qkv[l];
+    if (fuse && l > 0) {  // the previous layer's post-FFN step, then q/k/v
+      const ResNorm R{m->y, rc, rn, m->L[l - 1].ln_post_ffn, W.ln_in, c.eps};
+      if (tail)
+        W8A8_TRY(run_qkv_attention(att8, att8 ? (const void*)qq.wq : (const void*)W.wqkv, qq.inv_delta, qq.s_w,
+                                   m->qkv_dim, H, &R, nullptr, m->qkv, at, m->ws, m->sms, st));
+      else
+        W8A8_TRY(linear(m, att8, qq, W.wqkv, m->qkv_dim, H, nullptr, M, m->qkv, st, &R));
+      std::swap(rc, rn);
+    } else {
+      if (tr) W8A8_TRY(trace_copy(tr->a_in, l, m->a, H, 2));
+      if (tail)
+        W8A8_TRY(run_qkv_attention(att8, att8 ? (const void*)qq.wq : (const void*)W.wqkv, qq.inv_delta, qq.s_w,
+                                   m->qkv_dim, H, nullptr, m->a, m->qkv, at, m->ws, m->sms, st));
+      else
+        W8A8_TRY(linear(m, att8, qq, W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
+      if (tr) W8A8_TRY(trace_copy(tr->qkv, l, m->qkv, m->qkv_dim, 2));
+    }
+    if (tail) {
+      // the attention ran inside the q/k/v launch
+    } else if (attn_decode_supported(s)) {
       W8A8_TRY(launch_attn_decode(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, kc, vc, m->o, st));
     } else {
       W8A8_TRY(launch_qk_rope(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, m->q, kc, vc, st));
@@ -419,9 +447,11 @@ extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_l
   }
   m->attn_ws_bytes = aws;
   W8A8_MTRY(dalloc(m, reinterpret_cast<char**>(&m->attn_ws), aws));
+  W8A8_MTRY(dalloc(m, &m->tail_ws, kTailScratchBytes));
   cudaStream_t st = m->st;
   W8A8_MTRY(cudaMemsetAsync(m->ws, 0, W8A8_WS_RESERVED, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
   W8A8_MTRY(cudaMemsetAsync(m->attn_ws, 0, aws, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
+  W8A8_MTRY(cudaMemsetAsync(m->tail_ws, 0, kTailScratchBytes, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
   W8A8_MTRY(cudaMemsetAsync(m->stats, 0, ((size_t)c.layers * m->stats_stride() + H) * 4, st) == cudaSuccess
                 ? W8A8_OK
                 : W8A8_ERR_CUDA);

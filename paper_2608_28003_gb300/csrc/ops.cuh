@@ -40,5 +40,11 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
 // rn (decode only): the call's input is computed from the decoder's residual step inside the
 // decode GEMV (X is ignored); W8A8_ERR_SHAPE when the decode GEMV does not take the call.
 bool decode_gemv_takes(bool int8, int M, int N, int K, bool geglu, int sms);
+// The one-token q/k/v projection followed, in the same launch, by the decode attention of its
+// sequence (tail of the decode GEMV); rn as above (nullable), X ignored when rn is given.
+w8a8_status run_qkv_attention(bool int8, const void* W, const float* inv_delta, const float* s_w, int N, int K,
+                              const ResNorm* rn, const uint16_t* X, uint16_t* Y, const AttnTail& tail, void* ws,
+                              int sms, cudaStream_t st);
+bool qkv_attention_takes(bool int8, int N, int K, int sms);
 
 }  // namespace w8a8

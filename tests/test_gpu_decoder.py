@@ -199,6 +199,37 @@ def test_decode_kernel_count(B, setup):
     assert counts[(0b1001, 0b0010, 1)] - counts[(0, 0, 0)] == 1
 
 
+@pytest.mark.parametrize("mask", [OM.make_mask(), OM.Mask(frozenset({0, 3}), frozenset({1}), True)],
+                         ids=["bf16", "mixed"])
+def test_single_sequence_decode_matches_oracle(B, setup, mask):
+    """One sequence: the decode step runs its attention as the tail of the q/k/v GEMV (no attention
+    launch) with the residual step fused into q/k/v and gate/up; positions 24..27 cross the sliding
+    window of 8 on layers 1..3.  Against the oracle at batch 1 with the same prepared weights; the
+    graph replay equals an eager step; a step launches the position update, embedding + norm, four
+    kernels per layer, the last residual step and lm_head (W8A8 lm_head adds its quantiser)."""
+    dec, od, toks = setup[:3]
+    od1 = OD.OracleDecoder(od.cfg, od.w, batch=1, max_len=64)
+    od1.prep, od1.stats = od.prep, od.stats
+    fb, ab, lm = mask.bits()
+    dec.set_mask(fb, ab, lm)
+    t1 = np.ascontiguousarray(toks[:1])
+    ref_all, sens = _sensitivity(od1, t1, 28, mask)
+    tt = torch.from_numpy(t1).cuda()
+    buf = torch.empty(1, V, dtype=torch.float32, device="cuda")
+    dec.forward(tt[:, :24].contiguous(), 0, want_logits=False)
+    rows = []
+    for s in range(4):
+        lg, t = dec.decode_step(tt[:, 24 + s].contiguous(), 24 + s, logits=buf)
+        rows.append(lg.cpu().numpy()[0])
+        assert int(t.item()) == int(np.argmax(rows[-1]))
+    _close(np.stack(rows), ref_all[0, 24:28], sens[0, 24:28])
+    lg2, _ = dec.decode_step(tt[:, 27].contiguous(), 27, logits=buf)  # replayed at the same position
+    assert np.array_equal(lg2.cpu().numpy()[0], rows[-1])
+    lg3, _ = dec.forward(tt[:, 27:28].contiguous(), 27)  # eager forward of the same step
+    assert np.array_equal(lg3.cpu().numpy()[0], rows[-1])
+    assert dec.decode_kernels(1, want_logits=True) == 2 + 4 * L + 2 + (1 if lm else 0)
+
+
 def test_mask_controls(B, setup):
     dec = setup[0]
     dec.set_mask(0, 0, 0)
