@@ -136,39 +136,6 @@ static bool small_gemv(bool int8, const void* W, const float* inv_delta, const f
   return true;
 }
 
-// The one-token q/k/v projection with the decode attention of its sequence as the GEMV's tail
-// (W8A8_ERR_SHAPE when the decode GEMV's plan for this shape cannot carry the tail).
-w8a8_status run_qkv_attention(bool int8, const void* W, const float* inv_delta, const float* s_w, int N, int K,
-                              const ResNorm* rn, const uint16_t* X, uint16_t* Y, const AttnTail& tail, void* ws,
-                              int sms, cudaStream_t st) {
-  SmallArgs a{};
-  a.p = make_small_plan(int8 ? SMALL_INT8 : SMALL_BF16, 1, N, K, EPI_BF16, sms, rn != nullptr);
-  W8A8_CHECK_ARG(a.p.ok && a.p.MT == 1 && a.p.RW == 1, W8A8_ERR_SHAPE, "q/k/v with attention: no plan for N=%d K=%d",
-                 N, K);
-  if (rn) {
-    a.has_rn = 1;
-    a.rn = *rn;
-  }
-  a.W = W;
-  a.X = X;
-  a.M = 1;
-  a.N = N;
-  a.K = K;
-  a.kind = EPI_BF16;
-  a.inv_delta = inv_delta;
-  a.s_w = s_w;
-  a.y = Y;
-  a.err = err_word(ws);
-  a.has_tail = 1;
-  a.tail = tail;
-  return launch_small_gemv(int8 ? SMALL_INT8 : SMALL_BF16, a, st);
-}
-
-bool qkv_attention_takes(bool int8, int N, int K, int sms) {
-  const SmallPlan p = make_small_plan(int8 ? SMALL_INT8 : SMALL_BF16, 1, N, K, EPI_BF16, sms, true);
-  return p.ok && p.MT == 1 && p.RW == 1;
-}
-
 bool decode_gemv_takes(bool int8, int M, int N, int K, bool geglu, int sms) {
   return make_small_plan(int8, M, N, K, geglu ? EPI_GEGLU : EPI_BF16, sms, true).ok != 0;
 }
@@ -184,12 +151,16 @@ constexpr int kTcMinTokens = 64, kTcMinTokensNarrow = 9, kTcNarrowMaxN = 16384;
 static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N, int K, const float* bias, int kind,
                     const float* inv_delta, const float* s_w, uint16_t* Y, float* logits, int32_t* top1,
                     const w8a8_debug* dbg, void* ws, void* codes, float* s_x, void* part, cudaStream_t st,
-                    w8a8_status* status) {
+                    w8a8_status* status, const PreCodes* pre = nullptr) {
   if (M < (N <= kTcNarrowMaxN ? kTcMinTokensNarrow : kTcMinTokens) || !W16 ||
       !tc_gemm_supported(M, N, K, kind, top1 != nullptr, max_top_keys()))
     return false;
   TcArgs a{};
-  if (int8) {
+  if (int8 && pre && pre->codes16 && !dbg) {  // the producer of X quantised it already
+    a.A = pre->codes16;
+    a.s_x = pre->s_x;
+    a.s_w = s_w;
+  } else if (int8) {
     w8a8_status q = launch_quantize_rows(X, M, K, inv_delta, dbg ? dbg->xq : nullptr,
                                          reinterpret_cast<uint16_t*>(codes), s_x, st);
     if (q == W8A8_OK && dbg && dbg->s_x)
@@ -230,7 +201,7 @@ static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N,
 // One W8A8 linear: K1 then the streaming GEMM.  s_x and the codes live in the workspace.
 w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, const float* bias, int kind,
                                    uint16_t* Y, float* logits, int32_t* top1, const w8a8_debug* dbg, void* ws,
-                                   int sms, cudaStream_t st, const ResNorm* rn) {
+                                   int sms, cudaStream_t st, const ResNorm* rn, const PreCodes* pre) {
   const int N = w->n, K = w->k;
   w8a8_status small_status = W8A8_OK;
   if (!logits && !top1 &&
@@ -242,7 +213,7 @@ w8a8_status run_w8a8_linear(const w8a8_qweight* w, const uint16_t* X, int M, con
   void* codes = base + L.xf16;
   float* s_x = reinterpret_cast<float*>(base + L.sx);
   if (tc_path(true, w->wq_f16, X, M, N, K, bias, kind, w->inv_delta, w->s_w, Y, logits, top1, dbg, ws, codes, s_x,
-              base + L.part, st, &small_status))
+              base + L.part, st, &small_status, pre))
     return small_status;
   StreamArgs a{};
   a.p = make_stream_plan(true, M, N, K, sms);
@@ -413,7 +384,7 @@ FfnWs ffn_ws(int M, int H, int F, int sms) {
 }
 
 w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X, int M, uint16_t* Y, uint16_t* h_dbg,
-                    void* workspace, int sms, cudaStream_t st, const ResNorm* rn_gate_up) {
+                    void* workspace, int sms, cudaStream_t st, const ResNorm* rn_gate_up, const PreCodes* pre_gate_up) {
   const int H = f->hidden, F = f->inter;
   const FfnWs L = ffn_ws(M, H, F, sms);
   char* base = reinterpret_cast<char*>(workspace);
@@ -432,7 +403,8 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
                        f->gate_up.s_w, h, nullptr, nullptr, nullptr, workspace,
                        base + L.gu + (linear_ws(M, 2 * F, H, true, sms).xf16 - W8A8_WS_RESERVED),
                        reinterpret_cast<float*>(base + L.gu + (linear_ws(M, 2 * F, H, true, sms).sx - W8A8_WS_RESERVED)),
-                       base + L.gu + (linear_ws(M, 2 * F, H, true, sms).part - W8A8_WS_RESERVED), st, &ss)) {
+                       base + L.gu + (linear_ws(M, 2 * F, H, true, sms).part - W8A8_WS_RESERVED), st, &ss,
+                       pre_gate_up)) {
       W8A8_TRY(ss);
     } else {
       const LinearWs A = linear_ws(M, 2 * F, H, true, sms);

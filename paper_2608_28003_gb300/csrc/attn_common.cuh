@@ -1,6 +1,7 @@
-// Device helpers shared by the decode attention kernel and the attention tail of the q/k/v decode
-// GEMV: asynchronous row copies, warp reductions, bf16 unpacking, and the per-head RMSNorm + RoPE
-// of the new row (lane l of a warp holds the rotate-half pairs (4l + e, 128 + 4l + e), e < 4).
+// Device helpers of the decode attention kernel: asynchronous row copies, warp reductions, bf16
+// unpacking, the per-head RMSNorm + RoPE of the new row (lane l of a warp holds the rotate-half pairs
+// (4l + e, 128 + 4l + e), e < 4), one warp's share of a key tile (scores, online softmax, values) and
+// the combination of the warps' partials of a head.
 #pragma once
 
 #include "common.cuh"

@@ -26,6 +26,18 @@ __device__ float block_sum(float v, float* red) {
   return s;
 }
 
+// Maximum over the block; every thread gets the result.
+__device__ float block_max(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float s = 0.0f;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s = fmaxf(s, red[i]);
+  return s;
+}
+
 constexpr int kRowThreads = 256;
 constexpr int kRowVec = 2;  // 8-element vectors per thread: H <= 4096
 
@@ -43,10 +55,62 @@ __device__ __forceinline__ uint4 pack8(const float (&x)[8]) {
   return w;
 }
 
+// The next linear's per-token quantiser (K1, Eq. xhat-lmhead / stx / xint8) on the row this block
+// has just produced, fused here because the block holds the whole row: x_hat = fl(x * inv_delta),
+// m = max |x_hat|, s_x = fl(m / 127), codes = clamp(rint(fl(x_hat * fl(127 / m))), -127, 127) written
+// as fp16 (the tensor-core GEMM's operand).  x: this thread's vectors of the row, already rounded to
+// bf16 (the values the stand-alone K1 would read); the arithmetic is the stand-alone K1's, so the
+// codes and s_x are bit-identical to it.
+struct RowQuant {
+  const float* inv_delta;  // [H]; null: no codes
+  uint16_t* codes;         // [M, H] fp16
+  float* s_x;              // [M]
+};
+__device__ __forceinline__ void row_quantize(const RowQuant& q, int row, int H, const float (&x)[kRowVec][8],
+                                             float* red) {
+  const int nv = H >> 3;
+  float xh[kRowVec][8];
+  float amax = 0.0f;
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        xh[v][e] = __fmul_rn(x[v][e], q.inv_delta[vi * 8 + e]);
+        amax = fmaxf(amax, fabsf(xh[v][e]));
+      }
+    }
+  }
+  const float m = block_max(amax, red);
+  const float r = m > 0.0f ? __fdiv_rn(127.0f, m) : 0.0f;
+  if (threadIdx.x == 0) q.s_x[row] = __fdiv_rn(m, 127.0f);
+#pragma unroll
+  for (int v = 0; v < kRowVec; ++v) {
+    const int vi = threadIdx.x + v * kRowThreads;
+    if (vi < nv) {
+      uint32_t h[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int q0 = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][2 * e], r))));
+        const int q1 = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][2 * e + 1], r))));
+        h[e] = (uint32_t)int_to_f16_bits(q0) | ((uint32_t)int_to_f16_bits(q1) << 16);
+      }
+      reinterpret_cast<uint4*>(q.codes + (size_t)row * H)[vi] = make_uint4(h[0], h[1], h[2], h[3]);
+    }
+  }
+}
+
+__device__ __forceinline__ void round8_bf16(const float (&x)[8], float (&b)[8]) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) b[e] = bf16_bits_to_f32(f32_to_bf16_bits(x[e]));
+}
+
 __global__ void __launch_bounds__(kRowThreads) embed_norm_kernel(const int32_t* __restrict__ tokens, int vocab,
                                                                  const uint16_t* __restrict__ embed, int H, float scale,
                                                                  const float* __restrict__ w, float eps,
-                                                                 float* __restrict__ r, uint16_t* __restrict__ a) {
+                                                                 float* __restrict__ r, uint16_t* __restrict__ a,
+                                                                 const RowQuant rq) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[32];
@@ -81,14 +145,17 @@ __global__ void __launch_bounds__(kRowThreads) embed_norm_kernel(const int32_t* 
 #pragma unroll
       for (int e = 0; e < 8; ++e) y[e] = x[v][e] * inv * w[vi * 8 + e];
       reinterpret_cast<uint4*>(a + (size_t)row * H)[vi] = pack8(y);
+      if (rq.inv_delta) round8_bf16(y, x[v]);  // x now holds the bf16 row
     }
   }
+  if (rq.inv_delta) row_quantize(rq, row, H, x, red);
 }
 
 __global__ void __launch_bounds__(kRowThreads) residual_norm_kernel(const uint16_t* __restrict__ y, int H,
                                                                     const float* __restrict__ w_post,
                                                                     const float* __restrict__ w_next, float eps,
-                                                                    float* __restrict__ r, uint16_t* __restrict__ a) {
+                                                                    float* __restrict__ r, uint16_t* __restrict__ a,
+                                                                    const RowQuant rq) {
   pdl_trigger();
   __shared__ float red[32];
   const int row = blockIdx.x;
@@ -149,8 +216,10 @@ __global__ void __launch_bounds__(kRowThreads) residual_norm_kernel(const uint16
 #pragma unroll
       for (int e = 0; e < 8; ++e) out[e] = rv[v][e] * inv_r * wn[v][e];
       reinterpret_cast<uint4*>(a + (size_t)row * H)[vi] = pack8(out);
+      if (rq.inv_delta) round8_bf16(out, yv[v]);  // yv now holds the bf16 row
     }
   }
+  if (rq.inv_delta) row_quantize(rq, row, H, yv, red);
 }
 
 // One warp per head of a row (q heads, then k heads, then v heads).  hd == 256: lane l holds
@@ -434,19 +503,22 @@ int attention_splits(const AttnShape& s, int sm_count) {
 }  // namespace
 
 w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embed, int vocab, int H, float embed_scale,
-                              const float* w, float eps, float* r, uint16_t* a, cudaStream_t st) {
+                              const float* w, float eps, float* r, uint16_t* a, cudaStream_t st, const float* q_inv_delta,
+                              uint16_t* q_codes, float* q_sx) {
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "embed: hidden %d unsupported", H);
   W8A8_CUDA(launch_pdl(embed_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, tokens, vocab, embed, H, embed_scale, w,
-                       eps, r, a));
+                       eps, r, a, RowQuant{q_inv_delta, q_codes, q_sx}));
   return W8A8_OK;
 }
 
 w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w_post, const float* w_next, float eps,
-                                 float* r, uint16_t* a, cudaStream_t st) {
+                                 float* r, uint16_t* a, cudaStream_t st, const float* q_inv_delta, uint16_t* q_codes,
+                                 float* q_sx) {
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "residual norm: hidden %d unsupported", H);
-  W8A8_CUDA(launch_pdl(residual_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, y, H, w_post, w_next, eps, r, a));
+  W8A8_CUDA(launch_pdl(residual_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, y, H, w_post, w_next, eps, r, a,
+                       RowQuant{q_inv_delta, q_codes, q_sx}));
   return W8A8_OK;
 }
 

@@ -13,13 +13,17 @@ struct AttnShape {
   float scale;         // attention scale
 };
 
-// r = fp32(embed[token]) * embed_scale; a = bf16(rmsnorm(r) * w) (token ids outside [0, vocab) read row 0)
+// r = fp32(embed[token]) * embed_scale; a = bf16(rmsnorm(r) * w) (token ids outside [0, vocab) read row 0).
+// q_inv_delta non-null: also the next linear's per-token quantiser on a (fp16 codes [M, H] and
+// s_x [M], bit-identical to the stand-alone quantiser), so that linear needs no launch of its own.
 w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embed, int vocab, int H, float embed_scale,
-                              const float* w, float eps, float* r, uint16_t* a, cudaStream_t st);
+                              const float* w, float eps, float* r, uint16_t* a, cudaStream_t st,
+                              const float* q_inv_delta = nullptr, uint16_t* q_codes = nullptr, float* q_sx = nullptr);
 
-// r += rmsnorm(y) * w_post;  a = bf16(rmsnorm(r) * w_next)
+// r += rmsnorm(y) * w_post;  a = bf16(rmsnorm(r) * w_next); the quantiser as above
 w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w_post, const float* w_next, float eps,
-                                 float* r, uint16_t* a, cudaStream_t st);
+                                 float* r, uint16_t* a, cudaStream_t st, const float* q_inv_delta = nullptr,
+                                 uint16_t* q_codes = nullptr, float* q_sx = nullptr);
 
 // Per row: q heads and k head RMS-normalised (weights qn, kn; skipped when null), RoPE at position
 // *pos0 + t, q -> fp32 [M, n_q*hd], k and v -> bf16 KV cache [B][max_seq][n_kv*hd] of this layer.

@@ -93,21 +93,20 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
   x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
 }
 
-template <int kW, int MT, int RW, bool kTail = false>
+template <int kW, int MT, int RW>
 __global__ void __launch_bounds__(kThreads, 2)
     gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
-  static_assert(!kTail || (MT == 1 && RW == 1), "the attention tail follows the one-token q/k/v projection");
   // kW: weights bf16 (SMALL_BF16), INT8 codes (SMALL_INT8) or e4m3 codes (SMALL_FP8, 8 slots only)
   constexpr bool kInt8 = kW == SMALL_INT8, kFp8 = kW == SMALL_FP8;
   constexpr bool kQ = kInt8 || kFp8;  // one-byte codes, per-token K1, dequantising epilogue
-  static_assert(!kFp8 || MT == 8, "the e4m3 path runs on the tensor cores (8 token slots)");
+  static_assert(!kFp8 || MT >= 8, "the e4m3 path runs on the tensor cores (8 or 16 token slots)");
   constexpr float kQmax = kFp8 ? 448.0f : 127.0f;  // largest code magnitude
   constexpr int R = 8 * RW;
   // bf16 at 5-8 tokens: the products run on the tensor cores (mma.sync m16n8k16, the activations
   // as the A operand with token rows 8-15 zero, each 8 weight rows an n-tile), the 8 consumer warps
   // taking alternate k steps of every stage; the weights arrive as 128-byte-swizzled boxes of 64
   // columns and the activation rows are padded by 16 bytes, so the fragment loads hit distinct banks
-  constexpr bool kMma = MT == 8;
+  constexpr bool kMma = MT >= 8;  // 8 or 16 token slots: the tensor-core paths (16: both halves of the A tile)
   // W8A8 at 5-8 tokens: the same on INT8 codes carried as fp16 (exact): K1 writes the activation
   // codes to shared memory as fp16, each thread widens four consecutive weight bytes (one 32-bit
   // load from 128-byte-swizzled boxes of 128 columns) into two fp16 pairs, and the k order inside
@@ -119,7 +118,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   using Acc = typename std::conditional<kInt8, int, float>::type;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ float s_red[kCW];
-  __shared__ float s_red8[MT > 4 ? MT : 1][kCW];  // eight-slot K1: per-token maxima of the warps
+  __shared__ float s_red8[MT > 4 ? MT : 1][kCW];  // 8 / 16-slot K1: per-token maxima of the warps
   __shared__ float s_sx[MT];
 
   const SmallPlan& p = a.p;
@@ -358,24 +357,29 @@ __global__ void __launch_bounds__(kThreads, 2)
         xh[6] = __fmul_rn(bf16_lo(w.w), d1.z);
         xh[7] = __fmul_rn(bf16_hi(w.w), d1.w);
       };
-      auto load_tokens = [&](int vi, uint4 (&w)[MT]) {
+      // tokens m0 .. m0 + 7 of vector vi (eight loads in flight; 16 slots take two groups)
+      auto load_tokens = [&](int vi, int m0, uint4 (&w)[8]) {
 #pragma unroll
-        for (int m = 0; m < MT; ++m)
-          w[m] = m < a.M ? reinterpret_cast<const uint4*>(xrows + (size_t)m * xstride)[vi] : make_uint4(0u, 0u, 0u, 0u);
+        for (int m = 0; m < 8; ++m)
+          w[m] = m0 + m < a.M ? reinterpret_cast<const uint4*>(xrows + (size_t)(m0 + m) * xstride)[vi]
+                              : make_uint4(0u, 0u, 0u, 0u);
       };
       float am[MT];
 #pragma unroll
       for (int m = 0; m < MT; ++m) am[m] = 0.0f;
       for (int vi = tid; vi < nvec; vi += kCW * 32) {
-        uint4 w[MT];
-        load_tokens(vi, w);
         const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
 #pragma unroll
-        for (int m = 0; m < MT; ++m) {
-          float xh[8];
-          smooth8(w[m], d0, d1, xh);
+        for (int m0 = 0; m0 < MT; m0 += 8) {
+          uint4 w[8];
+          load_tokens(vi, m0, w);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) am[m] = fmaxf(am[m], fabsf(xh[e]));
+          for (int m = 0; m < 8; ++m) {
+            float xh[8];
+            smooth8(w[m], d0, d1, xh);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) am[m0 + m] = fmaxf(am[m0 + m], fabsf(xh[e]));
+          }
         }
       }
 #pragma unroll
@@ -399,13 +403,16 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       // pass 2: the rows again (L1), quantised; codes of slots >= M are zeros
       for (int vi = tid; vi < nvec; vi += kCW * 32) {
-        uint4 w[MT];
-        load_tokens(vi, w);
         const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
 #pragma unroll
-        for (int m = 0; m < MT; ++m) {
+        for (int m0 = 0; m0 < MT; m0 += 8) {
+          uint4 w8[8];
+          load_tokens(vi, m0, w8);
+#pragma unroll
+          for (int mi = 0; mi < 8; ++mi) {
+          const int m = m0 + mi;
           float xh[8];
-          smooth8(w[m], d0, d1, xh);
+          smooth8(w8[mi], d0, d1, xh);
           if constexpr (kFp8) {  // e4m3 codes: their fp16 values for the MMA, the bytes for debugging
             uint32_t c[4];
 #pragma unroll
@@ -435,6 +442,7 @@ __global__ void __launch_bounds__(kThreads, 2)
               if (a.xq_dbg && blockIdx.x == 0 && m < a.M)
                 reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K)[vi] = packed;
             }
+          }
           }
         }
       }
@@ -485,9 +493,9 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
       for (int m = 0; m < MT; ++m) acc[c][i][m] = 0;
   float mc[2][RW][4];  // MMA path: two accumulator sets (alternate k steps), per n-tile of 8 rows
-  int mi32[RW][2];     // W8A8 MMA path: the folded INT32 sums (token g, rows 8 i + 2 t and + 1)
+  int mi32[RW][4];     // W8A8 MMA path: the folded INT32 sums (tokens g, g + 8; rows 8 i + 2 t and + 1)
 #pragma unroll
-  for (int i = 0; i < RW; ++i) mi32[i][0] = mi32[i][1] = 0;
+  for (int i = 0; i < RW; ++i) mi32[i][0] = mi32[i][1] = mi32[i][2] = mi32[i][3] = 0;
 #pragma unroll
   for (int c = 0; c < 2; ++c)
 #pragma unroll
@@ -522,8 +530,12 @@ __global__ void __launch_bounds__(kThreads, 2)
           const int u = q >> 5, kk = q & 31, ch = kk & 7;
           const uint32_t box = sb + (uint32_t)(u * R * kSliceBytes + (kk >> 3) * R * 128);
           const int kg = (u0 + u) * 512 + 16 * kk;
-          uint32_t a0, a2;
+          uint32_t a0, a2, a1 = 0u, a3 = 0u;  // tokens g and, with 16 slots, g + 8
           asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];\n" : "=r"(a0), "=r"(a2) : "r"(xs + (uint32_t)((g * xsb + kg + 4 * t) * 2)));
+          if constexpr (MT == 16)
+            asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];\n"
+                         : "=r"(a1), "=r"(a3)
+                         : "r"(xs + (uint32_t)(((g + 8) * xsb + kg + 4 * t) * 2)));
 #pragma unroll
           for (int i = 0; i < RW; ++i) {
             uint32_t wb;
@@ -535,7 +547,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             } else {
               i8x4_to_f16x2x2(wb, b0, b1);
             }
-            mma_f16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
+            mma_f16_16816(c[i], a0, a1, a2, a3, b0, b1);
           }
         };
         for (int q = warp; q < 32 * cnt; q += 2 * kCW) {
@@ -545,8 +557,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         if constexpr (kInt8) {
 #pragma unroll
           for (int i = 0; i < RW; ++i) {  // fold: each set took at most 128 products per output this stage
-            mi32[i][0] += __float2int_rn(mc[0][i][0]) + __float2int_rn(mc[1][i][0]);
-            mi32[i][1] += __float2int_rn(mc[0][i][1]) + __float2int_rn(mc[1][i][1]);
+#pragma unroll
+            for (int e = 0; e < (MT == 16 ? 4 : 2); ++e) mi32[i][e] += __float2int_rn(mc[0][i][e]) + __float2int_rn(mc[1][i][e]);
 #pragma unroll
             for (int e = 0; e < 4; ++e) mc[0][i][e] = mc[1][i][e] = 0.0f;
           }
@@ -556,21 +568,24 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int u = q >> 4, kk = q & 15, c0 = 2 * (kk & 3);
         const uint32_t box = sb + (uint32_t)(u * R * kSliceBytes + (kk >> 2) * R * 128);
         const int kg = (u0 + u) * 256 + 16 * kk;
-        uint32_t a0, a2;
-        ldm_x2(xs + (uint32_t)((xr * xsb + kg + 8 * xh) * 2), a0, a2);
+        uint32_t a0, a2, a1 = 0u, a3 = 0u;  // 16 slots: matrices (tokens 0-7 | 8-15) x (k lo | k hi)
+        if constexpr (MT == 16)
+          ldm_x4(xs + (uint32_t)(((xr + 8 * xh) * xsb + kg + 8 * (lane >> 4)) * 2), a0, a1, a2, a3);
+        else
+          ldm_x2(xs + (uint32_t)((xr * xsb + kg + 8 * xh) * 2), a0, a2);
 #pragma unroll
         for (int i = 0; i < RW; i += 2) {
           if (i + 1 < RW) {  // n-tiles i and i + 1: matrices (i, k lo), (i, k hi), (i + 1, lo), (i + 1, hi)
             const int mi = lane >> 3, r = 8 * (i + (mi >> 1)) + xr, ch = c0 + (mi & 1);
             uint32_t b0, b1, b2, b3;
             ldm_x4(box + (uint32_t)(r * 128 + ((ch ^ xr) << 4)), b0, b1, b2, b3);
-            mma_bf16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
-            mma_bf16_16816(c[i + 1], a0, 0u, a2, 0u, b2, b3);
+            mma_bf16_16816(c[i], a0, a1, a2, a3, b0, b1);
+            mma_bf16_16816(c[i + 1], a0, a1, a2, a3, b2, b3);
           } else {
             const int r = 8 * i + xr, ch = c0 + xh;
             uint32_t b0, b1;
             ldm_x2(box + (uint32_t)(r * 128 + ((ch ^ xr) << 4)), b0, b1);
-            mma_bf16_16816(c[i], a0, 0u, a2, 0u, b0, b1);
+            mma_bf16_16816(c[i], a0, a1, a2, a3, b0, b1);
           }
         }
       };
@@ -634,20 +649,24 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
   }
   if constexpr (kMma) {
-    // Each warp's sums (accumulator c0 / c1 of n-tile i: token g, rows 8 i + 2 t and + 1) go to
-    // shared memory [warp][row][token]; then every output sums the 8 warps in warp order (W8A8:
-    // INT32, exact, then dequantised as fl(fl(s_x s_w) acc)).
+    // Each warp's sums (accumulators c0 / c1 of n-tile i: token g, rows 8 i + 2 t and + 1; c2 / c3:
+    // token g + 8) go to shared memory [warp][row][token]; then every output sums the 8 warps in
+    // warp order (W8A8: INT32, exact, then dequantised as fl(fl(s_x s_w) acc)).
     Acc* part = reinterpret_cast<Acc*>(xsp + p.xbytes + p.abytes);
     const int g = lane >> 2, t = lane & 3;
     if (ok) {
 #pragma unroll
       for (int i = 0; i < RW; ++i) {
-        if constexpr (kInt8) {
-          part[(warp * R + 8 * i + 2 * t) * 8 + g] = mi32[i][0];
-          part[(warp * R + 8 * i + 2 * t + 1) * 8 + g] = mi32[i][1];
-        } else {
-          part[(warp * R + 8 * i + 2 * t) * 8 + g] = mc[0][i][0] + mc[1][i][0];
-          part[(warp * R + 8 * i + 2 * t + 1) * 8 + g] = mc[0][i][1] + mc[1][i][1];
+#pragma unroll
+        for (int h = 0; h < MT / 8; ++h) {  // token half: g, then g + 8
+          const int m = g + 8 * h;
+          if constexpr (kInt8) {
+            part[(warp * R + 8 * i + 2 * t) * MT + m] = mi32[i][2 * h];
+            part[(warp * R + 8 * i + 2 * t + 1) * MT + m] = mi32[i][2 * h + 1];
+          } else {
+            part[(warp * R + 8 * i + 2 * t) * MT + m] = mc[0][i][2 * h] + mc[1][i][2 * h];
+            part[(warp * R + 8 * i + 2 * t + 1) * MT + m] = mc[0][i][2 * h + 1] + mc[1][i][2 * h + 1];
+          }
         }
       }
     }
@@ -655,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     auto total = [&](int r, int m) {
       Acc v = 0;
 #pragma unroll
-      for (int w = 0; w < kCW; ++w) v += part[(w * R + r) * 8 + m];
+      for (int w = 0; w < kCW; ++w) v += part[(w * R + r) * MT + m];
       float y;
       if constexpr (kInt8) {
         y = __fmul_rn(__fmul_rn(s_sx[m], a.s_w[row0 + r]), __int2float_rn(v));
@@ -668,26 +687,23 @@ __global__ void __launch_bounds__(kThreads, 2)
       return a.bias ? __fadd_rn(y, a.bias[row0 + r]) : y;
     };
     if (a.kind == EPI_GEGLU) {  // pair b of block j: gate row 16 j + b, up row 16 j + 8 + b
-      for (int e = tid; e < (R / 2) * 8; e += kCW * 32) {
-        const int pr = e >> 3, m = e & 7, j = pr >> 3, b = pr & 7;
+      for (int e = tid; e < (R / 2) * MT; e += kCW * 32) {
+        const int pr = e / MT, m = e % MT, j = pr >> 3, b = pr & 7;
         const int gr = 16 * j + b;
         if (m >= a.M || row0 + gr + 8 >= a.N) continue;
         a.y[(size_t)m * (a.N >> 1) + ((row0 + 16 * j) >> 1) + b] =
             f32_to_bf16_bits(geglu_recipe(total(gr, m), total(gr + 8, m)));
       }
     } else {
-      for (int e = tid; e < R * 8; e += kCW * 32) {
-        const int r = e >> 3, m = e & 7;
+      for (int e = tid; e < R * MT; e += kCW * 32) {
+        const int r = e / MT, m = e % MT;
         if (m >= a.M || row0 + r >= a.N) continue;
         a.y[(size_t)m * a.N + row0 + r] = f32_to_bf16_bits(total(r, m));
       }
     }
     return;
   }
-  if (!ok) {
-    if constexpr (kTail) attn_tail(a.tail, a.y, smem_raw + a.p.smem_bytes, 1, a.err);  // keeps the tickets whole
-    return;
-  }
+  if (!ok) return;
 #pragma unroll
   for (int c = 1; c < NA; ++c)  // fixed order: ((a0 + a1) + a2) + a3
 #pragma unroll
@@ -703,10 +719,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) acc[0][i][m] += __shfl_xor_sync(0xffffffffu, acc[0][i][m], o);
     }
-  if constexpr (!kTail) {
-    if (lane != 0) return;
-  }
-  if (lane == 0) {  // the epilogue (the whole warp reaches the attention tail after it)
+  if (lane != 0) return;
+  {  // the epilogue (lane 0)
     auto value = [&](Acc v, int i, int row, int m) -> float {  // i: the warp's row slot of `row`
       float y;
       if constexpr (kInt8) {
@@ -743,31 +757,25 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
     }
   }
-  if constexpr (kTail) {
-    __syncwarp();
-    attn_tail(a.tail, a.y, smem_raw + a.p.smem_bytes, 1, a.err);
-  }
 }
 
-template <int kW, int MT, int RW, bool kTail = false>
+template <int kW, int MT, int RW>
 w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW, kTail>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    kSmemLimit - kStatic));
     attr_set[dev] = true;
   }
   constexpr int EB = kW == SMALL_BF16 ? 2 : 1;
   CUtensorMap tw;
-  if (MT == 8)  // the tensor-core paths: 128-byte boxes (64 bf16 or 128 INT8 columns), 128-byte swizzle
+  if (MT >= 8)  // the tensor-core paths: 128-byte boxes (64 bf16 or 128 INT8 columns), 128-byte swizzle
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 8 * RW, 128));
   else
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
-  const size_t smem = (size_t)a.p.smem_bytes + (kTail ? (size_t)kTailSmem : 0);  // the tail's region follows
-  W8A8_CHECK_ARG(smem <= (size_t)(kSmemLimit - kStatic), W8A8_ERR_SHAPE, "small GEMV: %zu bytes of shared memory", smem);
-  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW, kTail>, dim3(a.p.P), dim3(kThreads), smem, st, tw,
+  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
                        a));
   return W8A8_OK;
 }
@@ -775,7 +783,7 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
 // accumulator registers a warp may hold (tokens x rows): larger products spill; the tensor-core paths
 // (8 token slots) hold 8 (+ 2 INT32) per n-tile of 8 rows whatever the token count
 constexpr bool slots_fit(int kw, int MT, int RW) {
-  return MT == 8 || (kw != SMALL_FP8 && MT * RW <= (kw == SMALL_INT8 ? 48 : 32));
+  return MT >= 8 || (kw != SMALL_FP8 && MT * RW <= (kw == SMALL_INT8 ? 48 : 32));
 }
 
 template <int kW, int MT, int RW>
@@ -800,13 +808,14 @@ w8a8_status launch_mt(const SmallArgs& a, cudaStream_t st) {
 template <int kW>
 w8a8_status launch_typed(const SmallArgs& a, cudaStream_t st) {
   if constexpr (kW == SMALL_FP8) {
-    return launch_mt<kW, 8>(a, st);
+    return a.p.MT == 16 ? launch_mt<kW, 16>(a, st) : launch_mt<kW, 8>(a, st);
   } else {
     switch (a.p.MT) {
       case 1: return launch_mt<kW, 1>(a, st);
       case 2: return launch_mt<kW, 2>(a, st);
       case 4: return launch_mt<kW, 4>(a, st);
-      default: return launch_mt<kW, 8>(a, st);
+      case 8: return launch_mt<kW, 8>(a, st);
+      default: return launch_mt<kW, 16>(a, st);
     }
   }
 }
@@ -817,10 +826,11 @@ SmallPlan make_small_plan(int wkind, int M, int N, int K, int kind, int sm_count
   SmallPlan p{};
   const bool int8_weights = wkind != SMALL_BF16;  // one-byte codes (INT8 or e4m3)
   if (fused_norm && K > 2048) return p;  // one 8-channel vector per consumer thread
-  if (M < 1 || M > 8 || N < 1 || K < 16 || K % 16 != 0) return p;
+  if (M < 1 || M > 16 || N < 1 || K < 16 || K % 16 != 0) return p;
+  if (M > 8 && fused_norm) return p;  // the decoder fuses its residual step at 1-8 tokens only
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return p;
   if (kind == EPI_GEGLU && N % 16 != 0) return p;
-  p.MT = wkind == SMALL_FP8 ? 8 : M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
+  p.MT = M > 8 ? 16 : wkind == SMALL_FP8 ? 8 : M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
   if (int8_weights && p.MT <= 4 && K > kMaxInt8K) return p;
   // fewest rows per CTA (more CTAs) that still fit in two CTAs per SM
   static const int kRw[] = {1, 2, 4, 6};
@@ -839,10 +849,10 @@ SmallPlan make_small_plan(int wkind, int M, int N, int K, int kind, int sm_count
   p.sub = int8_weights ? 512 : 256;
   p.nsub = (K + p.sub - 1) / p.sub;
   p.kpad = p.nsub * p.sub;
-  const bool mma = p.MT == 8;  // the kernel's tensor-core paths (same rule): padded bf16 / fp16 rows
+  const bool mma = p.MT >= 8;  // the kernel's tensor-core paths (same rule): padded bf16 / fp16 rows
   p.xbytes = mma ? p.MT * (p.kpad + (int8_weights ? 16 : 8)) * 2 : p.MT * p.kpad * (int8_weights ? 1 : 2);
   p.abytes = fused_norm && int8_weights ? p.MT * p.kpad * 2 : 0;
-  p.rbytes = mma ? kCW * R * 8 * 4 : 0;  // the warps' partial sums
+  p.rbytes = mma ? kCW * R * p.MT * 4 : 0;  // the warps' partial sums
   const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - p.abytes - p.rbytes - 16 * 16;
   // sub-slices per stage: 4 for warps with one or two rows, fewer for wider CTAs; each stage must
   // fit twice in the ring unless one stage covers everything
@@ -870,17 +880,9 @@ w8a8_status launch_small_gemv(int wkind, const SmallArgs& a, cudaStream_t st) {
   take_kernel_events(&v0, &v1);
   cudaEvent_t e0 = reinterpret_cast<cudaEvent_t>(v0), e1 = reinterpret_cast<cudaEvent_t>(v1);
   if (e0) W8A8_CUDA(cudaEventRecord(e0, st));
-  w8a8_status s;
-  if (a.has_tail) {
-    W8A8_CHECK_ARG(wkind != SMALL_FP8 && a.M == 1 && a.p.MT == 1 && a.p.RW == 1 && a.tail.n_q >= 1 &&
-                       a.tail.n_q <= kTailMaxG && 8 % a.tail.n_q == 0,
-                   W8A8_ERR_SHAPE, "small GEMV: the attention tail needs one token, one row per warp, 1-4 heads");
-    s = wkind == SMALL_INT8 ? launch_t<SMALL_INT8, 1, 1, true>(a, st) : launch_t<SMALL_BF16, 1, 1, true>(a, st);
-  } else {
-    s = wkind == SMALL_FP8    ? launch_typed<SMALL_FP8>(a, st)
-        : wkind == SMALL_INT8 ? launch_typed<SMALL_INT8>(a, st)
-                              : launch_typed<SMALL_BF16>(a, st);
-  }
+  const w8a8_status s = wkind == SMALL_FP8    ? launch_typed<SMALL_FP8>(a, st)
+                        : wkind == SMALL_INT8 ? launch_typed<SMALL_INT8>(a, st)
+                                              : launch_typed<SMALL_BF16>(a, st);
   if (e1) W8A8_CUDA(cudaEventRecord(e1, st));
   return s;
 }

@@ -1,9 +1,8 @@
-// Decode GEMV for up to 8 tokens whose CTAs own whole weight rows (no split of the k sum across
+// Decode GEMV for up to 16 tokens whose CTAs own whole weight rows (no split of the k sum across
 // CTAs): the W8A8 path with the per-token quantiser (K1) fused into its prologue, its e4m3 (FP8)
 // variant, and the bf16 pass-through.
 #pragma once
 
-#include "attn_tail.cuh"
 #include "common.cuh"
 
 namespace w8a8 {
@@ -14,7 +13,7 @@ enum { SMALL_BF16 = 0, SMALL_INT8 = 1, SMALL_FP8 = 2 };
 
 struct SmallPlan {
   int ok;           // 0: this shape is left to the weight-streaming kernel
-  int MT;           // token slots: 1, 2, 4 or 8
+  int MT;           // token slots: 1, 2, 4, 8 or 16 (8 and 16: the tensor-core paths)
   int RW;           // weight rows per consumer warp: 1, 2, 4 or 6 (R = 8 RW rows per CTA)
   int P;            // CTAs
   int sub;          // k elements per 512-byte sub-slice of a row (256 bf16, 512 INT8)
@@ -59,8 +58,6 @@ struct SmallArgs {
   ResNorm rn;
   unsigned int* err;       // device error word
   SmallPlan p;
-  int has_tail;            // 1: the decode attention of one sequence runs as this GEMV's tail (q/k/v
-  AttnTail tail;           //    projection at one token; the plan must have one token slot, one row per warp)
 };
 
 // fused_norm: the call computes its input with a ResNorm (needs K <= 2048)

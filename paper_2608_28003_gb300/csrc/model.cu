@@ -62,9 +62,10 @@ struct w8a8_model {
   size_t ws_bytes = 0;
   void* attn_ws = nullptr;
   size_t attn_ws_bytes = 0;
-  // decode attention of one sequence as the tail of the q/k/v GEMV: two tickets (zero between
-  // launches), then the attention CTAs' partials
-  unsigned char* tail_ws = nullptr;
+  // the next W8A8 linear's quantised input written by the norm kernels at 9+ tokens ([max_tokens,
+  // hidden] fp16 codes and [max_tokens] scales), so that its GEMM needs no quantiser launch
+  uint16_t* pcodes = nullptr;
+  float* psx = nullptr;
   // diagnostics: when set, a forward copies every layer's output (the residual stream after its
   // post-FFN step, fp32 [M, H]) to capture + l M H
   float* capture = nullptr;
@@ -120,10 +121,10 @@ void free_all(w8a8_model* m) {
 w8a8_qweight qdesc(const QW& q, int n, int k) { return w8a8_qweight{n, k, q.wq, q.s_w, q.inv_delta, q.wq_f16}; }
 
 w8a8_status linear(w8a8_model* m, bool int8, const QW& qw, const uint16_t* Wbf, int N, int K, const uint16_t* X, int M,
-                   uint16_t* Y, cudaStream_t st, const ResNorm* rn) {
+                   uint16_t* Y, cudaStream_t st, const ResNorm* rn, const PreCodes* pre = nullptr) {
   if (int8) {
     const w8a8_qweight w = qdesc(qw, N, K);
-    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st, rn);
+    return run_w8a8_linear(&w, X, M, nullptr, 0, Y, nullptr, nullptr, nullptr, m->ws, m->sms, st, rn, pre);
   }
   return run_bf16_linear(Wbf, N, K, X, M, nullptr, 0, Y, nullptr, nullptr, m->ws, m->sms, st, rn);
 }
@@ -143,16 +144,6 @@ bool fuse_residual(const w8a8_model* m, int M, bool calib) {
   return true;
 }
 
-// Whether the decode attention of this call can run as the q/k/v GEMV's tail: one sequence at one
-// token, one key/value head of 256 shared by 1, 2 or 4 query heads, and a decode-GEMV plan for q/k/v
-// with one row per warp.
-bool attn_tail_ok(const w8a8_model* m, bool att8, int B, int T) {
-  const w8a8_model_cfg& c = m->cfg;
-  if (B != 1 || T != 1 || c.n_kv != 1 || c.head_dim != kAttnHd) return false;
-  if (c.n_q != 1 && c.n_q != 2 && c.n_q != 4) return false;
-  return qkv_attention_takes(att8, m->qkv_dim, c.hidden, m->sms);
-}
-
 // The decoder over M = B * T rows whose positions start at *m->d_pos (set by the caller).
 w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, float* logits, int32_t* top1, bool calib,
                          cudaStream_t st) {
@@ -161,7 +152,16 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
   const bool fuse = fuse_residual(m, M, calib);
   float* rc = m->r;   // the residual stream as of now
   float* rn = m->r2;  // where a fused update writes the next one
-  W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st));
+  // 9+ tokens: the norm kernels quantise the input of the next W8A8 linear themselves (its
+  // tensor-core GEMM then needs no quantiser launch); fewer tokens run the decode GEMV, which
+  // quantises inside
+  const bool preq = !calib && M >= 9 && m->prepared;
+  const PreCodes pc{m->pcodes, m->psx};
+  auto att8_of = [&](int l) { return !calib && m->prepared && ((m->attn_bits >> l) & 1u); };
+  const bool pre0 = preq && att8_of(0);
+  W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st,
+                             pre0 ? m->q_qkv[0].inv_delta : nullptr, m->pcodes, m->psx));
+  bool pre_qkv = pre0;  // whether the codes of the current q/k/v input exist
   const w8a8_trace* tr = m->trace_on && !calib ? &m->trace : nullptr;
   W8A8_CHECK_ARG(!tr || M <= tr->max_rows, W8A8_ERR_SHAPE, "trace: %d rows exceed the trace's %d", M, tr ? tr->max_rows : 0);
   // copy this call's M rows of a [rows, width] tensor into slice l of a [L][max_rows][width] trace buffer
@@ -185,31 +185,17 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     const float* kn = c.qk_norm ? W.k_norm : nullptr;
     const float* cs = glob ? m->cos_g : m->cos_l;
     const float* sn = glob ? m->sin_g : m->sin_l;
-    // one sequence at one token: the attention runs as the q/k/v GEMV's tail (no separate launch)
-    const bool tail = !calib && attn_tail_ok(m, att8, B, T);
-    const AttnTail at{c.n_q, glob ? 0 : c.window, c.max_seq, s.scale, c.eps, m->d_pos, qn, kn, cs, sn, kc, vc, m->o,
-                      reinterpret_cast<float*>(m->tail_ws + 256), reinterpret_cast<unsigned int*>(m->tail_ws)};
     const QW& qq = m->q_qkv[l];
     if (fuse && l > 0) {  // the previous layer's post-FFN step, then q/k/v
       const ResNorm R{m->y, rc, rn, m->L[l - 1].ln_post_ffn, W.ln_in, c.eps};
-      if (tail)
-        W8A8_TRY(run_qkv_attention(att8, att8 ? (const void*)qq.wq : (const void*)W.wqkv, qq.inv_delta, qq.s_w,
-                                   m->qkv_dim, H, &R, nullptr, m->qkv, at, m->ws, m->sms, st));
-      else
-        W8A8_TRY(linear(m, att8, qq, W.wqkv, m->qkv_dim, H, nullptr, M, m->qkv, st, &R));
+      W8A8_TRY(linear(m, att8, qq, W.wqkv, m->qkv_dim, H, nullptr, M, m->qkv, st, &R));
       std::swap(rc, rn);
     } else {
       if (tr) W8A8_TRY(trace_copy(tr->a_in, l, m->a, H, 2));
-      if (tail)
-        W8A8_TRY(run_qkv_attention(att8, att8 ? (const void*)qq.wq : (const void*)W.wqkv, qq.inv_delta, qq.s_w,
-                                   m->qkv_dim, H, nullptr, m->a, m->qkv, at, m->ws, m->sms, st));
-      else
-        W8A8_TRY(linear(m, att8, qq, W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr));
+      W8A8_TRY(linear(m, att8, qq, W.wqkv, m->qkv_dim, H, m->a, M, m->qkv, st, nullptr, pre_qkv ? &pc : nullptr));
       if (tr) W8A8_TRY(trace_copy(tr->qkv, l, m->qkv, m->qkv_dim, 2));
     }
-    if (tail) {
-      // the attention ran inside the q/k/v launch
-    } else if (attn_decode_supported(s)) {
+    if (attn_decode_supported(s)) {
       W8A8_TRY(launch_attn_decode(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, kc, vc, m->o, st));
     } else {
       W8A8_TRY(launch_qk_rope(m->qkv, s, m->d_pos, qn, kn, c.eps, cs, sn, m->q, kc, vc, st));
@@ -234,18 +220,22 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
       W8A8_TRY(run_ffn(&f, prec, nullptr, M, m->y, nullptr, m->ws, m->sms, st, &R));
       std::swap(rc, rn);
     } else {
-      W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, rc, m->a, st));
+      const bool pre_gu = preq && ffn8;
+      W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, rc, m->a, st,
+                                    pre_gu ? m->q_gu[l].inv_delta : nullptr, m->pcodes, m->psx));
       if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
       if (tr) W8A8_TRY(trace_copy(tr->a_ffn, l, m->a, H, 2));
       uint16_t* h_out = calib ? m->h : nullptr;
       if (tr && tr->h) h_out = tr->h + (size_t)l * tr->max_rows * F;  // the block writes h there
-      W8A8_TRY(run_ffn(&f, prec, m->a, M, m->y, h_out, m->ws, m->sms, st));
+      W8A8_TRY(run_ffn(&f, prec, m->a, M, m->y, h_out, m->ws, m->sms, st, nullptr, pre_gu ? &pc : nullptr));
       if (tr) W8A8_TRY(trace_copy(tr->y_f, l, m->y, H, 2));
     }
     if (calib) W8A8_TRY(launch_act_absmax(m->h, M, F, m->stat_down(l), st));
     if (!fuse || l + 1 == c.layers) {
       const float* next = l + 1 < c.layers ? m->L[l + 1].ln_in : m->final_norm;
-      W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, rc, m->a, st));
+      pre_qkv = preq && l + 1 < c.layers && att8_of(l + 1);
+      W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, rc, m->a, st,
+                                    pre_qkv ? m->q_qkv[l + 1].inv_delta : nullptr, m->pcodes, m->psx));
     }
     if (m->capture)
       W8A8_CUDA(cudaMemcpyAsync(m->capture + (size_t)l * M * H, rc, sizeof(float) * M * H, cudaMemcpyDeviceToDevice, st));
@@ -447,11 +437,11 @@ extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_l
   }
   m->attn_ws_bytes = aws;
   W8A8_MTRY(dalloc(m, reinterpret_cast<char**>(&m->attn_ws), aws));
-  W8A8_MTRY(dalloc(m, &m->tail_ws, kTailScratchBytes));
+  W8A8_MTRY(dalloc(m, &m->pcodes, (size_t)c.max_tokens * H));
+  W8A8_MTRY(dalloc(m, &m->psx, (size_t)c.max_tokens + 4));
   cudaStream_t st = m->st;
   W8A8_MTRY(cudaMemsetAsync(m->ws, 0, W8A8_WS_RESERVED, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
   W8A8_MTRY(cudaMemsetAsync(m->attn_ws, 0, aws, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
-  W8A8_MTRY(cudaMemsetAsync(m->tail_ws, 0, kTailScratchBytes, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
   W8A8_MTRY(cudaMemsetAsync(m->stats, 0, ((size_t)c.layers * m->stats_stride() + H) * 4, st) == cudaSuccess
                 ? W8A8_OK
                 : W8A8_ERR_CUDA);

@@ -86,14 +86,16 @@ def _sensitivity(od, toks, T, mask):
     return ref, _rel_l2(pert, ref)
 
 
-def _close(gpu: np.ndarray, ref: np.ndarray, sens: np.ndarray):
+def _close(gpu: np.ndarray, ref: np.ndarray, sens: np.ndarray, plain: bool = False):
     """End-to-end tolerance, per position: relative L2 error <= max(1e-2, 1.5 x the oracle's own
     one-ulp sensitivity there).  Through 4 random layers a one-ulp change of one input element
     moves the oracle's logits by ~0.6 % (all bf16) and ~3 % (with W8A8 sublayers, whose INT8 codes
-    flip), so fp32-vs-fp64 rounding differences cannot be held to less.  Top-1 must agree wherever
-    the oracle's margin exceeds twice the row's largest error."""
+    flip), so fp32-vs-fp64 rounding differences cannot be held to less.  plain: the stated 1e-2
+    alone (the all-bf16 mask, whose sensitivity stays below it).  Top-1 must agree wherever the
+    oracle's margin exceeds twice the row's largest error.  Every step of every layer is held to
+    the oracle without this amplification in test_gpu_decoder_trace.py."""
     rel = _rel_l2(gpu, ref)
-    tol = np.maximum(1e-2, 1.5 * sens)
+    tol = np.full_like(rel, 1e-2) if plain else np.maximum(1e-2, 1.5 * sens)
     assert np.all(rel <= tol), (float(rel.max()), float(tol.min()))
     d = np.abs(gpu.astype(np.float64) - ref)
     err = d.max(axis=-1)
@@ -115,14 +117,15 @@ def test_decoder_prefill_and_decode_match_oracle(B, setup, mask):
     od.reset()
     ref = od.forward(toks[:, :24], 0, mask)["logits"]
     assert np.allclose(ref, ref_all[:, :24])
-    _close(logits.view(2, 24, V).cpu().numpy(), ref, sens[:, :24])
+    bf16_mask = not (fb or ab or lm)
+    _close(logits.view(2, 24, V).cpu().numpy(), ref, sens[:, :24], plain=bf16_mask)
     assert np.array_equal(top1.view(2, 24).cpu().numpy(), logits.view(2, 24, V).argmax(-1).cpu().numpy())
     buf = torch.empty(2, V, dtype=torch.float32, device="cuda")
     for s in range(4):  # positions 24..27 cross the sliding window of 8 on layers 1..3
         col = tt[:, 24 + s].contiguous()
         lg, t1 = dec.decode_step(col, 24 + s, logits=buf)
         r = od.forward(toks[:, 24 + s:25 + s], 24 + s, mask)["logits"][:, 0]
-        _close(lg.cpu().numpy(), r, sens[:, 24 + s])
+        _close(lg.cpu().numpy(), r, sens[:, 24 + s], plain=bf16_mask)
 
 
 @pytest.mark.parametrize("mask", [OM.make_mask(), OM.Mask(frozenset({1, 2}), frozenset({0}), True)],
@@ -202,11 +205,11 @@ def test_decode_kernel_count(B, setup):
 @pytest.mark.parametrize("mask", [OM.make_mask(), OM.Mask(frozenset({0, 3}), frozenset({1}), True)],
                          ids=["bf16", "mixed"])
 def test_single_sequence_decode_matches_oracle(B, setup, mask):
-    """One sequence: the decode step runs its attention as the tail of the q/k/v GEMV (no attention
-    launch) with the residual step fused into q/k/v and gate/up; positions 24..27 cross the sliding
-    window of 8 on layers 1..3.  Against the oracle at batch 1 with the same prepared weights; the
-    graph replay equals an eager step; a step launches the position update, embedding + norm, four
-    kernels per layer, the last residual step and lm_head (W8A8 lm_head adds its quantiser)."""
+    """One sequence (the headline decode): the residual step fused into q/k/v and gate/up, one-token
+    decode GEMVs and decode attention; positions 24..27 cross the sliding window of 8 on layers 1..3.
+    Against the oracle at batch 1 with the same prepared weights; the graph replay equals an eager
+    step; a step launches the position update, embedding + norm, five kernels per layer, the last
+    residual step and lm_head (W8A8 lm_head adds its quantiser)."""
     dec, od, toks = setup[:3]
     od1 = OD.OracleDecoder(od.cfg, od.w, batch=1, max_len=64)
     od1.prep, od1.stats = od.prep, od.stats
@@ -216,18 +219,18 @@ def test_single_sequence_decode_matches_oracle(B, setup, mask):
     ref_all, sens = _sensitivity(od1, t1, 28, mask)
     tt = torch.from_numpy(t1).cuda()
     buf = torch.empty(1, V, dtype=torch.float32, device="cuda")
-    dec.forward(tt[:, :24].contiguous(), 0, want_logits=False)
+    dec.forward(tt[:, :24].clone(), 0, want_logits=False)  # clone: a fresh, 16-byte aligned tensor
     rows = []
     for s in range(4):
-        lg, t = dec.decode_step(tt[:, 24 + s].contiguous(), 24 + s, logits=buf)
+        lg, t = dec.decode_step(tt[:, 24 + s].clone(), 24 + s, logits=buf)
         rows.append(lg.cpu().numpy()[0])
         assert int(t.item()) == int(np.argmax(rows[-1]))
     _close(np.stack(rows), ref_all[0, 24:28], sens[0, 24:28])
-    lg2, _ = dec.decode_step(tt[:, 27].contiguous(), 27, logits=buf)  # replayed at the same position
+    lg2, _ = dec.decode_step(tt[:, 27].clone(), 27, logits=buf)  # replayed at the same position
     assert np.array_equal(lg2.cpu().numpy()[0], rows[-1])
-    lg3, _ = dec.forward(tt[:, 27:28].contiguous(), 27)  # eager forward of the same step
+    lg3, _ = dec.forward(tt[:, 27:28].clone(), 27)  # eager forward of the same step
     assert np.array_equal(lg3.cpu().numpy()[0], rows[-1])
-    assert dec.decode_kernels(1, want_logits=True) == 2 + 4 * L + 2 + (1 if lm else 0)
+    assert dec.decode_kernels(1, want_logits=True) == 2 + 5 * L + 2 + (1 if lm else 0)
 
 
 def test_mask_controls(B, setup):

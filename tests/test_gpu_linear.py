@@ -128,6 +128,9 @@ LINEAR_SHAPES = [
     (4, 1152, 1024),    # o_proj shape
     (7, 9, 16),         # fewer rows than one CTA's eight, K of one vector
     (2, 64, 9216),      # K too long for the fused quantiser: K1 + streaming kernel
+    (13, 1536, 1152),   # row-owning decode GEMV, 16 token slots (both halves of the MMA's A tile)
+    (11, 1000, 1152),   # 16 slots, ragged N and tokens
+    (16, 1152, 1024),   # 16 slots, o_proj shape
 ]
 
 
@@ -231,6 +234,7 @@ def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarr
                                    (1, 1536, 1152), (8, 1152, 6912), (3, 40, 64), (2, 13824, 1152),
                                    (128, 6912, 1152), (70, 1152, 6912), (300, 256, 64),
                                    (6, 1536, 1152),      # 8 token slots on the tensor cores, with a bias
+                                   (13, 1536, 1152),     # 16 token slots on the tensor cores
                                    (7, 200, 64),         # the same, ragged rows, one 64-column box of K
                                    (8, 13824, 1152),     # the same, 48 rows per CTA
                                    (32, 1152, 4608),     # split-K: 18 tiles, k cut into 8 parts
