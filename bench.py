@@ -816,6 +816,14 @@ def sweep(B, dev, head, xh, flush, stream, peaks):
         row["fp8_vs_bf16"] = round(row["bf16_us"] / row["fp8_us"], 3)
         cmp[f"M{M}"] = row
     out["ffn_fp8_int8_bf16"] = cmp
+    # the exact integer routes' sustained rates (the rooflines of the INT8 paths): best of three
+    rp = {}
+    for route, name in ((0, "dp4a"), (1, "mma_sync_s8"), (2, "mma_sync_f16_on_int8_codes")):
+        rp[name] = round(max(B.route_peak(route) for _ in range(3)), 1)
+    rp["tcgen05_kind_f16_on_int8_codes"] = peaks.get("bf16_tflops")
+    rp["note"] = ("TOPS; tcgen05 kind::f16 runs fp16 operands at the bf16 rate, so the W8A8 prefill GEMM's "
+                  "route peak is the measured bf16 GEMM peak; FP8 (kind::f8f6f4) is twice it (nominal ratio)")
+    out["int8_route_peaks"] = rp
     lg = torch.empty(512, VOCAB, dtype=torch.float32, device=dev)
     tp = torch.empty(512, dtype=torch.int32, device=dev)
     for M in (1, 16, 128, 512):

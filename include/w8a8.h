@@ -71,6 +71,14 @@ w8a8_status w8a8_workspace_check(void* workspace, void* stream);
  * neither (NULL, NULL clears a pending request). */
 w8a8_status w8a8_set_kernel_events(void* start_event, void* stop_event);
 
+/* Measurement aid (no counterpart in the paper; not a compute entry point: it allocates and frees a
+ * small sink buffer and synchronises `stream`): the sustained rate, in TOPS (two ops per
+ * multiply-add), of an exact integer route for the INT8 GEMM on the current GPU, measured by one
+ * launch over every SM with CUDA events: route 0 = dp4a, 1 = mma.sync m16n8k32 s8 x s8 -> s32,
+ * 2 = mma.sync m16n8k16 fp16 x fp16 -> fp32 (the decode GEMV's tensor-core path on INT8 codes
+ * carried as fp16).  The tcgen05 route's rate is the fp16 / bf16 tensor rate (kind::f16). */
+w8a8_status w8a8_route_peak(int route, double* tops, void* stream);
+
 /* ---------------------------------------------------------------------------------------
  * Prepared W8A8 weight of one linear (produced by w8a8_prepare_weights /
  * w8a8_prepare_gate_up, owned by the caller).

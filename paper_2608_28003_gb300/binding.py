@@ -120,6 +120,7 @@ SIGNATURES = {
     "w8a8_last_error": (ctypes.c_char_p, []),
     "w8a8_workspace_check": (_i32, [_vp, _vp]),
     "w8a8_set_kernel_events": (_i32, [_vp, _vp]),
+    "w8a8_route_peak": (_i32, [_i32, ctypes.POINTER(ctypes.c_double), _vp]),
     "w8a8_act_absmax": (_i32, [_vp, _i32, _i32, _vp, _vp]),
     "w8a8_prepare_weights": (_i32, [_vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
     "w8a8_prepare_gate_up": (_i32, [_vp, _vp, _i32, _i32, _vp, _f32, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -232,6 +233,13 @@ def default_workspace() -> Workspace:
 def workspace_check(ws: "Workspace", stream=None) -> None:
     """Raise W8A8Error(ERR_TIMEOUT) if a kernel using `ws` recorded a device-side timeout."""
     _check("w8a8_workspace_check", lib().w8a8_workspace_check(_p(ws.buf), _stream(stream)))
+
+
+def route_peak(route: int, stream=None) -> float:
+    """Sustained TOPS of an exact integer route (0 dp4a, 1 mma.sync s8, 2 mma.sync fp16)."""
+    out = ctypes.c_double(0.0)
+    _check("w8a8_route_peak", lib().w8a8_route_peak(int(route), ctypes.byref(out), _stream(stream)))
+    return out.value
 
 
 def set_kernel_events(start, stop) -> None:

@@ -1063,14 +1063,6 @@ w8a8_status dispatch(TcArgs a, cudaStream_t st) {
   };
   const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
                c128 = cost(kBM, 128, 1.81, 2 * pairs), c64 = cost(kBM, 64, 2.7, 2 * pairs);
-  const bool pair = (c256 <= c192 && c256 <= c128 && c256 <= c64) || (c192 <= c128 && c192 <= c64);
-  // W8A8 on CTA pairs: 128-channel pair tiles.  Its accumulator is restarted every 1024 k (one slot
-  // per chunk), so wide tiles (two 256-column slots fill tensor memory) leave a tile's chunks no
-  // slot to overlap with the next tile's, and the epilogue's INT32 fold of two 32-column groups per
-  // warp spills; 128 columns give four slots and one group per warp.
-  if constexpr (kMode == kModeI8) {
-    if (pair) return launch_t2<kMode, 128>(a, st);
-  }
   if (c256 <= c192 && c256 <= c128 && c256 <= c64) return launch_t2<kMode, 256>(a, st);
   if (c192 <= c128 && c192 <= c64) return launch_t2<kMode, 192>(a, st);
   if (c128 <= c64) return launch_split<kMode, 128>(a, st);
