@@ -107,13 +107,27 @@ static unsigned int* err_word(void* ws) {
 
 // Decode-sized calls whose CTAs can own whole weight rows go to the row-owning GEMV (K1 fused
 // into it on the W8A8 path); returns false when the shape is left to the streaming kernel.
+// Partial row maxima passed from the FFN's gate/up launch to its down launch (see SmallArgs).
+struct RowMax {
+  float* out;                   // gate/up: [P][MT]
+  const float* next_inv_delta;  // gate/up: down's 1 / delta
+  const float* in;              // down: gate/up's rows
+  int n;                        // down: gate/up's CTA count
+};
+
 static bool small_gemv(bool int8, const void* W, const float* inv_delta, const float* s_w, const uint16_t* X, int M,
                        int N, int K, const float* bias, int kind, uint16_t* Y, const w8a8_debug* dbg, void* ws,
-                       const ResNorm* rn, int sms, cudaStream_t st, w8a8_status* status) {
+                       const ResNorm* rn, int sms, cudaStream_t st, w8a8_status* status, const RowMax* rm = nullptr) {
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return false;
   SmallArgs a{};
   a.p = make_small_plan(int8, M, N, K, kind, sms, rn != nullptr);
   if (!a.p.ok) return false;
+  if (rm) {
+    a.rowmax_out = rm->out;
+    a.next_inv_delta = rm->next_inv_delta;
+    a.rowmax_in = rm->in;
+    a.rowmax_n = rm->n;
+  }
   if (rn) {
     a.has_rn = 1;
     a.rn = *rn;
@@ -379,6 +393,8 @@ FfnWs ffn_ws(int M, int H, int F, int sms) {
   off += a.total - W8A8_WS_RESERVED;
   w.dn = off;
   off += b.total - W8A8_WS_RESERVED;
+  w.rowmax = off;  // gate/up's partial row maxima for down's quantiser (decode GEMV, 16 slots at most)
+  off += round_up((size_t)2 * std::max(sms, 1) * 16 * 4, 256);
   w.total = off;
   return w;
 }
@@ -392,10 +408,16 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
   // The two linears run one after the other on `stream` and share the FFN workspace's reserved
   // counters (each leaves them zero); their scratch regions are disjoint.
   if (precision == W8A8_PREC_W8A8) {
-    // gate/up: scratch at L.gu
+    // gate/up: scratch at L.gu.  At 5-16 tokens, when both linears run the decode GEMV's tensor-core
+    // path, gate/up's GeGLU epilogue also hands down the partial maxima of its quantiser's first pass.
     w8a8_status ss = W8A8_OK;
+    const SmallPlan pg = make_small_plan(true, M, 2 * F, H, EPI_GEGLU, sms, rn_gate_up != nullptr);
+    const SmallPlan pd = make_small_plan(true, M, H, F, EPI_BF16, sms, false);
+    const bool handoff = pg.ok && pd.ok && pg.MT >= 8 && pd.MT == pg.MT;
+    float* rowmax = reinterpret_cast<float*>(base + L.rowmax);
+    const RowMax rm_gu{rowmax, f->down.inv_delta, nullptr, 0}, rm_dn{nullptr, nullptr, rowmax, pg.P};
     if (small_gemv(true, f->gate_up.wq, f->gate_up.inv_delta, f->gate_up.s_w, X, M, 2 * F, H, nullptr, EPI_GEGLU, h,
-                   nullptr, workspace, rn_gate_up, sms, st, &ss)) {
+                   nullptr, workspace, rn_gate_up, sms, st, &ss, handoff ? &rm_gu : nullptr)) {
       W8A8_TRY(ss);
     } else if (rn_gate_up) {
       W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "fused residual norm: the decode GEMV does not take gate/up at M=%d", M);
@@ -427,7 +449,7 @@ w8a8_status run_ffn(const w8a8_ffn_weights* f, int precision, const uint16_t* X,
       W8A8_TRY(launch_stream_gemm(true, a, st));
     }
     if (small_gemv(true, f->down.wq, f->down.inv_delta, f->down.s_w, h, M, H, F, nullptr, EPI_BF16, Y, nullptr,
-                   workspace, nullptr, sms, st, &ss)) {
+                   workspace, nullptr, sms, st, &ss, handoff ? &rm_dn : nullptr)) {
       W8A8_TRY(ss);
     } else if (tc_path(true, f->down.wq_f16, h, M, H, F, nullptr, EPI_BF16, f->down.inv_delta, f->down.s_w, Y,
                        nullptr, nullptr, nullptr, workspace,

@@ -3,9 +3,11 @@
 // At decode the attention of a layer reads a few hundred cached key/value rows and one new row;
 // split over separate kernels (QK-norm + RoPE, then attention with a cross-CTA combine through
 // global memory) it costs several dependent round trips.  Here one launch does it all:
-//  * grid (kSplits, B, n_kv) in clusters of kSplits CTAs along x: CTA r of a cluster takes an
-//    equal share of the key positions of (sequence b, key/value head kvh); shares are at least
-//    kMinKeys long, so short contexts leave the trailing CTAs idle;
+//  * grid (kSplits, B, n_kv x G / hpc) in clusters of kSplits CTAs along x: a cluster takes hpc of
+//    the G query heads of (sequence b, key/value head kvh): all G at more than 8 sequences, one at up
+//    to 8 (G times the SMs, each CTA's warps on one head); CTA r of a cluster takes an equal share of
+//    the key positions; shares are at least kMinKeys long, so short contexts leave the trailing CTAs
+//    idle; the first cluster of a key/value head writes the new row to the cache;
 //  * before waiting for the preceding kernel (the q/k/v projection), each CTA starts copying its
 //    cached key/value rows (positions before the new one, written by earlier steps) into shared
 //    memory with cp.async, in tiles of 64 positions (one buffer: a share longer than a tile loads
@@ -14,7 +16,7 @@
 //    arithmetic of the prefill path (one warp per head, lane l holding the RoPE pairs
 //    (4l + e, 128 + 4l + e)); the CTA whose share ends at the new position also writes its key
 //    (bf16) and value to the cache and uses them from shared memory;
-//  * warp w handles query head w mod G and an even share (key group w / G) of each tile: one, two
+//  * warp w handles query head w mod hpc and an even share (key group w / hpc) of each tile: one, two
 //    or four lanes per key compute its dot product with the scaled query (read from shared
 //    memory; key rows padded to 528 bytes, chunks rotated per lane so that the lanes of a
 //    shared-memory phase hit different bank groups), then the warp updates its running max, sum
@@ -72,13 +74,18 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     attn_decode_kernel(const uint16_t* __restrict__ qkv, AttnShape s, const int* __restrict__ pos0,
                        const float* __restrict__ qn, const float* __restrict__ kn, float eps,
                        const float* __restrict__ rope_cos, const float* __restrict__ rope_sin,
-                       uint16_t* __restrict__ kcache, uint16_t* __restrict__ vcache, uint16_t* __restrict__ o) {
+                       uint16_t* __restrict__ kcache, uint16_t* __restrict__ vcache, uint16_t* __restrict__ o,
+                       int hpc) {
   extern __shared__ __align__(16) uint8_t sm[];
   pdl_trigger();
-  const int r = blockIdx.x, b = blockIdx.y, kvh = blockIdx.z;
-  const int G = s.n_q / s.n_kv, KG = kWarps / G;  // heads per key/value head; key groups per tile
+  // hpc query heads per cluster (1, or all G heads of a key/value head): blockIdx.z picks the
+  // key/value head and, with hpc < G, which hpc of its query heads this cluster takes
+  const int G = s.n_q / s.n_kv, KG = kWarps / hpc;  // heads per key/value head; key groups per tile
+  const int r = blockIdx.x, b = blockIdx.y, kvh = blockIdx.z / (G / hpc);
+  const int hq0 = kvh * G + (blockIdx.z % (G / hpc)) * hpc;  // this cluster's first query head
+  const bool writes_cache = hq0 == kvh * G;  // the first cluster of a key/value head stores its new row
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int hw = warp % G, gw = warp / G;         // this warp's head (within the group) and key group
+  const int hw = warp % hpc, gw = warp / hpc;     // this warp's head (within the cluster's) and key group
   // The position was set before this launch's chain began, and cached rows before it were
   // written by earlier launches: both may be read before waiting for the preceding kernel.
   const int pos = *pos0;
@@ -109,9 +116,9 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
   // norm weights and the RoPE row of this position: constants, read before the wait as well
   const float* cos_row = rope_cos + (size_t)pos * (kHd / 2);
   const float* sin_row = rope_sin + (size_t)pos * (kHd / 2);
-  const int kwarp = G;  // the warp that rotates the new key (G < 8 warps)
+  const int kwarp = hpc;  // the warp that rotates the new key (hpc < 8 warps)
   RopeConsts qc, kc2;
-  if (r < used && warp < G) load_rope_consts(qc, qn, cos_row, sin_row, lane);
+  if (r < used && warp < hpc) load_rope_consts(qc, qn, cos_row, sin_row, lane);
   if (owns_new && warp == kwarp) load_rope_consts(kc2, kn, cos_row, sin_row, lane);
 
   pdl_wait();
@@ -119,8 +126,8 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
   const int qkv_dim = (s.n_q + 2 * s.n_kv) * kHd;
   const uint16_t* src_row = qkv + (size_t)b * qkv_dim;
   if (r < used) {
-    if (warp < G) {
-      const uint16_t* src = src_row + (size_t)(kvh * G + warp) * kHd;
+    if (warp < hpc) {
+      const uint16_t* src = src_row + (size_t)(hq0 + warp) * kHd;
       const uint2 a = *reinterpret_cast<const uint2*>(src + 4 * lane);
       const uint2 c = *reinterpret_cast<const uint2*>(src + kHd / 2 + 4 * lane);
       float x1[4] = {bf16_lo(a.x), bf16_hi(a.x), bf16_lo(a.y), bf16_hi(a.y)};
@@ -144,16 +151,18 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
       u1.y = (uint32_t)f32_to_bf16_bits(x1[2]) | ((uint32_t)f32_to_bf16_bits(x1[3]) << 16);
       u2.x = (uint32_t)f32_to_bf16_bits(x2[0]) | ((uint32_t)f32_to_bf16_bits(x2[1]) << 16);
       u2.y = (uint32_t)f32_to_bf16_bits(x2[2]) | ((uint32_t)f32_to_bf16_bits(x2[3]) << 16);
-      uint16_t* kd = kcache + seq_base + (size_t)pos * row_stride;
-      *reinterpret_cast<uint2*>(kd + 4 * lane) = u1;
-      *reinterpret_cast<uint2*>(kd + kHd / 2 + 4 * lane) = u2;
+      if (writes_cache) {
+        uint16_t* kd = kcache + seq_base + (size_t)pos * row_stride;
+        *reinterpret_cast<uint2*>(kd + 4 * lane) = u1;
+        *reinterpret_cast<uint2*>(kd + kHd / 2 + 4 * lane) = u2;
+      }
       *reinterpret_cast<uint2*>(sm + kOffKNew + 8 * lane) = u1;
       *reinterpret_cast<uint2*>(sm + kOffKNew + kHd + 8 * lane) = u2;
     }
     if (owns_new && warp == kWarps - 1) {  // value head kvh: straight copy
       const uint16_t* src = src_row + (size_t)(s.n_q + s.n_kv + kvh) * kHd;
       const uint4 v = *reinterpret_cast<const uint4*>(src + 8 * lane);
-      *reinterpret_cast<uint4*>(vcache + seq_base + (size_t)pos * row_stride + 8 * lane) = v;
+      if (writes_cache) *reinterpret_cast<uint4*>(vcache + seq_base + (size_t)pos * row_stride + 8 * lane) = v;
       *reinterpret_cast<uint4*>(sm + kOffVNew + 16 * lane) = v;
     }
   }
@@ -186,9 +195,9 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     part[kHd + 1] = l;
   }
   __syncthreads();
-  if (warp < G) {
+  if (warp < hpc) {
     float M, Lc, y[8];
-    attn_combine_warps(reinterpret_cast<const float*>(sm + kOffPart), kPartFloats, G, KG, warp, lane, M, Lc, y);
+    attn_combine_warps(reinterpret_cast<const float*>(sm + kOffPart), kPartFloats, hpc, KG, warp, lane, M, Lc, y);
     const uint32_t dst = map_to_rank(sbase + kOffInbox + (uint32_t)((r * kMaxG + warp) * kPartFloats * 4), 0);
     st_cluster_f32x4(dst + 32 * lane, y[0], y[1], y[2], y[3]);
     st_cluster_f32x4(dst + 32 * lane + 16, y[4], y[5], y[6], y[7]);
@@ -198,7 +207,7 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     }
   }
   cluster_sync_all();  // release the pushes / acquire them in CTA 0
-  if (r == 0 && warp < G) {
+  if (r == 0 && warp < hpc) {
     const float* in = reinterpret_cast<const float*>(sm + kOffInbox);
     const float mi = lane < kSplits ? in[(lane * kMaxG + warp) * kPartFloats + kHd] : -INFINITY;
     const float li = lane < kSplits ? in[(lane * kMaxG + warp) * kPartFloats + kHd + 1] : 0.0f;
@@ -223,7 +232,7 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     w.y = (uint32_t)f32_to_bf16_bits(z[2]) | ((uint32_t)f32_to_bf16_bits(z[3]) << 16);
     w.z = (uint32_t)f32_to_bf16_bits(z[4]) | ((uint32_t)f32_to_bf16_bits(z[5]) << 16);
     w.w = (uint32_t)f32_to_bf16_bits(z[6]) | ((uint32_t)f32_to_bf16_bits(z[7]) << 16);
-    *reinterpret_cast<uint4*>(o + (size_t)b * (s.n_q * kHd) + (size_t)(kvh * G + warp) * kHd + 8 * lane) = w;
+    *reinterpret_cast<uint4*>(o + (size_t)b * (s.n_q * kHd) + (size_t)(hq0 + warp) * kHd + 8 * lane) = w;
   }
 }
 
@@ -248,8 +257,11 @@ w8a8_status launch_attn_decode(const uint16_t* qkv, const AttnShape& s, const in
     W8A8_CUDA(cudaFuncSetAttribute(attn_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem));
     attr_set[dev] = true;
   }
-  W8A8_CUDA(launch_pdl(attn_decode_kernel, dim3(kSplits, s.B, s.n_kv), dim3(kWarps * 32), (size_t)kSmem, st, qkv, s,
-                       pos0, qn, kn, eps, rope_cos, rope_sin, kcache, vcache, o));
+  // Few sequences: one cluster per query head (G times the SMs, every CTA's warps on one head, the
+  // cached rows read once per head); many: one cluster per key/value head (its G heads share the rows).
+  const int G = s.n_q / s.n_kv, hpc = s.B <= 8 ? 1 : G;
+  W8A8_CUDA(launch_pdl(attn_decode_kernel, dim3(kSplits, s.B, s.n_kv * (G / hpc)), dim3(kWarps * 32), (size_t)kSmem,
+                       st, qkv, s, pos0, qn, kn, eps, rope_cos, rope_sin, kcache, vcache, o, hpc));
   return W8A8_OK;
 }
 

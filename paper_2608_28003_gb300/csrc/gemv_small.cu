@@ -120,6 +120,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   __shared__ float s_red[kCW];
   __shared__ float s_red8[MT > 4 ? MT : 1][kCW];  // 8 / 16-slot K1: per-token maxima of the warps
   __shared__ float s_sx[MT];
+  __shared__ unsigned int s_hmax[MT];  // GeGLU epilogue: per-token max |h * 1/delta| of this CTA (float bits)
 
   const SmallPlan& p = a.p;
   const int S = p.stages, SB = p.stage_bytes, nst = p.nst, kpad = p.kpad, KS = p.ks, nsub = p.nsub;
@@ -367,7 +368,12 @@ __global__ void __launch_bounds__(kThreads, 2)
       float am[MT];
 #pragma unroll
       for (int m = 0; m < MT; ++m) am[m] = 0.0f;
-      for (int vi = tid; vi < nvec; vi += kCW * 32) {
+      if (a.rowmax_in) {  // the producer's partial maxima stand for pass 1 (the same fp32 products)
+        for (int i = tid; i < a.rowmax_n; i += kCW * 32)
+#pragma unroll
+          for (int m = 0; m < MT; ++m) am[m] = fmaxf(am[m], a.rowmax_in[(size_t)i * MT + m]);
+      }
+      for (int vi = a.rowmax_in ? nvec : tid; vi < nvec; vi += kCW * 32) {
         const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
 #pragma unroll
         for (int m0 = 0; m0 < MT; m0 += 8) {
@@ -687,12 +693,23 @@ __global__ void __launch_bounds__(kThreads, 2)
       return a.bias ? __fadd_rn(y, a.bias[row0 + r]) : y;
     };
     if (a.kind == EPI_GEGLU) {  // pair b of block j: gate row 16 j + b, up row 16 j + 8 + b
+      if (a.rowmax_out && tid < MT) s_hmax[tid] = 0u;
+      if (a.rowmax_out) named_bar_sync(1, kCW * 32);
       for (int e = tid; e < (R / 2) * MT; e += kCW * 32) {
         const int pr = e / MT, m = e % MT, j = pr >> 3, b = pr & 7;
         const int gr = 16 * j + b;
         if (m >= a.M || row0 + gr + 8 >= a.N) continue;
-        a.y[(size_t)m * (a.N >> 1) + ((row0 + 16 * j) >> 1) + b] =
-            f32_to_bf16_bits(geglu_recipe(total(gr, m), total(gr + 8, m)));
+        const int hc = ((row0 + 16 * j) >> 1) + b;  // h channel
+        const uint16_t hb = f32_to_bf16_bits(geglu_recipe(total(gr, m), total(gr + 8, m)));
+        a.y[(size_t)m * (a.N >> 1) + hc] = hb;
+        if (a.rowmax_out) {  // |x_hat| of the down projection's quantiser, as its K1 computes it
+          const float v = fabsf(__fmul_rn(bf16_bits_to_f32(hb), a.next_inv_delta[hc]));
+          if (!(v != v)) atomicMax(&s_hmax[m], __float_as_uint(v));  // K1's fmaxf passes over NaN too
+        }
+      }
+      if (a.rowmax_out) {
+        named_bar_sync(1, kCW * 32);
+        if (tid < MT) a.rowmax_out[(size_t)blockIdx.x * MT + tid] = __uint_as_float(s_hmax[tid]);
       }
     } else {
       for (int e = tid; e < R * MT; e += kCW * 32) {

@@ -58,6 +58,14 @@ struct SmallArgs {
   ResNorm rn;
   unsigned int* err;       // device error word
   SmallPlan p;
+  // The FFN's down projection at 5-16 tokens (token slots 8 or 16): the gate/up launch (GeGLU) writes,
+  // per CTA and token slot, the maximum of |fl(h * next_inv_delta)| over its h channels (rowmax_out
+  // [P][MT]); the down launch (W8A8) takes m_t as the maximum of rowmax_n such rows (rowmax_in) and
+  // skips the first pass of its quantiser.  Both nullable.
+  float* rowmax_out;
+  const float* next_inv_delta;  // [N / 2] the down projection's 1 / delta
+  const float* rowmax_in;
+  int rowmax_n;
 };
 
 // fused_norm: the call computes its input with a ResNorm (needs K <= 2048)

@@ -17,7 +17,7 @@ struct LinearWs {
   size_t xf16, sx, part, total;
 };
 struct FfnWs {
-  size_t h, gu, dn, total;
+  size_t h, gu, dn, rowmax, total;
 };
 LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms);
 FfnWs ffn_ws(int M, int H, int F, int sms);
