@@ -824,6 +824,27 @@ def sweep(B, dev, head, xh, flush, stream, peaks):
     rp["note"] = ("TOPS; tcgen05 kind::f16 runs fp16 operands at the bf16 rate, so the W8A8 prefill GEMM's "
                   "route peak is the measured bf16 GEMM peak; FP8 (kind::f8f6f4) is twice it (nominal ratio)")
     out["int8_route_peaks"] = rp
+    # the prefill GEMM alone (gate/up shape as a plain linear, 2048 x 1152 -> 13824): its kernel's
+    # tensor rate against its route's peak (bf16 and INT8-as-fp16: the measured bf16 peak; FP8: twice it)
+    Mg, Ng = 2048, 2 * INTER
+    _, wg = synth.weight(Ng, HIDDEN, seed=1)
+    _, xg, _ = synth.activations(Mg, HIDDEN, 8, seed=2)
+    wg, xg = wg.to(dev), xg.to(dev)
+    yg = torch.empty(Mg, Ng, dtype=torch.bfloat16, device=dev)
+    qg = B.prepare_weights(wg, B.act_absmax(xg), want_f16=True)
+    q8g = B.fp8_prepare_weights(wg, B.act_absmax(xg))
+    flops = 2 * Mg * Ng * HIDDEN
+    bf = peaks["bf16_tflops"]
+    for tag, fn, pk in (("w8a8", lambda: B.linear(qg, xg, out=yg, ws=ws), bf),
+                        ("bf16", lambda: B.linear_bf16(wg, xg, out=yg, ws=ws), bf),
+                        ("fp8", lambda: B.fp8_linear(q8g, xg, out=yg, ws=ws), 2 * bf)):
+        t = statistics.mean(timed_steps(fn, 10, 3, flush, stream, kev))
+        nm = f"gemm_{tag}_2048x1152x13824"
+        rec(nm, t, flops, (w8a8_bytes if tag != "bf16" else bf16_bytes)(Mg, Ng, HIDDEN), True)
+        kt = out[nm]["kernel_us"] * 1e-6
+        out[nm].update({"kernel_TOPS": round(flops / kt / 1e12, 1), "route_peak_TOPS": round(pk, 1),
+                        "route_frac": round(flops / kt / 1e12 / pk, 4)})
+    del wg, xg, yg, qg, q8g
     lg = torch.empty(512, VOCAB, dtype=torch.float32, device=dev)
     tp = torch.empty(512, dtype=torch.int32, device=dev)
     for M in (1, 16, 128, 512):

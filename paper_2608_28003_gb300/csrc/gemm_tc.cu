@@ -50,6 +50,17 @@ constexpr int kModeBf16 = TC_BF16, kModeI8 = TC_I8, kModeFp8 = TC_FP8;
 __host__ __device__ constexpr int bk_elems(int mode) { return mode == kModeFp8 ? kSwz : kSwz / 2; }
 __host__ __device__ constexpr int elem_bytes(int mode) { return mode == kModeFp8 ? 1 : 2; }
 constexpr int kKbPerChunk = 1024 / kBK;  // stages per exact fp32 chunk of 1024 k
+// W8A8 chunk length in stages for a range of len stages: the fewest chunks of at most kKbPerChunk
+// stages, of equal length (the last one shorter), so that the epilogue's fold of one chunk overlaps
+// the MMAs of a chunk as long as itself rather than those of a short remainder (1152 k: 576 + 576,
+// not 1024 + 128).
+__host__ __device__ constexpr int chunk_stages(int len) {
+  return len <= kKbPerChunk ? (len > 0 ? len : 1)
+                            : (len + (len + kKbPerChunk - 1) / kKbPerChunk - 1) / ((len + kKbPerChunk - 1) / kKbPerChunk);
+}
+__host__ __device__ constexpr int chunk_count(int len) {
+  return len <= 0 ? 1 : (len + chunk_stages(len) - 1) / chunk_stages(len);
+}
 constexpr int kEpiWarps = 16;                   // four per TMEM lane quarter: one per column quarter
 constexpr int kParts = kEpiWarps / 4;
 constexpr int kProdWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1;
@@ -153,22 +164,6 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // 32 consecutive fp32 values p[c0 .. c0 + 31] into w, 0 past n (c0 a multiple of 32, p 16-byte
 // aligned): eight 16-byte loads when the group lies inside n.  Every lane of a warp reads the same
 // addresses (a broadcast).
-__device__ __forceinline__ void ld_cols32(const float* p, int c0, int n, float (&w)[32]) {
-  if (c0 + 32 <= n) {
-    const float4* q = reinterpret_cast<const float4*>(p + c0);
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const float4 t = __ldg(q + k);
-      w[4 * k] = t.x;
-      w[4 * k + 1] = t.y;
-      w[4 * k + 2] = t.z;
-      w[4 * k + 3] = t.w;
-    }
-  } else {
-#pragma unroll
-    for (int j = 0; j < 32; ++j) w[j] = c0 + j < n ? __ldg(p + c0 + j) : 0.0f;
-  }
-}
 
 // The dequantising epilogue of one 32-column group: w holds s_w of the columns on entry and
 // fl(fl(s_x s_w) acc) (+ bias) on exit (Eq. gemm-final); acc is the INT32 sum (W8A8) or the fp32
@@ -180,17 +175,39 @@ __device__ __forceinline__ float acc_as_f32<int>(int v) { return __int2float_rn(
 template <>
 __device__ __forceinline__ float acc_as_f32<uint32_t>(uint32_t v) { return __uint_as_float(v); }
 
-template <typename T>
-__device__ __forceinline__ void dequant32(const TcArgs& a, float sx, int c0, const T* acc, float (&w)[32]) {
-  ld_cols32(a.s_w, c0, a.N, w);
+// Column values of the epilogue (s_w, bias) one column per lane: lane j holds column c0 + j of
+// each of the warp's NG groups, loaded at the start of a tile, before the wait for its
+// accumulator, so that the load latency overlaps the MMAs; element j of a group takes its values
+// from lane j with a shuffle.
+template <int NG>
+struct ColVals {
+  float sw[NG], b[NG];
+};
+template <int NG>
+__device__ __forceinline__ void load_colvals(const TcArgs& a, bool want_sw, int n0, int part, int bn, int lane,
+                                             ColVals<NG>& cv) {
 #pragma unroll
-  for (int j = 0; j < 32; ++j) w[j] = __fmul_rn(__fmul_rn(sx, w[j]), acc_as_f32<T>(acc[j]));
-  if (a.bias) {
-    float b[32];
-    ld_cols32(a.bias, c0, a.N, b);
-#pragma unroll
-    for (int j = 0; j < 32; ++j) w[j] = __fadd_rn(w[j], b[j]);
+  for (int i = 0; i < NG; ++i) {
+    const int c = n0 + 32 * (part + kParts * i) + lane;
+    const bool in = 32 * (part + kParts * i) < bn && c < a.N;
+    cv.sw[i] = want_sw && in ? __ldg(a.s_w + c) : 0.0f;
+    cv.b[i] = a.bias && in ? __ldg(a.bias + c) : 0.0f;
   }
+}
+// fl(fl(s_x s_w) acc) (+ bias) of one 32-column group (Eq. gemm-final); acc is the INT32 sum
+// (W8A8) or the fp32 one (FP8); sw / b are this lane's column values of the group.
+template <typename T>
+__device__ __forceinline__ void dequant32(bool has_bias, float sx, float sw, float b, const T* acc, float (&v)[32]) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    float y = __fmul_rn(__fmul_rn(sx, __shfl_sync(0xffffffffu, sw, j)), acc_as_f32<T>(acc[j]));
+    if (has_bias) y = __fadd_rn(y, __shfl_sync(0xffffffffu, b, j));
+    v[j] = y;
+  }
+}
+__device__ __forceinline__ void add_bias32(float b, float (&v)[32]) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __fadd_rn(v[j], __shfl_sync(0xffffffffu, b, j));
 }
 
 // ------------------------------------------------------------------ epilogue through TMA stores
@@ -366,8 +383,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int KS = a.ksplit > 1 ? a.ksplit : 1, units = tiles * KS;
   auto kb_lo = [&](int u) { return (int)((long long)(u % KS) * nkb / KS); };
   auto kb_hi = [&](int u) { return (int)((long long)(u % KS + 1) * nkb / KS); };
-  // accumulator chunks of a unit: W8A8 restarts every 1024 k counted from the unit's first stage
-  auto chunks_of = [&](int u) { return kInt8 ? (kb_hi(u) - kb_lo(u) + kKbPerChunk - 1) / kKbPerChunk : 1; };
+  // accumulator chunks of a unit: W8A8 restarts every chunk_stages(len) stages (at most 1024 k)
+  // counted from the unit's first stage
+  auto chunks_of = [&](int u) { return kInt8 ? chunk_count(kb_hi(u) - kb_lo(u)) : 1; };
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
                  done = acce0 + 8 * NSLOT;
 
@@ -448,7 +466,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(slot * SC);
-          const int kb0 = kInt8 ? ulo + c * kKbPerChunk : ulo, kb1 = kInt8 ? min(uhi, kb0 + kKbPerChunk) : uhi;
+          const int per = chunk_stages(uhi - ulo);
+          const int kb0 = kInt8 ? ulo + c * per : ulo, kb1 = kInt8 ? min(uhi, kb0 + per) : uhi;
           for (int kb = kb0; kb < kb1; ++kb, ++g) {
             const int s = g % S;
             if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
@@ -521,6 +540,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 32 * NG; ++j) isum[j] = 0;
         const int nch = chunks_of(u);
+        ColVals<NG> cv;  // before the first wait: the loads overlap the MMAs
+        if (KS == 1) load_colvals<NG>(a, true, n0, part, BN, lane, cv);
+        const float sx = KS == 1 && row < a.M ? a.s_x[row] : 0.0f;
         for (int c = 0; c < nch; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
@@ -556,7 +578,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else if (!ok) {
           break;
         }
-        const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
         for (int i = 0; i < NG; ++i) {
           const int g = part + kParts * i;
@@ -567,18 +588,24 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (n0 + 32 * g + j < a.N) a.acc_dbg[(size_t)row * a.N + n0 + 32 * g + j] = isum[32 * i + j];
           }
           float v[32];
-          dequant32(a, sx, n0 + 32 * g, &isum[32 * i], v);
+          dequant32(a.bias != nullptr, sx, cv.sw[i], cv.b[i], &isum[32 * i], v);
           emit32(32 * g, v);
         }
       } else {
+        constexpr int NG = (BN / 32 + kParts - 1) / kParts;
+        ColVals<NG> cv;  // before the wait: the loads overlap the MMAs
+        if (KS == 1) load_colvals<NG>(a, kFp8, n0, part, BN, lane, cv);
+        const float sx = kFp8 && KS == 1 && row < a.M ? a.s_x[row] : 0.0f;
         const int slot = q % NSLOT;
         if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
           ok = false;
           atomicOr(a.err, DEVERR_CONSUMER_WAIT);
         } else {
           tc_fence_after();
-#pragma unroll 1
-          for (int g = part; g < BN / 32; g += kParts) {
+#pragma unroll
+          for (int i = 0; i < NG; ++i) {
+            const int g = part + kParts * i;
+            if (g >= BN / 32) break;
             uint32_t r[32];
             tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
             if (KS > 1) {  // this part's fp32 sums go to the partials
@@ -587,16 +614,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             float v[32];
             if constexpr (kFp8) {
-              dequant32(a, row < a.M ? a.s_x[row] : 0.0f, n0 + 32 * g, r, v);
+              dequant32(a.bias != nullptr, sx, cv.sw[i], cv.b[i], r, v);
             } else {
 #pragma unroll
               for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-              if (a.bias) {
-                float b[32];
-                ld_cols32(a.bias, n0 + 32 * g, a.N, b);
-#pragma unroll
-                for (int j = 0; j < 32; ++j) v[j] = __fadd_rn(v[j], b[j]);
-              }
+              if (a.bias) add_bias32(cv.b[i], v);
             }
             emit32(32 * g, v);
           }
@@ -743,8 +765,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   const int NT = (a.N + BN - 1) / BN, tiles = NT * ((a.M + 2 * kBM - 1) / (2 * kBM));
   const int nkb = (a.K + BKe - 1) / BKe;
-  const int nchunks = kInt8 ? (nkb + kKbPerChunk - 1) / kKbPerChunk : 1;
-  const int kb_per_chunk = kInt8 ? kKbPerChunk : nkb;
+  const int nchunks = kInt8 ? chunk_count(nkb) : 1;
+  const int kb_per_chunk = kInt8 ? chunk_stages(nkb) : nkb;
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
                  done = acce0 + 8 * NSLOT;
 
@@ -866,6 +888,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         int isum[32 * NG];
 #pragma unroll
         for (int j = 0; j < 32 * NG; ++j) isum[j] = 0;
+        ColVals<NG> cv;  // before the first wait: the loads overlap the MMAs
+        load_colvals<NG>(a, true, n0, part, BN, lane, cv);
+        const float sx = row < a.M ? a.s_x[row] : 0.0f;
         for (int c = 0; c < nchunks; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
@@ -887,7 +912,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           mbar_arrive_cluster(acce_lead + 8 * slot);
         }
         if (!ok) break;
-        const float sx = row < a.M ? a.s_x[row] : 0.0f;
 #pragma unroll
         for (int i = 0; i < NG; ++i) {
           const int g = part + kParts * i;
@@ -898,10 +922,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               if (n0 + 32 * g + j < a.N) a.acc_dbg[(size_t)row * a.N + n0 + 32 * g + j] = isum[32 * i + j];
           }
           float v[32];
-          dequant32(a, sx, n0 + 32 * g, &isum[32 * i], v);
+          dequant32(a.bias != nullptr, sx, cv.sw[i], cv.b[i], &isum[32 * i], v);
           emit(32 * g, v);
         }
       } else {
+        constexpr int NG = (BN / 32 + kParts - 1) / kParts;
+        ColVals<NG> cv;  // before the wait: the loads overlap the MMAs
+        load_colvals<NG>(a, kFp8, n0, part, BN, lane, cv);
+        const float sx = kFp8 && row < a.M ? a.s_x[row] : 0.0f;
         const int slot = q % NSLOT;
         if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
           ok = false;
@@ -909,22 +937,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-#pragma unroll 1
-        for (int g = part; g < BN / 32; g += kParts) {
+#pragma unroll
+        for (int i = 0; i < NG; ++i) {
+          const int g = part + kParts * i;
+          if (g >= BN / 32) break;
           uint32_t r[32];
           tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
           float v[32];
           if constexpr (kFp8) {
-            dequant32(a, row < a.M ? a.s_x[row] : 0.0f, n0 + 32 * g, r, v);
+            dequant32(a.bias != nullptr, sx, cv.sw[i], cv.b[i], r, v);
           } else {
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-            if (a.bias) {
-              float b[32];
-              ld_cols32(a.bias, n0 + 32 * g, a.N, b);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) v[j] = __fadd_rn(v[j], b[j]);
-            }
+            if (a.bias) add_bias32(cv.b[i], v);
           }
           emit(32 * g, v);
         }
@@ -1062,9 +1087,15 @@ w8a8_status dispatch(TcArgs a, cudaStream_t st) {
     return (double)((t + slots - 1) / slots) * bn * unit;
   };
   const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
-               c128 = cost(kBM, 128, 1.81, 2 * pairs), c64 = cost(kBM, 64, 2.7, 2 * pairs);
-  if (c256 <= c192 && c256 <= c128 && c256 <= c64) return launch_t2<kMode, 256>(a, st);
-  if (c192 <= c128 && c192 <= c64) return launch_t2<kMode, 192>(a, st);
+               p128 = cost(2 * kBM, 128, 1.32, pairs), c128 = cost(kBM, 128, 1.81, 2 * pairs),
+               c64 = cost(kBM, 64, 2.7, 2 * pairs);
+  if (c256 <= c192 && c256 <= c128 && c256 <= c64 && c256 <= p128) return launch_t2<kMode, 256>(a, st);
+  if (c192 <= c128 && c192 <= c64 && c192 <= p128) return launch_t2<kMode, 192>(a, st);
+  // pairs on 256 x 128 tiles where the output is narrow but the single-CTA tiles would not be
+  // split over k (they fill more than half of the SMs): half the shared-memory operand traffic per
+  // MMA of a 128 x 128 tile on one CTA
+  const long long t128 = (long long)((a.N + 127) / 128) * ((a.M + kBM - 1) / kBM);
+  if (2 * t128 > device_sms() && p128 < c128 && p128 < c64) return launch_t2<kMode, 128>(a, st);
   if (c128 <= c64) return launch_split<kMode, 128>(a, st);
   return launch_split<kMode, 64>(a, st);  // few tokens: spread the weight stream over more SMs
 }
