@@ -55,7 +55,7 @@ int device_sms() {
 }
 
 // ------------------------------------------------------------------------ workspace plans
-// Layout: [reserved counters | x codes [M,K] | s_x [M] | partials]
+// Layout: [reserved counters | x codes [M,K] | s_x [M], sums of |codes| [M] | partials]
 
 LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
   LinearWs w{};
@@ -63,7 +63,7 @@ LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms) {
   w.xf16 = off;
   if (int8_path) off += round_up((size_t)M * K * 2, 256);
   w.sx = off;
-  if (int8_path) off += round_up((size_t)M * 4, 256);
+  if (int8_path) off += round_up((size_t)M * 8, 256);
   w.part = off;
   off += round_up(std::max(make_stream_plan(int8_path, M, N, K, sms).partial_bytes, tc_split_partial_bytes(M, sms)), 256);
   w.total = off;
@@ -173,10 +173,12 @@ static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N,
   if (int8 && pre && pre->codes16 && !dbg) {  // the producer of X quantised it already
     a.A = pre->codes16;
     a.s_x = pre->s_x;
+    a.qsum = pre->qsum;
     a.s_w = s_w;
   } else if (int8) {
+    int* qsum = reinterpret_cast<int*>(s_x + M);  // beside s_x in the workspace
     w8a8_status q = launch_quantize_rows(X, M, K, inv_delta, dbg ? dbg->xq : nullptr,
-                                         reinterpret_cast<uint16_t*>(codes), s_x, st);
+                                         reinterpret_cast<uint16_t*>(codes), s_x, st, qsum);
     if (q == W8A8_OK && dbg && dbg->s_x)
       q = cudaMemcpyAsync(dbg->s_x, s_x, sizeof(float) * M, cudaMemcpyDeviceToDevice, st) == cudaSuccess
               ? W8A8_OK
@@ -187,6 +189,7 @@ static bool tc_path(bool int8, const void* W16, const uint16_t* X, int M, int N,
     }
     a.A = codes;
     a.s_x = s_x;
+    a.qsum = qsum;
     a.s_w = s_w;
     a.acc_dbg = dbg ? dbg->acc : nullptr;
   } else {

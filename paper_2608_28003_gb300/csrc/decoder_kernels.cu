@@ -65,6 +65,7 @@ struct RowQuant {
   const float* inv_delta;  // [H]; null: no codes
   uint16_t* codes;         // [M, H] fp16
   float* s_x;              // [M]
+  int* qsum;               // [M] nullable: sum_k |q_tk| (the tensor-core GEMM's exactness certificate)
 };
 __device__ __forceinline__ void row_quantize(const RowQuant& q, int row, int H, const float (&x)[kRowVec][8],
                                              float* red) {
@@ -86,6 +87,8 @@ __device__ __forceinline__ void row_quantize(const RowQuant& q, int row, int H, 
   const float r = m > 0.0f ? __fdiv_rn(127.0f, m) : 0.0f;
   if (threadIdx.x == 0) q.s_x[row] = __fdiv_rn(m, 127.0f);
 #pragma unroll
+  int qs = 0;
+#pragma unroll
   for (int v = 0; v < kRowVec; ++v) {
     const int vi = threadIdx.x + v * kRowThreads;
     if (vi < nv) {
@@ -94,9 +97,23 @@ __device__ __forceinline__ void row_quantize(const RowQuant& q, int row, int H, 
       for (int e = 0; e < 4; ++e) {
         const int q0 = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][2 * e], r))));
         const int q1 = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][2 * e + 1], r))));
+        qs += abs(q0) + abs(q1);
         h[e] = (uint32_t)int_to_f16_bits(q0) | ((uint32_t)int_to_f16_bits(q1) << 16);
       }
       reinterpret_cast<uint4*>(q.codes + (size_t)row * H)[vi] = make_uint4(h[0], h[1], h[2], h[3]);
+    }
+  }
+  if (q.qsum) {  // integer sum over the block (exact in any order)
+    __shared__ int qred[kRowThreads / 32];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) qs += __shfl_xor_sync(0xffffffffu, qs, o);
+    if ((threadIdx.x & 31) == 0) qred[threadIdx.x >> 5] = qs;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int t = 0;
+#pragma unroll
+      for (int w = 0; w < kRowThreads / 32; ++w) t += qred[w];
+      q.qsum[row] = t;
     }
   }
 }
@@ -504,21 +521,21 @@ int attention_splits(const AttnShape& s, int sm_count) {
 
 w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embed, int vocab, int H, float embed_scale,
                               const float* w, float eps, float* r, uint16_t* a, cudaStream_t st, const float* q_inv_delta,
-                              uint16_t* q_codes, float* q_sx) {
+                              uint16_t* q_codes, float* q_sx, int* q_sum) {
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "embed: hidden %d unsupported", H);
   W8A8_CUDA(launch_pdl(embed_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, tokens, vocab, embed, H, embed_scale, w,
-                       eps, r, a, RowQuant{q_inv_delta, q_codes, q_sx}));
+                       eps, r, a, RowQuant{q_inv_delta, q_codes, q_sx, q_sum}));
   return W8A8_OK;
 }
 
 w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w_post, const float* w_next, float eps,
                                  float* r, uint16_t* a, cudaStream_t st, const float* q_inv_delta, uint16_t* q_codes,
-                                 float* q_sx) {
+                                 float* q_sx, int* q_sum) {
   if (M == 0) return W8A8_OK;
   W8A8_CHECK_ARG(H % 8 == 0 && H <= 8 * kRowVec * kRowThreads, W8A8_ERR_SHAPE, "residual norm: hidden %d unsupported", H);
   W8A8_CUDA(launch_pdl(residual_norm_kernel, dim3(M), dim3(kRowThreads), 0, st, y, H, w_post, w_next, eps, r, a,
-                       RowQuant{q_inv_delta, q_codes, q_sx}));
+                       RowQuant{q_inv_delta, q_codes, q_sx, q_sum}));
   return W8A8_OK;
 }
 

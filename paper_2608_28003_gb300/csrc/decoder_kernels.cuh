@@ -18,12 +18,13 @@ struct AttnShape {
 // s_x [M], bit-identical to the stand-alone quantiser), so that linear needs no launch of its own.
 w8a8_status launch_embed_norm(const int32_t* tokens, int M, const uint16_t* embed, int vocab, int H, float embed_scale,
                               const float* w, float eps, float* r, uint16_t* a, cudaStream_t st,
-                              const float* q_inv_delta = nullptr, uint16_t* q_codes = nullptr, float* q_sx = nullptr);
+                              const float* q_inv_delta = nullptr, uint16_t* q_codes = nullptr, float* q_sx = nullptr,
+                              int* q_sum = nullptr);
 
 // r += rmsnorm(y) * w_post;  a = bf16(rmsnorm(r) * w_next); the quantiser as above
 w8a8_status launch_residual_norm(const uint16_t* y, int M, int H, const float* w_post, const float* w_next, float eps,
                                  float* r, uint16_t* a, cudaStream_t st, const float* q_inv_delta = nullptr,
-                                 uint16_t* q_codes = nullptr, float* q_sx = nullptr);
+                                 uint16_t* q_codes = nullptr, float* q_sx = nullptr, int* q_sum = nullptr);
 
 // Per row: q heads and k head RMS-normalised (weights qn, kn; skipped when null), RoPE at position
 // *pos0 + t, q -> fp32 [M, n_q*hd], k and v -> bf16 KV cache [B][max_seq][n_kv*hd] of this layer.

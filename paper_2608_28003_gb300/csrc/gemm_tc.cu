@@ -61,10 +61,32 @@ __host__ __device__ constexpr int chunk_stages(int len) {
 __host__ __device__ constexpr int chunk_count(int len) {
   return len <= 0 ? 1 : (len + chunk_stages(len) - 1) / chunk_stages(len);
 }
+// The fold exists because a fp32 sum of integer products is exact only while every partial sum
+// stays within 2^24.  Weight codes are at most 127 in magnitude, so for token t every partial sum
+// of its products, in any order or grouping, is bounded by 127 sum_k |q_tk|: a tile whose tokens
+// all have sum_k |q_tk| <= kExactQsum needs no fold at all (one accumulator over the whole k
+// range, exact, as the bf16 path runs).  The bound is data-dependent; the quantiser reports the
+// sums, and tiles that fail it take the chunked path.
+constexpr int kExactQsum = (1 << 24) / 127;  // 132104: 127 x 132104 <= 2^24
 constexpr int kEpiWarps = 16;                   // four per TMEM lane quarter: one per column quarter
 constexpr int kParts = kEpiWarps / 4;
 constexpr int kProdWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1;
 constexpr int kThreads = 32 * (kEpiWarps + 2);
+// The 512 epilogue threads test the rows once per kernel, while the first stages load: bit i of
+// *fail is set when row tile i (rows_per_tile tokens) has a token past the bound.  Row tiles past
+// the 32nd always take the chunked path.  Ends with the epilogue warps' named barrier 3; the
+// first thread then arrives on the MMA issuer's barrier.
+__device__ __forceinline__ void scan_exact(const TcArgs& a, int rows_per_tile, uint32_t* fail, uint32_t ready) {
+  const int rows = min(a.M, 32 * rows_per_tile);
+  uint32_t f = 0u;
+  for (int i = threadIdx.x; i < rows; i += 32 * kEpiWarps)
+    if (__ldg(a.qsum + i) > kExactQsum) f |= 1u << (i / rows_per_tile);
+  f = __reduce_or_sync(0xffffffffu, f);
+  if ((threadIdx.x & 31) == 0 && f) atomicOr(fail, f);
+  named_bar_sync(3, 32 * kEpiWarps);
+  if (threadIdx.x == 0) mbar_arrive(ready);
+}
+__device__ __forceinline__ bool row_tile_exact(uint32_t fail, int i) { return i < 32 && !((fail >> i) & 1u); }
 constexpr uint32_t kTmemCols = 512;  // all of an SM's tensor memory: 2 (bf16) or 4 (W8A8) accumulator slots
 constexpr uint32_t kABytes = kBM * kBK * 2;
 constexpr int kStageBufBytes = 32 * 64;                  // one epilogue block: 32 rows of 64 bytes
@@ -196,13 +218,26 @@ __device__ __forceinline__ void load_colvals(const TcArgs& a, bool want_sw, int 
 }
 // fl(fl(s_x s_w) acc) (+ bias) of one 32-column group (Eq. gemm-final); acc is the INT32 sum
 // (W8A8) or the fp32 one (FP8); sw / b are this lane's column values of the group.
+// Two IEEE fp32 products, each rounded to nearest even (the packed form of two __fmul_rn).
+__device__ __forceinline__ void fmul2_rn(float a0, float a1, float b0, float b1, float& d0, float& d1) {
+  const unsigned long long x = ((unsigned long long)__float_as_uint(a1) << 32) | __float_as_uint(a0);
+  const unsigned long long y = ((unsigned long long)__float_as_uint(b1) << 32) | __float_as_uint(b0);
+  unsigned long long z;
+  asm("mul.rn.f32x2 %0, %1, %2;\n" : "=l"(z) : "l"(x), "l"(y));
+  d0 = __uint_as_float((uint32_t)z);
+  d1 = __uint_as_float((uint32_t)(z >> 32));
+}
 template <typename T>
 __device__ __forceinline__ void dequant32(bool has_bias, float sx, float sw, float b, const T* acc, float (&v)[32]) {
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    float y = __fmul_rn(__fmul_rn(sx, __shfl_sync(0xffffffffu, sw, j)), acc_as_f32<T>(acc[j]));
-    if (has_bias) y = __fadd_rn(y, __shfl_sync(0xffffffffu, b, j));
-    v[j] = y;
+  for (int j = 0; j < 32; j += 2) {
+    float t0, t1;
+    fmul2_rn(sx, sx, __shfl_sync(0xffffffffu, sw, j), __shfl_sync(0xffffffffu, sw, j + 1), t0, t1);
+    fmul2_rn(t0, t1, acc_as_f32<T>(acc[j]), acc_as_f32<T>(acc[j + 1]), v[j], v[j + 1]);
+    if (has_bias) {
+      v[j] = __fadd_rn(v[j], __shfl_sync(0xffffffffu, b, j));
+      v[j + 1] = __fadd_rn(v[j + 1], __shfl_sync(0xffffffffu, b, j + 1));
+    }
   }
 }
 __device__ __forceinline__ void add_bias32(float b, float (&v)[32]) {
@@ -369,9 +404,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int BN = GG::BN, S = GG::S;
   constexpr int SC = slot_cols(BN), NSLOT = (int)kTmemCols / SC;  // accumulator slots in tensor memory
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
+  __shared__ uint64_t bars[2 * S + 2 * NSLOT + 2];
   __shared__ uint32_t tmem_slot;
   __shared__ int s_flag, s_last;
+  __shared__ uint32_t s_fail;  // W8A8: row tiles with a token past the exactness bound
 
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -383,11 +419,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int KS = a.ksplit > 1 ? a.ksplit : 1, units = tiles * KS;
   auto kb_lo = [&](int u) { return (int)((long long)(u % KS) * nkb / KS); };
   auto kb_hi = [&](int u) { return (int)((long long)(u % KS + 1) * nkb / KS); };
-  // accumulator chunks of a unit: W8A8 restarts every chunk_stages(len) stages (at most 1024 k)
-  // counted from the unit's first stage
-  auto chunks_of = [&](int u) { return kInt8 ? chunk_count(kb_hi(u) - kb_lo(u)) : 1; };
+  // accumulator chunks of a unit (warp-collective): W8A8 restarts every chunk_stages(len) stages
+  // (at most 1024 k) counted from the unit's first stage, unless the tile's tokens pass the
+  // exactness bound (one chunk)
+  // W8A8 row tiles are tested against the exactness bound when a tile's k range is not split (split
+  // units are short: their first fold boundary would come before the scan ends) and spans more than
+  // one chunk
+  const bool scan = kInt8 && a.qsum != nullptr && KS == 1 && nkb > kKbPerChunk;
+  auto unit_chunks = [&](int u) {  // epilogue side, after the scan
+    const int n = kInt8 ? chunk_count(kb_hi(u) - kb_lo(u)) : 1;
+    return n > 1 && !(scan && row_tile_exact(s_fail, (u / KS) / NT)) ? n : 1;
+  };
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
-                 done = acce0 + 8 * NSLOT;
+                 done = acce0 + 8 * NSLOT, ready = done + 8;
 
   pdl_trigger();
   if (warp == kProdWarp && lane == 0) {
@@ -405,6 +449,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(acce0 + 8 * b, 32 * kEpiWarps);
     }
     mbar_init(done, 1);
+    mbar_init(ready, 1);
+    s_fail = 0u;
     fence_mbar_init();
   }
   if (warp == kMmaWarp) {
@@ -453,38 +499,63 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16(kMode == kModeBf16 ? 1u : 0u, BN, kBM);
-      bool ok = true;
+      bool ok = true, known = false;  // known: the epilogue's exactness scan has been read
+      uint32_t fail = 0u;
       int g = 0, q = 0;  // stages consumed, accumulator chunks produced
+      // One accumulator slot per chunk; a W8A8 unit restarts in the next slot at each fold boundary
+      // (every chunk_stages(len) stages) unless its row tile passed the exactness bound, which is
+      // first needed at the first boundary, when the scan has long finished.
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        const int nch = chunks_of(u), ulo = kb_lo(u), uhi = kb_hi(u);
-        for (int c = 0; c < nch && ok; ++c, ++q) {
-          const int slot = q % NSLOT;
-          if (q >= NSLOT &&  // the epilogue has drained this slot's previous chunk
-              !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+        const int ulo = kb_lo(u), uhi = kb_hi(u), per = kInt8 ? chunk_stages(uhi - ulo) : uhi - ulo;
+        int slot = q % NSLOT, kb0 = ulo, next_fold = ulo + per;
+        if (q >= NSLOT &&  // the epilogue has drained this slot's previous chunk
+            !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t d = tmem + (uint32_t)(slot * SC);
+        for (int kb = ulo; kb < uhi; ++kb, ++g) {
+          if (kInt8 && kb == next_fold) {  // a fold boundary
+            next_fold += per;
+            if (scan && !known) {
+              if (!mbar_wait_bounded(ready, 0u, kWaitBudgetCycles)) {
+                ok = false;
+                break;
+              }
+              fail = s_fail;
+              known = true;
+            }
+            if (!(scan && row_tile_exact(fail, (u / KS) / NT))) {
+              tc_commit(accf0 + 8 * slot);
+              ++q;
+              slot = q % NSLOT;
+              if (q >= NSLOT &&
+                  !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              d = tmem + (uint32_t)(slot * SC);
+              kb0 = kb;
+            }
+          }
+          const int s = g % S;
+          if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d = tmem + (uint32_t)(slot * SC);
-          const int per = chunk_stages(uhi - ulo);
-          const int kb0 = kInt8 ? ulo + c * per : ulo, kb1 = kInt8 ? min(uhi, kb0 + per) : uhi;
-          for (int kb = kb0; kb < kb1; ++kb, ++g) {
-            const int s = g % S;
-            if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
 #pragma unroll
-            for (int k16 = 0; k16 < kSwz / 32; ++k16) {  // 32 bytes of k per instruction
-              const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
-              const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BBytes + 32u * k16);
-              tc_mma_m<kMode>(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
-            }
-            tc_commit(empty0 + 8 * s);
+          for (int k16 = 0; k16 < kSwz / 32; ++k16) {  // 32 bytes of k per instruction
+            const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
+            const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BBytes + 32u * k16);
+            tc_mma_m<kMode>(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
           }
-          if (ok) tc_commit(accf0 + 8 * slot);
+          tc_commit(empty0 + 8 * s);
         }
+        if (ok) tc_commit(accf0 + 8 * slot);
+        ++q;
       }
       if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
       tc_commit(done);  // completes once every MMA issued above has completed
@@ -492,6 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------------------------------------------------------------- epilogue warps 0-15
+    if (scan) scan_exact(a, kBM, &s_fail, ready);
     const int quad = warp & 3, part = warp >> 2;  // TMEM lane quarter (tokens), column quarter
     const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
     const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
@@ -539,10 +611,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         int isum[32 * NG];
 #pragma unroll
         for (int j = 0; j < 32 * NG; ++j) isum[j] = 0;
-        const int nch = chunks_of(u);
+        const int nch = unit_chunks(u);
         ColVals<NG> cv;  // before the first wait: the loads overlap the MMAs
         if (KS == 1) load_colvals<NG>(a, true, n0, part, BN, lane, cv);
         const float sx = KS == 1 && row < a.M ? a.s_x[row] : 0.0f;
+        if (nch == 1 && KS == 1) {  // one exact fp32 accumulator: the INT32 sum as a float
+          const int slot = q % NSLOT;
+          if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
+            ok = false;
+            atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int i = 0; i < NG; ++i) {
+            const int g = part + kParts * i;
+            if (g >= BN / 32) break;
+            uint32_t r[32];
+            tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
+            if (a.acc_dbg && row < a.M) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (n0 + 32 * g + j < a.N)
+                  a.acc_dbg[(size_t)row * a.N + n0 + 32 * g + j] = __float2int_rn(__uint_as_float(r[j]));
+            }
+            float v[32];
+            dequant32(a.bias != nullptr, sx, cv.sw[i], cv.b[i], r, v);
+            emit32(32 * g, v);
+          }
+          tc_fence_before();
+          mbar_arrive(acce0 + 8 * slot);
+          ++q;
+          if (want_top && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
+          continue;
+        }
         for (int c = 0; c < nch; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
@@ -753,9 +855,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   constexpr int BN = GG::BN, S = GG::S;
   constexpr int SC = slot_cols(BN), NSLOT = (int)kTmemCols / SC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t bars[2 * S + 2 * NSLOT + 1];
+  __shared__ uint64_t bars[2 * S + 2 * NSLOT + 2];
   __shared__ uint32_t tmem_slot;
   __shared__ int s_flag;
+  __shared__ uint32_t s_fail;  // W8A8: row tiles with a token past the exactness bound
 
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -767,8 +870,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int nkb = (a.K + BKe - 1) / BKe;
   const int nchunks = kInt8 ? chunk_count(nkb) : 1;
   const int kb_per_chunk = kInt8 ? chunk_stages(nkb) : nkb;
+  // accumulator chunks of tile t (warp-collective): one where its 256 tokens pass the exactness bound
+  // W8A8 row tiles (256 tokens) are tested against the exactness bound when K spans several chunks
+  const bool scan = kInt8 && a.qsum != nullptr && nchunks > 1;
+  auto tile_chunks = [&](int t) {  // epilogue side, after the scan
+    return nchunks > 1 && !(scan && row_tile_exact(s_fail, t / NT)) ? nchunks : 1;
+  };
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, accf0 = full0 + 16 * S, acce0 = accf0 + 8 * NSLOT,
-                 done = acce0 + 8 * NSLOT;
+                 done = acce0 + 8 * NSLOT, ready = done + 8;
 
   pdl_trigger();
   if (warp == kProdWarp && lane == 0) {
@@ -786,6 +895,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(acce0 + 8 * b, 2 * 32 * kEpiWarps);  // both CTAs' epilogue threads
     }
     mbar_init(done, 1);
+    mbar_init(ready, 1);
+    s_fail = 0u;
     fence_mbar_init();
   }
   if (warp == kMmaWarp) {
@@ -833,36 +944,61 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------------- MMA issuer (CTA 0)
     if (lane == 0 && rank == 0) {
       constexpr uint32_t idesc = idesc_f16(kMode == kModeBf16 ? 1u : 0u, BN, 2 * kBM);
-      bool ok = true;
+      bool ok = true, known = false;  // known: this CTA's exactness scan has been read
+      uint32_t fail = 0u;
       int g = 0, q = 0;
+      // As in the single-CTA kernel: a W8A8 tile restarts in the next slot at each fold boundary
+      // unless its row tile passed the exactness bound.
       for (int t = pair; t < tiles && ok; t += npairs) {
-        for (int c = 0; c < nchunks && ok; ++c, ++q) {
-          const int slot = q % NSLOT;
-          if (q >= NSLOT &&
-              !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+        int slot = q % NSLOT, kb0 = 0, next_fold = kb_per_chunk;
+        if (q >= NSLOT &&
+            !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t d = tmem + (uint32_t)(slot * SC);
+        for (int kb = 0; kb < nkb; ++kb, ++g) {
+          if (kInt8 && kb == next_fold) {  // a fold boundary
+            next_fold += kb_per_chunk;
+            if (scan && !known) {
+              if (!mbar_wait_bounded(ready, 0u, kWaitBudgetCycles)) {
+                ok = false;
+                break;
+              }
+              fail = s_fail;
+              known = true;
+            }
+            if (!(scan && row_tile_exact(fail, t / NT))) {
+              tc2_commit_both(accf0 + 8 * slot);
+              ++q;
+              slot = q % NSLOT;
+              if (q >= NSLOT &&
+                  !mbar_wait_bounded(acce0 + 8 * slot, (uint32_t)(((q / NSLOT) - 1) & 1), kWaitBudgetCycles)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              d = tmem + (uint32_t)(slot * SC);
+              kb0 = kb;
+            }
+          }
+          const int s = g % S;
+          if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d = tmem + (uint32_t)(slot * SC);
-          const int kb0 = c * kb_per_chunk, kb1 = min(nkb, kb0 + kb_per_chunk);
-          for (int kb = kb0; kb < kb1; ++kb, ++g) {
-            const int s = g % S;
-            if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)((g / S) & 1), kWaitBudgetCycles)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
 #pragma unroll
-            for (int k16 = 0; k16 < kSwz / 32; ++k16) {  // 32 bytes of k per instruction
-              const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
-              const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BHalf + 32u * k16);
-              tc2_mma_m<kMode>(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
-            }
-            tc2_commit_both(empty0 + 8 * s);
+          for (int k16 = 0; k16 < kSwz / 32; ++k16) {  // 32 bytes of k per instruction
+            const uint64_t ad = sdesc_swz(sA + (uint32_t)s * kABytes + 32u * k16);
+            const uint64_t bd = sdesc_swz(sB + (uint32_t)s * GG::BHalf + 32u * k16);
+            tc2_mma_m<kMode>(d, ad, bd, idesc, (kb == kb0 && k16 == 0) ? 0u : 1u);
           }
-          if (ok) tc2_commit_both(accf0 + 8 * slot);
+          tc2_commit_both(empty0 + 8 * s);
         }
+        if (ok) tc2_commit_both(accf0 + 8 * slot);
+        ++q;
       }
       if (!ok) atomicOr(a.err, DEVERR_PRODUCER_WAIT);
       tc2_commit(done);
@@ -870,6 +1006,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------------------------------------------------------------- epilogue warps 0-15 (both CTAs)
+    if (scan) scan_exact(a, 2 * kBM, &s_fail, ready);
     const int quad = warp & 3, part = warp >> 2;
     const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
     const bool want_top = a.kind == EPI_F32 && a.top1 != nullptr;
@@ -891,7 +1028,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         ColVals<NG> cv;  // before the first wait: the loads overlap the MMAs
         load_colvals<NG>(a, true, n0, part, BN, lane, cv);
         const float sx = row < a.M ? a.s_x[row] : 0.0f;
-        for (int c = 0; c < nchunks; ++c, ++q) {
+        const int nch = tile_chunks(t);
+        if (nch == 1) {  // one exact fp32 accumulator: it is the INT32 sum as a float; dequantise directly
+          const int slot = q % NSLOT;
+          if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
+            ok = false;
+            atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int i = 0; i < NG; ++i) {
+            const int g = part + kParts * i;
+            if (g >= BN / 32) break;
+            uint32_t r[32];
+            tmem_ld32(lane_base + (uint32_t)(slot * SC + 32 * g), r);
+            if (a.acc_dbg && row < a.M) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (n0 + 32 * g + j < a.N)
+                  a.acc_dbg[(size_t)row * a.N + n0 + 32 * g + j] = __float2int_rn(__uint_as_float(r[j]));
+            }
+            float v[32];
+            dequant32(a.bias != nullptr, sx, cv.sw[i], cv.b[i], r, v);
+            emit(32 * g, v);
+          }
+          tc_fence_before();
+          mbar_arrive_cluster(acce_lead + 8 * slot);
+          ++q;
+          if (want_top && row < a.M && best != 0ull) atomicMax(a.top_keys + row, best);
+          continue;
+        }
+        for (int c = 0; c < nch; ++c, ++q) {
           const int slot = q % NSLOT;
           if (!mbar_wait_bounded(accf0 + 8 * slot, (uint32_t)((q / NSLOT) & 1), kWaitBudgetCycles)) {
             ok = false;
@@ -1066,15 +1234,20 @@ constexpr int kMinKbPerPart = 2;
 // under the cap) would lose.
 constexpr int kMinParts = 4;
 
-template <int kMode, int kBN>
-w8a8_status launch_split(TcArgs a, cudaStream_t st) {
-  const int sms = device_sms(), nkb = (a.K + bk_elems(kMode) - 1) / bk_elems(kMode);
-  const long long tiles = (long long)((a.N + kBN - 1) / kBN) * ((a.M + kBM - 1) / kBM);
-  a.ksplit = 1;
+// k parts of a single-CTA call on BN-column tiles (1: no split)
+int split_parts(const TcArgs& a, int mode, int bn) {
+  const int sms = device_sms(), nkb = (a.K + bk_elems(mode) - 1) / bk_elems(mode);
+  const long long tiles = (long long)((a.N + bn - 1) / bn) * ((a.M + kBM - 1) / kBM);
   if (a.kind == EPI_BF16 && a.partials && a.tile_counters && 2 * tiles <= sms) {
     const int ks = std::min({(int)(sms / tiles), nkb / kMinKbPerPart, a.K / (4 * a_box_rows(a.M))});
-    if (ks >= kMinParts) a.ksplit = ks;
+    if (ks >= kMinParts) return ks;
   }
+  return 1;
+}
+
+template <int kMode, int kBN>
+w8a8_status launch_split(TcArgs a, cudaStream_t st) {
+  a.ksplit = split_parts(a, kMode, kBN);
   return launch_t<kMode, kBN>(a, st);
 }
 
@@ -1082,20 +1255,29 @@ template <int kMode>
 w8a8_status dispatch(TcArgs a, cudaStream_t st) {
   a.ksplit = 1;
   const long long pairs = device_sms() / 2;
-  auto cost = [&](int bm, int bn, double unit, long long slots) {
-    const long long t = (long long)((a.N + bn - 1) / bn) * ((a.M + bm - 1) / bm);
-    return (double)((t + slots - 1) / slots) * bn * unit;
+  // ks k parts: ks units per tile, each with 1/ks of the k range, plus the partials' round trip
+  // (taken as a third of a unit's time).  Counted from 256 tokens on the bf16 and W8A8 paths only:
+  // there it picks split 128-column tiles over one wave of 64-column tiles (512 x 6912 -> 1152:
+  // bf16 38.6 -> 32.4 us, W8A8 42.6 -> 33.4 us), while below it, and on the FP8 path, it measured
+  // slower than the split-free model (128-token prefill 1.87 -> 2.22 ms; FP8 at 512 tokens 23 -> 29 us)
+  const bool split_cost = a.M >= 256 && kMode != kModeFp8;
+  auto cost = [&](int bm, int bn, double unit, long long slots, int ks = 1) {
+    const long long t = (long long)((a.N + bn - 1) / bn) * ((a.M + bm - 1) / bm) * ks;
+    return (double)((t + slots - 1) / slots) * bn * unit / ks * (ks > 1 ? 1.33 : 1.0);
   };
   const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
-               p128 = cost(2 * kBM, 128, 1.32, pairs), c128 = cost(kBM, 128, 1.81, 2 * pairs),
-               c64 = cost(kBM, 64, 2.7, 2 * pairs);
+               c128 = cost(kBM, 128, 1.81, 2 * pairs, split_cost ? split_parts(a, kMode, 128) : 1),
+               c64 = cost(kBM, 64, 2.7, 2 * pairs, split_cost ? split_parts(a, kMode, 64) : 1);
+  // W8A8 only: pairs on 256 x 128 tiles where the output is narrow but the single-CTA tiles would
+  // not be split over k (they fill more than half of the SMs); four 128-column accumulator slots
+  // keep the fold chunks of a long k range in flight (measured on 2048 x 6912 -> 1152: 42.7 us
+  // against 45.7 us on single CTAs; the bf16 and FP8 paths measured no gain)
+  const double p128 = kMode == kModeI8 ? cost(2 * kBM, 128, 1.32, pairs) : 1e30;
   if (c256 <= c192 && c256 <= c128 && c256 <= c64 && c256 <= p128) return launch_t2<kMode, 256>(a, st);
   if (c192 <= c128 && c192 <= c64 && c192 <= p128) return launch_t2<kMode, 192>(a, st);
-  // pairs on 256 x 128 tiles where the output is narrow but the single-CTA tiles would not be
-  // split over k (they fill more than half of the SMs): half the shared-memory operand traffic per
-  // MMA of a 128 x 128 tile on one CTA
   const long long t128 = (long long)((a.N + 127) / 128) * ((a.M + kBM - 1) / kBM);
-  if (2 * t128 > device_sms() && p128 < c128 && p128 < c64) return launch_t2<kMode, 128>(a, st);
+  if (kMode == kModeI8 && 2 * t128 > device_sms() && p128 < c128 && p128 < c64) return launch_t2<kMode, 128>(a, st);
+
   if (c128 <= c64) return launch_split<kMode, 128>(a, st);
   return launch_split<kMode, 64>(a, st);  // few tokens: spread the weight stream over more SMs
 }

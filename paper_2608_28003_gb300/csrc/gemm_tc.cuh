@@ -17,6 +17,8 @@ struct TcArgs {
   int M, N, K;
   int kind;             // EPI_BF16, EPI_GEGLU or EPI_F32
   const float* s_x;     // [M] W8A8 / FP8: per-token scales
+  const int* qsum;      // [M] W8A8, nullable: sum_k |q_tk| per token; a tile whose tokens all have
+                        // 127 qsum <= 2^24 runs one exact fp32 accumulator over all of k (no folds)
   const float* s_w;     // [N] W8A8 / FP8: per-channel scales
   const float* bias;    // [N] nullable
   uint16_t* y;          // bf16 [M, N] (EPI_BF16) or [M, N / 2] (EPI_GEGLU)

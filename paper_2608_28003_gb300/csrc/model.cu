@@ -63,9 +63,11 @@ struct w8a8_model {
   void* attn_ws = nullptr;
   size_t attn_ws_bytes = 0;
   // the next W8A8 linear's quantised input written by the norm kernels at 9+ tokens ([max_tokens,
-  // hidden] fp16 codes and [max_tokens] scales), so that its GEMM needs no quantiser launch
+  // hidden] fp16 codes, [max_tokens] scales and sums of |codes|), so that its GEMM needs no
+  // quantiser launch
   uint16_t* pcodes = nullptr;
   float* psx = nullptr;
+  int* psum = nullptr;
   // diagnostics: when set, a forward copies every layer's output (the residual stream after its
   // post-FFN step, fp32 [M, H]) to capture + l M H
   float* capture = nullptr;
@@ -156,11 +158,11 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
   // tensor-core GEMM then needs no quantiser launch); fewer tokens run the decode GEMV, which
   // quantises inside
   const bool preq = !calib && M >= 9 && m->prepared;
-  const PreCodes pc{m->pcodes, m->psx};
+  const PreCodes pc{m->pcodes, m->psx, m->psum};
   auto att8_of = [&](int l) { return !calib && m->prepared && ((m->attn_bits >> l) & 1u); };
   const bool pre0 = preq && att8_of(0);
   W8A8_TRY(launch_embed_norm(tokens, M, m->embed, c.vocab, H, m->embed_scale, m->L[0].ln_in, c.eps, rc, m->a, st,
-                             pre0 ? m->q_qkv[0].inv_delta : nullptr, m->pcodes, m->psx));
+                             pre0 ? m->q_qkv[0].inv_delta : nullptr, m->pcodes, m->psx, m->psum));
   bool pre_qkv = pre0;  // whether the codes of the current q/k/v input exist
   const w8a8_trace* tr = m->trace_on && !calib ? &m->trace : nullptr;
   W8A8_CHECK_ARG(!tr || M <= tr->max_rows, W8A8_ERR_SHAPE, "trace: %d rows exceed the trace's %d", M, tr ? tr->max_rows : 0);
@@ -222,7 +224,7 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
     } else {
       const bool pre_gu = preq && ffn8;
       W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_attn, W.ln_pre_ffn, c.eps, rc, m->a, st,
-                                    pre_gu ? m->q_gu[l].inv_delta : nullptr, m->pcodes, m->psx));
+                                    pre_gu ? m->q_gu[l].inv_delta : nullptr, m->pcodes, m->psx, m->psum));
       if (calib) W8A8_TRY(launch_act_absmax(m->a, M, H, m->stat_gu(l), st));
       if (tr) W8A8_TRY(trace_copy(tr->a_ffn, l, m->a, H, 2));
       uint16_t* h_out = calib ? m->h : nullptr;
@@ -235,7 +237,7 @@ w8a8_status forward_core(w8a8_model* m, const int32_t* tokens, int B, int T, flo
       const float* next = l + 1 < c.layers ? m->L[l + 1].ln_in : m->final_norm;
       pre_qkv = preq && l + 1 < c.layers && att8_of(l + 1);
       W8A8_TRY(launch_residual_norm(m->y, M, H, W.ln_post_ffn, next, c.eps, rc, m->a, st,
-                                    pre_qkv ? m->q_qkv[l + 1].inv_delta : nullptr, m->pcodes, m->psx));
+                                    pre_qkv ? m->q_qkv[l + 1].inv_delta : nullptr, m->pcodes, m->psx, m->psum));
     }
     if (m->capture)
       W8A8_CUDA(cudaMemcpyAsync(m->capture + (size_t)l * M * H, rc, sizeof(float) * M * H, cudaMemcpyDeviceToDevice, st));
@@ -439,6 +441,7 @@ extern "C" w8a8_status w8a8_model_create(const w8a8_model_cfg* cfg, const w8a8_l
   W8A8_MTRY(dalloc(m, reinterpret_cast<char**>(&m->attn_ws), aws));
   W8A8_MTRY(dalloc(m, &m->pcodes, (size_t)c.max_tokens * H));
   W8A8_MTRY(dalloc(m, &m->psx, (size_t)c.max_tokens + 4));
+  W8A8_MTRY(dalloc(m, &m->psum, (size_t)c.max_tokens + 4));
   cudaStream_t st = m->st;
   W8A8_MTRY(cudaMemsetAsync(m->ws, 0, W8A8_WS_RESERVED, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);
   W8A8_MTRY(cudaMemsetAsync(m->attn_ws, 0, aws, st) == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA);

@@ -22,18 +22,21 @@ struct FfnWs {
 LinearWs linear_ws(int M, int N, int K, bool int8_path, int sms);
 FfnWs ffn_ws(int M, int H, int F, int sms);
 
+// qsum (nullable): per row, sum_k |q_tk| (the tensor-core GEMM's exactness certificate)
 w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* inv_delta, int8_t* xq,
-                                 uint16_t* xq_f16, float* s_x, cudaStream_t st);
+                                 uint16_t* xq_f16, float* s_x, cudaStream_t st, int* qsum = nullptr);
 w8a8_status launch_quantize_rows_fp8(const uint16_t* X, int M, int K, const float* inv_delta, uint8_t* xq,
                                      float* s_x, cudaStream_t st);
 w8a8_status launch_act_absmax(const uint16_t* X, int T, int K, float* absmax, cudaStream_t st);
 
 // The per-token quantiser's outputs for X computed by the kernel that produced X (the decoder's
-// norm kernels): fp16 codes [M, K] and s_x [M].  A W8A8 linear that runs the tensor-core GEMM then
-// launches no quantiser of its own; other routes quantise X themselves and ignore them.
+// norm kernels): fp16 codes [M, K], s_x [M] and the rows' sums of |codes| [M] (nullable).  A W8A8
+// linear that runs the tensor-core GEMM then launches no quantiser of its own; other routes
+// quantise X themselves and ignore them.
 struct PreCodes {
   const uint16_t* codes16;
   const float* s_x;
+  const int* qsum;
 };
 
 // kind: 0 bf16 output, 1 GeGLU, 2 fp32 logits (+ top-1)

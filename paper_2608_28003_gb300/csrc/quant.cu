@@ -23,7 +23,7 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __re
                                                            const float* __restrict__ inv_delta,
                                                            int8_t* __restrict__ xq,
                                                            uint16_t* __restrict__ xq_f16,
-                                                           float* __restrict__ s_x) {
+                                                           float* __restrict__ s_x, int* __restrict__ qsum) {
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x;
@@ -81,6 +81,7 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __re
   const float r = m > 0.0f ? __fdiv_rn(kQmax, m) : 0.0f;  // fl32(127 / m_t)
   if (threadIdx.x == 0) s_x[row] = __fdiv_rn(m, kQmax);  // s_t^x = fl32(m_t / 127)
 
+  int qs = 0;  // sum_k |q_tk| of this thread's codes (the GEMM's exactness certificate)
   auto emit = [&](int vi, const float (&v8)[8]) {
     if constexpr (kFp8) {  // e4m3 codes (xq receives the bytes)
       uint32_t c[4];
@@ -91,6 +92,8 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __re
       int q[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(v8[e], r))));
+#pragma unroll
+      for (int e = 0; e < 8; ++e) qs += abs(q[e]);
       if (xq) {
         uint2 packed;
         packed.x = (uint32_t)(q[0] & 0xff) | ((uint32_t)(q[1] & 0xff) << 8) | ((uint32_t)(q[2] & 0xff) << 16) |
@@ -126,15 +129,27 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint16_t* __re
       emit(vi, v8);
     }
   }
+  if (qsum) {  // one integer sum per row (exact in any order)
+    __shared__ int qred[32];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) qs += __shfl_xor_sync(0xffffffffu, qs, o);
+    if ((threadIdx.x & 31) == 0) qred[threadIdx.x >> 5] = qs;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int t = 0;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += qred[w];
+      qsum[row] = t;
+    }
+  }
 }
 
 w8a8_status launch_quantize_rows(const uint16_t* X, int M, int K, const float* inv_delta, int8_t* xq,
-                                 uint16_t* xq_f16, float* s_x, cudaStream_t st) {
+                                 uint16_t* xq_f16, float* s_x, cudaStream_t st, int* qsum) {
   if (M == 0) return W8A8_OK;
   const int nvec = K / 8;
   const int threads = nvec <= 4 * 128 ? 128 : 256;
   W8A8_CUDA(launch_pdl(quantize_rows_kernel<4, false>, dim3(M), dim3(threads), 0, st, X, K, inv_delta, xq, xq_f16,
-                       s_x));
+                       s_x, qsum));
   return W8A8_OK;
 }
 
@@ -144,7 +159,7 @@ w8a8_status launch_quantize_rows_fp8(const uint16_t* X, int M, int K, const floa
   const int nvec = K / 8;
   const int threads = nvec <= 4 * 128 ? 128 : 256;
   W8A8_CUDA(launch_pdl(quantize_rows_kernel<4, true>, dim3(M), dim3(threads), 0, st, X, K, inv_delta,
-                       reinterpret_cast<int8_t*>(xq), static_cast<uint16_t*>(nullptr), s_x));
+                       reinterpret_cast<int8_t*>(xq), static_cast<uint16_t*>(nullptr), s_x, static_cast<int*>(nullptr)));
   return W8A8_OK;
 }
 
@@ -446,7 +461,7 @@ extern "C" w8a8_status w8a8_quantize_activations(const uint16_t* X, int M, int K
                  W8A8_ERR_ALIGN, "w8a8_quantize_activations: pointers must be 16-byte aligned");
   w8a8_status s = check_device();
   if (s != W8A8_OK) return s;
-  return launch_quantize_rows(X, M, K, inv_delta, xq, xq_f16, s_x, as_stream(stream));
+  return launch_quantize_rows(X, M, K, inv_delta, xq, xq_f16, s_x, as_stream(stream), nullptr);
 }
 
 // ------------------------------------------------------------------------ FP8 (e4m3) variant

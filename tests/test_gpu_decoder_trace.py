@@ -110,11 +110,13 @@ def f32(t):
     return t.float().numpy().astype(np.float64) if t.dtype != torch.float32 else t.numpy().astype(np.float64)
 
 
-def check_norm(got, want):
-    """bf16 RMSNorm outputs: fp32 (GPU) against fp64 (oracle) sums, one rounding apart at most."""
+def check_norm(got, want, what="", in_err=0.0):
+    """bf16 RMSNorm outputs: fp32 (GPU) against fp64 (oracle) sums, one rounding apart at most;
+    in_err bounds what an error of the norm's input (absolute, per element) contributes."""
     want = OW.round_to_bf16(want.astype(np.float32)).astype(np.float64)
-    assert np.all(np.abs(got - want) <= ulp_bf16(want) + 1e-30)
-    assert np.mean(got == want) > 0.99
+    bad = np.abs(got - want) > ulp_bf16(want) + in_err + 1e-30
+    assert not bad.any(), (what, np.argwhere(bad)[:5].tolist(), got[bad][:5].tolist(), want[bad][:5].tolist())
+    assert np.mean(got == want) > 0.99, what
 
 
 def check_linear(x, got, int8, prep_q, W32):
@@ -168,7 +170,7 @@ def check_layers(run, prep, tr, rows, positions, qkv_all, eta):
             r_prev = (w["embed"][toks[positions]].astype(np.float32) * np.float32(cfg.embed_scale)).astype(np.float64)
         else:
             r_prev = f32(tr["r"][l - 1, rows])
-        check_norm(a_in, OD.rmsnorm(r_prev, w["ln_in"][l], cfg.eps))
+        check_norm(a_in, OD.rmsnorm(r_prev, w["ln_in"][l], cfg.eps), ("a_in", l))
         qkv = f32(tr["qkv"][l, rows])
         check_linear(a_in, qkv, att8, prep["qkv"].get(l), w["wqkv"][l])
         attn = f32(tr["attn"][l, rows])
@@ -178,16 +180,21 @@ def check_layers(run, prep, tr, rows, positions, qkv_all, eta):
             assert np.all(np.abs(attn[i] - ref) <= 2 * ulp_bf16(ref) + eta * vmax), (l, int(p))
         y_o = f32(tr["y_o"][l, rows])
         check_linear(attn, y_o, att8, prep["o"].get(l), w["wo"][l])
-        r_mid = r_prev + OD.rmsnorm(y_o, w["ln_post_attn"][l], cfg.eps)
+        n_o = OD.rmsnorm(y_o, w["ln_post_attn"][l], cfg.eps)
+        r_mid = r_prev + n_o
         a_ffn = f32(tr["a_ffn"][l, rows])
-        check_norm(a_ffn, OD.rmsnorm(r_mid, w["ln_pre_ffn"][l], cfg.eps))
+        # the GPU forms r_mid in fp32 (not traced): a few roundings of |r_prev| + |n_o| at 2^-24 each,
+        # scaled by the pre-FFN norm (1 / rms(r_mid) times its weight)
+        inv = 1.0 / np.sqrt(np.mean(r_mid ** 2, axis=1, keepdims=True) + cfg.eps)
+        mid_err = 4 * 2.0 ** -24 * (np.abs(r_prev) + np.abs(n_o)) * inv * np.abs(w["ln_pre_ffn"][l])
+        check_norm(a_ffn, OD.rmsnorm(r_mid, w["ln_pre_ffn"][l], cfg.eps), ("a_ffn", l), mid_err)
         h, y_f = f32(tr["h"][l, rows]), f32(tr["y_f"][l, rows])
         check_ffn(a_ffn, h, y_f, ffn8, prep["ffn"].get(l), w, l)
         r = f32(tr["r"][l, rows])
         r_ref = r_mid + OD.rmsnorm(y_f, w["ln_post_ffn"][l], cfg.eps)
         assert np.all(np.abs(r - r_ref) <= 4e-6 * np.max(np.abs(r_ref), axis=1, keepdims=True)), l
     a_fin = f32(tr["a_fin"][rows])
-    check_norm(a_fin, OD.rmsnorm(f32(tr["r"][L - 1, rows]), w["final_norm"], cfg.eps))
+    check_norm(a_fin, OD.rmsnorm(f32(tr["r"][L - 1, rows]), w["final_norm"], cfg.eps), "a_fin")
     return a_fin
 
 
