@@ -221,6 +221,34 @@ def test_w8a8_accumulator_exact_at_extremes(B, K):
     assert np.array_equal(f32_of_bf16(Y), r["y"])
 
 
+@pytest.mark.parametrize("M,N,K,bad", [(640, 4608, 1152, (256, 512)),   # CTA pairs, 256-token row tiles
+                                       (1024, 1152, 6912, (128, 256))])  # single CTAs, 128-token row tiles
+def test_tc_exactness_bound_mixed_tiles(B, M, N, K, bad):
+    """The tensor-core GEMM keeps one fp32 accumulator per tile when every token of the row tile
+    has 127 sum_k |q| <= 2^24, and folds every 1024 k otherwise.  Here the rows of one tile are all
+    +-1 (every code +-127: sum 127 K, past the bound; acc up to 127^2 K > 2^24, which only the folds
+    keep exact) and the other tiles are small values with one spike per row (sums far below it), so
+    both paths run in one call; every INT32 sum and output is compared bit for bit."""
+    g = np.random.default_rng(M + K)
+    x = (0.05 * g.standard_normal((M, K))).astype(np.float32)
+    x[np.arange(M), g.integers(0, K, M)] = 1.0
+    lo, hi = bad
+    x[lo:hi] = np.where(g.random((hi - lo, K)) < 0.5, -1.0, 1.0)
+    w = np.where(g.random((N, K)) < 0.5, -0.5, 0.5).astype(np.float32)
+    w[0] = np.sign(x[lo]) * 0.5  # acc[lo, 0] = 127^2 K
+    xt, wt = torch.from_numpy(x).to(torch.bfloat16), torch.from_numpy(w).to(torch.bfloat16)
+    x = xt.float().numpy()
+    q = B.prepare_weights(cu(wt), None, 0.5, False, want_f16=True)
+    Y, dbg = B.linear(q, cu(xt), debug=True)
+    r = OW.w8a8_linear(x, OW.prepare_weights(wt.float().numpy(), None, smooth=False), out="bf16")
+    sums = np.abs(r["xq"].astype(np.int64)).sum(axis=1)
+    assert np.all(127 * sums[lo:hi] > 2 ** 24) and np.all(127 * np.delete(sums, np.s_[lo:hi]) <= 2 ** 24)
+    acc = dbg["acc"].cpu().numpy().astype(np.int64)
+    assert acc[lo, 0] == 127 * 127 * K
+    assert np.array_equal(acc, r["acc"])
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+
+
 # ---------------------------------------------------------------------- bf16 pass-through
 def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarray):
     K = X.shape[1]
