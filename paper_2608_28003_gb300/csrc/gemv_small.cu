@@ -556,9 +556,12 @@ __global__ void __launch_bounds__(kThreads, 2)
             mma_f16_16816(c[i], a0, a1, a2, a3, b0, b1);
           }
         };
-        for (int q = warp; q < 32 * cnt; q += 2 * kCW) {
+        // k steps up to K only: the padding past K (to whole 512-byte sub-slices) holds zeros on
+        // both operands, so its steps are skipped (1152 k: 72 of 96 steps)
+        const int nq = min(32 * cnt, (a.K - u0 * 512) / 16);
+        for (int q = warp; q < nq; q += 2 * kCW) {
           step8(q, mc[0]);
-          if (q + kCW < 32 * cnt) step8(q + kCW, mc[1]);
+          if (q + kCW < nq) step8(q + kCW, mc[1]);
         }
         if constexpr (kInt8) {
 #pragma unroll
@@ -595,9 +598,10 @@ __global__ void __launch_bounds__(kThreads, 2)
           }
         }
       };
-      for (int q = warp; q < 16 * cnt; q += 2 * kCW) {  // alternate steps feed the two accumulator sets
+      const int nq = min(16 * cnt, (a.K - u0 * 256) / 16);  // k steps up to K (the padding is zeros)
+      for (int q = warp; q < nq; q += 2 * kCW) {  // alternate steps feed the two accumulator sets
         step(q, mc[0]);
-        if (q + kCW < 16 * cnt) step(q + kCW, mc[1]);
+        if (q + kCW < nq) step(q + kCW, mc[1]);
       }
       }
       __syncwarp();
