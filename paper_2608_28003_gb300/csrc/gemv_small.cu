@@ -88,6 +88,21 @@ __device__ __forceinline__ void ldm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1
                : "r"(addr));
 }
 
+// Sixteen e4m3 codes (byte j of the vector = code j) as fp32 values (exact).
+__device__ __forceinline__ void e4m3x16_to_f32(const uint4& v, float (&x)[16]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t lo = e4m3x2_to_f16x2(w[i]), hi = e4m3x2_to_f16x2(w[i] >> 16);
+    const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&lo));
+    const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&hi));
+    x[4 * i] = a.x;
+    x[4 * i + 1] = a.y;
+    x[4 * i + 2] = b.x;
+    x[4 * i + 3] = b.y;
+  }
+}
+
 __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
   x[0] = bf16_lo(v.x); x[1] = bf16_hi(v.x); x[2] = bf16_lo(v.y); x[3] = bf16_hi(v.y);
   x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
@@ -96,10 +111,10 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
 template <int kW, int MT, int RW>
 __global__ void __launch_bounds__(kThreads, 2)
     gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
-  // kW: weights bf16 (SMALL_BF16), INT8 codes (SMALL_INT8) or e4m3 codes (SMALL_FP8, 8 slots only)
+  // kW: weights bf16 (SMALL_BF16), INT8 codes (SMALL_INT8) or e4m3 codes (SMALL_FP8: fp32 FMAs on the
+  // widened codes at 1-4 token slots, the tensor cores at 8 / 16)
   constexpr bool kInt8 = kW == SMALL_INT8, kFp8 = kW == SMALL_FP8;
   constexpr bool kQ = kInt8 || kFp8;  // one-byte codes, per-token K1, dequantising epilogue
-  static_assert(!kFp8 || MT >= 8, "the e4m3 path runs on the tensor cores (8 or 16 token slots)");
   constexpr float kQmax = kFp8 ? 448.0f : 127.0f;  // largest code magnitude
   constexpr int R = 8 * RW;
   // bf16 at 5-8 tokens: the products run on the tensor cores (mma.sync m16n8k16, the activations
@@ -319,9 +334,9 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
         for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red[i]);
         named_bar_sync(1, kCW * 32);  // s_red is reused by the next slot
-        const float r = mx > 0.0f ? __fdiv_rn(127.0f, mx) : 0.0f;  // fl32(127 / m_t)
+        const float r = mx > 0.0f ? __fdiv_rn(kQmax, mx) : 0.0f;  // fl32(127 / m_t)
         if (tid == 0) {
-          const float sx = __fdiv_rn(mx, 127.0f);  // s_t^x = fl32(m_t / 127)
+          const float sx = __fdiv_rn(mx, kQmax);  // s_t^x = fl32(m_t / 127)
           s_sx[m] = sx;
           if (live && a.s_x_dbg && blockIdx.x == 0) a.s_x_dbg[m] = sx;
         }
@@ -330,7 +345,14 @@ __global__ void __launch_bounds__(kThreads, 2)
           const int vi = tid + v * kCW * 32;
           if (vi < nvec) {
             uint2 packed = make_uint2(0u, 0u);
-            if (live) {
+            if (live && kFp8) {  // e4m3 codes (nearest even, saturating), one byte each
+              uint32_t c[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e)
+                c[e] = e4m3x2_of(__fmul_rn(xh[v][2 * e], r), __fmul_rn(xh[v][2 * e + 1], r));
+              packed = make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
+              if (a.xq_dbg && blockIdx.x == 0) *reinterpret_cast<uint2*>(a.xq_dbg + (size_t)m * a.K + 8 * vi) = packed;
+            } else if (live) {
               int q[8];
 #pragma unroll
               for (int e = 0; e < 8; ++e) q[e] = max(-127, min(127, __float2int_rn(__fmul_rn(xh[v][e], r))));
@@ -630,6 +652,24 @@ __global__ void __launch_bounds__(kThreads, 2)
               acc[u % NA][i][m] = t;
             }
           }
+        } else if constexpr (kFp8) {  // e4m3 codes widened to fp32 (exact products), fp32 FMAs
+          uint4 wv[RW];
+#pragma unroll
+          for (int i = 0; i < RW; ++i) wv[i] = lds128(sub + wlane + (uint32_t)((warp + 8 * i) * 256));
+#pragma unroll
+          for (int m = 0; m < MT; ++m) {
+            float xf[16];
+            e4m3x16_to_f32(lds128(xs + (uint32_t)(m * kpad + (u0 + u) * 512 + 16 * lane)), xf);
+#pragma unroll
+            for (int i = 0; i < RW; ++i) {
+              float wf[16];
+              e4m3x16_to_f32(wv[i], wf);
+              float t = acc[u % NA][i][m];
+#pragma unroll
+              for (int e = 0; e < 16; ++e) t = fmaf(wf[e], xf[e], t);
+              acc[u % NA][i][m] = t;
+            }
+          }
         } else {
           uint4 wv[RW];
 #pragma unroll
@@ -747,6 +787,8 @@ __global__ void __launch_bounds__(kThreads, 2)
       if constexpr (kInt8) {
         y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), __int2float_rn(v));
         if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row] = v;
+      } else if constexpr (kFp8) {
+        y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), v);
       } else {
         y = v;
       }
@@ -801,10 +843,11 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   return W8A8_OK;
 }
 
-// accumulator registers a warp may hold (tokens x rows): larger products spill; the tensor-core paths
-// (8 token slots) hold 8 (+ 2 INT32) per n-tile of 8 rows whatever the token count
+// accumulator registers a warp may hold (tokens x rows): larger products spill (e4m3 fewer: its
+// widened operands take 32 more); the tensor-core paths (8 / 16 token slots) hold 8 (+ 2 or 4
+// INT32) per n-tile of 8 rows whatever the token count
 constexpr bool slots_fit(int kw, int MT, int RW) {
-  return MT >= 8 || (kw != SMALL_FP8 && MT * RW <= (kw == SMALL_INT8 ? 48 : 32));
+  return MT >= 8 || MT * RW <= (kw == SMALL_INT8 ? 48 : kw == SMALL_FP8 ? 12 : 32);
 }
 
 template <int kW, int MT, int RW>
@@ -828,16 +871,12 @@ w8a8_status launch_mt(const SmallArgs& a, cudaStream_t st) {
 
 template <int kW>
 w8a8_status launch_typed(const SmallArgs& a, cudaStream_t st) {
-  if constexpr (kW == SMALL_FP8) {
-    return a.p.MT == 16 ? launch_mt<kW, 16>(a, st) : launch_mt<kW, 8>(a, st);
-  } else {
-    switch (a.p.MT) {
-      case 1: return launch_mt<kW, 1>(a, st);
-      case 2: return launch_mt<kW, 2>(a, st);
-      case 4: return launch_mt<kW, 4>(a, st);
-      case 8: return launch_mt<kW, 8>(a, st);
-      default: return launch_mt<kW, 16>(a, st);
-    }
+  switch (a.p.MT) {
+    case 1: return launch_mt<kW, 1>(a, st);
+    case 2: return launch_mt<kW, 2>(a, st);
+    case 4: return launch_mt<kW, 4>(a, st);
+    case 8: return launch_mt<kW, 8>(a, st);
+    default: return launch_mt<kW, 16>(a, st);
   }
 }
 
@@ -851,7 +890,9 @@ SmallPlan make_small_plan(int wkind, int M, int N, int K, int kind, int sm_count
   if (M > 8 && fused_norm) return p;  // the decoder fuses its residual step at 1-8 tokens only
   if (kind != EPI_BF16 && kind != EPI_GEGLU) return p;
   if (kind == EPI_GEGLU && N % 16 != 0) return p;
-  p.MT = M > 8 ? 16 : wkind == SMALL_FP8 ? 8 : M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
+  // e4m3: fp32 FMAs on the widened codes at 1-2 tokens (one token: 22 us per FFN block against 35 on
+  // the tensor cores); from 3 tokens the 8-slot tensor-core path (4 tokens x 6 rows of FMAs spill)
+  p.MT = M > 8 ? 16 : (wkind == SMALL_FP8 && M > 2) ? 8 : M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
   if (int8_weights && p.MT <= 4 && K > kMaxInt8K) return p;
   // fewest rows per CTA (more CTAs) that still fit in two CTAs per SM
   static const int kRw[] = {1, 2, 4, 6};

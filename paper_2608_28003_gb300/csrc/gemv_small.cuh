@@ -7,8 +7,8 @@
 
 namespace w8a8 {
 
-// Weight kinds: bf16, INT8 codes (W8A8), e4m3 codes (the FP8 variant; always 8 token slots on the
-// tensor cores).
+// Weight kinds: bf16, INT8 codes (W8A8), e4m3 codes (the FP8 variant: codes widened to fp32 for
+// FMAs at 1-4 token slots, to fp16 for the tensor cores at 8 / 16).
 enum { SMALL_BF16 = 0, SMALL_INT8 = 1, SMALL_FP8 = 2 };
 
 struct SmallPlan {
