@@ -66,19 +66,6 @@ __device__ __forceinline__ uint32_t f16x2_of(float lo, float hi) {
   asm("cvt.rn.f16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
 }
-// Four signed INT8 codes (bytes 0..3 of w) as two fp16 pairs (bytes 0, 1) and (2, 3), exactly:
-// byte b + 128 is placed under the exponent bits 0x64 (the half 1024 + b + 128), then 1152 is
-// subtracted.
-__device__ __forceinline__ void i8x4_to_f16x2x2(uint32_t w, uint32_t& lo, uint32_t& hi) {
-  const uint32_t u = w ^ 0x80808080u;
-  uint32_t p0, p1;
-  asm("prmt.b32 %0, %1, %2, 0x4140;\n" : "=r"(p0) : "r"(u), "r"(0x64646464u));
-  asm("prmt.b32 %0, %1, %2, 0x4342;\n" : "=r"(p1) : "r"(u), "r"(0x64646464u));
-  const uint32_t k1152 = 0x64806480u;  // (1152, 1152) as fp16
-  asm("sub.rn.f16x2 %0, %1, %2;\n" : "=r"(lo) : "r"(p0), "r"(k1152));
-  asm("sub.rn.f16x2 %0, %1, %2;\n" : "=r"(hi) : "r"(p1), "r"(k1152));
-}
-
 __device__ __forceinline__ void ldm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];\n" : "=r"(r0), "=r"(r1) : "r"(addr));
 }

@@ -44,7 +44,7 @@ def ffn(B):
     return c, f, prep
 
 
-@pytest.mark.parametrize("M", [1, 3, 5, 8, 9, 13, 16, 64])
+@pytest.mark.parametrize("M", [1, 3, 5, 8, 9, 13, 16, 24, 32, 64])
 def test_ffn_w8a8_bit_exact(B, ffn, M):
     c, f, prep = ffn
     x = c["x"][:M]

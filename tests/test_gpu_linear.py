@@ -249,6 +249,48 @@ def test_tc_exactness_bound_mixed_tiles(B, M, N, K, bad):
     assert np.array_equal(f32_of_bf16(Y), r["y"])
 
 
+WIDE_FEW_SHAPES = [
+    (7, 8208, 1040),     # ragged N (8208 = 64 x 128 + 16) and K (an odd number of 64-k steps)
+    (20, 8192, 1152),    # with a bias
+    (32, 13824, 1152),   # the gate/up shape at a decode batch of 32
+]
+
+
+@pytest.mark.parametrize("M,N,K", WIDE_FEW_SHAPES)
+def test_w8a8_wide_output_few_tokens_bit_exact(B, M, N, K):
+    """5-32 tokens on wide outputs with the INT8 codes only (no fp16 copy): the streaming kernel;
+    codes, scales, INT32 sums and outputs bit for bit."""
+    x32, x, w32, w, c32, c = _case(M, N, K, seed=M * 11 + N)
+    stat = OW.act_absmax(np.concatenate([c32, x32]))
+    q = B.prepare_weights(cu(w), cu(torch.from_numpy(stat)))  # INT8 codes only: no fp16 copy
+    bias = np.random.default_rng(3).standard_normal(N).astype(np.float32) if M == 20 else None
+    Y, dbg = B.linear(q, cu(x), bias=cu(torch.from_numpy(bias)) if bias is not None else None, debug=True)
+    r = OW.w8a8_linear(x32, OW.prepare_weights(w32, stat), bias=bias, out="bf16")
+    assert np.array_equal(dbg["xq"].cpu().numpy(), r["xq"])
+    assert np.array_equal(dbg["s_x"].cpu().numpy(), r["s_x"])
+    assert np.array_equal(dbg["acc"].cpu().numpy().astype(np.int64), r["acc"])
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+
+
+def test_w8a8_wide_output_few_tokens_at_extremes(B):
+    """Rows of +-1 (every code +-127) at 12 tokens on a wide output, K = 2048: acc[0, 0] = 127^2 K
+    exceeds 2^24, so the fp32 MMA sums of the streaming kernel must be folded into INT32 to come
+    out exact."""
+    M, N, K = 12, 8192, 2048
+    g = np.random.default_rng(5)
+    x = np.where(g.random((M, K)) < 0.5, -1.0, 1.0).astype(np.float32)
+    w = np.where(g.random((N, K)) < 0.5, -0.5, 0.5).astype(np.float32)
+    w[0] = np.sign(x[0]) * 0.5
+    xt, wt = torch.from_numpy(x).to(torch.bfloat16), torch.from_numpy(w).to(torch.bfloat16)
+    q = B.prepare_weights(cu(wt), None, 0.5, False)
+    Y, dbg = B.linear(q, cu(xt), debug=True)
+    r = OW.w8a8_linear(xt.float().numpy(), OW.prepare_weights(wt.float().numpy(), None, smooth=False), out="bf16")
+    acc = dbg["acc"].cpu().numpy().astype(np.int64)
+    assert acc[0, 0] == 127 * 127 * K > 2 ** 24
+    assert np.array_equal(acc, r["acc"])
+    assert np.array_equal(f32_of_bf16(Y), r["y"])
+
+
 # ---------------------------------------------------------------------- bf16 pass-through
 def _bf16_close(y_gpu: np.ndarray, X: np.ndarray, W: np.ndarray, y_ref: np.ndarray):
     K = X.shape[1]
