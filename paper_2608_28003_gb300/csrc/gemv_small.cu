@@ -35,8 +35,7 @@ namespace w8a8 {
 
 namespace {
 
-constexpr int kCW = 8;  // consumer warps
-constexpr int kThreads = (kCW + 1) * 32;
+constexpr int kCW = 8;  // consumer warps (16 on the tensor-core paths when the grid has one CTA per SM)
 constexpr int kSmemLimit = 227 * 1024;
 constexpr int kStatic = 2048;       // static shared memory of the kernel (reduction slots, scales) + slack
 constexpr int kSliceBytes = 512;    // bytes of one weight row per sub-slice
@@ -48,13 +47,13 @@ __device__ __forceinline__ float warp_sum32(float v) {
   return v;
 }
 
-// Sum over the 256 consumer threads in the residual-norm kernel's order (lane tree, then warps
-// 0..7 in turn); every consumer thread gets the result.
+// Sum over the first 256 consumer threads in the residual-norm kernel's order (lane tree, then
+// warps 0..7 in turn); each of them gets the result (barrier 2: those 256 threads only).
 __device__ __forceinline__ float consumer_sum(float v, float* red, int warp, int lane) {
   v = warp_sum32(v);
-  named_bar_sync(1, 256);
+  named_bar_sync(2, 256);
   if (lane == 0) red[warp] = v;
-  named_bar_sync(1, 256);
+  named_bar_sync(2, 256);
   float t = 0.0f;
 #pragma unroll
   for (int i = 0; i < 8; ++i) t += red[i];
@@ -95,8 +94,8 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&x)[8]) {
   x[4] = bf16_lo(v.z); x[5] = bf16_hi(v.z); x[6] = bf16_lo(v.w); x[7] = bf16_hi(v.w);
 }
 
-template <int kW, int MT, int RW>
-__global__ void __launch_bounds__(kThreads, 2)
+template <int kW, int MT, int RW, int CW>
+__global__ void __launch_bounds__((CW + 1) * 32, CW == 8 ? 2 : 1)
     gemv_small_kernel(const __grid_constant__ CUtensorMap tmW, const SmallArgs a) {
   // kW: weights bf16 (SMALL_BF16), INT8 codes (SMALL_INT8) or e4m3 codes (SMALL_FP8: fp32 FMAs on the
   // widened codes at 1-4 token slots, the tensor cores at 8 / 16)
@@ -119,8 +118,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   // accumulation (no fold).
   using Acc = typename std::conditional<kInt8, int, float>::type;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ float s_red[kCW];
-  __shared__ float s_red8[MT > 4 ? MT : 1][kCW];  // 8 / 16-slot K1: per-token maxima of the warps
+  __shared__ float s_red[CW];
+  __shared__ float s_red8[MT > 4 ? MT : 1][CW];  // 8 / 16-slot K1: per-token maxima of the warps
   __shared__ float s_sx[MT];
   __shared__ unsigned int s_hmax[MT];  // GeGLU epilogue: per-token max |h * 1/delta| of this CTA (float bits)
 
@@ -134,22 +133,28 @@ __global__ void __launch_bounds__(kThreads, 2)
   uint64_t* empty = full + S;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row0 = blockIdx.x * R;
+  if constexpr (CW != kCW) {  // the fused residual norm runs on 8 consumer warps only (not planned)
+    if (a.has_rn) {
+      if (threadIdx.x == 0) atomicOr(a.err, DEVERR_CONSUMER_WAIT);
+      return;
+    }
+  }
 
   pdl_trigger();
-  if (threadIdx.x == kCW * 32) {  // the producer thread: fetch the tensor map before the first copy needs it
+  if (threadIdx.x == CW * 32) {  // the producer thread: fetch the tensor map before the first copy needs it
     prefetch_tmap(&tmW);
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_u32(full + s), 1);
-      mbar_init(smem_u32(empty + s), kCW);
+      mbar_init(smem_u32(empty + s), CW);
     }
     fence_mbar_init();
   }
   __syncthreads();
 
   // ------------------------------------------------------------------------ producer thread
-  if (warp == kCW) {
+  if (warp == CW) {
     if (lane != 0) return;
     bool ok = true;
     int it = 0, s = 0;
@@ -209,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const float4* idl = reinterpret_cast<const float4*>(a.inv_delta);
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
-      const int vi = tid + v * kCW * 32;
+      const int vi = tid + v * CW * 32;
       if (vi < (a.K >> 3)) {
         idr[v][0] = idl[2 * vi];
         idr[v][1] = idl[2 * vi + 1];
@@ -279,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         *reinterpret_cast<uint4*>(as + (size_t)m * (kQ ? kpad : xsb) + 8 * tid) = w;
       }
     }
-    named_bar_sync(1, kCW * 32);
+    named_bar_sync(1, CW * 32);
     xrows = as;
     xstride = kpad;
   }
@@ -297,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 2)
           const uint4* src = reinterpret_cast<const uint4*>(xrows + (size_t)m * xstride);
 #pragma unroll
           for (int v = 0; v < 4; ++v) {
-            const int vi = tid + v * kCW * 32;
+            const int vi = tid + v * CW * 32;
             if (vi < nvec) {
               const uint4 w = src[vi];
               const float4 d0 = idr[v][0], d1 = idr[v][1];
@@ -316,11 +321,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         amax = warp_max(amax);
         if (lane == 0) s_red[warp] = amax;
-        named_bar_sync(1, kCW * 32);
+        named_bar_sync(1, CW * 32);
         float mx = 0.0f;
 #pragma unroll
-        for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red[i]);
-        named_bar_sync(1, kCW * 32);  // s_red is reused by the next slot
+        for (int i = 0; i < CW; ++i) mx = fmaxf(mx, s_red[i]);
+        named_bar_sync(1, CW * 32);  // s_red is reused by the next slot
         const float r = mx > 0.0f ? __fdiv_rn(kQmax, mx) : 0.0f;  // fl32(127 / m_t)
         if (tid == 0) {
           const float sx = __fdiv_rn(mx, kQmax);  // s_t^x = fl32(m_t / 127)
@@ -329,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
-          const int vi = tid + v * kCW * 32;
+          const int vi = tid + v * CW * 32;
           if (vi < nvec) {
             uint2 packed = make_uint2(0u, 0u);
             if (live && kFp8) {  // e4m3 codes (nearest even, saturating), one byte each
@@ -378,11 +383,11 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
       for (int m = 0; m < MT; ++m) am[m] = 0.0f;
       if (a.rowmax_in) {  // the producer's partial maxima stand for pass 1 (the same fp32 products)
-        for (int i = tid; i < a.rowmax_n; i += kCW * 32)
+        for (int i = tid; i < a.rowmax_n; i += CW * 32)
 #pragma unroll
           for (int m = 0; m < MT; ++m) am[m] = fmaxf(am[m], a.rowmax_in[(size_t)i * MT + m]);
       }
-      for (int vi = a.rowmax_in ? nvec : tid; vi < nvec; vi += kCW * 32) {
+      for (int vi = a.rowmax_in ? nvec : tid; vi < nvec; vi += CW * 32) {
         const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
 #pragma unroll
         for (int m0 = 0; m0 < MT; m0 += 8) {
@@ -402,13 +407,13 @@ __global__ void __launch_bounds__(kThreads, 2)
         const float v = warp_max(am[m]);
         if (lane == 0) s_red8[m][warp] = v;
       }
-      named_bar_sync(1, kCW * 32);
+      named_bar_sync(1, CW * 32);
       float rr[MT];
 #pragma unroll
       for (int m = 0; m < MT; ++m) {
         float mx = 0.0f;
 #pragma unroll
-        for (int i = 0; i < kCW; ++i) mx = fmaxf(mx, s_red8[m][i]);
+        for (int i = 0; i < CW; ++i) mx = fmaxf(mx, s_red8[m][i]);
         rr[m] = mx > 0.0f ? __fdiv_rn(kQmax, mx) : 0.0f;  // fl32(127 / m_t)
         if (tid == m) {
           const float sx = __fdiv_rn(mx, kQmax);  // s_t^x = fl32(m_t / 127); 0 for slots >= M
@@ -417,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
       }
       // pass 2: the rows again (L1), quantised; codes of slots >= M are zeros
-      for (int vi = tid; vi < nvec; vi += kCW * 32) {
+      for (int vi = tid; vi < nvec; vi += CW * 32) {
         const float4 d0 = idl[2 * vi], d1 = idl[2 * vi + 1];
 #pragma unroll
         for (int m0 = 0; m0 < MT; m0 += 8) {
@@ -464,13 +469,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     if constexpr (kMma) {  // fp16 codes: zeros from K to the padded length
       const int t8 = (kpad - a.K) >> 3;
-      for (int i = tid; i < MT * t8; i += kCW * 32) {
+      for (int i = tid; i < MT * t8; i += CW * 32) {
         const int m = i / t8, c = i - m * t8;
         *reinterpret_cast<uint4*>(xsp + ((size_t)m * xsb + a.K + 8 * c) * 2) = make_uint4(0u, 0u, 0u, 0u);
       }
     } else {  // INT8 codes: zeros from K to the padded length
       const int tail16 = (kpad - a.K) >> 4;
-      for (int i = tid; i < MT * tail16; i += kCW * 32) {
+      for (int i = tid; i < MT * tail16; i += CW * 32) {
         const int m = i / tail16, c = i - m * tail16;
         *reinterpret_cast<uint4*>(xsp + (size_t)m * kpad + a.K + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
       }
@@ -478,24 +483,24 @@ __global__ void __launch_bounds__(kThreads, 2)
   } else if (!a.has_rn) {
     const int vpr = kpad >> 3;  // 16-byte vectors per slot
     const int total = MT * vpr;
-    for (int i0 = tid; i0 < total; i0 += 4 * kCW * 32) {  // four loads in flight per thread
+    for (int i0 = tid; i0 < total; i0 += 4 * CW * 32) {  // four loads in flight per thread
       uint4 val[4];
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const int i = i0 + u * kCW * 32;
+        const int i = i0 + u * CW * 32;
         const int m = i / vpr, v = i - m * vpr;
         val[u] = make_uint4(0u, 0u, 0u, 0u);
         if (i < total && m < a.M && 8 * v < a.K) val[u] = reinterpret_cast<const uint4*>(a.X + (size_t)m * a.K)[v];
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const int i = i0 + u * kCW * 32;
+        const int i = i0 + u * CW * 32;
         const int m = i / vpr, v = i - m * vpr;
         if (i < total) *reinterpret_cast<uint4*>(xsp + ((size_t)m * xsb + 8 * v) * 2) = val[u];
       }
     }
   }
-  named_bar_sync(1, kCW * 32);
+  named_bar_sync(1, CW * 32);
 
   // NA independent accumulators per (row, token) keep the FMA / dp4a chains short when a warp has
   // few rows and tokens; sub-slice u of every stage feeds accumulator u mod NA.
@@ -568,9 +573,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         // k steps up to K only: the padding past K (to whole 512-byte sub-slices) holds zeros on
         // both operands, so its steps are skipped (1152 k: 72 of 96 steps)
         const int nq = min(32 * cnt, (a.K - u0 * 512) / 16);
-        for (int q = warp; q < nq; q += 2 * kCW) {
+        for (int q = warp; q < nq; q += 2 * CW) {
           step8(q, mc[0]);
-          if (q + kCW < nq) step8(q + kCW, mc[1]);
+          if (q + CW < nq) step8(q + CW, mc[1]);
         }
         if constexpr (kInt8) {
 #pragma unroll
@@ -608,9 +613,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
       };
       const int nq = min(16 * cnt, (a.K - u0 * 256) / 16);  // k steps up to K (the padding is zeros)
-      for (int q = warp; q < nq; q += 2 * kCW) {  // alternate steps feed the two accumulator sets
+      for (int q = warp; q < nq; q += 2 * CW) {  // alternate steps feed the two accumulator sets
         step(q, mc[0]);
-        if (q + kCW < nq) step(q + kCW, mc[1]);
+        if (q + CW < nq) step(q + CW, mc[1]);
       }
       }
       __syncwarp();
@@ -707,11 +712,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
       }
     }
-    if (!named_bar_all(1, kCW * 32, ok)) return;
+    if (!named_bar_all(1, CW * 32, ok)) return;
     auto total = [&](int r, int m) {
       Acc v = 0;
 #pragma unroll
-      for (int w = 0; w < kCW; ++w) v += part[(w * R + r) * MT + m];
+      for (int w = 0; w < CW; ++w) v += part[(w * R + r) * MT + m];
       float y;
       if constexpr (kInt8) {
         y = __fmul_rn(__fmul_rn(s_sx[m], a.s_w[row0 + r]), __int2float_rn(v));
@@ -725,8 +730,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     };
     if (a.kind == EPI_GEGLU) {  // pair b of block j: gate row 16 j + b, up row 16 j + 8 + b
       if (a.rowmax_out && tid < MT) s_hmax[tid] = 0u;
-      if (a.rowmax_out) named_bar_sync(1, kCW * 32);
-      for (int e = tid; e < (R / 2) * MT; e += kCW * 32) {
+      if (a.rowmax_out) named_bar_sync(1, CW * 32);
+      for (int e = tid; e < (R / 2) * MT; e += CW * 32) {
         const int pr = e / MT, m = e % MT, j = pr >> 3, b = pr & 7;
         const int gr = 16 * j + b;
         if (m >= a.M || row0 + gr + 8 >= a.N) continue;
@@ -739,11 +744,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
       }
       if (a.rowmax_out) {
-        named_bar_sync(1, kCW * 32);
+        named_bar_sync(1, CW * 32);
         if (tid < MT) a.rowmax_out[(size_t)blockIdx.x * MT + tid] = __uint_as_float(s_hmax[tid]);
       }
     } else {
-      for (int e = tid; e < R * MT; e += kCW * 32) {
+      for (int e = tid; e < R * MT; e += CW * 32) {
         const int r = e / MT, m = e % MT;
         if (m >= a.M || row0 + r >= a.N) continue;
         a.y[(size_t)m * a.N + row0 + r] = f32_to_bf16_bits(total(r, m));
@@ -809,13 +814,13 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 }
 
-template <int kW, int MT, int RW>
+template <int kW, int MT, int RW, int CW>
 w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
   static bool attr_set[64] = {};
   int dev = 0;
   W8A8_CUDA(cudaGetDevice(&dev));
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    W8A8_CUDA(cudaFuncSetAttribute(gemv_small_kernel<kW, MT, RW, CW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    kSmemLimit - kStatic));
     attr_set[dev] = true;
   }
@@ -825,8 +830,8 @@ w8a8_status launch_t(const SmallArgs& a, cudaStream_t st) {
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 128 / EB, 8 * RW, 128));
   else
     W8A8_TRY(make_tmap_2d(&tw, a.W, EB, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K * EB, 256, 8 * RW, 0));
-  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW>, dim3(a.p.P), dim3(kThreads), (size_t)a.p.smem_bytes, st, tw,
-                       a));
+  W8A8_CUDA(launch_pdl(gemv_small_kernel<kW, MT, RW, CW>, dim3(a.p.P), dim3((CW + 1) * 32), (size_t)a.p.smem_bytes, st,
+                       tw, a));
   return W8A8_OK;
 }
 
@@ -840,7 +845,10 @@ constexpr bool slots_fit(int kw, int MT, int RW) {
 template <int kW, int MT, int RW>
 w8a8_status launch_checked(const SmallArgs& a, cudaStream_t st) {
   if constexpr (slots_fit(kW, MT, RW)) {
-    return launch_t<kW, MT, RW>(a, st);
+    if constexpr (MT >= 8 && RW == 1) {
+      if (a.p.cw == 16) return launch_t<kW, MT, RW, 16>(a, st);
+    }
+    return launch_t<kW, MT, RW, kCW>(a, st);
   } else {
     W8A8_CHECK_ARG(false, W8A8_ERR_SHAPE, "small GEMV: %d tokens x %d rows per warp not built", MT, RW);
   }
@@ -901,7 +909,11 @@ SmallPlan make_small_plan(int wkind, int M, int N, int K, int kind, int sm_count
   const bool mma = p.MT >= 8;  // the kernel's tensor-core paths (same rule): padded bf16 / fp16 rows
   p.xbytes = mma ? p.MT * (p.kpad + (int8_weights ? 16 : 8)) * 2 : p.MT * p.kpad * (int8_weights ? 1 : 2);
   p.abytes = fused_norm && int8_weights ? p.MT * p.kpad * 2 : 0;
-  p.rbytes = mma ? kCW * R * p.MT * 4 : 0;  // the warps' partial sums
+  // 16 consumer warps where a tensor-core grid has one CTA per SM (one row block per warp group
+  // of 8 rows: the down and o projections at 5-16 tokens): twice the warps to hide the MMA and
+  // widening latencies of a CTA that has the SM to itself
+  p.cw = mma && p.RW == 1 && p.P <= sm_count && !fused_norm ? 16 : kCW;
+  p.rbytes = mma ? p.cw * R * p.MT * 4 : 0;  // the warps' partial sums
   const int budget = kSmemLimit / cps - kStatic - 1024 - p.xbytes - p.abytes - p.rbytes - 16 * 16;
   // sub-slices per stage: 4 for warps with one or two rows, fewer for wider CTAs; each stage must
   // fit twice in the ring unless one stage covers everything

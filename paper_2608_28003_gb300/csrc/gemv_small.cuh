@@ -27,6 +27,7 @@ struct SmallPlan {
   int abytes;       // W8A8 with a fused residual norm: the bf16 rows it produces, before K1
   int rbytes;       // 5-8 tokens (tensor-core paths): the consumer warps' partial sums
   int smem_bytes;
+  int cw;           // consumer warps: 8, or 16 on the tensor-core paths when the grid has one CTA per SM
 };
 
 // The decoder's residual step in front of a decode linear, fused into the GEMV's prologue:
