@@ -70,6 +70,104 @@ __device__ __forceinline__ void st_cluster_f32x4(uint32_t addr, float a, float b
   asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
                : "memory");
 }
+// One query head per CTA (the cluster's head), thread t owning output dim t (256 threads, head dim
+// 256).  Per key tile: half-warp h scores keys h, h + 16, ... (lane i of the half holds dims of
+// chunks i and i + 16 of the key row and of the query, kept in registers; four shuffles sum the
+// half); every warp then takes the tile's max and its weights p_j = e^(s_j - m) (lane i: keys i and
+// i + 32) into its own shared-memory row, and thread t adds sum_j p_j v_jt to its running output.
+// The CTA's (m, l, o) partial goes to CTA 0's inbox (one distributed shared memory store per dim),
+// and after one cluster barrier CTA 0 combines the partials, thread t its dim.
+template <typename Stage>
+__device__ __forceinline__ void head_keys_one(uint8_t* sm, uint32_t sbase, Stage& stage, int kb, int ke, int ntiles,
+                                              int pos, int r, int b, int hq0, const AttnShape& s,
+                                              uint16_t* __restrict__ o) {
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int half = t >> 4, l16 = lane & 15;
+  const float* qs = reinterpret_cast<const float*>(sm + kOffQ);
+  float4 q[4];  // dims 8 l16 .. 8 l16 + 7 and 128 + 8 l16 .. 128 + 8 l16 + 7
+  q[0] = reinterpret_cast<const float4*>(qs + 8 * l16)[0];
+  q[1] = reinterpret_cast<const float4*>(qs + 8 * l16)[1];
+  q[2] = reinterpret_cast<const float4*>(qs + kHd / 2 + 8 * l16)[0];
+  q[3] = reinterpret_cast<const float4*>(qs + kHd / 2 + 8 * l16)[1];
+  float* sc = reinterpret_cast<float*>(sm + kOffPart);   // [kTile] scores of the tile
+  float* pw = sc + kTile + warp * kTile;                 // this warp's weights of the tile
+  float m = -INFINITY, l = 0.0f, acc = 0.0f;
+  for (int ti = 0; ti < ntiles; ++ti) {
+    cp_async_wait<0>();
+    __syncthreads();
+    const int j0 = kb + ti * kTile, nt = min(kTile, ke - j0);
+    const uint8_t* kt = sm + kOffBuf;
+    const uint8_t* vt = kt + kTile * kKRow;
+    for (int jb = 0; jb < nt; jb += 2 * kWarps) {  // warp-uniform trip count: the shuffles below take every lane
+      const int j = jb + half;
+      const bool live = j < nt;
+      const uint8_t* kr = j0 + j == pos ? sm + kOffKNew : kt + (live ? j : 0) * kKRow;
+      const uint4 ka = reinterpret_cast<const uint4*>(kr)[l16];
+      const uint4 kc = reinterpret_cast<const uint4*>(kr)[l16 + 16];
+      float x[8], d0 = 0.0f, d1 = 0.0f;
+      unpack8_bf16(ka, x);
+      d0 = fmaf(q[0].x, x[0], d0); d0 = fmaf(q[0].y, x[1], d0); d0 = fmaf(q[0].z, x[2], d0); d0 = fmaf(q[0].w, x[3], d0);
+      d0 = fmaf(q[1].x, x[4], d0); d0 = fmaf(q[1].y, x[5], d0); d0 = fmaf(q[1].z, x[6], d0); d0 = fmaf(q[1].w, x[7], d0);
+      unpack8_bf16(kc, x);
+      d1 = fmaf(q[2].x, x[0], d1); d1 = fmaf(q[2].y, x[1], d1); d1 = fmaf(q[2].z, x[2], d1); d1 = fmaf(q[2].w, x[3], d1);
+      d1 = fmaf(q[3].x, x[4], d1); d1 = fmaf(q[3].y, x[5], d1); d1 = fmaf(q[3].z, x[6], d1); d1 = fmaf(q[3].w, x[7], d1);
+      float dsum = d0 + d1;
+#pragma unroll
+      for (int of = 8; of > 0; of >>= 1) dsum += __shfl_xor_sync(0xffffffffu, dsum, of);  // within the half
+      if (live && l16 == 0) sc[j] = dsum;
+    }
+    __syncthreads();
+    const float s0 = lane < nt ? sc[lane] : -INFINITY, s1 = lane + 32 < nt ? sc[lane + 32] : -INFINITY;
+    const float m_new = fmaxf(m, warp_max_f(fmaxf(s0, s1)));
+    const float corr = expf(m - m_new);  // 0 on the first tile (m = -inf)
+    const float p0 = lane < nt ? expf(s0 - m_new) : 0.0f, p1 = lane + 32 < nt ? expf(s1 - m_new) : 0.0f;
+    pw[lane] = p0;
+    pw[lane + 32] = p1;
+    l = l * corr + warp_sum_f(p0 + p1);
+    m = m_new;
+    __syncwarp();
+    float a4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    int j = 0;
+    for (; j + 4 <= nt; j += 4) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint8_t* vr = j0 + j + u == pos ? sm + kOffVNew : vt + (j + u) * kVRow;
+        a4[u] = fmaf(pw[j + u], bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(vr)[t]), a4[u]);
+      }
+    }
+    for (; j < nt; ++j) {
+      const uint8_t* vr = j0 + j == pos ? sm + kOffVNew : vt + j * kVRow;
+      a4[0] = fmaf(pw[j], bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(vr)[t]), a4[0]);
+    }
+    acc = fmaf(acc, corr, (a4[0] + a4[1]) + (a4[2] + a4[3]));
+    __syncthreads();  // the buffer, the scores and the weights are reused by the next tile
+    if (ti + 1 < ntiles) stage(ti + 1);
+  }
+  const uint32_t dst = map_to_rank(sbase + kOffInbox + (uint32_t)(r * kMaxG * kPartFloats * 4), 0);
+  st_cluster_f32(dst + 4 * t, acc);
+  if (t == 0) {
+    st_cluster_f32(dst + kHd * 4, m);
+    st_cluster_f32(dst + (kHd + 1) * 4, l);
+  }
+  cluster_sync_all();  // release the pushes / acquire them in CTA 0
+  if (r != 0) return;
+  const float* in = reinterpret_cast<const float*>(sm + kOffInbox);
+  float mr[kSplits], M = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kSplits; ++i) {
+    mr[i] = in[i * kMaxG * kPartFloats + kHd];
+    M = fmaxf(M, mr[i]);
+  }
+  float L = 0.0f, y = 0.0f;
+#pragma unroll
+  for (int i = 0; i < kSplits; ++i) {
+    const float f = mr[i] == -INFINITY ? 0.0f : expf(mr[i] - M);
+    L = fmaf(in[i * kMaxG * kPartFloats + kHd + 1], f, L);
+    y = fmaf(in[i * kMaxG * kPartFloats + t], f, y);
+  }
+  o[(size_t)b * (s.n_q * kHd) + (size_t)hq0 * kHd + t] = f32_to_bf16_bits(y / L);
+}
+
 __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     attn_decode_kernel(const uint16_t* __restrict__ qkv, AttnShape s, const int* __restrict__ pos0,
                        const float* __restrict__ qn, const float* __restrict__ kn, float eps,
@@ -167,6 +265,11 @@ __global__ void __cluster_dims__(kSplits, 1, 1) __launch_bounds__(kWarps * 32)
     }
   }
   __syncthreads();
+
+  if (hpc == 1) {  // one head per cluster: see head_keys_one
+    head_keys_one(sm, sbase, stage, kb, ke, ntiles, pos, r, b, hq0, s, o);
+    return;
+  }
 
   // ---- this warp's keys of every tile
   const float* qs = reinterpret_cast<const float*>(sm + kOffQ) + hw * kHd;
