@@ -772,45 +772,64 @@ __global__ void __launch_bounds__((CW + 1) * 32, CW == 8 ? 2 : 1)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) acc[0][i][m] += __shfl_xor_sync(0xffffffffu, acc[0][i][m], o);
     }
-  if (lane != 0) return;
-  {  // the epilogue (lane 0)
-    auto value = [&](Acc v, int i, int row, int m) -> float {  // i: the warp's row slot of `row`
-      float y;
-      if constexpr (kInt8) {
-        y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), __int2float_rn(v));
-        if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row] = v;
-      } else if constexpr (kFp8) {
-        y = __fmul_rn(__fmul_rn(s_sx[m], swr[i]), v);
-      } else {
-        y = v;
-      }
-      return a.bias ? __fadd_rn(y, bir[i]) : y;
-    };
-    if (a.kind == EPI_GEGLU) {
-#pragma unroll
-      for (int j = 0; j < RW / 2; ++j) {
-        const int gi = row0 + 16 * j + warp, ui = gi + 8;
-        if (ui >= a.N) continue;
-        const int hid = ((row0 + 16 * j) >> 1) + warp;
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-          if (m >= a.M) break;
-          const float g = value(acc[0][2 * j][m], 2 * j, gi, m), u = value(acc[0][2 * j + 1][m], 2 * j + 1, ui, m);
-          a.y[(size_t)m * (a.N >> 1) + hid] = f32_to_bf16_bits(geglu_recipe(g, u));
-        }
-      }
+  // The epilogue: lane e of the warp writes the warp's output e (every lane holds every sum), so
+  // the outputs' arithmetic (dequantisation, GeGLU) runs side by side on the lanes instead of in
+  // turn on one lane.  Lane e picks its sums, scales and bias by selects, not by indexing.
+  auto value = [&](Acc v, float sw, float bi, int row, int m) -> float {
+    float y;
+    if constexpr (kInt8) {
+      y = __fmul_rn(__fmul_rn(s_sx[m], sw), __int2float_rn(v));
+      if (a.acc_dbg) a.acc_dbg[(size_t)m * a.N + row] = v;
+    } else if constexpr (kFp8) {
+      y = __fmul_rn(__fmul_rn(s_sx[m], sw), v);
     } else {
-#pragma unroll
-      for (int i = 0; i < RW; ++i) {
-        const int row = row0 + warp + 8 * i;
-        if (row >= a.N) continue;
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-          if (m >= a.M) break;
-          a.y[(size_t)m * a.N + row] = f32_to_bf16_bits(value(acc[0][i][m], i, row, m));
-        }
-      }
+      y = v;
     }
+    return a.bias ? __fadd_rn(y, bi) : y;
+  };
+  if (a.kind == EPI_GEGLU) {  // output e = (pair j, token m): gate row slot 2 j, up row slot 2 j + 1
+    if (lane >= (RW / 2) * MT) return;
+    const int j = lane / MT, m = lane - j * MT;
+    Acc ga = 0, ua = 0;
+    float sg = 0.0f, su = 0.0f, bg = 0.0f, bu = 0.0f;
+#pragma unroll
+    for (int jj = 0; jj < RW / 2; ++jj) {
+      if (jj == j) {
+        sg = swr[2 * jj];
+        su = swr[2 * jj + 1];
+        bg = bir[2 * jj];
+        bu = bir[2 * jj + 1];
+      }
+#pragma unroll
+      for (int mm = 0; mm < MT; ++mm)
+        if (jj == j && mm == m) {
+          ga = acc[0][2 * jj][mm];
+          ua = acc[0][2 * jj + 1][mm];
+        }
+    }
+    const int gi = row0 + 16 * j + warp, ui = gi + 8;
+    if (ui >= a.N || m >= a.M) return;
+    const int hid = ((row0 + 16 * j) >> 1) + warp;
+    const float g = value(ga, sg, bg, gi, m), u = value(ua, su, bu, ui, m);
+    a.y[(size_t)m * (a.N >> 1) + hid] = f32_to_bf16_bits(geglu_recipe(g, u));
+  } else {  // output e = (row slot i, token m)
+    if (lane >= RW * MT) return;
+    const int i = lane / MT, m = lane - i * MT;
+    Acc av = 0;
+    float sw = 0.0f, bi = 0.0f;
+#pragma unroll
+    for (int ii = 0; ii < RW; ++ii) {
+      if (ii == i) {
+        sw = swr[ii];
+        bi = bir[ii];
+      }
+#pragma unroll
+      for (int mm = 0; mm < MT; ++mm)
+        if (ii == i && mm == m) av = acc[0][ii][mm];
+    }
+    const int row = row0 + warp + 8 * i;
+    if (row >= a.N || m >= a.M) return;
+    a.y[(size_t)m * a.N + row] = f32_to_bf16_bits(value(av, sw, bi, row, m));
   }
 }
 
