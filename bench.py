@@ -49,7 +49,7 @@ HIDDEN, INTER, VOCAB, LAYERS = 1152, 6912, 262144, 26
 PREFILL = 128
 # DRAM bytes read + written per launch of the decode GEMV, averaged over the roofline mix's launches
 # (ncu over one decode step of `--profile-workload decode4`, the same shapes)
-GEMV_MIX_TRAFFIC = 11170645
+GEMV_MIX_TRAFFIC = 11170354
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 WORKLOAD = ("decode, 26-layer Gemma-3-1B-shaped decoder (H 1152, 4q/1kv x 256, FFN 6912, V 262144), mask FFN 5+5 + "
