@@ -16,14 +16,18 @@
 //    arithmetic of the prefill path (one warp per head, lane l holding the RoPE pairs
 //    (4l + e, 128 + 4l + e)); the CTA whose share ends at the new position also writes its key
 //    (bf16) and value to the cache and uses them from shared memory;
-//  * warp w handles query head w mod hpc and an even share (key group w / hpc) of each tile: one, two
-//    or four lanes per key compute its dot product with the scaled query (read from shared
-//    memory; key rows padded to 528 bytes, chunks rotated per lane so that the lanes of a
-//    shared-memory phase hit different bank groups), then the warp updates its running max, sum
-//    and output (lane l: dims 8l .. 8l+7) over its keys;
-//  * the warps of a head combine their partial (m, l, o) inside the CTA; each CTA then stores its
-//    per-head partials into CTA 0's shared memory (distributed shared memory stores, released by
-//    one cluster barrier), and CTA 0 combines them and writes the output row.
+//  * one head per CTA (up to 8 sequences): thread t owns output dim t; per tile, half-warps score
+//    the keys (the query in registers, a 16-lane shuffle sum per key), every warp takes the tile's
+//    max and weights into its own shared-memory row, and thread t adds sum_j p_j v_jt; the CTA's
+//    partial (m, l, o) goes to CTA 0's shared memory as one distributed shared memory store per
+//    dim, and after one cluster barrier CTA 0 combines the partials, thread t its dim;
+//  * G heads per CTA (more sequences): warp w handles query head w mod hpc and an even share (key
+//    group w / hpc) of each tile: one, two or four lanes per key compute its dot product with the
+//    scaled query (read from shared memory; key rows padded to 528 bytes, chunks rotated per lane
+//    so that the lanes of a shared-memory phase hit different bank groups), then the warp updates
+//    its running max, sum and output (lane l: dims 8l .. 8l+7) over its keys; the warps of a head
+//    combine their partial (m, l, o) inside the CTA, each CTA stores its per-head partials into
+//    CTA 0's shared memory (released by one cluster barrier), and CTA 0 combines them.
 #include <cmath>
 
 #include "attn_common.cuh"
