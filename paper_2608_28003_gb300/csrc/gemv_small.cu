@@ -10,7 +10,8 @@
 //    sub-slices of 512 bytes per row (each one or
 //    two unswizzled boxes of R rows x 256 elements), so that small-R calls still move enough bytes
 //    per pipeline round trip;
-//  * the 8 consumer warps wait for the preceding kernel and stage the activations in shared
+//  * the consumer warps (8; 16 on the tensor-core paths of a grid with one CTA per SM) wait for
+//    the preceding kernel and stage the activations in shared
 //    memory, optionally computing them first from the decoder's residual step (residual add and
 //    the two RMSNorms, fused here instead of a separate launch).  The W8A8 path quantises them
 //    there, with the arithmetic of the stand-alone per-token quantiser (Eq. stx / xint8,
@@ -19,10 +20,10 @@
 //    a row's 512 bytes (consecutive lanes read consecutive bytes: no bank conflicts);
 //  * INT8: four dp4a per 16 bytes and token, exact INT32 sums (Eq. gemm-final); bf16: fp32 FMAs,
 //    sub-slice u of a stage feeding accumulator u mod NA, summed in a fixed order at the end;
-//  * the lanes' sums meet in a butterfly (every lane ends with the same value) and lane 0 runs the
-//    epilogue: dequantisation fl(fl(s_x s_w) acc) (Eq. gemm-final), bias, GeGLU of the FFN section
-//    on interleaved gate/up rows (blocks of 8: rows 16q .. 16q+7 are gate rows 8q .. 8q+7, the next
-//    8 the matching up rows; warp w holds both rows of a pair).
+//  * the lanes' sums meet in a butterfly (every lane ends with the same value) and lane e runs the
+//    epilogue of the warp's output e: dequantisation fl(fl(s_x s_w) acc) (Eq. gemm-final), bias,
+//    GeGLU of the FFN section on interleaved gate/up rows (blocks of 8: rows 16q .. 16q+7 are gate
+//    rows 8q .. 8q+7, the next 8 the matching up rows; warp w holds both rows of a pair).
 // Waits are bounded as in the weight-streaming kernel (error word, no hang).
 #include <algorithm>
 #include <type_traits>
