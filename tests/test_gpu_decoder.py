@@ -133,13 +133,26 @@ def test_decoder_prefill_and_decode_match_oracle(B, setup, mask):
 def test_decode_batch8_matches_oracle(B, setup, mask):
     """Eight sequences: a 12-token prefill (tensor-core GEMM) and one decode step whose linears run
     the row-owning GEMV with eight token slots (bf16: on the tensor cores, with the residual norm
-    fused into q/k/v and gate/up), against an oracle decoder of batch 8 with the same statistics."""
+    fused into q/k/v and gate/up) and whose attention runs one query head per CTA, against an
+    oracle decoder of batch 8 with the same statistics."""
+    _decode_batch_matches_oracle(B, setup, mask, 8)
+
+
+def test_decode_batch12_matches_oracle(B, setup):
+    """Twelve sequences (more than eight): the decode step's attention runs all query heads of a
+    key/value head in one CTA (warps split by head and key group), its linears the 16-slot GEMV
+    (ragged: 12 of 16 slots), its residual steps the stand-alone norm kernels."""
+    _decode_batch_matches_oracle(B, setup, OM.make_mask(), 12)
+
+
+def _decode_batch_matches_oracle(B, setup, mask, nb):
     flat = setup[4]
     f32, bf, norms = synth.decoder_weights(L, H, F, V, seed=5)
     w = {k: [t.cuda() for t in v] if isinstance(v, list) else v.cuda() for k, v in bf.items()}
     n = {k: [torch.from_numpy(a).cuda() for a in v] if isinstance(v, list) else torch.from_numpy(v).cuda()
          for k, v in norms.items()}
-    cfg = B.DecoderConfig(layers=L, vocab=V, window=8, global_layers=(0,), max_batch=8, max_seq=64, max_tokens=128)
+    cfg = B.DecoderConfig(layers=L, vocab=V, window=8, global_layers=(0,), max_batch=nb, max_seq=64,
+                          max_tokens=max(128, 12 * nb))
     dec = B.Decoder(cfg, w, n)
     dec.set_stats(flat)
     dec.prepare()
@@ -147,20 +160,20 @@ def test_decode_batch8_matches_oracle(B, setup, mask):
     dec.set_mask(fb, ab, lm)
     ow = dict(f32)
     ow.update(norms)
-    od = OD.OracleDecoder(OD.DecoderConfig(layers=L, vocab=V, window=8, global_layers=(0,)), ow, batch=8, max_len=64)
+    od = OD.OracleDecoder(OD.DecoderConfig(layers=L, vocab=V, window=8, global_layers=(0,)), ow, batch=nb, max_len=64)
     od.prepare(stats=setup[1].stats)  # the statistics the GPU decoder was given (flat)
-    toks = synth.tokens(8 * 13, V, seed=7).reshape(8, 13)
+    toks = synth.tokens(nb * 13, V, seed=7).reshape(nb, 13)
     ref_all, sens = _sensitivity(od, toks, 13, mask)
     tt = torch.from_numpy(toks).cuda()
     dec.forward(tt[:, :12].contiguous(), 0, want_logits=False)
-    buf = torch.empty(8, V, dtype=torch.float32, device="cuda")
+    buf = torch.empty(nb, V, dtype=torch.float32, device="cuda")
     lg, t1 = dec.decode_step(tt[:, 12].contiguous(), 12, logits=buf)
     # One perturbation per sequence is a noisy estimate of how far rounding differences travel
     # (with W8A8 sublayers they flip INT8 codes): the same GPU decoder run on these sequences in
-    # pairs differs from this batch of eight by 1.6-2.5 % already in the prefill, where the
+    # pairs differs from the batch of eight by 1.6-2.5 % already in the prefill, where the
     # kernels are the same and only the token count (tiling, split-K) changes.  So the scale is
-    # the largest estimate over the eight sequences.
-    _close(lg.cpu().numpy(), ref_all[:, 12], np.full(8, sens[:, 12].max()))
+    # the largest estimate over the batch's sequences.
+    _close(lg.cpu().numpy(), ref_all[:, 12], np.full(nb, sens[:, 12].max()))
     assert np.array_equal(t1.cpu().numpy(), lg.argmax(-1).cpu().numpy())
     dec.close()
 
