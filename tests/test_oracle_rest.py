@@ -390,3 +390,31 @@ def test_decoder_sublayers_enter_through_their_post_norms():
         assert np.abs(scaled(name, factor, part) - base).max() < 1e-3 * scale, (name, part)
     for name, factor in (("ln_post_attn", 2), ("ln_post_ffn", 2), ("wg", 2)):
         assert np.abs(scaled(name, factor) - base).max() > 0.05 * scale, name
+
+
+def test_qk_norm_precedes_rope():
+    """QK-norm, then RoPE: a rotation keeps each (i, i + d/2) pair's length, so the cached key of
+    one token stays the same length at every position even when the norm's multipliers differ
+    between the two dims of a pair.  Normalising after the rotation would weight the rotated
+    coordinates, and the length would then depend on the position, as the direct check of the two
+    orders on a random vector shows.  The same token at positions 0..5 of one sequence reaches
+    layer 0 with the same input, so its raw key row is the same at each position."""
+    cfg, w = _composition_decoder()
+    d, half = cfg.head_dim, cfg.head_dim // 2
+    kn = np.array([0.25, 1.0, 4.0, 0.5, 3.0, 0.5, 1.0, 2.0], F32)  # pair (i, i + 4): unequal weights
+    w["k_norm"] = [kn]
+    dec = decoder.OracleDecoder(cfg, w, batch=1, max_len=8)
+    dec.forward(np.full((1, 6), 9), 0, want_logits=False)
+    keys = dec.kc[0, 0, :6, :d]
+    lengths = np.linalg.norm(keys, axis=-1)
+    assert np.all(np.abs(lengths / lengths[0] - 1.0) < 2.0 ** -6), lengths  # bf16 rounding of the cache
+    # the other order on a random row: the length moves with the position by far more than that
+    x = np.random.default_rng(3).standard_normal((1, d))
+    pos = np.arange(6)
+    other = np.stack([decoder.rmsnorm(decoder.rope(x, pos[i:i + 1], cfg.rope_global, d), kn, cfg.eps)[0]
+                      for i in range(6)])
+    ol = np.linalg.norm(other, axis=-1)
+    assert np.abs(ol / ol[0] - 1.0).max() > 0.05, ol
+    this = decoder.rope(np.repeat(decoder.rmsnorm(x, kn, cfg.eps), 6, axis=0), pos, cfg.rope_global, d)
+    assert np.allclose(np.linalg.norm(this, axis=-1), np.linalg.norm(decoder.rmsnorm(x, kn, cfg.eps)))
+    assert half * 2 == d
