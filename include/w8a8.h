@@ -403,6 +403,20 @@ w8a8_status w8a8_model_set_trace(w8a8_model* m, const w8a8_trace* t);
  * graph must exist: W8A8_ERR_INVALID_ARG before the first decode step of this (B, mask). */
 w8a8_status w8a8_model_decode_kernels(const w8a8_model* m, int B, int want_logits, int* kernels);
 
+/* Test and measurement aid with no counterpart in the paper (host only, no device access): the
+ * launch plan the decode GEMV (the row-owning kernel behind w8a8_linear, w8a8_linear_bf16,
+ * w8a8_ffn_block and the decoder at 1-16 tokens) makes for an [N, K] linear over M tokens.
+ * weight_kind: 0 bf16, 1 INT8 codes, 2 e4m3 codes; geglu: the FFN's gate/up epilogue; fused_norm:
+ * the decoder's residual step computed in the prologue; sms: the device's SM count.  out receives
+ * W8A8_PLAN_FIELDS ints: taken (0: the shape goes to another kernel, every field 0), token slots,
+ * weight rows per warp, CTAs, CTAs per SM, consumer warps, 512-byte sub-slices per stage, pipeline
+ * steps, ring stages, stage bytes, activation bytes, residual-row bytes, partial-sum bytes, dynamic
+ * shared memory bytes, padded K, sub-slices over K.  W8A8_ERR_INVALID_ARG for a null out, a weight
+ * kind outside 0-2 or sms < 1. */
+#define W8A8_PLAN_FIELDS 16
+w8a8_status w8a8_decode_gemv_plan(int weight_kind, int M, int N, int K, int geglu, int fused_norm, int sms,
+                                  int* out);
+
 /* Negative log-likelihood of targets under softmax(logits) per row (LM Head section's
  * perplexity): nll[i] = logsumexp(logits[i, :]) - logits[i, targets[i]], fp32. */
 w8a8_status w8a8_token_nll(const float* logits, const int32_t* targets, int M, int V, float* nll, void* stream);

@@ -158,6 +158,7 @@ SIGNATURES = {
     "w8a8_decoder_forward": (_i32, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_decoder_decode_step": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_model_decode_kernels": (_i32, [_vp, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
+    "w8a8_decode_gemv_plan": (_i32, [_i32, _i32, _i32, _i32, _i32, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_model_set_trace": (_i32, [_vp, ctypes.POINTER(TraceC)]),
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
@@ -582,6 +583,21 @@ def greedy_order(gain_ms, top1, ppl_delta, min_top1: float = 0.989, max_ppl_delt
     k = lib().w8a8_greedy_order(arr(gain_ms, ctypes.c_float), arr(top1, ctypes.c_float),
                                 arr(ppl_delta, ctypes.c_float), n, float(min_top1), float(max_ppl_delta), order)
     return list(order[:k])
+
+
+PLAN_FIELDS = ("taken", "slots", "rows_per_warp", "ctas", "ctas_per_sm", "consumer_warps", "subslices_per_stage",
+               "steps", "stages", "stage_bytes", "x_bytes", "resid_bytes", "partial_bytes", "smem_bytes", "kpad",
+               "subslices")
+WEIGHT_KINDS = {"bf16": 0, "int8": 1, "fp8": 2}
+
+
+def decode_gemv_plan(weight_kind: str, M: int, N: int, K: int, geglu: bool = False, fused_norm: bool = False,
+                     sms: int = 152) -> dict:
+    """The decode GEMV's launch plan for an [N, K] linear over M tokens (host only)."""
+    out = (ctypes.c_int32 * len(PLAN_FIELDS))()
+    _check("w8a8_decode_gemv_plan", lib().w8a8_decode_gemv_plan(WEIGHT_KINDS[weight_kind], M, N, K, int(geglu),
+                                                                int(fused_norm), sms, out))
+    return dict(zip(PLAN_FIELDS, list(out)))
 
 
 def choose_mask(latency, top1, ppl_delta, n_int8, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> int:

@@ -311,6 +311,20 @@ using namespace w8a8;
 
 extern "C" int w8a8_abi_version(void) { return 2; }
 
+extern "C" w8a8_status w8a8_decode_gemv_plan(int weight_kind, int M, int N, int K, int geglu, int fused_norm, int sms,
+                                             int* out) {
+  W8A8_CHECK_ARG(out, W8A8_ERR_INVALID_ARG, "w8a8_decode_gemv_plan: null out");
+  W8A8_CHECK_ARG(weight_kind >= SMALL_BF16 && weight_kind <= SMALL_FP8 && sms > 0, W8A8_ERR_INVALID_ARG,
+                 "w8a8_decode_gemv_plan: weight kind %d or SM count %d out of range", weight_kind, sms);
+  const SmallPlan p = make_small_plan(weight_kind, M, N, K, geglu ? EPI_GEGLU : EPI_BF16, sms, fused_norm != 0);
+  const int v[W8A8_PLAN_FIELDS] = {p.ok,     p.MT,          p.RW,         p.P,          p.P > sms ? 2 : 1,
+                                   p.cw,     p.ks,          p.nst,        p.stages,     p.stage_bytes,
+                                   p.xbytes, p.abytes,      p.rbytes,     p.smem_bytes, p.kpad,
+                                   p.nsub};
+  for (int i = 0; i < W8A8_PLAN_FIELDS; ++i) out[i] = p.ok ? v[i] : 0;
+  return W8A8_OK;
+}
+
 extern "C" w8a8_status w8a8_set_kernel_events(void* start_event, void* stop_event) {
   W8A8_CHECK_ARG((start_event == nullptr) == (stop_event == nullptr), W8A8_ERR_INVALID_ARG,
                  "w8a8_set_kernel_events: give both events or neither");

@@ -1,0 +1,100 @@
+"""CPU checks of the decode GEMV's launch plan (host logic, no GPU): for every decoder linear at 1-16
+tokens, in every weight kind, a plan that takes the shape covers it, fits the shared memory of the
+CTAs it puts on an SM, keeps its weight ring double-buffered (or holds the whole stream) and picks
+16 consumer warps only where its rules allow; the decoder's own shapes land where the kernel
+design puts them."""
+import pytest
+
+SMEM_PER_SM = 227 * 1024   # shared memory a CTA may use on GB300
+STATIC_SMEM = 2048         # the kernel's static shared memory (reduction slots, scales) and slack
+SMS = 152
+
+# the Gemma-3-1B-shaped decoder's linears: (N, K, GeGLU epilogue, residual step fusable)
+SHAPES = {
+    "qkv": (1536, 1152, False, True),
+    "o": (1152, 1024, False, False),
+    "gate_up": (13824, 1152, True, True),
+    "down": (1152, 6912, False, False),
+}
+
+
+@pytest.fixture(scope="module")
+def B():
+    from paper_2608_28003_gb300 import build
+    build.build()
+    from paper_2608_28003_gb300 import binding
+    return binding
+
+
+def plans(B):
+    for kind in ("bf16", "int8", "fp8"):
+        for name, (N, K, geglu, fusable) in SHAPES.items():
+            for M in range(1, 17):
+                for fused in ((False, True) if fusable else (False,)):
+                    yield kind, name, M, N, K, geglu, fused, B.decode_gemv_plan(kind, M, N, K, geglu, fused, SMS)
+
+
+def test_every_plan_covers_its_shape_and_fits(B):
+    taken = 0
+    for kind, name, M, N, K, geglu, fused, p in plans(B):
+        what = (kind, name, M, fused)
+        if not p["taken"]:
+            assert all(v == 0 for v in p.values()), what
+            continue
+        taken += 1
+        assert p["slots"] in (1, 2, 4, 8, 16) and p["slots"] >= M, what
+        assert p["slots"] == 1 or p["slots"] // 2 < M or (kind == "fp8" and p["slots"] == 8), what
+        R = 8 * p["rows_per_warp"]
+        assert p["ctas"] == -(-N // R), what                       # every output row, once
+        assert p["ctas_per_sm"] == (2 if p["ctas"] > SMS else 1), what
+        sub = 256 if kind == "bf16" else 512                      # k elements per 512-byte row slice
+        assert p["subslices"] == -(-K // sub) and p["kpad"] == p["subslices"] * sub >= K, what
+        assert p["subslices_per_stage"] in (1, 2, 4), what
+        assert p["steps"] == -(-p["subslices"] // p["subslices_per_stage"]), what
+        assert p["stage_bytes"] == p["subslices_per_stage"] * R * 512, what
+        assert min(p["steps"], 2) <= p["stages"] <= min(16, p["steps"]), what
+        assert p["smem_bytes"] == (1024 + p["stages"] * p["stage_bytes"] + p["x_bytes"] + p["resid_bytes"]
+                                   + p["partial_bytes"] + 16 * p["stages"]), what
+        assert p["ctas_per_sm"] * (p["smem_bytes"] + STATIC_SMEM) <= SMEM_PER_SM, what
+        if geglu:
+            assert p["rows_per_warp"] % 2 == 0, what                # gate and up rows in pairs
+        if fused:
+            assert M <= 8 and K <= 2048, what                       # one 8-channel vector per thread
+        mma = p["slots"] >= 8
+        assert (p["partial_bytes"] > 0) == mma, what
+        sixteen = mma and p["rows_per_warp"] == 1 and p["ctas"] <= SMS and not fused
+        assert p["consumer_warps"] == (16 if sixteen else 8), what
+        if mma:
+            assert p["partial_bytes"] == p["consumer_warps"] * R * p["slots"] * 4, what
+    assert taken > 150  # of the 288 shape, token-count and fusion combinations
+
+
+def test_decoder_shapes_route_as_designed(B):
+    P = lambda *a, **k: B.decode_gemv_plan(*a, sms=SMS, **k)  # noqa: E731
+    # one token: q/k/v with the residual step fused, 8 rows per CTA on 192 CTAs
+    p = P("bf16", 1, 1536, 1152, fused_norm=True)
+    assert (p["taken"], p["slots"], p["rows_per_warp"], p["ctas"], p["consumer_warps"]) == (1, 1, 1, 192, 8)
+    # gate/up + GeGLU: 48 rows per CTA (three gate/up pairs per warp), two CTAs per SM
+    for kind in ("bf16", "int8"):
+        p = P(kind, 1, 13824, 1152, geglu=True, fused_norm=True)
+        assert (p["rows_per_warp"], p["ctas"], p["ctas_per_sm"]) == (6, 288, 2)
+    # down and o: one CTA per SM; 16 consumer warps on the tensor-core paths (5-8 tokens)
+    for M, warps in ((1, 8), (4, 8), (8, 16)):
+        p = P("int8", M, 1152, 6912)
+        assert (p["taken"], p["ctas"], p["consumer_warps"]) == (1, 144, warps), M
+    # the residual step is fused at 1-8 tokens only; K = 6912 rows of 16 token slots do not fit
+    assert not P("bf16", 9, 1536, 1152, fused_norm=True)["taken"]
+    assert P("bf16", 9, 1536, 1152)["taken"]
+    assert not P("bf16", 16, 1152, 6912)["taken"]
+    assert not P("int8", 16, 1152, 6912)["taken"]
+    # e4m3 codes: fp32 FMAs at 1-2 tokens, the 8-slot tensor-core path from 3
+    assert P("fp8", 2, 1152, 1024)["slots"] == 2
+    assert P("fp8", 3, 1152, 1024)["slots"] == 8
+
+
+def test_plan_rejects_bad_arguments(B):
+    with pytest.raises(B.W8A8Error):
+        B.decode_gemv_plan("bf16", 1, 1152, 1024, sms=0)
+    out = (B.ctypes.c_int32 * len(B.PLAN_FIELDS))()
+    assert B.lib().w8a8_decode_gemv_plan(3, 1, 1152, 1024, 0, 0, SMS, out) != 0  # weight kind out of range
+    assert B.lib().w8a8_decode_gemv_plan(0, 1, 1152, 1024, 0, 0, SMS, None) != 0
