@@ -417,6 +417,17 @@ w8a8_status w8a8_model_decode_kernels(const w8a8_model* m, int B, int want_logit
 w8a8_status w8a8_decode_gemv_plan(int weight_kind, int M, int N, int K, int geglu, int fused_norm, int sms,
                                   int* out);
 
+/* Test and measurement aid with no counterpart in the paper (host only, no device access): the
+ * plan of the persistent weight-streaming kernel behind the lm_head (and W8A8 linears prepared
+ * without the fp16 code copy) for an [N, K] linear over M tokens.  out receives
+ * W8A8_STREAM_PLAN_FIELDS ints: dp4a GEMV (1) or MMA streaming (0), whole 128-row groups per CTA,
+ * dp4a token slots (0 on the MMA path), 8-token blocks per token group, tokens per group, token
+ * groups, 128-row weight groups, k elements per stage, k chunks per row group, CTAs, CTAs per SM,
+ * ring stages, stage bytes, dynamic shared memory bytes, partial-sum bytes.  W8A8_ERR_INVALID_ARG
+ * for a null out, M, N < 1, K < 16 or sms < 1. */
+#define W8A8_STREAM_PLAN_FIELDS 15
+w8a8_status w8a8_stream_gemm_plan(int int8_weights, int M, int N, int K, int sms, int* out);
+
 /* Negative log-likelihood of targets under softmax(logits) per row (LM Head section's
  * perplexity): nll[i] = logsumexp(logits[i, :]) - logits[i, targets[i]], fp32. */
 w8a8_status w8a8_token_nll(const float* logits, const int32_t* targets, int M, int V, float* nll, void* stream);

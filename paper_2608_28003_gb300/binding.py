@@ -159,6 +159,7 @@ SIGNATURES = {
     "w8a8_decoder_decode_step": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp, _vp]),
     "w8a8_model_decode_kernels": (_i32, [_vp, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_decode_gemv_plan": (_i32, [_i32, _i32, _i32, _i32, _i32, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
+    "w8a8_stream_gemm_plan": (_i32, [_i32, _i32, _i32, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_model_set_trace": (_i32, [_vp, ctypes.POINTER(TraceC)]),
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
@@ -598,6 +599,18 @@ def decode_gemv_plan(weight_kind: str, M: int, N: int, K: int, geglu: bool = Fal
     _check("w8a8_decode_gemv_plan", lib().w8a8_decode_gemv_plan(WEIGHT_KINDS[weight_kind], M, N, K, int(geglu),
                                                                 int(fused_norm), sms, out))
     return dict(zip(PLAN_FIELDS, list(out)))
+
+
+STREAM_PLAN_FIELDS = ("dp4a", "whole", "slots", "blocks", "tokens_per_group", "token_groups", "row_groups",
+                      "kc", "k_chunks", "ctas", "ctas_per_sm", "stages", "stage_bytes", "smem_bytes",
+                      "partial_bytes")
+
+
+def stream_gemm_plan(int8_weights: bool, M: int, N: int, K: int, sms: int = 152) -> dict:
+    """The weight-streaming kernel's plan for an [N, K] linear over M tokens (host only)."""
+    out = (ctypes.c_int32 * len(STREAM_PLAN_FIELDS))()
+    _check("w8a8_stream_gemm_plan", lib().w8a8_stream_gemm_plan(int(int8_weights), M, N, K, sms, out))
+    return dict(zip(STREAM_PLAN_FIELDS, list(out)))
 
 
 def choose_mask(latency, top1, ppl_delta, n_int8, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> int:

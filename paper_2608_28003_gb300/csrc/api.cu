@@ -325,6 +325,19 @@ extern "C" w8a8_status w8a8_decode_gemv_plan(int weight_kind, int M, int N, int 
   return W8A8_OK;
 }
 
+extern "C" w8a8_status w8a8_stream_gemm_plan(int int8_weights, int M, int N, int K, int sms, int* out) {
+  W8A8_CHECK_ARG(out, W8A8_ERR_INVALID_ARG, "w8a8_stream_gemm_plan: null out");
+  W8A8_CHECK_ARG(M >= 1 && N >= 1 && K >= 16 && sms > 0, W8A8_ERR_INVALID_ARG,
+                 "w8a8_stream_gemm_plan: M=%d, N=%d, K=%d or SM count %d out of range", M, N, K, sms);
+  const StreamPlan p = make_stream_plan(int8_weights != 0, M, N, K, sms);
+  const int v[W8A8_STREAM_PLAN_FIELDS] = {p.dp4a, p.whole, p.dp4a ? p.MT : 0, p.NB, p.TOK,
+                                          p.Z,    p.G,     p.KC,               p.C,  p.P,
+                                          p.dp4a || p.NB <= 4 ? 2 : 1,        p.stages,
+                                          p.stage_bytes,   p.smem_bytes,       (int)p.partial_bytes};
+  for (int i = 0; i < W8A8_STREAM_PLAN_FIELDS; ++i) out[i] = v[i];
+  return W8A8_OK;
+}
+
 extern "C" w8a8_status w8a8_set_kernel_events(void* start_event, void* stop_event) {
   W8A8_CHECK_ARG((start_event == nullptr) == (stop_event == nullptr), W8A8_ERR_INVALID_ARG,
                  "w8a8_set_kernel_events: give both events or neither");

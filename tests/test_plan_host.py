@@ -98,3 +98,52 @@ def test_plan_rejects_bad_arguments(B):
     out = (B.ctypes.c_int32 * len(B.PLAN_FIELDS))()
     assert B.lib().w8a8_decode_gemv_plan(3, 1, 1152, 1024, 0, 0, SMS, out) != 0  # weight kind out of range
     assert B.lib().w8a8_decode_gemv_plan(0, 1, 1152, 1024, 0, 0, SMS, None) != 0
+
+
+STREAM_STATIC = 8192  # the streaming kernel's static shared memory (barrier flags, top-1 keys)
+
+
+def test_stream_plan_covers_its_shape_and_fits(B):
+    """The persistent weight-streaming kernel (lm_head-sized outputs, 1-63 tokens): its token
+    groups, 128-row groups and k chunks cover the call, every CTA has a unit, the grid holds at
+    most its CTAs per SM on every SM, the ring fits beside them, and whole row groups per CTA
+    (no partial tiles) use the widest k chunk."""
+    for int8 in (True, False):
+        for N in (262144, 13824, 1152):
+            for K in (1152, 6912):
+                for M in range(1, 64):
+                    p = B.stream_gemm_plan(int8, M, N, K, SMS)
+                    what = (int8, N, K, M)
+                    dp4a = int8 and M <= 4 and 4 * K <= 32768
+                    assert p["dp4a"] == int(dp4a), what
+                    if dp4a:
+                        assert p["slots"] in (1, 2, 4) and p["slots"] >= M and p["slots"] // 2 < M, what
+                        assert p["tokens_per_group"] == p["slots"] and p["token_groups"] == 1, what
+                        assert p["ctas_per_sm"] == 2, what
+                    else:
+                        nb = 1 if M <= 8 else 2 if M <= 16 else 4 if M <= 32 else 8
+                        assert p["blocks"] == nb and p["tokens_per_group"] == 8 * nb, what
+                        assert p["token_groups"] == -(-M // (8 * nb)), what
+                        assert p["ctas_per_sm"] == (2 if nb <= 4 else 1), what
+                    assert p["row_groups"] == -(-N // 128), what
+                    assert p["k_chunks"] == -(-K // p["kc"]) and p["k_chunks"] * p["kc"] >= K, what
+                    units = p["token_groups"] * p["row_groups"] * p["k_chunks"]
+                    assert 1 <= p["ctas"] <= min(units, p["ctas_per_sm"] * SMS, 8192), what
+                    assert p["whole"] == int(p["token_groups"] * p["row_groups"] >= p["ctas"]), what
+                    if p["whole"]:
+                        assert p["kc"] == (256 if int8 else 128), what
+                    assert 2 <= p["stages"] <= 8, what
+                    assert p["ctas_per_sm"] * (p["smem_bytes"] + STREAM_STATIC) <= SMEM_PER_SM, what
+                    assert p["partial_bytes"] == p["ctas"] * 2 * 128 * p["tokens_per_group"] * 4, what
+
+
+def test_lm_head_routes_as_designed(B):
+    # one token: the dp4a GEMV, two CTAs per SM over 2048 whole 128-row groups
+    p = B.stream_gemm_plan(True, 1, 262144, 1152, SMS)
+    assert (p["dp4a"], p["ctas"], p["ctas_per_sm"], p["whole"]) == (1, 2 * SMS, 2, 1)
+    # 5-32 tokens: the MMA streaming kernel with two CTAs per SM; from 33, one
+    for M, cps in ((5, 2), (16, 2), (32, 2), (33, 1), (63, 1)):
+        p = B.stream_gemm_plan(True, M, 262144, 1152, SMS)
+        assert (p["dp4a"], p["ctas_per_sm"], p["ctas"]) == (0, cps, cps * SMS), M
+    with pytest.raises(B.W8A8Error):
+        B.stream_gemm_plan(True, 0, 262144, 1152, SMS)
