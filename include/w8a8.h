@@ -428,6 +428,16 @@ w8a8_status w8a8_decode_gemv_plan(int weight_kind, int M, int N, int K, int gegl
 #define W8A8_STREAM_PLAN_FIELDS 15
 w8a8_status w8a8_stream_gemm_plan(int int8_weights, int M, int N, int K, int sms, int* out);
 
+/* Test and measurement aid with no counterpart in the paper (host only, no device access): the
+ * tile shape and k split the tcgen05 GEMM takes for an [N, K] linear over M tokens.  mode: 0 bf16,
+ * 1 INT8 codes (carried as fp16), 2 e4m3; kind: 0 bf16 output, 1 GeGLU, 2 fp32 logits; split_ok:
+ * the caller's workspace holds the partials and tile counters a k split needs; sms: the SM count.
+ * out[0] = 1 for CTA pairs on 256-token tiles, 0 for single CTAs on 128-token tiles; out[1] = the
+ * tile's channels (256, 192 or 128 on pairs; 128 or 64 on single CTAs); out[2] = the k parts of a
+ * single-CTA tile (1: no split).  W8A8_ERR_INVALID_ARG for a null out, a mode or kind out of range or
+ * sms < 2; W8A8_ERR_SHAPE where the GEMM does not take the shape (K or N not a multiple of 16). */
+w8a8_status w8a8_tc_gemm_plan(int mode, int M, int N, int K, int kind, int split_ok, int sms, int* out);
+
 /* Negative log-likelihood of targets under softmax(logits) per row (LM Head section's
  * perplexity): nll[i] = logsumexp(logits[i, :]) - logits[i, targets[i]], fp32. */
 w8a8_status w8a8_token_nll(const float* logits, const int32_t* targets, int M, int V, float* nll, void* stream);

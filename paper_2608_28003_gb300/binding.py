@@ -160,6 +160,7 @@ SIGNATURES = {
     "w8a8_model_decode_kernels": (_i32, [_vp, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_decode_gemv_plan": (_i32, [_i32, _i32, _i32, _i32, _i32, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_stream_gemm_plan": (_i32, [_i32, _i32, _i32, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
+    "w8a8_tc_gemm_plan": (_i32, [_i32, _i32, _i32, _i32, _i32, _i32, _i32, ctypes.POINTER(ctypes.c_int32)]),
     "w8a8_model_set_trace": (_i32, [_vp, ctypes.POINTER(TraceC)]),
     "w8a8_token_nll": (_i32, [_vp, _vp, _i32, _i32, _vp, _vp]),
     "w8a8_choose_mask": (_i32, [_fp, _fp, _fp, ctypes.POINTER(ctypes.c_int32), _i32, _f32, _f32]),
@@ -611,6 +612,19 @@ def stream_gemm_plan(int8_weights: bool, M: int, N: int, K: int, sms: int = 152)
     out = (ctypes.c_int32 * len(STREAM_PLAN_FIELDS))()
     _check("w8a8_stream_gemm_plan", lib().w8a8_stream_gemm_plan(int(int8_weights), M, N, K, sms, out))
     return dict(zip(STREAM_PLAN_FIELDS, list(out)))
+
+
+TC_MODES = {"bf16": 0, "int8": 1, "fp8": 2}
+EPILOGUES = {"bf16": 0, "geglu": 1, "f32": 2}
+
+
+def tc_gemm_plan(mode: str, M: int, N: int, K: int, kind: str = "bf16", split_ok: bool = True,
+                 sms: int = 152) -> tuple:
+    """(pair, channels per tile, k parts) the tcgen05 GEMM takes for an [N, K] linear over M tokens."""
+    out = (ctypes.c_int32 * 3)()
+    _check("w8a8_tc_gemm_plan", lib().w8a8_tc_gemm_plan(TC_MODES[mode], M, N, K, EPILOGUES[kind], int(split_ok),
+                                                        sms, out))
+    return tuple(out)
 
 
 def choose_mask(latency, top1, ppl_delta, n_int8, min_top1: float = 0.989, max_ppl_delta: float = 0.01) -> int:

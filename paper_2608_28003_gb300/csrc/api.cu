@@ -325,6 +325,20 @@ extern "C" w8a8_status w8a8_decode_gemv_plan(int weight_kind, int M, int N, int 
   return W8A8_OK;
 }
 
+extern "C" w8a8_status w8a8_tc_gemm_plan(int mode, int M, int N, int K, int kind, int split_ok, int sms, int* out) {
+  W8A8_CHECK_ARG(out, W8A8_ERR_INVALID_ARG, "w8a8_tc_gemm_plan: null out");
+  W8A8_CHECK_ARG(mode >= TC_BF16 && mode <= TC_FP8 && kind >= EPI_BF16 && kind <= EPI_F32 && sms > 1,
+                 W8A8_ERR_INVALID_ARG, "w8a8_tc_gemm_plan: mode %d, kind %d or SM count %d out of range", mode,
+                 kind, sms);
+  W8A8_CHECK_ARG(tc_gemm_supported(M, N, K, kind, false, 0), W8A8_ERR_SHAPE,
+                 "w8a8_tc_gemm_plan: M=%d, N=%d, K=%d is not a tensor-core GEMM shape", M, N, K);
+  const TcChoice c = tc_choose(mode, M, N, K, kind, split_ok != 0, sms);
+  out[0] = c.pair;
+  out[1] = c.bn;
+  out[2] = c.ksplit;
+  return W8A8_OK;
+}
+
 extern "C" w8a8_status w8a8_stream_gemm_plan(int int8_weights, int M, int N, int K, int sms, int* out) {
   W8A8_CHECK_ARG(out, W8A8_ERR_INVALID_ARG, "w8a8_stream_gemm_plan: null out");
   W8A8_CHECK_ARG(M >= 1 && N >= 1 && K >= 16 && sms > 0, W8A8_ERR_INVALID_ARG,

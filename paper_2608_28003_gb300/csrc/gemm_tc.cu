@@ -1159,52 +1159,61 @@ constexpr int kMinKbPerPart = 2;
 // under the cap) would lose.
 constexpr int kMinParts = 4;
 
-// k parts of a single-CTA call on BN-column tiles (1: no split)
-int split_parts(const TcArgs& a, int mode, int bn) {
-  const int sms = device_sms(), nkb = (a.K + bk_elems(mode) - 1) / bk_elems(mode);
-  const long long tiles = (long long)((a.N + bn - 1) / bn) * ((a.M + kBM - 1) / kBM);
-  if (a.kind == EPI_BF16 && a.partials && a.tile_counters && 2 * tiles <= sms) {
-    const int ks = std::min({(int)(sms / tiles), nkb / kMinKbPerPart, a.K / (4 * a_box_rows(a.M))});
+// k parts of a single-CTA call on BN-column tiles (1: no split); split_ok: the caller gave the
+// partials and tile counters the split needs
+int split_parts(int mode, int M, int N, int K, int kind, bool split_ok, int bn, int sms) {
+  const int nkb = (K + bk_elems(mode) - 1) / bk_elems(mode);
+  const long long tiles = (long long)((N + bn - 1) / bn) * ((M + kBM - 1) / kBM);
+  if (kind == EPI_BF16 && split_ok && 2 * tiles <= sms) {
+    const int ks = std::min({(int)(sms / tiles), nkb / kMinKbPerPart, K / (4 * a_box_rows(M))});
     if (ks >= kMinParts) return ks;
   }
   return 1;
 }
 
-template <int kMode, int kBN>
-w8a8_status launch_split(TcArgs a, cudaStream_t st) {
-  a.ksplit = split_parts(a, kMode, kBN);
-  return launch_t<kMode, kBN>(a, st);
-}
+}  // namespace
 
-template <int kMode>
-w8a8_status dispatch(TcArgs a, cudaStream_t st) {
-  a.ksplit = 1;
-  const long long pairs = device_sms() / 2;
+TcChoice tc_choose(int mode, int M, int N, int K, int kind, bool split_ok, int sms) {
+  const long long pairs = sms / 2;
   // ks k parts: ks units per tile, each with 1/ks of the k range, plus the partials' round trip
   // (taken as a third of a unit's time).  Counted from 256 tokens on the bf16 and W8A8 paths only:
   // there it picks split 128-column tiles over one wave of 64-column tiles (512 x 6912 -> 1152:
   // bf16 38.6 -> 32.4 us, W8A8 42.6 -> 33.4 us), while below it, and on the FP8 path, it measured
   // slower than the split-free model (128-token prefill 1.87 -> 2.22 ms; FP8 at 512 tokens 23 -> 29 us)
-  const bool split_cost = a.M >= 256 && kMode != kModeFp8;
+  const bool split_cost = M >= 256 && mode != kModeFp8;
   auto cost = [&](int bm, int bn, double unit, long long slots, int ks = 1) {
-    const long long t = (long long)((a.N + bn - 1) / bn) * ((a.M + bm - 1) / bm) * ks;
+    const long long t = (long long)((N + bn - 1) / bn) * ((M + bm - 1) / bm) * ks;
     return (double)((t + slots - 1) / slots) * bn * unit / ks * (ks > 1 ? 1.33 : 1.0);
   };
   const double c256 = cost(2 * kBM, 256, 1.0, pairs), c192 = cost(2 * kBM, 192, 1.32, pairs),
-               c128 = cost(kBM, 128, 1.81, 2 * pairs, split_cost ? split_parts(a, kMode, 128) : 1),
-               c64 = cost(kBM, 64, 2.7, 2 * pairs, split_cost ? split_parts(a, kMode, 64) : 1);
+               c128 = cost(kBM, 128, 1.81, 2 * pairs, split_cost ? split_parts(mode, M, N, K, kind, split_ok, 128, sms) : 1),
+               c64 = cost(kBM, 64, 2.7, 2 * pairs, split_cost ? split_parts(mode, M, N, K, kind, split_ok, 64, sms) : 1);
   // W8A8 only: pairs on 256 x 128 tiles where the output is narrow but the single-CTA tiles would
   // not be split over k (they fill more than half of the SMs); four 128-column accumulator slots
   // keep the fold chunks of a long k range in flight (measured on 2048 x 6912 -> 1152: 42.7 us
   // against 45.7 us on single CTAs; the bf16 and FP8 paths measured no gain)
-  const double p128 = kMode == kModeI8 ? cost(2 * kBM, 128, 1.32, pairs) : 1e30;
-  if (c256 <= c192 && c256 <= c128 && c256 <= c64 && c256 <= p128) return launch_t2<kMode, 256>(a, st);
-  if (c192 <= c128 && c192 <= c64 && c192 <= p128) return launch_t2<kMode, 192>(a, st);
-  const long long t128 = (long long)((a.N + 127) / 128) * ((a.M + kBM - 1) / kBM);
-  if (kMode == kModeI8 && 2 * t128 > device_sms() && p128 < c128 && p128 < c64) return launch_t2<kMode, 128>(a, st);
+  const double p128 = mode == kModeI8 ? cost(2 * kBM, 128, 1.32, pairs) : 1e30;
+  if (c256 <= c192 && c256 <= c128 && c256 <= c64 && c256 <= p128) return TcChoice{1, 256, 1};
+  if (c192 <= c128 && c192 <= c64 && c192 <= p128) return TcChoice{1, 192, 1};
+  const long long t128 = (long long)((N + 127) / 128) * ((M + kBM - 1) / kBM);
+  if (mode == kModeI8 && 2 * t128 > sms && p128 < c128 && p128 < c64) return TcChoice{1, 128, 1};
+  if (c128 <= c64) return TcChoice{0, 128, split_parts(mode, M, N, K, kind, split_ok, 128, sms)};
+  return TcChoice{0, 64, split_parts(mode, M, N, K, kind, split_ok, 64, sms)};  // few tokens: spread the weights
+}
 
-  if (c128 <= c64) return launch_split<kMode, 128>(a, st);
-  return launch_split<kMode, 64>(a, st);  // few tokens: spread the weight stream over more SMs
+namespace {
+
+template <int kMode>
+w8a8_status dispatch(TcArgs a, cudaStream_t st) {
+  const TcChoice c = tc_choose(kMode, a.M, a.N, a.K, a.kind, a.partials && a.tile_counters, device_sms());
+  a.ksplit = c.ksplit;
+  if (c.pair) {
+    if (c.bn == 256) return launch_t2<kMode, 256>(a, st);
+    if (c.bn == 192) return launch_t2<kMode, 192>(a, st);
+    return launch_t2<kMode, 128>(a, st);
+  }
+  if (c.bn == 128) return launch_t<kMode, 128>(a, st);
+  return launch_t<kMode, 64>(a, st);
 }
 
 }  // namespace

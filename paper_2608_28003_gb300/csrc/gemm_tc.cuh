@@ -37,6 +37,17 @@ struct TcArgs {
 // Shapes the tensor-core GEMM takes: K a multiple of 16, N a multiple of 16, top-1 for at most
 // max_top rows.
 bool tc_gemm_supported(int M, int N, int K, int kind, bool want_top, int max_top);
+
+// The tile shape and k split the tcgen05 GEMM takes for a call (host only): pair = 1 for CTA pairs
+// on 256-token tiles of bn = 256, 192 or 128 channels, 0 for single CTAs on 128-token tiles of bn =
+// 128 or 64 channels; ksplit = the k parts of a single-CTA tile (1: none).  mode: TC_BF16, TC_I8 or
+// TC_FP8; kind: the epilogue; split_ok: partials and tile counters are available; sms: SM count.
+struct TcChoice {
+  int pair;
+  int bn;
+  int ksplit;
+};
+TcChoice tc_choose(int mode, int M, int N, int K, int kind, bool split_ok, int sms);
 // Workspace bytes the split-K partials of an M-token call may take (an upper bound over N and K,
 // non-decreasing in M).
 size_t tc_split_partial_bytes(int M, int sms);

@@ -147,3 +147,49 @@ def test_lm_head_routes_as_designed(B):
         assert (p["dp4a"], p["ctas_per_sm"], p["ctas"]) == (0, cps, cps * SMS), M
     with pytest.raises(B.W8A8Error):
         B.stream_gemm_plan(True, 0, 262144, 1152, SMS)
+
+
+def test_tc_gemm_choice_rules(B):
+    """The tcgen05 GEMM's tile choice over a grid of shapes: a k split only on single-CTA tiles of a
+    bf16-output call that has its partials, at least four parts, one unit per SM at most, and each
+    part at least two stages of k; pairs only on 256-token tiles."""
+    for mode in ("bf16", "int8", "fp8"):
+        for kind in ("bf16", "geglu", "f32"):
+            for split_ok in (False, True):
+                for M in (1, 8, 16, 32, 64, 128, 256, 300, 512, 2048):
+                    for N in (1152, 1536, 6912, 13824, 262144):
+                        for K in (1024, 1152, 6912):
+                            pair, bn, ks = B.tc_gemm_plan(mode, M, N, K, kind, split_ok, SMS)
+                            what = (mode, kind, split_ok, M, N, K)
+                            assert (pair, bn) in ((1, 256), (1, 192), (1, 128), (0, 128), (0, 64)), what
+                            if pair == 1 and bn == 128:
+                                assert mode == "int8", what      # the narrow pair tile is W8A8's
+                            if ks > 1:
+                                assert not pair and kind == "bf16" and split_ok, what
+                                tiles = -(-N // bn) * -(-M // 128)
+                                bk = 128 if mode == "fp8" else 64  # k elements per 128-byte stage row
+                                assert ks >= 4 and ks * tiles <= SMS and 2 * ks <= -(-K // bk), what
+                                assert 2 * tiles <= SMS, what
+                            else:
+                                assert ks == 1, what
+
+
+def test_tc_gemm_routes_decoder_shapes_as_designed(B):
+    P = lambda *a, **k: B.tc_gemm_plan(*a, sms=SMS, **k)  # noqa: E731
+    # 2048-token prefill: gate/up on 256 x 256 pair tiles in every mode; W8A8 down on 256 x 128 pairs
+    for mode in ("bf16", "int8", "fp8"):
+        assert P(mode, 2048, 13824, 1152, "geglu") == (1, 256, 1)
+    assert P("int8", 2048, 1152, 6912) == (1, 128, 1)
+    assert P("bf16", 2048, 1152, 6912) == (0, 128, 1)
+    # 512 tokens: the down projection on split 128-column tiles (four parts), bf16 and W8A8
+    assert P("bf16", 512, 1152, 6912) == (0, 128, 4) == P("int8", 512, 1152, 6912)
+    # decode batches: q/k/v, o and down at 32 tokens split over 6-8 parts of 64-column tiles
+    assert P("bf16", 32, 1536, 1152) == (0, 64, 6)
+    assert P("bf16", 32, 1152, 1024) == (0, 64, 8)
+    assert P("bf16", 32, 1152, 6912) == (0, 64, 8)
+    # without the partials' workspace, no split
+    assert P("bf16", 32, 1152, 6912, split_ok=False) == (0, 64, 1)
+    # fp32 logits (lm_head) never split
+    assert P("bf16", 64, 262144, 1152, "f32")[2] == 1
+    with pytest.raises(B.W8A8Error):
+        P("bf16", 32, 1152, 1000)  # K not a multiple of 16
