@@ -193,3 +193,37 @@ def test_tc_gemm_routes_decoder_shapes_as_designed(B):
     assert P("bf16", 64, 262144, 1152, "f32")[2] == 1
     with pytest.raises(B.W8A8Error):
         P("bf16", 32, 1152, 1000)  # K not a multiple of 16
+
+
+RESERVED = 65536  # W8A8_WS_RESERVED: the split-K and top-1 counters at the start of a workspace
+
+
+def _ceil(x, a=256):
+    return -(-x // a) * a
+
+
+def test_workspace_sizes_cover_every_region(B):
+    """The workspace a caller allocates from the size queries holds the reserved counters, the
+    activation codes and scales, and the larger of the two kernels' partial sums (the streaming
+    kernel's plan, the tcgen05 GEMM's k split: one unit per SM at most); the FFN block's holds h and
+    both linears' regions and the row-maxima hand-off.  Sizes grow with the token count."""
+    for N, K in ((1536, 1152), (1152, 1024), (13824, 1152), (1152, 6912), (262144, 1152)):
+        prev = prev_bf = 0
+        for M in (1, 2, 4, 5, 8, 9, 16, 33, 64, 128, 300, 512, 2048):
+            total = B._size("w8a8_linear_workspace_size", M, N, K)
+            rows = M if M >= 128 else -(-M // 8) * 8
+            parts = max(B.stream_gemm_plan(True, M, N, K, SMS)["partial_bytes"], SMS * 128 * min(rows, 128) * 4)
+            assert total == RESERVED + _ceil(2 * M * K) + _ceil(8 * M) + _ceil(parts), (M, N, K)
+            assert total % 256 == 0 and total >= prev
+            prev = total
+            bf = B._size("w8a8_linear_bf16_workspace_size", M, N, K)
+            parts_bf = max(B.stream_gemm_plan(False, M, N, K, SMS)["partial_bytes"], SMS * 128 * min(rows, 128) * 4)
+            assert bf == RESERVED + _ceil(parts_bf) and bf >= prev_bf, (M, N, K)
+            prev_bf = bf
+    for M in (1, 8, 16, 64, 512, 2048):
+        H, F = 1152, 6912
+        ffn = B._size("w8a8_ffn_workspace_size", M, H, F)
+        gu = B._size("w8a8_linear_workspace_size", M, 2 * F, H) - RESERVED
+        dn = B._size("w8a8_linear_workspace_size", M, H, F) - RESERVED
+        assert ffn == RESERVED + _ceil(2 * M * F) + gu + dn + _ceil(2 * SMS * 16 * 4), M
+        assert B._size("w8a8_lm_head_workspace_size", M, 262144, H) == B._size("w8a8_linear_workspace_size", M, 262144, H)
